@@ -1,0 +1,250 @@
+/*
+ * tda.h -- C ABI of the GB300 (sm_103a) training-data-attribution hot path.
+ *
+ * The library turns per-example weight gradients of linear layers, given in
+ * factored form, into seeded Kronecker-projected features, preconditions the
+ * queries with a damped Fisher inverse and scores queries against training
+ * examples (dattri-LLM paper, Sec. 3.2 and App. A.2, A.4, B.2, B.3).
+ *
+ * Notation. A linear layer z = W a has W in R^{N_o x N_i}. For one example with
+ * T token positions the paper's factors are a in R^{N_i x T} and g = Dz in
+ * R^{N_o x T}, and the weight gradient is DW = g a^T = sum_t g_t a_t^T
+ * (Eq. 1). This ABI stores an example's factors token-major:
+ *     A[t][c] = a_t[c]   (T x d_in,  d_in  = N_i)
+ *     B[t][r] = g_t[r]   (T x d_out, d_out = N_o)
+ * and a batch of N examples as A[N][T][d_in], B[N][T][d_out], C-contiguous.
+ * A padded token is a zero row in both A and B; it contributes nothing.
+ *
+ * Projection (Eq. 2, App. A.2). P_a (k_in x d_in) and P_g (k_out x d_out) are
+ * Rademacher maps with entries s/sqrt(k), s in {+1,-1}, k the map's output
+ * dimension. s is generated from (seed, layer, side, row, col) by a
+ * counter-based hash; the matrices never exist in device memory. A projected
+ * feature is the k_out x k_in matrix
+ *     Phi = P_g DW P_a^T = (B S_out)^T (A S_in) / sqrt(k_in k_out)
+ * stored row-major (feature index i*k_in + j), D = k_in*k_out features.
+ *
+ * Conventions shared by every entry point:
+ *  - All pointers to tensors are DEVICE pointers (cudaMalloc'd, or from a
+ *    caching allocator) unless a comment says host. The caller owns every
+ *    buffer; the library allocates no device memory. Scratch is passed in as
+ *    `ws` of `ws_bytes`, sized by tda_workspace_size().
+ *  - `stream` is a cudaStream_t (NULL = legacy default stream). Every call is
+ *    asynchronous on that stream unless its comment says otherwise.
+ *  - Arguments are validated on the host before any launch; a failing call
+ *    launches nothing and returns a non-zero tda_status. tda_last_error()
+ *    returns a thread-local message describing the last failure.
+ *  - Device-side bounded waits that time out set a device error word instead
+ *    of hanging; tda_device_status() synchronises the stream and reports it.
+ *  - Nothing throws across the ABI.
+ */
+#ifndef TDA_H
+#define TDA_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef enum {
+    TDA_OK = 0,
+    TDA_ERR_INVALID_ARG = 1, /* null pointer, bad size, misalignment, bad enum */
+    TDA_ERR_UNSUPPORTED = 2, /* valid request with no kernel for it (e.g. route) */
+    TDA_ERR_WORKSPACE = 3,   /* ws smaller than tda_workspace_size() */
+    TDA_ERR_CUDA = 4,        /* a CUDA runtime call failed; see tda_last_error */
+    TDA_ERR_NOT_SPD = 5,     /* F + lambda I was not positive definite */
+    TDA_ERR_TIMEOUT = 6      /* a device-side bounded wait expired */
+} tda_status;
+
+typedef enum { TDA_F32 = 0, TDA_BF16 = 1, TDA_F64 = 2 } tda_dtype;
+
+/* TDA_PROJ_IDENTITY requires k_in == d_in and k_out == d_out and uses P = I
+ * (no 1/sqrt(k) scale), so Phi = DW exactly: the unprojected gradient. */
+typedef enum { TDA_PROJ_RADEMACHER = 0, TDA_PROJ_IDENTITY = 1 } tda_proj_kind;
+
+/* Routes (Sec. 3.2 "FLOP-aware routing", App. A.4):
+ *  FACTORED    -- project the factors, then contract over tokens (Eq. 2);
+ *  MATERIALIZE -- form DW = g a^T (Eq. 1), then project it / dot it;
+ *  GRAM        -- factored inner products, sum_{t,s} <a_t,a_s><g_t,g_s> (Eq. 4). */
+typedef enum {
+    TDA_ROUTE_AUTO = -1,
+    TDA_ROUTE_FACTORED = 0,
+    TDA_ROUTE_MATERIALIZE = 1,
+    TDA_ROUTE_GRAM = 2
+} tda_route_id;
+
+/* Operations the cost model routes (App. A.4: per layer and per operation). */
+typedef enum {
+    TDA_OP_PROJECT = 0,             /* n1 examples -> n1 projected features      */
+    TDA_OP_SIMILARITY_PROJECTED = 1,/* n1 x n2 inner products of projected grads */
+    TDA_OP_SIMILARITY_EXACT = 2     /* n1 x n2 inner products of unprojected DW  */
+} tda_op;
+
+/* One linear layer. seed and layer must be identical for every gradient that
+ * will be compared (App. A.2: the per-layer base seed is held fixed). */
+typedef struct {
+    int64_t d_in;   /* N_i, input width  */
+    int64_t d_out;  /* N_o, output width */
+    int64_t T;      /* token positions per example */
+    int32_t k_in;   /* k_a, projected input dimension  */
+    int32_t k_out;  /* k_g, projected output dimension */
+    uint64_t seed;  /* base seed of the projection */
+    uint32_t layer; /* layer index mixed into the seed */
+    int32_t kind;   /* tda_proj_kind */
+} tda_layer_desc;
+
+/* ---------------------------------------------------------------------------
+ * tda_proj_entries -- write the sign matrix S (rows x cols, int8 in {+1,-1},
+ * or {0,1} for the identity kind) of one projection side, exactly as the
+ * projection kernels generate it on chip. side 0 = input factor a (S_in,
+ * rows = d_in, cols = k_in); side 1 = output gradient g (S_out, rows = d_out,
+ * cols = k_out). P = S / sqrt(cols). Seeds per layer and side: App. A.2.
+ * out: device, rows*cols bytes, row-major. cols in [1, 1024].
+ * ------------------------------------------------------------------------- */
+tda_status tda_proj_entries(uint64_t seed, uint32_t layer, int32_t side, int32_t kind,
+                            int64_t rows, int32_t cols, int8_t* out, void* stream);
+
+/* ---------------------------------------------------------------------------
+ * tda_workspace_size -- bytes of scratch `ws` that the matching call needs
+ * (op PROJECT -> tda_project; op SIMILARITY_EXACT -> tda_similarity_exact).
+ * n1 = examples (or queries), n2 = train examples (similarity only).
+ * route AUTO resolves through tda_route() first. Host only; no device work.
+ * ------------------------------------------------------------------------- */
+tda_status tda_workspace_size(tda_op op, const tda_layer_desc* L, tda_dtype dtype,
+                              int64_t n1, int64_t n2, tda_route_id route, size_t* bytes);
+
+/* ---------------------------------------------------------------------------
+ * tda_project -- projected per-example gradients of one layer (Eq. 1, Eq. 2).
+ *   dtype  TDA_BF16 or TDA_F32: element type of A and B. Accumulation is fp32.
+ *   A      device, A[N][T][d_in], 16-byte aligned.
+ *   B      device, B[N][T][d_out], 16-byte aligned.
+ *   phi    device fp32, N rows of D = k_in*k_out features, row n at
+ *          phi + n*ld_phi (ld_phi >= D); overwritten.
+ *   route  FACTORED (Eq. 2 on the factors), MATERIALIZE (DW first), or AUTO
+ *          (tda_route's choice for TDA_OP_PROJECT).
+ * Both routes give the same result up to rounding (App. A.4).
+ * bf16 requires d_in % 8 == 0 and d_out % 8 == 0; fp32 requires % 4.
+ * ------------------------------------------------------------------------- */
+tda_status tda_project(const tda_layer_desc* L, tda_dtype dtype, const void* A, const void* B,
+                       int64_t N, float* phi, int64_t ld_phi, tda_route_id route,
+                       void* ws, size_t ws_bytes, void* stream);
+
+/* ---------------------------------------------------------------------------
+ * tda_similarity_exact -- unprojected gradient inner products
+ *   S[q][i] = beta*S[q][i] + <DW_q, DW_i>_F
+ * for n_q query and n_t train examples of one layer (Eq. 4's left side).
+ *   route GRAM computes sum_{t,s} <a_t^q,a_s^i><g_t^q,g_s^i> (Eq. 4) without
+ *   forming DW; MATERIALIZE forms DW (Eq. 1) in ws and takes Frobenius dots;
+ *   AUTO asks tda_route (TDA_OP_SIMILARITY_EXACT).
+ *   Aq/Bq: [n_q][T][d], At/Bt: [n_t][T][d], dtype as in tda_project.
+ *   S: device fp32, row q at S + q*ld_S (ld_S >= n_t). beta 0 overwrites.
+ * ------------------------------------------------------------------------- */
+tda_status tda_similarity_exact(const tda_layer_desc* L, tda_dtype dtype,
+                                const void* Aq, const void* Bq, int64_t n_q,
+                                const void* At, const void* Bt, int64_t n_t,
+                                float* S, int64_t ld_S, float beta, tda_route_id route,
+                                void* ws, size_t ws_bytes, void* stream);
+
+/* ---------------------------------------------------------------------------
+ * tda_precondition -- damped Fisher inverse on the query side (App. B.3: a
+ * curvature fit over the training gradients, then per-layer preconditioning
+ * of the queries; App. B.2: damping in units of the mean eigenvalue).
+ *
+ * `state` is a device buffer of tda_precondition_state_bytes(D, state_dtype)
+ * bytes: an 8-double header followed by a D x D matrix of state_dtype
+ * (TDA_F32 or TDA_F64). The ops, in order of use:
+ *   TDA_PC_RESET      zero the state.
+ *   TDA_PC_FIT_ACCUM  M += Phi^T Phi over n feature rows (phi, ld_phi).
+ *                     Called once per streamed chunk of training features.
+ *   TDA_PC_FACTOR     F = M / n_total; lambda = lambda_abs +
+ *                     lambda_rel_mean_eig * tr(F)/D; M <- L with
+ *                     L L^T = F + lambda I (lower Cholesky, in place).
+ *                     A non-positive pivot is recorded in the header;
+ *                     tda_precondition_info() reports it (TDA_ERR_NOT_SPD).
+ *   TDA_PC_APPLY      qhat = (F + lambda I)^{-1} q for n_q rows of q (fp32,
+ *                     ld_q); qhat has state_dtype (fp64 rows for an F64
+ *                     state), row stride ld_qhat. After a failed FACTOR the
+ *                     rows are NaN.
+ * Arguments not used by an op are ignored (may be 0/NULL).
+ * ------------------------------------------------------------------------- */
+#define TDA_PC_RESET 0
+#define TDA_PC_FIT_ACCUM 1
+#define TDA_PC_FACTOR 2
+#define TDA_PC_APPLY 3
+
+size_t tda_precondition_state_bytes(int64_t D, tda_dtype state_dtype);
+
+tda_status tda_precondition(int32_t op, int64_t D, tda_dtype state_dtype, void* state,
+                            const float* phi, int64_t n, int64_t ld_phi,
+                            int64_t n_total, double lambda_abs, double lambda_rel_mean_eig,
+                            const float* q, int64_t n_q, int64_t ld_q,
+                            void* qhat, int64_t ld_qhat, void* stream);
+
+/* Synchronises `stream` and copies the state header to host `info[4]`:
+ * {lambda used, tr(F)/D, failed pivot (0 = SPD), n_total}. Returns
+ * TDA_ERR_NOT_SPD if the last FACTOR failed. */
+tda_status tda_precondition_info(int64_t D, tda_dtype state_dtype, const void* state,
+                                 double* info, void* stream);
+
+/* ---------------------------------------------------------------------------
+ * tda_score -- S[q][i] = beta*S[q][i] + sum_f Qhat[q][f] Phi[i][f]
+ * (gradient inner products; GradDot when Qhat = Q, Sec. 3.2 / Eq. 4).
+ *   Qhat  device, n_q rows of D, q_dtype TDA_F32 or TDA_F64, row stride ld_q.
+ *         With TDA_F64 the sum is accumulated in fp64.
+ *   Phi   device fp32, n_t rows of D, row stride ld_phi.
+ *   S     device fp32, row stride ld_S >= n_t. beta 0 overwrites (S may hold
+ *         garbage); beta 1 accumulates layers.
+ * ------------------------------------------------------------------------- */
+tda_status tda_score(const void* Qhat, tda_dtype q_dtype, int64_t n_q, int64_t ld_q,
+                     const float* Phi, int64_t n_t, int64_t ld_phi, int64_t D,
+                     float* S, int64_t ld_S, float beta, void* stream);
+
+/* ---------------------------------------------------------------------------
+ * tda_topk -- per query row of S (n_q x n_t, fp32, row stride ld_S), the k
+ * largest scores in descending order; ties go to the smaller train index.
+ * idx: device int32 [n_q][k]; val: device fp32 [n_q][k] (may be NULL).
+ * 1 <= k <= min(n_t, 1024). A NaN score is treated as larger than +inf (it
+ * ranks first), so it is visible in the output.
+ * ------------------------------------------------------------------------- */
+tda_status tda_topk(const float* S, int64_t n_q, int64_t n_t, int64_t ld_S, int32_t k,
+                    int32_t* idx, float* val, void* stream);
+
+/* ---------------------------------------------------------------------------
+ * tda_route -- the FLOP-aware route choice (Sec. 3.2, App. A.4, Table 2).
+ * Host only, no device work. cost_out[r] = estimated cost of route r
+ * (FACTORED, MATERIALIZE, GRAM); -1 for a route that cannot produce the op's
+ * result. In the default model the cost is the route's flop count (2 flops
+ * per multiply-add); after tda_route_calibrate() it is the estimated seconds
+ * max(flops / rate_r, bytes_r / bandwidth) with rates measured on the device.
+ * The cheapest route wins; ties prefer GRAM, then FACTORED, then MATERIALIZE.
+ * ------------------------------------------------------------------------- */
+tda_status tda_route(const tda_layer_desc* L, tda_op op, int64_t n1, int64_t n2,
+                     tda_dtype dtype, tda_route_id* chosen, double* cost_out);
+
+/* Measures per-route throughput on the current device with short synthetic
+ * launches of the route kernels inside the caller's scratch `ws` (at least
+ * TDA_CALIBRATE_WS_BYTES bytes, contents destroyed), synchronises `stream`,
+ * then switches tda_route to the time model. rates_out (host, may be NULL)
+ * receives 4 doubles: flop/s of the factored, materialise and Gram kernels
+ * and the streaming bytes/s of the factored kernel. */
+#define TDA_CALIBRATE_WS_BYTES ((size_t)768 << 20)
+tda_status tda_route_calibrate(void* ws, size_t ws_bytes, void* stream, double* rates_out);
+/* 0 = flop model (the paper's), 1 = calibrated time model. */
+tda_status tda_route_set_model(int32_t model);
+
+/* Synchronises `stream`, then reads and clears the device error word.
+ * Returns TDA_ERR_TIMEOUT if a kernel's bounded wait expired since the last
+ * check, TDA_ERR_CUDA on a CUDA error, else TDA_OK. */
+tda_status tda_device_status(void* stream);
+
+/* Thread-local message of the last failing call on this thread ("" if none). */
+const char* tda_last_error(void);
+
+/* ABI version: major*10000 + minor*100 + patch. */
+int32_t tda_version(void);
+
+#ifdef __cplusplus
+}
+#endif
+#endif /* TDA_H */
