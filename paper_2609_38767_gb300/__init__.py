@@ -1,0 +1,194 @@
+"""GB300 (sm_103a) training-data-attribution hot path of the dattri-LLM paper.
+
+Python binding of the C ABI in ``include/tda.h``: every function here has the
+name and argument order of its C entry point and only marshals arguments
+(torch tensors become device pointers, ``stream=None`` becomes torch's current
+CUDA stream). All computation happens in ``libtda.so``. Importing this package
+loads nothing; the first call loads the library and raises if it is missing,
+so there is no silent CPU path.
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+import threading
+
+__all__ = [
+    "LayerDesc", "TdaError", "load", "tda_proj_entries", "tda_workspace_size", "tda_project",
+    "tda_similarity_exact", "tda_precondition_state_bytes", "tda_precondition",
+    "tda_precondition_info", "tda_score", "tda_topk", "tda_route", "tda_route_calibrate",
+    "tda_route_set_model", "tda_device_status", "tda_last_error", "tda_version",
+]
+
+_HERE = os.path.dirname(os.path.abspath(__file__))
+_lock = threading.Lock()
+_lib = None
+
+# enums of include/tda.h
+TDA_OK, TDA_ERR_INVALID_ARG, TDA_ERR_UNSUPPORTED, TDA_ERR_WORKSPACE = 0, 1, 2, 3
+TDA_ERR_CUDA, TDA_ERR_NOT_SPD, TDA_ERR_TIMEOUT = 4, 5, 6
+TDA_F32, TDA_BF16, TDA_F64 = 0, 1, 2
+TDA_PROJ_RADEMACHER, TDA_PROJ_IDENTITY = 0, 1
+TDA_ROUTE_AUTO, TDA_ROUTE_FACTORED, TDA_ROUTE_MATERIALIZE, TDA_ROUTE_GRAM = -1, 0, 1, 2
+TDA_OP_PROJECT, TDA_OP_SIMILARITY_PROJECTED, TDA_OP_SIMILARITY_EXACT = 0, 1, 2
+TDA_PC_RESET, TDA_PC_FIT_ACCUM, TDA_PC_FACTOR, TDA_PC_APPLY = 0, 1, 2, 3
+TDA_CALIBRATE_WS_BYTES = 768 << 20
+_STATUS = {0: "TDA_OK", 1: "TDA_ERR_INVALID_ARG", 2: "TDA_ERR_UNSUPPORTED", 3: "TDA_ERR_WORKSPACE",
+           4: "TDA_ERR_CUDA", 5: "TDA_ERR_NOT_SPD", 6: "TDA_ERR_TIMEOUT"}
+
+
+class LayerDesc(ctypes.Structure):
+    """tda_layer_desc."""
+    _fields_ = [("d_in", ctypes.c_int64), ("d_out", ctypes.c_int64), ("T", ctypes.c_int64),
+                ("k_in", ctypes.c_int32), ("k_out", ctypes.c_int32), ("seed", ctypes.c_uint64),
+                ("layer", ctypes.c_uint32), ("kind", ctypes.c_int32)]
+
+    def __init__(self, d_in, d_out, T, k_in, k_out, seed=0, layer=0, kind=TDA_PROJ_RADEMACHER):
+        super().__init__(d_in, d_out, T, k_in, k_out, seed, layer, kind)
+
+
+class TdaError(RuntimeError):
+    def __init__(self, status: int, message: str):
+        super().__init__(f"{_STATUS.get(status, status)}: {message}")
+        self.status = status
+
+
+def lib_path(name: str = "libtda.so") -> str:
+    return os.path.join(_HERE, name)
+
+
+def load() -> ctypes.CDLL:
+    """Load libtda.so (built by ``build.build()``); raises if it is absent."""
+    global _lib
+    with _lock:
+        if _lib is not None:
+            return _lib
+        path = lib_path()
+        if not os.path.exists(path):
+            raise ImportError(f"{path} is missing: run paper_2609_38767_gb300.build.build() first")
+        lib = ctypes.CDLL(path)
+        P, I32, I64, U32, U64 = ctypes.c_void_p, ctypes.c_int32, ctypes.c_int64, ctypes.c_uint32, ctypes.c_uint64
+        D, F, SZ = ctypes.c_double, ctypes.c_float, ctypes.c_size_t
+        LP = ctypes.POINTER(LayerDesc)
+        sig = {
+            "tda_proj_entries": (I32, [U64, U32, I32, I32, I64, I32, P, P]),
+            "tda_workspace_size": (I32, [I32, LP, I32, I64, I64, I32, ctypes.POINTER(SZ)]),
+            "tda_project": (I32, [LP, I32, P, P, I64, P, I64, I32, P, SZ, P]),
+            "tda_similarity_exact": (I32, [LP, I32, P, P, I64, P, P, I64, P, I64, F, I32, P, SZ, P]),
+            "tda_precondition_state_bytes": (SZ, [I64, I32]),
+            "tda_precondition": (I32, [I32, I64, I32, P, P, I64, I64, I64, D, D, P, I64, I64, P, I64, P]),
+            "tda_precondition_info": (I32, [I64, I32, P, ctypes.POINTER(D), P]),
+            "tda_score": (I32, [P, I32, I64, I64, P, I64, I64, I64, P, I64, F, P]),
+            "tda_topk": (I32, [P, I64, I64, I64, I32, P, P, P]),
+            "tda_route": (I32, [LP, I32, I64, I64, I32, ctypes.POINTER(I32), ctypes.POINTER(D)]),
+            "tda_route_calibrate": (I32, [P, SZ, P, ctypes.POINTER(D)]),
+            "tda_route_set_model": (I32, [I32]),
+            "tda_device_status": (I32, [P]),
+            "tda_last_error": (ctypes.c_char_p, []),
+            "tda_version": (I32, []),
+        }
+        for name, (res, args) in sig.items():
+            fn = getattr(lib, name)
+            fn.restype = res
+            fn.argtypes = args
+        _lib = lib
+        return lib
+
+
+def _ptr(x):
+    """Device (or host) address of a tensor, an int, or None."""
+    if x is None:
+        return None
+    if isinstance(x, int):
+        return x
+    return x.data_ptr()
+
+
+def _stream(stream):
+    if stream is None:
+        import torch
+        return torch.cuda.current_stream().cuda_stream
+    if isinstance(stream, int):
+        return stream
+    return stream.cuda_stream
+
+
+def _check(status: int) -> None:
+    if status != TDA_OK:
+        raise TdaError(status, load().tda_last_error().decode())
+
+
+def tda_last_error() -> str:
+    return load().tda_last_error().decode()
+
+
+def tda_version() -> int:
+    return int(load().tda_version())
+
+
+def tda_proj_entries(seed, layer, side, kind, rows, cols, out, stream=None):
+    _check(load().tda_proj_entries(seed, layer, side, kind, rows, cols, _ptr(out), _stream(stream)))
+
+
+def tda_workspace_size(op, L, dtype, n1, n2, route=TDA_ROUTE_AUTO) -> int:
+    b = ctypes.c_size_t(0)
+    _check(load().tda_workspace_size(op, ctypes.byref(L), dtype, n1, n2, route, ctypes.byref(b)))
+    return int(b.value)
+
+
+def tda_project(L, dtype, A, B, N, phi, ld_phi, route=TDA_ROUTE_AUTO, ws=None, ws_bytes=0, stream=None):
+    _check(load().tda_project(ctypes.byref(L), dtype, _ptr(A), _ptr(B), N, _ptr(phi), ld_phi, route,
+                              _ptr(ws), ws_bytes, _stream(stream)))
+
+
+def tda_similarity_exact(L, dtype, Aq, Bq, n_q, At, Bt, n_t, S, ld_S, beta=0.0, route=TDA_ROUTE_AUTO,
+                         ws=None, ws_bytes=0, stream=None):
+    _check(load().tda_similarity_exact(ctypes.byref(L), dtype, _ptr(Aq), _ptr(Bq), n_q, _ptr(At), _ptr(Bt),
+                                       n_t, _ptr(S), ld_S, beta, route, _ptr(ws), ws_bytes, _stream(stream)))
+
+
+def tda_precondition_state_bytes(D, state_dtype) -> int:
+    return int(load().tda_precondition_state_bytes(D, state_dtype))
+
+
+def tda_precondition(op, D, state_dtype, state, phi=None, n=0, ld_phi=0, n_total=0, lambda_abs=0.0,
+                     lambda_rel_mean_eig=0.0, q=None, n_q=0, ld_q=0, qhat=None, ld_qhat=0, stream=None):
+    _check(load().tda_precondition(op, D, state_dtype, _ptr(state), _ptr(phi), n, ld_phi, n_total,
+                                   lambda_abs, lambda_rel_mean_eig, _ptr(q), n_q, ld_q, _ptr(qhat),
+                                   ld_qhat, _stream(stream)))
+
+
+def tda_precondition_info(D, state_dtype, state, stream=None) -> list[float]:
+    info = (ctypes.c_double * 4)()
+    _check(load().tda_precondition_info(D, state_dtype, _ptr(state), info, _stream(stream)))
+    return list(info)
+
+
+def tda_score(Qhat, q_dtype, n_q, ld_q, Phi, n_t, ld_phi, D, S, ld_S, beta=0.0, stream=None):
+    _check(load().tda_score(_ptr(Qhat), q_dtype, n_q, ld_q, _ptr(Phi), n_t, ld_phi, D, _ptr(S), ld_S,
+                            beta, _stream(stream)))
+
+
+def tda_topk(S, n_q, n_t, ld_S, k, idx, val=None, stream=None):
+    _check(load().tda_topk(_ptr(S), n_q, n_t, ld_S, k, _ptr(idx), _ptr(val), _stream(stream)))
+
+
+def tda_route(L, op, n1, n2, dtype) -> tuple[int, list[float]]:
+    chosen = ctypes.c_int32(0)
+    cost = (ctypes.c_double * 3)()
+    _check(load().tda_route(ctypes.byref(L), op, n1, n2, dtype, ctypes.byref(chosen), cost))
+    return int(chosen.value), list(cost)
+
+
+def tda_route_calibrate(ws, ws_bytes, stream=None) -> list[float]:
+    rates = (ctypes.c_double * 4)()
+    _check(load().tda_route_calibrate(_ptr(ws), ws_bytes, _stream(stream), rates))
+    return list(rates)
+
+
+def tda_route_set_model(model: int) -> None:
+    _check(load().tda_route_set_model(model))
+
+
+def tda_device_status(stream=None) -> None:
+    _check(load().tda_device_status(_stream(stream)))

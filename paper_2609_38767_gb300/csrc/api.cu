@@ -1,0 +1,421 @@
+// api.cu -- the extern "C" entry points of libtda.so (include/tda.h):
+// host-side argument validation, route selection and kernel dispatch.
+#include <stdarg.h>
+#include <stdio.h>
+#include <string.h>
+
+#include <cmath>
+#include <mutex>
+
+#include "tda_internal.cuh"
+
+namespace tda {
+
+static thread_local char g_msg[512] = "";
+
+tda_status fail(tda_status st, const char* fmt, ...) {
+    va_list ap;
+    va_start(ap, fmt);
+    vsnprintf(g_msg, sizeof(g_msg), fmt, ap);
+    va_end(ap);
+    return st;
+}
+
+tda_status cuda_check(cudaError_t e, const char* what) {
+    if (e == cudaSuccess) return TDA_OK;
+    return fail(TDA_ERR_CUDA, "%s: %s (%s)", what, cudaGetErrorName(e), cudaGetErrorString(e));
+}
+
+// The device error word: bounded waits that expire OR bits into it.
+__device__ unsigned int g_error_word;
+
+unsigned int* device_error_word() {
+    static std::mutex mu;
+    static unsigned int* cache[64] = {};
+    int dev = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return nullptr;
+    std::lock_guard<std::mutex> lock(mu);
+    if (!cache[dev]) {
+        void* p = nullptr;
+        if (cudaGetSymbolAddress(&p, g_error_word) != cudaSuccess) return nullptr;
+        cache[dev] = (unsigned int*)p;
+    }
+    return cache[dev];
+}
+
+float projection_scale(const tda_layer_desc& L);
+
+// ---------------------------------------------------------------------------
+// Route cost model (Sec. 3.2, App. A.4, Table 2): flop counts at 2 flops per
+// multiply-add, or, after calibration, estimated seconds.
+// ---------------------------------------------------------------------------
+static std::mutex g_route_mu;
+static int g_route_model = 0;
+static double g_rate[3] = {0, 0, 0};  // flop/s of the factored, materialise, Gram kernels
+static double g_bw = 0;               // bytes/s
+
+struct RouteCounts {
+    double flops[3];
+    double bytes[3];
+};
+
+void set_route_rates(const double rate[3], double bw) {
+    std::lock_guard<std::mutex> lock(g_route_mu);
+    for (int r = 0; r < 3; ++r) g_rate[r] = rate[r];
+    g_bw = bw;
+    g_route_model = (rate[0] > 0 && bw > 0) ? 1 : 0;
+}
+
+static RouteCounts route_counts(const tda_layer_desc& L, tda_op op, int64_t n1, int64_t n2,
+                                tda_dtype dt) {
+    const double B1 = (double)n1, B2 = (double)n2, T = (double)L.T;
+    const double Ni = (double)L.d_in, No = (double)L.d_out, ka = (double)L.k_in, kg = (double)L.k_out;
+    const double el = dt == TDA_F32 ? 4.0 : 2.0;
+    const double factors = T * (Ni + No) * el;  // one example's factor bytes
+    const double proj = 2.0 * T * (Ni * ka + No * kg);
+    const double contract = 2.0 * T * ka * kg;
+    const double build = 2.0 * T * Ni * No;
+    const double dense = 2.0 * No * Ni * ka + 2.0 * No * ka * kg;
+    RouteCounts c;
+    if (op == TDA_OP_PROJECT) {
+        c.flops[0] = B1 * (proj + contract);
+        c.flops[1] = B1 * (build + dense);
+        c.flops[2] = -1;
+        c.bytes[0] = B1 * (factors + 4.0 * ka * kg);
+        c.bytes[1] = B1 * (factors + 8.0 * Ni * No + 4.0 * ka * kg);
+        c.bytes[2] = -1;
+    } else if (op == TDA_OP_SIMILARITY_PROJECTED) {
+        c.flops[0] = (B1 + B2) * (proj + contract) + B1 * B2 * 2.0 * ka * kg;
+        c.flops[1] = (B1 + B2) * (build + dense) + B1 * B2 * 2.0 * ka * kg;
+        c.flops[2] = (B1 + B2) * proj + B1 * B2 * 2.0 * T * T * (ka + kg);
+        c.bytes[0] = (B1 + B2) * (factors + 4.0 * ka * kg);
+        c.bytes[1] = (B1 + B2) * (factors + 8.0 * Ni * No);
+        c.bytes[2] = (B1 + B2) * factors + B1 * B2 * 4.0 * T * (ka + kg);
+    } else {
+        c.flops[0] = -1;
+        c.flops[1] = (B1 + B2) * build + B1 * B2 * 2.0 * Ni * No;
+        c.flops[2] = B1 * B2 * 2.0 * T * T * (Ni + No);
+        c.bytes[0] = -1;
+        c.bytes[1] = (B1 + B2) * (factors + 4.0 * Ni * No) + B1 * B2 * 0.0;
+        c.bytes[2] = B1 * B2 * factors;
+    }
+    return c;
+}
+
+static tda_status validate_layer(const tda_layer_desc* L, bool need_k) {
+    if (!L) return fail(TDA_ERR_INVALID_ARG, "layer descriptor is NULL");
+    if (L->d_in < 1 || L->d_out < 1 || L->T < 0)
+        return fail(TDA_ERR_INVALID_ARG, "bad layer sizes d_in=%lld d_out=%lld T=%lld",
+                    (long long)L->d_in, (long long)L->d_out, (long long)L->T);
+    if (L->kind != TDA_PROJ_RADEMACHER && L->kind != TDA_PROJ_IDENTITY)
+        return fail(TDA_ERR_INVALID_ARG, "bad projection kind %d", L->kind);
+    if (need_k) {
+        if (L->k_in < 1 || L->k_out < 1)
+            return fail(TDA_ERR_INVALID_ARG, "bad projection dims k_in=%d k_out=%d", L->k_in, L->k_out);
+        if (L->kind == TDA_PROJ_IDENTITY && (L->k_in != L->d_in || L->k_out != L->d_out))
+            return fail(TDA_ERR_INVALID_ARG, "identity projection needs k_in == d_in, k_out == d_out");
+    }
+    return TDA_OK;
+}
+
+static tda_status validate_factors(const tda_layer_desc* L, tda_dtype dt, const void* A,
+                                   const void* B, int64_t n, const char* who) {
+    if (dt != TDA_F32 && dt != TDA_BF16)
+        return fail(TDA_ERR_INVALID_ARG, "%s: dtype must be TDA_F32 or TDA_BF16", who);
+    if (n < 0) return fail(TDA_ERR_INVALID_ARG, "%s: negative example count", who);
+    if (n > 0 && L->T > 0) {
+        if (!A || !B) return fail(TDA_ERR_INVALID_ARG, "%s: NULL factor pointer", who);
+        if (((uintptr_t)A & 15) || ((uintptr_t)B & 15))
+            return fail(TDA_ERR_INVALID_ARG, "%s: factors must be 16-byte aligned", who);
+        const int64_t q = dt == TDA_BF16 ? 8 : 4;
+        if (L->d_in % q || L->d_out % q)
+            return fail(TDA_ERR_INVALID_ARG, "%s: d_in and d_out must be multiples of %lld", who,
+                        (long long)q);
+    }
+    return TDA_OK;
+}
+
+static tda_route_id choose(const RouteCounts& c, double* cost_out) {
+    double cost[3];
+    std::lock_guard<std::mutex> lock(g_route_mu);
+    for (int r = 0; r < 3; ++r) {
+        if (c.flops[r] < 0) {
+            cost[r] = -1;
+        } else if (g_route_model == 1 && g_rate[r] > 0 && g_bw > 0) {
+            cost[r] = std::fmax(c.flops[r] / g_rate[r], c.bytes[r] / g_bw);
+        } else {
+            cost[r] = c.flops[r];
+        }
+    }
+    static const int pref[3] = {TDA_ROUTE_GRAM, TDA_ROUTE_FACTORED, TDA_ROUTE_MATERIALIZE};
+    int best = -1;
+    for (int p = 0; p < 3; ++p) {
+        const int r = pref[p];
+        if (cost[r] < 0) continue;
+        if (best < 0 || cost[r] < cost[best]) best = r;
+    }
+    if (cost_out)
+        for (int r = 0; r < 3; ++r) cost_out[r] = cost[r];
+    return (tda_route_id)best;
+}
+
+}  // namespace tda
+
+using namespace tda;
+
+extern "C" {
+
+const char* tda_last_error(void) { return g_msg; }
+
+int32_t tda_version(void) { return 100; }
+
+tda_status tda_proj_entries(uint64_t seed, uint32_t layer, int32_t side, int32_t kind, int64_t rows,
+                            int32_t cols, int8_t* out, void* stream) {
+    g_msg[0] = 0;
+    if (side != 0 && side != 1) return fail(TDA_ERR_INVALID_ARG, "side must be 0 or 1");
+    if (kind != TDA_PROJ_RADEMACHER && kind != TDA_PROJ_IDENTITY)
+        return fail(TDA_ERR_INVALID_ARG, "bad projection kind %d", kind);
+    if (rows < 0 || cols < 1 || cols > 1024) return fail(TDA_ERR_INVALID_ARG, "bad rows/cols");
+    if (rows > 0 && !out) return fail(TDA_ERR_INVALID_ARG, "out is NULL");
+    return cuda_check(launch_proj_entries(side_key(seed, layer, side), kind, rows, cols, out,
+                                          (cudaStream_t)stream),
+                      "tda_proj_entries launch");
+}
+
+tda_status tda_route(const tda_layer_desc* L, tda_op op, int64_t n1, int64_t n2, tda_dtype dtype,
+                     tda_route_id* chosen, double* cost_out) {
+    g_msg[0] = 0;
+    if (op < TDA_OP_PROJECT || op > TDA_OP_SIMILARITY_EXACT)
+        return fail(TDA_ERR_INVALID_ARG, "bad op %d", (int)op);
+    tda_status st = validate_layer(L, op != TDA_OP_SIMILARITY_EXACT);
+    if (st) return st;
+    if (n1 < 0 || n2 < 0) return fail(TDA_ERR_INVALID_ARG, "negative batch size");
+    if (!chosen) return fail(TDA_ERR_INVALID_ARG, "chosen is NULL");
+    *chosen = choose(route_counts(*L, op, n1, n2, dtype), cost_out);
+    return TDA_OK;
+}
+
+tda_status tda_route_set_model(int32_t model) {
+    g_msg[0] = 0;
+    if (model != 0 && model != 1) return fail(TDA_ERR_INVALID_ARG, "model must be 0 or 1");
+    std::lock_guard<std::mutex> lock(g_route_mu);
+    if (model == 1 && !(g_rate[0] > 0 && g_bw > 0))
+        return fail(TDA_ERR_INVALID_ARG, "time model needs tda_route_calibrate() first");
+    g_route_model = model;
+    return TDA_OK;
+}
+
+tda_status tda_workspace_size(tda_op op, const tda_layer_desc* L, tda_dtype dtype, int64_t n1,
+                              int64_t n2, tda_route_id route, size_t* bytes) {
+    g_msg[0] = 0;
+    if (!bytes) return fail(TDA_ERR_INVALID_ARG, "bytes is NULL");
+    *bytes = 0;
+    tda_status st = validate_layer(L, op != TDA_OP_SIMILARITY_EXACT);
+    if (st) return st;
+    if (route == TDA_ROUTE_AUTO) {
+        st = tda_route(L, op, n1, n2, dtype, &route, nullptr);
+        if (st) return st;
+    }
+    if (op == TDA_OP_PROJECT) {
+        if (route == TDA_ROUTE_MATERIALIZE) *bytes = materialize_ws_bytes_per_example(*L);
+        return TDA_OK;
+    }
+    if (op == TDA_OP_SIMILARITY_EXACT) {
+        if (route == TDA_ROUTE_MATERIALIZE) *bytes = similarity_materialize_ws_bytes(*L, n1, 1);
+        return TDA_OK;
+    }
+    return fail(TDA_ERR_UNSUPPORTED, "no workspace query for op %d", (int)op);
+}
+
+tda_status tda_project(const tda_layer_desc* L, tda_dtype dtype, const void* A, const void* B,
+                       int64_t N, float* phi, int64_t ld_phi, tda_route_id route, void* ws,
+                       size_t ws_bytes, void* stream) {
+    g_msg[0] = 0;
+    tda_status st = validate_layer(L, true);
+    if (st) return st;
+    if ((st = validate_factors(L, dtype, A, B, N, "tda_project"))) return st;
+    const int64_t D = (int64_t)L->k_in * L->k_out;
+    if (N > 0 && !phi) return fail(TDA_ERR_INVALID_ARG, "phi is NULL");
+    if (ld_phi < D) return fail(TDA_ERR_INVALID_ARG, "ld_phi (%lld) < k_in*k_out (%lld)",
+                                (long long)ld_phi, (long long)D);
+    if (N > 2147483647LL) return fail(TDA_ERR_INVALID_ARG, "N too large");
+    if (route == TDA_ROUTE_AUTO) {
+        tda_route_id r;
+        if ((st = tda_route(L, TDA_OP_PROJECT, N, 0, dtype, &r, nullptr))) return st;
+        route = r;
+    }
+    cudaStream_t s = (cudaStream_t)stream;
+    if (N == 0) return TDA_OK;
+    if (L->T == 0) return cuda_check(cudaMemset2DAsync(phi, ld_phi * 4, 0, D * 4, N, s), "zero phi");
+    if (route == TDA_ROUTE_FACTORED) {
+        if (dtype == TDA_BF16 && project_tc_supported(*L, A, B)) {
+            unsigned int* err = device_error_word();
+            if (!err) return fail(TDA_ERR_CUDA, "cannot resolve the device error word");
+            return cuda_check(launch_project_tc(*L, A, B, N, phi, ld_phi, err, s), "project (tcgen05)");
+        }
+        return cuda_check(launch_project_simt(*L, dtype, A, B, N, phi, ld_phi, s), "project (simt)");
+    }
+    if (route == TDA_ROUTE_MATERIALIZE) {
+        const size_t need = materialize_ws_bytes_per_example(*L);
+        if (!ws || ws_bytes < need)
+            return fail(TDA_ERR_WORKSPACE, "materialise route needs >= %zu bytes of ws, got %zu", need,
+                        ws_bytes);
+        return cuda_check(launch_project_materialized(*L, dtype, A, B, N, phi, ld_phi, ws, ws_bytes, s),
+                          "project (materialise)");
+    }
+    return fail(TDA_ERR_UNSUPPORTED, "route %d cannot produce projected features", (int)route);
+}
+
+tda_status tda_similarity_exact(const tda_layer_desc* L, tda_dtype dtype, const void* Aq,
+                                const void* Bq, int64_t n_q, const void* At, const void* Bt,
+                                int64_t n_t, float* S, int64_t ld_S, float beta, tda_route_id route,
+                                void* ws, size_t ws_bytes, void* stream) {
+    g_msg[0] = 0;
+    tda_status st = validate_layer(L, false);
+    if (st) return st;
+    if ((st = validate_factors(L, dtype, Aq, Bq, n_q, "tda_similarity_exact (queries)"))) return st;
+    if ((st = validate_factors(L, dtype, At, Bt, n_t, "tda_similarity_exact (train)"))) return st;
+    if (n_q > 65535) return fail(TDA_ERR_INVALID_ARG, "n_q must be <= 65535");
+    if (n_q > 0 && n_t > 0 && !S) return fail(TDA_ERR_INVALID_ARG, "S is NULL");
+    if (ld_S < n_t) return fail(TDA_ERR_INVALID_ARG, "ld_S < n_t");
+    if (route == TDA_ROUTE_AUTO) {
+        tda_route_id r;
+        if ((st = tda_route(L, TDA_OP_SIMILARITY_EXACT, n_q, n_t, dtype, &r, nullptr))) return st;
+        route = r;
+    }
+    cudaStream_t s = (cudaStream_t)stream;
+    if (n_q == 0 || n_t == 0) return TDA_OK;
+    if (L->T == 0) {
+        // DW = 0: the inner products are 0
+        return cuda_check(launch_score(S, TDA_F32, n_q, 0, S, n_t, 0, 0, S, ld_S, beta, s), "zero S");
+    }
+    if (route == TDA_ROUTE_GRAM)
+        return cuda_check(launch_similarity_gram(*L, dtype, Aq, Bq, n_q, At, Bt, n_t, S, ld_S, beta, s),
+                          "similarity (gram)");
+    if (route == TDA_ROUTE_MATERIALIZE) {
+        const size_t need = similarity_materialize_ws_bytes(*L, n_q, 1);
+        if (!ws || ws_bytes < need)
+            return fail(TDA_ERR_WORKSPACE, "materialise route needs >= %zu bytes of ws, got %zu", need,
+                        ws_bytes);
+        return cuda_check(launch_similarity_materialized(*L, dtype, Aq, Bq, n_q, At, Bt, n_t, S, ld_S,
+                                                         beta, ws, ws_bytes, s),
+                          "similarity (materialise)");
+    }
+    return fail(TDA_ERR_UNSUPPORTED, "route %d cannot produce exact similarities", (int)route);
+}
+
+size_t tda_precondition_state_bytes(int64_t D, tda_dtype state_dtype) {
+    if (D < 1 || (state_dtype != TDA_F32 && state_dtype != TDA_F64)) return 0;
+    const size_t el = state_dtype == TDA_F64 ? 8 : 4;
+    return kPcHeaderDoubles * sizeof(double) + (size_t)D * (size_t)D * el;
+}
+
+tda_status tda_precondition(int32_t op, int64_t D, tda_dtype state_dtype, void* state,
+                            const float* phi, int64_t n, int64_t ld_phi, int64_t n_total,
+                            double lambda_abs, double lambda_rel_mean_eig, const float* q,
+                            int64_t n_q, int64_t ld_q, void* qhat, int64_t ld_qhat, void* stream) {
+    g_msg[0] = 0;
+    if (D < 1) return fail(TDA_ERR_INVALID_ARG, "D must be >= 1");
+    if (state_dtype != TDA_F32 && state_dtype != TDA_F64)
+        return fail(TDA_ERR_INVALID_ARG, "state dtype must be TDA_F32 or TDA_F64");
+    if (!state) return fail(TDA_ERR_INVALID_ARG, "state is NULL");
+    if ((uintptr_t)state & 15) return fail(TDA_ERR_INVALID_ARG, "state must be 16-byte aligned");
+    cudaStream_t s = (cudaStream_t)stream;
+    switch (op) {
+        case TDA_PC_RESET:
+            return cuda_check(cudaMemsetAsync(state, 0, tda_precondition_state_bytes(D, state_dtype), s),
+                              "reset state");
+        case TDA_PC_FIT_ACCUM:
+            if (n < 0) return fail(TDA_ERR_INVALID_ARG, "negative n");
+            if (n > 0 && !phi) return fail(TDA_ERR_INVALID_ARG, "phi is NULL");
+            if (ld_phi < D) return fail(TDA_ERR_INVALID_ARG, "ld_phi < D");
+            if (D > 65535 * 64LL) return fail(TDA_ERR_INVALID_ARG, "D too large");
+            return cuda_check(launch_pc_fit(D, state_dtype, state, phi, n, ld_phi, s), "fit");
+        case TDA_PC_FACTOR:
+            if (n_total < 1) return fail(TDA_ERR_INVALID_ARG, "n_total must be >= 1");
+            if (!(lambda_abs >= 0) || !(lambda_rel_mean_eig >= 0) ||
+                !(lambda_abs > 0 || lambda_rel_mean_eig > 0))
+                return fail(TDA_ERR_INVALID_ARG, "damping must be >= 0 and not both zero");
+            return cuda_check(launch_pc_factor(D, state_dtype, state, n_total, lambda_abs,
+                                               lambda_rel_mean_eig, s),
+                              "factor");
+        case TDA_PC_APPLY: {
+            if (n_q < 0) return fail(TDA_ERR_INVALID_ARG, "negative n_q");
+            if (n_q > 0 && (!q || !qhat)) return fail(TDA_ERR_INVALID_ARG, "q/qhat is NULL");
+            if (ld_q < D || ld_qhat < D) return fail(TDA_ERR_INVALID_ARG, "ld_q/ld_qhat < D");
+            const size_t el = state_dtype == TDA_F64 ? 8 : 4;
+            if ((size_t)D * el > 200 * 1024)
+                return fail(TDA_ERR_UNSUPPORTED, "APPLY keeps one row in shared memory: D*%zu > 200 KiB", el);
+            return cuda_check(launch_pc_apply(D, state_dtype, state, q, n_q, ld_q, qhat, ld_qhat, s),
+                              "apply");
+        }
+        default:
+            return fail(TDA_ERR_INVALID_ARG, "bad precondition op %d", op);
+    }
+}
+
+tda_status tda_precondition_info(int64_t D, tda_dtype state_dtype, const void* state, double* info,
+                                 void* stream) {
+    g_msg[0] = 0;
+    if (!state || !info) return fail(TDA_ERR_INVALID_ARG, "NULL argument");
+    (void)D;
+    (void)state_dtype;
+    cudaStream_t s = (cudaStream_t)stream;
+    double h[kPcHeaderDoubles];
+    tda_status st = cuda_check(cudaMemcpyAsync(h, state, sizeof(h), cudaMemcpyDeviceToHost, s), "read header");
+    if (st) return st;
+    if ((st = cuda_check(cudaStreamSynchronize(s), "sync"))) return st;
+    info[0] = h[kPcLambda];
+    info[1] = h[kPcMeanEig];
+    info[2] = h[kPcFailedPivot];
+    info[3] = h[kPcNTotal];
+    if (h[kPcFailedPivot] != 0.0)
+        return fail(TDA_ERR_NOT_SPD, "F + lambda I not positive definite at pivot %.0f", h[kPcFailedPivot]);
+    return TDA_OK;
+}
+
+tda_status tda_score(const void* Qhat, tda_dtype q_dtype, int64_t n_q, int64_t ld_q, const float* Phi,
+                     int64_t n_t, int64_t ld_phi, int64_t D, float* S, int64_t ld_S, float beta,
+                     void* stream) {
+    g_msg[0] = 0;
+    if (q_dtype != TDA_F32 && q_dtype != TDA_F64)
+        return fail(TDA_ERR_INVALID_ARG, "Qhat dtype must be TDA_F32 or TDA_F64");
+    if (n_q < 0 || n_t < 0 || D < 0) return fail(TDA_ERR_INVALID_ARG, "negative size");
+    if (n_q > 65535LL * 64) return fail(TDA_ERR_INVALID_ARG, "n_q too large");
+    if (n_q > 0 && n_t > 0) {
+        if (!S) return fail(TDA_ERR_INVALID_ARG, "S is NULL");
+        if (D > 0 && (!Qhat || !Phi)) return fail(TDA_ERR_INVALID_ARG, "Qhat/Phi is NULL");
+    }
+    if (ld_q < D || ld_phi < D || ld_S < n_t) return fail(TDA_ERR_INVALID_ARG, "leading dimension too small");
+    return cuda_check(launch_score(Qhat, q_dtype, n_q, ld_q, Phi, n_t, ld_phi, D, S, ld_S, beta,
+                                   (cudaStream_t)stream),
+                      "score");
+}
+
+tda_status tda_topk(const float* S, int64_t n_q, int64_t n_t, int64_t ld_S, int32_t k, int32_t* idx,
+                    float* val, void* stream) {
+    g_msg[0] = 0;
+    if (n_q < 0 || n_t < 0) return fail(TDA_ERR_INVALID_ARG, "negative size");
+    if (k < 1 || k > 1024 || k > n_t) return fail(TDA_ERR_INVALID_ARG, "need 1 <= k <= min(n_t, 1024)");
+    if (n_t > 0xFFFFFFFFLL) return fail(TDA_ERR_INVALID_ARG, "n_t too large");
+    if (ld_S < n_t) return fail(TDA_ERR_INVALID_ARG, "ld_S < n_t");
+    if (n_q > 0 && (!S || !idx)) return fail(TDA_ERR_INVALID_ARG, "S/idx is NULL");
+    return cuda_check(launch_topk(S, n_q, n_t, ld_S, k, idx, val, (cudaStream_t)stream), "topk");
+}
+
+tda_status tda_device_status(void* stream) {
+    g_msg[0] = 0;
+    tda_status st = cuda_check(cudaStreamSynchronize((cudaStream_t)stream), "stream sync");
+    if (st) return st;
+    unsigned int w = 0;
+    if ((st = cuda_check(cudaMemcpyFromSymbol(&w, g_error_word, sizeof(w)), "read error word"))) return st;
+    if (w) {
+        unsigned int z = 0;
+        cudaMemcpyToSymbol(g_error_word, &z, sizeof(z));
+        if (w & kErrTimeout) return fail(TDA_ERR_TIMEOUT, "a device-side bounded wait expired (word %#x)", w);
+        return fail(TDA_ERR_CUDA, "device reported an inconsistent launch (word %#x)", w);
+    }
+    return TDA_OK;
+}
+
+}  // extern "C"

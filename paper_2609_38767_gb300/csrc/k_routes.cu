@@ -1,0 +1,311 @@
+// k_routes.cu -- the materialised route (b) and the factorised Gram route (c)
+// (Sec. 3.2 "FLOP-aware routing", App. A.4, Table 2), CUDA-core versions.
+//
+// Route (b): G = DW = g a^T, G[r][c] = sum_t B[t][r] A[t][c] (Eq. 1), then
+//   projection: Phi = scale * S_out^T G S_in   (same result as Eq. 2), or
+//   exact similarity: <G_q, G_i>_F.
+// Route (c): <DW_q, DW_i>_F = sum_{t,s} <a_t^q, a_s^i> <g_t^q, g_s^i> (Eq. 4),
+//   never forming DW.
+#include <cuda_bf16.h>
+
+#include "tda_internal.cuh"
+
+namespace tda {
+namespace {
+
+constexpr int kT = 64;   // tile edge
+constexpr int kK = 32;   // contraction chunk
+constexpr int kTh = 256;
+
+__device__ __forceinline__ float ld1(const float* p) { return __ldg(p); }
+__device__ __forceinline__ float ld1(const __nv_bfloat16* p) { return __bfloat162float(*p); }
+
+// Batched G_e = B_e^T A_e for examples e in [e0, e0+nb); G row-major d_out x d_in.
+template <typename T>
+__global__ void __launch_bounds__(kTh)
+materialize_kernel(const T* __restrict__ A, const T* __restrict__ B, int64_t e0, int64_t Tn,
+                   int64_t d_in, int64_t d_out, float* __restrict__ G) {
+    __shared__ float Bs[kK][kT + 1];
+    __shared__ float As[kK][kT + 1];
+    const int64_t e = e0 + blockIdx.z;
+    const T* Ae = A + e * Tn * d_in;
+    const T* Be = B + e * Tn * d_out;
+    float* Ge = G + (int64_t)blockIdx.z * d_out * d_in;
+    const int64_t r0 = (int64_t)blockIdx.y * kT, c0 = (int64_t)blockIdx.x * kT;
+    const int tid = threadIdx.x, ty = tid / 16, tx = tid % 16;
+    float acc[4][4] = {};
+    for (int64_t t0 = 0; t0 < Tn; t0 += kK) {
+        for (int x = tid; x < kK * kT; x += kTh) {
+            const int tt = x / kT, cc = x % kT;
+            const int64_t t = t0 + tt;
+            Bs[tt][cc] = (t < Tn && r0 + cc < d_out) ? ld1(Be + t * d_out + r0 + cc) : 0.f;
+            As[tt][cc] = (t < Tn && c0 + cc < d_in) ? ld1(Ae + t * d_in + c0 + cc) : 0.f;
+        }
+        __syncthreads();
+#pragma unroll 8
+        for (int tt = 0; tt < kK; ++tt)
+#pragma unroll
+            for (int u = 0; u < 4; ++u)
+#pragma unroll
+                for (int v = 0; v < 4; ++v)
+                    acc[u][v] = fmaf(Bs[tt][ty * 4 + u], As[tt][tx * 4 + v], acc[u][v]);
+        __syncthreads();
+    }
+#pragma unroll
+    for (int u = 0; u < 4; ++u)
+#pragma unroll
+        for (int v = 0; v < 4; ++v) {
+            const int64_t r = r0 + ty * 4 + u, c = c0 + tx * 4 + v;
+            if (r < d_out && c < d_in) Ge[r * d_in + c] = acc[u][v];
+        }
+}
+
+__device__ __forceinline__ float signed_term(uint64_t w, int bit, float v) {
+    return ((w >> bit) & 1u) ? -v : v;
+}
+
+// X_e[r][j] = sum_c G_e[r][c] S_in[c][j]   (rows r of d_out, columns j of k_in)
+__global__ void __launch_bounds__(kTh)
+sign_right_kernel(const float* __restrict__ G, int64_t d_out, int64_t d_in, int k_in,
+                  uint64_t key, int kind, float* __restrict__ X) {
+    __shared__ float Gs[kT][kT + 1];  // [r][c]
+    __shared__ uint64_t Ws[kT];
+    const float* Ge = G + (int64_t)blockIdx.z * d_out * d_in;
+    float* Xe = X + (int64_t)blockIdx.z * d_out * k_in;
+    const int64_t r0 = (int64_t)blockIdx.y * kT;
+    const int j0 = blockIdx.x * kT;
+    const int tid = threadIdx.x, ty = tid / 16, tx = tid % 16;
+    float acc[4][4] = {};
+    for (int64_t c0 = 0; c0 < d_in; c0 += kT) {
+        for (int x = tid; x < kT * kT; x += kTh) {
+            const int rr = x / kT, cc = x % kT;
+            Gs[rr][cc] = (r0 + rr < d_out && c0 + cc < d_in) ? Ge[(r0 + rr) * d_in + c0 + cc] : 0.f;
+        }
+        if (tid < kT) Ws[tid] = sign_word(key, (uint32_t)(j0 + tid), (uint64_t)(c0 >> 6));
+        __syncthreads();
+        if (kind == TDA_PROJ_RADEMACHER) {
+            uint64_t w[4];
+#pragma unroll
+            for (int v = 0; v < 4; ++v) w[v] = Ws[tx * 4 + v];
+            for (int cc = 0; cc < kT; ++cc)
+#pragma unroll
+                for (int u = 0; u < 4; ++u) {
+                    const float g = Gs[ty * 4 + u][cc];
+#pragma unroll
+                    for (int v = 0; v < 4; ++v) acc[u][v] += signed_term(w[v], cc, g);
+                }
+        } else {
+#pragma unroll
+            for (int v = 0; v < 4; ++v) {
+                const int64_t j = j0 + tx * 4 + v;
+                if (j >= c0 && j < c0 + kT)
+#pragma unroll
+                    for (int u = 0; u < 4; ++u) acc[u][v] += Gs[ty * 4 + u][j - c0];
+            }
+        }
+        __syncthreads();
+    }
+#pragma unroll
+    for (int u = 0; u < 4; ++u)
+#pragma unroll
+        for (int v = 0; v < 4; ++v) {
+            const int64_t r = r0 + ty * 4 + u;
+            const int j = j0 + tx * 4 + v;
+            if (r < d_out && j < k_in) Xe[r * k_in + j] = acc[u][v];
+        }
+}
+
+// Phi_e[i][j] = scale * sum_r S_out[r][i] X_e[r][j]
+__global__ void __launch_bounds__(kTh)
+sign_left_kernel(const float* __restrict__ X, int64_t d_out, int k_in, int k_out, uint64_t key,
+                 int kind, float scale, int64_t e0, float* __restrict__ phi, int64_t ld_phi) {
+    __shared__ float Xs[kT][kT + 1];  // [r][j]
+    __shared__ uint64_t Ws[kT];
+    const float* Xe = X + (int64_t)blockIdx.z * d_out * k_in;
+    const int i0 = blockIdx.y * kT, j0 = blockIdx.x * kT;
+    const int tid = threadIdx.x, ty = tid / 16, tx = tid % 16;
+    float acc[4][4] = {};
+    for (int64_t rb = 0; rb < d_out; rb += kT) {
+        for (int x = tid; x < kT * kT; x += kTh) {
+            const int rr = x / kT, jj = x % kT;
+            Xs[rr][jj] = (rb + rr < d_out && j0 + jj < k_in) ? Xe[(rb + rr) * k_in + j0 + jj] : 0.f;
+        }
+        if (tid < kT) Ws[tid] = sign_word(key, (uint32_t)(i0 + tid), (uint64_t)(rb >> 6));
+        __syncthreads();
+        if (kind == TDA_PROJ_RADEMACHER) {
+            uint64_t w[4];
+#pragma unroll
+            for (int u = 0; u < 4; ++u) w[u] = Ws[ty * 4 + u];
+            for (int rr = 0; rr < kT; ++rr)
+#pragma unroll
+                for (int v = 0; v < 4; ++v) {
+                    const float x = Xs[rr][tx * 4 + v];
+#pragma unroll
+                    for (int u = 0; u < 4; ++u) acc[u][v] += signed_term(w[u], rr, x);
+                }
+        } else {
+#pragma unroll
+            for (int u = 0; u < 4; ++u) {
+                const int64_t i = i0 + ty * 4 + u;
+                if (i >= rb && i < rb + kT)
+#pragma unroll
+                    for (int v = 0; v < 4; ++v) acc[u][v] += Xs[i - rb][tx * 4 + v];
+            }
+        }
+        __syncthreads();
+    }
+    const int64_t e = e0 + blockIdx.z;
+#pragma unroll
+    for (int u = 0; u < 4; ++u)
+#pragma unroll
+        for (int v = 0; v < 4; ++v) {
+            const int i = i0 + ty * 4 + u, j = j0 + tx * 4 + v;
+            if (i < k_out && j < k_in) phi[e * ld_phi + (int64_t)i * k_in + j] = acc[u][v] * scale;
+        }
+}
+
+// Route (c): one CTA per (train i, query q) pair, 16x16 token tiles; each
+// thread owns one (t, s) pair of the tile and forms <a_t,a_s> <g_t,g_s>.
+template <typename T>
+__global__ void __launch_bounds__(kTh)
+gram_kernel(const T* __restrict__ Aq, const T* __restrict__ Bq, const T* __restrict__ At,
+            const T* __restrict__ Bt, int64_t Tn, int64_t d_in, int64_t d_out,
+            float* __restrict__ S, int64_t ld_S, float beta) {
+    constexpr int TT = 16, KC = 64;
+    __shared__ float Xq[TT][KC + 1];
+    __shared__ float Xi[TT][KC + 1];
+    __shared__ float red[kTh];
+    const int64_t i = blockIdx.x, q = blockIdx.y;
+    const int tid = threadIdx.x, tl = tid / TT, sl = tid % TT;
+    float total = 0.f;
+    for (int64_t t0 = 0; t0 < Tn; t0 += TT) {
+        for (int64_t s0 = 0; s0 < Tn; s0 += TT) {
+            float dots[2];
+            for (int side = 0; side < 2; ++side) {
+                const int64_t d = side == 0 ? d_in : d_out;
+                const T* xq = (side == 0 ? Aq + q * Tn * d_in : Bq + q * Tn * d_out);
+                const T* xi = (side == 0 ? At + i * Tn * d_in : Bt + i * Tn * d_out);
+                float acc = 0.f;
+                for (int64_t c0 = 0; c0 < d; c0 += KC) {
+                    for (int x = tid; x < TT * KC; x += kTh) {
+                        const int rr = x / KC, cc = x % KC;
+                        const int64_t c = c0 + cc;
+                        Xq[rr][cc] = (t0 + rr < Tn && c < d) ? ld1(xq + (t0 + rr) * d + c) : 0.f;
+                        Xi[rr][cc] = (s0 + rr < Tn && c < d) ? ld1(xi + (s0 + rr) * d + c) : 0.f;
+                    }
+                    __syncthreads();
+#pragma unroll 16
+                    for (int cc = 0; cc < KC; ++cc) acc = fmaf(Xq[tl][cc], Xi[sl][cc], acc);
+                    __syncthreads();
+                }
+                dots[side] = acc;
+            }
+            total = fmaf(dots[0], dots[1], total);
+        }
+    }
+    red[tid] = total;
+    __syncthreads();
+    for (int w = kTh / 2; w > 0; w >>= 1) {
+        if (tid < w) red[tid] += red[tid + w];
+        __syncthreads();
+    }
+    if (tid == 0) {
+        float* dst = S + q * ld_S + i;
+        *dst = (beta == 0.f) ? red[0] : beta * (*dst) + red[0];
+    }
+}
+
+template <typename T>
+void launch_materialize(const void* A, const void* B, int64_t e0, int64_t nb,
+                        const tda_layer_desc& L, float* G, cudaStream_t s) {
+    dim3 grid((unsigned)((L.d_in + kT - 1) / kT), (unsigned)((L.d_out + kT - 1) / kT), (unsigned)nb);
+    materialize_kernel<T><<<grid, kTh, 0, s>>>((const T*)A, (const T*)B, e0, L.T, L.d_in, L.d_out, G);
+}
+
+}  // namespace
+
+float projection_scale(const tda_layer_desc& L);
+
+size_t materialize_ws_bytes_per_example(const tda_layer_desc& L) {
+    return sizeof(float) * (size_t)(L.d_out * L.d_in + L.d_out * (int64_t)L.k_in);
+}
+
+cudaError_t launch_project_materialized(const tda_layer_desc& L, tda_dtype dt, const void* A,
+                                        const void* B, int64_t N, float* phi, int64_t ld_phi,
+                                        void* ws, size_t ws_bytes, cudaStream_t s) {
+    const size_t per = materialize_ws_bytes_per_example(L);
+    int64_t nb = (int64_t)(ws_bytes / per);
+    if (nb < 1) return cudaErrorInvalidValue;
+    if (nb > 65535) nb = 65535;
+    const uint64_t key_in = side_key(L.seed, L.layer, 0);
+    const uint64_t key_out = side_key(L.seed, L.layer, 1);
+    const float scale = projection_scale(L);
+    for (int64_t e0 = 0; e0 < N; e0 += nb) {
+        const int64_t cnt = (N - e0) < nb ? (N - e0) : nb;
+        float* G = (float*)ws;
+        float* X = G + cnt * L.d_out * L.d_in;
+        if (dt == TDA_BF16)
+            launch_materialize<__nv_bfloat16>(A, B, e0, cnt, L, G, s);
+        else
+            launch_materialize<float>(A, B, e0, cnt, L, G, s);
+        dim3 g2((unsigned)((L.k_in + kT - 1) / kT), (unsigned)((L.d_out + kT - 1) / kT), (unsigned)cnt);
+        sign_right_kernel<<<g2, kTh, 0, s>>>(G, L.d_out, L.d_in, L.k_in, key_in, L.kind, X);
+        dim3 g3((unsigned)((L.k_in + kT - 1) / kT), (unsigned)((L.k_out + kT - 1) / kT), (unsigned)cnt);
+        sign_left_kernel<<<g3, kTh, 0, s>>>(X, L.d_out, L.k_in, L.k_out, key_out, L.kind, scale, e0,
+                                            phi, ld_phi);
+        cudaError_t e = cudaGetLastError();
+        if (e != cudaSuccess) return e;
+    }
+    return cudaSuccess;
+}
+
+size_t similarity_materialize_ws_bytes(const tda_layer_desc& L, int64_t n_q, int64_t chunk) {
+    return sizeof(float) * (size_t)((n_q + chunk) * L.d_out * L.d_in);
+}
+
+cudaError_t launch_similarity_materialized(const tda_layer_desc& L, tda_dtype dt, const void* Aq,
+                                           const void* Bq, int64_t n_q, const void* At,
+                                           const void* Bt, int64_t n_t, float* S, int64_t ld_S,
+                                           float beta, void* ws, size_t ws_bytes, cudaStream_t s) {
+    const int64_t gsz = L.d_out * L.d_in;
+    const int64_t room = (int64_t)(ws_bytes / (sizeof(float) * (size_t)gsz)) - n_q;
+    if (room < 1) return cudaErrorInvalidValue;
+    int64_t chunk = room < 65535 ? room : 65535;
+    float* Gq = (float*)ws;
+    float* Gt = Gq + n_q * gsz;
+    for (int64_t q0 = 0; q0 < n_q; q0 += 65535) {
+        const int64_t cnt = (n_q - q0) < 65535 ? (n_q - q0) : 65535;
+        if (dt == TDA_BF16)
+            launch_materialize<__nv_bfloat16>(Aq, Bq, q0, cnt, L, Gq + q0 * gsz, s);
+        else
+            launch_materialize<float>(Aq, Bq, q0, cnt, L, Gq + q0 * gsz, s);
+    }
+    for (int64_t i0 = 0; i0 < n_t; i0 += chunk) {
+        const int64_t cnt = (n_t - i0) < chunk ? (n_t - i0) : chunk;
+        if (dt == TDA_BF16)
+            launch_materialize<__nv_bfloat16>(At, Bt, i0, cnt, L, Gt, s);
+        else
+            launch_materialize<float>(At, Bt, i0, cnt, L, Gt, s);
+        cudaError_t e = launch_score(Gq, TDA_F32, n_q, gsz, Gt, cnt, gsz, gsz, S + i0, ld_S, beta, s);
+        if (e != cudaSuccess) return e;
+    }
+    return cudaGetLastError();
+}
+
+cudaError_t launch_similarity_gram(const tda_layer_desc& L, tda_dtype dt, const void* Aq,
+                                   const void* Bq, int64_t n_q, const void* At, const void* Bt,
+                                   int64_t n_t, float* S, int64_t ld_S, float beta,
+                                   cudaStream_t s) {
+    if (n_q == 0 || n_t == 0) return cudaSuccess;
+    dim3 grid((unsigned)n_t, (unsigned)n_q);
+    if (dt == TDA_BF16)
+        gram_kernel<__nv_bfloat16><<<grid, kTh, 0, s>>>(
+            (const __nv_bfloat16*)Aq, (const __nv_bfloat16*)Bq, (const __nv_bfloat16*)At,
+            (const __nv_bfloat16*)Bt, L.T, L.d_in, L.d_out, S, ld_S, beta);
+    else
+        gram_kernel<float><<<grid, kTh, 0, s>>>((const float*)Aq, (const float*)Bq, (const float*)At,
+                                                (const float*)Bt, L.T, L.d_in, L.d_out, S, ld_S, beta);
+    return cudaGetLastError();
+}
+
+}  // namespace tda

@@ -1,0 +1,194 @@
+// k_score.cu -- score GEMM S = beta*S + Qhat Phi^T (gradient inner products,
+// Sec. 3.2 / Eq. 4's left side; GradDot when Qhat = Q) and per-row top-k.
+#include <float.h>
+
+#include "tda_internal.cuh"
+
+namespace tda {
+namespace {
+
+constexpr int kST = 64;   // output tile edge (queries x train)
+constexpr int kSK = 32;   // feature chunk
+constexpr int kSThreads = 256;
+
+// TQ: element type of Qhat; TA: accumulation type (double when Qhat is fp64).
+template <typename TQ, typename TA>
+__global__ void __launch_bounds__(kSThreads)
+score_kernel(const TQ* __restrict__ Q, int64_t n_q, int64_t ld_q, const float* __restrict__ P,
+             int64_t n_t, int64_t ld_p, int64_t D, float* __restrict__ S, int64_t ld_S,
+             float beta) {
+    __shared__ TA Qs[kSK][kST + 1];
+    __shared__ TA Ps[kSK][kST + 1];
+    const int tid = threadIdx.x;
+    const int64_t q0 = (int64_t)blockIdx.y * kST, i0 = (int64_t)blockIdx.x * kST;
+    const int ty = tid / 16, tx = tid % 16;
+    TA acc[4][4];
+#pragma unroll
+    for (int a = 0; a < 4; ++a)
+#pragma unroll
+        for (int b = 0; b < 4; ++b) acc[a][b] = (TA)0;
+
+    for (int64_t f0 = 0; f0 < D; f0 += kSK) {
+        for (int e = tid; e < kSK * kST; e += kSThreads) {
+            const int rr = e / kSK, ff = e % kSK;
+            const int64_t f = f0 + ff;
+            const int64_t q = q0 + rr, i = i0 + rr;
+            Qs[ff][rr] = (q < n_q && f < D) ? (TA)Q[q * ld_q + f] : (TA)0;
+            Ps[ff][rr] = (i < n_t && f < D) ? (TA)P[i * ld_p + f] : (TA)0;
+        }
+        __syncthreads();
+#pragma unroll 8
+        for (int ff = 0; ff < kSK; ++ff) {
+            TA a[4], b[4];
+#pragma unroll
+            for (int u = 0; u < 4; ++u) a[u] = Qs[ff][ty * 4 + u];
+#pragma unroll
+            for (int u = 0; u < 4; ++u) b[u] = Ps[ff][tx * 4 + u];
+#pragma unroll
+            for (int u = 0; u < 4; ++u)
+#pragma unroll
+                for (int v = 0; v < 4; ++v) acc[u][v] += a[u] * b[v];
+        }
+        __syncthreads();
+    }
+#pragma unroll
+    for (int u = 0; u < 4; ++u)
+#pragma unroll
+        for (int v = 0; v < 4; ++v) {
+            const int64_t q = q0 + ty * 4 + u, i = i0 + tx * 4 + v;
+            if (q < n_q && i < n_t) {
+                float* dst = S + q * ld_S + i;
+                *dst = (beta == 0.f) ? (float)acc[u][v] : (float)((TA)beta * (TA)(*dst) + acc[u][v]);
+            }
+        }
+}
+
+// ---------------------------------------------------------------------------
+// Top-k. Each entry gets a 64-bit key whose descending order is "score
+// descending, then index ascending": the high word maps the float to an
+// order-preserving unsigned (NaN largest, -0 folded into +0), the low word is
+// ~index. Keys are distinct, so the k-th largest key splits the row exactly.
+// One CTA per row: 8 passes of an 8-bit radix select find that key, the k
+// winners are gathered and bitonic-sorted in shared memory.
+// ---------------------------------------------------------------------------
+constexpr int kTopThreads = 512;
+constexpr int kTopMaxK = 1024;
+
+__device__ __forceinline__ uint64_t topk_key(float v, int64_t i) {
+    uint32_t u = __float_as_uint(v);
+    uint32_t o;
+    if (v != v)
+        o = 0xFFFFFFFFu;
+    else if (v == 0.f)
+        o = 0x80000000u;
+    else
+        o = (u & 0x80000000u) ? ~u : (u | 0x80000000u);
+    return ((uint64_t)o << 32) | (uint64_t)(~(uint32_t)i);
+}
+
+__global__ void __launch_bounds__(kTopThreads)
+topk_kernel(const float* __restrict__ S, int64_t n_t, int64_t ld_S, int32_t k,
+            int32_t* __restrict__ idx, float* __restrict__ val) {
+    __shared__ unsigned int hist[256];
+    __shared__ uint64_t sel[kTopMaxK];
+    __shared__ uint64_t s_prefix, s_mask;
+    __shared__ int s_remaining;
+    __shared__ unsigned int s_count;
+    const int64_t q = blockIdx.x;
+    const float* row = S + q * ld_S;
+    const int tid = threadIdx.x;
+    if (tid == 0) {
+        s_prefix = 0;
+        s_mask = 0;
+        s_remaining = k;
+        s_count = 0;
+    }
+    for (int pass = 0; pass < 8; ++pass) {
+        const int shift = 56 - 8 * pass;
+        for (int b = tid; b < 256; b += kTopThreads) hist[b] = 0;
+        __syncthreads();
+        const uint64_t prefix = s_prefix, mask = s_mask;
+        for (int64_t i = tid; i < n_t; i += kTopThreads) {
+            const uint64_t key = topk_key(row[i], i);
+            if ((key & mask) == prefix) atomicAdd(&hist[(key >> shift) & 255u], 1u);
+        }
+        __syncthreads();
+        if (tid == 0) {
+            int rem = s_remaining;
+            unsigned int cum = 0;
+            int digit = 0;
+            for (int b = 255; b >= 0; --b) {
+                if (cum + hist[b] >= (unsigned)rem) {
+                    digit = b;
+                    break;
+                }
+                cum += hist[b];
+            }
+            s_remaining = rem - (int)cum;
+            s_prefix = prefix | ((uint64_t)digit << shift);
+            s_mask = mask | ((uint64_t)255 << shift);
+        }
+        __syncthreads();
+    }
+    const uint64_t kth = s_prefix;  // the k-th largest key
+    int P = 1;
+    while (P < k) P <<= 1;
+    for (int e = tid; e < P; e += kTopThreads) sel[e] = 0;
+    __syncthreads();
+    for (int64_t i = tid; i < n_t; i += kTopThreads) {
+        const uint64_t key = topk_key(row[i], i);
+        if (key >= kth) {
+            const unsigned int slot = atomicAdd(&s_count, 1u);
+            if (slot < (unsigned)k) sel[slot] = key;
+        }
+    }
+    __syncthreads();
+    // bitonic sort, descending
+    for (int size = 2; size <= P; size <<= 1) {
+        for (int stride = size >> 1; stride > 0; stride >>= 1) {
+            for (int e = tid; e < P; e += kTopThreads) {
+                const int partner = e ^ stride;
+                if (partner > e) {
+                    const bool desc = ((e & size) == 0);
+                    const uint64_t a = sel[e], b = sel[partner];
+                    if (desc ? (a < b) : (a > b)) {
+                        sel[e] = b;
+                        sel[partner] = a;
+                    }
+                }
+            }
+            __syncthreads();
+        }
+    }
+    for (int e = tid; e < k; e += kTopThreads) {
+        const uint32_t i = ~(uint32_t)(sel[e] & 0xFFFFFFFFu);
+        const bool ok = (int64_t)i < n_t;  // always true when exactly k keys were selected
+        idx[q * k + e] = ok ? (int32_t)i : -1;
+        if (val) val[q * k + e] = ok ? row[i] : __int_as_float(0x7fc00000);
+    }
+}
+
+}  // namespace
+
+cudaError_t launch_score(const void* Qhat, tda_dtype qdt, int64_t n_q, int64_t ld_q,
+                         const float* Phi, int64_t n_t, int64_t ld_phi, int64_t D, float* S,
+                         int64_t ld_S, float beta, cudaStream_t s) {
+    if (n_q == 0 || n_t == 0) return cudaSuccess;
+    dim3 grid((unsigned)((n_t + kST - 1) / kST), (unsigned)((n_q + kST - 1) / kST));
+    if (qdt == TDA_F64)
+        score_kernel<double, double><<<grid, kSThreads, 0, s>>>(
+            (const double*)Qhat, n_q, ld_q, Phi, n_t, ld_phi, D, S, ld_S, beta);
+    else
+        score_kernel<float, float><<<grid, kSThreads, 0, s>>>(
+            (const float*)Qhat, n_q, ld_q, Phi, n_t, ld_phi, D, S, ld_S, beta);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_topk(const float* S, int64_t n_q, int64_t n_t, int64_t ld_S, int32_t k,
+                        int32_t* idx, float* val, cudaStream_t s) {
+    if (n_q == 0) return cudaSuccess;
+    topk_kernel<<<(unsigned)n_q, kTopThreads, 0, s>>>(S, n_t, ld_S, k, idx, val);
+    return cudaGetLastError();
+}
+
+}  // namespace tda

@@ -1,0 +1,107 @@
+// tda_internal.cuh -- internal declarations shared by the CUDA translation
+// units of libtda.so (kernels and the C-ABI layer). Not installed.
+#pragma once
+
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+#include "../../include/tda.h"
+
+namespace tda {
+
+// ---------------------------------------------------------------------------
+// Counter-based Rademacher signs (App. A.2: Rademacher maps, two sides with
+// distinct seeds derived from one per-layer base seed).
+//
+// side_key(seed, layer, side) = mix(mix(seed + G*(layer+1)) + G*(side+1))
+// entry (r, c) of a side's d x k sign matrix = bit (r mod 64) of
+//   mix(side_key + G*(((c << 32) | (r >> 6)) + 1)),  set bit -> -1.
+// mix is the SplitMix64 output function. One 64-bit word therefore holds the
+// signs of 64 consecutive rows of one column: exactly one 128-byte row of a
+// K-major bf16 operand tile with a 64-wide K chunk.
+// ---------------------------------------------------------------------------
+constexpr uint64_t kGamma = 0x9E3779B97F4A7C15ull;
+
+__host__ __device__ __forceinline__ uint64_t mix64(uint64_t z) {
+    z = (z ^ (z >> 30)) * 0xBF58476D1CE4E5B9ull;
+    z = (z ^ (z >> 27)) * 0x94D049BB133111EBull;
+    return z ^ (z >> 31);
+}
+
+__host__ __device__ __forceinline__ uint64_t side_key(uint64_t seed, uint32_t layer, int side) {
+    uint64_t base = mix64(seed + kGamma * ((uint64_t)layer + 1u));
+    return mix64(base + kGamma * ((uint64_t)(uint32_t)side + 1u));
+}
+
+// Sign word of column c for rows [64*rb, 64*rb + 64).
+__host__ __device__ __forceinline__ uint64_t sign_word(uint64_t key, uint32_t c, uint64_t rb) {
+    return mix64(key + kGamma * ((((uint64_t)c << 32) | rb) + 1u));
+}
+
+// Error bits written by kernels into the device error word.
+enum : unsigned int {
+    kErrTimeout = 1u,    // a bounded mbarrier / flag wait expired
+    kErrBadLaunch = 2u,  // a kernel found its launch geometry inconsistent
+};
+
+// Device address of the library's error word on the current device.
+unsigned int* device_error_word();
+
+// Thread-local error message helpers (api.cu).
+tda_status fail(tda_status st, const char* fmt, ...);
+tda_status cuda_check(cudaError_t e, const char* what);
+
+// ---------------------------------------------------------------------------
+// Kernel launchers (one per translation unit). All return cudaError_t from
+// cudaGetLastError() after the launch; arguments are validated by the caller.
+// ---------------------------------------------------------------------------
+
+cudaError_t launch_proj_entries(uint64_t key, int kind, int64_t rows, int32_t cols, int8_t* out,
+                                cudaStream_t s);
+
+// Generic (SIMT) projection, any shape, fp32 or bf16 inputs.
+cudaError_t launch_project_simt(const tda_layer_desc& L, tda_dtype dt, const void* A, const void* B,
+                                int64_t N, float* phi, int64_t ld_phi, cudaStream_t s);
+
+// tcgen05 / TMA projection for bf16 inputs. Returns cudaErrorNotSupported if
+// the shape has no tensor-core instantiation (caller falls back to SIMT).
+bool project_tc_supported(const tda_layer_desc& L, const void* A, const void* B);
+cudaError_t launch_project_tc(const tda_layer_desc& L, const void* A, const void* B, int64_t N,
+                              float* phi, int64_t ld_phi, unsigned int* err, cudaStream_t s);
+
+// Route (b): materialise G = B^T A for nb examples into ws, then project it.
+size_t materialize_ws_bytes_per_example(const tda_layer_desc& L);
+cudaError_t launch_project_materialized(const tda_layer_desc& L, tda_dtype dt, const void* A,
+                                        const void* B, int64_t N, float* phi, int64_t ld_phi,
+                                        void* ws, size_t ws_bytes, cudaStream_t s);
+
+// Unprojected similarity, routes (b) and (c).
+size_t similarity_materialize_ws_bytes(const tda_layer_desc& L, int64_t n_q, int64_t chunk);
+cudaError_t launch_similarity_materialized(const tda_layer_desc& L, tda_dtype dt, const void* Aq,
+                                           const void* Bq, int64_t n_q, const void* At,
+                                           const void* Bt, int64_t n_t, float* S, int64_t ld_S,
+                                           float beta, void* ws, size_t ws_bytes, cudaStream_t s);
+cudaError_t launch_similarity_gram(const tda_layer_desc& L, tda_dtype dt, const void* Aq,
+                                   const void* Bq, int64_t n_q, const void* At, const void* Bt,
+                                   int64_t n_t, float* S, int64_t ld_S, float beta, cudaStream_t s);
+
+// Preconditioner.
+cudaError_t launch_pc_fit(int64_t D, tda_dtype sdt, void* state, const float* phi, int64_t n,
+                          int64_t ld, cudaStream_t s);
+cudaError_t launch_pc_factor(int64_t D, tda_dtype sdt, void* state, int64_t n_total,
+                             double lambda_abs, double lambda_rel, cudaStream_t s);
+cudaError_t launch_pc_apply(int64_t D, tda_dtype sdt, const void* state, const float* q,
+                            int64_t n_q, int64_t ld_q, void* qhat, int64_t ld_qhat,
+                            cudaStream_t s);
+
+// Scores and ranking.
+cudaError_t launch_score(const void* Qhat, tda_dtype qdt, int64_t n_q, int64_t ld_q,
+                         const float* Phi, int64_t n_t, int64_t ld_phi, int64_t D, float* S,
+                         int64_t ld_S, float beta, cudaStream_t s);
+cudaError_t launch_topk(const float* S, int64_t n_q, int64_t n_t, int64_t ld_S, int32_t k,
+                        int32_t* idx, float* val, cudaStream_t s);
+
+// State header layout of the preconditioner (doubles).
+enum { kPcLambda = 0, kPcMeanEig = 1, kPcFailedPivot = 2, kPcNTotal = 3, kPcHeaderDoubles = 8 };
+
+}  // namespace tda

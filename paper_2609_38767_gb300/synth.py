@@ -137,3 +137,41 @@ def to_f64(x: np.ndarray, dtype: str) -> np.ndarray:
     if dtype == "bf16":
         return bf16_bits_to_f32(x).astype(np.float64)
     return np.asarray(x, dtype=np.float32).astype(np.float64)
+
+
+# ------------------------------------------------------------------ device side
+_synth_lib = None
+
+
+def _load_device_lib():
+    global _synth_lib
+    if _synth_lib is None:
+        import ctypes
+        import os
+
+        path = os.path.join(os.path.dirname(os.path.abspath(__file__)), "libtda_synth.so")
+        if not os.path.exists(path):
+            raise ImportError(f"{path} is missing: run paper_2609_38767_gb300.build.build() first")
+        lib = ctypes.CDLL(path)
+        u64, i64, i32 = ctypes.c_uint64, ctypes.c_int64, ctypes.c_int32
+        lib.tda_synth_fill.restype = i32
+        lib.tda_synth_fill.argtypes = [ctypes.c_void_p, i32, i32, u64, u64, i64, i64, i64, i64,
+                                       ctypes.c_float, u64, u64, u64, ctypes.c_void_p]
+        _synth_lib = lib
+    return _synth_lib
+
+
+def fill_device(out, seed: int, stream: int, n: int, T: int, d: int, sigma: float = 1.0,
+                dist: int = DIST_NORMAL, e0: int = 0, mask_p: float = 0.0,
+                mask_seed: int = SEED_MASK, mask_stream: int = 0, cuda_stream=None) -> None:
+    """Fill a device tensor (fp32 or bf16, n*T*d elements) with the generator's values."""
+    import torch
+
+    dt = {torch.float32: 0, torch.bfloat16: 1}[out.dtype]
+    assert out.is_cuda and out.is_contiguous() and out.numel() >= n * T * d
+    s = cuda_stream if cuda_stream is not None else torch.cuda.current_stream().cuda_stream
+    rc = _load_device_lib().tda_synth_fill(out.data_ptr(), dt, dist, seed, stream, e0, n, T, d,
+                                           float(sigma), mask_seed, mask_stream,
+                                           mask_threshold(mask_p), s)
+    if rc != 0:
+        raise RuntimeError(f"tda_synth_fill failed ({rc})")

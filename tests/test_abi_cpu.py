@@ -1,0 +1,111 @@
+"""C-ABI checks that need no GPU: the library builds and loads, exports every
+declared symbol, validates arguments on the host, and its host-only route
+cost model agrees with the oracle's (App. A.4, Table 2)."""
+import ctypes
+import os
+import re
+
+import numpy as np
+import pytest
+
+import paper_2609_38767_gb300 as tda
+from paper_2609_38767_gb300 import build as tbuild
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+
+
+@pytest.fixture(scope="module")
+def libs():
+    return tbuild.build()
+
+
+def _declared(header):
+    text = open(os.path.join(ROOT, "include", header)).read()
+    text = re.sub(r"/\*.*?\*/", "", text, flags=re.S)
+    return sorted(set(re.findall(r"\b(tda_\w+)\s*\(", text)))
+
+
+@pytest.mark.parametrize("header,lib", [("tda.h", "libtda.so"), ("tda_synth.h", "libtda_synth.so")])
+def test_every_declared_symbol_is_exported(libs, header, lib):
+    so = ctypes.CDLL(libs[lib])
+    names = _declared(header)
+    assert names, header
+    missing = [n for n in names if not hasattr(so, n)]
+    assert not missing, missing
+
+
+def test_layer_desc_layout_matches_header():
+    assert ctypes.sizeof(tda.LayerDesc) == 48
+    assert tda.LayerDesc.seed.offset == 32 and tda.LayerDesc.kind.offset == 44
+
+
+def test_version_and_state_bytes(libs):
+    assert tda.tda_version() >= 100
+    assert tda.tda_precondition_state_bytes(256, tda.TDA_F64) == 64 + 256 * 256 * 8
+    assert tda.tda_precondition_state_bytes(10, tda.TDA_F32) == 64 + 400
+    assert tda.tda_precondition_state_bytes(0, tda.TDA_F32) == 0
+
+
+def _err(fn, *a, **k):
+    with pytest.raises(tda.TdaError) as e:
+        fn(*a, **k)
+    return e.value.status
+
+
+def test_host_validation_rejects_bad_arguments(libs):
+    L = tda.LayerDesc(64, 64, 8, 16, 16)
+    s = 0  # never reached: validation fails first
+    assert _err(tda.tda_project, L, tda.TDA_BF16, None, None, 4, None, 256, stream=s) == tda.TDA_ERR_INVALID_ARG
+    assert _err(tda.tda_project, L, tda.TDA_BF16, 16, 16, 4, 16, 100, stream=s) == tda.TDA_ERR_INVALID_ARG
+    assert _err(tda.tda_project, L, tda.TDA_BF16, 8, 16, 4, 16, 256, stream=s) == tda.TDA_ERR_INVALID_ARG
+    assert _err(tda.tda_project, L, 7, 16, 16, 4, 16, 256, stream=s) == tda.TDA_ERR_INVALID_ARG
+    bad = tda.LayerDesc(60, 64, 8, 16, 16)  # d_in not a multiple of 8 for bf16
+    assert _err(tda.tda_project, bad, tda.TDA_BF16, 16, 16, 4, 16, 256, stream=s) == tda.TDA_ERR_INVALID_ARG
+    ident = tda.LayerDesc(64, 64, 8, 16, 16, kind=tda.TDA_PROJ_IDENTITY)
+    assert _err(tda.tda_project, ident, tda.TDA_F32, 16, 16, 4, 16, 256, stream=s) == tda.TDA_ERR_INVALID_ARG
+    assert _err(tda.tda_project, L, tda.TDA_BF16, 16, 16, 4, 16, 256, route=tda.TDA_ROUTE_MATERIALIZE,
+                ws=None, ws_bytes=0, stream=s) == tda.TDA_ERR_WORKSPACE
+    assert _err(tda.tda_project, L, tda.TDA_BF16, 16, 16, 4, 16, 256, route=tda.TDA_ROUTE_GRAM,
+                stream=s) == tda.TDA_ERR_UNSUPPORTED
+    assert _err(tda.tda_topk, 16, 2, 10, 10, 11, 16, stream=s) == tda.TDA_ERR_INVALID_ARG
+    assert _err(tda.tda_topk, 16, 2, 10, 10, 0, 16, stream=s) == tda.TDA_ERR_INVALID_ARG
+    assert _err(tda.tda_score, 16, tda.TDA_BF16, 2, 8, 16, 3, 8, 8, 16, 3, stream=s) == tda.TDA_ERR_INVALID_ARG
+    assert _err(tda.tda_score, 16, tda.TDA_F32, 2, 4, 16, 3, 8, 8, 16, 3, stream=s) == tda.TDA_ERR_INVALID_ARG
+    assert _err(tda.tda_precondition, 9, 8, tda.TDA_F64, 16, stream=s) == tda.TDA_ERR_INVALID_ARG
+    assert _err(tda.tda_precondition, tda.TDA_PC_FACTOR, 8, tda.TDA_F64, 16, n_total=0, lambda_abs=1.0,
+                stream=s) == tda.TDA_ERR_INVALID_ARG
+    assert _err(tda.tda_precondition, tda.TDA_PC_FACTOR, 8, tda.TDA_F64, 16, n_total=4, stream=s) \
+        == tda.TDA_ERR_INVALID_ARG
+    assert _err(tda.tda_proj_entries, 0, 0, 2, 0, 4, 4, 16, stream=s) == tda.TDA_ERR_INVALID_ARG
+    assert _err(tda.tda_route_set_model, 1) == tda.TDA_ERR_INVALID_ARG
+    assert _err(tda.tda_route_calibrate, None, 0, stream=s) == tda.TDA_ERR_WORKSPACE
+    assert "ws" in tda.tda_last_error()
+
+
+SHAPES = [
+    # (n1, n2, T, d_in, d_out, k_in, k_out)
+    (1, 8, 32, 1024, 1024, 64, 64), (1, 8, 2048, 1024, 1024, 64, 64), (64, 4096, 512, 2048, 8192, 32, 32),
+    (128, 2 ** 24 // 8, 8, 8192, 8192, 64, 64), (128, 2 ** 24 // 8192, 8192, 8192, 8192, 64, 64),
+    (8, 64, 32, 256, 256, 16, 16), (3, 5, 1, 24, 40, 8, 8), (512, 16384, 2048, 12288, 49152, 128, 128),
+]
+
+
+@pytest.mark.parametrize("shape", SHAPES)
+@pytest.mark.parametrize("op", [tda.TDA_OP_PROJECT, tda.TDA_OP_SIMILARITY_PROJECTED, tda.TDA_OP_SIMILARITY_EXACT])
+def test_route_flop_model_matches_oracle(libs, orc, shape, op):
+    n1, n2, T, di, do, ki, ko = shape
+    L = tda.LayerDesc(di, do, T, ki, ko)
+    chosen, cost = tda.tda_route(L, op, n1, n2, tda.TDA_BF16)
+    best, ocost = orc.route_costs(op, n1, n2, T, di, do, ki, ko)
+    assert chosen == best
+    np.testing.assert_allclose(cost, ocost, rtol=1e-12)
+
+
+def test_workspace_sizes(libs):
+    L = tda.LayerDesc(256, 128, 32, 16, 16)
+    assert tda.tda_workspace_size(tda.TDA_OP_PROJECT, L, tda.TDA_F32, 10, 0, tda.TDA_ROUTE_FACTORED) == 0
+    assert tda.tda_workspace_size(tda.TDA_OP_PROJECT, L, tda.TDA_F32, 10, 0,
+                                  tda.TDA_ROUTE_MATERIALIZE) == 4 * (128 * 256 + 128 * 16)
+    assert tda.tda_workspace_size(tda.TDA_OP_SIMILARITY_EXACT, L, tda.TDA_F32, 3, 9,
+                                  tda.TDA_ROUTE_MATERIALIZE) == 4 * 4 * 128 * 256
+    assert tda.tda_workspace_size(tda.TDA_OP_SIMILARITY_EXACT, L, tda.TDA_F32, 3, 9, tda.TDA_ROUTE_GRAM) == 0

@@ -1,0 +1,267 @@
+"""GPU parity: every entry point of libtda.so, called through the C ABI, against
+the fp64 oracle on the same seeded inputs. Tolerances: projected features and
+score matrices within a relative Frobenius error of 1e-5 for fp32 factors and
+2e-2 for bf16 factors (fp32 accumulation); sign entries, indices and top-k
+bit-exact."""
+import numpy as np
+import pytest
+import torch
+
+import paper_2609_38767_gb300 as tda
+from paper_2609_38767_gb300 import build as tbuild
+from paper_2609_38767_gb300 import synth
+
+pytestmark = pytest.mark.gpu
+
+TOL = {"f32": 1e-5, "bf16": 2e-2}
+
+
+@pytest.fixture(scope="module")
+def dev():
+    assert torch.cuda.is_available(), "GPU tests need a CUDA device"
+    tbuild.build()
+    tda.load()
+    return torch.device("cuda:0")
+
+
+def rel_fro(x, ref):
+    x = np.asarray(x, dtype=np.float64)
+    ref = np.asarray(ref, dtype=np.float64)
+    return float(np.linalg.norm(x - ref) / max(np.linalg.norm(ref), 1e-300))
+
+
+def make_factors(n, T, d_in, d_out, dtype, stream, sigma_b=0.1, mask_p=0.0, dist=0, e0=0, query=False):
+    off = synth.QUERY_STREAM_OFFSET if query else 0
+    ms = 1000 if query else 0
+    A = synth.factors(synth.SEED_A, stream + off, n, T, d_in, 1.0, dist, e0, dtype, mask_p, mask_stream=ms)
+    B = synth.factors(synth.SEED_B, stream + off, n, T, d_out, sigma_b, 0, e0, dtype, mask_p, mask_stream=ms)
+    return A, B
+
+
+def to_dev(x, dtype, device):
+    if dtype == "bf16":
+        return torch.from_numpy(x.view(np.int16)).view(torch.bfloat16).to(device)
+    return torch.from_numpy(x).to(device)
+
+
+TD = {"f32": tda.TDA_F32, "bf16": tda.TDA_BF16}
+
+
+def gpu_project(L, dtype, A, B, N, route, device, ld=None):
+    D = L.k_in * L.k_out
+    ld = ld or D
+    phi = torch.full((N, ld), float("nan"), dtype=torch.float32, device=device)
+    ws, wsb = None, 0
+    if route == tda.TDA_ROUTE_MATERIALIZE:
+        wsb = tda.tda_workspace_size(tda.TDA_OP_PROJECT, L, TD[dtype], N, 0, route) * min(N, 3)
+        ws = torch.empty(wsb, dtype=torch.uint8, device=device)
+    tda.tda_project(L, TD[dtype], A, B, N, phi, ld, route, ws, wsb)
+    tda.tda_device_status()
+    return phi[:, :D].cpu().numpy().reshape(N, L.k_out, L.k_in), phi
+
+
+# ------------------------------------------------------------------ generator and signs
+def test_device_generator_matches_numpy(dev):
+    for dtype, dist, mask in [("f32", 0, 0.0), ("bf16", 0, 0.01), ("bf16", 1, 0.0), ("f32", 1, 0.05)]:
+        n, T, d = 3, 37, 48
+        ref = synth.factors(5, 7, n, T, d, 0.37, dist, 11, dtype, mask)
+        out = torch.empty(n * T * d, dtype=torch.bfloat16 if dtype == "bf16" else torch.float32, device=dev)
+        synth.fill_device(out, 5, 7, n, T, d, 0.37, dist, 11, mask)
+        got = out.cpu()
+        got = got.view(torch.int16).numpy().view(np.uint16) if dtype == "bf16" else got.numpy()
+        np.testing.assert_array_equal(got.reshape(ref.shape), ref)
+
+
+@pytest.mark.parametrize("rows,cols,side,layer", [(300, 48, 0, 0), (4096, 64, 1, 3), (130, 128, 0, 223),
+                                                  (64, 16, 1, 7)])
+def test_proj_entries_bit_exact(dev, orc, rows, cols, side, layer):
+    out = torch.zeros(rows * cols, dtype=torch.int8, device=dev)
+    tda.tda_proj_entries(12345, layer, side, 0, rows, cols, out)
+    np.testing.assert_array_equal(out.cpu().numpy().reshape(rows, cols),
+                                  orc.proj_entries(12345, layer, side, rows, cols))
+    ident = torch.zeros(40 * 40, dtype=torch.int8, device=dev)
+    tda.tda_proj_entries(0, 0, 0, 1, 40, 40, ident)
+    np.testing.assert_array_equal(ident.cpu().numpy().reshape(40, 40), np.eye(40, dtype=np.int8))
+
+
+# ------------------------------------------------------------------ projection
+PROJ_CASES = [
+    # (N, T, d_in, d_out, k_in, k_out, dtype, kind)
+    (64, 32, 256, 256, 16, 16, "f32", 0),        # the 256x256 fp32 layer, k = 16
+    (5, 45, 200, 136, 32, 48, "bf16", 0),        # ragged T, d and k
+    (3, 130, 512, 1024, 32, 32, "bf16", 0),      # T over one 128-token tile
+    (4, 19, 96, 160, 80, 72, "f32", 0),          # k over one 64-wide tile
+    (2, 7, 24, 16, 24, 16, "f32", 1),            # identity map: Phi = DW
+    (3, 64, 256, 512, 128, 64, "bf16", 0),       # wide k
+    (2, 257, 128, 128, 64, 64, "bf16", 0),       # tokens spanning 3 tiles
+]
+
+
+@pytest.mark.parametrize("case", PROJ_CASES)
+@pytest.mark.parametrize("route", [tda.TDA_ROUTE_FACTORED, tda.TDA_ROUTE_MATERIALIZE])
+def test_project_matches_oracle(dev, orc, case, route):
+    N, T, di, do, ki, ko, dtype, kind = case
+    A, B = make_factors(N, T, di, do, dtype, stream=3, mask_p=0.02)
+    L = tda.LayerDesc(di, do, T, ki, ko, seed=99, layer=5, kind=kind)
+    got, _ = gpu_project(L, dtype, to_dev(A, dtype, dev), to_dev(B, dtype, dev), N, route, dev)
+    ref = orc.project(synth.to_f64(A, dtype), synth.to_f64(B, dtype), ki, ko, 99, 5, kind)
+    err = rel_fro(got, ref)
+    assert err <= TOL[dtype], err
+    for n in range(N):  # per example as well
+        assert rel_fro(got[n], ref[n]) <= TOL[dtype]
+
+
+def test_project_leading_dimension_and_edge_sizes(dev, orc):
+    N, T, di, do, ki, ko = 4, 20, 64, 32, 16, 8
+    A, B = make_factors(N, T, di, do, "f32", stream=4)
+    L = tda.LayerDesc(di, do, T, ki, ko, seed=1, layer=2)
+    got, phi = gpu_project(L, "f32", to_dev(A, "f32", dev), to_dev(B, "f32", dev), N,
+                           tda.TDA_ROUTE_FACTORED, dev, ld=200)
+    assert torch.isnan(phi[:, ki * ko:]).all()  # untouched padding
+    ref = orc.project(synth.to_f64(A, "f32"), synth.to_f64(B, "f32"), ki, ko, 1, 2)
+    assert rel_fro(got, ref) <= 1e-5
+    # T = 0: DW = 0; N = 0: nothing to do
+    L0 = tda.LayerDesc(di, do, 0, ki, ko)
+    phi0 = torch.full((3, ki * ko), 7.0, device=dev)
+    tda.tda_project(L0, tda.TDA_F32, None, None, 3, phi0, ki * ko)
+    assert (phi0 == 0).all()
+    tda.tda_project(L, tda.TDA_F32, None, None, 0, None, ki * ko)
+    tda.tda_device_status()
+
+
+# ------------------------------------------------------------------ exact similarity
+@pytest.mark.parametrize("dtype", ["f32", "bf16"])
+@pytest.mark.parametrize("route", [tda.TDA_ROUTE_GRAM, tda.TDA_ROUTE_MATERIALIZE, tda.TDA_ROUTE_AUTO])
+def test_similarity_exact_matches_oracle(dev, orc, dtype, route):
+    nq, nt, T, di, do = 3, 5, 21, 40, 24
+    Aq, Bq = make_factors(nq, T, di, do, dtype, stream=6, query=True)
+    At, Bt = make_factors(nt, T, di, do, dtype, stream=6)
+    L = tda.LayerDesc(di, do, T, 1, 1)
+    S = torch.full((nq, nt + 3), 0.5, device=dev)
+    wsb = tda.tda_workspace_size(tda.TDA_OP_SIMILARITY_EXACT, L, TD[dtype], nq, nt, route) * 2
+    ws = torch.empty(max(wsb, 1), dtype=torch.uint8, device=dev)
+    tda.tda_similarity_exact(L, TD[dtype], to_dev(Aq, dtype, dev), to_dev(Bq, dtype, dev), nq,
+                             to_dev(At, dtype, dev), to_dev(Bt, dtype, dev), nt, S, nt + 3, 1.0, route,
+                             ws, wsb)
+    tda.tda_device_status()
+    ref = orc.similarity(synth.to_f64(Aq, dtype), synth.to_f64(Bq, dtype), synth.to_f64(At, dtype),
+                         synth.to_f64(Bt, dtype)) + 0.5
+    assert rel_fro(S[:, :nt].cpu().numpy(), ref) <= TOL[dtype]
+    assert (S[:, nt:] == 0.5).all()
+
+
+# ------------------------------------------------------------------ preconditioned scores
+def _precond_pipeline(dev, orc, N, Nq, T, di, do, k, dtype, sdt, lam_abs, lam_rel, mask_p=0.0):
+    A, B = make_factors(N, T, di, do, dtype, stream=8, mask_p=mask_p)
+    Aq, Bq = make_factors(Nq, T, di, do, dtype, stream=8, mask_p=mask_p, query=True)
+    L = tda.LayerDesc(di, do, T, k, k, seed=0, layer=0)
+    D = k * k
+    _, phi = gpu_project(L, dtype, to_dev(A, dtype, dev), to_dev(B, dtype, dev), N, tda.TDA_ROUTE_FACTORED, dev)
+    _, q = gpu_project(L, dtype, to_dev(Aq, dtype, dev), to_dev(Bq, dtype, dev), Nq, tda.TDA_ROUTE_FACTORED, dev)
+    state = torch.empty(tda.tda_precondition_state_bytes(D, sdt), dtype=torch.uint8, device=dev)
+    tda.tda_precondition(tda.TDA_PC_RESET, D, sdt, state)
+    half = N // 2  # two streamed chunks
+    tda.tda_precondition(tda.TDA_PC_FIT_ACCUM, D, sdt, state, phi=phi, n=half, ld_phi=D)
+    tda.tda_precondition(tda.TDA_PC_FIT_ACCUM, D, sdt, state, phi=phi[half:], n=N - half, ld_phi=D)
+    tda.tda_precondition(tda.TDA_PC_FACTOR, D, sdt, state, n_total=N, lambda_abs=lam_abs,
+                         lambda_rel_mean_eig=lam_rel)
+    qhat = torch.empty((Nq, D), dtype=torch.float64 if sdt == tda.TDA_F64 else torch.float32, device=dev)
+    tda.tda_precondition(tda.TDA_PC_APPLY, D, sdt, state, q=q, n_q=Nq, ld_q=D, qhat=qhat, ld_qhat=D)
+    S = torch.empty((Nq, N), device=dev)
+    tda.tda_score(qhat, sdt, Nq, D, phi, N, D, D, S, N)
+    info = tda.tda_precondition_info(D, sdt, state)
+    tda.tda_device_status()
+    # oracle, end to end from the same input bits
+    fo = orc.project(synth.to_f64(A, dtype), synth.to_f64(B, dtype), k, k, 0, 0).reshape(N, D)
+    fq = orc.project(synth.to_f64(Aq, dtype), synth.to_f64(Bq, dtype), k, k, 0, 0).reshape(Nq, D)
+    F = orc.fisher(fo)
+    lam = orc.damping(F, lam_abs, lam_rel)
+    Sref = orc.score(orc.precondition(F, lam, fq), fo)
+    return S.cpu().numpy(), Sref, info, lam
+
+
+def test_preconditioned_scores_fp32_layer_fp64_state(dev, orc):
+    # d 256 -> 256, fp32, T = 32, 64 train / 8 query, k = 16, lambda = 1e-3
+    S, Sref, info, lam = _precond_pipeline(dev, orc, 64, 8, 32, 256, 256, 16, "f32", tda.TDA_F64, 1e-3, 0.0)
+    assert abs(info[0] - lam) <= 1e-12 * lam and info[2] == 0 and info[3] == 64
+    assert rel_fro(S, Sref) <= 1e-5
+
+
+def test_preconditioned_scores_bf16_fp32_state_relative_damping(dev, orc):
+    S, Sref, info, lam = _precond_pipeline(dev, orc, 96, 16, 40, 128, 192, 16, "bf16", tda.TDA_F32,
+                                           0.0, 1e-2, mask_p=0.01)
+    assert abs(info[0] - lam) <= 1e-5 * lam
+    assert rel_fro(S, Sref) <= 2e-2
+
+
+def test_precondition_not_spd_is_reported(dev):
+    D = 8
+    state = torch.empty(tda.tda_precondition_state_bytes(D, tda.TDA_F32), dtype=torch.uint8, device=dev)
+    tda.tda_precondition(tda.TDA_PC_RESET, D, tda.TDA_F32, state)
+    phi = torch.ones((2, D), device=dev)
+    tda.tda_precondition(tda.TDA_PC_FIT_ACCUM, D, tda.TDA_F32, state, phi=phi, n=2, ld_phi=D)
+    # make the accumulated matrix indefinite by hand
+    m = state[64:].view(torch.float32).view(D, D)
+    m[3, 3] = -100.0
+    tda.tda_precondition(tda.TDA_PC_FACTOR, D, tda.TDA_F32, state, n_total=2, lambda_abs=1e-3)
+    with pytest.raises(tda.TdaError) as e:
+        tda.tda_precondition_info(D, tda.TDA_F32, state)
+    assert e.value.status == tda.TDA_ERR_NOT_SPD
+    q = torch.ones((1, D), device=dev)
+    qh = torch.zeros((1, D), device=dev)
+    tda.tda_precondition(tda.TDA_PC_APPLY, D, tda.TDA_F32, state, q=q, n_q=1, ld_q=D, qhat=qh, ld_qhat=D)
+    assert torch.isnan(qh).all()
+
+
+# ------------------------------------------------------------------ score and top-k
+@pytest.mark.parametrize("qdt", [tda.TDA_F32, tda.TDA_F64])
+def test_score_and_accumulate(dev, orc, qdt):
+    rng = np.random.default_rng(0)
+    nq, nt, D = 70, 133, 1029
+    Q = rng.standard_normal((nq, D)).astype(np.float32)
+    P = rng.standard_normal((nt, D)).astype(np.float32)
+    Qd = torch.from_numpy(Q).to(dev).to(torch.float64 if qdt == tda.TDA_F64 else torch.float32)
+    S = torch.full((nq, nt), 2.0, device=dev)
+    tda.tda_score(Qd, qdt, nq, D, torch.from_numpy(P).to(dev), nt, D, D, S, nt, beta=1.0)
+    tda.tda_device_status()
+    ref = orc.score(Q, P) + 2.0
+    assert rel_fro(S.cpu().numpy(), ref) <= 1e-5
+
+
+def test_topk_selection_bit_exact_on_gpu_scores(dev, orc):
+    rng = np.random.default_rng(1)
+    nq, nt, k = 9, 5000, 100
+    S = (np.round(rng.standard_normal((nq, nt)) * 64) / 64).astype(np.float32)  # many ties
+    S[0, :] = 0.0
+    S[1, 17] = -0.0
+    Sd = torch.from_numpy(S).to(dev)
+    idx = torch.empty((nq, k), dtype=torch.int32, device=dev)
+    val = torch.empty((nq, k), device=dev)
+    tda.tda_topk(Sd, nq, nt, nt, k, idx, val)
+    tda.tda_device_status()
+    oi, ov = orc.topk(S.astype(np.float64), k)
+    np.testing.assert_array_equal(idx.cpu().numpy(), oi)
+    np.testing.assert_array_equal(val.cpu().numpy(), ov.astype(np.float32))
+
+
+@pytest.mark.parametrize("k", [1, 7, 1024])
+def test_topk_sizes(dev, orc, k):
+    rng = np.random.default_rng(k)
+    nq, nt = 3, 1500
+    S = rng.standard_normal((nq, nt)).astype(np.float32)
+    idx = torch.empty((nq, k), dtype=torch.int32, device=dev)
+    tda.tda_topk(torch.from_numpy(S).to(dev), nq, nt, nt, k, idx, None)
+    oi, _ = orc.topk(S.astype(np.float64), k)
+    np.testing.assert_array_equal(idx.cpu().numpy(), oi)
+
+
+def test_route_auto_and_calibration(dev, orc):
+    ws = torch.empty(tda.TDA_CALIBRATE_WS_BYTES, dtype=torch.uint8, device=dev)
+    rates = tda.tda_route_calibrate(ws, tda.TDA_CALIBRATE_WS_BYTES)
+    assert all(r > 0 for r in rates), rates
+    L = tda.LayerDesc(2048, 2048, 512, 32, 32)
+    chosen, cost = tda.tda_route(L, tda.TDA_OP_PROJECT, 4096, 0, tda.TDA_BF16)
+    assert chosen == tda.TDA_ROUTE_FACTORED and cost[0] < cost[1]
+    tda.tda_route_set_model(0)
+    chosen, cost = tda.tda_route(L, tda.TDA_OP_SIMILARITY_EXACT, 1, 8, tda.TDA_BF16)
+    assert chosen == orc.route_costs(2, 1, 8, 512, 2048, 2048)[0]
