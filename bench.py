@@ -1,0 +1,422 @@
+#!/usr/bin/env python3
+"""Throughput of the attribution hot path on GB300.
+
+Workload: one Llama-style 1B transformer block, bf16 -- linears q/k/v/o
+2048x2048, gate/up 2048->8192, down 8192->2048; T = 512 tokens; 4096 train and
+64 query examples; factors A ~ N(0,1), B ~ N(0,1e-3) with 1% of tokens masked
+in both; seeded Kronecker Rademacher projection k_in = k_out = 32 per linear
+(1024 features per linear, 7168 per example).
+
+One step = one pass of the whole path over the block: route choice per linear
+(host cost model), factored projection of every train and query example
+through all 7 linears, per-linear Fisher fit over the train features, damped
+inverse (lambda = 1e-2 x mean eigenvalue) applied to the queries, the 64 x 4096
+score matrix and the top-100 train indices per query.
+
+value: train examples attributed per second with the factors resident in HBM
+(198 GB, larger than L2, so no flush is needed between steps). e2e: the same
+metric through tda_project_host with the factors in pinned host memory, the
+H2D copies and the D2H read of the top-k inside the timed region.
+
+--impl reference times the fp64 CPU oracle on a bounded sample of the same
+workload on the host cores (the only other place this file runs the oracle).
+"""
+from __future__ import annotations
+
+import argparse
+import json
+import math
+import os
+import statistics
+import subprocess
+import sys
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+LINEARS = [("q", 2048, 2048), ("k", 2048, 2048), ("v", 2048, 2048), ("o", 2048, 2048),
+           ("gate", 2048, 8192), ("up", 2048, 8192), ("down", 8192, 2048)]
+METRIC = "train examples attributed/sec (project+score)"
+
+
+def parse_args():
+    p = argparse.ArgumentParser()
+    p.add_argument("--gpus", type=int, default=1)
+    p.add_argument("--steps", type=int, default=5)
+    p.add_argument("--warmup", type=int, default=3)
+    p.add_argument("--impl", default="ours", choices=["ours", "reference"])
+    p.add_argument("--n-train", type=int, default=4096)
+    p.add_argument("--n-query", type=int, default=64)
+    p.add_argument("--T", type=int, default=512)
+    p.add_argument("--k", type=int, default=32)
+    p.add_argument("--topk", type=int, default=100)
+    p.add_argument("--no-precondition", action="store_true")
+    p.add_argument("--e2e-steps", type=int, default=2)
+    p.add_argument("--no-e2e", action="store_true")
+    p.add_argument("--no-cpu-baseline", action="store_true")
+    p.add_argument("--pool", type=int, default=32, help="pinned host examples per linear for e2e")
+    return p.parse_args()
+
+
+def workload(args):
+    return {
+        "workload": "llama1b_block_bf16",
+        "linears": {n: [di, do] for n, di, do in LINEARS},
+        "T": args.T, "n_train": args.n_train, "n_query": args.n_query,
+        "k_in": args.k, "k_out": args.k, "features_per_example": len(LINEARS) * args.k * args.k,
+        "factors": "A~N(0,1), B~N(0,1e-3), 1% tokens masked (seeded synthetic)",
+        "method": "GradDot" if args.no_precondition else "(F+lambda I)^-1-preconditioned, lambda=1e-2*mean eig",
+        "topk": args.topk, "l2": "inputs larger than L2 (no flush)",
+    }
+
+
+# ---------------------------------------------------------------------------- clocks
+class ClockSampler:
+    FIELDS = ("clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,clocks_event_reasons.hw_slowdown,"
+              "clocks_event_reasons.hw_thermal_slowdown,clocks_event_reasons.sw_thermal_slowdown,"
+              "clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, index):
+        self.index = index
+        self.proc = None
+
+    def start(self):
+        try:
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", "-i", str(self.index), f"--query-gpu={self.FIELDS}", "--format=csv,noheader,nounits",
+                 "-lms", "100"], stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+        except OSError:
+            self.proc = None
+
+    def stop(self):
+        if self.proc is None:
+            return None
+        self.proc.terminate()
+        try:
+            out, _ = self.proc.communicate(timeout=5)
+        except subprocess.TimeoutExpired:
+            self.proc.kill()
+            out, _ = self.proc.communicate()
+        rows = []
+        for line in out.splitlines():
+            parts = [x.strip() for x in line.split(",")]
+            if len(parts) < 8:
+                continue
+            try:
+                rows.append((float(parts[0]), float(parts[1]), parts[4:8]))
+            except ValueError:
+                continue
+        if not rows:
+            return None
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        reasons = sorted({names[i] for _, _, flags in rows for i, f in enumerate(flags) if f.lower() == "active"})
+        return {"sm_mhz": statistics.median(r[0] for r in rows), "sm_max_mhz": max(r[1] for r in rows),
+                "reasons": reasons, "samples": len(rows)}
+
+
+# ---------------------------------------------------------------------------- oracle (CPU)
+def oracle_sample(args, n_s, n_q_s, factors_of):
+    """Time the fp64 oracle on n_s train and n_q_s query examples of the block and
+    extrapolate to the full workload's examples/s. factors_of(role, l, e0, n)
+    returns float64 arrays (A, B) for n examples."""
+    import numpy as np
+
+    import oracle
+
+    oracle.build()
+    threads = os.cpu_count() or 1
+    oracle.set_threads(threads)
+    k, D = args.k, args.k * args.k
+    t_train = t_query = t_fisher = t_factor = 0.0
+    phis, qs = [], []
+    for li, (_, di, do) in enumerate(LINEARS):
+        A, B = factors_of("train", li, 0, n_s)
+        t0 = time.perf_counter()
+        phis.append(oracle.project(A, B, k, k, 0, li).reshape(n_s, D))
+        t_train += time.perf_counter() - t0
+        Aq, Bq = factors_of("query", li, 0, n_q_s)
+        t0 = time.perf_counter()
+        qs.append(oracle.project(Aq, Bq, k, k, 0, li).reshape(n_q_s, D))
+        t_query += time.perf_counter() - t0
+        if not args.no_precondition:
+            t0 = time.perf_counter()
+            F = oracle.fisher(phis[-1])
+            t_fisher += time.perf_counter() - t0
+            t0 = time.perf_counter()
+            qs[-1] = oracle.precondition(F, oracle.damping(F, 0.0, 1e-2), qs[-1])
+            t_factor += time.perf_counter() - t0
+    t0 = time.perf_counter()
+    S = oracle.score(np.concatenate(qs, 1), np.concatenate(phis, 1))
+    oracle.topk(S, min(args.topk, n_s))
+    t_score = time.perf_counter() - t0
+    N, Nq = args.n_train, args.n_query
+    total = (t_train + t_fisher + t_score * Nq / n_q_s) * N / n_s + t_query * Nq / n_q_s + t_factor
+    sample = (f"{n_s} train + {n_q_s} query examples (fp64, {threads} threads) through all 7 linears, Fisher/Cholesky/score on them; "
+              f"per-train-example parts scaled by {N}/{n_s}, query parts by {Nq}/{n_q_s}, factorisation once")
+    return N / total, threads, sample, t_train + t_query + t_fisher + t_factor + t_score
+
+
+def reference_main(args):
+    """--impl reference: the oracle as it stands on the host cores, same config and metric."""
+    import numpy as np
+
+    from paper_2609_38767_gb300 import synth
+
+    rank = int(os.environ.get("RANK", "0"))
+    if rank != 0:
+        return 0
+    sb = math.sqrt(1e-3)
+
+    cache = {}
+
+    def factors_of(role, li, e0, n):
+        # two generated examples per (role, linear), cycled to n: the oracle's work
+        # does not depend on the values, and generation stays out of the timing
+        key = (role, li)
+        if key not in cache:
+            di, do = LINEARS[li][1], LINEARS[li][2]
+            off = synth.QUERY_STREAM_OFFSET if role == "query" else 0
+            ms = 1000 if role == "query" else 0
+            A = synth.factors(synth.SEED_A, li + off, 2, args.T, di, 1.0, 0, 0, "bf16", 0.01, mask_stream=ms)
+            B = synth.factors(synth.SEED_B, li + off, 2, args.T, do, sb, 0, 0, "bf16", 0.01, mask_stream=ms)
+            cache[key] = (synth.to_f64(A, "bf16"), synth.to_f64(B, "bf16"))
+        A, B = cache[key]
+        reps = (n + 1) // 2
+        return np.tile(A, (reps, 1, 1))[:n], np.tile(B, (reps, 1, 1))[:n]
+
+    threads = os.cpu_count() or 1
+    n_s, n_q_s = max(2, threads), 2
+    vals, secs = [], []
+    sample = ""
+    for i in range(args.warmup + args.steps):
+        v, cores, sample, s = oracle_sample(args, n_s, n_q_s, factors_of)
+        if i >= args.warmup:
+            vals.append(v)
+            secs.append(s)
+    value = statistics.median(vals)
+    line = {
+        "impl": "reference", "metric": METRIC, "value": value, "unit": "examples/s", "n_gpus": args.gpus,
+        "steps": args.steps, "warmup": args.warmup, "ms_per_step": 1e3 * args.n_train / value,
+        "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+        "config": workload(args),
+        "cpu_baseline": {"value": value, "unit": "examples/s", "cores": cores, "kind": "oracle", "sample": sample},
+        "e2e": {"value": value, "unit": "examples/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
+    }
+    print(json.dumps(line), flush=True)
+    return 0
+
+
+# ---------------------------------------------------------------------------- GPU arm
+def main():
+    args = parse_args()
+    if args.impl == "reference":
+        return reference_main(args)
+
+    import numpy as np
+    import torch
+
+    import paper_2609_38767_gb300 as tda
+    from paper_2609_38767_gb300 import build as tbuild
+    from paper_2609_38767_gb300 import synth
+
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    torch.cuda.set_device(local)
+    dist = None
+    if world > 1:
+        import torch.distributed as dist
+        dist.init_process_group("nccl", device_id=torch.device("cuda", local))
+    if rank == 0:
+        tbuild.build()
+    if dist:
+        dist.barrier()
+    tda.load()
+    dev = torch.device("cuda", local)
+    stream = torch.cuda.current_stream()
+    T, N, Nq, k = args.T, args.n_train, args.n_query, args.k
+    D = k * k
+    nl = len(LINEARS)
+    DT = D * nl
+    sb = math.sqrt(1e-3)
+
+    # ---- device-resident synthetic factors (untimed)
+    At, Bt, Aq, Bq = [], [], [], []
+    for li, (_, di, do) in enumerate(LINEARS):
+        for store, n, role in ((At, N, 0), (Aq, Nq, 1)):
+            x = torch.empty(n * T * di, dtype=torch.bfloat16, device=dev)
+            synth.fill_device(x, synth.SEED_A, li + (synth.QUERY_STREAM_OFFSET if role else 0), n, T, di, 1.0,
+                              mask_p=0.01, mask_stream=1000 if role else 0)
+            store.append(x)
+        for store, n, role in ((Bt, N, 0), (Bq, Nq, 1)):
+            x = torch.empty(n * T * do, dtype=torch.bfloat16, device=dev)
+            synth.fill_device(x, synth.SEED_B, li + (synth.QUERY_STREAM_OFFSET if role else 0), n, T, do, sb,
+                              mask_p=0.01, mask_stream=1000 if role else 0)
+            store.append(x)
+    Phi = torch.empty((N, DT), dtype=torch.float32, device=dev)
+    Q = torch.empty((Nq, DT), dtype=torch.float32, device=dev)
+    Qh = torch.empty((Nq, DT), dtype=torch.float32, device=dev)
+    S = torch.empty((Nq, N), dtype=torch.float32, device=dev)
+    idx = torch.empty((Nq, args.topk), dtype=torch.int32, device=dev)
+    val = torch.empty((Nq, args.topk), dtype=torch.float32, device=dev)
+    sbytes = tda.tda_precondition_state_bytes(D, tda.TDA_F32)
+    states = [torch.empty(sbytes, dtype=torch.uint8, device=dev) for _ in LINEARS]
+    layers = [tda.LayerDesc(di, do, T, k, k, seed=0, layer=li) for li, (_, di, do) in enumerate(LINEARS)]
+    torch.cuda.synchronize()
+
+    ev = []  # (start, end, algorithmic bytes) per projection launch of the train set
+
+    def attribute(project, record=False):
+        routes = [tda.tda_route(L, tda.TDA_OP_PROJECT, N, 0, tda.TDA_BF16)[0] for L in layers]
+        for li, L in enumerate(layers):
+            if record:
+                e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+                e0.record(stream)
+            project("train", li, L, routes[li])
+            if record:
+                e1.record(stream)
+                ev.append((e0, e1, N * (T * (L.d_in + L.d_out) * 2 + 4 * D)))
+        for li, L in enumerate(layers):
+            project("query", li, L, routes[li])
+        target = Q
+        if not args.no_precondition:
+            for li in range(nl):
+                st = states[li]
+                tda.tda_precondition(tda.TDA_PC_RESET, D, tda.TDA_F32, st)
+                tda.tda_precondition(tda.TDA_PC_FIT_ACCUM, D, tda.TDA_F32, st, phi=Phi[:, li * D:], n=N, ld_phi=DT)
+                tda.tda_precondition(tda.TDA_PC_FACTOR, D, tda.TDA_F32, st, n_total=N, lambda_rel_mean_eig=1e-2)
+                tda.tda_precondition(tda.TDA_PC_APPLY, D, tda.TDA_F32, st, q=Q[:, li * D:], n_q=Nq, ld_q=DT,
+                                     qhat=Qh[:, li * D:], ld_qhat=DT)
+            target = Qh
+        tda.tda_score(target, tda.TDA_F32, Nq, DT, Phi, N, DT, DT, S, N, 0.0)
+        tda.tda_topk(S, Nq, N, N, args.topk, idx, val)
+
+    def project_dev(role, li, L, route):
+        if role == "train":
+            tda.tda_project(L, tda.TDA_BF16, At[li], Bt[li], N, Phi[:, li * D:], DT, route)
+        else:
+            tda.tda_project(L, tda.TDA_BF16, Aq[li], Bq[li], Nq, Q[:, li * D:], DT, route)
+
+    for _ in range(args.warmup):
+        attribute(project_dev)
+    tda.tda_device_status()
+    if dist:
+        dist.barrier()
+    torch.cuda.synchronize()
+    clocks = ClockSampler(local)
+    clocks.start()
+    time.sleep(0.3)
+    launches0 = tda.tda_launch_count()
+    t_start, t_end = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    t_start.record(stream)
+    for _ in range(args.steps):
+        attribute(project_dev, record=True)
+    t_end.record(stream)
+    torch.cuda.synchronize()
+    launches = tda.tda_launch_count() - launches0
+    ck = clocks.stop()
+    tda.tda_device_status()
+    ms = t_start.elapsed_time(t_end) / args.steps
+    if dist:
+        t = torch.tensor([ms], device=dev)
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        ms = float(t.item())
+        dist.barrier()
+    value = world * N / (ms * 1e-3)
+    proj_ms = sum(a.elapsed_time(b) for a, b, _ in ev)
+    proj_bytes = sum(x for _, _, x in ev)
+    peaks = {}
+    try:
+        with open(os.path.join(ROOT, "MEASURED_PEAKS.json")) as f:
+            peaks = json.load(f)
+    except OSError:
+        pass
+    hbm = float(peaks.get("hbm_gbs", 6800.0))
+    achieved = proj_bytes / (proj_ms * 1e-3) / 1e9
+    roofline = {"bound": "hbm", "kernel": "factored projection (train, 7 linears)", "achieved": achieved,
+                "peak": hbm, "unit": "GB/s", "frac": achieved / hbm, "traffic": None,
+                "peak_source": "MEASURED_PEAKS.json hbm_gbs" if peaks else "fallback 6.8 TB/s",
+                "share_of_step": proj_ms / (ms * args.steps)}
+
+    # ---- e2e through tda_project_host with pinned host factors
+    e2e = None
+    if not args.no_e2e:
+        P = min(args.pool, N)
+        pools = []
+        for li, (_, di, do) in enumerate(LINEARS):
+            a = torch.empty(P * T * di, dtype=torch.bfloat16).pin_memory()
+            b = torch.empty(P * T * do, dtype=torch.bfloat16).pin_memory()
+            a.copy_(At[li][: P * T * di])
+            b.copy_(Bt[li][: P * T * do])
+            qa = torch.empty(Nq * T * di, dtype=torch.bfloat16).pin_memory()
+            qb = torch.empty(Nq * T * do, dtype=torch.bfloat16).pin_memory()
+            qa.copy_(Aq[li])
+            qb.copy_(Bq[li])
+            pools.append((a, b, qa, qb))
+        wsb = 2 * P * T * max(di + do for _, di, do in LINEARS) * 2
+        ws = torch.empty(wsb, dtype=torch.uint8, device=dev)
+        idx_h = torch.empty((Nq, args.topk), dtype=torch.int32).pin_memory()
+        val_h = torch.empty((Nq, args.topk), dtype=torch.float32).pin_memory()
+
+        def project_host(role, li, L, route):
+            a, b, qa, qb = pools[li]
+            if role == "train":
+                for e0 in range(0, N, P):
+                    n = min(P, N - e0)
+                    tda.tda_project_host(L, tda.TDA_BF16, a, b, n, Phi[e0:, li * D:], DT, ws, wsb)
+            else:
+                tda.tda_project_host(L, tda.TDA_BF16, qa, qb, Nq, Q[:, li * D:], DT, ws, wsb)
+
+        def e2e_step():
+            attribute(project_host)
+            idx_h.copy_(idx, non_blocking=True)
+            val_h.copy_(val, non_blocking=True)
+            stream.synchronize()
+
+        e2e_step()
+        if dist:
+            dist.barrier()
+        torch.cuda.synchronize()
+        t0 = time.perf_counter()
+        for _ in range(args.e2e_steps):
+            e2e_step()
+        e2e_s = (time.perf_counter() - t0) / args.e2e_steps
+        if dist:
+            t = torch.tensor([e2e_s], device=dev)
+            dist.all_reduce(t, op=dist.ReduceOp.MAX)
+            e2e_s = float(t.item())
+        h2d = N * T * sum(di + do for _, di, do in LINEARS) * 2 + Nq * T * sum(di + do for _, di, do in LINEARS) * 2
+        e2e = {"value": world * N / e2e_s, "unit": "examples/s", "h2d_bytes_per_step": h2d,
+               "d2h_bytes_per_step": Nq * args.topk * 8, "ms_per_step": e2e_s * 1e3,
+               "host_pool_examples": P}
+
+    cpu = None
+    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+        def factors_of(role, li, e0, n):
+            src_a, src_b = (At, Bt) if role == "train" else (Aq, Bq)
+            di, do = LINEARS[li][1], LINEARS[li][2]
+            a = src_a[li][e0 * T * di:(e0 + n) * T * di].float().cpu().numpy().astype(np.float64)
+            b = src_b[li][e0 * T * do:(e0 + n) * T * do].float().cpu().numpy().astype(np.float64)
+            return a.reshape(n, T, di), b.reshape(n, T, do)
+
+        threads = os.cpu_count() or 1
+        v, cores, sample, _ = oracle_sample(args, max(2, threads), 2, factors_of)
+        cpu = {"value": v, "unit": "examples/s", "cores": cores, "kind": "oracle", "sample": sample}
+
+    if rank == 0:
+        line = {
+            "metric": METRIC, "value": value, "unit": "examples/s", "n_gpus": world, "steps": args.steps,
+            "warmup": args.warmup, "ms_per_step": ms, "higher_is_better": True, "scaling": "weak",
+            "vs_baseline": None, "dtype": "bf16", "data": "synthetic", "config": workload(args),
+            "roofline": roofline, "cpu_baseline": cpu, "e2e": e2e, "gpu_launches": launches,
+            "clocks": ck,
+        }
+        print(json.dumps(line), flush=True)
+    if dist:
+        dist.destroy_process_group()
+    return 0
+
+
+if __name__ == "__main__":
+    sys.exit(main())

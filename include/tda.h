@@ -131,6 +131,23 @@ tda_status tda_project(const tda_layer_desc* L, tda_dtype dtype, const void* A, 
                        void* ws, size_t ws_bytes, void* stream);
 
 /* ---------------------------------------------------------------------------
+ * tda_project_host -- tda_project (route FACTORED) for factors held in HOST
+ * memory. A_h[N][T][d_in] and B_h[N][T][d_out] are copied chunk by chunk into
+ * two halves of the device scratch `ws` on a copy stream owned by the library
+ * and projected on `stream` as they land (App. A.2: factors are projected as
+ * they arrive and never buffered whole). Page-locked host memory
+ * (cudaHostAlloc / cudaHostRegister) lets copies overlap compute; pageable
+ * memory works but serialises. The host buffers must stay unchanged until
+ * `stream` has completed. ws: >= tda_project_host_ws_min() bytes (one example
+ * per half), 256-byte aligned; larger ws means larger chunks. Calls on one
+ * device serialise their enqueueing on a library mutex.
+ * ------------------------------------------------------------------------- */
+size_t tda_project_host_ws_min(const tda_layer_desc* L, tda_dtype dtype);
+tda_status tda_project_host(const tda_layer_desc* L, tda_dtype dtype, const void* A_h, const void* B_h,
+                            int64_t N, float* phi, int64_t ld_phi, void* ws, size_t ws_bytes,
+                            void* stream);
+
+/* ---------------------------------------------------------------------------
  * tda_similarity_exact -- unprojected gradient inner products
  *   S[q][i] = beta*S[q][i] + <DW_q, DW_i>_F
  * for n_q query and n_t train examples of one layer (Eq. 4's left side).
@@ -243,6 +260,10 @@ const char* tda_last_error(void);
 
 /* ABI version: major*10000 + minor*100 + patch. */
 int32_t tda_version(void);
+
+/* Number of kernel launches this library has issued in this process (all
+ * devices, all threads). Host only; for counting launches in a timed region. */
+uint64_t tda_launch_count(void);
 
 #ifdef __cplusplus
 }

@@ -15,9 +15,10 @@ import threading
 
 __all__ = [
     "LayerDesc", "TdaError", "load", "tda_proj_entries", "tda_workspace_size", "tda_project",
+    "tda_project_host_ws_min", "tda_project_host",
     "tda_similarity_exact", "tda_precondition_state_bytes", "tda_precondition",
     "tda_precondition_info", "tda_score", "tda_topk", "tda_route", "tda_route_calibrate",
-    "tda_route_set_model", "tda_device_status", "tda_last_error", "tda_version",
+    "tda_route_set_model", "tda_device_status", "tda_last_error", "tda_version", "tda_launch_count",
 ]
 
 _HERE = os.path.dirname(os.path.abspath(__file__))
@@ -74,6 +75,8 @@ def load() -> ctypes.CDLL:
             "tda_proj_entries": (I32, [U64, U32, I32, I32, I64, I32, P, P]),
             "tda_workspace_size": (I32, [I32, LP, I32, I64, I64, I32, ctypes.POINTER(SZ)]),
             "tda_project": (I32, [LP, I32, P, P, I64, P, I64, I32, P, SZ, P]),
+            "tda_project_host_ws_min": (SZ, [LP, I32]),
+            "tda_project_host": (I32, [LP, I32, P, P, I64, P, I64, P, SZ, P]),
             "tda_similarity_exact": (I32, [LP, I32, P, P, I64, P, P, I64, P, I64, F, I32, P, SZ, P]),
             "tda_precondition_state_bytes": (SZ, [I64, I32]),
             "tda_precondition": (I32, [I32, I64, I32, P, P, I64, I64, I64, D, D, P, I64, I64, P, I64, P]),
@@ -86,6 +89,7 @@ def load() -> ctypes.CDLL:
             "tda_device_status": (I32, [P]),
             "tda_last_error": (ctypes.c_char_p, []),
             "tda_version": (I32, []),
+            "tda_launch_count": (U64, []),
         }
         for name, (res, args) in sig.items():
             fn = getattr(lib, name)
@@ -126,6 +130,10 @@ def tda_version() -> int:
     return int(load().tda_version())
 
 
+def tda_launch_count() -> int:
+    return int(load().tda_launch_count())
+
+
 def tda_proj_entries(seed, layer, side, kind, rows, cols, out, stream=None):
     _check(load().tda_proj_entries(seed, layer, side, kind, rows, cols, _ptr(out), _stream(stream)))
 
@@ -139,6 +147,15 @@ def tda_workspace_size(op, L, dtype, n1, n2, route=TDA_ROUTE_AUTO) -> int:
 def tda_project(L, dtype, A, B, N, phi, ld_phi, route=TDA_ROUTE_AUTO, ws=None, ws_bytes=0, stream=None):
     _check(load().tda_project(ctypes.byref(L), dtype, _ptr(A), _ptr(B), N, _ptr(phi), ld_phi, route,
                               _ptr(ws), ws_bytes, _stream(stream)))
+
+
+def tda_project_host_ws_min(L, dtype) -> int:
+    return int(load().tda_project_host_ws_min(ctypes.byref(L), dtype))
+
+
+def tda_project_host(L, dtype, A_h, B_h, N, phi, ld_phi, ws, ws_bytes, stream=None):
+    _check(load().tda_project_host(ctypes.byref(L), dtype, _ptr(A_h), _ptr(B_h), N, _ptr(phi), ld_phi,
+                                   _ptr(ws), ws_bytes, _stream(stream)))
 
 
 def tda_similarity_exact(L, dtype, Aq, Bq, n_q, At, Bt, n_t, S, ld_S, beta=0.0, route=TDA_ROUTE_AUTO,

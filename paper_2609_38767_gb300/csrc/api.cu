@@ -5,6 +5,7 @@
 #include <string.h>
 
 #include <cmath>
+#include <atomic>
 #include <mutex>
 
 #include "tda_internal.cuh"
@@ -25,6 +26,9 @@ tda_status cuda_check(cudaError_t e, const char* what) {
     if (e == cudaSuccess) return TDA_OK;
     return fail(TDA_ERR_CUDA, "%s: %s (%s)", what, cudaGetErrorName(e), cudaGetErrorString(e));
 }
+
+static std::atomic<uint64_t> g_launches{0};
+void note_launches(uint64_t n) { g_launches.fetch_add(n, std::memory_order_relaxed); }
 
 // The device error word: bounded waits that expire OR bits into it.
 __device__ unsigned int g_error_word;
@@ -168,6 +172,8 @@ extern "C" {
 const char* tda_last_error(void) { return g_msg; }
 
 int32_t tda_version(void) { return 100; }
+
+uint64_t tda_launch_count(void) { return g_launches.load(std::memory_order_relaxed); }
 
 tda_status tda_proj_entries(uint64_t seed, uint32_t layer, int32_t side, int32_t kind, int64_t rows,
                             int32_t cols, int8_t* out, void* stream) {

@@ -289,14 +289,17 @@ pc_apply_kernel(int64_t D, const void* state, const float* __restrict__ q, int64
 template <typename TS>
 cudaError_t factor_impl(int64_t D, void* state, int64_t n_total, double la, double lr,
                         cudaStream_t s) {
+    note_launches(2);
     pc_prepare_kernel<TS><<<1, 256, 0, s>>>(D, state, n_total, la, lr);
     int64_t blocks = (D * D + 255) / 256;
     if (blocks > 152 * 32) blocks = 152 * 32;
     pc_scale_kernel<TS><<<(unsigned)blocks, 256, 0, s>>>(D, state);
     for (int64_t k0 = 0; k0 < D; k0 += kNB) {
+        note_launches(1);
         pc_chol_diag_kernel<TS><<<1, 256, 0, s>>>(D, state, k0);
         const int64_t rest = D - k0 - kNB;
         if (rest > 0) {
+            note_launches(2);
             pc_chol_panel_kernel<TS><<<(unsigned)((rest + 127) / 128), 128, 0, s>>>(D, state, k0);
             const unsigned t = (unsigned)((rest + kFT - 1) / kFT);
             pc_chol_update_kernel<TS><<<dim3(t, t), 256, 0, s>>>(D, state, k0);
@@ -311,6 +314,7 @@ cudaError_t launch_pc_fit(int64_t D, tda_dtype sdt, void* state, const float* ph
                           int64_t ld, cudaStream_t s) {
     if (n == 0) return cudaSuccess;
     const unsigned t = (unsigned)((D + kFT - 1) / kFT);
+    note_launches(1);
     if (sdt == TDA_F64)
         pc_fit_kernel<double><<<dim3(t, t), 256, 0, s>>>(D, state, phi, n, ld);
     else
@@ -331,6 +335,7 @@ cudaError_t launch_pc_apply(int64_t D, tda_dtype sdt, const void* state, const f
     const size_t el = sdt == TDA_F64 ? sizeof(double) : sizeof(float);
     const size_t smem = (size_t)D * el;
     cudaError_t e;
+    note_launches(1);
     if (sdt == TDA_F64) {
         e = cudaFuncSetAttribute(pc_apply_kernel<double>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                  (int)smem);

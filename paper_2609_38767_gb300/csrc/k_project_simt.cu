@@ -138,6 +138,7 @@ cudaError_t launch_proj_entries(uint64_t key, int kind, int64_t rows, int32_t co
     if (total == 0) return cudaSuccess;
     int64_t blocks = (total + 255) / 256;
     if (blocks > 152 * 64) blocks = 152 * 64;
+    note_launches(1);
     proj_entries_kernel<<<(unsigned)blocks, 256, 0, s>>>(key, kind, rows, cols, out);
     return cudaGetLastError();
 }
@@ -155,6 +156,7 @@ cudaError_t launch_project_simt(const tda_layer_desc& L, tda_dtype dt, const voi
     dim3 grid((unsigned)N, (unsigned)((L.k_out + kTile - 1) / kTile),
               (unsigned)((L.k_in + kTile - 1) / kTile));
     const float scale = projection_scale(L);
+    note_launches(1);
     if (dt == TDA_BF16)
         project_simt_kernel<__nv_bfloat16><<<grid, kThreads, 0, s>>>(
             (const __nv_bfloat16*)A, (const __nv_bfloat16*)B, L.T, L.d_in, L.d_out, L.k_in,

@@ -219,6 +219,7 @@ template <typename T>
 void launch_materialize(const void* A, const void* B, int64_t e0, int64_t nb,
                         const tda_layer_desc& L, float* G, cudaStream_t s) {
     dim3 grid((unsigned)((L.d_in + kT - 1) / kT), (unsigned)((L.d_out + kT - 1) / kT), (unsigned)nb);
+    note_launches(1);
     materialize_kernel<T><<<grid, kTh, 0, s>>>((const T*)A, (const T*)B, e0, L.T, L.d_in, L.d_out, G);
 }
 
@@ -249,6 +250,7 @@ cudaError_t launch_project_materialized(const tda_layer_desc& L, tda_dtype dt, c
         else
             launch_materialize<float>(A, B, e0, cnt, L, G, s);
         dim3 g2((unsigned)((L.k_in + kT - 1) / kT), (unsigned)((L.d_out + kT - 1) / kT), (unsigned)cnt);
+        note_launches(2);
         sign_right_kernel<<<g2, kTh, 0, s>>>(G, L.d_out, L.d_in, L.k_in, key_in, L.kind, X);
         dim3 g3((unsigned)((L.k_in + kT - 1) / kT), (unsigned)((L.k_out + kT - 1) / kT), (unsigned)cnt);
         sign_left_kernel<<<g3, kTh, 0, s>>>(X, L.d_out, L.k_in, L.k_out, key_out, L.kind, scale, e0,
@@ -298,6 +300,7 @@ cudaError_t launch_similarity_gram(const tda_layer_desc& L, tda_dtype dt, const 
                                    cudaStream_t s) {
     if (n_q == 0 || n_t == 0) return cudaSuccess;
     dim3 grid((unsigned)n_t, (unsigned)n_q);
+    note_launches(1);
     if (dt == TDA_BF16)
         gram_kernel<__nv_bfloat16><<<grid, kTh, 0, s>>>(
             (const __nv_bfloat16*)Aq, (const __nv_bfloat16*)Bq, (const __nv_bfloat16*)At,

@@ -175,6 +175,7 @@ cudaError_t launch_score(const void* Qhat, tda_dtype qdt, int64_t n_q, int64_t l
                          int64_t ld_S, float beta, cudaStream_t s) {
     if (n_q == 0 || n_t == 0) return cudaSuccess;
     dim3 grid((unsigned)((n_t + kST - 1) / kST), (unsigned)((n_q + kST - 1) / kST));
+    note_launches(1);
     if (qdt == TDA_F64)
         score_kernel<double, double><<<grid, kSThreads, 0, s>>>(
             (const double*)Qhat, n_q, ld_q, Phi, n_t, ld_phi, D, S, ld_S, beta);
@@ -187,6 +188,7 @@ cudaError_t launch_score(const void* Qhat, tda_dtype qdt, int64_t n_q, int64_t l
 cudaError_t launch_topk(const float* S, int64_t n_q, int64_t n_t, int64_t ld_S, int32_t k,
                         int32_t* idx, float* val, cudaStream_t s) {
     if (n_q == 0) return cudaSuccess;
+    note_launches(1);
     topk_kernel<<<(unsigned)n_q, kTopThreads, 0, s>>>(S, n_t, ld_S, k, idx, val);
     return cudaGetLastError();
 }

@@ -1,0 +1,98 @@
+// stream_host.cu -- tda_project_host: the factored projection of factors that
+// live in host memory. App. A.2 applies the projection as the factors arrive,
+// so raw factors are never buffered whole; here they stream through two
+// device staging halves of the caller's scratch: the copy of chunk c+1 (on a
+// library-owned copy stream) overlaps the projection of chunk c (on the
+// caller's stream).
+#include <mutex>
+
+#include "tda_internal.cuh"
+
+namespace tda {
+namespace {
+
+struct HostPipe {
+    bool ready = false;
+    cudaStream_t copy = nullptr;
+    cudaEvent_t copied[2] = {nullptr, nullptr};
+    cudaEvent_t done[2] = {nullptr, nullptr};
+    std::mutex mu;
+};
+
+HostPipe g_pipes[64];
+
+cudaError_t pipe_for_device(HostPipe** out) {
+    int dev = 0;
+    cudaError_t e = cudaGetDevice(&dev);
+    if (e != cudaSuccess) return e;
+    if (dev < 0 || dev >= 64) return cudaErrorInvalidDevice;
+    HostPipe& p = g_pipes[dev];
+    *out = &p;
+    if (p.ready) return cudaSuccess;
+    if ((e = cudaStreamCreateWithFlags(&p.copy, cudaStreamNonBlocking)) != cudaSuccess) return e;
+    for (int b = 0; b < 2; ++b) {
+        if ((e = cudaEventCreateWithFlags(&p.copied[b], cudaEventDisableTiming)) != cudaSuccess) return e;
+        if ((e = cudaEventCreateWithFlags(&p.done[b], cudaEventDisableTiming)) != cudaSuccess) return e;
+    }
+    p.ready = true;
+    return cudaSuccess;
+}
+
+}  // namespace
+}  // namespace tda
+
+using namespace tda;
+
+extern "C" size_t tda_project_host_ws_min(const tda_layer_desc* L, tda_dtype dtype) {
+    if (!L || L->T < 0 || L->d_in < 1 || L->d_out < 1) return 0;
+    const size_t el = dtype == TDA_F32 ? 4 : 2;
+    const size_t per = (size_t)L->T * (size_t)(L->d_in + L->d_out) * el;
+    return 2 * (((per + 255) / 256) * 256);
+}
+
+extern "C" tda_status tda_project_host(const tda_layer_desc* L, tda_dtype dtype, const void* A_h,
+                                       const void* B_h, int64_t N, float* phi, int64_t ld_phi,
+                                       void* ws, size_t ws_bytes, void* stream) {
+    if (!L) return fail(TDA_ERR_INVALID_ARG, "layer descriptor is NULL");
+    if (dtype != TDA_F32 && dtype != TDA_BF16) return fail(TDA_ERR_INVALID_ARG, "dtype must be F32 or BF16");
+    if (N < 0) return fail(TDA_ERR_INVALID_ARG, "negative N");
+    if (N > 0 && L->T > 0 && (!A_h || !B_h)) return fail(TDA_ERR_INVALID_ARG, "NULL host factor pointer");
+    const size_t need = tda_project_host_ws_min(L, dtype);
+    if (need == 0) return fail(TDA_ERR_INVALID_ARG, "bad layer sizes");
+    if (!ws || ws_bytes < need)
+        return fail(TDA_ERR_WORKSPACE, "tda_project_host needs >= %zu bytes of ws, got %zu", need, ws_bytes);
+    if ((uintptr_t)ws & 255) return fail(TDA_ERR_INVALID_ARG, "ws must be 256-byte aligned");
+    if (N == 0 || L->T == 0)
+        return tda_project(L, dtype, ws, ws, N, phi, ld_phi, TDA_ROUTE_FACTORED, nullptr, 0, stream);
+
+    HostPipe* p = nullptr;
+    tda_status st = cuda_check(pipe_for_device(&p), "copy pipeline setup");
+    if (st) return st;
+    std::lock_guard<std::mutex> lock(p->mu);
+    const size_t el = dtype == TDA_F32 ? 4 : 2;
+    const size_t a_ex = (size_t)L->T * L->d_in * el, b_ex = (size_t)L->T * L->d_out * el;
+    const size_t half = (ws_bytes / 2) & ~(size_t)255;
+    int64_t chunk = (int64_t)(half / (a_ex + b_ex));
+    if (chunk > N) chunk = N;
+    cudaStream_t s = (cudaStream_t)stream;
+    for (int64_t c0 = 0, c = 0; c0 < N; c0 += chunk, ++c) {
+        const int b = (int)(c & 1);
+        const int64_t cnt = (N - c0) < chunk ? (N - c0) : chunk;
+        char* dA = (char*)ws + (size_t)b * half;
+        char* dB = dA + (size_t)chunk * a_ex;
+        if ((st = cuda_check(cudaStreamWaitEvent(p->copy, p->done[b], 0), "wait buffer"))) return st;
+        if ((st = cuda_check(cudaMemcpyAsync(dA, (const char*)A_h + (size_t)c0 * a_ex, (size_t)cnt * a_ex,
+                                             cudaMemcpyHostToDevice, p->copy), "copy A")))
+            return st;
+        if ((st = cuda_check(cudaMemcpyAsync(dB, (const char*)B_h + (size_t)c0 * b_ex, (size_t)cnt * b_ex,
+                                             cudaMemcpyHostToDevice, p->copy), "copy B")))
+            return st;
+        if ((st = cuda_check(cudaEventRecord(p->copied[b], p->copy), "record copy"))) return st;
+        if ((st = cuda_check(cudaStreamWaitEvent(s, p->copied[b], 0), "wait copy"))) return st;
+        if ((st = tda_project(L, dtype, dA, dB, cnt, phi + c0 * ld_phi, ld_phi, TDA_ROUTE_FACTORED, nullptr, 0,
+                              stream)))
+            return st;
+        if ((st = cuda_check(cudaEventRecord(p->done[b], s), "record done"))) return st;
+    }
+    return TDA_OK;
+}

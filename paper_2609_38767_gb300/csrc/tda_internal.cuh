@@ -44,6 +44,9 @@ enum : unsigned int {
     kErrBadLaunch = 2u,  // a kernel found its launch geometry inconsistent
 };
 
+// Host-side count of kernels this library has launched (tda_launch_count).
+void note_launches(uint64_t n);
+
 // Device address of the library's error word on the current device.
 unsigned int* device_error_word();
 

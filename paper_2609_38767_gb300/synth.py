@@ -63,16 +63,21 @@ def word(key: np.uint64, n: np.ndarray) -> np.ndarray:
         return mix64(np.uint64(key) + GAMMA * (np.asarray(n, dtype=np.uint64) + np.uint64(1)))
 
 
+_PAIR = np.uint64(0x0000FFFF0000FFFF)
+_LO32 = np.uint64(0xFFFFFFFF)
+
+
 def normal(key: np.uint64, i: np.ndarray) -> np.ndarray:
     i = np.asarray(i, dtype=np.uint64)
-    s = np.zeros(i.shape, dtype=np.int64)
+    s = np.zeros(i.shape, dtype=np.uint64)
     with np.errstate(over="ignore"):
         base = i * np.uint64(3)
         for j in range(3):
             w = word(key, base + np.uint64(j))
-            for q in range(4):
-                s += ((w >> np.uint64(16 * q)) & np.uint64(0xFFFF)).astype(np.int64)
-    return (s + 6 - 393216).astype(np.float32) / np.float32(65536.0)
+            # sum of the four 16-bit fields: pairwise in two 32-bit lanes, then the lanes
+            p = (w & _PAIR) + ((w >> np.uint64(16)) & _PAIR)
+            s += (p & _LO32) + (p >> np.uint64(32))
+    return (s.astype(np.int64) + (6 - 393216)).astype(np.float32) / np.float32(65536.0)
 
 
 def student_t4(key: np.uint64, i: np.ndarray) -> np.ndarray:
@@ -116,10 +121,16 @@ def factors(seed: int, stream: int, n: int, T: int, d: int, sigma: float = 1.0,
     e = np.arange(e0, e0 + n, dtype=np.uint64)[:, None, None]
     t = np.arange(T, dtype=np.uint64)[None, :, None]
     c = np.arange(d, dtype=np.uint64)[None, None, :]
-    with np.errstate(over="ignore"):
-        idx = (e * np.uint64(T) + t) * np.uint64(d) + c
-    v = normal(key, idx) if dist == DIST_NORMAL else student_t4(key, idx)
-    v = (v * np.float32(sigma)).astype(np.float32)
+    gen = normal if dist == DIST_NORMAL else student_t4
+    v = np.empty((n, T, d), dtype=np.float32)
+    flat = v.reshape(-1)
+    chunk = max(1, (1 << 16) // max(d, 1))  # token rows per chunk, cache-sized
+    rows = (e * np.uint64(T) + t).reshape(-1)  # global token index of each (example, token) row
+    for r0 in range(0, rows.size, chunk):
+        r = rows[r0:r0 + chunk, None]
+        with np.errstate(over="ignore"):
+            idx = r * np.uint64(d) + c.reshape(1, -1)
+        flat[r0 * d:(r0 + r.shape[0]) * d] = (gen(key, idx) * np.float32(sigma)).astype(np.float32).reshape(-1)
     thr = mask_threshold(mask_p)
     if thr > 0:
         mkey = stream_key(mask_seed, mask_stream)
