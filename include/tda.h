@@ -148,6 +148,32 @@ tda_status tda_project_host(const tda_layer_desc* L, tda_dtype dtype, const void
                             void* stream);
 
 /* ---------------------------------------------------------------------------
+ * tda_project_materialized_noalloc -- tda_project with route MATERIALIZE for
+ * callers that cannot allocate device memory: the library keeps its own
+ * scratch in a fixed device array of tda_noalloc_scratch_bytes() bytes
+ * (64 MiB), held on every GPU that loads libtda.so until the process exits.
+ * (The paper has no counterpart; this is a deployment convenience.)
+ * Intended for code that cannot call cudaMalloc or supply a workspace where it
+ * projects, e.g. a plugin inside a host program that owns all device memory,
+ * or a loop that must not pay cudaMalloc's implicit device synchronisation.
+ *   Arguments as tda_project; A, B, phi are still the caller's buffers.
+ *   Rejects (TDA_ERR_WORKSPACE) a layer whose per-example scratch,
+ *   4*(d_out*d_in + d_out*k_in) bytes, exceeds the array.
+ *   The first call on a device, with that device current, resolves the
+ *   array's device address (cudaGetSymbolAddress); make that first call
+ *   before any stream capture.
+ *   Every call shares the one array and leaves its contents behind; the
+ *   kernels overwrite what they read, so nothing needs clearing. Calls whose
+ *   work overlaps on the GPU (different streams, or host threads without
+ *   ordering) race on the array: serialise them on one stream.
+ *   No cudaMalloc, cudaFree or allocating library routine is called.
+ * ------------------------------------------------------------------------- */
+size_t tda_noalloc_scratch_bytes(void);
+tda_status tda_project_materialized_noalloc(const tda_layer_desc* L, tda_dtype dtype, const void* A,
+                                            const void* B, int64_t N, float* phi, int64_t ld_phi,
+                                            void* stream);
+
+/* ---------------------------------------------------------------------------
  * tda_similarity_exact -- unprojected gradient inner products
  *   S[q][i] = beta*S[q][i] + <DW_q, DW_i>_F
  * for n_q query and n_t train examples of one layer (Eq. 4's left side).
