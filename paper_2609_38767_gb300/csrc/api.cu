@@ -47,8 +47,6 @@ unsigned int* device_error_word() {
     return cache[dev];
 }
 
-float projection_scale(const tda_layer_desc& L);
-
 // ---------------------------------------------------------------------------
 // Route cost model (Sec. 3.2, App. A.4, Table 2): flop counts at 2 flops per
 // multiply-add, or, after calibration, estimated seconds.

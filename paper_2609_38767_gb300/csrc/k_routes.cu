@@ -225,8 +225,6 @@ void launch_materialize(const void* A, const void* B, int64_t e0, int64_t nb,
 
 }  // namespace
 
-float projection_scale(const tda_layer_desc& L);
-
 size_t materialize_ws_bytes_per_example(const tda_layer_desc& L) {
     return sizeof(float) * (size_t)(L.d_out * L.d_in + L.d_out * (int64_t)L.k_in);
 }

@@ -44,6 +44,9 @@ enum : unsigned int {
     kErrBadLaunch = 2u,  // a kernel found its launch geometry inconsistent
 };
 
+// 1/sqrt(k_in k_out) for Rademacher maps, 1 for the identity map (App. A.2).
+float projection_scale(const tda_layer_desc& L);
+
 // Host-side count of kernels this library has launched (tda_launch_count).
 void note_launches(uint64_t n);
 

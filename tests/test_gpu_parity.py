@@ -265,3 +265,47 @@ def test_route_auto_and_calibration(dev, orc):
     tda.tda_route_set_model(0)
     chosen, cost = tda.tda_route(L, tda.TDA_OP_SIMILARITY_EXACT, 1, 8, tda.TDA_BF16)
     assert chosen == orc.route_costs(2, 1, 8, 512, 2048, 2048)[0]
+
+
+# ------------------------------------------------------------------ tensor-core projection specifics
+def test_tc_projection_signs_bit_exact(dev, orc):
+    # One-hot factors: A_n = I (T = d_in tokens), B_n = e_r at token t only, so
+    # Phi_n / scale = outer(S_out[r, :], S_in[t, :]) exactly -- the signs the
+    # tensor-core kernel generated on chip, compared bit for bit with the oracle's.
+    d, k, N = 128, 32, 4
+    picks = [(0, 5), (77, 127), (127, 64), (31, 0)]  # (t, r) per example
+    A = np.zeros((N, d, d), dtype=np.float32)
+    B = np.zeros((N, d, d), dtype=np.float32)
+    for n, (t, r) in enumerate(picks):
+        A[n] = np.eye(d, dtype=np.float32)
+        B[n, t, r] = 1.0
+    Ab = torch.from_numpy(A).to(dev).to(torch.bfloat16)
+    Bb = torch.from_numpy(B).to(dev).to(torch.bfloat16)
+    L = tda.LayerDesc(d, d, d, k, k, seed=2024, layer=9)
+    got, _ = gpu_project(L, "bf16", Ab, Bb, N, tda.TDA_ROUTE_FACTORED, dev)
+    S_in = orc.proj_entries(2024, 9, 0, d, k).astype(np.float32)
+    S_out = orc.proj_entries(2024, 9, 1, d, k).astype(np.float32)
+    for n, (t, r) in enumerate(picks):
+        np.testing.assert_array_equal(got[n] * k, np.outer(S_out[r], S_in[t]))
+
+
+TC_CASES = [
+    # (N, T, d_in, d_out, k, dtype): persistent loop, ragged K chunks, T = 1, T over tiles
+    (400, 200, 64, 72, 16, "bf16"),
+    (7, 1, 136, 200, 32, "bf16"),
+    (5, 129, 136, 64, 64, "bf16"),
+    (3, 384, 1024, 256, 32, "bf16"),
+    (160, 16, 2048, 2048, 32, "bf16"),
+]
+
+
+@pytest.mark.parametrize("case", TC_CASES)
+def test_tc_projection_matches_oracle(dev, orc, case):
+    N, T, di, do, k, dtype = case
+    A, B = make_factors(N, T, di, do, dtype, stream=11, sigma_b=0.03, mask_p=0.01)
+    L = tda.LayerDesc(di, do, T, k, k, seed=5, layer=3)
+    got, _ = gpu_project(L, dtype, to_dev(A, dtype, dev), to_dev(B, dtype, dev), N, tda.TDA_ROUTE_FACTORED, dev)
+    ref = orc.project(synth.to_f64(A, dtype), synth.to_f64(B, dtype), k, k, 5, 3)
+    assert rel_fro(got, ref) <= TOL[dtype]
+    worst = max(rel_fro(got[n], ref[n]) for n in range(N))
+    assert worst <= TOL[dtype], worst
