@@ -334,7 +334,9 @@ def main():
         pass
     hbm = float(peaks.get("hbm_gbs", 6800.0))
     achieved = proj_bytes / (proj_ms * 1e-3) / 1e9
-    roofline = {"bound": "hbm", "kernel": "factored projection (train, 7 linears)", "achieved": achieved,
+    engines = sorted({tda.tda_project_engine(L, tda.TDA_BF16, At[li], Bt[li]) for li, L in enumerate(layers)})
+    roofline = {"bound": "hbm", "kernel": "factored projection (train, 7 linears)",
+                "engine": "tcgen05" if engines == [1] else ("cuda-core" if engines == [0] else "mixed"), "achieved": achieved,
                 "peak": hbm, "unit": "GB/s", "frac": achieved / hbm, "traffic": None,
                 "peak_source": "MEASURED_PEAKS.json hbm_gbs" if peaks else "fallback 6.8 TB/s",
                 "share_of_step": proj_ms / (ms * args.steps)}

@@ -130,6 +130,12 @@ tda_status tda_project(const tda_layer_desc* L, tda_dtype dtype, const void* A, 
                        int64_t N, float* phi, int64_t ld_phi, tda_route_id route,
                        void* ws, size_t ws_bytes, void* stream);
 
+/* Which kernel tda_project (route FACTORED) would run for these arguments on
+ * the current device: 1 = the tcgen05/TMA tensor-core kernel (bf16, k_in ==
+ * k_out in {16, 32, 64}, sm_103), 0 = the CUDA-core kernel, negative = the
+ * arguments are invalid. Host only; for tests and benchmark reports. */
+int32_t tda_project_engine(const tda_layer_desc* L, tda_dtype dtype, const void* A, const void* B);
+
 /* ---------------------------------------------------------------------------
  * tda_project_host -- tda_project (route FACTORED) for factors held in HOST
  * memory. A_h[N][T][d_in] and B_h[N][T][d_out] are copied chunk by chunk into

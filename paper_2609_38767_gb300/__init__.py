@@ -15,7 +15,7 @@ import threading
 
 __all__ = [
     "LayerDesc", "TdaError", "load", "tda_proj_entries", "tda_workspace_size", "tda_project",
-    "tda_project_host_ws_min", "tda_project_host", "tda_noalloc_scratch_bytes",
+    "tda_project_engine", "tda_project_host_ws_min", "tda_project_host", "tda_noalloc_scratch_bytes",
     "tda_project_materialized_noalloc",
     "tda_similarity_exact", "tda_precondition_state_bytes", "tda_precondition",
     "tda_precondition_info", "tda_score", "tda_topk", "tda_route", "tda_route_calibrate",
@@ -76,6 +76,7 @@ def load() -> ctypes.CDLL:
             "tda_proj_entries": (I32, [U64, U32, I32, I32, I64, I32, P, P]),
             "tda_workspace_size": (I32, [I32, LP, I32, I64, I64, I32, ctypes.POINTER(SZ)]),
             "tda_project": (I32, [LP, I32, P, P, I64, P, I64, I32, P, SZ, P]),
+            "tda_project_engine": (I32, [LP, I32, P, P]),
             "tda_project_host_ws_min": (SZ, [LP, I32]),
             "tda_project_host": (I32, [LP, I32, P, P, I64, P, I64, P, SZ, P]),
             "tda_noalloc_scratch_bytes": (SZ, []),
@@ -150,6 +151,10 @@ def tda_workspace_size(op, L, dtype, n1, n2, route=TDA_ROUTE_AUTO) -> int:
 def tda_project(L, dtype, A, B, N, phi, ld_phi, route=TDA_ROUTE_AUTO, ws=None, ws_bytes=0, stream=None):
     _check(load().tda_project(ctypes.byref(L), dtype, _ptr(A), _ptr(B), N, _ptr(phi), ld_phi, route,
                               _ptr(ws), ws_bytes, _stream(stream)))
+
+
+def tda_project_engine(L, dtype, A, B) -> int:
+    return int(load().tda_project_engine(ctypes.byref(L), dtype, _ptr(A), _ptr(B)))
 
 
 def tda_project_host_ws_min(L, dtype) -> int:

@@ -270,6 +270,12 @@ tda_status tda_project(const tda_layer_desc* L, tda_dtype dtype, const void* A, 
     return fail(TDA_ERR_UNSUPPORTED, "route %d cannot produce projected features", (int)route);
 }
 
+int32_t tda_project_engine(const tda_layer_desc* L, tda_dtype dtype, const void* A, const void* B) {
+    g_msg[0] = 0;
+    if (validate_layer(L, true) || validate_factors(L, dtype, A, B, 1, "tda_project_engine")) return -1;
+    return (dtype == TDA_BF16 && project_tc_supported(*L, A, B)) ? 1 : 0;
+}
+
 tda_status tda_similarity_exact(const tda_layer_desc* L, tda_dtype dtype, const void* Aq,
                                 const void* Bq, int64_t n_q, const void* At, const void* Bt,
                                 int64_t n_t, float* S, int64_t ld_S, float beta, tda_route_id route,

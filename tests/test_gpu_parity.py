@@ -282,6 +282,7 @@ def test_tc_projection_signs_bit_exact(dev, orc):
     Ab = torch.from_numpy(A).to(dev).to(torch.bfloat16)
     Bb = torch.from_numpy(B).to(dev).to(torch.bfloat16)
     L = tda.LayerDesc(d, d, d, k, k, seed=2024, layer=9)
+    assert tda.tda_project_engine(L, tda.TDA_BF16, Ab, Bb) == 1
     got, _ = gpu_project(L, "bf16", Ab, Bb, N, tda.TDA_ROUTE_FACTORED, dev)
     S_in = orc.proj_entries(2024, 9, 0, d, k).astype(np.float32)
     S_out = orc.proj_entries(2024, 9, 1, d, k).astype(np.float32)
@@ -304,7 +305,9 @@ def test_tc_projection_matches_oracle(dev, orc, case):
     N, T, di, do, k, dtype = case
     A, B = make_factors(N, T, di, do, dtype, stream=11, sigma_b=0.03, mask_p=0.01)
     L = tda.LayerDesc(di, do, T, k, k, seed=5, layer=3)
-    got, _ = gpu_project(L, dtype, to_dev(A, dtype, dev), to_dev(B, dtype, dev), N, tda.TDA_ROUTE_FACTORED, dev)
+    Ad, Bd = to_dev(A, dtype, dev), to_dev(B, dtype, dev)
+    assert tda.tda_project_engine(L, TD[dtype], Ad, Bd) == 1  # the tensor-core kernel runs
+    got, _ = gpu_project(L, dtype, Ad, Bd, N, tda.TDA_ROUTE_FACTORED, dev)
     ref = orc.project(synth.to_f64(A, dtype), synth.to_f64(B, dtype), k, k, 5, 3)
     assert rel_fro(got, ref) <= TOL[dtype]
     worst = max(rel_fro(got[n], ref[n]) for n in range(N))
