@@ -261,7 +261,7 @@ def main():
     idx = torch.empty((Nq, args.topk), dtype=torch.int32, device=dev)
     val = torch.empty((Nq, args.topk), dtype=torch.float32, device=dev)
     sbytes = tda.tda_precondition_state_bytes(D, tda.TDA_F32)
-    states = [torch.empty(sbytes, dtype=torch.uint8, device=dev) for _ in LINEARS]
+    state = torch.empty(nl * sbytes, dtype=torch.uint8, device=dev)  # all 7 layers, back to back
     layers = [tda.LayerDesc(di, do, T, k, k, seed=0, layer=li) for li, (_, di, do) in enumerate(LINEARS)]
     torch.cuda.synchronize()
 
@@ -281,13 +281,12 @@ def main():
             project("query", li, L, routes[li])
         target = Q
         if not args.no_precondition:
-            for li in range(nl):
-                st = states[li]
-                tda.tda_precondition(tda.TDA_PC_RESET, D, tda.TDA_F32, st)
-                tda.tda_precondition(tda.TDA_PC_FIT_ACCUM, D, tda.TDA_F32, st, phi=Phi[:, li * D:], n=N, ld_phi=DT)
-                tda.tda_precondition(tda.TDA_PC_FACTOR, D, tda.TDA_F32, st, n_total=N, lambda_rel_mean_eig=1e-2)
-                tda.tda_precondition(tda.TDA_PC_APPLY, D, tda.TDA_F32, st, q=Q[:, li * D:], n_q=Nq, ld_q=DT,
-                                     qhat=Qh[:, li * D:], ld_qhat=DT)
+            # one batched call per op for the 7 layers (layer l's features at column l*D)
+            tda.tda_precondition(tda.TDA_PC_RESET, nl, D, tda.TDA_F32, state)
+            tda.tda_precondition(tda.TDA_PC_FIT_ACCUM, nl, D, tda.TDA_F32, state, phi=Phi, n=N, ld_phi=DT)
+            tda.tda_precondition(tda.TDA_PC_FACTOR, nl, D, tda.TDA_F32, state, n_total=N, lambda_rel_mean_eig=1e-2)
+            tda.tda_precondition(tda.TDA_PC_APPLY, nl, D, tda.TDA_F32, state, q=Q, n_q=Nq, ld_q=DT, qhat=Qh,
+                                 ld_qhat=DT)
             target = Qh
         tda.tda_score(target, tda.TDA_F32, Nq, DT, Phi, N, DT, DT, S, N, 0.0)
         tda.tda_topk(S, Nq, N, N, args.topk, idx, val)

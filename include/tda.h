@@ -198,23 +198,29 @@ tda_status tda_similarity_exact(const tda_layer_desc* L, tda_dtype dtype,
 /* ---------------------------------------------------------------------------
  * tda_precondition -- damped Fisher inverse on the query side (App. B.3: a
  * curvature fit over the training gradients, then per-layer preconditioning
- * of the queries; App. B.2: damping in units of the mean eigenvalue).
+ * of the queries; App. B.2: damping in units of the mean eigenvalue), for
+ * n_layers independent layers of D features each in one call.
  *
- * `state` is a device buffer of tda_precondition_state_bytes(D, state_dtype)
- * bytes: an 8-double header followed by a D x D matrix of state_dtype
- * (TDA_F32 or TDA_F64). The ops, in order of use:
+ * Feature layout: layer l's D features of example (or query) row r are at
+ * phi[r*ld_phi + l*D + f], q[r*ld_q + l*D + f], qhat[r*ld_qhat + l*D + f]:
+ * the layers' features side by side in each row (n_layers = 1: one layer).
+ *
+ * `state` is a device buffer of n_layers * tda_precondition_state_bytes(D,
+ * state_dtype) bytes, 16-byte aligned: per layer a 64-byte header, the D x D
+ * matrix M and the inverses of M's 32 x 32 diagonal blocks, all in
+ * state_dtype (TDA_F32 or TDA_F64). The ops, in order of use:
  *   TDA_PC_RESET      zero the state.
- *   TDA_PC_FIT_ACCUM  M += Phi^T Phi over n feature rows (phi, ld_phi).
- *                     Called once per streamed chunk of training features.
- *   TDA_PC_FACTOR     F = M / n_total; lambda = lambda_abs +
- *                     lambda_rel_mean_eig * tr(F)/D; M <- L with
- *                     L L^T = F + lambda I (lower Cholesky, in place).
- *                     A non-positive pivot is recorded in the header;
- *                     tda_precondition_info() reports it (TDA_ERR_NOT_SPD).
- *   TDA_PC_APPLY      qhat = (F + lambda I)^{-1} q for n_q rows of q (fp32,
- *                     ld_q); qhat has state_dtype (fp64 rows for an F64
- *                     state), row stride ld_qhat. After a failed FACTOR the
- *                     rows are NaN.
+ *   TDA_PC_FIT_ACCUM  M_l += Phi_l^T Phi_l over n feature rows. Call once per
+ *                     streamed chunk of training features.
+ *   TDA_PC_FACTOR     F_l = M_l / n_total; lambda_l = lambda_abs +
+ *                     lambda_rel_mean_eig * tr(F_l)/D; factor F_l + lambda_l I
+ *                     = L L^T (Cholesky) into the state. A non-positive pivot
+ *                     is recorded in the layer's header; tda_precondition_info
+ *                     reports it (TDA_ERR_NOT_SPD).
+ *   TDA_PC_APPLY      qhat_l = (F_l + lambda_l I)^{-1} q_l for n_q query rows
+ *                     (q fp32; qhat in state_dtype, i.e. fp64 rows for an F64
+ *                     state). Layers whose FACTOR failed get NaN rows.
+ *                     Needs D <= 40960 (F32) or 20480 (F64).
  * Arguments not used by an op are ignored (may be 0/NULL).
  * ------------------------------------------------------------------------- */
 #define TDA_PC_RESET 0
@@ -222,18 +228,20 @@ tda_status tda_similarity_exact(const tda_layer_desc* L, tda_dtype dtype,
 #define TDA_PC_FACTOR 2
 #define TDA_PC_APPLY 3
 
+/* Bytes of ONE layer's state (a multiple of 256). */
 size_t tda_precondition_state_bytes(int64_t D, tda_dtype state_dtype);
 
-tda_status tda_precondition(int32_t op, int64_t D, tda_dtype state_dtype, void* state,
+tda_status tda_precondition(int32_t op, int32_t n_layers, int64_t D, tda_dtype state_dtype, void* state,
                             const float* phi, int64_t n, int64_t ld_phi,
                             int64_t n_total, double lambda_abs, double lambda_rel_mean_eig,
                             const float* q, int64_t n_q, int64_t ld_q,
                             void* qhat, int64_t ld_qhat, void* stream);
 
-/* Synchronises `stream` and copies the state header to host `info[4]`:
- * {lambda used, tr(F)/D, failed pivot (0 = SPD), n_total}. Returns
- * TDA_ERR_NOT_SPD if the last FACTOR failed. */
-tda_status tda_precondition_info(int64_t D, tda_dtype state_dtype, const void* state,
+/* Synchronises `stream` and copies each layer's header to host
+ * info[4*l .. 4*l+3] = {lambda used, tr(F)/D, failed pivot (0 = SPD), n_total}
+ * (info holds 4*n_layers doubles). Returns TDA_ERR_NOT_SPD if the last FACTOR
+ * failed for any layer. */
+tda_status tda_precondition_info(int32_t n_layers, int64_t D, tda_dtype state_dtype, const void* state,
                                  double* info, void* stream);
 
 /* ---------------------------------------------------------------------------

@@ -83,8 +83,8 @@ def load() -> ctypes.CDLL:
             "tda_project_materialized_noalloc": (I32, [LP, I32, P, P, I64, P, I64, P]),
             "tda_similarity_exact": (I32, [LP, I32, P, P, I64, P, P, I64, P, I64, F, I32, P, SZ, P]),
             "tda_precondition_state_bytes": (SZ, [I64, I32]),
-            "tda_precondition": (I32, [I32, I64, I32, P, P, I64, I64, I64, D, D, P, I64, I64, P, I64, P]),
-            "tda_precondition_info": (I32, [I64, I32, P, ctypes.POINTER(D), P]),
+            "tda_precondition": (I32, [I32, I32, I64, I32, P, P, I64, I64, I64, D, D, P, I64, I64, P, I64, P]),
+            "tda_precondition_info": (I32, [I32, I64, I32, P, ctypes.POINTER(D), P]),
             "tda_score": (I32, [P, I32, I64, I64, P, I64, I64, I64, P, I64, F, P]),
             "tda_topk": (I32, [P, I64, I64, I64, I32, P, P, P]),
             "tda_route": (I32, [LP, I32, I64, I64, I32, ctypes.POINTER(I32), ctypes.POINTER(D)]),
@@ -185,16 +185,16 @@ def tda_precondition_state_bytes(D, state_dtype) -> int:
     return int(load().tda_precondition_state_bytes(D, state_dtype))
 
 
-def tda_precondition(op, D, state_dtype, state, phi=None, n=0, ld_phi=0, n_total=0, lambda_abs=0.0,
+def tda_precondition(op, n_layers, D, state_dtype, state, phi=None, n=0, ld_phi=0, n_total=0, lambda_abs=0.0,
                      lambda_rel_mean_eig=0.0, q=None, n_q=0, ld_q=0, qhat=None, ld_qhat=0, stream=None):
-    _check(load().tda_precondition(op, D, state_dtype, _ptr(state), _ptr(phi), n, ld_phi, n_total,
+    _check(load().tda_precondition(op, n_layers, D, state_dtype, _ptr(state), _ptr(phi), n, ld_phi, n_total,
                                    lambda_abs, lambda_rel_mean_eig, _ptr(q), n_q, ld_q, _ptr(qhat),
                                    ld_qhat, _stream(stream)))
 
 
-def tda_precondition_info(D, state_dtype, state, stream=None) -> list[float]:
-    info = (ctypes.c_double * 4)()
-    _check(load().tda_precondition_info(D, state_dtype, _ptr(state), info, _stream(stream)))
+def tda_precondition_info(n_layers, D, state_dtype, state, stream=None) -> list[float]:
+    info = (ctypes.c_double * (4 * n_layers))()
+    _check(load().tda_precondition_info(n_layers, D, state_dtype, _ptr(state), info, _stream(stream)))
     return list(info)
 
 

@@ -317,46 +317,49 @@ tda_status tda_similarity_exact(const tda_layer_desc* L, tda_dtype dtype, const 
 size_t tda_precondition_state_bytes(int64_t D, tda_dtype state_dtype) {
     if (D < 1 || (state_dtype != TDA_F32 && state_dtype != TDA_F64)) return 0;
     const size_t el = state_dtype == TDA_F64 ? 8 : 4;
-    return kPcHeaderDoubles * sizeof(double) + (size_t)D * (size_t)D * el;
+    const size_t nblk = (size_t)((D + 31) / 32);
+    const size_t raw = kPcHeaderDoubles * sizeof(double) + ((size_t)D * (size_t)D + nblk * 1024) * el;
+    return (raw + 255) & ~(size_t)255;
 }
 
-tda_status tda_precondition(int32_t op, int64_t D, tda_dtype state_dtype, void* state,
+tda_status tda_precondition(int32_t op, int32_t n_layers, int64_t D, tda_dtype state_dtype, void* state,
                             const float* phi, int64_t n, int64_t ld_phi, int64_t n_total,
                             double lambda_abs, double lambda_rel_mean_eig, const float* q,
                             int64_t n_q, int64_t ld_q, void* qhat, int64_t ld_qhat, void* stream) {
     g_msg[0] = 0;
-    if (D < 1) return fail(TDA_ERR_INVALID_ARG, "D must be >= 1");
+    if (n_layers < 1 || n_layers > 65535) return fail(TDA_ERR_INVALID_ARG, "n_layers must be in [1, 65535]");
+    if (D < 1 || D > (1LL << 20)) return fail(TDA_ERR_INVALID_ARG, "D must be in [1, 2^20]");
     if (state_dtype != TDA_F32 && state_dtype != TDA_F64)
         return fail(TDA_ERR_INVALID_ARG, "state dtype must be TDA_F32 or TDA_F64");
     if (!state) return fail(TDA_ERR_INVALID_ARG, "state is NULL");
     if ((uintptr_t)state & 15) return fail(TDA_ERR_INVALID_ARG, "state must be 16-byte aligned");
+    const int64_t width = (int64_t)n_layers * D;  // features per row across the layers
     cudaStream_t s = (cudaStream_t)stream;
     switch (op) {
         case TDA_PC_RESET:
-            return cuda_check(cudaMemsetAsync(state, 0, tda_precondition_state_bytes(D, state_dtype), s),
+            return cuda_check(cudaMemsetAsync(state, 0, (size_t)n_layers * tda_precondition_state_bytes(D, state_dtype), s),
                               "reset state");
         case TDA_PC_FIT_ACCUM:
             if (n < 0) return fail(TDA_ERR_INVALID_ARG, "negative n");
             if (n > 0 && !phi) return fail(TDA_ERR_INVALID_ARG, "phi is NULL");
-            if (ld_phi < D) return fail(TDA_ERR_INVALID_ARG, "ld_phi < D");
-            if (D > 65535 * 64LL) return fail(TDA_ERR_INVALID_ARG, "D too large");
-            return cuda_check(launch_pc_fit(D, state_dtype, state, phi, n, ld_phi, s), "fit");
+            if (ld_phi < width) return fail(TDA_ERR_INVALID_ARG, "ld_phi < n_layers*D");
+            return cuda_check(launch_pc_fit(n_layers, D, state_dtype, state, phi, n, ld_phi, s), "fit");
         case TDA_PC_FACTOR:
             if (n_total < 1) return fail(TDA_ERR_INVALID_ARG, "n_total must be >= 1");
             if (!(lambda_abs >= 0) || !(lambda_rel_mean_eig >= 0) ||
                 !(lambda_abs > 0 || lambda_rel_mean_eig > 0))
                 return fail(TDA_ERR_INVALID_ARG, "damping must be >= 0 and not both zero");
-            return cuda_check(launch_pc_factor(D, state_dtype, state, n_total, lambda_abs,
+            return cuda_check(launch_pc_factor(n_layers, D, state_dtype, state, n_total, lambda_abs,
                                                lambda_rel_mean_eig, s),
                               "factor");
         case TDA_PC_APPLY: {
             if (n_q < 0) return fail(TDA_ERR_INVALID_ARG, "negative n_q");
             if (n_q > 0 && (!q || !qhat)) return fail(TDA_ERR_INVALID_ARG, "q/qhat is NULL");
-            if (ld_q < D || ld_qhat < D) return fail(TDA_ERR_INVALID_ARG, "ld_q/ld_qhat < D");
-            const size_t el = state_dtype == TDA_F64 ? 8 : 4;
-            if ((size_t)D * el > 200 * 1024)
-                return fail(TDA_ERR_UNSUPPORTED, "APPLY keeps one row in shared memory: D*%zu > 200 KiB", el);
-            return cuda_check(launch_pc_apply(D, state_dtype, state, q, n_q, ld_q, qhat, ld_qhat, s),
+            if (ld_q < width || ld_qhat < width) return fail(TDA_ERR_INVALID_ARG, "ld_q/ld_qhat < n_layers*D");
+            if (D > precondition_apply_max_d(state_dtype))
+                return fail(TDA_ERR_UNSUPPORTED, "APPLY keeps a query row in shared memory: D > %lld",
+                            (long long)precondition_apply_max_d(state_dtype));
+            return cuda_check(launch_pc_apply(n_layers, D, state_dtype, state, q, n_q, ld_q, qhat, ld_qhat, s),
                               "apply");
         }
         default:
@@ -364,23 +367,35 @@ tda_status tda_precondition(int32_t op, int64_t D, tda_dtype state_dtype, void* 
     }
 }
 
-tda_status tda_precondition_info(int64_t D, tda_dtype state_dtype, const void* state, double* info,
-                                 void* stream) {
+tda_status tda_precondition_info(int32_t n_layers, int64_t D, tda_dtype state_dtype, const void* state,
+                                 double* info, void* stream) {
     g_msg[0] = 0;
     if (!state || !info) return fail(TDA_ERR_INVALID_ARG, "NULL argument");
-    (void)D;
-    (void)state_dtype;
+    if (n_layers < 1) return fail(TDA_ERR_INVALID_ARG, "n_layers must be >= 1");
+    const size_t per = tda_precondition_state_bytes(D, state_dtype);
+    if (!per) return fail(TDA_ERR_INVALID_ARG, "bad D or state dtype");
     cudaStream_t s = (cudaStream_t)stream;
-    double h[kPcHeaderDoubles];
-    tda_status st = cuda_check(cudaMemcpyAsync(h, state, sizeof(h), cudaMemcpyDeviceToHost, s), "read header");
-    if (st) return st;
-    if ((st = cuda_check(cudaStreamSynchronize(s), "sync"))) return st;
-    info[0] = h[kPcLambda];
-    info[1] = h[kPcMeanEig];
-    info[2] = h[kPcFailedPivot];
-    info[3] = h[kPcNTotal];
-    if (h[kPcFailedPivot] != 0.0)
-        return fail(TDA_ERR_NOT_SPD, "F + lambda I not positive definite at pivot %.0f", h[kPcFailedPivot]);
+    double fail_at = 0;
+    int fail_layer = -1;
+    for (int32_t l = 0; l < n_layers; ++l) {
+        double h[kPcHeaderDoubles];
+        tda_status st = cuda_check(
+            cudaMemcpyAsync(h, (const char*)state + (size_t)l * per, sizeof(h), cudaMemcpyDeviceToHost, s),
+            "read header");
+        if (st) return st;
+        if ((st = cuda_check(cudaStreamSynchronize(s), "sync"))) return st;
+        info[4 * l + 0] = h[kPcLambda];
+        info[4 * l + 1] = h[kPcMeanEig];
+        info[4 * l + 2] = h[kPcFailedPivot];
+        info[4 * l + 3] = h[kPcNTotal];
+        if (h[kPcFailedPivot] != 0.0 && fail_layer < 0) {
+            fail_layer = l;
+            fail_at = h[kPcFailedPivot];
+        }
+    }
+    if (fail_layer >= 0)
+        return fail(TDA_ERR_NOT_SPD, "layer %d: F + lambda I not positive definite at pivot %.0f", fail_layer,
+                    fail_at);
     return TDA_OK;
 }
 
@@ -391,7 +406,7 @@ tda_status tda_score(const void* Qhat, tda_dtype q_dtype, int64_t n_q, int64_t l
     if (q_dtype != TDA_F32 && q_dtype != TDA_F64)
         return fail(TDA_ERR_INVALID_ARG, "Qhat dtype must be TDA_F32 or TDA_F64");
     if (n_q < 0 || n_t < 0 || D < 0) return fail(TDA_ERR_INVALID_ARG, "negative size");
-    if (n_q > 65535LL * 64) return fail(TDA_ERR_INVALID_ARG, "n_q too large");
+    if (n_q > 65535LL * 32) return fail(TDA_ERR_INVALID_ARG, "n_q too large");
     if (n_q > 0 && n_t > 0) {
         if (!S) return fail(TDA_ERR_INVALID_ARG, "S is NULL");
         if (D > 0 && (!Qhat || !Phi)) return fail(TDA_ERR_INVALID_ARG, "Qhat/Phi is NULL");

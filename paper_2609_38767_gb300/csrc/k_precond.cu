@@ -1,16 +1,26 @@
-// k_precond.cu -- damped Fisher preconditioner of the queries.
+// k_precond.cu -- damped Fisher preconditioner of the queries, for a batch of
+// layers with the same feature count D.
 //
 // App. B.3: curvature-based methods fit a curvature matrix over the training
 // gradients and precondition the queries layer by layer; App. B.2: damping is
 // a multiple of the layer's mean eigenvalue. On projected features phi (D per
-// example) the fit is the empirical Fisher F = (1/N) sum_i phi_i phi_i^T, and a
-// query q becomes qhat = (F + lambda I)^{-1} q.
+// example and layer) the fit is the empirical Fisher F = (1/N) sum_i phi_i
+// phi_i^T, and a query q becomes qhat = (F + lambda I)^{-1} q.
 //
-// State (caller-owned): kPcHeaderDoubles doubles of header, then M (D x D,
-// float or double). FIT accumulates M += Phi^T Phi; FACTOR turns M into the
-// lower Cholesky factor L of M/n_total + lambda I (blocked right-looking:
-// diagonal block, panel triangular solve, trailing update); APPLY solves
-// L L^T x = q by blocked forward and backward substitution.
+// Per-layer state (caller-owned, tda_precondition_state_bytes each, layers
+// back to back): 64-byte header | M (D x D) | Dinv (ceil(D/32) blocks of
+// 32 x 32), elements float or double. After FACTOR, M holds L strictly below
+// its 32 x 32 diagonal blocks; each diagonal block of L is held as its inverse
+// in Dinv.
+//   FIT     M += Phi^T Phi (lower 128x128 tiles; register-blocked SYRK)
+//   FACTOR  M <- L, L L^T = M/n_total + lambda I: right-looking Cholesky in
+//           32-column steps; each step factors the diagonal block inside every
+//           panel CTA (so it needs no launch of its own), solves the panel, then
+//           updates the trailing lower triangle. The inverse of every diagonal
+//           block is kept in Dinv.
+//   APPLY   forward and backward block substitution; with Dinv each 32-row
+//           block step is a small matrix product instead of a serial chain.
+// Every launch covers all layers of the call (grid z or y = layer).
 #include <math.h>
 
 #include "tda_internal.cuh"
@@ -18,70 +28,150 @@
 namespace tda {
 namespace {
 
-constexpr int kFT = 64;  // fit tile edge
-constexpr int kFK = 32;  // rows per fit chunk
 constexpr int kNB = 32;  // Cholesky / substitution block
 
 template <typename TS>
-__device__ __forceinline__ TS* mat_of(void* state) {
-    return (TS*)((char*)state + kPcHeaderDoubles * sizeof(double));
-}
+struct St {
+    char* base;
+    int64_t D;
+    size_t bytes;
+    __device__ __forceinline__ double* header(int l) const { return (double*)(base + (size_t)l * bytes); }
+    __device__ __forceinline__ TS* M(int l) const { return (TS*)(base + (size_t)l * bytes + 64); }
+    __device__ __forceinline__ TS* Dinv(int l) const { return M(l) + D * D; }
+};
+
 template <typename TS>
-__device__ __forceinline__ const TS* mat_of(const void* state) {
-    return (const TS*)((const char*)state + kPcHeaderDoubles * sizeof(double));
+St<TS> state_of(void* state, int64_t D) {
+    St<TS> s;
+    s.base = (char*)state;
+    s.D = D;
+    s.bytes = tda_precondition_state_bytes(D, sizeof(TS) == 8 ? TDA_F64 : TDA_F32);
+    return s;
 }
 
-// M[a][b] += sum_n phi[n][a] phi[n][b], 64 x 64 tiles, 256 threads x 4x4.
-template <typename TS>
+// ---------------------------------------------------------------- FIT (fp32)
+// Tile 128 x 128 of M for rows a0.., cols b0.. (b-tile <= a-tile), K = rows of
+// Phi in chunks of 16. Thread (ty, tx) of 16 x 16 owns rows {ty*4+u, 64+ty*4+u}
+// and columns {tx*4+v, 64+tx*4+v}: 8 x 8 accumulators, float4 shared reads.
+constexpr int kFT = 128, kFK = 16;
+
 __global__ void __launch_bounds__(256)
-pc_fit_kernel(int64_t D, void* state, const float* __restrict__ phi, int64_t n, int64_t ld) {
-    __shared__ TS Xa[kFK][kFT + 1];
-    __shared__ TS Xb[kFK][kFT + 1];
-    TS* M = mat_of<TS>(state);
-    const int tid = threadIdx.x, ty = tid / 16, tx = tid % 16;
+fit_f32_kernel(St<float> st, const float* __restrict__ phi, int64_t n, int64_t ld) {
+    if (blockIdx.x > blockIdx.y) return;  // upper tile: M is used through its lower triangle
+    __shared__ __align__(16) float Xa[kFK][kFT];
+    __shared__ __align__(16) float Xb[kFK][kFT];
+    const int l = blockIdx.z;
+    const int64_t D = st.D;
+    const float* ph = phi + (int64_t)l * D;
     const int64_t a0 = (int64_t)blockIdx.y * kFT, b0 = (int64_t)blockIdx.x * kFT;
-    TS acc[4][4];
+    const int tid = threadIdx.x, ty = tid >> 4, tx = tid & 15;
+    float acc[8][8];
 #pragma unroll
-    for (int u = 0; u < 4; ++u)
+    for (int u = 0; u < 8; ++u)
 #pragma unroll
-        for (int v = 0; v < 4; ++v) acc[u][v] = (TS)0;
+        for (int v = 0; v < 8; ++v) acc[u][v] = 0.f;
+    const bool vec = ((ld & 3) == 0) && ((D & 3) == 0) && (((uintptr_t)ph & 15) == 0);
     for (int64_t r0 = 0; r0 < n; r0 += kFK) {
-        for (int e = tid; e < kFK * kFT; e += 256) {
-            const int rr = e / kFT, cc = e % kFT;
+        // 16 rows x 128 columns per operand: 512 float4 each, 2 per thread
+#pragma unroll
+        for (int h = 0; h < 2; ++h) {
+            const int e = tid + h * 256;
+            const int rr = e >> 5, c4 = (e & 31) * 4;
             const int64_t r = r0 + rr;
-            Xa[rr][cc] = (r < n && a0 + cc < D) ? (TS)phi[r * ld + a0 + cc] : (TS)0;
-            Xb[rr][cc] = (r < n && b0 + cc < D) ? (TS)phi[r * ld + b0 + cc] : (TS)0;
+            float4 va = make_float4(0.f, 0.f, 0.f, 0.f), vb = va;
+            if (r < n) {
+                const float* row = ph + r * ld;
+                if (vec && a0 + c4 + 3 < D) {
+                    va = *reinterpret_cast<const float4*>(row + a0 + c4);
+                } else {
+                    float t[4];
+                    for (int i = 0; i < 4; ++i) t[i] = (a0 + c4 + i < D) ? row[a0 + c4 + i] : 0.f;
+                    va = make_float4(t[0], t[1], t[2], t[3]);
+                }
+                if (vec && b0 + c4 + 3 < D) {
+                    vb = *reinterpret_cast<const float4*>(row + b0 + c4);
+                } else {
+                    float t[4];
+                    for (int i = 0; i < 4; ++i) t[i] = (b0 + c4 + i < D) ? row[b0 + c4 + i] : 0.f;
+                    vb = make_float4(t[0], t[1], t[2], t[3]);
+                }
+            }
+            *reinterpret_cast<float4*>(&Xa[rr][c4]) = va;
+            *reinterpret_cast<float4*>(&Xb[rr][c4]) = vb;
         }
         __syncthreads();
-#pragma unroll 8
-        for (int rr = 0; rr < kFK; ++rr) {
-            TS x[4], y[4];
 #pragma unroll
-            for (int u = 0; u < 4; ++u) x[u] = Xa[rr][ty * 4 + u];
+        for (int k = 0; k < kFK; ++k) {
+            const float4 x0 = *reinterpret_cast<const float4*>(&Xa[k][ty * 4]);
+            const float4 x1 = *reinterpret_cast<const float4*>(&Xa[k][64 + ty * 4]);
+            const float4 y0 = *reinterpret_cast<const float4*>(&Xb[k][tx * 4]);
+            const float4 y1 = *reinterpret_cast<const float4*>(&Xb[k][64 + tx * 4]);
+            const float x[8] = {x0.x, x0.y, x0.z, x0.w, x1.x, x1.y, x1.z, x1.w};
+            const float y[8] = {y0.x, y0.y, y0.z, y0.w, y1.x, y1.y, y1.z, y1.w};
 #pragma unroll
-            for (int v = 0; v < 4; ++v) y[v] = Xb[rr][tx * 4 + v];
+            for (int u = 0; u < 8; ++u)
 #pragma unroll
-            for (int u = 0; u < 4; ++u)
-#pragma unroll
-                for (int v = 0; v < 4; ++v) acc[u][v] += x[u] * y[v];
+                for (int v = 0; v < 8; ++v) acc[u][v] = fmaf(x[u], y[v], acc[u][v]);
         }
         __syncthreads();
     }
+    float* M = st.M(l);
 #pragma unroll
+    for (int u = 0; u < 8; ++u) {
+        const int64_t a = a0 + (u < 4 ? ty * 4 + u : 64 + ty * 4 + (u - 4));
+        if (a >= D) continue;
+#pragma unroll
+        for (int v = 0; v < 8; ++v) {
+            const int64_t b = b0 + (v < 4 ? tx * 4 + v : 64 + tx * 4 + (v - 4));
+            if (b < D) M[a * D + b] += acc[u][v];
+        }
+    }
+}
+
+// ---------------------------------------------------------------- FIT (fp64)
+__global__ void __launch_bounds__(256)
+fit_f64_kernel(St<double> st, const float* __restrict__ phi, int64_t n, int64_t ld) {
+    if (blockIdx.x > blockIdx.y) return;
+    constexpr int T = 64, K = 32;
+    __shared__ double Xa[K][T + 1];
+    __shared__ double Xb[K][T + 1];
+    const int l = blockIdx.z;
+    const int64_t D = st.D;
+    const float* ph = phi + (int64_t)l * D;
+    const int tid = threadIdx.x, ty = tid / 16, tx = tid % 16;
+    const int64_t a0 = (int64_t)blockIdx.y * T, b0 = (int64_t)blockIdx.x * T;
+    double acc[4][4] = {};
+    for (int64_t r0 = 0; r0 < n; r0 += K) {
+        for (int e = tid; e < K * T; e += 256) {
+            const int rr = e / T, cc = e % T;
+            const int64_t r = r0 + rr;
+            Xa[rr][cc] = (r < n && a0 + cc < D) ? (double)ph[r * ld + a0 + cc] : 0.0;
+            Xb[rr][cc] = (r < n && b0 + cc < D) ? (double)ph[r * ld + b0 + cc] : 0.0;
+        }
+        __syncthreads();
+        for (int rr = 0; rr < K; ++rr)
+#pragma unroll
+            for (int u = 0; u < 4; ++u)
+#pragma unroll
+                for (int v = 0; v < 4; ++v) acc[u][v] += Xa[rr][ty * 4 + u] * Xb[rr][tx * 4 + v];
+        __syncthreads();
+    }
+    double* M = st.M(l);
     for (int u = 0; u < 4; ++u)
-#pragma unroll
         for (int v = 0; v < 4; ++v) {
             const int64_t a = a0 + ty * 4 + u, b = b0 + tx * 4 + v;
             if (a < D && b < D) M[a * D + b] += acc[u][v];
         }
 }
 
-// Header: trace -> mean eigenvalue of F = M/n_total, and lambda.
+// ---------------------------------------------------------------- FACTOR
+// Header: mean eigenvalue of F = M/n_total is tr(M)/(n_total D); lambda.
 template <typename TS>
-__global__ void pc_prepare_kernel(int64_t D, void* state, int64_t n_total, double lambda_abs,
-                                  double lambda_rel) {
+__global__ void prepare_kernel(St<TS> st, int64_t n_total, double lambda_abs, double lambda_rel) {
     __shared__ double part[256];
-    const TS* M = mat_of<TS>((const void*)state);
+    const int l = blockIdx.x;
+    const int64_t D = st.D;
+    const TS* M = st.M(l);
     double s = 0.0;
     for (int64_t a = threadIdx.x; a < D; a += blockDim.x) s += (double)M[a * D + a];
     part[threadIdx.x] = s;
@@ -91,7 +181,7 @@ __global__ void pc_prepare_kernel(int64_t D, void* state, int64_t n_total, doubl
         __syncthreads();
     }
     if (threadIdx.x == 0) {
-        double* h = (double*)state;
+        double* h = st.header(l);
         const double mean_eig = part[0] / (double)n_total / (double)D;
         h[kPcLambda] = lambda_abs + lambda_rel * mean_eig;
         h[kPcMeanEig] = mean_eig;
@@ -100,97 +190,117 @@ __global__ void pc_prepare_kernel(int64_t D, void* state, int64_t n_total, doubl
     }
 }
 
-// M <- M / n_total + lambda I
+// Lower triangle of M <- M / n_total + lambda I.
 template <typename TS>
-__global__ void pc_scale_kernel(int64_t D, void* state) {
-    const double* h = (const double*)state;
-    TS* M = mat_of<TS>(state);
-    const TS inv = (TS)(1.0 / h[kPcNTotal]);
-    const TS lam = (TS)h[kPcLambda];
-    const int64_t total = D * D;
-    for (int64_t e = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; e < total;
+__global__ void scale_kernel(St<TS> st, int n_layers) {
+    const int64_t D = st.D, per = D * D;
+    for (int64_t e = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; e < per * n_layers;
          e += (int64_t)gridDim.x * blockDim.x) {
-        const int64_t a = e / D, b = e - a * D;
-        TS v = M[e] * inv;
-        if (a == b) v += lam;
-        M[e] = v;
+        const int l = (int)(e / per);
+        const int64_t r = e - (int64_t)l * per, a = r / D, b = r - a * D;
+        if (b > a) continue;
+        const double* h = st.header(l);
+        TS* M = st.M(l);
+        TS v = M[r] * (TS)(1.0 / h[kPcNTotal]);
+        if (a == b) v += (TS)h[kPcLambda];
+        M[r] = v;
     }
 }
 
-// Factor the nb x nb diagonal block at k0 in shared memory (unblocked,
-// right-looking). A non-positive pivot records its 1-based global index.
+// One 32-column step at k0, grid (layer, row chunk): every CTA factors the
+// diagonal block in shared memory (one warp), then solves x L_kk^T = a for 256
+// panel rows. Row chunk 0 also writes L_kk and its inverse (into Dinv).
 template <typename TS>
-__global__ void __launch_bounds__(256) pc_chol_diag_kernel(int64_t D, void* state, int64_t k0) {
-    __shared__ TS Ls[kNB][kNB + 1];
-    TS* M = mat_of<TS>(state);
-    double* h = (double*)state;
-    const int nb = (int)((D - k0) < kNB ? (D - k0) : kNB);
-    for (int e = threadIdx.x; e < nb * nb; e += blockDim.x) {
-        const int i = e / nb, j = e % nb;
-        Ls[i][j] = M[(k0 + i) * D + k0 + j];
-    }
-    __syncthreads();
-    for (int j = 0; j < nb; ++j) {
-        if (threadIdx.x == 0) {
-            const TS p = Ls[j][j];
-            if (!(p > (TS)0)) {
-                if (h[kPcFailedPivot] == 0.0) h[kPcFailedPivot] = (double)(k0 + j + 1);
-                Ls[j][j] = (TS)NAN;
-            } else {
-                Ls[j][j] = sqrt(p);
-            }
-        }
-        __syncthreads();
-        const TS piv = Ls[j][j];
-        for (int i = j + 1 + threadIdx.x; i < nb; i += blockDim.x) Ls[i][j] /= piv;
-        __syncthreads();
-        for (int e = threadIdx.x; e < nb * nb; e += blockDim.x) {
-            const int i = e / nb, c = e % nb;
-            if (i > j && c > j && c <= i) Ls[i][c] -= Ls[i][j] * Ls[c][j];
-        }
-        __syncthreads();
-    }
-    for (int e = threadIdx.x; e < nb * nb; e += blockDim.x) {
-        const int i = e / nb, j = e % nb;
-        M[(k0 + i) * D + k0 + j] = (j <= i) ? Ls[i][j] : (TS)0;
-    }
-}
-
-// Panel: rows i >= k0+nb solve x L_kk^T = a for their nb entries of block column k0.
-template <typename TS>
-__global__ void __launch_bounds__(128) pc_chol_panel_kernel(int64_t D, void* state, int64_t k0) {
+__global__ void __launch_bounds__(256) panel_kernel(St<TS> st, int64_t k0) {
     __shared__ TS Lk[kNB][kNB + 1];
-    TS* M = mat_of<TS>(state);
+    const int l = blockIdx.x;
+    const int64_t D = st.D;
+    TS* M = st.M(l);
     const int nb = (int)((D - k0) < kNB ? (D - k0) : kNB);
-    for (int e = threadIdx.x; e < nb * nb; e += blockDim.x) {
-        const int i = e / nb, j = e % nb;
-        Lk[i][j] = M[(k0 + i) * D + k0 + j];
+    const int tid = threadIdx.x, lane = tid & 31;
+    for (int e = tid; e < kNB * kNB; e += blockDim.x) {
+        const int i = e / kNB, j = e % kNB;
+        TS v;
+        if (i < nb && j < nb)
+            v = (j <= i) ? M[(k0 + i) * D + k0 + j] : (TS)0;
+        else
+            v = (i == j) ? (TS)1 : (TS)0;  // identity padding of a ragged last block
+        Lk[i][j] = v;
     }
     __syncthreads();
-    const int64_t i = k0 + nb + (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
+    if (tid < 32) {
+        int bad = -1;
+        for (int j = 0; j < kNB; ++j) {
+            const TS p = Lk[j][j];
+            const bool ok = p > (TS)0;
+            if (!ok && bad < 0) bad = j;
+            const TS piv = ok ? (TS)sqrt((double)p) : (TS)NAN;
+            __syncwarp();
+            if (lane == j) Lk[j][j] = piv;
+            if (lane > j) Lk[lane][j] /= piv;
+            __syncwarp();
+            if (lane > j)
+                for (int c = j + 1; c <= lane; ++c) Lk[lane][c] -= Lk[lane][j] * Lk[c][j];
+            __syncwarp();
+        }
+        if (blockIdx.y == 0 && lane == 0 && bad >= 0 && bad < nb) {
+            double* h = st.header(l);
+            if (h[kPcFailedPivot] == 0.0) h[kPcFailedPivot] = (double)(k0 + bad + 1);
+        }
+    }
+    __syncthreads();
+    // The diagonal block of M is left as it is: other CTAs of this launch read
+    // it, and later steps use the block only through its inverse in Dinv.
+    if (blockIdx.y == 0) {
+        // inverse of the (padded) diagonal block: lane c solves L X[:, c] = e_c
+        if (tid < 32) {
+            TS* Di = st.Dinv(l) + (k0 / kNB) * (kNB * kNB);
+            const int c = lane;
+            TS x[kNB];
+#pragma unroll
+            for (int i = 0; i < kNB; ++i) {
+                TS s = (i == c) ? (TS)1 : (TS)0;
+#pragma unroll
+                for (int m = 0; m < i; ++m) s -= Lk[i][m] * x[m];
+                x[i] = (i < c) ? (TS)0 : s / Lk[i][i];
+            }
+#pragma unroll
+            for (int i = 0; i < kNB; ++i) Di[i * kNB + c] = x[i];
+        }
+    }
+    const int64_t i = k0 + nb + (int64_t)blockIdx.y * blockDim.x + tid;
     if (i >= D) return;
     TS x[kNB];
-    for (int j = 0; j < nb; ++j) {
-        TS s = M[i * D + k0 + j];
+#pragma unroll
+    for (int j = 0; j < kNB; ++j) x[j] = (j < nb) ? M[i * D + k0 + j] : (TS)0;
+#pragma unroll
+    for (int j = 0; j < kNB; ++j) {
+        TS s = x[j];
+#pragma unroll
         for (int m = 0; m < j; ++m) s -= x[m] * Lk[j][m];
         x[j] = s / Lk[j][j];
     }
-    for (int j = 0; j < nb; ++j) M[i * D + k0 + j] = x[j];
+#pragma unroll
+    for (int j = 0; j < kNB; ++j)
+        if (j < nb) M[i * D + k0 + j] = x[j];
 }
 
 // Trailing update of the lower triangle: M[i][j] -= sum_m L[i][m] L[j][m] over
-// the panel columns m in [k0, k0+nb), for i >= j >= k0+nb. 64x64 tiles.
+// the panel columns m in [k0, k0+nb), i >= j >= k0+nb. 64x64 tiles, grid z = layer.
 template <typename TS>
-__global__ void __launch_bounds__(256) pc_chol_update_kernel(int64_t D, void* state, int64_t k0) {
-    if (blockIdx.x > blockIdx.y) return;  // strictly-upper tile
-    __shared__ TS Pi[kNB][kFT + 1];
-    __shared__ TS Pj[kNB][kFT + 1];
-    TS* M = mat_of<TS>(state);
+__global__ void __launch_bounds__(256) update_kernel(St<TS> st, int64_t k0) {
+    if (blockIdx.x > blockIdx.y) return;
+    constexpr int T = 64;
+    __shared__ TS Pi[kNB][T + 1];
+    __shared__ TS Pj[kNB][T + 1];
+    const int l = blockIdx.z;
+    const int64_t D = st.D;
+    TS* M = st.M(l);
     const int nb = (int)((D - k0) < kNB ? (D - k0) : kNB);
     const int64_t s0 = k0 + nb;
-    const int64_t i0 = s0 + (int64_t)blockIdx.y * kFT, j0 = s0 + (int64_t)blockIdx.x * kFT;
+    const int64_t i0 = s0 + (int64_t)blockIdx.y * T, j0 = s0 + (int64_t)blockIdx.x * T;
     const int tid = threadIdx.x, ty = tid / 16, tx = tid % 16;
-    for (int e = tid; e < kNB * kFT; e += 256) {
+    for (int e = tid; e < kNB * T; e += 256) {
         const int r = e / kNB, m = e % kNB;
         Pi[m][r] = (i0 + r < D && m < nb) ? M[(i0 + r) * D + k0 + m] : (TS)0;
         Pj[m][r] = (j0 + r < D && m < nb) ? M[(j0 + r) * D + k0 + m] : (TS)0;
@@ -201,11 +311,17 @@ __global__ void __launch_bounds__(256) pc_chol_update_kernel(int64_t D, void* st
     for (int u = 0; u < 4; ++u)
 #pragma unroll
         for (int v = 0; v < 4; ++v) acc[u][v] = (TS)0;
+#pragma unroll 8
     for (int m = 0; m < kNB; ++m) {
+        TS a[4], b[4];
+#pragma unroll
+        for (int u = 0; u < 4; ++u) a[u] = Pi[m][ty * 4 + u];
+#pragma unroll
+        for (int v = 0; v < 4; ++v) b[v] = Pj[m][tx * 4 + v];
 #pragma unroll
         for (int u = 0; u < 4; ++u)
 #pragma unroll
-            for (int v = 0; v < 4; ++v) acc[u][v] += Pi[m][ty * 4 + u] * Pj[m][tx * 4 + v];
+            for (int v = 0; v < 4; ++v) acc[u][v] += a[u] * b[v];
     }
 #pragma unroll
     for (int u = 0; u < 4; ++u)
@@ -216,140 +332,178 @@ __global__ void __launch_bounds__(256) pc_chol_update_kernel(int64_t D, void* st
         }
 }
 
-// One CTA per query row: forward (L y = q) then backward (L^T x = y)
-// substitution in blocks of kNB rows; y and x live in shared memory.
-template <typename TS>
+// ---------------------------------------------------------------- APPLY
+// grid (query group, layer). G query rows per CTA; y[G][D] in shared memory.
+// Forward, block b:  r = q_b - L_{b,<b} y_<b ;  y_b = Dinv_b r
+// Backward, block b: r = y_b - L_{>b,b}^T x_>b ;  x_b = Dinv_b^T r
+template <typename TS, int G>
 __global__ void __launch_bounds__(256)
-pc_apply_kernel(int64_t D, const void* state, const float* __restrict__ q, int64_t ld_q,
-                TS* __restrict__ out, int64_t ld_out) {
+apply_kernel(St<TS> st, const float* __restrict__ q, int64_t n_q, int64_t ld_q, TS* __restrict__ out,
+             int64_t ld_out) {
     extern __shared__ __align__(16) unsigned char smem_raw[];
-    TS* y = (TS*)smem_raw;             // D entries
-    __shared__ TS part[8][kNB];        // per-warp partial sums
-    __shared__ TS r[kNB];
-    const TS* L = mat_of<TS>(state);
-    const double* h = (const double*)state;
-    const int64_t row = blockIdx.x;
-    const float* qr = q + row * ld_q;
-    TS* xo = out + row * ld_out;
+    TS* y = (TS*)smem_raw;  // [G][D]
+    __shared__ TS part[8][G][kNB];
+    __shared__ TS r[G][kNB];
+    const int l = blockIdx.y;
+    const int64_t D = st.D;
+    const TS* L = st.M(l);
+    const TS* Dv = st.Dinv(l);
+    const double* h = st.header(l);
+    const int64_t g0 = (int64_t)blockIdx.x * G;
+    const int gn = (int)((n_q - g0) < G ? (n_q - g0) : G);
     const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
     if (h[kPcFailedPivot] != 0.0) {
-        for (int64_t i = tid; i < D; i += blockDim.x) xo[i] = (TS)NAN;
+        for (int g = 0; g < gn; ++g)
+            for (int64_t i = tid; i < D; i += blockDim.x) out[(g0 + g) * ld_out + (int64_t)l * D + i] = (TS)NAN;
         return;
     }
-    // forward: y[i] = (q[i] - sum_{m<i} L[i][m] y[m]) / L[i][i]
-    for (int64_t b0 = 0; b0 < D; b0 += kNB) {
+    const int64_t nblk = (D + kNB - 1) / kNB;
+    // forward
+    for (int64_t bi = 0; bi < nblk; ++bi) {
+        const int64_t b0 = bi * kNB;
         const int nb = (int)((D - b0) < kNB ? (D - b0) : kNB);
-        // r[ii] = q[b0+ii] - sum_{m < b0} L[b0+ii][m] y[m]; warps split rows
-        for (int ii = warp; ii < nb; ii += 8) {
-            TS s = (TS)0;
-            for (int64_t m = lane; m < b0; m += 32) s += L[(b0 + ii) * D + m] * y[m];
-            for (int o = 16; o > 0; o >>= 1) s += __shfl_xor_sync(0xffffffffu, s, o);
-            if (lane == 0) r[ii] = (TS)qr[b0 + ii] - s;
-        }
-        __syncthreads();
-        if (warp == 0) {
-            for (int ii = 0; ii < nb; ++ii) {
-                TS s = (lane < ii) ? L[(b0 + ii) * D + b0 + lane] * y[b0 + lane] : (TS)0;
+        for (int ii = warp; ii < kNB; ii += 8) {
+            TS acc[G];
+#pragma unroll
+            for (int g = 0; g < G; ++g) acc[g] = (TS)0;
+            if (ii < nb)
+                for (int64_t m = lane; m < b0; m += 32) {
+                    const TS lv = L[(b0 + ii) * D + m];
+#pragma unroll
+                    for (int g = 0; g < G; ++g) acc[g] += lv * y[g * D + m];
+                }
+#pragma unroll
+            for (int g = 0; g < G; ++g) {
+                TS s = acc[g];
                 for (int o = 16; o > 0; o >>= 1) s += __shfl_xor_sync(0xffffffffu, s, o);
-                if (lane == 0) y[b0 + ii] = (r[ii] - s) / L[(b0 + ii) * D + b0 + ii];
-                __syncwarp();
+                if (lane == 0)
+                    r[g][ii] = (ii < nb && g < gn) ? (TS)q[(g0 + g) * ld_q + (int64_t)l * D + b0 + ii] - s : (TS)0;
             }
         }
         __syncthreads();
+        for (int e = tid; e < G * kNB; e += blockDim.x) {
+            const int g = e / kNB, i = e % kNB;
+            TS s = (TS)0;
+            for (int j = 0; j <= i; ++j) s += Dv[bi * kNB * kNB + i * kNB + j] * r[g][j];
+            if (i < nb) y[g * D + b0 + i] = s;
+        }
+        __syncthreads();
     }
-    // backward: x[i] = (y[i] - sum_{m>i} L[m][i] x[m]) / L[i][i]; x overwrites y
-    const int64_t nblk = (D + kNB - 1) / kNB;
+    // backward (x overwrites y)
     for (int64_t bi = nblk - 1; bi >= 0; --bi) {
         const int64_t b0 = bi * kNB;
         const int nb = (int)((D - b0) < kNB ? (D - b0) : kNB);
         const int64_t e0 = b0 + nb;
-        // lane = column ii of the block, warps stride over solved rows m >= e0
-        TS s = (TS)0;
+        TS acc[G];
+#pragma unroll
+        for (int g = 0; g < G; ++g) acc[g] = (TS)0;
         if (lane < nb)
-            for (int64_t m = e0 + warp; m < D; m += 8) s += L[m * D + b0 + lane] * y[m];
-        part[warp][lane] = s;
-        __syncthreads();
-        if (warp == 0) {
-            TS t = (TS)0;
-            for (int w = 0; w < 8; ++w) t += part[w][lane];
-            if (lane < nb) r[lane] = y[b0 + lane] - t;
-            __syncwarp();
-            for (int ii = nb - 1; ii >= 0; --ii) {
-                TS u = (lane > ii && lane < nb) ? L[(b0 + lane) * D + b0 + ii] * y[b0 + lane] : (TS)0;
-                for (int o = 16; o > 0; o >>= 1) u += __shfl_xor_sync(0xffffffffu, u, o);
-                if (lane == 0) y[b0 + ii] = (r[ii] - u) / L[(b0 + ii) * D + b0 + ii];
-                __syncwarp();
+            for (int64_t m = e0 + warp; m < D; m += 8) {
+                const TS lv = L[m * D + b0 + lane];
+#pragma unroll
+                for (int g = 0; g < G; ++g) acc[g] += lv * y[g * D + m];
             }
+#pragma unroll
+        for (int g = 0; g < G; ++g) part[warp][g][lane] = acc[g];
+        __syncthreads();
+        for (int e = tid; e < G * kNB; e += blockDim.x) {
+            const int g = e / kNB, i = e % kNB;
+            TS t = (TS)0;
+            for (int w = 0; w < 8; ++w) t += part[w][g][i];
+            r[g][i] = (i < nb) ? y[g * D + b0 + i] - t : (TS)0;
+        }
+        __syncthreads();
+        for (int e = tid; e < G * kNB; e += blockDim.x) {
+            const int g = e / kNB, i = e % kNB;
+            TS s = (TS)0;
+            for (int j = i; j < kNB; ++j) s += Dv[bi * kNB * kNB + j * kNB + i] * r[g][j];
+            if (i < nb) y[g * D + b0 + i] = s;
         }
         __syncthreads();
     }
-    for (int64_t i = tid; i < D; i += blockDim.x) xo[i] = y[i];
+    for (int g = 0; g < gn; ++g)
+        for (int64_t i = tid; i < D; i += blockDim.x) out[(g0 + g) * ld_out + (int64_t)l * D + i] = y[g * D + i];
 }
 
 template <typename TS>
-cudaError_t factor_impl(int64_t D, void* state, int64_t n_total, double la, double lr,
+cudaError_t factor_impl(int n_layers, int64_t D, void* state, int64_t n_total, double la, double lr,
                         cudaStream_t s) {
+    St<TS> st = state_of<TS>(state, D);
     note_launches(2);
-    pc_prepare_kernel<TS><<<1, 256, 0, s>>>(D, state, n_total, la, lr);
-    int64_t blocks = (D * D + 255) / 256;
-    if (blocks > 152 * 32) blocks = 152 * 32;
-    pc_scale_kernel<TS><<<(unsigned)blocks, 256, 0, s>>>(D, state);
+    prepare_kernel<TS><<<n_layers, 256, 0, s>>>(st, n_total, la, lr);
+    int64_t blocks = (D * D * n_layers + 255) / 256;
+    if (blocks > 152 * 16) blocks = 152 * 16;
+    scale_kernel<TS><<<(unsigned)blocks, 256, 0, s>>>(st, n_layers);
     for (int64_t k0 = 0; k0 < D; k0 += kNB) {
-        note_launches(1);
-        pc_chol_diag_kernel<TS><<<1, 256, 0, s>>>(D, state, k0);
         const int64_t rest = D - k0 - kNB;
+        const unsigned chunks = (unsigned)(rest > 0 ? (rest + 255) / 256 : 1);
+        note_launches(1);
+        panel_kernel<TS><<<dim3(n_layers, chunks), 256, 0, s>>>(st, k0);
         if (rest > 0) {
-            note_launches(2);
-            pc_chol_panel_kernel<TS><<<(unsigned)((rest + 127) / 128), 128, 0, s>>>(D, state, k0);
-            const unsigned t = (unsigned)((rest + kFT - 1) / kFT);
-            pc_chol_update_kernel<TS><<<dim3(t, t), 256, 0, s>>>(D, state, k0);
+            const unsigned t = (unsigned)((rest + 63) / 64);
+            note_launches(1);
+            update_kernel<TS><<<dim3(t, t, n_layers), 256, 0, s>>>(st, k0);
         }
     }
+    return cudaGetLastError();
+}
+
+template <typename TS, int G>
+cudaError_t apply_impl(int n_layers, int64_t D, const void* state, const float* q, int64_t n_q, int64_t ld_q,
+                       void* qhat, int64_t ld_qhat, cudaStream_t s) {
+    St<TS> st = state_of<TS>(const_cast<void*>(state), D);
+    const size_t smem = (size_t)G * D * sizeof(TS);
+    cudaError_t e = cudaFuncSetAttribute(apply_kernel<TS, G>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                         (int)smem);
+    if (e != cudaSuccess) return e;
+    note_launches(1);
+    apply_kernel<TS, G><<<dim3((unsigned)((n_q + G - 1) / G), n_layers), 256, smem, s>>>(st, q, n_q, ld_q,
+                                                                                     (TS*)qhat, ld_qhat);
     return cudaGetLastError();
 }
 
 }  // namespace
 
-cudaError_t launch_pc_fit(int64_t D, tda_dtype sdt, void* state, const float* phi, int64_t n,
+int64_t precondition_apply_max_d(tda_dtype sdt) {
+    // one query row of D elements must fit the shared-memory budget of APPLY
+    return (int64_t)(160 * 1024) / (sdt == TDA_F64 ? 8 : 4);
+}
+
+cudaError_t launch_pc_fit(int n_layers, int64_t D, tda_dtype sdt, void* state, const float* phi, int64_t n,
                           int64_t ld, cudaStream_t s) {
     if (n == 0) return cudaSuccess;
-    const unsigned t = (unsigned)((D + kFT - 1) / kFT);
-    note_launches(1);
-    if (sdt == TDA_F64)
-        pc_fit_kernel<double><<<dim3(t, t), 256, 0, s>>>(D, state, phi, n, ld);
-    else
-        pc_fit_kernel<float><<<dim3(t, t), 256, 0, s>>>(D, state, phi, n, ld);
-    return cudaGetLastError();
-}
-
-cudaError_t launch_pc_factor(int64_t D, tda_dtype sdt, void* state, int64_t n_total,
-                             double lambda_abs, double lambda_rel, cudaStream_t s) {
-    if (sdt == TDA_F64) return factor_impl<double>(D, state, n_total, lambda_abs, lambda_rel, s);
-    return factor_impl<float>(D, state, n_total, lambda_abs, lambda_rel, s);
-}
-
-cudaError_t launch_pc_apply(int64_t D, tda_dtype sdt, const void* state, const float* q,
-                            int64_t n_q, int64_t ld_q, void* qhat, int64_t ld_qhat,
-                            cudaStream_t s) {
-    if (n_q == 0) return cudaSuccess;
-    const size_t el = sdt == TDA_F64 ? sizeof(double) : sizeof(float);
-    const size_t smem = (size_t)D * el;
-    cudaError_t e;
     note_launches(1);
     if (sdt == TDA_F64) {
-        e = cudaFuncSetAttribute(pc_apply_kernel<double>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                 (int)smem);
-        if (e != cudaSuccess) return e;
-        pc_apply_kernel<double><<<(unsigned)n_q, 256, smem, s>>>(D, state, q, ld_q, (double*)qhat,
-                                                                  ld_qhat);
+        const unsigned t = (unsigned)((D + 63) / 64);
+        fit_f64_kernel<<<dim3(t, t, n_layers), 256, 0, s>>>(state_of<double>(state, D), phi, n, ld);
     } else {
-        e = cudaFuncSetAttribute(pc_apply_kernel<float>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                 (int)smem);
-        if (e != cudaSuccess) return e;
-        pc_apply_kernel<float><<<(unsigned)n_q, 256, smem, s>>>(D, state, q, ld_q, (float*)qhat,
-                                                                 ld_qhat);
+        const unsigned t = (unsigned)((D + kFT - 1) / kFT);
+        fit_f32_kernel<<<dim3(t, t, n_layers), 256, 0, s>>>(state_of<float>(state, D), phi, n, ld);
     }
     return cudaGetLastError();
+}
+
+cudaError_t launch_pc_factor(int n_layers, int64_t D, tda_dtype sdt, void* state, int64_t n_total,
+                             double lambda_abs, double lambda_rel, cudaStream_t s) {
+    if (sdt == TDA_F64) return factor_impl<double>(n_layers, D, state, n_total, lambda_abs, lambda_rel, s);
+    return factor_impl<float>(n_layers, D, state, n_total, lambda_abs, lambda_rel, s);
+}
+
+cudaError_t launch_pc_apply(int n_layers, int64_t D, tda_dtype sdt, const void* state, const float* q,
+                            int64_t n_q, int64_t ld_q, void* qhat, int64_t ld_qhat, cudaStream_t s) {
+    if (n_q == 0) return cudaSuccess;
+    const size_t el = sdt == TDA_F64 ? 8 : 4;
+    const size_t budget = 160 * 1024;
+    if (sdt == TDA_F64) {
+        if ((size_t)D * el * 8 <= budget)
+            return apply_impl<double, 8>(n_layers, D, state, q, n_q, ld_q, qhat, ld_qhat, s);
+        if ((size_t)D * el * 2 <= budget)
+            return apply_impl<double, 2>(n_layers, D, state, q, n_q, ld_q, qhat, ld_qhat, s);
+        return apply_impl<double, 1>(n_layers, D, state, q, n_q, ld_q, qhat, ld_qhat, s);
+    }
+    if ((size_t)D * el * 8 <= budget) return apply_impl<float, 8>(n_layers, D, state, q, n_q, ld_q, qhat, ld_qhat, s);
+    if ((size_t)D * el * 2 <= budget) return apply_impl<float, 2>(n_layers, D, state, q, n_q, ld_q, qhat, ld_qhat, s);
+    return apply_impl<float, 1>(n_layers, D, state, q, n_q, ld_q, qhat, ld_qhat, s);
 }
 
 }  // namespace tda

@@ -7,55 +7,82 @@
 namespace tda {
 namespace {
 
-constexpr int kST = 64;   // output tile edge (queries x train)
+constexpr int kTQ = 32;   // queries per tile
+constexpr int kTT = 64;   // train examples per tile
 constexpr int kSK = 32;   // feature chunk
 constexpr int kSThreads = 256;
 
-// TQ: element type of Qhat; TA: accumulation type (double when Qhat is fp64).
+__device__ __forceinline__ void load4(const float* p, bool ok, bool vec, float* out, int64_t lim) {
+    if (ok && vec) {
+        const float4 v = *reinterpret_cast<const float4*>(p);
+        out[0] = v.x; out[1] = v.y; out[2] = v.z; out[3] = v.w;
+    } else {
+        for (int i = 0; i < 4; ++i) out[i] = (ok && i < lim) ? p[i] : 0.f;
+    }
+}
+__device__ __forceinline__ void load4(const double* p, bool ok, bool, double* out, int64_t lim) {
+    for (int i = 0; i < 4; ++i) out[i] = (ok && i < lim) ? p[i] : 0.0;
+}
+
+// S tile (32 queries x 64 train) = Qhat_tile Phi_tile^T over D in chunks of 32.
+// Thread (tq = tid/32, tt = tid%32) owns queries tq*4..+3 and train tt, tt+32.
+// Operands are read 16 bytes at a time along the feature axis (coalesced) and
+// staged transposed ([feature][row], padded) in shared memory.
 template <typename TQ, typename TA>
 __global__ void __launch_bounds__(kSThreads)
 score_kernel(const TQ* __restrict__ Q, int64_t n_q, int64_t ld_q, const float* __restrict__ P,
              int64_t n_t, int64_t ld_p, int64_t D, float* __restrict__ S, int64_t ld_S,
              float beta) {
-    __shared__ TA Qs[kSK][kST + 1];
-    __shared__ TA Ps[kSK][kST + 1];
+    __shared__ TA Qs[kSK][kTQ + 1];
+    __shared__ TA Ps[kSK][kTT + 1];
     const int tid = threadIdx.x;
-    const int64_t q0 = (int64_t)blockIdx.y * kST, i0 = (int64_t)blockIdx.x * kST;
-    const int ty = tid / 16, tx = tid % 16;
-    TA acc[4][4];
+    const int64_t q0 = (int64_t)blockIdx.y * kTQ, i0 = (int64_t)blockIdx.x * kTT;
+    const int tq = tid >> 5, tt = tid & 31;
+    const bool vq = (sizeof(TQ) == 4) && ((ld_q & 3) == 0) && (((uintptr_t)Q & 15) == 0);
+    const bool vp = ((ld_p & 3) == 0) && (((uintptr_t)P & 15) == 0);
+    TA acc[4][2];
 #pragma unroll
-    for (int a = 0; a < 4; ++a)
-#pragma unroll
-        for (int b = 0; b < 4; ++b) acc[a][b] = (TA)0;
+    for (int a = 0; a < 4; ++a) acc[a][0] = acc[a][1] = (TA)0;
 
     for (int64_t f0 = 0; f0 < D; f0 += kSK) {
-        for (int e = tid; e < kSK * kST; e += kSThreads) {
-            const int rr = e / kSK, ff = e % kSK;
-            const int64_t f = f0 + ff;
-            const int64_t q = q0 + rr, i = i0 + rr;
-            Qs[ff][rr] = (q < n_q && f < D) ? (TA)Q[q * ld_q + f] : (TA)0;
-            Ps[ff][rr] = (i < n_t && f < D) ? (TA)P[i * ld_p + f] : (TA)0;
+        {   // Q tile: 32 rows x 32 features, one 4-wide load per thread
+            const int r = tid >> 3, k4 = (tid & 7) * 4;
+            const int64_t q = q0 + r, f = f0 + k4;
+            TQ v[4];
+            load4(Q + q * ld_q + f, q < n_q && f < D, vq && f + 3 < D, v, D - f);
+#pragma unroll
+            for (int i = 0; i < 4; ++i) Qs[k4 + i][r] = (TA)v[i];
+        }
+#pragma unroll
+        for (int h = 0; h < 2; ++h) {  // Phi tile: 64 rows x 32 features
+            const int e = tid + h * kSThreads;
+            const int r = e >> 3, k4 = (e & 7) * 4;
+            const int64_t i = i0 + r, f = f0 + k4;
+            float v[4];
+            load4(P + i * ld_p + f, i < n_t && f < D, vp && f + 3 < D, v, D - f);
+#pragma unroll
+            for (int u = 0; u < 4; ++u) Ps[k4 + u][r] = (TA)v[u];
         }
         __syncthreads();
 #pragma unroll 8
-        for (int ff = 0; ff < kSK; ++ff) {
-            TA a[4], b[4];
+        for (int k = 0; k < kSK; ++k) {
+            TA a[4];
 #pragma unroll
-            for (int u = 0; u < 4; ++u) a[u] = Qs[ff][ty * 4 + u];
+            for (int u = 0; u < 4; ++u) a[u] = Qs[k][tq * 4 + u];
+            const TA b0 = Ps[k][tt], b1 = Ps[k][tt + 32];
 #pragma unroll
-            for (int u = 0; u < 4; ++u) b[u] = Ps[ff][tx * 4 + u];
-#pragma unroll
-            for (int u = 0; u < 4; ++u)
-#pragma unroll
-                for (int v = 0; v < 4; ++v) acc[u][v] += a[u] * b[v];
+            for (int u = 0; u < 4; ++u) {
+                acc[u][0] += a[u] * b0;
+                acc[u][1] += a[u] * b1;
+            }
         }
         __syncthreads();
     }
 #pragma unroll
     for (int u = 0; u < 4; ++u)
 #pragma unroll
-        for (int v = 0; v < 4; ++v) {
-            const int64_t q = q0 + ty * 4 + u, i = i0 + tx * 4 + v;
+        for (int v = 0; v < 2; ++v) {
+            const int64_t q = q0 + tq * 4 + u, i = i0 + tt + 32 * v;
             if (q < n_q && i < n_t) {
                 float* dst = S + q * ld_S + i;
                 *dst = (beta == 0.f) ? (float)acc[u][v] : (float)((TA)beta * (TA)(*dst) + acc[u][v]);
@@ -174,7 +201,7 @@ cudaError_t launch_score(const void* Qhat, tda_dtype qdt, int64_t n_q, int64_t l
                          const float* Phi, int64_t n_t, int64_t ld_phi, int64_t D, float* S,
                          int64_t ld_S, float beta, cudaStream_t s) {
     if (n_q == 0 || n_t == 0) return cudaSuccess;
-    dim3 grid((unsigned)((n_t + kST - 1) / kST), (unsigned)((n_q + kST - 1) / kST));
+    dim3 grid((unsigned)((n_t + kTT - 1) / kTT), (unsigned)((n_q + kTQ - 1) / kTQ));
     note_launches(1);
     if (qdt == TDA_F64)
         score_kernel<double, double><<<grid, kSThreads, 0, s>>>(

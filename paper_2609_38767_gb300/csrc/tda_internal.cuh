@@ -91,14 +91,15 @@ cudaError_t launch_similarity_gram(const tda_layer_desc& L, tda_dtype dt, const 
                                    const void* Bq, int64_t n_q, const void* At, const void* Bt,
                                    int64_t n_t, float* S, int64_t ld_S, float beta, cudaStream_t s);
 
-// Preconditioner.
-cudaError_t launch_pc_fit(int64_t D, tda_dtype sdt, void* state, const float* phi, int64_t n,
+// Preconditioner, n_layers layers of D features each (layer l's columns at
+// offset l*D of every feature row).
+int64_t precondition_apply_max_d(tda_dtype sdt);
+cudaError_t launch_pc_fit(int n_layers, int64_t D, tda_dtype sdt, void* state, const float* phi, int64_t n,
                           int64_t ld, cudaStream_t s);
-cudaError_t launch_pc_factor(int64_t D, tda_dtype sdt, void* state, int64_t n_total,
+cudaError_t launch_pc_factor(int n_layers, int64_t D, tda_dtype sdt, void* state, int64_t n_total,
                              double lambda_abs, double lambda_rel, cudaStream_t s);
-cudaError_t launch_pc_apply(int64_t D, tda_dtype sdt, const void* state, const float* q,
-                            int64_t n_q, int64_t ld_q, void* qhat, int64_t ld_qhat,
-                            cudaStream_t s);
+cudaError_t launch_pc_apply(int n_layers, int64_t D, tda_dtype sdt, const void* state, const float* q,
+                            int64_t n_q, int64_t ld_q, void* qhat, int64_t ld_qhat, cudaStream_t s);
 
 // Scores and ranking.
 cudaError_t launch_score(const void* Qhat, tda_dtype qdt, int64_t n_q, int64_t ld_q,

@@ -41,8 +41,10 @@ def test_layer_desc_layout_matches_header():
 
 def test_version_and_state_bytes(libs):
     assert tda.tda_version() >= 100
-    assert tda.tda_precondition_state_bytes(256, tda.TDA_F64) == 64 + 256 * 256 * 8
-    assert tda.tda_precondition_state_bytes(10, tda.TDA_F32) == 64 + 400
+    def rup(x):
+        return (x + 255) // 256 * 256
+    assert tda.tda_precondition_state_bytes(256, tda.TDA_F64) == rup(64 + (256 * 256 + 8 * 1024) * 8)
+    assert tda.tda_precondition_state_bytes(10, tda.TDA_F32) == rup(64 + (100 + 1024) * 4)
     assert tda.tda_precondition_state_bytes(0, tda.TDA_F32) == 0
 
 
@@ -71,10 +73,15 @@ def test_host_validation_rejects_bad_arguments(libs):
     assert _err(tda.tda_topk, 16, 2, 10, 10, 0, 16, stream=s) == tda.TDA_ERR_INVALID_ARG
     assert _err(tda.tda_score, 16, tda.TDA_BF16, 2, 8, 16, 3, 8, 8, 16, 3, stream=s) == tda.TDA_ERR_INVALID_ARG
     assert _err(tda.tda_score, 16, tda.TDA_F32, 2, 4, 16, 3, 8, 8, 16, 3, stream=s) == tda.TDA_ERR_INVALID_ARG
-    assert _err(tda.tda_precondition, 9, 8, tda.TDA_F64, 16, stream=s) == tda.TDA_ERR_INVALID_ARG
-    assert _err(tda.tda_precondition, tda.TDA_PC_FACTOR, 8, tda.TDA_F64, 16, n_total=0, lambda_abs=1.0,
+    assert _err(tda.tda_precondition, 9, 1, 8, tda.TDA_F64, 16, stream=s) == tda.TDA_ERR_INVALID_ARG
+    assert _err(tda.tda_precondition, tda.TDA_PC_RESET, 0, 8, tda.TDA_F64, 16, stream=s) == tda.TDA_ERR_INVALID_ARG
+    assert _err(tda.tda_precondition, tda.TDA_PC_FIT_ACCUM, 3, 8, tda.TDA_F32, 16, phi=16, n=4, ld_phi=16,
+                stream=s) == tda.TDA_ERR_INVALID_ARG  # ld_phi < 3*8
+    assert _err(tda.tda_precondition, tda.TDA_PC_APPLY, 1, 50000, tda.TDA_F32, 16, q=16, n_q=1, ld_q=50000,
+                qhat=16, ld_qhat=50000, stream=s) == tda.TDA_ERR_UNSUPPORTED
+    assert _err(tda.tda_precondition, tda.TDA_PC_FACTOR, 1, 8, tda.TDA_F64, 16, n_total=0, lambda_abs=1.0,
                 stream=s) == tda.TDA_ERR_INVALID_ARG
-    assert _err(tda.tda_precondition, tda.TDA_PC_FACTOR, 8, tda.TDA_F64, 16, n_total=4, stream=s) \
+    assert _err(tda.tda_precondition, tda.TDA_PC_FACTOR, 1, 8, tda.TDA_F64, 16, n_total=4, stream=s) \
         == tda.TDA_ERR_INVALID_ARG
     assert _err(tda.tda_proj_entries, 0, 0, 2, 0, 4, 4, 16, stream=s) == tda.TDA_ERR_INVALID_ARG
     assert _err(tda.tda_route_set_model, 1) == tda.TDA_ERR_INVALID_ARG

@@ -159,17 +159,17 @@ def _precond_pipeline(dev, orc, N, Nq, T, di, do, k, dtype, sdt, lam_abs, lam_re
     _, phi = gpu_project(L, dtype, to_dev(A, dtype, dev), to_dev(B, dtype, dev), N, tda.TDA_ROUTE_FACTORED, dev)
     _, q = gpu_project(L, dtype, to_dev(Aq, dtype, dev), to_dev(Bq, dtype, dev), Nq, tda.TDA_ROUTE_FACTORED, dev)
     state = torch.empty(tda.tda_precondition_state_bytes(D, sdt), dtype=torch.uint8, device=dev)
-    tda.tda_precondition(tda.TDA_PC_RESET, D, sdt, state)
+    tda.tda_precondition(tda.TDA_PC_RESET, 1, D, sdt, state)
     half = N // 2  # two streamed chunks
-    tda.tda_precondition(tda.TDA_PC_FIT_ACCUM, D, sdt, state, phi=phi, n=half, ld_phi=D)
-    tda.tda_precondition(tda.TDA_PC_FIT_ACCUM, D, sdt, state, phi=phi[half:], n=N - half, ld_phi=D)
-    tda.tda_precondition(tda.TDA_PC_FACTOR, D, sdt, state, n_total=N, lambda_abs=lam_abs,
+    tda.tda_precondition(tda.TDA_PC_FIT_ACCUM, 1, D, sdt, state, phi=phi, n=half, ld_phi=D)
+    tda.tda_precondition(tda.TDA_PC_FIT_ACCUM, 1, D, sdt, state, phi=phi[half:], n=N - half, ld_phi=D)
+    tda.tda_precondition(tda.TDA_PC_FACTOR, 1, D, sdt, state, n_total=N, lambda_abs=lam_abs,
                          lambda_rel_mean_eig=lam_rel)
     qhat = torch.empty((Nq, D), dtype=torch.float64 if sdt == tda.TDA_F64 else torch.float32, device=dev)
-    tda.tda_precondition(tda.TDA_PC_APPLY, D, sdt, state, q=q, n_q=Nq, ld_q=D, qhat=qhat, ld_qhat=D)
+    tda.tda_precondition(tda.TDA_PC_APPLY, 1, D, sdt, state, q=q, n_q=Nq, ld_q=D, qhat=qhat, ld_qhat=D)
     S = torch.empty((Nq, N), device=dev)
     tda.tda_score(qhat, sdt, Nq, D, phi, N, D, D, S, N)
-    info = tda.tda_precondition_info(D, sdt, state)
+    info = tda.tda_precondition_info(1, D, sdt, state)
     tda.tda_device_status()
     # oracle, end to end from the same input bits
     fo = orc.project(synth.to_f64(A, dtype), synth.to_f64(B, dtype), k, k, 0, 0).reshape(N, D)
@@ -197,19 +197,19 @@ def test_preconditioned_scores_bf16_fp32_state_relative_damping(dev, orc):
 def test_precondition_not_spd_is_reported(dev):
     D = 8
     state = torch.empty(tda.tda_precondition_state_bytes(D, tda.TDA_F32), dtype=torch.uint8, device=dev)
-    tda.tda_precondition(tda.TDA_PC_RESET, D, tda.TDA_F32, state)
+    tda.tda_precondition(tda.TDA_PC_RESET, 1, D, tda.TDA_F32, state)
     phi = torch.ones((2, D), device=dev)
-    tda.tda_precondition(tda.TDA_PC_FIT_ACCUM, D, tda.TDA_F32, state, phi=phi, n=2, ld_phi=D)
+    tda.tda_precondition(tda.TDA_PC_FIT_ACCUM, 1, D, tda.TDA_F32, state, phi=phi, n=2, ld_phi=D)
     # make the accumulated matrix indefinite by hand
     m = state[64:].view(torch.float32).view(D, D)
     m[3, 3] = -100.0
-    tda.tda_precondition(tda.TDA_PC_FACTOR, D, tda.TDA_F32, state, n_total=2, lambda_abs=1e-3)
+    tda.tda_precondition(tda.TDA_PC_FACTOR, 1, D, tda.TDA_F32, state, n_total=2, lambda_abs=1e-3)
     with pytest.raises(tda.TdaError) as e:
-        tda.tda_precondition_info(D, tda.TDA_F32, state)
+        tda.tda_precondition_info(1, D, tda.TDA_F32, state)
     assert e.value.status == tda.TDA_ERR_NOT_SPD
     q = torch.ones((1, D), device=dev)
     qh = torch.zeros((1, D), device=dev)
-    tda.tda_precondition(tda.TDA_PC_APPLY, D, tda.TDA_F32, state, q=q, n_q=1, ld_q=D, qhat=qh, ld_qhat=D)
+    tda.tda_precondition(tda.TDA_PC_APPLY, 1, D, tda.TDA_F32, state, q=q, n_q=1, ld_q=D, qhat=qh, ld_qhat=D)
     assert torch.isnan(qh).all()
 
 
@@ -312,3 +312,33 @@ def test_tc_projection_matches_oracle(dev, orc, case):
     assert rel_fro(got, ref) <= TOL[dtype]
     worst = max(rel_fro(got[n], ref[n]) for n in range(N))
     assert worst <= TOL[dtype], worst
+
+
+@pytest.mark.parametrize("sdt,D,lam_abs,lam_rel,tol", [(tda.TDA_F64, 70, 1e-3, 0.0, 1e-9),
+                                                       (tda.TDA_F32, 96, 0.0, 1e-2, 1e-4),
+                                                       (tda.TDA_F32, 1000, 0.0, 1e-2, 1e-3)])
+def test_precondition_batched_layers_match_oracle(dev, orc, sdt, D, lam_abs, lam_rel, tol):
+    # three layers side by side in each feature row, ragged D, streamed in two chunks
+    rng = np.random.default_rng(D)
+    nl, N, Nq = 3, 150, 11
+    phi = (rng.standard_normal((N, nl * D)) * rng.uniform(0.5, 2.0, nl * D)).astype(np.float32)
+    q = rng.standard_normal((Nq, nl * D)).astype(np.float32)
+    per = tda.tda_precondition_state_bytes(D, sdt)
+    state = torch.empty(nl * per, dtype=torch.uint8, device=dev)
+    phid, qd = torch.from_numpy(phi).to(dev), torch.from_numpy(q).to(dev)
+    tda.tda_precondition(tda.TDA_PC_RESET, nl, D, sdt, state)
+    tda.tda_precondition(tda.TDA_PC_FIT_ACCUM, nl, D, sdt, state, phi=phid, n=70, ld_phi=nl * D)
+    tda.tda_precondition(tda.TDA_PC_FIT_ACCUM, nl, D, sdt, state, phi=phid[70:], n=N - 70, ld_phi=nl * D)
+    tda.tda_precondition(tda.TDA_PC_FACTOR, nl, D, sdt, state, n_total=N, lambda_abs=lam_abs,
+                         lambda_rel_mean_eig=lam_rel)
+    qh = torch.empty((Nq, nl * D), dtype=torch.float64 if sdt == tda.TDA_F64 else torch.float32, device=dev)
+    tda.tda_precondition(tda.TDA_PC_APPLY, nl, D, sdt, state, q=qd, n_q=Nq, ld_q=nl * D, qhat=qh, ld_qhat=nl * D)
+    info = tda.tda_precondition_info(nl, D, sdt, state)
+    tda.tda_device_status()
+    got = qh.cpu().numpy().astype(np.float64)
+    for l in range(nl):
+        F = orc.fisher(phi[:, l * D:(l + 1) * D].astype(np.float64))
+        lam = orc.damping(F, lam_abs, lam_rel)
+        assert abs(info[4 * l] - lam) <= 1e-5 * lam and info[4 * l + 2] == 0
+        ref = orc.precondition(F, lam, q[:, l * D:(l + 1) * D].astype(np.float64))
+        assert rel_fro(got[:, l * D:(l + 1) * D], ref) <= tol
