@@ -201,7 +201,7 @@ def test_precondition_not_spd_is_reported(dev):
     phi = torch.ones((2, D), device=dev)
     tda.tda_precondition(tda.TDA_PC_FIT_ACCUM, 1, D, tda.TDA_F32, state, phi=phi, n=2, ld_phi=D)
     # make the accumulated matrix indefinite by hand
-    m = state[64:].view(torch.float32).view(D, D)
+    m = state[64:64 + 4 * D * D].view(torch.float32).view(D, D)
     m[3, 3] = -100.0
     tda.tda_precondition(tda.TDA_PC_FACTOR, 1, D, tda.TDA_F32, state, n_total=2, lambda_abs=1e-3)
     with pytest.raises(tda.TdaError) as e:
