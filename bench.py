@@ -56,7 +56,15 @@ def parse_args():
     p.add_argument("--no-e2e", action="store_true")
     p.add_argument("--no-cpu-baseline", action="store_true")
     p.add_argument("--pool", type=int, default=32, help="pinned host examples per linear for e2e")
-    return p.parse_args()
+    p.add_argument("--linears", default="q,k,v,o,gate,up,down",
+                   help="subset of the block's linears (profiling of a smaller case)")
+    p.add_argument("--project-only", action="store_true",
+                   help="time only the train projection (kernel profiling; not the metric's step)")
+    a = p.parse_args()
+    names = a.linears.split(",")
+    global LINEARS
+    LINEARS = [x for x in LINEARS if x[0] in names]
+    return a
 
 
 def workload(args):
@@ -68,6 +76,7 @@ def workload(args):
         "factors": "A~N(0,1), B~N(0,1e-3), 1% tokens masked (seeded synthetic)",
         "method": "GradDot" if args.no_precondition else "(F+lambda I)^-1-preconditioned, lambda=1e-2*mean eig",
         "topk": args.topk, "l2": "inputs larger than L2 (no flush)",
+        **({"mode": "project-only (kernel profiling)"} if args.project_only else {}),
     }
 
 
@@ -277,6 +286,8 @@ def main():
             if record:
                 e1.record(stream)
                 ev.append((e0, e1, N * (T * (L.d_in + L.d_out) * 2 + 4 * D)))
+        if args.project_only:
+            return
         for li, L in enumerate(layers):
             project("query", li, L, routes[li])
         target = Q
@@ -342,7 +353,7 @@ def main():
 
     # ---- e2e through tda_project_host with pinned host factors
     e2e = None
-    if not args.no_e2e:
+    if not args.no_e2e and not args.project_only:
         P = min(args.pool, N)
         pools = []
         for li, (_, di, do) in enumerate(LINEARS):
@@ -393,7 +404,7 @@ def main():
                "host_pool_examples": P}
 
     cpu = None
-    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+    if rank == 0 and world == 1 and not args.no_cpu_baseline and not args.project_only:
         def factors_of(role, li, e0, n):
             src_a, src_b = (At, Bt) if role == "train" else (Aq, Bq)
             di, do = LINEARS[li][1], LINEARS[li][2]

@@ -344,6 +344,7 @@ apply_kernel(St<TS> st, const float* __restrict__ q, int64_t n_q, int64_t ld_q, 
     TS* y = (TS*)smem_raw;  // [G][D]
     __shared__ TS part[8][G][kNB];
     __shared__ TS r[G][kNB];
+    __shared__ TS Dsm[kNB][kNB + 1];  // inverse of the current diagonal block
     const int l = blockIdx.y;
     const int64_t D = st.D;
     const TS* L = st.M(l);
@@ -362,6 +363,7 @@ apply_kernel(St<TS> st, const float* __restrict__ q, int64_t n_q, int64_t ld_q, 
     for (int64_t bi = 0; bi < nblk; ++bi) {
         const int64_t b0 = bi * kNB;
         const int nb = (int)((D - b0) < kNB ? (D - b0) : kNB);
+        for (int e = tid; e < kNB * kNB; e += blockDim.x) Dsm[e / kNB][e % kNB] = Dv[bi * kNB * kNB + e];
         for (int ii = warp; ii < kNB; ii += 8) {
             TS acc[G];
 #pragma unroll
@@ -384,7 +386,7 @@ apply_kernel(St<TS> st, const float* __restrict__ q, int64_t n_q, int64_t ld_q, 
         for (int e = tid; e < G * kNB; e += blockDim.x) {
             const int g = e / kNB, i = e % kNB;
             TS s = (TS)0;
-            for (int j = 0; j <= i; ++j) s += Dv[bi * kNB * kNB + i * kNB + j] * r[g][j];
+            for (int j = 0; j <= i; ++j) s += Dsm[i][j] * r[g][j];
             if (i < nb) y[g * D + b0 + i] = s;
         }
         __syncthreads();
@@ -394,6 +396,7 @@ apply_kernel(St<TS> st, const float* __restrict__ q, int64_t n_q, int64_t ld_q, 
         const int64_t b0 = bi * kNB;
         const int nb = (int)((D - b0) < kNB ? (D - b0) : kNB);
         const int64_t e0 = b0 + nb;
+        for (int e = tid; e < kNB * kNB; e += blockDim.x) Dsm[e / kNB][e % kNB] = Dv[bi * kNB * kNB + e];
         TS acc[G];
 #pragma unroll
         for (int g = 0; g < G; ++g) acc[g] = (TS)0;
@@ -416,7 +419,7 @@ apply_kernel(St<TS> st, const float* __restrict__ q, int64_t n_q, int64_t ld_q, 
         for (int e = tid; e < G * kNB; e += blockDim.x) {
             const int g = e / kNB, i = e % kNB;
             TS s = (TS)0;
-            for (int j = i; j < kNB; ++j) s += Dv[bi * kNB * kNB + j * kNB + i] * r[g][j];
+            for (int j = i; j < kNB; ++j) s += Dsm[j][i] * r[g][j];
             if (i < nb) y[g * D + b0 + i] = s;
         }
         __syncthreads();
@@ -501,7 +504,7 @@ cudaError_t launch_pc_apply(int n_layers, int64_t D, tda_dtype sdt, const void* 
             return apply_impl<double, 2>(n_layers, D, state, q, n_q, ld_q, qhat, ld_qhat, s);
         return apply_impl<double, 1>(n_layers, D, state, q, n_q, ld_q, qhat, ld_qhat, s);
     }
-    if ((size_t)D * el * 8 <= budget) return apply_impl<float, 8>(n_layers, D, state, q, n_q, ld_q, qhat, ld_qhat, s);
+    if ((size_t)D * el * 4 <= budget) return apply_impl<float, 4>(n_layers, D, state, q, n_q, ld_q, qhat, ld_qhat, s);
     if ((size_t)D * el * 2 <= budget) return apply_impl<float, 2>(n_layers, D, state, q, n_q, ld_q, qhat, ld_qhat, s);
     return apply_impl<float, 1>(n_layers, D, state, q, n_q, ld_q, qhat, ld_qhat, s);
 }
