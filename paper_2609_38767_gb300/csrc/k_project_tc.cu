@@ -18,8 +18,9 @@
 // Warp roles (256 threads, one persistent CTA per SM):
 //   warp 0  TMA producer: 128x64 bf16 factor tiles into the stage ring
 //   warp 1  TMEM allocator; lane 0 issues the MMAs
-//   warp 2  sign generator: k x 64 bf16 +-1 tiles into the stage ring
-//   warp 3  idle
+//   warps 2-3  sign generators: k x 64 bf16 +-1 tiles into the stage ring,
+//           each warp one half of every 128-byte row (one warp alone falls
+//           behind the HBM stream)
 //   warps 4-7  epilogue: TMEM -> registers -> shared -> token contraction
 // Accumulators are double-buffered in TMEM, so the epilogue of one tile
 // overlaps the MMAs of the next. Every wait is bounded (about 1 s); on expiry
@@ -186,12 +187,14 @@ __host__ __device__ constexpr uint32_t idesc_bf16(int M, int N) {
     return (1u << 4) | (1u << 7) | (1u << 10) | ((uint32_t)(N >> 3) << 17) | ((uint32_t)(M >> 4) << 24);
 }
 
-// Row n of a K-major 128B-swizzled sign tile: the 64 signs of column n over
-// the K chunk, as bf16 +1 (0x3F80) or -1 (0xBF80).
-__device__ __forceinline__ void write_sign_row(uint8_t* tile, int n, uint64_t w) {
+// Half `half` (16-byte chunks 4*half .. 4*half+3) of row n of a K-major
+// 128B-swizzled sign tile: signs of column n over the K chunk, as bf16 +1
+// (0x3F80) or -1 (0xBF80). Two generator warps each write one half.
+__device__ __forceinline__ void write_sign_half(uint8_t* tile, int n, uint64_t w, int half) {
     uint8_t* row = tile + (n >> 3) * 1024 + (n & 7) * 128;
 #pragma unroll
-    for (int c = 0; c < 8; ++c) {
+    for (int cc = 0; cc < 4; ++cc) {
+        const int c = cc + 4 * half;
         const uint32_t bits = (uint32_t)(w >> (8 * c)) & 0xFFu;
         uint32_t q[4];
 #pragma unroll
@@ -217,7 +220,7 @@ project_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant
     float* stY = stX + kTileM * C::kStageLd;      // [128][K+4] Bt rows
     uint64_t* bars = (uint64_t*)(stY + kTileM * C::kStageLd);
     uint64_t* full = bars;                        // TMA landed        (count 1 + tx)
-    uint64_t* sready = bars + C::kStages;         // signs written     (count 1)
+    uint64_t* sready = bars + C::kStages;         // signs written     (count 2)
     uint64_t* empty = bars + 2 * C::kStages;      // MMAs done reading (count 1)
     uint64_t* tfull = bars + 3 * C::kStages;      // [2] accumulators ready
     uint64_t* tempty = tfull + 2;                 // [2] accumulators drained (count 4)
@@ -229,7 +232,7 @@ project_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant
     if (threadIdx.x == 0) {
         for (int s = 0; s < C::kStages; ++s) {
             mbar_init(smem_u32(&full[s]), 1);
-            mbar_init(smem_u32(&sready[s]), 1);
+            mbar_init(smem_u32(&sready[s]), 2);
             mbar_init(smem_u32(&empty[s]), 1);
         }
         for (int b = 0; b < 2; ++b) {
@@ -327,8 +330,8 @@ project_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant
                 atomicOr(p.err, kErrTimeout);
                 break;
             }
-    } else if (warp == 2) {
-        // ---------------- sign generator
+    } else if (warp == 2 || warp == 3) {
+        // ---------------- sign generators (two warps, one half-row each)
         uint32_t ring = 0;
         bool ok = true;
         for (int64_t n = blockIdx.x; ok && n < p.N; n += gridDim.x)
@@ -348,7 +351,8 @@ project_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant
                     const uint64_t key = side_b ? p.key_out : p.key_in;
                     const uint64_t rb = (uint64_t)(side_b ? kc - p.nk_in : kc);
                     uint8_t* tile = sS + (size_t)s * C::kSignBytes;
-                    for (int col = lane; col < K; col += 32) write_sign_row(tile, col, sign_word(key, (uint32_t)col, rb));
+                    for (int col = lane; col < K; col += 32)
+                        write_sign_half(tile, col, sign_word(key, (uint32_t)col, rb), warp - 2);
                     fence_proxy_async();
                     __syncwarp();
                     if (lane == 0) mbar_arrive(smem_u32(&sready[s]));
