@@ -39,6 +39,15 @@ LINEARS = [("q", 2048, 2048), ("k", 2048, 2048), ("v", 2048, 2048), ("o", 2048, 
            ("gate", 2048, 8192), ("up", 2048, 8192), ("down", 8192, 2048)]
 METRIC = "train examples attributed/sec (project+score)"
 
+# DRAM traffic of the tensor-core projection kernel, from one ncu capture
+# (dram__bytes_read.sum + dram__bytes_write.sum) of 608 examples of the 2048x2048
+# linear (profiles/tc_projection_q608.md): measured bytes over algorithmic bytes.
+# Launches of other linears are scaled by their algorithmic bytes (traffic is
+# one read of every factor byte, so it grows in proportion). Valid only for the
+# kernel source it was measured on; any change makes the bench report null.
+TRAFFIC_RATIO = 1.0011893
+TRAFFIC_KERNEL_SHA256 = "56100eb3d1ce2c3d3d1f80b60e922da63ac79b26b764db4bec77b526f36e4eb2"
+
 
 def parse_args():
     p = argparse.ArgumentParser()
@@ -345,9 +354,15 @@ def main():
     hbm = float(peaks.get("hbm_gbs", 6800.0))
     achieved = proj_bytes / (proj_ms * 1e-3) / 1e9
     engines = sorted({tda.tda_project_engine(L, tda.TDA_BF16, At[li], Bt[li]) for li, L in enumerate(layers)})
+    import hashlib
+    with open(os.path.join(ROOT, "paper_2609_38767_gb300", "csrc", "k_project_tc.cu"), "rb") as f:
+        same_kernel = hashlib.sha256(f.read()).hexdigest() == TRAFFIC_KERNEL_SHA256
+    per_launch = proj_bytes / max(len(ev), 1)
     roofline = {"bound": "hbm", "kernel": "factored projection (train, 7 linears)",
                 "engine": "tcgen05" if engines == [1] else ("cuda-core" if engines == [0] else "mixed"), "achieved": achieved,
-                "peak": hbm, "unit": "GB/s", "frac": achieved / hbm, "traffic": None,
+                "peak": hbm, "unit": "GB/s", "frac": achieved / hbm,
+                "traffic": TRAFFIC_RATIO * per_launch if (same_kernel and engines == [1]) else None,
+                "algorithmic_bytes_per_launch": per_launch,
                 "peak_source": "MEASURED_PEAKS.json hbm_gbs" if peaks else "fallback 6.8 TB/s",
                 "share_of_step": proj_ms / (ms * args.steps)}
 
