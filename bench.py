@@ -64,7 +64,7 @@ def parse_args():
     p.add_argument("--e2e-steps", type=int, default=2)
     p.add_argument("--no-e2e", action="store_true")
     p.add_argument("--no-cpu-baseline", action="store_true")
-    p.add_argument("--pool", type=int, default=32, help="pinned host examples per linear for e2e")
+    p.add_argument("--pool", type=int, default=128, help="pinned host examples per linear for e2e")
     p.add_argument("--linears", default="q,k,v,o,gate,up,down",
                    help="subset of the block's linears (profiling of a smaller case)")
     p.add_argument("--project-only", action="store_true",
@@ -402,6 +402,16 @@ def main():
             stream.synchronize()
 
         e2e_step()
+        # raw pinned-host -> device bandwidth on this machine, the ceiling of the e2e leg
+        hb = pools[0][0]
+        db = torch.empty_like(hb, device=dev)
+        torch.cuda.synchronize()
+        t0 = time.perf_counter()
+        for _ in range(3):
+            db.copy_(hb, non_blocking=True)
+        torch.cuda.synchronize()
+        h2d_gbs = 3 * hb.numel() * 2 / (time.perf_counter() - t0) / 1e9
+        del db
         if dist:
             dist.barrier()
         torch.cuda.synchronize()
@@ -416,7 +426,8 @@ def main():
         h2d = N * T * sum(di + do for _, di, do in LINEARS) * 2 + Nq * T * sum(di + do for _, di, do in LINEARS) * 2
         e2e = {"value": world * N / e2e_s, "unit": "examples/s", "h2d_bytes_per_step": h2d,
                "d2h_bytes_per_step": Nq * args.topk * 8, "ms_per_step": e2e_s * 1e3,
-               "host_pool_examples": P}
+               "host_pool_examples": P, "h2d_gbs_measured": h2d_gbs,
+               "h2d_bound_examples_per_s": world * N / (h2d / (h2d_gbs * 1e9))}
 
     cpu = None
     if rank == 0 and world == 1 and not args.no_cpu_baseline and not args.project_only:
