@@ -52,7 +52,7 @@ struct Cfg {
     static constexpr size_t kSmemA = (size_t)kStages * kTileBytes;
     static constexpr size_t kSmemS = (size_t)kStages * kSignBytes;
     static constexpr size_t kSmemStage = 2ull * kTileM * kStageLd * 4;
-    static constexpr size_t kSmemBars = 8 * (3 * kStages + 5) + 16;
+    static constexpr size_t kSmemBars = 8 * (3 * kStages + 7) + 16;
     static constexpr size_t kSmem = 1024 + kSmemA + kSmemS + kSmemStage + kSmemBars;
     // contraction blocking: 16 row groups x 8 column groups of threads
     static constexpr int RB = K / 16 > 0 ? K / 16 : 1;
@@ -66,6 +66,7 @@ struct Params {
     float* phi;
     unsigned int* err;
     int n_ttiles, nk_in, nk_out;
+    int cs;  // CTAs per cluster sharing one example's token tiles (1, 2 or 4)
 };
 
 // ---------------------------------------------------------------- PTX helpers
@@ -164,6 +165,54 @@ __device__ __forceinline__ void tmem_ld16(uint32_t taddr, float* v) {
 #pragma unroll
     for (int i = 0; i < 16; ++i) v[i] = __uint_as_float(r[i]);
 }
+// ---- thread-block cluster helpers (distributed shared memory)
+__device__ __forceinline__ uint32_t cluster_rank() {
+    uint32_t r;
+    asm volatile("mov.u32 %0, %%cluster_ctarank;" : "=r"(r));
+    return r;
+}
+__device__ __forceinline__ void cluster_sync() {
+    asm volatile("barrier.cluster.arrive.release.aligned;\n barrier.cluster.wait.acquire.aligned;" ::: "memory");
+}
+// Address of the same shared-memory location in CTA `rank` of this cluster.
+__device__ __forceinline__ uint32_t map_rank(uint32_t saddr, uint32_t rank) {
+    uint32_t r;
+    asm volatile("mapa.shared::cluster.u32 %0, %1, %2;" : "=r"(r) : "r"(saddr), "r"(rank));
+    return r;
+}
+__device__ __forceinline__ void st_cluster_f32(uint32_t addr, float v) {
+    asm volatile("st.shared::cluster.f32 [%0], %1;" ::"r"(addr), "f"(v) : "memory");
+}
+__device__ __forceinline__ void fence_acq_rel_cluster() { asm volatile("fence.acq_rel.cluster;" ::: "memory"); }
+// Arrive (release, cluster scope) on the barrier at local address `bar` of CTA `rank`.
+__device__ __forceinline__ void mbar_arrive_remote(uint32_t bar, uint32_t rank) {
+    asm volatile("mbarrier.arrive.release.cluster.shared::cluster.b64 _, [%0];" ::"r"(map_rank(bar, rank))
+                 : "memory");
+}
+__device__ __forceinline__ bool mbar_try_wait_cluster(uint32_t bar, uint32_t parity) {
+    uint32_t ok;
+    asm volatile(
+        "{\n .reg .pred p;\n mbarrier.try_wait.parity.acquire.cluster.shared::cta.b64 p, [%1], %2;\n selp.u32 %0, 1, 0, p;\n}"
+        : "=r"(ok)
+        : "r"(bar), "r"(parity)
+        : "memory");
+    return ok != 0;
+}
+__device__ __forceinline__ bool wait_bounded_cluster(uint32_t bar, uint32_t parity, volatile int* abort,
+                                                     unsigned int* err) {
+    const uint64_t t0 = global_ns();
+#pragma unroll 1
+    while (true) {
+        if (mbar_try_wait_cluster(bar, parity)) return true;
+        if (*abort) return false;
+        if (global_ns() - t0 > kTimeoutNs) {
+            atomicOr(err, kErrTimeout);
+            *abort = 1;
+            return false;
+        }
+    }
+}
+
 // OR of `v` over the 128 epilogue threads, through named barrier 1.
 __device__ __forceinline__ bool epi_any(bool v) {
     uint32_t r;
@@ -225,7 +274,9 @@ project_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant
     uint64_t* tfull = bars + 3 * C::kStages;      // [2] accumulators ready
     uint64_t* tempty = tfull + 2;                 // [2] accumulators drained (count 4)
     uint64_t* mma_done = tempty + 2;
-    uint32_t* tmem_slot = (uint32_t*)(mma_done + 1);
+    uint64_t* red_go = mma_done + 1;              // leader -> member: write your partial (count 1)
+    uint64_t* red_full = red_go + 1;              // members -> leader: partials written (count cs-1)
+    uint32_t* tmem_slot = (uint32_t*)(red_full + 1);
     volatile int* abort = (volatile int*)(tmem_slot + 1);
 
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
@@ -240,6 +291,8 @@ project_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant
             mbar_init(smem_u32(&tempty[b]), 4);
         }
         mbar_init(smem_u32(mma_done), 1);
+        mbar_init(smem_u32(red_go), 1);
+        mbar_init(smem_u32(red_full), p.cs > 1 ? p.cs - 1 : 1);
         *abort = 0;
         fence_mbar_init();
     }
@@ -249,8 +302,11 @@ project_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant
     }
     tc_fence_before();
     __syncthreads();
+    cluster_sync();  // every CTA's barriers exist before any remote arrive
     tc_fence_after();
     const uint32_t tmem = *tmem_slot;
+    // examples are shared out per cluster; token tiles per CTA rank within it
+    const uint32_t crank = cluster_rank(), cid = blockIdx.x / p.cs, ncl = gridDim.x / p.cs;
 
     const int nk_tot = p.nk_in + p.nk_out;
     if (warp == 0 && lane == 0) {
@@ -260,8 +316,8 @@ project_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant
         for (int s = 0; s < C::kStages; ++s) issued[s] = false;
         uint32_t ring = 0;
         bool ok = true;
-        for (int64_t n = blockIdx.x; ok && n < p.N; n += gridDim.x)
-            for (int tt = 0; ok && tt < p.n_ttiles; ++tt)
+        for (int64_t n = cid; ok && n < p.N; n += ncl)
+            for (int tt = (int)crank; ok && tt < p.n_ttiles; tt += p.cs)
                 for (int kc = 0; kc < nk_tot; ++kc, ++ring) {
                     const int s = ring % C::kStages;
                     const uint32_t ph = (ring / C::kStages) & 1u;
@@ -292,8 +348,8 @@ project_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant
         uint32_t ring = 0, tile = 0;
         bool ok = true;
         const uint32_t idesc = idesc_bf16(kTileM, K);
-        for (int64_t n = blockIdx.x; ok && n < p.N; n += gridDim.x)
-            for (int tt = 0; ok && tt < p.n_ttiles; ++tt, ++tile) {
+        for (int64_t n = cid; ok && n < p.N; n += ncl)
+            for (int tt = (int)crank; ok && tt < p.n_ttiles; tt += p.cs, ++tile) {
                 const uint32_t b = tile & 1u, use = tile >> 1;
                 if (!wait_bounded(smem_u32(&tempty[b]), (use & 1u) ^ 1u, abort, p.err)) {
                     ok = false;
@@ -334,8 +390,8 @@ project_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant
         // ---------------- sign generators (two warps, one half-row each)
         uint32_t ring = 0;
         bool ok = true;
-        for (int64_t n = blockIdx.x; ok && n < p.N; n += gridDim.x)
-            for (int tt = 0; ok && tt < p.n_ttiles; ++tt)
+        for (int64_t n = cid; ok && n < p.N; n += ncl)
+            for (int tt = (int)crank; ok && tt < p.n_ttiles; tt += p.cs)
                 for (int kc = 0; kc < nk_tot; ++kc, ++ring) {
                     const int s = ring % C::kStages;
                     const uint32_t ph = (ring / C::kStages) & 1u;
@@ -363,15 +419,15 @@ project_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant
         const int et = threadIdx.x - 128;
         const int row = q * 32 + lane;   // token within the tile
         const int rg = et >> 3, cg = et & 7;
-        uint32_t tile = 0;
+        uint32_t tile = 0, red_use = 0;
         bool stop = false;
-        for (int64_t n = blockIdx.x; !stop && n < p.N; n += gridDim.x) {
+        for (int64_t n = cid; !stop && n < p.N; n += ncl) {
             float acc[C::RB][C::CB];
 #pragma unroll
             for (int a = 0; a < C::RB; ++a)
 #pragma unroll
                 for (int c = 0; c < C::CB; ++c) acc[a][c] = 0.f;
-            for (int tt = 0; tt < p.n_ttiles; ++tt, ++tile) {
+            for (int tt = (int)crank; tt < p.n_ttiles; tt += p.cs, ++tile) {
                 const uint32_t b = tile & 1u, use = tile >> 1;
                 bool got = true;
                 if (lane == 0) got = wait_bounded(smem_u32(&tfull[b]), use & 1u, abort, p.err);
@@ -410,6 +466,43 @@ project_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant
                 epi_sync();
             }
             if (stop) break;
+            if (p.cs > 1) {
+                // Cluster reduction of the partial Phi blocks into the leader (rank
+                // 0). The leader's staging buffer (free between tiles) receives
+                // member r's partial at offset (r-1)*K*K, thread-major.
+                constexpr int kPer = C::RB * C::CB;
+                const uint32_t slot = smem_u32(stX) + (uint32_t)(et * kPer) * 4u;
+                bool got = true;
+                if (crank == 0) {
+                    if (et == 0)
+                        for (int r = 1; r < p.cs; ++r) mbar_arrive_remote(smem_u32(red_go), (uint32_t)r);
+                    if (lane == 0) got = wait_bounded_cluster(smem_u32(red_full), red_use & 1u, abort, p.err);
+                    got = __shfl_sync(0xffffffffu, got, 0);
+                    if (epi_any(!got)) break;
+                    for (int r = 1; r < p.cs; ++r) {
+                        const float* part = stX + (r - 1) * K * K + et * kPer;
+#pragma unroll
+                        for (int a = 0; a < C::RB; ++a)
+#pragma unroll
+                            for (int c = 0; c < C::CB; ++c) acc[a][c] += part[a * C::CB + c];
+                    }
+                    epi_sync();  // partials consumed; staging free for the next tile
+                } else {
+                    if (lane == 0) got = wait_bounded_cluster(smem_u32(red_go), red_use & 1u, abort, p.err);
+                    got = __shfl_sync(0xffffffffu, got, 0);
+                    if (epi_any(!got)) break;
+                    const uint32_t dst = map_rank(slot, 0) + (crank - 1) * (uint32_t)(K * K) * 4u;
+#pragma unroll
+                    for (int a = 0; a < C::RB; ++a)
+#pragma unroll
+                        for (int c = 0; c < C::CB; ++c) st_cluster_f32(dst + (uint32_t)(a * C::CB + c) * 4u, acc[a][c]);
+                    fence_acq_rel_cluster();
+                    epi_sync();
+                    if (et == 0) mbar_arrive_remote(smem_u32(red_full), 0u);
+                }
+                ++red_use;
+                if (crank != 0) continue;
+            }
             float* out = p.phi + n * p.ld_phi;
 #pragma unroll
             for (int a = 0; a < C::RB; ++a)
@@ -425,6 +518,7 @@ project_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant
         tc_fence_after();
         tmem_dealloc(tmem, C::kTmemCols);
     }
+    cluster_sync();  // no CTA leaves while a peer may still write to it
 }
 
 // ---------------------------------------------------------------- host side
@@ -499,9 +593,33 @@ cudaError_t launch_k(const tda_layer_desc& L, const void* A, const void* B, int6
     cudaError_t e = cudaFuncSetAttribute(project_tc_kernel<K>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                          (int)C::kSmem);
     if (e != cudaSuccess) return e;
-    const int64_t grid = N < sms ? N : sms;
+    // Fewer examples than SMs: a cluster of cs CTAs shares each example's token
+    // tiles and reduces the partial features through distributed shared memory.
+    int cs = 1;
+    if (N < sms) cs = (2 * N >= sms) ? 2 : 4;
+    while (cs > 1 && cs > p.n_ttiles) cs >>= 1;
+    p.cs = cs;
+    cudaLaunchConfig_t cfg = {};
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeClusterDimension;
+    attr[0].val.clusterDim.x = (unsigned)cs;
+    attr[0].val.clusterDim.y = 1;
+    attr[0].val.clusterDim.z = 1;
+    cfg.blockDim = dim3(kThreads);
+    cfg.dynamicSmemBytes = C::kSmem;
+    cfg.stream = s;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    int64_t clusters = N;
+    int max_clusters = 0;
+    cfg.gridDim = dim3((unsigned)(cs * (sms / cs)));
+    if (cudaOccupancyMaxActiveClusters(&max_clusters, project_tc_kernel<K>, &cfg) != cudaSuccess || max_clusters < 1)
+        max_clusters = sms / cs;
+    if (clusters > max_clusters) clusters = max_clusters;
+    cfg.gridDim = dim3((unsigned)(clusters * cs));
     note_launches(1);
-    project_tc_kernel<K><<<(unsigned)grid, kThreads, C::kSmem, s>>>(tmA, tmB, p);
+    e = cudaLaunchKernelEx(&cfg, project_tc_kernel<K>, tmA, tmB, p);
+    if (e != cudaSuccess) return e;
     return cudaGetLastError();
 }
 

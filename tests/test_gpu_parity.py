@@ -297,6 +297,11 @@ TC_CASES = [
     (5, 129, 136, 64, 64, "bf16"),
     (3, 384, 1024, 256, 32, "bf16"),
     (160, 16, 2048, 2048, 32, "bf16"),
+    # fewer examples than SMs: clusters of CTAs split an example's token tiles
+    (2, 1024, 256, 512, 32, "bf16"),    # 4-CTA clusters, 2 tiles per CTA
+    (50, 300, 128, 64, 16, "bf16"),     # 4-CTA clusters; more clusters than fit
+    (64, 512, 512, 256, 64, "bf16"),    # 2-CTA clusters (the query batch shape)
+    (1, 384, 64, 64, 32, "bf16"),       # one example over 2 CTAs, uneven tiles
 ]
 
 
