@@ -45,8 +45,8 @@ METRIC = "train examples attributed/sec (project+score)"
 # Launches of other linears are scaled by their algorithmic bytes (traffic is
 # one read of every factor byte, so it grows in proportion). Valid only for the
 # kernel source it was measured on; any change makes the bench report null.
-TRAFFIC_RATIO = 1.0011893
-TRAFFIC_KERNEL_SHA256 = "56100eb3d1ce2c3d3d1f80b60e922da63ac79b26b764db4bec77b526f36e4eb2"
+TRAFFIC_RATIO = 1.0011866
+TRAFFIC_KERNEL_SHA256 = "087a05225e94f716b8f93767e3f2054d12d9654fcd132411b2bc97752a13bb69"
 
 
 def parse_args():
