@@ -272,50 +272,47 @@ def main():
             synth.fill_device(x, synth.SEED_B, li + (synth.QUERY_STREAM_OFFSET if role else 0), n, T, do, sb,
                               mask_p=0.01, mask_stream=1000 if role else 0)
             store.append(x)
-    Phi = torch.empty((N, DT), dtype=torch.float32, device=dev)
-    Q = torch.empty((Nq, DT), dtype=torch.float32, device=dev)
-    Qh = torch.empty((Nq, DT), dtype=torch.float32, device=dev)
-    S = torch.empty((Nq, N), dtype=torch.float32, device=dev)
-    idx = torch.empty((Nq, args.topk), dtype=torch.int32, device=dev)
-    val = torch.empty((Nq, args.topk), dtype=torch.float32, device=dev)
-    sbytes = tda.tda_precondition_state_bytes(D, tda.TDA_F32)
-    state = torch.empty(nl * sbytes, dtype=torch.uint8, device=dev)  # all 7 layers, back to back
-    layers = [tda.LayerDesc(di, do, T, k, k, seed=0, layer=li) for li, (_, di, do) in enumerate(LINEARS)]
+    from paper_2609_38767_gb300.block import BlockPipeline
+
+    pipe = BlockPipeline([(di, do) for _, di, do in LINEARS], T, k, N, Nq, topk=args.topk,
+                         precondition=not args.no_precondition, lambda_rel=1e-2, device=dev)
+    layers, Phi, Q, idx, val = pipe.layers, pipe.Phi, pipe.Q, pipe.idx, pipe.val
     torch.cuda.synchronize()
 
     ev = []  # (start, end, algorithmic bytes) per projection launch of the train set
 
     def attribute(project, record=False):
-        routes = [tda.tda_route(L, tda.TDA_OP_PROJECT, N, 0, tda.TDA_BF16)[0] for L in layers]
-        for li, L in enumerate(layers):
-            if record:
-                e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-                e0.record(stream)
-            project("train", li, L, routes[li])
-            if record:
-                e1.record(stream)
-                ev.append((e0, e1, N * (T * (L.d_in + L.d_out) * 2 + 4 * D)))
-        if args.project_only:
-            return
-        for li, L in enumerate(layers):
-            project("query", li, L, routes[li])
-        target = Q
-        if not args.no_precondition:
-            # one batched call per op for the 7 layers (layer l's features at column l*D)
-            tda.tda_precondition(tda.TDA_PC_RESET, nl, D, tda.TDA_F32, state)
-            tda.tda_precondition(tda.TDA_PC_FIT_ACCUM, nl, D, tda.TDA_F32, state, phi=Phi, n=N, ld_phi=DT)
-            tda.tda_precondition(tda.TDA_PC_FACTOR, nl, D, tda.TDA_F32, state, n_total=N, lambda_rel_mean_eig=1e-2)
-            tda.tda_precondition(tda.TDA_PC_APPLY, nl, D, tda.TDA_F32, state, q=Q, n_q=Nq, ld_q=DT, qhat=Qh,
-                                 ld_qhat=DT)
-            target = Qh
-        tda.tda_score(target, tda.TDA_F32, Nq, DT, Phi, N, DT, DT, S, N, 0.0)
-        tda.tda_topk(S, Nq, N, N, args.topk, idx, val)
+        marks = {}
 
-    def project_dev(role, li, L, route):
+        def before(li):
+            if record:
+                e0 = torch.cuda.Event(enable_timing=True)
+                e0.record(stream)
+                marks[li] = e0
+
+        def train(li, L, route, phi, ld):
+            before(li)
+            project("train", li, L, route, phi, ld)
+
+        def after(li):
+            if record:
+                e1 = torch.cuda.Event(enable_timing=True)
+                e1.record(stream)
+                L = layers[li]
+                ev.append((marks[li], e1, N * (T * (L.d_in + L.d_out) * 2 + 4 * D)))
+
+        if args.project_only:
+            for li, (L, route) in enumerate(zip(layers, pipe.routes())):
+                train(li, L, route, Phi[:, li * D:], DT)
+                after(li)
+            return
+        pipe.run(train, lambda li, L, route, phi, ld: project("query", li, L, route, phi, ld), after)
+
+    def project_dev(role, li, L, route, phi, ld):
         if role == "train":
-            tda.tda_project(L, tda.TDA_BF16, At[li], Bt[li], N, Phi[:, li * D:], DT, route)
+            tda.tda_project(L, tda.TDA_BF16, At[li], Bt[li], N, phi, ld, route)
         else:
-            tda.tda_project(L, tda.TDA_BF16, Aq[li], Bq[li], Nq, Q[:, li * D:], DT, route)
+            tda.tda_project(L, tda.TDA_BF16, Aq[li], Bq[li], Nq, phi, ld, route)
 
     for _ in range(args.warmup):
         attribute(project_dev)
@@ -386,14 +383,14 @@ def main():
         idx_h = torch.empty((Nq, args.topk), dtype=torch.int32).pin_memory()
         val_h = torch.empty((Nq, args.topk), dtype=torch.float32).pin_memory()
 
-        def project_host(role, li, L, route):
+        def project_host(role, li, L, route, phi, ld):
             a, b, qa, qb = pools[li]
             if role == "train":
                 for e0 in range(0, N, P):
                     n = min(P, N - e0)
-                    tda.tda_project_host(L, tda.TDA_BF16, a, b, n, Phi[e0:, li * D:], DT, ws, wsb)
+                    tda.tda_project_host(L, tda.TDA_BF16, a, b, n, phi[e0:], ld, ws, wsb)
             else:
-                tda.tda_project_host(L, tda.TDA_BF16, qa, qb, Nq, Q[:, li * D:], DT, ws, wsb)
+                tda.tda_project_host(L, tda.TDA_BF16, qa, qb, Nq, phi, ld, ws, wsb)
 
         def e2e_step():
             attribute(project_host)

@@ -1,0 +1,69 @@
+"""One attribution pass over a block of linear layers, through the C ABI.
+
+A transformer block's linears (e.g. q, k, v, o, gate, up, down) share the token
+count T and the projection size k. For a batch of train and query examples the
+pass is: route choice per linear (Sec. 3.2 / App. A.4 cost model), factored
+projection of every example through every linear (Eq. 2), the per-linear Fisher
+fit and damped inverse applied to the queries (App. B.2, B.3), the query x train
+score matrix summed over the linears (Eq. 4's left side) and the top-k train
+indices per query. Every step is a libtda.so call; this class only owns the
+device buffers and the order of the calls.
+
+Feature layout: linear l's k*k features of an example sit at columns
+[l*k*k, (l+1)*k*k) of one row, so the preconditioner handles all linears in one
+batched call and the score is one GEMM over all features.
+"""
+from __future__ import annotations
+
+import torch
+
+import paper_2609_38767_gb300 as tda
+
+
+class BlockPipeline:
+    def __init__(self, linears, T, k, n_train, n_query, *, topk=100, precondition=True,
+                 lambda_abs=0.0, lambda_rel=1e-2, seed=0, layer0=0, device="cuda"):
+        self.layers = [tda.LayerDesc(di, do, T, k, k, seed=seed, layer=layer0 + i)
+                       for i, (di, do) in enumerate(linears)]
+        self.N, self.Nq, self.D = n_train, n_query, k * k
+        self.nl = len(self.layers)
+        self.DT = self.D * self.nl
+        self.topk, self.precondition = topk, precondition
+        self.lambda_abs, self.lambda_rel = lambda_abs, lambda_rel
+        dev = torch.device(device)
+        self.Phi = torch.empty((n_train, self.DT), dtype=torch.float32, device=dev)
+        self.Q = torch.empty((n_query, self.DT), dtype=torch.float32, device=dev)
+        self.Qh = torch.empty((n_query, self.DT), dtype=torch.float32, device=dev)
+        self.S = torch.empty((n_query, n_train), dtype=torch.float32, device=dev)
+        self.idx = torch.empty((n_query, topk), dtype=torch.int32, device=dev)
+        self.val = torch.empty((n_query, topk), dtype=torch.float32, device=dev)
+        per = tda.tda_precondition_state_bytes(self.D, tda.TDA_F32)
+        self.state = torch.empty(self.nl * per, dtype=torch.uint8, device=dev)
+
+    def routes(self):
+        return [tda.tda_route(L, tda.TDA_OP_PROJECT, self.N, 0, tda.TDA_BF16)[0] for L in self.layers]
+
+    def run(self, project_train, project_query, after_train_linear=None):
+        """project_train(li, L, route, phi_view, ld) fills train features of linear li;
+        project_query likewise for the queries. after_train_linear(li) is called after
+        each train projection (e.g. to record timing events)."""
+        routes = self.routes()
+        D, DT = self.D, self.DT
+        for li, L in enumerate(self.layers):
+            project_train(li, L, routes[li], self.Phi[:, li * D:], DT)
+            if after_train_linear:
+                after_train_linear(li)
+        for li, L in enumerate(self.layers):
+            project_query(li, L, routes[li], self.Q[:, li * D:], DT)
+        target = self.Q
+        if self.precondition:
+            nl, st, f32 = self.nl, self.state, tda.TDA_F32
+            tda.tda_precondition(tda.TDA_PC_RESET, nl, D, f32, st)
+            tda.tda_precondition(tda.TDA_PC_FIT_ACCUM, nl, D, f32, st, phi=self.Phi, n=self.N, ld_phi=DT)
+            tda.tda_precondition(tda.TDA_PC_FACTOR, nl, D, f32, st, n_total=self.N, lambda_abs=self.lambda_abs,
+                                 lambda_rel_mean_eig=self.lambda_rel)
+            tda.tda_precondition(tda.TDA_PC_APPLY, nl, D, f32, st, q=self.Q, n_q=self.Nq, ld_q=DT,
+                                 qhat=self.Qh, ld_qhat=DT)
+            target = self.Qh
+        tda.tda_score(target, tda.TDA_F32, self.Nq, DT, self.Phi, self.N, DT, DT, self.S, self.N, 0.0)
+        tda.tda_topk(self.S, self.Nq, self.N, self.N, self.topk, self.idx, self.val)

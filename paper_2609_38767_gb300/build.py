@@ -56,6 +56,20 @@ def _compile(src: str, extra: list[str]) -> str:
     return obj
 
 
+def build_synth_cpu() -> str:
+    """gcc build of the CPU side of the input generator (OpenMP, no FP contraction)."""
+    src = os.path.join(CSRC, "synth_cpu.c")
+    target = lib_path("libtda_synth_cpu.so")
+    if _stale(target, [src]):
+        cmd = ["gcc", "-O2", "-std=c11", "-fPIC", "-shared", "-fopenmp", "-ffp-contract=off",
+               "-o", target + ".tmp", src, "-lm"]
+        r = subprocess.run(cmd, capture_output=True, text=True)
+        if r.returncode != 0:
+            raise RuntimeError(f"gcc failed for {src}:\n{r.stderr}")
+        os.replace(target + ".tmp", target)
+    return target
+
+
 def build(verbose: bool = False, extra: list[str] | None = None) -> dict[str, str]:
     """Build every library that is out of date; returns {name: path}."""
     os.makedirs(BUILD, exist_ok=True)
@@ -76,6 +90,7 @@ def build(verbose: bool = False, extra: list[str] | None = None) -> dict[str, st
                 if verbose:
                     print("built", target)
             out[name] = target
+    out["libtda_synth_cpu.so"] = build_synth_cpu()
     return out
 
 

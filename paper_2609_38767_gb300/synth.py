@@ -29,6 +29,8 @@ one rounding per operation):
 """
 from __future__ import annotations
 
+import os
+
 import numpy as np
 
 GAMMA = np.uint64(0x9E3779B97F4A7C15)
@@ -113,10 +115,49 @@ def mask_threshold(p: float) -> int:
     return min(int(float(p) * 18446744073709551616.0), (1 << 64) - 1)
 
 
+_cpu_lib = None
+
+
+def _load_cpu_lib():
+    """The C implementation of this generator (libtda_synth_cpu.so), or None if not built."""
+    global _cpu_lib
+    if _cpu_lib is None:
+        import ctypes
+
+        path = os.path.join(os.path.dirname(os.path.abspath(__file__)), "libtda_synth_cpu.so")
+        if not os.path.exists(path):
+            return None
+        lib = ctypes.CDLL(path)
+        u64, i64, i32 = ctypes.c_uint64, ctypes.c_int64, ctypes.c_int32
+        lib.tda_synth_fill_cpu.restype = i32
+        lib.tda_synth_fill_cpu.argtypes = [ctypes.c_void_p, i32, i32, u64, u64, i64, i64, i64, i64,
+                                           ctypes.c_float, u64, u64, u64]
+        _cpu_lib = lib
+    return _cpu_lib
+
+
 def factors(seed: int, stream: int, n: int, T: int, d: int, sigma: float = 1.0,
             dist: int = DIST_NORMAL, e0: int = 0, dtype: str = "bf16",
-            mask_p: float = 0.0, mask_seed: int = SEED_MASK, mask_stream: int = 0) -> np.ndarray:
-    """X[n][T][d] as float32, or as uint16 bf16 bit patterns when dtype == 'bf16'."""
+            mask_p: float = 0.0, mask_seed: int = SEED_MASK, mask_stream: int = 0,
+            impl: str = "auto") -> np.ndarray:
+    """X[n][T][d] as float32, or as uint16 bf16 bit patterns when dtype == 'bf16'.
+
+    impl 'numpy' evaluates the definition with numpy; 'c' (or 'auto' when the
+    library is built) uses the identical C implementation, which is faster."""
+    lib = _load_cpu_lib() if impl in ("auto", "c") else None
+    if impl == "c" and lib is None:
+        raise ImportError("libtda_synth_cpu.so is not built")
+    if lib is not None:
+        out = np.empty((n, T, d), dtype=np.uint16 if dtype == "bf16" else np.float32)
+        rc = lib.tda_synth_fill_cpu(out.ctypes.data, 1 if dtype == "bf16" else 0, dist, seed, stream, e0, n, T, d,
+                                    float(sigma), mask_seed, mask_stream, mask_threshold(mask_p))
+        if rc != 0:
+            raise ValueError("tda_synth_fill_cpu: bad argument")
+        return out
+    return _factors_numpy(seed, stream, n, T, d, sigma, dist, e0, dtype, mask_p, mask_seed, mask_stream)
+
+
+def _factors_numpy(seed, stream, n, T, d, sigma, dist, e0, dtype, mask_p, mask_seed, mask_stream):
     key = stream_key(seed, stream)
     e = np.arange(e0, e0 + n, dtype=np.uint64)[:, None, None]
     t = np.arange(T, dtype=np.uint64)[None, :, None]
@@ -126,11 +167,21 @@ def factors(seed: int, stream: int, n: int, T: int, d: int, sigma: float = 1.0,
     flat = v.reshape(-1)
     chunk = max(1, (1 << 16) // max(d, 1))  # token rows per chunk, cache-sized
     rows = (e * np.uint64(T) + t).reshape(-1)  # global token index of each (example, token) row
-    for r0 in range(0, rows.size, chunk):
+
+    def fill(r0):
         r = rows[r0:r0 + chunk, None]
         with np.errstate(over="ignore"):
             idx = r * np.uint64(d) + c.reshape(1, -1)
         flat[r0 * d:(r0 + r.shape[0]) * d] = (gen(key, idx) * np.float32(sigma)).astype(np.float32).reshape(-1)
+
+    starts = range(0, rows.size, chunk)
+    if rows.size * d >= (1 << 22):  # numpy releases the GIL: fill chunks on all cores
+        from concurrent.futures import ThreadPoolExecutor
+        with ThreadPoolExecutor(max_workers=os.cpu_count() or 1) as ex:
+            list(ex.map(fill, starts))
+    else:
+        for r0 in starts:
+            fill(r0)
     thr = mask_threshold(mask_p)
     if thr > 0:
         mkey = stream_key(mask_seed, mask_stream)

@@ -1,0 +1,185 @@
+"""Parity at the workloads' full sizes, on sampled outputs the oracle computes
+one by one, and through properties that hold at any size.
+
+* Llama-1B block (the benchmark's workload and launch configuration): 4096 train
+  and 64 query examples resident, the whole pass of BlockPipeline; sampled
+  feature rows and GradDot scores against the oracle, top-k selection bit-exact,
+  the preconditioner's solve checked by its residual.
+* Llama-3-8B layer shapes (k = 64, T = 1024): one streamed chunk of 256 train
+  examples through the 7 linears of a layer.
+* Large-model layer shapes (k = 128, T = 2048, Student-t activations), factors
+  streamed from pinned host memory through tda_project_host.
+* The 8192 x 8192 linear of the route sweep: exact similarity by both routes.
+Tolerances: relative Frobenius error 2e-2 for bf16 factors (spec bound).
+"""
+import math
+
+import numpy as np
+import pytest
+import torch
+
+import paper_2609_38767_gb300 as tda
+from paper_2609_38767_gb300 import build as tbuild
+from paper_2609_38767_gb300 import synth
+from paper_2609_38767_gb300.block import BlockPipeline
+
+pytestmark = pytest.mark.gpu
+TOL = 2e-2
+
+
+@pytest.fixture(scope="module")
+def dev():
+    assert torch.cuda.is_available(), "GPU tests need a CUDA device"
+    tbuild.build()
+    tda.load()
+    return torch.device("cuda:0")
+
+
+def rel_fro(x, ref):
+    x, ref = np.asarray(x, np.float64), np.asarray(ref, np.float64)
+    return float(np.linalg.norm(x - ref) / np.linalg.norm(ref))
+
+
+def fill(n, T, d, seed, stream, sigma, dist, mask_p, mask_stream, dev):
+    x = torch.empty(n * T * d, dtype=torch.bfloat16, device=dev)
+    synth.fill_device(x, seed, stream, n, T, d, sigma, dist, 0, mask_p, mask_stream=mask_stream)
+    return x
+
+
+def oracle_example(orc, e, role, li, T, di, do, k, sig_b, dist_a, mask_p, layer):
+    off, ms = (synth.QUERY_STREAM_OFFSET, 1000) if role == "query" else (0, 0)
+    A = synth.factors(synth.SEED_A, li + off, 1, T, di, 1.0, dist_a, e, "bf16", mask_p, mask_stream=ms)
+    B = synth.factors(synth.SEED_B, li + off, 1, T, do, sig_b, 0, e, "bf16", mask_p, mask_stream=ms)
+    return orc.project(synth.to_f64(A, "bf16"), synth.to_f64(B, "bf16"), k, k, 0, layer)[0].reshape(-1)
+
+
+def run_block(dev, linears, T, k, N, Nq, sig_b, dist_a, mask_p, topk):
+    At, Bt, Aq, Bq = [], [], [], []
+    for li, (di, do) in enumerate(linears):
+        At.append(fill(N, T, di, synth.SEED_A, li, 1.0, dist_a, mask_p, 0, dev))
+        Bt.append(fill(N, T, do, synth.SEED_B, li, sig_b, 0, mask_p, 0, dev))
+        Aq.append(fill(Nq, T, di, synth.SEED_A, li + synth.QUERY_STREAM_OFFSET, 1.0, dist_a, mask_p, 1000, dev))
+        Bq.append(fill(Nq, T, do, synth.SEED_B, li + synth.QUERY_STREAM_OFFSET, sig_b, 0, mask_p, 1000, dev))
+    pipe = BlockPipeline(linears, T, k, N, Nq, topk=topk, precondition=True, lambda_rel=1e-2, device=dev)
+    for li, L in enumerate(pipe.layers):
+        assert tda.tda_project_engine(L, tda.TDA_BF16, At[li], Bt[li]) == 1
+    pipe.run(lambda li, L, r, phi, ld: tda.tda_project(L, tda.TDA_BF16, At[li], Bt[li], N, phi, ld, r),
+             lambda li, L, r, phi, ld: tda.tda_project(L, tda.TDA_BF16, Aq[li], Bq[li], Nq, phi, ld, r))
+    S_plain = torch.empty((Nq, N), device=dev)  # GradDot (unpreconditioned) on the same features
+    tda.tda_score(pipe.Q, tda.TDA_F32, Nq, pipe.DT, pipe.Phi, N, pipe.DT, pipe.DT, S_plain, N)
+    info = tda.tda_precondition_info(pipe.nl, pipe.D, tda.TDA_F32, pipe.state)
+    tda.tda_device_status()
+    del At, Bt, Aq, Bq
+    return pipe, S_plain, info
+
+
+def check_block(orc, pipe, S_plain, info, linears, T, k, sig_b, dist_a, mask_p, train_s, query_s, rng):
+    D, N, Nq = k * k, pipe.N, pipe.Nq
+    phi = {e: pipe.Phi[e].cpu().numpy() for e in train_s}
+    qf = {e: pipe.Q[e].cpu().numpy() for e in query_s}
+    ophi = {e: np.concatenate([oracle_example(orc, e, "train", li, T, di, do, k, sig_b, dist_a, mask_p, li)
+                               for li, (di, do) in enumerate(linears)]) for e in train_s}
+    oq = {e: np.concatenate([oracle_example(orc, e, "query", li, T, di, do, k, sig_b, dist_a, mask_p, li)
+                             for li, (di, do) in enumerate(linears)]) for e in query_s}
+    for e in train_s:
+        assert rel_fro(phi[e], ophi[e]) <= TOL, ("train", e)
+        for li in range(len(linears)):
+            assert rel_fro(phi[e][li * D:(li + 1) * D], ophi[e][li * D:(li + 1) * D]) <= TOL
+    for e in query_s:
+        assert rel_fro(qf[e], oq[e]) <= TOL, ("query", e)
+    # GradDot scores of the sampled pairs, oracle features on both sides
+    Sp = S_plain.cpu().numpy()
+    got = np.array([[Sp[q, i] for i in train_s] for q in query_s])
+    ref = np.array([[float(oq[q] @ ophi[i]) for i in train_s] for q in query_s])
+    assert rel_fro(got, ref) <= TOL
+    # top-k: selection on the GPU's own score matrix is bit-exact
+    S = pipe.S.cpu().numpy()
+    oi, ov = orc.topk(S.astype(np.float64), pipe.topk)
+    np.testing.assert_array_equal(pipe.idx.cpu().numpy(), oi)
+    np.testing.assert_array_equal(pipe.val.cpu().numpy(), ov.astype(np.float32))
+    # the solve: (F + lambda I) qhat = q for every linear, F from the features it was fitted on
+    Phi64 = pipe.Phi.cpu().numpy().astype(np.float64)
+    Qh = pipe.Qh.cpu().numpy().astype(np.float64)
+    Q = pipe.Q.cpu().numpy().astype(np.float64)
+    for li in range(len(linears)):
+        P = Phi64[:, li * D:(li + 1) * D]
+        tr = float((P * P).sum()) / N
+        lam = 1e-2 * tr / D
+        assert abs(info[4 * li] - lam) <= 1e-4 * lam
+        X = Qh[:, li * D:(li + 1) * D]
+        R = (X @ P.T) @ P / N + lam * X - Q[:, li * D:(li + 1) * D]
+        assert np.linalg.norm(R) <= 1e-3 * np.linalg.norm(Q[:, li * D:(li + 1) * D]), li
+    return got, ref
+
+
+LLAMA1B = [(2048, 2048)] * 4 + [(2048, 8192)] * 2 + [(8192, 2048)]
+LLAMA8B = [(4096, 4096), (4096, 1024), (4096, 1024), (4096, 4096), (4096, 14336), (4096, 14336), (14336, 4096)]
+
+
+def test_llama1b_block_full_size(dev, orc):
+    # 4096 train / 64 query, T = 512, k = 32, B ~ N(0, 1e-3), 1% masked tokens
+    sb = math.sqrt(1e-3)
+    pipe, S_plain, info = run_block(dev, LLAMA1B, 512, 32, 4096, 64, sb, 0, 0.01, 100)
+    rng = np.random.default_rng(0)
+    train_s = [0, int(rng.integers(1, 4095)), 4095]
+    check_block(orc, pipe, S_plain, info, LLAMA1B, 512, 32, sb, 0, 0.01, train_s, [0, 63], rng)
+
+
+def test_llama8b_layer_chunk_full_shapes(dev, orc):
+    # one streamed chunk of 256 train examples, 16 queries, T = 1024, k = 64
+    pipe, S_plain, info = run_block(dev, LLAMA8B, 1024, 64, 256, 16, 0.1, 0, 0.0, 100)
+    check_block(orc, pipe, S_plain, info, LLAMA8B, 1024, 64, 0.1, 0, 0.0, [0, 255], [7], np.random.default_rng(1))
+
+
+@pytest.mark.parametrize("li,di,do", [(1, 12288, 1536), (4, 12288, 49152)])
+def test_large_model_layer_from_pinned_host(dev, orc, li, di, do):
+    # T = 2048, k = 128, A ~ Student-t(4), B ~ N(0, 1e-4); factors in pinned host memory
+    T, k, n, sb = 2048, 128, 2, 0.01
+    A = synth.factors(synth.SEED_A, li, n, T, di, 1.0, synth.DIST_STUDENT_T4, 0, "bf16")
+    B = synth.factors(synth.SEED_B, li, n, T, do, sb, 0, 0, "bf16")
+    Ah = torch.from_numpy(A.view(np.int16)).view(torch.bfloat16).pin_memory()
+    Bh = torch.from_numpy(B.view(np.int16)).view(torch.bfloat16).pin_memory()
+    L = tda.LayerDesc(di, do, T, k, k, seed=0, layer=li)
+    wsb = 2 * tda.tda_project_host_ws_min(L, tda.TDA_BF16)
+    ws = torch.empty(wsb, dtype=torch.uint8, device=dev)
+    phi = torch.empty((n, k * k), device=dev)
+    tda.tda_project_host(L, tda.TDA_BF16, Ah, Bh, n, phi, k * k, ws, wsb)
+    tda.tda_device_status()
+    ref = orc.project(synth.to_f64(A, "bf16"), synth.to_f64(B, "bf16"), k, k, 0, li)
+    got = phi.cpu().numpy().reshape(n, k, k)
+    for e in range(n):
+        assert rel_fro(got[e], ref[e]) <= TOL
+
+
+def test_topk_at_large_model_query_shape(dev, orc):
+    # 512 queries x 16384 train, top-100, descending with ties to the lower index
+    rng = np.random.default_rng(2)
+    S = (rng.standard_normal((512, 16384)) * 32).round().astype(np.float32)  # many exact ties
+    Sd = torch.from_numpy(S).to(dev)
+    idx = torch.empty((512, 100), dtype=torch.int32, device=dev)
+    val = torch.empty((512, 100), device=dev)
+    tda.tda_topk(Sd, 512, 16384, 16384, 100, idx, val)
+    oi, ov = orc.topk(S.astype(np.float64), 100)
+    np.testing.assert_array_equal(idx.cpu().numpy(), oi)
+    np.testing.assert_array_equal(val.cpu().numpy(), ov.astype(np.float32))
+
+
+@pytest.mark.parametrize("T", [8, 32])
+def test_route_sweep_linear_exact_similarity(dev, orc, T):
+    # 8192 x 8192 linear, A, B ~ N(0, 1): Gram route and materialise route vs the oracle
+    d, nq, nt = 8192, 2, 2
+    Aq = synth.factors(synth.SEED_A, 1000, nq, T, d, 1.0, dtype="bf16")
+    Bq = synth.factors(synth.SEED_B, 1000, nq, T, d, 1.0, dtype="bf16")
+    At = synth.factors(synth.SEED_A, 0, nt, T, d, 1.0, dtype="bf16")
+    Bt = synth.factors(synth.SEED_B, 0, nt, T, d, 1.0, dtype="bf16")
+    to = lambda x: torch.from_numpy(x.view(np.int16)).view(torch.bfloat16).to(dev)
+    L = tda.LayerDesc(d, d, T, 1, 1)
+    ref = orc.similarity(synth.to_f64(Aq, "bf16"), synth.to_f64(Bq, "bf16"), synth.to_f64(At, "bf16"),
+                         synth.to_f64(Bt, "bf16"))
+    for route in (tda.TDA_ROUTE_GRAM, tda.TDA_ROUTE_MATERIALIZE):
+        wsb = max(tda.tda_workspace_size(tda.TDA_OP_SIMILARITY_EXACT, L, tda.TDA_BF16, nq, nt, route), 1)
+        ws = torch.empty(wsb, dtype=torch.uint8, device=dev)
+        S = torch.empty((nq, nt), device=dev)
+        tda.tda_similarity_exact(L, tda.TDA_BF16, to(Aq), to(Bq), nq, to(At), to(Bt), nt, S, nt, 0.0, route, ws, wsb)
+        tda.tda_device_status()
+        assert rel_fro(S.cpu().numpy(), ref) <= TOL, route

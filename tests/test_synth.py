@@ -55,3 +55,13 @@ def test_sigma_scales_in_fp32():
     a = synth.factors(1, 0, 2, 3, 8, sigma=1.0, dtype="f32")
     b = synth.factors(1, 0, 2, 3, 8, sigma=0.1, dtype="f32")
     np.testing.assert_array_equal(b, (a * np.float32(0.1)).astype(np.float32))
+
+
+def test_c_generator_matches_numpy_definition():
+    from paper_2609_38767_gb300 import build
+
+    build.build_synth_cpu()
+    for dtype, dist, mask in [("f32", 0, 0.0), ("bf16", 0, 0.01), ("bf16", 1, 0.0), ("f32", 1, 0.05)]:
+        a = synth.factors(5, 7, 3, 37, 48, 0.37, dist, 11, dtype, mask, impl="numpy")
+        b = synth.factors(5, 7, 3, 37, 48, 0.37, dist, 11, dtype, mask, impl="c")
+        np.testing.assert_array_equal(a, b)
