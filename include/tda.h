@@ -290,6 +290,13 @@ tda_status tda_route_calibrate(void* ws, size_t ws_bytes, void* stream, double* 
 /* 0 = flop model (the paper's), 1 = calibrated time model. */
 tda_status tda_route_set_model(int32_t model);
 
+/* Self-test of the failure path: launches one thread that waits on an
+ * mbarrier nothing arrives on, bounded by timeout_ns (at most 2 s) of
+ * %globaltimer, exactly like the tensor-core kernels' waits. The wait runs
+ * out, the kernel records the timeout and returns; the next
+ * tda_device_status() reports TDA_ERR_TIMEOUT and the context stays usable. */
+tda_status tda_selftest_bounded_wait(uint64_t timeout_ns, void* stream);
+
 /* Synchronises `stream`, then reads and clears the device error word.
  * Returns TDA_ERR_TIMEOUT if a kernel's bounded wait expired since the last
  * check, TDA_ERR_CUDA on a CUDA error, else TDA_OK. */

@@ -19,7 +19,7 @@ __all__ = [
     "tda_project_materialized_noalloc",
     "tda_similarity_exact", "tda_precondition_state_bytes", "tda_precondition",
     "tda_precondition_info", "tda_score", "tda_topk", "tda_route", "tda_route_calibrate",
-    "tda_route_set_model", "tda_device_status", "tda_last_error", "tda_version", "tda_launch_count",
+    "tda_route_set_model", "tda_device_status", "tda_selftest_bounded_wait", "tda_last_error", "tda_version", "tda_launch_count",
 ]
 
 _HERE = os.path.dirname(os.path.abspath(__file__))
@@ -91,6 +91,7 @@ def load() -> ctypes.CDLL:
             "tda_route_calibrate": (I32, [P, SZ, P, ctypes.POINTER(D)]),
             "tda_route_set_model": (I32, [I32]),
             "tda_device_status": (I32, [P]),
+            "tda_selftest_bounded_wait": (I32, [U64, P]),
             "tda_last_error": (ctypes.c_char_p, []),
             "tda_version": (I32, []),
             "tda_launch_count": (U64, []),
@@ -222,6 +223,10 @@ def tda_route_calibrate(ws, ws_bytes, stream=None) -> list[float]:
 
 def tda_route_set_model(model: int) -> None:
     _check(load().tda_route_set_model(model))
+
+
+def tda_selftest_bounded_wait(timeout_ns, stream=None) -> None:
+    _check(load().tda_selftest_bounded_wait(timeout_ns, _stream(stream)))
 
 
 def tda_device_status(stream=None) -> None:

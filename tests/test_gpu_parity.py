@@ -347,3 +347,19 @@ def test_precondition_batched_layers_match_oracle(dev, orc, sdt, D, lam_abs, lam
         assert abs(info[4 * l] - lam) <= 1e-5 * lam and info[4 * l + 2] == 0
         ref = orc.precondition(F, lam, q[:, l * D:(l + 1) * D].astype(np.float64))
         assert rel_fro(got[:, l * D:(l + 1) * D], ref) <= tol
+
+
+def test_bounded_wait_times_out_and_context_survives(dev, orc):
+    # a wait on a barrier nothing arrives on runs out after 50 ms; the error word reports it
+    tda.tda_device_status()
+    tda.tda_selftest_bounded_wait(50_000_000)
+    with pytest.raises(tda.TdaError) as e:
+        tda.tda_device_status()
+    assert e.value.status == tda.TDA_ERR_TIMEOUT
+    tda.tda_device_status()  # the word was cleared
+    # the context is still usable: a projection afterwards matches the oracle
+    A, B = make_factors(3, 40, 64, 64, "bf16", stream=12)
+    L = tda.LayerDesc(64, 64, 40, 16, 16, seed=1, layer=1)
+    got, _ = gpu_project(L, "bf16", to_dev(A, "bf16", dev), to_dev(B, "bf16", dev), 3, tda.TDA_ROUTE_FACTORED, dev)
+    ref = orc.project(synth.to_f64(A, "bf16"), synth.to_f64(B, "bf16"), 16, 16, 1, 1)
+    assert rel_fro(got, ref) <= TOL["bf16"]
