@@ -55,7 +55,7 @@ St<TS> state_of(void* state, int64_t D) {
 // and columns {tx*4+v, 64+tx*4+v}: 8 x 8 accumulators, float4 shared reads.
 constexpr int kFT = 128, kFK = 16;
 
-__global__ void __launch_bounds__(256)
+__global__ void __launch_bounds__(256, 2)
 fit_f32_kernel(St<float> st, const float* __restrict__ phi, int64_t n, int64_t ld) {
     if (blockIdx.x > blockIdx.y) return;  // upper tile: M is used through its lower triangle
     __shared__ __align__(16) float Xa[kFK][kFT];
@@ -229,20 +229,28 @@ __global__ void __launch_bounds__(256) panel_kernel(St<TS> st, int64_t k0) {
     }
     __syncthreads();
     if (tid < 32) {
+        // Lane i holds row i of the block in registers; step j broadcasts the
+        // pivot and the scaled column j with warp shuffles (right-looking).
+        TS r[kNB];
+#pragma unroll
+        for (int c = 0; c < kNB; ++c) r[c] = Lk[lane][c];
         int bad = -1;
+#pragma unroll
         for (int j = 0; j < kNB; ++j) {
-            const TS p = Lk[j][j];
+            const TS p = __shfl_sync(0xffffffffu, r[j], j);
             const bool ok = p > (TS)0;
             if (!ok && bad < 0) bad = j;
             const TS piv = ok ? (TS)sqrt((double)p) : (TS)NAN;
-            __syncwarp();
-            if (lane == j) Lk[j][j] = piv;
-            if (lane > j) Lk[lane][j] /= piv;
-            __syncwarp();
-            if (lane > j)
-                for (int c = j + 1; c <= lane; ++c) Lk[lane][c] -= Lk[lane][j] * Lk[c][j];
-            __syncwarp();
+            if (lane == j) r[j] = piv;
+            if (lane > j) r[j] /= piv;
+#pragma unroll
+            for (int c = j + 1; c < kNB; ++c) {
+                const TS v = __shfl_sync(0xffffffffu, r[j], c);  // L[c][j]
+                if (lane >= c) r[c] -= r[j] * v;
+            }
         }
+#pragma unroll
+        for (int c = 0; c < kNB; ++c) Lk[lane][c] = (c <= lane) ? r[c] : (TS)0;
         if (blockIdx.y == 0 && lane == 0 && bad >= 0 && bad < nb) {
             double* h = st.header(l);
             if (h[kPcFailedPivot] == 0.0) h[kPcFailedPivot] = (double)(k0 + bad + 1);
