@@ -377,6 +377,7 @@ apply_kernel(St<TS> st, const float* __restrict__ q, int64_t n_q, int64_t ld_q, 
 #pragma unroll
             for (int g = 0; g < G; ++g) acc[g] = (TS)0;
             if (ii < nb)
+#pragma unroll 8
                 for (int64_t m = lane; m < b0; m += 32) {
                     const TS lv = L[(b0 + ii) * D + m];
 #pragma unroll
@@ -409,6 +410,7 @@ apply_kernel(St<TS> st, const float* __restrict__ q, int64_t n_q, int64_t ld_q, 
 #pragma unroll
         for (int g = 0; g < G; ++g) acc[g] = (TS)0;
         if (lane < nb)
+#pragma unroll 8
             for (int64_t m = e0 + warp; m < D; m += 8) {
                 const TS lv = L[m * D + b0 + lane];
 #pragma unroll
