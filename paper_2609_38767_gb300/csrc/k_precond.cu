@@ -240,7 +240,7 @@ __global__ void __launch_bounds__(256) panel_kernel(St<TS> st, int64_t k0) {
             const TS p = __shfl_sync(0xffffffffu, r[j], j);
             const bool ok = p > (TS)0;
             if (!ok && bad < 0) bad = j;
-            const TS piv = ok ? (TS)sqrt((double)p) : (TS)NAN;
+            const TS piv = ok ? sqrt(p) : (TS)NAN;  // sqrtf for a float state
             if (lane == j) r[j] = piv;
             if (lane > j) r[j] /= piv;
 #pragma unroll
