@@ -107,7 +107,8 @@ tda_status tda_proj_entries(uint64_t seed, uint32_t layer, int32_t side, int32_t
 
 /* ---------------------------------------------------------------------------
  * tda_workspace_size -- bytes of scratch `ws` that the matching call needs
- * (op PROJECT -> tda_project; op SIMILARITY_EXACT -> tda_similarity_exact).
+ * (op PROJECT -> tda_project; SIMILARITY_PROJECTED -> tda_similarity_projected;
+ * SIMILARITY_EXACT -> tda_similarity_exact), for one train example per chunk.
  * n1 = examples (or queries), n2 = train examples (similarity only).
  * route AUTO resolves through tda_route() first. Host only; no device work.
  * ------------------------------------------------------------------------- */
@@ -194,6 +195,26 @@ tda_status tda_similarity_exact(const tda_layer_desc* L, tda_dtype dtype,
                                 const void* At, const void* Bt, int64_t n_t,
                                 float* S, int64_t ld_S, float beta, tda_route_id route,
                                 void* ws, size_t ws_bytes, void* stream);
+
+/* ---------------------------------------------------------------------------
+ * tda_similarity_projected -- inner products of PROJECTED gradients,
+ *   S[q][i] = beta*S[q][i] + <Phi_q, Phi_i>,  Phi = P_g DW P_a^T (Eq. 2),
+ * by any of the three routes that give this result (App. A.4: routing per
+ * operation; exact arithmetic gives the same S):
+ *   FACTORED    project both sides' factors (Eq. 2), then dot the features;
+ *   MATERIALIZE form DW (Eq. 1), project it, then dot the features;
+ *   GRAM        project the factors per token (a~_t = P_a a_t, g~_t = P_g g_t)
+ *               and apply Eq. 4 to them, never forming Phi;
+ *   AUTO        tda_route(TDA_OP_SIMILARITY_PROJECTED).
+ * Arguments as tda_similarity_exact. ws: >= tda_workspace_size(
+ * TDA_OP_SIMILARITY_PROJECTED, L, dtype, n_q, n_t, route) bytes, 256-byte
+ * aligned; more ws lets train examples go through in larger chunks.
+ * ------------------------------------------------------------------------- */
+tda_status tda_similarity_projected(const tda_layer_desc* L, tda_dtype dtype,
+                                    const void* Aq, const void* Bq, int64_t n_q,
+                                    const void* At, const void* Bt, int64_t n_t,
+                                    float* S, int64_t ld_S, float beta, tda_route_id route,
+                                    void* ws, size_t ws_bytes, void* stream);
 
 /* ---------------------------------------------------------------------------
  * tda_precondition -- damped Fisher inverse on the query side (App. B.3: a

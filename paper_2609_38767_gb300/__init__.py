@@ -17,7 +17,7 @@ __all__ = [
     "LayerDesc", "TdaError", "load", "tda_proj_entries", "tda_workspace_size", "tda_project",
     "tda_project_engine", "tda_project_host_ws_min", "tda_project_host", "tda_noalloc_scratch_bytes",
     "tda_project_materialized_noalloc",
-    "tda_similarity_exact", "tda_precondition_state_bytes", "tda_precondition",
+    "tda_similarity_projected", "tda_similarity_exact", "tda_precondition_state_bytes", "tda_precondition",
     "tda_precondition_info", "tda_score", "tda_topk", "tda_route", "tda_route_calibrate",
     "tda_route_set_model", "tda_device_status", "tda_selftest_bounded_wait", "tda_last_error", "tda_version", "tda_launch_count",
 ]
@@ -81,6 +81,7 @@ def load() -> ctypes.CDLL:
             "tda_project_host": (I32, [LP, I32, P, P, I64, P, I64, P, SZ, P]),
             "tda_noalloc_scratch_bytes": (SZ, []),
             "tda_project_materialized_noalloc": (I32, [LP, I32, P, P, I64, P, I64, P]),
+            "tda_similarity_projected": (I32, [LP, I32, P, P, I64, P, P, I64, P, I64, F, I32, P, SZ, P]),
             "tda_similarity_exact": (I32, [LP, I32, P, P, I64, P, P, I64, P, I64, F, I32, P, SZ, P]),
             "tda_precondition_state_bytes": (SZ, [I64, I32]),
             "tda_precondition": (I32, [I32, I32, I64, I32, P, P, I64, I64, I64, D, D, P, I64, I64, P, I64, P]),
@@ -174,6 +175,12 @@ def tda_noalloc_scratch_bytes() -> int:
 def tda_project_materialized_noalloc(L, dtype, A, B, N, phi, ld_phi, stream=None):
     _check(load().tda_project_materialized_noalloc(ctypes.byref(L), dtype, _ptr(A), _ptr(B), N, _ptr(phi),
                                                    ld_phi, _stream(stream)))
+
+
+def tda_similarity_projected(L, dtype, Aq, Bq, n_q, At, Bt, n_t, S, ld_S, beta=0.0, route=TDA_ROUTE_AUTO,
+                             ws=None, ws_bytes=0, stream=None):
+    _check(load().tda_similarity_projected(ctypes.byref(L), dtype, _ptr(Aq), _ptr(Bq), n_q, _ptr(At), _ptr(Bt),
+                                           n_t, _ptr(S), ld_S, beta, route, _ptr(ws), ws_bytes, _stream(stream)))
 
 
 def tda_similarity_exact(L, dtype, Aq, Bq, n_q, At, Bt, n_t, S, ld_S, beta=0.0, route=TDA_ROUTE_AUTO,

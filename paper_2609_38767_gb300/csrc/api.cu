@@ -209,6 +209,8 @@ tda_status tda_route_set_model(int32_t model) {
     return TDA_OK;
 }
 
+static size_t simproj_ws(const tda_layer_desc& L, int64_t n_q, int64_t chunk, tda_route_id route);
+
 tda_status tda_workspace_size(tda_op op, const tda_layer_desc* L, tda_dtype dtype, int64_t n1,
                               int64_t n2, tda_route_id route, size_t* bytes) {
     g_msg[0] = 0;
@@ -226,6 +228,10 @@ tda_status tda_workspace_size(tda_op op, const tda_layer_desc* L, tda_dtype dtyp
     }
     if (op == TDA_OP_SIMILARITY_EXACT) {
         if (route == TDA_ROUTE_MATERIALIZE) *bytes = similarity_materialize_ws_bytes(*L, n1, 1);
+        return TDA_OK;
+    }
+    if (op == TDA_OP_SIMILARITY_PROJECTED) {
+        *bytes = simproj_ws(*L, n1, 1, route);
         return TDA_OK;
     }
     return fail(TDA_ERR_UNSUPPORTED, "no workspace query for op %d", (int)op);
@@ -312,6 +318,80 @@ tda_status tda_similarity_exact(const tda_layer_desc* L, tda_dtype dtype, const 
                           "similarity (materialise)");
     }
     return fail(TDA_ERR_UNSUPPORTED, "route %d cannot produce exact similarities", (int)route);
+}
+
+// Workspace of tda_similarity_projected for a train chunk of `chunk` examples.
+static size_t simproj_ws(const tda_layer_desc& L, int64_t n_q, int64_t chunk, tda_route_id route) {
+    const size_t D = (size_t)L.k_in * (size_t)L.k_out;
+    if (route == TDA_ROUTE_GRAM) return project_factors_bytes_per_example(L) * (size_t)(n_q + chunk);
+    size_t b = sizeof(float) * D * (size_t)(n_q + chunk);
+    if (route == TDA_ROUTE_MATERIALIZE) b += materialize_ws_bytes_per_example(L);
+    return b;
+}
+
+tda_status tda_similarity_projected(const tda_layer_desc* L, tda_dtype dtype, const void* Aq, const void* Bq,
+                                    int64_t n_q, const void* At, const void* Bt, int64_t n_t, float* S,
+                                    int64_t ld_S, float beta, tda_route_id route, void* ws, size_t ws_bytes,
+                                    void* stream) {
+    g_msg[0] = 0;
+    tda_status st = validate_layer(L, true);
+    if (st) return st;
+    if ((st = validate_factors(L, dtype, Aq, Bq, n_q, "tda_similarity_projected (queries)"))) return st;
+    if ((st = validate_factors(L, dtype, At, Bt, n_t, "tda_similarity_projected (train)"))) return st;
+    if (n_q > 65535) return fail(TDA_ERR_INVALID_ARG, "n_q must be <= 65535");
+    if (n_q > 0 && n_t > 0 && !S) return fail(TDA_ERR_INVALID_ARG, "S is NULL");
+    if (ld_S < n_t) return fail(TDA_ERR_INVALID_ARG, "ld_S < n_t");
+    if (route == TDA_ROUTE_AUTO) {
+        tda_route_id r;
+        if ((st = tda_route(L, TDA_OP_SIMILARITY_PROJECTED, n_q, n_t, dtype, &r, nullptr))) return st;
+        route = r;
+    }
+    if (route != TDA_ROUTE_FACTORED && route != TDA_ROUTE_MATERIALIZE && route != TDA_ROUTE_GRAM)
+        return fail(TDA_ERR_INVALID_ARG, "bad route %d", (int)route);
+    cudaStream_t s = (cudaStream_t)stream;
+    if (n_q == 0 || n_t == 0) return TDA_OK;
+    const size_t need = simproj_ws(*L, n_q, 1, route);
+    if (!ws || ws_bytes < need)
+        return fail(TDA_ERR_WORKSPACE, "tda_similarity_projected needs >= %zu bytes of ws, got %zu", need, ws_bytes);
+    if ((uintptr_t)ws & 255) return fail(TDA_ERR_INVALID_ARG, "ws must be 256-byte aligned");
+    const int64_t D = (int64_t)L->k_in * L->k_out;
+    const size_t el = dtype == TDA_F32 ? 4 : 2;
+    const size_t a_ex = (size_t)L->T * L->d_in * el, b_ex = (size_t)L->T * L->d_out * el;
+    if (route == TDA_ROUTE_GRAM) {
+        const size_t per = project_factors_bytes_per_example(*L);
+        float* Yq = (float*)ws;
+        float* Yt = (float*)((char*)ws + per * (size_t)n_q);
+        int64_t chunk = (int64_t)((ws_bytes - per * (size_t)n_q) / per);
+        if (chunk > n_t) chunk = n_t;
+        if (chunk > 65535) chunk = 65535;
+        if ((st = cuda_check(launch_project_factors(*L, dtype, Aq, Bq, 0, n_q, Yq, s), "project factors (queries)")))
+            return st;
+        for (int64_t i0 = 0; i0 < n_t; i0 += chunk) {
+            const int64_t c = (n_t - i0) < chunk ? (n_t - i0) : chunk;
+            if ((st = cuda_check(launch_project_factors(*L, dtype, At, Bt, i0, c, Yt, s), "project factors (train)")))
+                return st;
+            if ((st = cuda_check(launch_gram_projected(*L, Yq, n_q, Yt, c, S + i0, ld_S, beta, s), "gram (projected)")))
+                return st;
+        }
+        return TDA_OK;
+    }
+    // routes a and b: features of the queries, then of train chunks, then scores
+    const size_t mat = route == TDA_ROUTE_MATERIALIZE ? materialize_ws_bytes_per_example(*L) : 0;
+    float* Fq = (float*)ws;
+    float* Ft = Fq + (size_t)n_q * D;
+    int64_t chunk = (int64_t)((ws_bytes - mat - sizeof(float) * (size_t)D * (size_t)n_q) / (sizeof(float) * (size_t)D));
+    if (chunk > n_t) chunk = n_t;
+    void* mws = route == TDA_ROUTE_MATERIALIZE ? (void*)(Ft + (size_t)chunk * D) : nullptr;
+    if ((st = tda_project(L, dtype, Aq, Bq, n_q, Fq, D, route, mws, mat, stream))) return st;
+    for (int64_t i0 = 0; i0 < n_t; i0 += chunk) {
+        const int64_t c = (n_t - i0) < chunk ? (n_t - i0) : chunk;
+        if ((st = tda_project(L, dtype, (const char*)At + (size_t)i0 * a_ex, (const char*)Bt + (size_t)i0 * b_ex, c, Ft,
+                              D, route, mws, mat, stream)))
+            return st;
+        if ((st = cuda_check(launch_score(Fq, TDA_F32, n_q, D, Ft, c, D, D, S + i0, ld_S, beta, s), "score")))
+            return st;
+    }
+    return TDA_OK;
 }
 
 size_t tda_precondition_state_bytes(int64_t D, tda_dtype state_dtype) {

@@ -170,7 +170,7 @@ template <typename T>
 __global__ void __launch_bounds__(kTh)
 gram_kernel(const T* __restrict__ Aq, const T* __restrict__ Bq, const T* __restrict__ At,
             const T* __restrict__ Bt, int64_t Tn, int64_t d_in, int64_t d_out,
-            float* __restrict__ S, int64_t ld_S, float beta) {
+            float* __restrict__ S, int64_t ld_S, float beta, float alpha) {
     constexpr int TT = 16, KC = 64;
     __shared__ float Xq[TT][KC + 1];
     __shared__ float Xi[TT][KC + 1];
@@ -211,7 +211,54 @@ gram_kernel(const T* __restrict__ Aq, const T* __restrict__ Bq, const T* __restr
     }
     if (tid == 0) {
         float* dst = S + q * ld_S + i;
-        *dst = (beta == 0.f) ? red[0] : beta * (*dst) + red[0];
+        *dst = (beta == 0.f) ? alpha * red[0] : beta * (*dst) + alpha * red[0];
+    }
+}
+
+// Projected factors of examples [e0, e0+n): At[e][t][j] = sum_c A[t][c] S_in[c][j],
+// Bt[e][t][i] = sum_r B[t][r] S_out[r][i] (fp32, unscaled signs). One CTA per
+// (example, 64-token chunk); thread (t = tid/4, 16 columns at (tid%4)*16).
+template <typename T>
+__global__ void __launch_bounds__(kTh)
+project_factors_kernel(const T* __restrict__ X, int64_t e0, int64_t Tn, int64_t d, int k, uint64_t key,
+                       int kind, float* __restrict__ Y) {
+    __shared__ float Xs[64][kT + 1];  // 64 tokens x 64 features
+    __shared__ uint64_t Ws[256];
+    const int64_t e = e0 + blockIdx.y;
+    const int64_t t0 = (int64_t)blockIdx.x * 64;
+    const T* Xe = X + e * Tn * d;
+    float* Ye = Y + (int64_t)blockIdx.y * Tn * k;
+    const int tid = threadIdx.x, tl = tid >> 2, cq = (tid & 3) * 16;
+    for (int j0 = 0; j0 < k; j0 += 64) {
+        float acc[16];
+#pragma unroll
+        for (int q = 0; q < 16; ++q) acc[q] = 0.f;
+        for (int64_t c0 = 0; c0 < d; c0 += kT) {
+            __syncthreads();
+            for (int x = tid; x < 64 * kT; x += kTh) {
+                const int tt = x / kT, cc = x % kT;
+                Xs[tt][cc] = (t0 + tt < Tn && c0 + cc < d) ? ld1(Xe + (t0 + tt) * d + c0 + cc) : 0.f;
+            }
+            if (tid < 64) Ws[tid] = sign_word(key, (uint32_t)(j0 + tid), (uint64_t)(c0 >> 6));
+            __syncthreads();
+            if (kind == TDA_PROJ_RADEMACHER) {
+                for (int cc = 0; cc < kT; ++cc) {
+                    const float v = Xs[tl][cc];
+#pragma unroll
+                    for (int q = 0; q < 16; ++q) acc[q] += signed_term(Ws[cq + q], cc, v);
+                }
+            } else {
+#pragma unroll
+                for (int q = 0; q < 16; ++q) {
+                    const int64_t j = j0 + cq + q;
+                    if (j >= c0 && j < c0 + kT) acc[q] += Xs[tl][j - c0];
+                }
+            }
+        }
+        if (t0 + tl < Tn)
+#pragma unroll
+            for (int q = 0; q < 16; ++q)
+                if (j0 + cq + q < k) Ye[(t0 + tl) * k + j0 + cq + q] = acc[q];
     }
 }
 
@@ -302,10 +349,48 @@ cudaError_t launch_similarity_gram(const tda_layer_desc& L, tda_dtype dt, const 
     if (dt == TDA_BF16)
         gram_kernel<__nv_bfloat16><<<grid, kTh, 0, s>>>(
             (const __nv_bfloat16*)Aq, (const __nv_bfloat16*)Bq, (const __nv_bfloat16*)At,
-            (const __nv_bfloat16*)Bt, L.T, L.d_in, L.d_out, S, ld_S, beta);
+            (const __nv_bfloat16*)Bt, L.T, L.d_in, L.d_out, S, ld_S, beta, 1.f);
     else
         gram_kernel<float><<<grid, kTh, 0, s>>>((const float*)Aq, (const float*)Bq, (const float*)At,
-                                                (const float*)Bt, L.T, L.d_in, L.d_out, S, ld_S, beta);
+                                                (const float*)Bt, L.T, L.d_in, L.d_out, S, ld_S, beta, 1.f);
+    return cudaGetLastError();
+}
+
+size_t project_factors_bytes_per_example(const tda_layer_desc& L) {
+    return sizeof(float) * (size_t)(L.T * ((int64_t)L.k_in + L.k_out));
+}
+
+// Projected factors of n examples into Y: At block (n x T x k_in) then Bt block.
+cudaError_t launch_project_factors(const tda_layer_desc& L, tda_dtype dt, const void* A, const void* B, int64_t e0,
+                                   int64_t n, float* Y, cudaStream_t s) {
+    if (n == 0 || L.T == 0) return cudaSuccess;
+    const uint64_t key_in = side_key(L.seed, L.layer, 0), key_out = side_key(L.seed, L.layer, 1);
+    float* Ya = Y;
+    float* Yb = Y + n * L.T * L.k_in;
+    dim3 grid((unsigned)((L.T + 63) / 64), (unsigned)n);
+    note_launches(2);
+    if (dt == TDA_BF16) {
+        project_factors_kernel<__nv_bfloat16><<<grid, kTh, 0, s>>>((const __nv_bfloat16*)A, e0, L.T, L.d_in, L.k_in,
+                                                                   key_in, L.kind, Ya);
+        project_factors_kernel<__nv_bfloat16><<<grid, kTh, 0, s>>>((const __nv_bfloat16*)B, e0, L.T, L.d_out,
+                                                                   L.k_out, key_out, L.kind, Yb);
+    } else {
+        project_factors_kernel<float><<<grid, kTh, 0, s>>>((const float*)A, e0, L.T, L.d_in, L.k_in, key_in, L.kind, Ya);
+        project_factors_kernel<float><<<grid, kTh, 0, s>>>((const float*)B, e0, L.T, L.d_out, L.k_out, key_out, L.kind,
+                                                           Yb);
+    }
+    return cudaGetLastError();
+}
+
+// Eq. 4 on projected factors: S = beta*S + scale^2 * sum_{t,s} <a~,a~><g~,g~>.
+cudaError_t launch_gram_projected(const tda_layer_desc& L, const float* Yq, int64_t n_q, const float* Yt,
+                                  int64_t n_t, float* S, int64_t ld_S, float beta, cudaStream_t s) {
+    if (n_q == 0 || n_t == 0) return cudaSuccess;
+    const float sc = projection_scale(L);
+    dim3 grid((unsigned)n_t, (unsigned)n_q);
+    note_launches(1);
+    gram_kernel<float><<<grid, kTh, 0, s>>>(Yq, Yq + n_q * L.T * L.k_in, Yt, Yt + n_t * L.T * L.k_in, L.T, L.k_in,
+                                            L.k_out, S, ld_S, beta, sc * sc);
     return cudaGetLastError();
 }
 

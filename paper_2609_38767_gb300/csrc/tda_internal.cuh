@@ -91,6 +91,14 @@ cudaError_t launch_similarity_gram(const tda_layer_desc& L, tda_dtype dt, const 
                                    const void* Bq, int64_t n_q, const void* At, const void* Bt,
                                    int64_t n_t, float* S, int64_t ld_S, float beta, cudaStream_t s);
 
+// Projected factors (a~ = S_in^T a, g~ = S_out^T g per token, unscaled) and the
+// Gram identity on them (projected-similarity route c).
+size_t project_factors_bytes_per_example(const tda_layer_desc& L);
+cudaError_t launch_project_factors(const tda_layer_desc& L, tda_dtype dt, const void* A, const void* B, int64_t e0,
+                                   int64_t n, float* Y, cudaStream_t s);
+cudaError_t launch_gram_projected(const tda_layer_desc& L, const float* Yq, int64_t n_q, const float* Yt,
+                                  int64_t n_t, float* S, int64_t ld_S, float beta, cudaStream_t s);
+
 // Preconditioner, n_layers layers of D features each (layer l's columns at
 // offset l*D of every feature row).
 int64_t precondition_apply_max_d(tda_dtype sdt);

@@ -116,3 +116,10 @@ def test_workspace_sizes(libs):
     assert tda.tda_workspace_size(tda.TDA_OP_SIMILARITY_EXACT, L, tda.TDA_F32, 3, 9,
                                   tda.TDA_ROUTE_MATERIALIZE) == 4 * 4 * 128 * 256
     assert tda.tda_workspace_size(tda.TDA_OP_SIMILARITY_EXACT, L, tda.TDA_F32, 3, 9, tda.TDA_ROUTE_GRAM) == 0
+    D = 16 * 16
+    assert tda.tda_workspace_size(tda.TDA_OP_SIMILARITY_PROJECTED, L, tda.TDA_F32, 3, 9,
+                                  tda.TDA_ROUTE_FACTORED) == 4 * D * 4
+    assert tda.tda_workspace_size(tda.TDA_OP_SIMILARITY_PROJECTED, L, tda.TDA_F32, 3, 9,
+                                  tda.TDA_ROUTE_MATERIALIZE) == 4 * D * 4 + 4 * (128 * 256 + 128 * 16)
+    assert tda.tda_workspace_size(tda.TDA_OP_SIMILARITY_PROJECTED, L, tda.TDA_F32, 3, 9,
+                                  tda.TDA_ROUTE_GRAM) == 4 * 32 * (16 + 16) * 4

@@ -363,3 +363,26 @@ def test_bounded_wait_times_out_and_context_survives(dev, orc):
     got, _ = gpu_project(L, "bf16", to_dev(A, "bf16", dev), to_dev(B, "bf16", dev), 3, tda.TDA_ROUTE_FACTORED, dev)
     ref = orc.project(synth.to_f64(A, "bf16"), synth.to_f64(B, "bf16"), 16, 16, 1, 1)
     assert rel_fro(got, ref) <= TOL["bf16"]
+
+
+@pytest.mark.parametrize("dtype", ["f32", "bf16"])
+@pytest.mark.parametrize("route", [tda.TDA_ROUTE_FACTORED, tda.TDA_ROUTE_MATERIALIZE, tda.TDA_ROUTE_GRAM,
+                                   tda.TDA_ROUTE_AUTO])
+def test_similarity_projected_routes_match_oracle(dev, orc, dtype, route):
+    # projected-gradient inner products by the three routes (App. A.4), train side
+    # streamed through a workspace that holds only a few examples at a time
+    nq, nt, T, di, do, k = 3, 11, 37, 64, 48, 16
+    Aq, Bq = make_factors(nq, T, di, do, dtype, stream=13, query=True)
+    At, Bt = make_factors(nt, T, di, do, dtype, stream=13)
+    L = tda.LayerDesc(di, do, T, k, k, seed=4, layer=2)
+    base = tda.tda_workspace_size(tda.TDA_OP_SIMILARITY_PROJECTED, L, TD[dtype], nq, nt, route)
+    wsb = base + 3 * (4 * k * k + 4 * T * 2 * k)  # room for a few more train examples per chunk
+    ws = torch.empty(wsb, dtype=torch.uint8, device=dev)
+    S = torch.full((nq, nt), 1.5, device=dev)
+    tda.tda_similarity_projected(L, TD[dtype], to_dev(Aq, dtype, dev), to_dev(Bq, dtype, dev), nq,
+                                 to_dev(At, dtype, dev), to_dev(Bt, dtype, dev), nt, S, nt, 2.0, route, ws, wsb)
+    tda.tda_device_status()
+    fq = orc.project(synth.to_f64(Aq, dtype), synth.to_f64(Bq, dtype), k, k, 4, 2)
+    ft = orc.project(synth.to_f64(At, dtype), synth.to_f64(Bt, dtype), k, k, 4, 2)
+    ref = orc.score(fq, ft) + 2.0 * 1.5
+    assert rel_fro(S.cpu().numpy(), ref) <= TOL[dtype]
