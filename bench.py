@@ -280,9 +280,16 @@ def main():
     torch.cuda.synchronize()
 
     ev = []  # (start, end, algorithmic bytes) per projection launch of the train set
+    phase_ev = []  # (name, event) marks of the timed steps
 
     def attribute(project, record=False):
         marks = {}
+
+        def mark(name):
+            if record:
+                e = torch.cuda.Event(enable_timing=True)
+                e.record(stream)
+                phase_ev.append((name, e))
 
         def before(li):
             if record:
@@ -306,7 +313,7 @@ def main():
                 train(li, L, route, Phi[:, li * D:], DT)
                 after(li)
             return
-        pipe.run(train, lambda li, L, route, phi, ld: project("query", li, L, route, phi, ld), after)
+        pipe.run(train, lambda li, L, route, phi, ld: project("query", li, L, route, phi, ld), after, mark)
 
     def project_dev(role, li, L, route, phi, ld):
         if role == "train":
@@ -362,6 +369,29 @@ def main():
                 "algorithmic_bytes_per_launch": per_launch,
                 "peak_source": "MEASURED_PEAKS.json hbm_gbs" if peaks else "fallback 6.8 TB/s",
                 "share_of_step": proj_ms / (ms * args.steps)}
+
+    # ---- every phase of the step against its own ceiling
+    alu = 152 * 128 * 2 * float(peaks.get("sm_max_mhz", 2070.0)) * 1e6 / 1e12  # fp32 FMA TFLOP/s
+    ph = {}
+    for (name, e0), (_, e1) in zip(phase_ev, phase_ev[1:]):
+        if name is not None:
+            ph[name] = ph.get(name, 0.0) + e0.elapsed_time(e1) / args.steps
+    Dn = float(D)
+    per_unit = {
+        "project_train": ("hbm", sum(N * (T * (L.d_in + L.d_out) * 2 + 4 * D) for L in layers), hbm, "GB/s"),
+        "project_query": ("hbm", sum(Nq * (T * (L.d_in + L.d_out) * 2 + 4 * D) for L in layers), hbm, "GB/s"),
+        "fisher_fit": ("alu", nl * N * Dn * (Dn + 1), alu, "TFLOP/s"),
+        "factor": ("latency", nl * Dn ** 3 / 3, alu, "TFLOP/s"),
+        "apply": ("latency", nl * 2 * 2 * Dn * Dn * Nq, alu, "TFLOP/s"),
+        "score": ("alu", 2.0 * Nq * N * DT, alu, "TFLOP/s"),
+        "topk": ("latency", 8.0 * Nq * N * 4, hbm, "GB/s"),
+    }
+    phases = {}
+    for name, ms_ in ph.items():
+        bound, work, peak, unit = per_unit[name]
+        rate = work / (ms_ * 1e-3) / (1e9 if unit == "GB/s" else 1e12)
+        phases[name] = {"ms": ms_, "bound": bound, "achieved": rate, "peak": peak, "unit": unit,
+                        "frac": rate / peak}
 
     # ---- e2e through tda_project_host with pinned host factors
     e2e = None
@@ -444,7 +474,7 @@ def main():
             "metric": METRIC, "value": value, "unit": "examples/s", "n_gpus": world, "steps": args.steps,
             "warmup": args.warmup, "ms_per_step": ms, "higher_is_better": True, "scaling": "weak",
             "vs_baseline": None, "dtype": "bf16", "data": "synthetic", "config": workload(args),
-            "roofline": roofline, "cpu_baseline": cpu, "e2e": e2e, "gpu_launches": launches,
+            "roofline": roofline, "phases": phases, "cpu_baseline": cpu, "e2e": e2e, "gpu_launches": launches,
             "clocks": ck,
         }
         print(json.dumps(line), flush=True)

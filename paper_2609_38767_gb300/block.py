@@ -43,27 +43,37 @@ class BlockPipeline:
     def routes(self):
         return [tda.tda_route(L, tda.TDA_OP_PROJECT, self.N, 0, tda.TDA_BF16)[0] for L in self.layers]
 
-    def run(self, project_train, project_query, after_train_linear=None):
+    def run(self, project_train, project_query, after_train_linear=None, mark=None):
         """project_train(li, L, route, phi_view, ld) fills train features of linear li;
         project_query likewise for the queries. after_train_linear(li) is called after
-        each train projection (e.g. to record timing events)."""
+        each train projection; mark(name) before each phase and mark(None) at the end
+        (e.g. to record timing events on the stream)."""
+        mark = mark or (lambda name: None)
         routes = self.routes()
         D, DT = self.D, self.DT
+        mark("project_train")
         for li, L in enumerate(self.layers):
             project_train(li, L, routes[li], self.Phi[:, li * D:], DT)
             if after_train_linear:
                 after_train_linear(li)
+        mark("project_query")
         for li, L in enumerate(self.layers):
             project_query(li, L, routes[li], self.Q[:, li * D:], DT)
         target = self.Q
         if self.precondition:
             nl, st, f32 = self.nl, self.state, tda.TDA_F32
+            mark("fisher_fit")
             tda.tda_precondition(tda.TDA_PC_RESET, nl, D, f32, st)
             tda.tda_precondition(tda.TDA_PC_FIT_ACCUM, nl, D, f32, st, phi=self.Phi, n=self.N, ld_phi=DT)
+            mark("factor")
             tda.tda_precondition(tda.TDA_PC_FACTOR, nl, D, f32, st, n_total=self.N, lambda_abs=self.lambda_abs,
                                  lambda_rel_mean_eig=self.lambda_rel)
+            mark("apply")
             tda.tda_precondition(tda.TDA_PC_APPLY, nl, D, f32, st, q=self.Q, n_q=self.Nq, ld_q=DT,
                                  qhat=self.Qh, ld_qhat=DT)
             target = self.Qh
+        mark("score")
         tda.tda_score(target, tda.TDA_F32, self.Nq, DT, self.Phi, self.N, DT, DT, self.S, self.N, 0.0)
+        mark("topk")
         tda.tda_topk(self.S, self.Nq, self.N, self.N, self.topk, self.idx, self.val)
+        mark(None)
