@@ -269,7 +269,10 @@ tda_status tda_precondition_info(int32_t n_layers, int64_t D, tda_dtype state_dt
  * tda_score -- S[q][i] = beta*S[q][i] + sum_f Qhat[q][f] Phi[i][f]
  * (gradient inner products; GradDot when Qhat = Q, Sec. 3.2 / Eq. 4).
  *   Qhat  device, n_q rows of D, q_dtype TDA_F32 or TDA_F64, row stride ld_q.
- *         With TDA_F64 the sum is accumulated in fp64.
+ *         With TDA_F64 the sum is accumulated in fp64 (CUDA cores). With
+ *         TDA_F32 on sm_103 (aligned rows, D >= 64) the sum runs on the tensor
+ *         cores as three TF32 products per element pair (hi*hi + hi*lo + lo*hi
+ *         of the split x = hi + lo), accurate to about fp32 rounding.
  *   Phi   device fp32, n_t rows of D, row stride ld_phi.
  *   S     device fp32, row stride ld_S >= n_t. beta 0 overwrites (S may hold
  *         garbage); beta 1 accumulates layers.
@@ -277,6 +280,11 @@ tda_status tda_precondition_info(int32_t n_layers, int64_t D, tda_dtype state_dt
 tda_status tda_score(const void* Qhat, tda_dtype q_dtype, int64_t n_q, int64_t ld_q,
                      const float* Phi, int64_t n_t, int64_t ld_phi, int64_t D,
                      float* S, int64_t ld_S, float beta, void* stream);
+
+/* Which kernel tda_score would run: 1 = tcgen05 3xTF32 GEMM (fp32 Qhat,
+ * 16-byte aligned rows, D >= 64, sm_103), 0 = the CUDA-core kernel. Host only. */
+int32_t tda_score_engine(const void* Qhat, tda_dtype q_dtype, int64_t n_q, int64_t ld_q, const float* Phi,
+                         int64_t n_t, int64_t ld_phi, int64_t D);
 
 /* ---------------------------------------------------------------------------
  * tda_topk -- per query row of S (n_q x n_t, fp32, row stride ld_S), the k

@@ -18,7 +18,7 @@ __all__ = [
     "tda_project_engine", "tda_project_host_ws_min", "tda_project_host", "tda_noalloc_scratch_bytes",
     "tda_project_materialized_noalloc",
     "tda_similarity_projected", "tda_similarity_exact", "tda_precondition_state_bytes", "tda_precondition",
-    "tda_precondition_info", "tda_score", "tda_topk", "tda_route", "tda_route_calibrate",
+    "tda_precondition_info", "tda_score", "tda_score_engine", "tda_topk", "tda_route", "tda_route_calibrate",
     "tda_route_set_model", "tda_device_status", "tda_selftest_bounded_wait", "tda_last_error", "tda_version", "tda_launch_count",
 ]
 
@@ -88,6 +88,7 @@ def load() -> ctypes.CDLL:
             "tda_precondition_info": (I32, [I32, I64, I32, P, ctypes.POINTER(D), P]),
             "tda_score": (I32, [P, I32, I64, I64, P, I64, I64, I64, P, I64, F, P]),
             "tda_topk": (I32, [P, I64, I64, I64, I32, P, P, P]),
+            "tda_score_engine": (I32, [P, I32, I64, I64, P, I64, I64, I64]),
             "tda_route": (I32, [LP, I32, I64, I64, I32, ctypes.POINTER(I32), ctypes.POINTER(D)]),
             "tda_route_calibrate": (I32, [P, SZ, P, ctypes.POINTER(D)]),
             "tda_route_set_model": (I32, [I32]),
@@ -209,6 +210,10 @@ def tda_precondition_info(n_layers, D, state_dtype, state, stream=None) -> list[
 def tda_score(Qhat, q_dtype, n_q, ld_q, Phi, n_t, ld_phi, D, S, ld_S, beta=0.0, stream=None):
     _check(load().tda_score(_ptr(Qhat), q_dtype, n_q, ld_q, _ptr(Phi), n_t, ld_phi, D, _ptr(S), ld_S,
                             beta, _stream(stream)))
+
+
+def tda_score_engine(Qhat, q_dtype, n_q, ld_q, Phi, n_t, ld_phi, D) -> int:
+    return int(load().tda_score_engine(_ptr(Qhat), q_dtype, n_q, ld_q, _ptr(Phi), n_t, ld_phi, D))
 
 
 def tda_topk(S, n_q, n_t, ld_S, k, idx, val=None, stream=None):

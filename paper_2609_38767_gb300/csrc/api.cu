@@ -492,9 +492,21 @@ tda_status tda_score(const void* Qhat, tda_dtype q_dtype, int64_t n_q, int64_t l
         if (D > 0 && (!Qhat || !Phi)) return fail(TDA_ERR_INVALID_ARG, "Qhat/Phi is NULL");
     }
     if (ld_q < D || ld_phi < D || ld_S < n_t) return fail(TDA_ERR_INVALID_ARG, "leading dimension too small");
+    if (n_q > 0 && n_t > 0 && score_tc_supported(q_dtype, Qhat, n_q, ld_q, Phi, n_t, ld_phi, D)) {
+        unsigned int* err = device_error_word();
+        if (!err) return fail(TDA_ERR_CUDA, "cannot resolve the device error word");
+        return cuda_check(launch_score_tc((const float*)Qhat, n_q, ld_q, Phi, n_t, ld_phi, D, S, ld_S, beta, err,
+                                          (cudaStream_t)stream),
+                          "score (tcgen05)");
+    }
     return cuda_check(launch_score(Qhat, q_dtype, n_q, ld_q, Phi, n_t, ld_phi, D, S, ld_S, beta,
                                    (cudaStream_t)stream),
                       "score");
+}
+
+int32_t tda_score_engine(const void* Qhat, tda_dtype q_dtype, int64_t n_q, int64_t ld_q, const float* Phi,
+                         int64_t n_t, int64_t ld_phi, int64_t D) {
+    return score_tc_supported(q_dtype, Qhat, n_q, ld_q, Phi, n_t, ld_phi, D) ? 1 : 0;
 }
 
 tda_status tda_topk(const float* S, int64_t n_q, int64_t n_t, int64_t ld_S, int32_t k, int32_t* idx,

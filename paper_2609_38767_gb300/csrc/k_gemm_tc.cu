@@ -1,0 +1,367 @@
+// k_gemm_tc.cu -- the score GEMM on the 5th-generation tensor cores:
+//   S[n][m] = beta * S[n][m] + sum_k Phi[m][k] * Qhat[n][k]
+// (gradient inner products between training features Phi and preconditioned
+// query features Qhat, Sec. 3.2 / Eq. 4's left side) for fp32 operands.
+//
+// fp32 accuracy from TF32 tensor cores ("3xTF32"): every operand x is split as
+// x = hi + lo with hi = x truncated to TF32 (exact) and lo = x - hi (exact in
+// fp32); the product is hi*hi' + hi*lo' + lo*hi', dropping lo*lo' (relative
+// size ~2^-22). Each K=8 step therefore issues three tcgen05.mma.kind::tf32.
+//
+// CTA tile: 128 rows of Phi (MMA M, one TMEM lane each) x BN query columns
+// (MMA N). Warps 0-3 load 128-byte row chunks with coalesced 16-byte loads,
+// split them and store hi and lo in the 128B-swizzled K-major operand layout
+// of a stage; lane 0 of warp 4 issues the MMAs; warps 4-7 read the fp32
+// accumulator tile from TMEM. A thread-block cluster of cs CTAs splits K; the
+// members' partial tiles are summed into the leader CTA over distributed shared
+// memory (deterministic, no workspace) before the leader writes S. All waits
+// are bounded (see tc_ptx.cuh).
+#include <cuda.h>
+
+#include "tda_internal.cuh"
+
+namespace tda {
+namespace {
+
+#include "tc_ptx.cuh"
+
+constexpr int kThreads = 256;
+constexpr int kBM = 128;       // Phi rows per tile
+constexpr int kKC = 32;        // fp32 elements per K chunk (one 128-byte operand row)
+constexpr uint32_t kRowBytes = kKC * 4;
+
+template <int BN>
+struct GCfg {
+    static constexpr int kStages = BN <= 64 ? 4 : (BN <= 128 ? 3 : 2);
+    static constexpr uint32_t kABytes = kBM * kRowBytes;   // 16 KiB
+    static constexpr uint32_t kBBytes = BN * kRowBytes;
+    static constexpr uint32_t kStageBytes = 2 * kABytes + 2 * kBBytes;  // hi and lo of both operands
+    static constexpr uint32_t kTmemCols = BN < 32 ? 32 : BN;
+    static constexpr size_t kSmem = 1024 + (size_t)kStages * kStageBytes + 8 * (2 * kStages + 4) + 16;  // + barriers, TMEM slot, abort flag
+};
+
+struct GParams {
+    const float* A;  // Phi, n_t rows
+    const float* B;  // Qhat, n_q rows
+    float* S;
+    int64_t n_t, n_q, K, lda, ldb, ld_S;
+    float beta;
+    int cs, tiles_n;
+    unsigned int* err;
+};
+
+// Instruction descriptor, kind::tf32: tf32 A and B (format 2), fp32 D, both K-major.
+__host__ __device__ constexpr uint32_t idesc_tf32(int M, int N) {
+    return (1u << 4) | (2u << 7) | (2u << 10) | ((uint32_t)(N >> 3) << 17) | ((uint32_t)(M >> 4) << 24);
+}
+__device__ __forceinline__ void mma_tf32(uint32_t d_tmem, uint64_t adesc, uint64_t bdesc, uint32_t idesc,
+                                         uint32_t accumulate) {
+    asm volatile(
+        "{\n .reg .pred p;\n setp.ne.b32 p, %4, 0;\n tcgen05.mma.cta_group::1.kind::tf32 [%0], %1, %2, %3, p;\n}" ::"r"(
+            d_tmem),
+        "l"(adesc), "l"(bdesc), "r"(idesc), "r"(accumulate)
+        : "memory");
+}
+__device__ __forceinline__ void split_tf32(float x, float& hi, float& lo) {
+    hi = __uint_as_float(__float_as_uint(x) & 0xFFFFE000u);
+    lo = x - hi;
+}
+
+// Rows [r0, r0+rows) of a row-major fp32 matrix, K chunk kc, into the hi and lo
+// tiles (row r at r*128 bytes, 16-byte chunk c at (c ^ (r & 7)) * 16). The 128
+// producer threads cover 4 rows x 8 chunks per pass; out-of-range is zero.
+__device__ __forceinline__ void load_split(const float* __restrict__ X, int64_t ld, int64_t nrows, int64_t K,
+                                           int64_t r0, int rows, int64_t k0, uint8_t* hi, uint8_t* lo, int pt) {
+    const int c = pt & 7;
+    const int64_t kk = k0 + c * 4;
+    for (int rr = pt >> 3; rr < rows; rr += 16) {
+        const int64_t r = r0 + rr;
+        float4 v = make_float4(0.f, 0.f, 0.f, 0.f);
+        if (r < nrows) {
+            const float* p = X + r * ld + kk;
+            if (kk + 3 < K) {
+                v = __ldg(reinterpret_cast<const float4*>(p));
+            } else {
+                v.x = kk < K ? p[0] : 0.f;
+                v.y = kk + 1 < K ? p[1] : 0.f;
+                v.z = kk + 2 < K ? p[2] : 0.f;
+                v.w = 0.f;
+            }
+        }
+        float4 h, l;
+        split_tf32(v.x, h.x, l.x);
+        split_tf32(v.y, h.y, l.y);
+        split_tf32(v.z, h.z, l.z);
+        split_tf32(v.w, h.w, l.w);
+        const uint32_t off = (uint32_t)rr * kRowBytes + (uint32_t)((c ^ (rr & 7)) << 4);
+        *reinterpret_cast<float4*>(hi + off) = h;
+        *reinterpret_cast<float4*>(lo + off) = l;
+    }
+}
+
+template <int BN>
+__global__ void __launch_bounds__(kThreads, 1) score3x_kernel(const GParams p) {
+    using C = GCfg<BN>;
+    extern __shared__ uint8_t smem_raw[];
+    uint8_t* smem = (uint8_t*)(((uintptr_t)smem_raw + 1023) & ~(uintptr_t)1023);
+    uint64_t* bars = (uint64_t*)(smem + (size_t)C::kStages * C::kStageBytes);
+    uint64_t* full = bars;                   // count 4 (producer warps)
+    uint64_t* empty = bars + C::kStages;     // count 1 (MMA commit)
+    uint64_t* tfull = empty + C::kStages;    // count 1
+    uint64_t* red_go = tfull + 1;            // count 1 (leader's remote arrive)
+    uint64_t* red_full = red_go + 1;         // count cs-1
+    uint64_t* mma_done = red_full + 1;       // count 1
+    uint32_t* tmem_slot = (uint32_t*)(mma_done + 1);
+    volatile int* abort = (volatile int*)(tmem_slot + 1);
+
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    if (threadIdx.x == 0) {
+        for (int s = 0; s < C::kStages; ++s) {
+            mbar_init(smem_u32(&full[s]), 4);
+            mbar_init(smem_u32(&empty[s]), 1);
+        }
+        mbar_init(smem_u32(tfull), 1);
+        mbar_init(smem_u32(red_go), 1);
+        mbar_init(smem_u32(red_full), p.cs > 1 ? p.cs - 1 : 1);
+        mbar_init(smem_u32(mma_done), 1);
+        *abort = 0;
+        fence_mbar_init();
+    }
+    if (warp == 4) {
+        tmem_alloc(smem_u32(tmem_slot), C::kTmemCols);
+        tmem_relinquish();
+    }
+    tc_fence_before();
+    __syncthreads();
+    cluster_sync();
+    tc_fence_after();
+    const uint32_t tmem = *tmem_slot;
+
+    const uint32_t crank = cluster_rank();
+    const int64_t tile = blockIdx.x / p.cs;
+    const int64_t m0 = (tile / p.tiles_n) * kBM, n0 = (tile % p.tiles_n) * BN;
+    const int64_t nkc = (p.K + kKC - 1) / kKC;
+    const int64_t per = (nkc + p.cs - 1) / p.cs;
+    const int64_t kc0 = crank * per, kc1 = (kc0 + per) < nkc ? (kc0 + per) : nkc;
+
+    if (warp < 4) {
+        // ---------------- producers: global fp32 -> split -> swizzled smem
+        const int pt = threadIdx.x;
+        uint32_t it = 0;
+        for (int64_t kc = kc0; kc < kc1; ++kc, ++it) {
+            const int s = it % C::kStages;
+            const uint32_t ph = (it / C::kStages) & 1u;
+            bool got = true;
+            if (lane == 0) got = wait_bounded(smem_u32(&empty[s]), ph ^ 1u, abort, p.err);
+            got = __shfl_sync(0xffffffffu, got, 0);
+            __syncwarp();
+            if (!got) break;
+            uint8_t* st = smem + (size_t)s * C::kStageBytes;
+            load_split(p.A, p.lda, p.n_t, p.K, m0, kBM, kc * kKC, st, st + C::kABytes, pt);
+            load_split(p.B, p.ldb, p.n_q, p.K, n0, BN, kc * kKC, st + 2 * C::kABytes,
+                       st + 2 * C::kABytes + C::kBBytes, pt);
+            fence_proxy_async();
+            __syncwarp();
+            if (lane == 0) mbar_arrive(smem_u32(&full[s]));
+        }
+    } else {
+        if (warp == 4 && lane == 0) {
+            // ---------------- MMA issuer
+            const uint32_t idesc = idesc_tf32(kBM, BN);
+            uint32_t it = 0;
+            bool ok = true;
+            for (int64_t kc = kc0; kc < kc1; ++kc, ++it) {
+                const int s = it % C::kStages;
+                const uint32_t ph = (it / C::kStages) & 1u;
+                if (!wait_bounded(smem_u32(&full[s]), ph, abort, p.err)) {
+                    ok = false;
+                    break;
+                }
+                tc_fence_after();
+                const uint32_t st = smem_u32(smem + (size_t)s * C::kStageBytes);
+                const uint64_t ahi = sw128_desc(st), alo = sw128_desc(st + C::kABytes);
+                const uint64_t bhi = sw128_desc(st + 2 * C::kABytes), blo = sw128_desc(st + 2 * C::kABytes + C::kBBytes);
+#pragma unroll
+                for (int k = 0; k < kKC / 8; ++k) {  // K = 8 tf32 = 32 bytes per instruction
+                    const uint32_t first = (it == 0 && k == 0) ? 0u : 1u;
+                    mma_tf32(tmem, ahi + 2 * k, bhi + 2 * k, idesc, first);
+                    mma_tf32(tmem, ahi + 2 * k, blo + 2 * k, idesc, 1u);
+                    mma_tf32(tmem, alo + 2 * k, bhi + 2 * k, idesc, 1u);
+                }
+                mma_commit(smem_u32(&empty[s]));
+            }
+            if (ok) mma_commit(smem_u32(tfull));
+            mma_commit(smem_u32(mma_done));
+            const uint64_t t0 = global_ns();
+            while (!mbar_try_wait(smem_u32(mma_done), 0))
+                if (global_ns() - t0 > kTimeoutNs) {
+                    atomicOr(p.err, kErrTimeout);
+                    break;
+                }
+        }
+        __syncwarp();
+        // ---------------- epilogue (warps 4-7): TMEM -> (cluster reduction) -> S
+        const int q = warp & 3;
+        const int row = q * 32 + lane;  // Phi row within the tile
+        const bool empty_k = kc1 <= kc0;
+        bool got = true;
+        if (!empty_k) {
+            if (lane == 0) got = wait_bounded(smem_u32(tfull), 0, abort, p.err);
+            got = __shfl_sync(0xffffffffu, got, 0);
+        }
+        float acc[BN];
+        if (!epi_any(!got)) {
+            tc_fence_after();
+            const uint32_t tbase = tmem + ((uint32_t)(q * 32) << 16);
+#pragma unroll
+            for (int c0 = 0; c0 < BN; c0 += 16) {
+                if (empty_k) {
+#pragma unroll
+                    for (int i = 0; i < 16; ++i) acc[c0 + i] = 0.f;
+                } else {
+                    tmem_ld16(tbase + c0, acc + c0);
+                }
+            }
+            tc_fence_before();
+            bool ok = true;
+            if (p.cs > 1) {
+                // partial tiles of members 1..cs-1 land in the leader's stage buffers
+                float* red = (float*)smem;
+                const uint32_t slot = smem_u32(red) + (uint32_t)(row * BN) * 4u;
+                if (crank == 0) {
+                    if (threadIdx.x == 128)
+                        for (int r = 1; r < p.cs; ++r) mbar_arrive_remote(smem_u32(red_go), (uint32_t)r);
+                    bool g2 = true;
+                    if (lane == 0) g2 = wait_bounded_cluster(smem_u32(red_full), 0, abort, p.err);
+                    g2 = __shfl_sync(0xffffffffu, g2, 0);
+                    ok = !epi_any(!g2);
+                    if (ok)
+                        for (int r = 1; r < p.cs; ++r) {
+                            const float* part = red + (size_t)(r - 1) * kBM * BN + (size_t)row * BN;
+#pragma unroll
+                            for (int c = 0; c < BN; c += 4) {
+                                const float4 v = *reinterpret_cast<const float4*>(part + c);
+                                acc[c] += v.x;
+                                acc[c + 1] += v.y;
+                                acc[c + 2] += v.z;
+                                acc[c + 3] += v.w;
+                            }
+                        }
+                } else {
+                    bool g2 = true;
+                    if (lane == 0) g2 = wait_bounded_cluster(smem_u32(red_go), 0, abort, p.err);
+                    g2 = __shfl_sync(0xffffffffu, g2, 0);
+                    ok = !epi_any(!g2);
+                    if (ok) {
+                        const uint32_t dst = map_rank(slot, 0) + (crank - 1) * (uint32_t)(kBM * BN) * 4u;
+#pragma unroll
+                        for (int c = 0; c < BN; ++c) st_cluster_f32(dst + (uint32_t)c * 4u, acc[c]);
+                        fence_acq_rel_cluster();
+                        epi_sync();
+                        if (threadIdx.x == 128) mbar_arrive_remote(smem_u32(red_full), 0u);
+                    }
+                    ok = false;  // members write nothing to S
+                }
+            }
+            if (ok) {
+                const int64_t m = m0 + row;
+                if (m < p.n_t) {
+#pragma unroll
+                    for (int c = 0; c < BN; ++c) {
+                        const int64_t n = n0 + c;
+                        if (n < p.n_q) {
+                            float* dst = p.S + n * p.ld_S + m;
+                            *dst = (p.beta == 0.f) ? acc[c] : p.beta * (*dst) + acc[c];
+                        }
+                    }
+                }
+            }
+        }
+    }
+
+    tc_fence_before();
+    __syncthreads();
+    if (warp == 4) {
+        tc_fence_after();
+        tmem_dealloc(tmem, C::kTmemCols);
+    }
+    cluster_sync();
+}
+
+template <int BN>
+cudaError_t launch_bn(GParams p, cudaStream_t s) {
+    using C = GCfg<BN>;
+    static int sms = 0;
+    if (!sms) {
+        int dev = 0;
+        cudaGetDevice(&dev);
+        cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+        if (sms <= 0) sms = 1;
+    }
+    const int64_t tiles_m = (p.n_t + kBM - 1) / kBM, tiles_n = (p.n_q + BN - 1) / BN;
+    const int64_t tiles = tiles_m * tiles_n;
+    const int64_t nkc = (p.K + kKC - 1) / kKC;
+    int cs = 1;
+    while (cs < 4 && tiles * cs * 2 <= sms && nkc >= 8 * cs * 2) cs *= 2;
+    // the leader's stage buffers must hold the members' partial tiles
+    while (cs > 1 && (size_t)(cs - 1) * kBM * BN * 4 > (size_t)C::kStages * C::kStageBytes) cs >>= 1;
+    p.cs = cs;
+    p.tiles_n = (int)tiles_n;
+    cudaError_t e = cudaFuncSetAttribute(score3x_kernel<BN>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)C::kSmem);
+    if (e != cudaSuccess) return e;
+    cudaLaunchConfig_t cfg = {};
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeClusterDimension;
+    attr[0].val.clusterDim.x = (unsigned)cs;
+    attr[0].val.clusterDim.y = 1;
+    attr[0].val.clusterDim.z = 1;
+    cfg.gridDim = dim3((unsigned)(tiles * cs));
+    cfg.blockDim = dim3(kThreads);
+    cfg.dynamicSmemBytes = C::kSmem;
+    cfg.stream = s;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    note_launches(1);
+    e = cudaLaunchKernelEx(&cfg, score3x_kernel<BN>, p);
+    if (e != cudaSuccess) return e;
+    return cudaGetLastError();
+}
+
+}  // namespace
+
+bool score_tc_supported(tda_dtype qdt, const void* Qhat, int64_t n_q, int64_t ld_q, const float* Phi, int64_t n_t,
+                        int64_t ld_phi, int64_t D) {
+    static int sm103 = -1;
+    if (sm103 < 0) {
+        int dev = 0, major = 0, minor = 0;
+        cudaGetDevice(&dev);
+        cudaDeviceGetAttribute(&major, cudaDevAttrComputeCapabilityMajor, dev);
+        cudaDeviceGetAttribute(&minor, cudaDevAttrComputeCapabilityMinor, dev);
+        sm103 = (major == 10 && minor == 3) ? 1 : 0;
+    }
+    if (!sm103 || qdt != TDA_F32) return false;
+    if (n_q < 1 || n_t < 1 || D < 64 || n_q > (1LL << 24) || n_t > (1LL << 31) / kBM * kBM) return false;
+    if ((ld_q & 3) || (ld_phi & 3)) return false;
+    if (((uintptr_t)Qhat & 15) || ((uintptr_t)Phi & 15)) return false;
+    return true;
+}
+
+cudaError_t launch_score_tc(const float* Qhat, int64_t n_q, int64_t ld_q, const float* Phi, int64_t n_t, int64_t ld_phi,
+                            int64_t D, float* S, int64_t ld_S, float beta, unsigned int* err, cudaStream_t s) {
+    GParams p{};
+    p.A = Phi;
+    p.B = Qhat;
+    p.S = S;
+    p.n_t = n_t;
+    p.n_q = n_q;
+    p.K = D;
+    p.lda = ld_phi;
+    p.ldb = ld_q;
+    p.ld_S = ld_S;
+    p.beta = beta;
+    p.err = err;
+    if (n_q <= 64) return launch_bn<64>(p, s);
+    return launch_bn<128>(p, s);
+}
+
+}  // namespace tda

@@ -386,3 +386,20 @@ def test_similarity_projected_routes_match_oracle(dev, orc, dtype, route):
     ft = orc.project(synth.to_f64(At, dtype), synth.to_f64(Bt, dtype), k, k, 4, 2)
     ref = orc.score(fq, ft) + 2.0 * 1.5
     assert rel_fro(S.cpu().numpy(), ref) <= TOL[dtype]
+
+
+@pytest.mark.parametrize("nq,nt,D,beta", [(8, 64, 256, 0.0), (70, 300, 1024, 1.0), (64, 4096, 7168, 0.0),
+                                          (3, 130, 100, 0.5), (200, 257, 64, 0.0)])
+def test_score_tensor_core_matches_oracle(dev, orc, nq, nt, D, beta):
+    # fp32 scores on tcgen05 (3xTF32, cluster split-K): within the fp32 tolerance
+    rng = np.random.default_rng(nq + nt + D)
+    Q = rng.standard_normal((nq, D)).astype(np.float32)
+    P = (rng.standard_normal((nt, D)) * rng.uniform(0.1, 10.0, (nt, 1))).astype(np.float32)
+    Qd, Pd = torch.from_numpy(Q).to(dev), torch.from_numpy(P).to(dev)
+    assert tda.tda_score_engine(Qd, tda.TDA_F32, nq, D, Pd, nt, D, D) == 1
+    S0 = rng.standard_normal((nq, nt)).astype(np.float32)
+    S = torch.from_numpy(S0).to(dev)
+    tda.tda_score(Qd, tda.TDA_F32, nq, D, Pd, nt, D, D, S, nt, beta=beta)
+    tda.tda_device_status()
+    ref = orc.score(Q, P) + beta * S0.astype(np.float64)
+    assert rel_fro(S.cpu().numpy(), ref) <= 1e-5
