@@ -36,7 +36,11 @@ struct GCfg {
     static constexpr uint32_t kABytes = kBM * kRowBytes;   // 16 KiB
     static constexpr uint32_t kBBytes = BN * kRowBytes;
     static constexpr uint32_t kStageBytes = 2 * kABytes + 2 * kBBytes;  // hi and lo of both operands
-    static constexpr uint32_t kTmemCols = BN < 32 ? 32 : BN;
+    // K chunks rotate over kAcc accumulators (all 512 TMEM columns): each sees
+    // 1/kAcc of the additions, which bounds the tensor core's fp32 accumulation
+    // error; the epilogue sums them on CUDA cores with round-to-nearest.
+    static constexpr int kAcc = 512 / BN < 8 ? 512 / BN : 8;
+    static constexpr uint32_t kTmemCols = 512;
     static constexpr size_t kSmem = 1024 + (size_t)kStages * kStageBytes + 8 * (2 * kStages + 4) + 16;  // + barriers, TMEM slot, abort flag
 };
 
@@ -183,10 +187,11 @@ __global__ void __launch_bounds__(kThreads, 1) score3x_kernel(const GParams p) {
                 const uint64_t bhi = sw128_desc(st + 2 * C::kABytes), blo = sw128_desc(st + 2 * C::kABytes + C::kBBytes);
 #pragma unroll
                 for (int k = 0; k < kKC / 8; ++k) {  // K = 8 tf32 = 32 bytes per instruction
-                    const uint32_t first = (it == 0 && k == 0) ? 0u : 1u;
-                    mma_tf32(tmem, ahi + 2 * k, bhi + 2 * k, idesc, first);
-                    mma_tf32(tmem, ahi + 2 * k, blo + 2 * k, idesc, 1u);
-                    mma_tf32(tmem, alo + 2 * k, bhi + 2 * k, idesc, 1u);
+                    const uint32_t d = tmem + (it % C::kAcc) * BN;
+                    const uint32_t first = (it < (uint32_t)C::kAcc && k == 0) ? 0u : 1u;
+                    mma_tf32(d, ahi + 2 * k, bhi + 2 * k, idesc, first);
+                    mma_tf32(d, ahi + 2 * k, blo + 2 * k, idesc, 1u);
+                    mma_tf32(d, alo + 2 * k, bhi + 2 * k, idesc, 1u);
                 }
                 mma_commit(smem_u32(&empty[s]));
             }
@@ -213,13 +218,16 @@ __global__ void __launch_bounds__(kThreads, 1) score3x_kernel(const GParams p) {
         if (!epi_any(!got)) {
             tc_fence_after();
             const uint32_t tbase = tmem + ((uint32_t)(q * 32) << 16);
+            const int used = (int)((kc1 - kc0) < C::kAcc ? (kc1 - kc0) : C::kAcc);  // accumulators written
 #pragma unroll
             for (int c0 = 0; c0 < BN; c0 += 16) {
-                if (empty_k) {
 #pragma unroll
-                    for (int i = 0; i < 16; ++i) acc[c0 + i] = 0.f;
-                } else {
-                    tmem_ld16(tbase + c0, acc + c0);
+                for (int i = 0; i < 16; ++i) acc[c0 + i] = 0.f;
+                for (int a = 0; a < used; ++a) {
+                    float v[16];
+                    tmem_ld16(tbase + a * BN + c0, v);
+#pragma unroll
+                    for (int i = 0; i < 16; ++i) acc[c0 + i] += v[i];
                 }
             }
             tc_fence_before();
