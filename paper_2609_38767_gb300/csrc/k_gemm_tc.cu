@@ -74,12 +74,18 @@ __device__ __forceinline__ void split_tf32(float x, float& hi, float& lo) {
 // Rows [r0, r0+rows) of a row-major fp32 matrix, K chunk kc, into the hi and lo
 // tiles (row r at r*128 bytes, 16-byte chunk c at (c ^ (r & 7)) * 16). The 128
 // producer threads cover 4 rows x 8 chunks per pass; out-of-range is zero.
+// ROWS is a compile-time multiple of 16 so that all of a thread's loads issue
+// before the first one is consumed.
+template <int ROWS>
 __device__ __forceinline__ void load_split(const float* __restrict__ X, int64_t ld, int64_t nrows, int64_t K,
-                                           int64_t r0, int rows, int64_t k0, uint8_t* hi, uint8_t* lo, int pt) {
+                                           int64_t r0, int64_t k0, uint8_t* hi, uint8_t* lo, int pt) {
+    constexpr int kPer = ROWS / 16;
     const int c = pt & 7;
     const int64_t kk = k0 + c * 4;
-    for (int rr = pt >> 3; rr < rows; rr += 16) {
-        const int64_t r = r0 + rr;
+    float4 vals[kPer];
+#pragma unroll
+    for (int u = 0; u < kPer; ++u) {
+        const int64_t r = r0 + (pt >> 3) + 16 * u;
         float4 v = make_float4(0.f, 0.f, 0.f, 0.f);
         if (r < nrows) {
             const float* p = X + r * ld + kk;
@@ -92,6 +98,12 @@ __device__ __forceinline__ void load_split(const float* __restrict__ X, int64_t 
                 v.w = 0.f;
             }
         }
+        vals[u] = v;
+    }
+#pragma unroll
+    for (int u = 0; u < kPer; ++u) {
+        const int rr = (pt >> 3) + 16 * u;
+        const float4 v = vals[u];
         float4 h, l;
         split_tf32(v.x, h.x, l.x);
         split_tf32(v.y, h.y, l.y);
@@ -161,9 +173,9 @@ __global__ void __launch_bounds__(kThreads, 1) score3x_kernel(const GParams p) {
             __syncwarp();
             if (!got) break;
             uint8_t* st = smem + (size_t)s * C::kStageBytes;
-            load_split(p.A, p.lda, p.n_t, p.K, m0, kBM, kc * kKC, st, st + C::kABytes, pt);
-            load_split(p.B, p.ldb, p.n_q, p.K, n0, BN, kc * kKC, st + 2 * C::kABytes,
-                       st + 2 * C::kABytes + C::kBBytes, pt);
+            load_split<kBM>(p.A, p.lda, p.n_t, p.K, m0, kc * kKC, st, st + C::kABytes, pt);
+            load_split<BN>(p.B, p.ldb, p.n_q, p.K, n0, kc * kKC, st + 2 * C::kABytes,
+                           st + 2 * C::kABytes + C::kBBytes, pt);
             fence_proxy_async();
             __syncwarp();
             if (lane == 0) mbar_arrive(smem_u32(&full[s]));
