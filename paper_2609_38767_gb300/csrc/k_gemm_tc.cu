@@ -308,6 +308,197 @@ __global__ void __launch_bounds__(kThreads, 1) score3x_kernel(const GParams p) {
     cluster_sync();
 }
 
+// ---------------------------------------------------------------------------
+// Fisher fit on the tensor cores: M_l += Phi_l^T Phi_l for the lower 128 x 128
+// tiles of every layer l (layer l's features at column l*D of each row of Phi).
+// The operand tiles are features x examples, K-major: 32 examples per chunk.
+// Lane l of a producer warp loads example row e0+l, 16 bytes at a time, and
+// writes the four features transposed into the swizzled layout (conflict-free:
+// the 32 lanes hit 32 distinct banks).
+template <int ROWS>
+__device__ __forceinline__ void load_split_t(const float* __restrict__ X, int64_t ld, int64_t nrows, int64_t D,
+                                             int64_t f0, int64_t e0, uint8_t* hi, uint8_t* lo, int pt) {
+    constexpr int kPer = ROWS / 16;  // float4 groups per thread: 4 warps x 4 features x kPer
+    const int lane = pt & 31, w = pt >> 5;
+    const int64_t e = e0 + lane;
+    float4 vals[kPer];
+#pragma unroll
+    for (int j = 0; j < kPer; ++j) {
+        const int64_t f = f0 + (ROWS / 4) * w + 4 * j;
+        float4 v = make_float4(0.f, 0.f, 0.f, 0.f);
+        if (e < nrows) {
+            const float* p = X + e * ld + f;
+            if (f + 3 < D) {
+                v = __ldg(reinterpret_cast<const float4*>(p));
+            } else {
+                v.x = f < D ? p[0] : 0.f;
+                v.y = f + 1 < D ? p[1] : 0.f;
+                v.z = f + 2 < D ? p[2] : 0.f;
+                v.w = 0.f;
+            }
+        }
+        vals[j] = v;
+    }
+#pragma unroll
+    for (int j = 0; j < kPer; ++j) {
+        const float in[4] = {vals[j].x, vals[j].y, vals[j].z, vals[j].w};
+#pragma unroll
+        for (int i = 0; i < 4; ++i) {
+            const int fr = (ROWS / 4) * w + 4 * j + i;  // feature row of the tile
+            const uint32_t off = (uint32_t)fr * kRowBytes + (uint32_t)((((lane >> 2) ^ (fr & 7)) << 4) + (lane & 3) * 4);
+            float h, l;
+            split_tf32(in[i], h, l);
+            *reinterpret_cast<float*>(hi + off) = h;
+            *reinterpret_cast<float*>(lo + off) = l;
+        }
+    }
+}
+
+struct FParams {
+    const float* phi;
+    char* state;       // layer states, `bytes` apart; M at +64
+    size_t bytes;
+    int64_t D, n, ld;
+    int tiles;         // lower tiles per layer
+    unsigned int* err;
+};
+
+__global__ void __launch_bounds__(kThreads, 1) fit3x_kernel(const FParams p) {
+    constexpr int BN = 128;
+    using C = GCfg<BN>;
+    extern __shared__ uint8_t smem_raw[];
+    uint8_t* smem = (uint8_t*)(((uintptr_t)smem_raw + 1023) & ~(uintptr_t)1023);
+    uint64_t* bars = (uint64_t*)(smem + (size_t)C::kStages * C::kStageBytes);
+    uint64_t* full = bars;
+    uint64_t* empty = bars + C::kStages;
+    uint64_t* tfull = empty + C::kStages;
+    uint64_t* mma_done = tfull + 1;
+    uint32_t* tmem_slot = (uint32_t*)(mma_done + 3);
+    volatile int* abort = (volatile int*)(tmem_slot + 1);
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    if (threadIdx.x == 0) {
+        for (int s = 0; s < C::kStages; ++s) {
+            mbar_init(smem_u32(&full[s]), 4);
+            mbar_init(smem_u32(&empty[s]), 1);
+        }
+        mbar_init(smem_u32(tfull), 1);
+        mbar_init(smem_u32(mma_done), 1);
+        *abort = 0;
+        fence_mbar_init();
+    }
+    if (warp == 4) {
+        tmem_alloc(smem_u32(tmem_slot), C::kTmemCols);
+        tmem_relinquish();
+    }
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+    const uint32_t tmem = *tmem_slot;
+
+    const int layer = blockIdx.x / p.tiles;
+    const int t = blockIdx.x - layer * p.tiles;
+    int by = (int)((sqrtf(8.f * t + 1.f) - 1.f) * 0.5f);  // lower-tile index -> (by, bx), bx <= by
+    while ((by + 1) * (by + 2) / 2 <= t) ++by;
+    while (by * (by + 1) / 2 > t) --by;
+    const int bx = t - by * (by + 1) / 2;
+    const int64_t a0 = (int64_t)by * kBM, b0 = (int64_t)bx * BN;
+    const float* ph = p.phi + (int64_t)layer * p.D;
+    const int64_t nkc = (p.n + kKC - 1) / kKC;
+
+    if (warp < 4) {
+        uint32_t it = 0;
+        for (int64_t kc = 0; kc < nkc; ++kc, ++it) {
+            const int s = it % C::kStages;
+            const uint32_t phz = (it / C::kStages) & 1u;
+            bool got = true;
+            if (lane == 0) got = wait_bounded(smem_u32(&empty[s]), phz ^ 1u, abort, p.err);
+            got = __shfl_sync(0xffffffffu, got, 0);
+            __syncwarp();
+            if (!got) break;
+            uint8_t* st = smem + (size_t)s * C::kStageBytes;
+            load_split_t<kBM>(ph, p.ld, p.n, p.D, a0, kc * kKC, st, st + C::kABytes, threadIdx.x);
+            load_split_t<BN>(ph, p.ld, p.n, p.D, b0, kc * kKC, st + 2 * C::kABytes, st + 2 * C::kABytes + C::kBBytes,
+                             threadIdx.x);
+            fence_proxy_async();
+            __syncwarp();
+            if (lane == 0) mbar_arrive(smem_u32(&full[s]));
+        }
+    } else {
+        if (warp == 4 && lane == 0) {
+            const uint32_t idesc = idesc_tf32(kBM, BN);
+            uint32_t it = 0;
+            bool ok = true;
+            for (int64_t kc = 0; kc < nkc; ++kc, ++it) {
+                const int s = it % C::kStages;
+                const uint32_t phz = (it / C::kStages) & 1u;
+                if (!wait_bounded(smem_u32(&full[s]), phz, abort, p.err)) {
+                    ok = false;
+                    break;
+                }
+                tc_fence_after();
+                const uint32_t st = smem_u32(smem + (size_t)s * C::kStageBytes);
+                const uint64_t ahi = sw128_desc(st), alo = sw128_desc(st + C::kABytes);
+                const uint64_t bhi = sw128_desc(st + 2 * C::kABytes), blo = sw128_desc(st + 2 * C::kABytes + C::kBBytes);
+#pragma unroll
+                for (int k = 0; k < kKC / 8; ++k) {
+                    const uint32_t d = tmem + (it % C::kAcc) * BN;
+                    const uint32_t first = (it < (uint32_t)C::kAcc && k == 0) ? 0u : 1u;
+                    mma_tf32(d, ahi + 2 * k, bhi + 2 * k, idesc, first);
+                    mma_tf32(d, ahi + 2 * k, blo + 2 * k, idesc, 1u);
+                    mma_tf32(d, alo + 2 * k, bhi + 2 * k, idesc, 1u);
+                }
+                mma_commit(smem_u32(&empty[s]));
+            }
+            if (ok) mma_commit(smem_u32(tfull));
+            mma_commit(smem_u32(mma_done));
+            const uint64_t t0 = global_ns();
+            while (!mbar_try_wait(smem_u32(mma_done), 0))
+                if (global_ns() - t0 > kTimeoutNs) {
+                    atomicOr(p.err, kErrTimeout);
+                    break;
+                }
+        }
+        __syncwarp();
+        const int q = warp & 3;
+        const int row = q * 32 + lane;
+        bool got = true;
+        if (lane == 0) got = wait_bounded(smem_u32(tfull), 0, abort, p.err);
+        got = __shfl_sync(0xffffffffu, got, 0);
+        if (!epi_any(!got)) {
+            tc_fence_after();
+            const uint32_t tbase = tmem + ((uint32_t)(q * 32) << 16);
+            const int used = (int)(nkc < C::kAcc ? nkc : C::kAcc);
+            const int64_t a = a0 + row;
+            float* M = (float*)(p.state + (size_t)layer * p.bytes + 64);
+#pragma unroll
+            for (int c0 = 0; c0 < BN; c0 += 16) {
+                float acc[16];
+#pragma unroll
+                for (int i = 0; i < 16; ++i) acc[i] = 0.f;
+                for (int u = 0; u < used; ++u) {
+                    float v[16];
+                    tmem_ld16(tbase + u * BN + c0, v);
+#pragma unroll
+                    for (int i = 0; i < 16; ++i) acc[i] += v[i];
+                }
+                if (a < p.D)
+#pragma unroll
+                    for (int i = 0; i < 16; ++i) {
+                        const int64_t b = b0 + c0 + i;
+                        if (b < p.D) M[a * p.D + b] += acc[i];
+                    }
+            }
+            tc_fence_before();
+        }
+    }
+    tc_fence_before();
+    __syncthreads();
+    if (warp == 4) {
+        tc_fence_after();
+        tmem_dealloc(tmem, C::kTmemCols);
+    }
+}
+
 template <int BN>
 cudaError_t launch_bn(GParams p, cudaStream_t s) {
     using C = GCfg<BN>;
@@ -382,6 +573,35 @@ cudaError_t launch_score_tc(const float* Qhat, int64_t n_q, int64_t ld_q, const 
     p.err = err;
     if (n_q <= 64) return launch_bn<64>(p, s);
     return launch_bn<128>(p, s);
+}
+
+bool fit_tc_supported(int64_t D, const float* phi, int64_t ld) {
+    int dev = 0, major = 0, minor = 0;
+    cudaGetDevice(&dev);
+    cudaDeviceGetAttribute(&major, cudaDevAttrComputeCapabilityMajor, dev);
+    cudaDeviceGetAttribute(&minor, cudaDevAttrComputeCapabilityMinor, dev);
+    if (!(major == 10 && minor == 3)) return false;
+    return D >= 128 && (D & 3) == 0 && (ld & 3) == 0 && ((uintptr_t)phi & 15) == 0;
+}
+
+cudaError_t launch_fit_tc(int n_layers, int64_t D, void* state, size_t state_bytes, const float* phi, int64_t n,
+                          int64_t ld, unsigned int* err, cudaStream_t s) {
+    using C = GCfg<128>;
+    const int64_t nt = (D + kBM - 1) / kBM;
+    FParams p{};
+    p.phi = phi;
+    p.state = (char*)state;
+    p.bytes = state_bytes;
+    p.D = D;
+    p.n = n;
+    p.ld = ld;
+    p.tiles = (int)(nt * (nt + 1) / 2);
+    p.err = err;
+    cudaError_t e = cudaFuncSetAttribute(fit3x_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)C::kSmem);
+    if (e != cudaSuccess) return e;
+    note_launches(1);
+    fit3x_kernel<<<(unsigned)(p.tiles * n_layers), kThreads, C::kSmem, s>>>(p);
+    return cudaGetLastError();
 }
 
 }  // namespace tda

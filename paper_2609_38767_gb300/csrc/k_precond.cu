@@ -485,6 +485,11 @@ int64_t precondition_apply_max_d(tda_dtype sdt) {
 cudaError_t launch_pc_fit(int n_layers, int64_t D, tda_dtype sdt, void* state, const float* phi, int64_t n,
                           int64_t ld, cudaStream_t s) {
     if (n == 0) return cudaSuccess;
+    if (sdt == TDA_F32 && fit_tc_supported(D, phi, ld)) {
+        unsigned int* err = device_error_word();
+        if (err)
+            return launch_fit_tc(n_layers, D, state, tda_precondition_state_bytes(D, TDA_F32), phi, n, ld, err, s);
+    }
     note_launches(1);
     if (sdt == TDA_F64) {
         const unsigned t = (unsigned)((D + 63) / 64);
