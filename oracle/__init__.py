@@ -59,6 +59,9 @@ def _load():
             "oracle_project_materialized": (None, [I64, I64, I64, I64, I64, I64, U64, U32, I32, D, D, D]),
             "oracle_similarity_materialized": (None, [I64, I64, I64, I64, D, D, I64, D, D, D]),
             "oracle_similarity_gram": (None, [I64, I64, I64, I64, D, D, I64, D, D, D]),
+            "oracle_sq_norms_materialized": (None, [I64, I64, I64, I64, D, D, D]),
+            "oracle_sq_norms_gram": (None, [I64, I64, I64, I64, D, D, D]),
+            "oracle_cosine": (None, [I64, I64, D, D, D, D]),
             "oracle_fisher": (None, [I64, I64, D, D]),
             "oracle_damping": (ctypes.c_double, [I64, D, ctypes.c_double, ctypes.c_double]),
             "oracle_cholesky": (I32, [I64, D]),
@@ -157,6 +160,24 @@ def similarity(Aq, Bq, At, Bt, route: str = "gram") -> np.ndarray:
     return S
 
 
+def sq_norms(A, B, route: str = "gram") -> np.ndarray:
+    """Squared Frobenius norms of the N per-example gradients (N,T,d) factors."""
+    A, B = _f64(A), _f64(B)
+    N, T, d_in = A.shape
+    d_out = B.shape[2]
+    out = np.empty(N)
+    fn = _load().oracle_sq_norms_gram if route == "gram" else _load().oracle_sq_norms_materialized
+    fn(N, T, d_in, d_out, _p(A), _p(B), _p(out))
+    return out
+
+
+def cosine(S, nq, nt) -> np.ndarray:
+    S, nq, nt = _f64(S), _f64(nq), _f64(nt)
+    C = np.empty_like(S)
+    _load().oracle_cosine(S.shape[0], S.shape[1], _p(S), _p(nq), _p(nt), _p(C))
+    return C
+
+
 # ---------------------------------------------------------------- preconditioning
 def fisher(phi) -> np.ndarray:
     phi = _f64(phi)
@@ -213,7 +234,7 @@ def topk(S, k: int) -> tuple[np.ndarray, np.ndarray]:
 
 
 # ---------------------------------------------------------------- routing
-OP_PROJECT, OP_SIM_PROJECTED, OP_SIM_EXACT = 0, 1, 2
+OP_PROJECT, OP_SIM_PROJECTED, OP_SIM_EXACT, OP_NORM_PROJECTED, OP_NORM_EXACT = 0, 1, 2, 3, 4
 
 
 def route_costs(op: int, n1: int, n2: int, T: int, d_in: int, d_out: int,

@@ -240,6 +240,40 @@ void oracle_similarity_gram(int64_t T, int64_t d_in, int64_t d_out,
 }
 
 /* ------------------------------------------------------------------------ */
+/* Norms and cosine                                                         */
+/* ------------------------------------------------------------------------ */
+
+void oracle_sq_norms_materialized(int64_t N, int64_t T, int64_t d_in, int64_t d_out,
+                                  const double* A, const double* B, double* out) {
+#ifdef _OPENMP
+#pragma omp parallel for schedule(dynamic, 1) num_threads(g_threads)
+#endif
+    for (int64_t n = 0; n < N; ++n) {
+        double* G = (double*)malloc(sizeof(double) * (size_t)(d_out * d_in));
+        oracle_materialize(T, d_in, d_out, A + n * T * d_in, B + n * T * d_out, G);
+        double s = 0.0;
+        for (int64_t e = 0; e < d_out * d_in; ++e) s += G[e] * G[e];
+        out[n] = s;
+        free(G);
+    }
+}
+
+void oracle_sq_norms_gram(int64_t N, int64_t T, int64_t d_in, int64_t d_out,
+                          const double* A, const double* B, double* out) {
+    for (int64_t n = 0; n < N; ++n)
+        oracle_similarity_gram(T, d_in, d_out, 1, A + n * T * d_in, B + n * T * d_out,
+                               1, A + n * T * d_in, B + n * T * d_out, out + n);
+}
+
+/* LESS-style cosine: the inner product over the product of the two norms. */
+void oracle_cosine(int64_t n_q, int64_t n_t, const double* S, const double* nq,
+                   const double* nt, double* C) {
+    for (int64_t q = 0; q < n_q; ++q)
+        for (int64_t i = 0; i < n_t; ++i)
+            C[q * n_t + i] = S[q * n_t + i] / sqrt(nq[q] * nt[i]);
+}
+
+/* ------------------------------------------------------------------------ */
 /* Preconditioning                                                          */
 /* ------------------------------------------------------------------------ */
 
@@ -395,11 +429,21 @@ int32_t oracle_route_costs(int32_t op, int64_t n1, int64_t n2, int64_t T,
         cost[0] = (B1 + B2) * (proj_factors + contract) + B1 * B2 * 2.0 * ka * kg;
         cost[1] = (B1 + B2) * (build + project_dense) + B1 * B2 * 2.0 * ka * kg;
         cost[2] = (B1 + B2) * proj_factors + B1 * B2 * 2.0 * t * t * (ka + kg);
-    } else {
+    } else if (op == 2) {
         /* Table 2 as printed: materialised vs factorised cross-Gram */
         cost[0] = -1.0;
         cost[1] = (B1 + B2) * build + B1 * B2 * 2.0 * Ni * No;
         cost[2] = B1 * B2 * 2.0 * t * t * (Ni + No);
+    } else if (op == 3) {
+        /* norms of projected gradients: Table 2 with B1 = B2 = 1 per example */
+        cost[0] = B1 * (proj_factors + contract + 2.0 * ka * kg);
+        cost[1] = B1 * (build + project_dense + 2.0 * ka * kg);
+        cost[2] = B1 * (proj_factors + 2.0 * t * t * (ka + kg));
+    } else {
+        /* norms of unprojected gradients */
+        cost[0] = -1.0;
+        cost[1] = B1 * (build + 2.0 * Ni * No);
+        cost[2] = B1 * 2.0 * t * t * (Ni + No);
     }
     /* cheapest valid route; ties prefer the factorised (Gram) route, then the
      * factored projection, then materialisation */

@@ -89,6 +89,20 @@ void oracle_similarity_gram(int64_t T, int64_t d_in, int64_t d_out,
                             int64_t n_q, const double* Aq, const double* Bq,
                             int64_t n_t, const double* At, const double* Bt, double* S);
 
+/* ---- per-example gradient norms (App. A.4: norms are routed like Gram
+ *      matrices) and cosine scores ---- */
+
+/* ||DW||_F^2 of each of N examples: materialised (Eq. 1, sum of squares). */
+void oracle_sq_norms_materialized(int64_t N, int64_t T, int64_t d_in, int64_t d_out,
+                                  const double* A, const double* B, double* out);
+/* ||DW||_F^2 by Eq. 4 with both sides the same example:
+ * sum_{t,s} <a_t, a_s> <g_t, g_s>. */
+void oracle_sq_norms_gram(int64_t N, int64_t T, int64_t d_in, int64_t d_out,
+                          const double* A, const double* B, double* out);
+/* Cosine scores C[q][i] = S[q][i] / sqrt(nq[q] * nt[i]) from squared norms. */
+void oracle_cosine(int64_t n_q, int64_t n_t, const double* S, const double* nq,
+                   const double* nt, double* C);
+
 /* ---- curvature preconditioning of the queries (App. B.2, B.3) ---- */
 
 /* F = (1/N) sum_i phi_i phi_i^T (D x D). */
@@ -115,7 +129,9 @@ void oracle_topk(int64_t n_q, int64_t n_t, const double* S, int32_t k,
 /* ---- FLOP cost of each route (App. A.4, Table 2) ---- */
 
 /* op 0 = project N=n1 examples; op 1 = n1 x n2 similarity of projected
- * gradients; op 2 = n1 x n2 exact (unprojected) similarity.
+ * gradients; op 2 = n1 x n2 exact (unprojected) similarity; op 3 = squared
+ * norms of n1 projected gradients; op 4 = squared norms of n1 unprojected
+ * gradients.
  * cost[0] factored, cost[1] materialised, cost[2] Gram; a route that does not
  * produce the op's result gets -1. Returns the index of the cheapest route
  * (ties go to the lower index, i.e. the factored side). */

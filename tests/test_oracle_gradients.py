@@ -142,3 +142,31 @@ def test_gram_on_projected_factors_equals_projected_scores(orc):
     ft = orc.project(At, Bt, k_in, k_out, seed=3, layer=7)
     Sg = orc.similarity(Aq @ P_in, Bq @ P_out, At @ P_in, Bt @ P_out, route="gram")
     np.testing.assert_allclose(orc.score(fq, ft), Sg, rtol=1e-12)
+
+
+def test_squared_norms_two_routes_and_brute_force(orc):
+    # App. A.4 routes norms like Gram matrices: ||DW||^2 by Eq. 1 and by Eq. 4 agree
+    rng = np.random.default_rng(10)
+    N, T, di, do = 4, 6, 9, 7
+    A, B = _rand(rng, N, T, di), _rand(rng, N, T, do)
+    g = orc.sq_norms(A, B, "gram")
+    m = orc.sq_norms(A, B, "materialized")
+    brute = np.array([float((orc.materialize(A[n], B[n]) ** 2).sum()) for n in range(N)])
+    np.testing.assert_allclose(g, brute, rtol=1e-12)
+    np.testing.assert_allclose(m, brute, rtol=1e-12)
+    # a rank-one gradient g a^T (T = 1) has norm ||g||^2 ||a||^2
+    one = orc.sq_norms(A[:, :1], B[:, :1])
+    np.testing.assert_allclose(one, (A[:, 0] ** 2).sum(1) * (B[:, 0] ** 2).sum(1), rtol=1e-13)
+
+
+def test_cosine_properties(orc):
+    rng = np.random.default_rng(11)
+    X = rng.standard_normal((5, 12))
+    S = orc.score(X, X)
+    n = (X ** 2).sum(1)
+    C = orc.cosine(S, n, n)
+    np.testing.assert_allclose(np.diag(C), 1.0, rtol=1e-14)
+    assert np.abs(C).max() <= 1 + 1e-12
+    # invariant to scaling either side
+    C2 = orc.cosine(orc.score(3 * X, X), 9 * n, n)
+    np.testing.assert_allclose(C2, C, rtol=1e-13)

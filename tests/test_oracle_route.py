@@ -45,3 +45,16 @@ def test_projection_shrinks_the_factorised_regime(orc):
 def test_tiny_T_prefers_gram_for_projected_similarity(orc, T):
     best, _ = orc.route_costs(orc.OP_SIM_PROJECTED, 8, 8, T, 256, 256, 64, 64)
     assert best == 2
+
+
+def test_norm_costs_are_table2_with_one_example_per_side(orc):
+    n, T, di, do, k = 5, 16, 64, 32, 8
+    _, c = orc.route_costs(orc.OP_NORM_EXACT, n, 0, T, di, do)
+    assert c[0] == -1
+    assert c[1] == n * (2 * T * di * do + 2 * di * do)
+    assert c[2] == n * 2 * T * T * (di + do)
+    _, cp = orc.route_costs(orc.OP_NORM_PROJECTED, n, 0, T, di, do, k, k)
+    assert cp[2] == n * (2 * T * (di * k + do * k) + 2 * T * T * (2 * k))
+    # long sequences favour materialising for exact norms, short ones the Gram route
+    assert orc.route_costs(orc.OP_NORM_EXACT, 1, 0, 4, 1024, 1024)[0] == 2
+    assert orc.route_costs(orc.OP_NORM_EXACT, 1, 0, 4096, 1024, 1024)[0] == 1
