@@ -78,7 +78,9 @@ typedef enum {
 typedef enum {
     TDA_OP_PROJECT = 0,             /* n1 examples -> n1 projected features      */
     TDA_OP_SIMILARITY_PROJECTED = 1,/* n1 x n2 inner products of projected grads */
-    TDA_OP_SIMILARITY_EXACT = 2     /* n1 x n2 inner products of unprojected DW  */
+    TDA_OP_SIMILARITY_EXACT = 2,    /* n1 x n2 inner products of unprojected DW  */
+    TDA_OP_NORM_PROJECTED = 3,      /* n1 squared norms of projected gradients   */
+    TDA_OP_NORM_EXACT = 4           /* n1 squared norms of unprojected DW        */
 } tda_op;
 
 /* One linear layer. seed and layer must be identical for every gradient that
@@ -215,6 +217,25 @@ tda_status tda_similarity_projected(const tda_layer_desc* L, tda_dtype dtype,
                                     const void* At, const void* Bt, int64_t n_t,
                                     float* S, int64_t ld_S, float beta, tda_route_id route,
                                     void* ws, size_t ws_bytes, void* stream);
+
+/* ---------------------------------------------------------------------------
+ * tda_norms -- squared Frobenius norms of per-example gradients, routed like
+ * the cross-Gram matrices (App. A.4: "for cross-Gram matrices and for
+ * per-example norms alike"); with tda_cosine they give LESS-style cosine
+ * scores. op TDA_OP_NORM_PROJECTED: ||Phi_i||^2 of the projected gradient
+ * (routes FACTORED, MATERIALIZE, GRAM on projected factors); op
+ * TDA_OP_NORM_EXACT: ||DW_i||_F^2 (routes MATERIALIZE, GRAM by Eq. 4 with
+ * both sides example i). AUTO asks tda_route. out: device fp32[N].
+ * ws >= tda_workspace_size(op, L, dtype, N, 0, route) (0 for exact GRAM).
+ * ------------------------------------------------------------------------- */
+tda_status tda_norms(tda_op op, const tda_layer_desc* L, tda_dtype dtype, const void* A, const void* B,
+                     int64_t N, float* out, tda_route_id route, void* ws, size_t ws_bytes, void* stream);
+
+/* tda_cosine -- S[q][i] <- S[q][i] / sqrt(nq[q] * nt[i]) in place, nq and nt
+ * squared norms (device fp32, e.g. from tda_norms); IEEE division semantics
+ * (a zero norm gives inf or NaN, visibly). */
+tda_status tda_cosine(float* S, int64_t n_q, int64_t n_t, int64_t ld_S, const float* nq, const float* nt,
+                      void* stream);
 
 /* ---------------------------------------------------------------------------
  * tda_precondition -- damped Fisher inverse on the query side (App. B.3: a

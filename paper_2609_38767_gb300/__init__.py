@@ -17,7 +17,7 @@ __all__ = [
     "LayerDesc", "TdaError", "load", "tda_proj_entries", "tda_workspace_size", "tda_project",
     "tda_project_engine", "tda_project_host_ws_min", "tda_project_host", "tda_noalloc_scratch_bytes",
     "tda_project_materialized_noalloc",
-    "tda_similarity_projected", "tda_similarity_exact", "tda_precondition_state_bytes", "tda_precondition",
+    "tda_similarity_projected", "tda_similarity_exact", "tda_norms", "tda_cosine", "tda_precondition_state_bytes", "tda_precondition",
     "tda_precondition_info", "tda_score", "tda_score_engine", "tda_topk", "tda_route", "tda_route_calibrate",
     "tda_route_set_model", "tda_device_status", "tda_selftest_bounded_wait", "tda_last_error", "tda_version", "tda_launch_count",
 ]
@@ -33,6 +33,7 @@ TDA_F32, TDA_BF16, TDA_F64 = 0, 1, 2
 TDA_PROJ_RADEMACHER, TDA_PROJ_IDENTITY = 0, 1
 TDA_ROUTE_AUTO, TDA_ROUTE_FACTORED, TDA_ROUTE_MATERIALIZE, TDA_ROUTE_GRAM = -1, 0, 1, 2
 TDA_OP_PROJECT, TDA_OP_SIMILARITY_PROJECTED, TDA_OP_SIMILARITY_EXACT = 0, 1, 2
+TDA_OP_NORM_PROJECTED, TDA_OP_NORM_EXACT = 3, 4
 TDA_PC_RESET, TDA_PC_FIT_ACCUM, TDA_PC_FACTOR, TDA_PC_APPLY = 0, 1, 2, 3
 TDA_CALIBRATE_WS_BYTES = 768 << 20
 _STATUS = {0: "TDA_OK", 1: "TDA_ERR_INVALID_ARG", 2: "TDA_ERR_UNSUPPORTED", 3: "TDA_ERR_WORKSPACE",
@@ -82,6 +83,8 @@ def load() -> ctypes.CDLL:
             "tda_noalloc_scratch_bytes": (SZ, []),
             "tda_project_materialized_noalloc": (I32, [LP, I32, P, P, I64, P, I64, P]),
             "tda_similarity_projected": (I32, [LP, I32, P, P, I64, P, P, I64, P, I64, F, I32, P, SZ, P]),
+            "tda_norms": (I32, [I32, LP, I32, P, P, I64, P, I32, P, SZ, P]),
+            "tda_cosine": (I32, [P, I64, I64, I64, P, P, P]),
             "tda_similarity_exact": (I32, [LP, I32, P, P, I64, P, P, I64, P, I64, F, I32, P, SZ, P]),
             "tda_precondition_state_bytes": (SZ, [I64, I32]),
             "tda_precondition": (I32, [I32, I32, I64, I32, P, P, I64, I64, I64, D, D, P, I64, I64, P, I64, P]),
@@ -182,6 +185,15 @@ def tda_similarity_projected(L, dtype, Aq, Bq, n_q, At, Bt, n_t, S, ld_S, beta=0
                              ws=None, ws_bytes=0, stream=None):
     _check(load().tda_similarity_projected(ctypes.byref(L), dtype, _ptr(Aq), _ptr(Bq), n_q, _ptr(At), _ptr(Bt),
                                            n_t, _ptr(S), ld_S, beta, route, _ptr(ws), ws_bytes, _stream(stream)))
+
+
+def tda_norms(op, L, dtype, A, B, N, out, route=TDA_ROUTE_AUTO, ws=None, ws_bytes=0, stream=None):
+    _check(load().tda_norms(op, ctypes.byref(L), dtype, _ptr(A), _ptr(B), N, _ptr(out), route, _ptr(ws), ws_bytes,
+                            _stream(stream)))
+
+
+def tda_cosine(S, n_q, n_t, ld_S, nq, nt, stream=None):
+    _check(load().tda_cosine(_ptr(S), n_q, n_t, ld_S, _ptr(nq), _ptr(nt), _stream(stream)))
 
 
 def tda_similarity_exact(L, dtype, Aq, Bq, n_q, At, Bt, n_t, S, ld_S, beta=0.0, route=TDA_ROUTE_AUTO,

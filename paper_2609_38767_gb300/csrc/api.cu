@@ -93,13 +93,27 @@ static RouteCounts route_counts(const tda_layer_desc& L, tda_op op, int64_t n1, 
         c.bytes[0] = (B1 + B2) * (factors + 4.0 * ka * kg);
         c.bytes[1] = (B1 + B2) * (factors + 8.0 * Ni * No);
         c.bytes[2] = (B1 + B2) * factors + B1 * B2 * 4.0 * T * (ka + kg);
-    } else {
+    } else if (op == TDA_OP_SIMILARITY_EXACT) {
         c.flops[0] = -1;
         c.flops[1] = (B1 + B2) * build + B1 * B2 * 2.0 * Ni * No;
         c.flops[2] = B1 * B2 * 2.0 * T * T * (Ni + No);
         c.bytes[0] = -1;
-        c.bytes[1] = (B1 + B2) * (factors + 4.0 * Ni * No) + B1 * B2 * 0.0;
+        c.bytes[1] = (B1 + B2) * (factors + 4.0 * Ni * No);
         c.bytes[2] = B1 * B2 * factors;
+    } else if (op == TDA_OP_NORM_PROJECTED) {
+        c.flops[0] = B1 * (proj + contract + 2.0 * ka * kg);
+        c.flops[1] = B1 * (build + dense + 2.0 * ka * kg);
+        c.flops[2] = B1 * (proj + 2.0 * T * T * (ka + kg));
+        c.bytes[0] = B1 * (factors + 8.0 * ka * kg);
+        c.bytes[1] = B1 * (factors + 8.0 * Ni * No);
+        c.bytes[2] = B1 * (factors + 8.0 * T * (ka + kg));
+    } else {
+        c.flops[0] = -1;
+        c.flops[1] = B1 * (build + 2.0 * Ni * No);
+        c.flops[2] = B1 * 2.0 * T * T * (Ni + No);
+        c.bytes[0] = -1;
+        c.bytes[1] = B1 * (factors + 8.0 * Ni * No);
+        c.bytes[2] = B1 * factors;
     }
     return c;
 }
@@ -189,9 +203,8 @@ tda_status tda_proj_entries(uint64_t seed, uint32_t layer, int32_t side, int32_t
 tda_status tda_route(const tda_layer_desc* L, tda_op op, int64_t n1, int64_t n2, tda_dtype dtype,
                      tda_route_id* chosen, double* cost_out) {
     g_msg[0] = 0;
-    if (op < TDA_OP_PROJECT || op > TDA_OP_SIMILARITY_EXACT)
-        return fail(TDA_ERR_INVALID_ARG, "bad op %d", (int)op);
-    tda_status st = validate_layer(L, op != TDA_OP_SIMILARITY_EXACT);
+    if (op < TDA_OP_PROJECT || op > TDA_OP_NORM_EXACT) return fail(TDA_ERR_INVALID_ARG, "bad op %d", (int)op);
+    tda_status st = validate_layer(L, op != TDA_OP_SIMILARITY_EXACT && op != TDA_OP_NORM_EXACT);
     if (st) return st;
     if (n1 < 0 || n2 < 0) return fail(TDA_ERR_INVALID_ARG, "negative batch size");
     if (!chosen) return fail(TDA_ERR_INVALID_ARG, "chosen is NULL");
@@ -210,13 +223,14 @@ tda_status tda_route_set_model(int32_t model) {
 }
 
 static size_t simproj_ws(const tda_layer_desc& L, int64_t n_q, int64_t chunk, tda_route_id route);
+static size_t norms_ws(const tda_layer_desc& L, tda_op op, int64_t chunk, tda_route_id route);
 
 tda_status tda_workspace_size(tda_op op, const tda_layer_desc* L, tda_dtype dtype, int64_t n1,
                               int64_t n2, tda_route_id route, size_t* bytes) {
     g_msg[0] = 0;
     if (!bytes) return fail(TDA_ERR_INVALID_ARG, "bytes is NULL");
     *bytes = 0;
-    tda_status st = validate_layer(L, op != TDA_OP_SIMILARITY_EXACT);
+    tda_status st = validate_layer(L, op != TDA_OP_SIMILARITY_EXACT && op != TDA_OP_NORM_EXACT);
     if (st) return st;
     if (route == TDA_ROUTE_AUTO) {
         st = tda_route(L, op, n1, n2, dtype, &route, nullptr);
@@ -232,6 +246,14 @@ tda_status tda_workspace_size(tda_op op, const tda_layer_desc* L, tda_dtype dtyp
     }
     if (op == TDA_OP_SIMILARITY_PROJECTED) {
         *bytes = simproj_ws(*L, n1, 1, route);
+        return TDA_OK;
+    }
+    if (op == TDA_OP_NORM_PROJECTED) {
+        *bytes = norms_ws(*L, op, 1, route);
+        return TDA_OK;
+    }
+    if (op == TDA_OP_NORM_EXACT) {
+        *bytes = norms_ws(*L, op, 1, route);
         return TDA_OK;
     }
     return fail(TDA_ERR_UNSUPPORTED, "no workspace query for op %d", (int)op);
@@ -392,6 +414,105 @@ tda_status tda_similarity_projected(const tda_layer_desc* L, tda_dtype dtype, co
             return st;
     }
     return TDA_OK;
+}
+
+// Workspace of tda_norms for `chunk` examples at a time.
+static size_t norms_ws(const tda_layer_desc& L, tda_op op, int64_t chunk, tda_route_id route) {
+    if (op == TDA_OP_NORM_EXACT) {
+        if (route == TDA_ROUTE_GRAM) return 0;
+        return sizeof(float) * (size_t)(L.d_out * L.d_in) * (size_t)chunk;
+    }
+    if (route == TDA_ROUTE_GRAM) return project_factors_bytes_per_example(L) * (size_t)chunk;
+    size_t b = sizeof(float) * (size_t)L.k_in * (size_t)L.k_out * (size_t)chunk;
+    if (route == TDA_ROUTE_MATERIALIZE) b += (materialize_ws_bytes_per_example(L) + 255) & ~(size_t)255;
+    return b;
+}
+
+tda_status tda_norms(tda_op op, const tda_layer_desc* L, tda_dtype dtype, const void* A, const void* B, int64_t N,
+                     float* out, tda_route_id route, void* ws, size_t ws_bytes, void* stream) {
+    g_msg[0] = 0;
+    if (op != TDA_OP_NORM_PROJECTED && op != TDA_OP_NORM_EXACT)
+        return fail(TDA_ERR_INVALID_ARG, "op must be TDA_OP_NORM_PROJECTED or TDA_OP_NORM_EXACT");
+    tda_status st = validate_layer(L, op == TDA_OP_NORM_PROJECTED);
+    if (st) return st;
+    if ((st = validate_factors(L, dtype, A, B, N, "tda_norms"))) return st;
+    if (N > 0 && !out) return fail(TDA_ERR_INVALID_ARG, "out is NULL");
+    if (route == TDA_ROUTE_AUTO) {
+        tda_route_id r;
+        if ((st = tda_route(L, op, N, 0, dtype, &r, nullptr))) return st;
+        route = r;
+    }
+    if (op == TDA_OP_NORM_EXACT && route == TDA_ROUTE_FACTORED)
+        return fail(TDA_ERR_UNSUPPORTED, "exact norms have no factored-projection route");
+    if (route != TDA_ROUTE_FACTORED && route != TDA_ROUTE_MATERIALIZE && route != TDA_ROUTE_GRAM)
+        return fail(TDA_ERR_INVALID_ARG, "bad route %d", (int)route);
+    cudaStream_t s = (cudaStream_t)stream;
+    if (N == 0) return TDA_OK;
+    if (L->T == 0) return cuda_check(cudaMemsetAsync(out, 0, sizeof(float) * (size_t)N, s), "zero norms");
+    if (op == TDA_OP_NORM_EXACT && route == TDA_ROUTE_GRAM)
+        return cuda_check(launch_gram_self(*L, dtype, A, B, N, L->d_in, L->d_out, 1.f, out, s), "norms (gram)");
+    const size_t need = norms_ws(*L, op, 1, route);
+    if (!ws || ws_bytes < need)
+        return fail(TDA_ERR_WORKSPACE, "tda_norms needs >= %zu bytes of ws, got %zu", need, ws_bytes);
+    if ((uintptr_t)ws & 255) return fail(TDA_ERR_INVALID_ARG, "ws must be 256-byte aligned");
+    const size_t el = dtype == TDA_F32 ? 4 : 2;
+    const size_t a_ex = (size_t)L->T * L->d_in * el, b_ex = (size_t)L->T * L->d_out * el;
+    if (op == TDA_OP_NORM_EXACT) {  // materialise DW per example, sum of squares
+        const int64_t gsz = L->d_out * L->d_in;
+        int64_t chunk = (int64_t)(ws_bytes / (sizeof(float) * (size_t)gsz));
+        if (chunk > N) chunk = N;
+        if (chunk > 65535) chunk = 65535;
+        for (int64_t i0 = 0; i0 < N; i0 += chunk) {
+            const int64_t c = (N - i0) < chunk ? (N - i0) : chunk;
+            if ((st = cuda_check(launch_materialize_G(*L, dtype, A, B, i0, c, (float*)ws, s), "materialise")))
+                return st;
+            if ((st = cuda_check(launch_row_sq_norms((const float*)ws, c, gsz, gsz, out + i0, s), "norms")))
+                return st;
+        }
+        return TDA_OK;
+    }
+    if (route == TDA_ROUTE_GRAM) {  // Eq. 4 on the projected factors of each example with itself
+        const size_t per = project_factors_bytes_per_example(*L);
+        int64_t chunk = (int64_t)(ws_bytes / per);
+        if (chunk > N) chunk = N;
+        if (chunk > 65535) chunk = 65535;
+        const float sc = projection_scale(*L);
+        for (int64_t i0 = 0; i0 < N; i0 += chunk) {
+            const int64_t c = (N - i0) < chunk ? (N - i0) : chunk;
+            float* Y = (float*)ws;
+            if ((st = cuda_check(launch_project_factors(*L, dtype, A, B, i0, c, Y, s), "project factors"))) return st;
+            if ((st = cuda_check(launch_gram_self(*L, TDA_F32, Y, Y + c * L->T * L->k_in, c, L->k_in, L->k_out,
+                                                  sc * sc, out + i0, s),
+                                 "norms (projected gram)")))
+                return st;
+        }
+        return TDA_OK;
+    }
+    // routes a and b: features in ws, then row sums of squares
+    const int64_t D = (int64_t)L->k_in * L->k_out;
+    // [materialisation scratch, 256-aligned | features of `chunk` examples]
+    const size_t mat =
+        route == TDA_ROUTE_MATERIALIZE ? (materialize_ws_bytes_per_example(*L) + 255) & ~(size_t)255 : 0;
+    int64_t chunk = (int64_t)((ws_bytes - mat) / (sizeof(float) * (size_t)D));
+    if (chunk > N) chunk = N;
+    void* mws = mat ? ws : nullptr;
+    float* F = (float*)((char*)ws + mat);
+    for (int64_t i0 = 0; i0 < N; i0 += chunk) {
+        const int64_t c = (N - i0) < chunk ? (N - i0) : chunk;
+        if ((st = tda_project(L, dtype, (const char*)A + (size_t)i0 * a_ex, (const char*)B + (size_t)i0 * b_ex, c, F, D,
+                              route, mws, mat, stream)))
+            return st;
+        if ((st = cuda_check(launch_row_sq_norms(F, c, D, D, out + i0, s), "norms"))) return st;
+    }
+    return TDA_OK;
+}
+
+tda_status tda_cosine(float* S, int64_t n_q, int64_t n_t, int64_t ld_S, const float* nq, const float* nt,
+                      void* stream) {
+    g_msg[0] = 0;
+    if (n_q < 0 || n_t < 0 || ld_S < n_t) return fail(TDA_ERR_INVALID_ARG, "bad sizes");
+    if (n_q > 0 && n_t > 0 && (!S || !nq || !nt)) return fail(TDA_ERR_INVALID_ARG, "NULL argument");
+    return cuda_check(launch_cosine(S, n_q, n_t, ld_S, nq, nt, (cudaStream_t)stream), "cosine");
 }
 
 size_t tda_precondition_state_bytes(int64_t D, tda_dtype state_dtype) {

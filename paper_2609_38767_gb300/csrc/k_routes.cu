@@ -170,12 +170,12 @@ template <typename T>
 __global__ void __launch_bounds__(kTh)
 gram_kernel(const T* __restrict__ Aq, const T* __restrict__ Bq, const T* __restrict__ At,
             const T* __restrict__ Bt, int64_t Tn, int64_t d_in, int64_t d_out,
-            float* __restrict__ S, int64_t ld_S, float beta, float alpha) {
+            float* __restrict__ S, int64_t ld_S, float beta, float alpha, int self_pairs) {
     constexpr int TT = 16, KC = 64;
     __shared__ float Xq[TT][KC + 1];
     __shared__ float Xi[TT][KC + 1];
     __shared__ float red[kTh];
-    const int64_t i = blockIdx.x, q = blockIdx.y;
+    const int64_t i = blockIdx.x, q = self_pairs ? blockIdx.x : blockIdx.y;  // self: <DW_i, DW_i>
     const int tid = threadIdx.x, tl = tid / TT, sl = tid % TT;
     float total = 0.f;
     for (int64_t t0 = 0; t0 < Tn; t0 += TT) {
@@ -349,10 +349,10 @@ cudaError_t launch_similarity_gram(const tda_layer_desc& L, tda_dtype dt, const 
     if (dt == TDA_BF16)
         gram_kernel<__nv_bfloat16><<<grid, kTh, 0, s>>>(
             (const __nv_bfloat16*)Aq, (const __nv_bfloat16*)Bq, (const __nv_bfloat16*)At,
-            (const __nv_bfloat16*)Bt, L.T, L.d_in, L.d_out, S, ld_S, beta, 1.f);
+            (const __nv_bfloat16*)Bt, L.T, L.d_in, L.d_out, S, ld_S, beta, 1.f, 0);
     else
         gram_kernel<float><<<grid, kTh, 0, s>>>((const float*)Aq, (const float*)Bq, (const float*)At,
-                                                (const float*)Bt, L.T, L.d_in, L.d_out, S, ld_S, beta, 1.f);
+                                                (const float*)Bt, L.T, L.d_in, L.d_out, S, ld_S, beta, 1.f, 0);
     return cudaGetLastError();
 }
 
@@ -390,7 +390,79 @@ cudaError_t launch_gram_projected(const tda_layer_desc& L, const float* Yq, int6
     dim3 grid((unsigned)n_t, (unsigned)n_q);
     note_launches(1);
     gram_kernel<float><<<grid, kTh, 0, s>>>(Yq, Yq + n_q * L.T * L.k_in, Yt, Yt + n_t * L.T * L.k_in, L.T, L.k_in,
-                                            L.k_out, S, ld_S, beta, sc * sc);
+                                            L.k_out, S, ld_S, beta, sc * sc, 0);
+    return cudaGetLastError();
+}
+
+// ---------------------------------------------------------------- norms
+namespace {
+// out[r] = sum_f X[r][f]^2 (one warp per row)
+__global__ void row_sq_norms_kernel(const float* __restrict__ X, int64_t n, int64_t D, int64_t ld,
+                                    float* __restrict__ out) {
+    const int64_t r = (int64_t)blockIdx.x * (blockDim.x / 32) + threadIdx.x / 32;
+    const int lane = threadIdx.x & 31;
+    if (r >= n) return;
+    float s = 0.f;
+    for (int64_t f = lane; f < D; f += 32) {
+        const float v = X[r * ld + f];
+        s = fmaf(v, v, s);
+    }
+    for (int o = 16; o > 0; o >>= 1) s += __shfl_xor_sync(0xffffffffu, s, o);
+    if (lane == 0) out[r] = s;
+}
+// C[q][i] = S[q][i] / sqrt(nq[q] * nt[i])
+__global__ void cosine_kernel(float* __restrict__ S, int64_t n_q, int64_t n_t, int64_t ld_S,
+                              const float* __restrict__ nq, const float* __restrict__ nt) {
+    const int64_t total = n_q * n_t;
+    for (int64_t e = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; e < total;
+         e += (int64_t)gridDim.x * blockDim.x) {
+        const int64_t q = e / n_t, i = e - q * n_t;
+        S[q * ld_S + i] = S[q * ld_S + i] / sqrtf(nq[q] * nt[i]);
+    }
+}
+}  // namespace
+
+cudaError_t launch_row_sq_norms(const float* X, int64_t n, int64_t D, int64_t ld, float* out, cudaStream_t s) {
+    if (n == 0) return cudaSuccess;
+    note_launches(1);
+    row_sq_norms_kernel<<<(unsigned)((n + 7) / 8), 256, 0, s>>>(X, n, D, ld, out);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_cosine(float* S, int64_t n_q, int64_t n_t, int64_t ld_S, const float* nq, const float* nt,
+                          cudaStream_t s) {
+    if (n_q == 0 || n_t == 0) return cudaSuccess;
+    int64_t blocks = (n_q * n_t + 255) / 256;
+    if (blocks > 152 * 32) blocks = 152 * 32;
+    note_launches(1);
+    cosine_kernel<<<(unsigned)blocks, 256, 0, s>>>(S, n_q, n_t, ld_S, nq, nt);
+    return cudaGetLastError();
+}
+
+// ||DW_i||^2 for i in [0, n) by Eq. 4 with both sides example i (unprojected,
+// or on projected factors Y laid out as in launch_project_factors with alpha =
+// scale^2).
+cudaError_t launch_gram_self(const tda_layer_desc& L, tda_dtype dt, const void* A, const void* B, int64_t n,
+                             int64_t d_in, int64_t d_out, float alpha, float* out, cudaStream_t s) {
+    if (n == 0) return cudaSuccess;
+    note_launches(1);
+    if (dt == TDA_BF16)
+        gram_kernel<__nv_bfloat16><<<(unsigned)n, kTh, 0, s>>>((const __nv_bfloat16*)A, (const __nv_bfloat16*)B,
+                                                               (const __nv_bfloat16*)A, (const __nv_bfloat16*)B, L.T,
+                                                               d_in, d_out, out, 0, 0.f, alpha, 1);
+    else
+        gram_kernel<float><<<(unsigned)n, kTh, 0, s>>>((const float*)A, (const float*)B, (const float*)A,
+                                                       (const float*)B, L.T, d_in, d_out, out, 0, 0.f, alpha, 1);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_materialize_G(const tda_layer_desc& L, tda_dtype dt, const void* A, const void* B, int64_t e0,
+                                 int64_t n, float* G, cudaStream_t s) {
+    if (n == 0) return cudaSuccess;
+    if (dt == TDA_BF16)
+        launch_materialize<__nv_bfloat16>(A, B, e0, n, L, G, s);
+    else
+        launch_materialize<float>(A, B, e0, n, L, G, s);
     return cudaGetLastError();
 }
 

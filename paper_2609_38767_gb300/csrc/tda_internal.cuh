@@ -99,6 +99,15 @@ cudaError_t launch_project_factors(const tda_layer_desc& L, tda_dtype dt, const 
 cudaError_t launch_gram_projected(const tda_layer_desc& L, const float* Yq, int64_t n_q, const float* Yt,
                                   int64_t n_t, float* S, int64_t ld_S, float beta, cudaStream_t s);
 
+// Norms and cosine.
+cudaError_t launch_materialize_G(const tda_layer_desc& L, tda_dtype dt, const void* A, const void* B, int64_t e0,
+                                 int64_t n, float* G, cudaStream_t s);
+cudaError_t launch_row_sq_norms(const float* X, int64_t n, int64_t D, int64_t ld, float* out, cudaStream_t s);
+cudaError_t launch_cosine(float* S, int64_t n_q, int64_t n_t, int64_t ld_S, const float* nq, const float* nt,
+                          cudaStream_t s);
+cudaError_t launch_gram_self(const tda_layer_desc& L, tda_dtype dt, const void* A, const void* B, int64_t n,
+                             int64_t d_in, int64_t d_out, float alpha, float* out, cudaStream_t s);
+
 // Preconditioner, n_layers layers of D features each (layer l's columns at
 // offset l*D of every feature row).
 int64_t precondition_apply_max_d(tda_dtype sdt);

@@ -98,7 +98,8 @@ SHAPES = [
 
 
 @pytest.mark.parametrize("shape", SHAPES)
-@pytest.mark.parametrize("op", [tda.TDA_OP_PROJECT, tda.TDA_OP_SIMILARITY_PROJECTED, tda.TDA_OP_SIMILARITY_EXACT])
+@pytest.mark.parametrize("op", [tda.TDA_OP_PROJECT, tda.TDA_OP_SIMILARITY_PROJECTED, tda.TDA_OP_SIMILARITY_EXACT,
+                                tda.TDA_OP_NORM_PROJECTED, tda.TDA_OP_NORM_EXACT])
 def test_route_flop_model_matches_oracle(libs, orc, shape, op):
     n1, n2, T, di, do, ki, ko = shape
     L = tda.LayerDesc(di, do, T, ki, ko)
@@ -123,3 +124,26 @@ def test_workspace_sizes(libs):
                                   tda.TDA_ROUTE_MATERIALIZE) == 4 * D * 4 + 4 * (128 * 256 + 128 * 16)
     assert tda.tda_workspace_size(tda.TDA_OP_SIMILARITY_PROJECTED, L, tda.TDA_F32, 3, 9,
                                   tda.TDA_ROUTE_GRAM) == 4 * 32 * (16 + 16) * 4
+    # norms: one example at a time per chunk
+    assert tda.tda_workspace_size(tda.TDA_OP_NORM_PROJECTED, L, tda.TDA_F32, 3, 0, tda.TDA_ROUTE_FACTORED) == 4 * D
+    assert tda.tda_workspace_size(tda.TDA_OP_NORM_PROJECTED, L, tda.TDA_F32, 3, 0,
+                                  tda.TDA_ROUTE_MATERIALIZE) == 4 * D + 4 * (128 * 256 + 128 * 16)
+    assert tda.tda_workspace_size(tda.TDA_OP_NORM_PROJECTED, L, tda.TDA_F32, 3, 0,
+                                  tda.TDA_ROUTE_GRAM) == 4 * 32 * (16 + 16)
+    assert tda.tda_workspace_size(tda.TDA_OP_NORM_EXACT, L, tda.TDA_F32, 3, 0,
+                                  tda.TDA_ROUTE_MATERIALIZE) == 4 * 128 * 256
+    assert tda.tda_workspace_size(tda.TDA_OP_NORM_EXACT, L, tda.TDA_F32, 3, 0, tda.TDA_ROUTE_GRAM) == 0
+
+
+def test_norm_entry_validation(libs):
+    L = tda.LayerDesc(64, 64, 8, 16, 16)
+    s = 0
+    assert _err(tda.tda_norms, tda.TDA_OP_PROJECT, L, tda.TDA_F32, 16, 16, 4, 16, stream=s) \
+        == tda.TDA_ERR_INVALID_ARG
+    assert _err(tda.tda_norms, tda.TDA_OP_NORM_EXACT, L, tda.TDA_F32, 16, 16, 4, 16,
+                route=tda.TDA_ROUTE_FACTORED, stream=s) == tda.TDA_ERR_UNSUPPORTED
+    assert _err(tda.tda_norms, tda.TDA_OP_NORM_PROJECTED, L, tda.TDA_F32, 16, 16, 4, 16,
+                route=tda.TDA_ROUTE_FACTORED, stream=s) == tda.TDA_ERR_WORKSPACE
+    assert _err(tda.tda_norms, tda.TDA_OP_NORM_PROJECTED, L, tda.TDA_F32, 16, 16, 4, None, stream=s) \
+        == tda.TDA_ERR_INVALID_ARG
+    assert _err(tda.tda_cosine, 16, 2, 8, 4, 16, 16, stream=s) == tda.TDA_ERR_INVALID_ARG

@@ -403,3 +403,65 @@ def test_score_tensor_core_matches_oracle(dev, orc, nq, nt, D, beta):
     tda.tda_device_status()
     ref = orc.score(Q, P) + beta * S0.astype(np.float64)
     assert rel_fro(S.cpu().numpy(), ref) <= 1e-5
+
+
+@pytest.mark.gpu
+@pytest.mark.parametrize("dtype", ["f32", "bf16"])
+@pytest.mark.parametrize("op,route", [("proj", tda.TDA_ROUTE_FACTORED), ("proj", tda.TDA_ROUTE_MATERIALIZE),
+                                      ("proj", tda.TDA_ROUTE_GRAM), ("exact", tda.TDA_ROUTE_MATERIALIZE),
+                                      ("exact", tda.TDA_ROUTE_GRAM), ("proj", tda.TDA_ROUTE_AUTO)])
+def test_norms_and_cosine_match_oracle(dev, orc, dtype, op, route):
+    # per-example squared norms routed like Gram matrices (App. A.4), then cosine scores
+    n, nq, T, di, do, k = 9, 3, 29, 64, 40, 16
+    A, B = make_factors(n, T, di, do, dtype, stream=21)
+    Aq, Bq = make_factors(nq, T, di, do, dtype, stream=21, query=True)
+    L = tda.LayerDesc(di, do, T, k, k, seed=6, layer=1)
+    opc = tda.TDA_OP_NORM_PROJECTED if op == "proj" else tda.TDA_OP_NORM_EXACT
+    r = route if route != tda.TDA_ROUTE_AUTO else tda.tda_route(L, opc, n, 0, TD[dtype])[0]
+    wsb = tda.tda_workspace_size(opc, L, TD[dtype], n, 0, r) * 3 + 256
+    ws = torch.empty(max(wsb, 256), dtype=torch.uint8, device=dev)
+    out = torch.full((n,), -1.0, device=dev)
+    tda.tda_norms(opc, L, TD[dtype], to_dev(A, dtype, dev), to_dev(B, dtype, dev), n, out, route, ws, wsb)
+    tda.tda_device_status()
+    A64, B64 = synth.to_f64(A, dtype), synth.to_f64(B, dtype)
+    if op == "proj":
+        ref = (orc.project(A64, B64, k, k, 6, 1) ** 2).reshape(n, -1).sum(1)
+    else:
+        ref = orc.sq_norms(A64, B64, "materialized")
+    tol = 1e-5 if dtype == "f32" else 2e-2
+    np.testing.assert_allclose(out.cpu().numpy(), ref, rtol=tol)
+    if op == "proj":
+        # cosine of projected query/train features from device norms and scores
+        nqd = torch.empty(nq, device=dev)
+        tda.tda_norms(opc, L, TD[dtype], to_dev(Aq, dtype, dev), to_dev(Bq, dtype, dev), nq, nqd, route, ws, wsb)
+        fq = orc.project(synth.to_f64(Aq, dtype), synth.to_f64(Bq, dtype), k, k, 6, 1)
+        ft = orc.project(A64, B64, k, k, 6, 1)
+        S0 = orc.score(fq, ft)
+        S = torch.from_numpy(S0.astype(np.float32)).to(dev)
+        tda.tda_cosine(S, nq, n, n, nqd, out)
+        tda.tda_device_status()
+        C = orc.cosine(S0, (fq ** 2).reshape(nq, -1).sum(1), ref)
+        assert rel_fro(S.cpu().numpy(), C) <= (1e-5 if dtype == "f32" else 2e-2)
+        assert np.abs(S.cpu().numpy()).max() <= 1 + 1e-5
+
+
+@pytest.mark.gpu
+def test_norms_edge_cases(dev, orc):
+    # empty batch, T = 0 (zero gradients), a workspace that holds one example at a time
+    L = tda.LayerDesc(32, 32, 0, 8, 8)
+    out = torch.full((4,), 7.0, device=dev)
+    z = torch.empty(16, device=dev)
+    tda.tda_norms(tda.TDA_OP_NORM_EXACT, L, tda.TDA_F32, z, z, 4, out, tda.TDA_ROUTE_GRAM)
+    tda.tda_norms(tda.TDA_OP_NORM_PROJECTED, L, tda.TDA_F32, z, z, 0, out, tda.TDA_ROUTE_FACTORED)
+    tda.tda_device_status()
+    assert (out.cpu() == 0).all()
+    n, T, di, do = 5, 3, 24, 16
+    A, B = make_factors(n, T, di, do, "f32", stream=22)
+    L = tda.LayerDesc(di, do, T, 8, 8)
+    wsb = tda.tda_workspace_size(tda.TDA_OP_NORM_EXACT, L, tda.TDA_F32, n, 0, tda.TDA_ROUTE_MATERIALIZE)
+    ws = torch.empty(wsb, dtype=torch.uint8, device=dev)
+    out = torch.empty(n, device=dev)
+    tda.tda_norms(tda.TDA_OP_NORM_EXACT, L, tda.TDA_F32, to_dev(A, "f32", dev), to_dev(B, "f32", dev), n, out,
+                  tda.TDA_ROUTE_MATERIALIZE, ws, wsb)
+    tda.tda_device_status()
+    np.testing.assert_allclose(out.cpu().numpy(), orc.sq_norms(A, B, "gram"), rtol=1e-5)
