@@ -44,9 +44,19 @@ METRIC = "train examples attributed/sec (project+score)"
 # linear (profiles/tc_projection_q608.md): measured bytes over algorithmic bytes.
 # Launches of other linears are scaled by their algorithmic bytes (traffic is
 # one read of every factor byte, so it grows in proportion). Valid only for the
-# kernel source it was measured on; any change makes the bench report null.
-TRAFFIC_RATIO = 1.0011866
-TRAFFIC_KERNEL_SHA256 = "087a05225e94f716b8f93767e3f2054d12d9654fcd132411b2bc97752a13bb69"
+# kernel source it was measured on (the kernel file and its PTX helper header);
+# any change makes the bench report null.
+TRAFFIC_RATIO = 1.0012034
+TRAFFIC_KERNEL_SHA256 = "b4f57a1af080d252db6404531c012344fbdf83c022585a542317c2fbe29ac851"
+
+
+def projection_kernel_sha256():
+    import hashlib
+    h = hashlib.sha256()
+    for name in ("k_project_tc.cu", "tc_ptx.cuh"):
+        with open(os.path.join(ROOT, "paper_2609_38767_gb300", "csrc", name), "rb") as f:
+            h.update(f.read())
+    return h.hexdigest()
 
 
 def parse_args():
@@ -358,9 +368,7 @@ def main():
     hbm = float(peaks.get("hbm_gbs", 6800.0))
     achieved = proj_bytes / (proj_ms * 1e-3) / 1e9
     engines = sorted({tda.tda_project_engine(L, tda.TDA_BF16, At[li], Bt[li]) for li, L in enumerate(layers)})
-    import hashlib
-    with open(os.path.join(ROOT, "paper_2609_38767_gb300", "csrc", "k_project_tc.cu"), "rb") as f:
-        same_kernel = hashlib.sha256(f.read()).hexdigest() == TRAFFIC_KERNEL_SHA256
+    same_kernel = projection_kernel_sha256() == TRAFFIC_KERNEL_SHA256
     per_launch = proj_bytes / max(len(ev), 1)
     roofline = {"bound": "hbm", "kernel": "factored projection (train, 7 linears)",
                 "engine": "tcgen05" if engines == [1] else ("cuda-core" if engines == [0] else "mixed"), "achieved": achieved,
