@@ -66,6 +66,12 @@ def _load():
             "oracle_damping": (ctypes.c_double, [I64, D, ctypes.c_double, ctypes.c_double]),
             "oracle_cholesky": (I32, [I64, D]),
             "oracle_precondition": (I32, [I64, D, ctypes.c_double, I64, D, D]),
+            "oracle_kfac_covariances": (None, [I64, I64, I64, I64, I64, I64, U64, U32, I32, D, D, D, D]),
+            "oracle_sym_eig": (I32, [I64, D, D, D]),
+            "oracle_kfac_eigenvalues": (None, [I64, I64, D, D, D]),
+            "oracle_ekfac_eigenvalues": (None, [I64, I64, I64, D, D, D, D]),
+            "oracle_kfac_damping": (ctypes.c_double, [I64, I64, D, ctypes.c_double, ctypes.c_double]),
+            "oracle_kfac_precondition": (None, [I64, I64, D, D, D, ctypes.c_double, I64, D, D]),
             "oracle_score": (None, [I64, I64, I64, D, D, D]),
             "oracle_topk": (None, [I64, I64, D, I32, ctypes.POINTER(I32), D]),
             "oracle_route_costs": (I32, [I32, I64, I64, I64, I64, I64, I64, I64, D]),
@@ -208,6 +214,57 @@ def precondition(F, lam: float, Q) -> np.ndarray:
     st = int(_load().oracle_precondition(D, _p(F), lam, Q.shape[0], _p(Q), _p(out)))
     if st != 0:
         raise np.linalg.LinAlgError(f"F + lambda I not positive definite (minor {st})")
+    return out
+
+
+# ---------------------------------------------------------------- K-FAC / EK-FAC
+def kfac_covariances(A, B, k_in: int, k_out: int, seed: int, layer: int, kind: int = 0):
+    """A (N,T,d_in), B (N,T,d_out) -> (Ca (k_in,k_in), Cg (k_out,k_out)), token-averaged."""
+    A, B = _f64(A), _f64(B)
+    N, T, d_in = A.shape
+    d_out = B.shape[2]
+    Ca, Cg = np.empty((k_in, k_in)), np.empty((k_out, k_out))
+    _load().oracle_kfac_covariances(N, T, d_in, d_out, k_in, k_out, seed, layer, kind, _p(A), _p(B),
+                                    _p(Ca), _p(Cg))
+    return Ca, Cg
+
+
+def sym_eig(C):
+    """-> (w ascending, U with eigenvectors in columns, sweeps)."""
+    C = _f64(C)
+    n = C.shape[0]
+    w, U = np.empty(n), np.empty((n, n))
+    sweeps = int(_load().oracle_sym_eig(n, _p(C), _p(w), _p(U)))
+    return w, U, sweeps
+
+
+def kfac_eigenvalues(wa, wg) -> np.ndarray:
+    wa, wg = _f64(wa), _f64(wg)
+    Lam = np.empty((wg.size, wa.size))
+    _load().oracle_kfac_eigenvalues(wa.size, wg.size, _p(wa), _p(wg), _p(Lam))
+    return Lam
+
+
+def ekfac_eigenvalues(phi, Ua, Ug) -> np.ndarray:
+    phi, Ua, Ug = _f64(phi), _f64(Ua), _f64(Ug)
+    k_in, k_out = Ua.shape[0], Ug.shape[0]
+    N = phi.shape[0]
+    Lam = np.empty((k_out, k_in))
+    _load().oracle_ekfac_eigenvalues(N, k_in, k_out, _p(phi), _p(Ua), _p(Ug), _p(Lam))
+    return Lam
+
+
+def kfac_damping(Lam, lambda_abs: float, lambda_rel: float) -> float:
+    Lam = _f64(Lam)
+    return float(_load().oracle_kfac_damping(Lam.shape[1], Lam.shape[0], _p(Lam), lambda_abs, lambda_rel))
+
+
+def kfac_precondition(Ua, Ug, Lam, lam: float, Q) -> np.ndarray:
+    Ua, Ug, Lam, Q = _f64(Ua), _f64(Ug), _f64(Lam), _f64(Q)
+    k_in, k_out = Ua.shape[0], Ug.shape[0]
+    Q = Q.reshape(-1, k_out * k_in)
+    out = np.empty_like(Q)
+    _load().oracle_kfac_precondition(k_in, k_out, _p(Ua), _p(Ug), _p(Lam), lam, Q.shape[0], _p(Q), _p(out))
     return out
 
 

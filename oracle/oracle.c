@@ -353,6 +353,210 @@ int32_t oracle_precondition(int64_t D, const double* F, double lambda,
 }
 
 /* ------------------------------------------------------------------------ */
+/* Kronecker-factored curvature on projected factors                        */
+/* ------------------------------------------------------------------------ */
+
+void oracle_kfac_covariances(int64_t N, int64_t T, int64_t d_in, int64_t d_out,
+                             int64_t k_in, int64_t k_out, uint64_t seed, uint32_t layer,
+                             int32_t kind, const double* A, const double* B,
+                             double* Ca, double* Cg) {
+    double* P_in = (double*)malloc(sizeof(double) * (size_t)(d_in * k_in));
+    double* P_out = (double*)malloc(sizeof(double) * (size_t)(d_out * k_out));
+    oracle_proj_matrix(seed, layer, 0, kind, d_in, k_in, P_in);
+    oracle_proj_matrix(seed, layer, 1, kind, d_out, k_out, P_out);
+    /* per-example sums first (examples in parallel), then their sum in example order */
+    double* pa = (double*)calloc((size_t)(N > 0 ? N : 1) * (size_t)(k_in * k_in), sizeof(double));
+    double* pg = (double*)calloc((size_t)(N > 0 ? N : 1) * (size_t)(k_out * k_out), sizeof(double));
+#ifdef _OPENMP
+#pragma omp parallel for schedule(dynamic, 1) num_threads(g_threads)
+#endif
+    for (int64_t n = 0; n < N; ++n) {
+        const double* An = A + n * T * d_in;
+        const double* Bn = B + n * T * d_out;
+        double* at = (double*)malloc(sizeof(double) * (size_t)k_in);
+        double* gt = (double*)malloc(sizeof(double) * (size_t)k_out);
+        for (int64_t t = 0; t < T; ++t) {
+            for (int64_t j = 0; j < k_in; ++j) {
+                double s = 0.0;
+                for (int64_t c = 0; c < d_in; ++c) s += An[t * d_in + c] * P_in[c * k_in + j];
+                at[j] = s;
+            }
+            for (int64_t i = 0; i < k_out; ++i) {
+                double s = 0.0;
+                for (int64_t r = 0; r < d_out; ++r) s += Bn[t * d_out + r] * P_out[r * k_out + i];
+                gt[i] = s;
+            }
+            for (int64_t j = 0; j < k_in; ++j)
+                for (int64_t j2 = 0; j2 < k_in; ++j2) pa[n * k_in * k_in + j * k_in + j2] += at[j] * at[j2];
+            for (int64_t i = 0; i < k_out; ++i)
+                for (int64_t i2 = 0; i2 < k_out; ++i2) pg[n * k_out * k_out + i * k_out + i2] += gt[i] * gt[i2];
+        }
+        free(at);
+        free(gt);
+    }
+    const double M = (double)N * (double)T;
+    for (int64_t e = 0; e < k_in * k_in; ++e) {
+        double s = 0.0;
+        for (int64_t n = 0; n < N; ++n) s += pa[n * k_in * k_in + e];
+        Ca[e] = M > 0 ? s / M : 0.0;
+    }
+    for (int64_t e = 0; e < k_out * k_out; ++e) {
+        double s = 0.0;
+        for (int64_t n = 0; n < N; ++n) s += pg[n * k_out * k_out + e];
+        Cg[e] = M > 0 ? s / M : 0.0;
+    }
+    free(pa);
+    free(pg);
+    free(P_in);
+    free(P_out);
+}
+
+/* Cyclic Jacobi: sweep the pairs (p, q), p < q, in row order; each rotation
+ * J(p, q, theta) zeroes the (p, q) entry of A <- J^T A J, and V <- V J
+ * accumulates the eigenvectors. Stop once the off-diagonal Frobenius norm is
+ * at most 1e-15 of the matrix's. */
+int32_t oracle_sym_eig(int64_t n, const double* C, double* w, double* U) {
+    double* A = (double*)malloc(sizeof(double) * (size_t)(n * n > 0 ? n * n : 1));
+    memcpy(A, C, sizeof(double) * (size_t)(n * n));
+    for (int64_t i = 0; i < n; ++i)
+        for (int64_t j = 0; j < n; ++j) U[i * n + j] = i == j ? 1.0 : 0.0;
+    double fro = 0.0;
+    for (int64_t e = 0; e < n * n; ++e) fro += A[e] * A[e];
+    int32_t sweeps = -1;
+    for (int32_t sweep = 0; sweep <= 100; ++sweep) {
+        double off = 0.0;
+        for (int64_t i = 0; i < n; ++i)
+            for (int64_t j = 0; j < n; ++j)
+                if (i != j) off += A[i * n + j] * A[i * n + j];
+        if (off <= 1e-30 * fro) {
+            sweeps = sweep;
+            break;
+        }
+        if (sweep == 100) break;
+        for (int64_t p = 0; p < n - 1; ++p)
+            for (int64_t q = p + 1; q < n; ++q) {
+                const double apq = A[p * n + q];
+                if (apq == 0.0) continue;
+                /* tan(theta) as the smaller root of t^2 + 2 tau t - 1 = 0 */
+                const double tau = (A[q * n + q] - A[p * n + p]) / (2.0 * apq);
+                const double t = (tau >= 0 ? 1.0 : -1.0) / (fabs(tau) + sqrt(1.0 + tau * tau));
+                const double c = 1.0 / sqrt(1.0 + t * t), s = t * c;
+                for (int64_t k = 0; k < n; ++k) { /* A <- A J (columns p, q) */
+                    const double akp = A[k * n + p], akq = A[k * n + q];
+                    A[k * n + p] = c * akp - s * akq;
+                    A[k * n + q] = s * akp + c * akq;
+                }
+                for (int64_t k = 0; k < n; ++k) { /* A <- J^T A (rows p, q) */
+                    const double apk = A[p * n + k], aqk = A[q * n + k];
+                    A[p * n + k] = c * apk - s * aqk;
+                    A[q * n + k] = s * apk + c * aqk;
+                }
+                for (int64_t k = 0; k < n; ++k) { /* V <- V J */
+                    const double vkp = U[k * n + p], vkq = U[k * n + q];
+                    U[k * n + p] = c * vkp - s * vkq;
+                    U[k * n + q] = s * vkp + c * vkq;
+                }
+            }
+    }
+    /* sort ascending (selection sort), permuting eigenvector columns along */
+    for (int64_t i = 0; i < n; ++i) w[i] = A[i * n + i];
+    for (int64_t i = 0; i < n; ++i) {
+        int64_t m = i;
+        for (int64_t j = i + 1; j < n; ++j)
+            if (w[j] < w[m]) m = j;
+        if (m != i) {
+            const double tw = w[i];
+            w[i] = w[m];
+            w[m] = tw;
+            for (int64_t k = 0; k < n; ++k) {
+                const double tu = U[k * n + i];
+                U[k * n + i] = U[k * n + m];
+                U[k * n + m] = tu;
+            }
+        }
+    }
+    free(A);
+    return sweeps;
+}
+
+void oracle_kfac_eigenvalues(int64_t k_in, int64_t k_out, const double* wa, const double* wg,
+                             double* Lam) {
+    for (int64_t r = 0; r < k_out; ++r)
+        for (int64_t c = 0; c < k_in; ++c) Lam[r * k_in + c] = wg[r] * wa[c];
+}
+
+/* X = Ug^T V Ua for one k_out x k_in matrix V */
+static void to_eigenbasis(int64_t k_in, int64_t k_out, const double* Ua, const double* Ug,
+                          const double* V, double* X) {
+    double* Y = (double*)malloc(sizeof(double) * (size_t)(k_out * k_in));
+    for (int64_t r = 0; r < k_out; ++r) /* Y = V Ua */
+        for (int64_t c = 0; c < k_in; ++c) {
+            double s = 0.0;
+            for (int64_t j = 0; j < k_in; ++j) s += V[r * k_in + j] * Ua[j * k_in + c];
+            Y[r * k_in + c] = s;
+        }
+    for (int64_t r = 0; r < k_out; ++r) /* X = Ug^T Y */
+        for (int64_t c = 0; c < k_in; ++c) {
+            double s = 0.0;
+            for (int64_t i = 0; i < k_out; ++i) s += Ug[i * k_out + r] * Y[i * k_in + c];
+            X[r * k_in + c] = s;
+        }
+    free(Y);
+}
+
+void oracle_ekfac_eigenvalues(int64_t N, int64_t k_in, int64_t k_out, const double* phi,
+                              const double* Ua, const double* Ug, double* Lam) {
+    const int64_t D = k_in * k_out;
+    double* X = (double*)malloc(sizeof(double) * (size_t)((N > 0 ? N : 1) * D));
+#ifdef _OPENMP
+#pragma omp parallel for schedule(dynamic, 1) num_threads(g_threads)
+#endif
+    for (int64_t n = 0; n < N; ++n) to_eigenbasis(k_in, k_out, Ua, Ug, phi + n * D, X + n * D);
+    for (int64_t e = 0; e < D; ++e) {
+        double s = 0.0;
+        for (int64_t n = 0; n < N; ++n) s += X[n * D + e] * X[n * D + e];
+        Lam[e] = N > 0 ? s / (double)N : 0.0;
+    }
+    free(X);
+}
+
+double oracle_kfac_damping(int64_t k_in, int64_t k_out, const double* Lam, double lambda_abs,
+                           double lambda_rel) {
+    double s = 0.0;
+    for (int64_t e = 0; e < k_in * k_out; ++e) s += Lam[e];
+    return lambda_abs + lambda_rel * s / (double)(k_in * k_out);
+}
+
+void oracle_kfac_precondition(int64_t k_in, int64_t k_out, const double* Ua, const double* Ug,
+                              const double* Lam, double lambda, int64_t n_q, const double* Q,
+                              double* Qhat) {
+    const int64_t D = k_in * k_out;
+#ifdef _OPENMP
+#pragma omp parallel for schedule(dynamic, 1) num_threads(g_threads)
+#endif
+    for (int64_t q = 0; q < n_q; ++q) {
+        double* X = (double*)malloc(sizeof(double) * (size_t)D);
+        double* Y = (double*)malloc(sizeof(double) * (size_t)D);
+        to_eigenbasis(k_in, k_out, Ua, Ug, Q + q * D, X);
+        for (int64_t e = 0; e < D; ++e) X[e] /= Lam[e] + lambda;
+        for (int64_t r = 0; r < k_out; ++r) /* Y = X Ua^T */
+            for (int64_t c = 0; c < k_in; ++c) {
+                double s = 0.0;
+                for (int64_t j = 0; j < k_in; ++j) s += X[r * k_in + j] * Ua[c * k_in + j];
+                Y[r * k_in + c] = s;
+            }
+        for (int64_t r = 0; r < k_out; ++r) /* Qhat = Ug Y */
+            for (int64_t c = 0; c < k_in; ++c) {
+                double s = 0.0;
+                for (int64_t i = 0; i < k_out; ++i) s += Ug[r * k_out + i] * Y[i * k_in + c];
+                Qhat[q * D + r * k_in + c] = s;
+            }
+        free(X);
+        free(Y);
+    }
+}
+
+/* ------------------------------------------------------------------------ */
 /* Scores and top-k                                                         */
 /* ------------------------------------------------------------------------ */
 

@@ -116,6 +116,43 @@ int32_t oracle_cholesky(int64_t D, double* M);
 int32_t oracle_precondition(int64_t D, const double* F, double lambda,
                             int64_t n_q, const double* Q, double* Qhat);
 
+/* ---- Kronecker-factored curvature on the projected factors (K-FAC of
+ *      Martens & Grosse 2015, EK-FAC of George et al. 2018; the paper applies
+ *      them to projected factors unchanged, App. A.2, and damps by a multiple
+ *      of each layer's mean eigenvalue, App. B.2) ---- */
+
+/* Token-averaged second moments of the projected factors of N examples:
+ * Ca = (1/(N T)) sum_i sum_t a~_t a~_t^T (k_in x k_in) and
+ * Cg = (1/(N T)) sum_i sum_t g~_t g~_t^T (k_out x k_out), a~_t = P_a a_t,
+ * g~_t = P_g g_t with the seeded maps. */
+void oracle_kfac_covariances(int64_t N, int64_t T, int64_t d_in, int64_t d_out,
+                             int64_t k_in, int64_t k_out, uint64_t seed, uint32_t layer,
+                             int32_t kind, const double* A, const double* B,
+                             double* Ca, double* Cg);
+/* Symmetric eigendecomposition C = U diag(w) U^T by the cyclic Jacobi method
+ * (Golub & Van Loan, Matrix Computations, Sec. 8.5): eigenvalues ascending in
+ * w, eigenvectors in the columns of U (row-major n x n). Returns the number of
+ * sweeps, or -1 if 100 sweeps did not converge. */
+int32_t oracle_sym_eig(int64_t n, const double* C, double* w, double* U);
+/* K-FAC eigenvalues of Cg (x) Ca in the Kronecker eigenbasis:
+ * Lam[r][c] = wg[r] * wa[c] (k_out x k_in). */
+void oracle_kfac_eigenvalues(int64_t k_in, int64_t k_out, const double* wa, const double* wg,
+                             double* Lam);
+/* EK-FAC eigenvalue correction: the mean over the N training features of the
+ * squared coordinates in the Kronecker eigenbasis,
+ * Lam[r][c] = (1/N) sum_i ((Ug^T Phi_i Ua)[r][c])^2. */
+void oracle_ekfac_eigenvalues(int64_t N, int64_t k_in, int64_t k_out, const double* phi,
+                              const double* Ua, const double* Ug, double* Lam);
+/* lambda = lambda_abs + lambda_rel * mean(Lam). */
+double oracle_kfac_damping(int64_t k_in, int64_t k_out, const double* Lam, double lambda_abs,
+                           double lambda_rel);
+/* Qhat = Ug [(Ug^T Q Ua) / (Lam + lambda)] Ua^T for n_q query features
+ * (each k_out x k_in, row-major), the inverse of the damped curvature
+ * applied in its eigenbasis. */
+void oracle_kfac_precondition(int64_t k_in, int64_t k_out, const double* Ua, const double* Ug,
+                              const double* Lam, double lambda, int64_t n_q, const double* Q,
+                              double* Qhat);
+
 /* ---- scores and ranking ---- */
 
 /* S[q][i] = sum_f Qhat[q][f] Phi[i][f]. */
