@@ -79,6 +79,9 @@ def parse_args():
                    help="subset of the block's linears (profiling of a smaller case)")
     p.add_argument("--project-only", action="store_true",
                    help="time only the train projection (kernel profiling; not the metric's step)")
+    p.add_argument("--route-sweep", action="store_true",
+                   help="route cost-model sweep on one 8192x8192 bf16 linear (chosen vs measured fastest route)")
+    p.add_argument("--sweep-T", default="8,32,128,512,2048,8192")
     a = p.parse_args()
     names = a.linears.split(",")
     global LINEARS
@@ -236,10 +239,123 @@ def reference_main(args):
 
 
 # ---------------------------------------------------------------------------- GPU arm
+def route_sweep_main(args):
+    """One 8192x8192 bf16 linear, A, B ~ N(0,1), k = 64, 128 queries, N_train = 2^24 / T for each T:
+    every route of every op is timed on the device and extrapolated to the full N_train by a
+    two-point linear fit in the train count (t = a + b n); the route the Table 2 flop model
+    picks and the one the calibrated model picks are reported beside the measured fastest."""
+    import torch
+
+    import paper_2609_38767_gb300 as tda
+    from paper_2609_38767_gb300 import build as tbuild
+    from paper_2609_38767_gb300 import synth
+
+    tbuild.build()
+    tda.load()
+    dev = torch.device("cuda", 0)
+    torch.cuda.set_device(dev)
+    d, k, nq = 8192, 64, 128
+    D = k * k
+    cal_ws = torch.empty(tda.TDA_CALIBRATE_WS_BYTES, dtype=torch.uint8, device=dev)
+    rates = tda.tda_route_calibrate(cal_ws, tda.TDA_CALIBRATE_WS_BYTES)
+    del cal_ws
+    names = {0: "factored", 1: "materialize", 2: "gram"}
+    ops = [(tda.TDA_OP_PROJECT, "project", (0, 1)), (tda.TDA_OP_SIMILARITY_PROJECTED, "similarity_projected", (0, 1, 2)),
+           (tda.TDA_OP_SIMILARITY_EXACT, "similarity_exact", (1, 2))]
+    out = {"mode": "route-sweep", "linear": [d, d], "k": k, "n_query": nq, "dtype": "bf16",
+           "calibrated_rates_tflops": [r / 1e12 for r in rates[:3]], "calibrated_bw_gbs": rates[3] / 1e9,
+           "points": []}
+    stream = torch.cuda.current_stream()
+    for T in [int(x) for x in args.sweep_T.split(",")]:
+        N = 2 ** 24 // T
+        L = tda.LayerDesc(d, d, T, k, k, seed=0, layer=0)
+        ex_bytes = T * 2 * d * 2
+        P = max(1, min(N, int(16e9 // ex_bytes)))
+        A = torch.empty(P * T * d, dtype=torch.bfloat16, device=dev)
+        B = torch.empty_like(A)
+        Aq = torch.empty(nq * T * d, dtype=torch.bfloat16, device=dev)
+        Bq = torch.empty_like(Aq)
+        for x, seed, st in ((A, synth.SEED_A, 0), (B, synth.SEED_B, 0), (Aq, synth.SEED_A, 1000), (Bq, synth.SEED_B, 1000)):
+            synth.fill_device(x, seed, st, x.numel() // (T * d), T, d, 1.0)
+        phi = torch.empty(P * D, dtype=torch.float32, device=dev)
+        S = torch.empty(nq * P, dtype=torch.float32, device=dev)
+
+        def run(op, route, n_q, n_t, ws, wsb):
+            done = 0
+            while done < n_t:
+                c = min(P, n_t - done)
+                if op == tda.TDA_OP_PROJECT:
+                    tda.tda_project(L, tda.TDA_BF16, A, B, c, phi, D, route, ws, wsb)
+                elif op == tda.TDA_OP_SIMILARITY_PROJECTED:
+                    tda.tda_similarity_projected(L, tda.TDA_BF16, Aq, Bq, n_q, A, B, c, S, c, 0.0, route, ws, wsb)
+                else:
+                    tda.tda_similarity_exact(L, tda.TDA_BF16, Aq, Bq, n_q, A, B, c, S, c, 0.0, route, ws, wsb)
+                done += c
+
+        def timed(op, route, n_q, n_t, ws, wsb):
+            e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            e0.record(stream)
+            run(op, route, n_q, n_t, ws, wsb)
+            e1.record(stream)
+            e1.synchronize()
+            return e0.elapsed_time(e1) * 1e-3
+
+        point = {"T": T, "n_train": N, "pool_examples": P, "ops": {}}
+        for op, opname, routes in ops:
+            rec = {"flop_model_choice": names[tda.tda_route(L, op, nq, N, tda.TDA_BF16)[0]]}
+            tda.tda_route_set_model(1)
+            ch, est = tda.tda_route(L, op, nq, N, tda.TDA_BF16)
+            tda.tda_route_set_model(0)
+            rec["calibrated_choice"] = names[ch]
+            rec["calibrated_estimate_s"] = {names[r]: est[r] for r in routes}
+            meas = {}
+            for r in routes:
+                # pure pair-cost route (exact Gram): fewer queries when one train example is slow
+                n_q = nq
+                if op == tda.TDA_OP_SIMILARITY_EXACT and r == 2:
+                    per = 2.0 * T * T * 2 * d / 20e12  # seconds per pair at a conservative 20 TFLOP/s
+                    n_q = max(1, min(nq, int(0.5 / per)))
+                n1 = 1 if op != tda.TDA_OP_PROJECT else min(P, 8)
+                wsb = max(tda.tda_workspace_size(op, L, tda.TDA_BF16, n_q, P, r), 256)
+                if op == tda.TDA_OP_SIMILARITY_PROJECTED:
+                    wsb = max(wsb, min(2 << 30, tda.tda_workspace_size(op, L, tda.TDA_BF16, n_q, P, r) * 16))
+                ws = torch.empty(wsb, dtype=torch.uint8, device=dev)
+                timed(op, r, n_q, n1, ws, wsb)  # warm-up
+                t1 = timed(op, r, n_q, n1, ws, wsb)
+                while t1 < 0.05 and n1 < N:
+                    n1 = min(N, n1 * max(2, int(0.1 / max(t1, 1e-6))))
+                    t1 = timed(op, r, n_q, n1, ws, wsb)
+                if 2 * n1 <= N:
+                    t2 = timed(op, r, n_q, 2 * n1, ws, wsb)
+                    b = max((t2 - t1) / n1, 0.0)
+                    a = max(t1 - b * n1, 0.0)
+                else:
+                    a, b = 0.0, t1 / n1
+                full = (a + b * N) * (nq / n_q)
+                meas[names[r]] = {"seconds": full, "timed_train_examples": [n1, 2 * n1 if 2 * n1 <= N else n1],
+                                  "timed_queries": n_q, "extrapolated": n1 < N or n_q < nq}
+                del ws
+                torch.cuda.synchronize()
+            fastest = min(meas, key=lambda x: meas[x]["seconds"])
+            rec["measured"] = meas
+            rec["measured_fastest"] = fastest
+            rec["calibrated_over_fastest"] = meas[rec["calibrated_choice"]]["seconds"] / meas[fastest]["seconds"]
+            rec["flop_model_over_fastest"] = meas[rec["flop_model_choice"]]["seconds"] / meas[fastest]["seconds"]
+            point["ops"][opname] = rec
+        tda.tda_device_status()
+        out["points"].append(point)
+        print(json.dumps(point), file=sys.stderr, flush=True)
+        del A, B, Aq, Bq, phi, S
+        torch.cuda.empty_cache()
+    print(json.dumps(out))
+
+
 def main():
     args = parse_args()
     if args.impl == "reference":
         return reference_main(args)
+    if args.route_sweep:
+        return route_sweep_main(args)
 
     import numpy as np
     import torch

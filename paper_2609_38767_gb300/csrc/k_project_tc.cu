@@ -1,15 +1,26 @@
 // k_project_tc.cu -- factored projection (Eq. 2) on the 5th-generation tensor
 // cores of sm_103a: tcgen05.mma with TMEM accumulators, operands staged in
-// shared memory by TMA (factors) and by a generator warp (signs).
+// shared memory by TMA (factors) and by generator warps (signs).
 //
-// For every example n and every 128-token tile of it:
+// For every 128-row token tile:
 //   At = A_tile S_in   (128 x k_in,  K = d_in)    tcgen05, accumulators in TMEM
 //   Bt = B_tile S_out  (128 x k_out, K = d_out)   tcgen05, accumulators in TMEM
-//   Phi_n += Bt^T At   (k_out x k_in, over the 128 tokens) on CUDA cores, fp32
+//   Phi_n += Bt^T At   (k_out x k_in, over the tile's tokens of example n) on
+//                      CUDA cores, fp32
 // and finally Phi_n *= 1/sqrt(k_in k_out). The signs S (App. A.2) come from the
 // counter hash: one 64-bit word gives the 64 signs of one column over one
 // 64-row K chunk, which is one 128-byte row of the K-major, 128B-swizzled
 // operand tile, so the projection matrices never touch global memory.
+//
+// Token tiles: for T > 64 a tile is 128 consecutive tokens of one example (the
+// last one zero-filled past T); for T <= 64 a tile packs floor(128 / T) whole
+// examples (the factors of consecutive examples are consecutive rows), so short
+// sequences do not leave most of each MMA empty.
+//
+// A pipeline stage holds G token tiles (G = 2 for large batches) that share
+// one sign tile: the signs of a K chunk do not depend on the tokens, so
+// generating them once for G tiles halves the generators' work and the MMA
+// commits per byte streamed.
 //
 // The kernel streams every factor byte once from HBM; at k <= 64 its
 // arithmetic intensity (~k flop/B) is far below the tensor-core ridge, so it
@@ -19,13 +30,12 @@
 //   warp 0  TMA producer: 128x64 bf16 factor tiles into the stage ring
 //   warp 1  TMEM allocator; lane 0 issues the MMAs
 //   warps 2-3  sign generators: k x 64 bf16 +-1 tiles into the stage ring,
-//           each warp one half of every 128-byte row (one warp alone falls
-//           behind the HBM stream)
+//           each warp one half of every 128-byte row
 //   warps 4-7  epilogue: TMEM -> registers -> shared -> token contraction
-// Accumulators are double-buffered in TMEM, so the epilogue of one tile
-// overlaps the MMAs of the next. Every wait is bounded (about 1 s); on expiry
-// the kernel records kErrTimeout in the device error word, drains its copies,
-// frees its TMEM and returns.
+// Accumulators are double-buffered in TMEM, so the epilogue of one group of
+// tiles overlaps the MMAs of the next. Every wait is bounded (about 1 s); on
+// expiry the kernel records kErrTimeout in the device error word, drains its
+// copies, frees its TMEM and returns.
 #include <cuda.h>
 #include <cuda_bf16.h>
 
@@ -40,35 +50,74 @@ constexpr int kThreads = 256;
 constexpr int kTileM = 128;            // tokens per tile (MMA M)
 constexpr int kChunkK = 64;            // K elements per stage (128 bytes of bf16)
 constexpr uint32_t kTileBytes = kTileM * kChunkK * 2;  // 16 KiB per factor tile
+constexpr size_t kSmemMax = 232448;    // 227 KiB of dynamic shared memory per CTA
+constexpr int kMaxStages = 12;
 
-template <int K>
+template <int K, int G>
 struct Cfg {
-    static constexpr int kStages = K <= 32 ? 8 : 6;
-    static constexpr uint32_t kSignBytes = K * 128;  // K rows x 128 bytes
-    static constexpr int kStageLd = K + 4;           // padded fp32 staging row
-    static constexpr int kAccCols = 2 * K;           // At | Bt in one accumulator buffer
-    static constexpr uint32_t kTmemCols = 2 * kAccCols < 32 ? 32 : 2 * kAccCols;
-    static constexpr size_t kSmemA = (size_t)kStages * kTileBytes;
-    static constexpr size_t kSmemS = (size_t)kStages * kSignBytes;
+    static constexpr uint32_t kSignBytes = K * 128;                       // K rows x 128 bytes
+    static constexpr uint32_t kStageBytes = G * kTileBytes + kSignBytes;  // G factor tiles, then signs
+    static constexpr int kStageLd = K + 4;                                // padded fp32 staging row
+    static constexpr int kAccCols = 2 * K;                                // At | Bt of one tile
+    static constexpr int kBufCols = G * kAccCols;                         // one accumulator buffer
+    static constexpr uint32_t kTmemCols = 2 * kBufCols < 32 ? 32 : 2 * kBufCols;
     static constexpr size_t kSmemStage = 2ull * kTileM * kStageLd * 4;
+    static constexpr size_t kSmemBarsMax = 8 * (3 * kMaxStages + 7) + 16;
+    static constexpr int kFit = (int)((kSmemMax - 1024 - kSmemStage - kSmemBarsMax) / kStageBytes);
+    static constexpr int kStages = kFit > kMaxStages ? kMaxStages : kFit;
     static constexpr size_t kSmemBars = 8 * (3 * kStages + 7) + 16;
-    static constexpr size_t kSmem = 1024 + kSmemA + kSmemS + kSmemStage + kSmemBars;
+    static constexpr size_t kSmem = 1024 + (size_t)kStages * kStageBytes + kSmemStage + kSmemBars;
     // contraction blocking: 16 row groups x 8 column groups of threads
     static constexpr int RB = K / 16 > 0 ? K / 16 : 1;
     static constexpr int CB = K / 8;
+    static_assert(kStages >= 3 && kSmem <= kSmemMax, "shared memory per CTA");
+    static_assert(kStageBytes % 1024 == 0 && kTmemCols <= 512, "operand alignment / TMEM columns");
 };
 
 struct Params {
     int64_t N, T, d_in, d_out, ld_phi;
+    int64_t n_slots;  // example slots: examples (pack == 1) or groups of `pack` examples
     uint64_t key_in, key_out;
     float scale;
     float* phi;
     unsigned int* err;
-    int n_ttiles, nk_in, nk_out;
-    int cs;  // CTAs per cluster sharing one example's token tiles (1, 2 or 4)
+    int n_ttiles;     // token tiles per slot
+    int pack;         // examples per token tile (T <= 64), else 1
+    int nk_in, nk_out;
+    int cs;           // CTAs per cluster sharing one example's token tiles (1, 2 or 4)
 };
 
 #include "tc_ptx.cuh"
+
+// The sequence of token tiles ("units") one CTA works on, identical for every
+// warp role: example slots cid, cid + ncl, ... and, within a slot, the token
+// tiles crank, crank + cs, ...
+struct Units {
+    int64_t x;
+    int tt;
+    __device__ __forceinline__ void first(uint32_t cid, uint32_t crank) {
+        x = cid;
+        tt = (int)crank;
+    }
+    // Next group of up to G units into gx/gt; returns how many (0 = finished).
+    template <int G>
+    __device__ __forceinline__ int take(const Params& p, uint32_t ncl, uint32_t crank, int64_t* gx, int* gt) {
+        int n = 0;
+#pragma unroll
+        for (int u = 0; u < G; ++u)
+            if (x < p.n_slots) {
+                gx[u] = x;
+                gt[u] = tt;
+                ++n;
+                tt += p.cs;
+                if (tt >= p.n_ttiles) {
+                    tt = (int)crank;
+                    x += ncl;
+                }
+            }
+        return n;
+    }
+};
 
 // Half `half` (16-byte chunks 4*half .. 4*half+3) of row n of a K-major
 // 128B-swizzled sign tile: signs of column n over the K chunk, as bf16 +1
@@ -90,16 +139,15 @@ __device__ __forceinline__ void write_sign_half(uint8_t* tile, int n, uint64_t w
     }
 }
 
-template <int K>
+template <int K, int G>
 __global__ void __launch_bounds__(kThreads, 1)
 project_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
                   const Params p) {
-    using C = Cfg<K>;
+    using C = Cfg<K, G>;
     extern __shared__ uint8_t smem_raw[];
     uint8_t* smem = (uint8_t*)(((uintptr_t)smem_raw + 1023) & ~(uintptr_t)1023);
-    uint8_t* sA = smem;
-    uint8_t* sS = sA + C::kSmemA;
-    float* stX = (float*)(sS + C::kSmemS);        // [128][K+4] At rows
+    uint8_t* sA = smem;                           // kStages x [G factor tiles | sign tile]
+    float* stX = (float*)(sA + (size_t)C::kStages * C::kStageBytes);  // [128][K+4] At rows
     float* stY = stX + kTileM * C::kStageLd;      // [128][K+4] Bt rows
     uint64_t* bars = (uint64_t*)(stY + kTileM * C::kStageLd);
     uint64_t* full = bars;                        // TMA landed        (count 1 + tx)
@@ -139,34 +187,41 @@ project_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant
     cluster_sync();  // every CTA's barriers exist before any remote arrive
     tc_fence_after();
     const uint32_t tmem = *tmem_slot;
-    // examples are shared out per cluster; token tiles per CTA rank within it
     const uint32_t crank = cluster_rank(), cid = blockIdx.x / p.cs, ncl = gridDim.x / p.cs;
-
     const int nk_tot = p.nk_in + p.nk_out;
+    int64_t gx[G];
+    int gt[G];
+    Units it;
+    it.first(cid, crank);
+
     if (warp == 0 && lane == 0) {
         // ---------------- TMA producer
-        uint32_t last_par[16];
-        bool issued[16];
+        uint32_t last_par[kMaxStages];
+        bool issued[kMaxStages];
         for (int s = 0; s < C::kStages; ++s) issued[s] = false;
         uint32_t ring = 0;
         bool ok = true;
-        for (int64_t n = cid; ok && n < p.N; n += ncl)
-            for (int tt = (int)crank; ok && tt < p.n_ttiles; tt += p.cs)
-                for (int kc = 0; kc < nk_tot; ++kc, ++ring) {
-                    const int s = ring % C::kStages;
-                    const uint32_t ph = (ring / C::kStages) & 1u;
-                    if (!wait_bounded(smem_u32(&empty[s]), ph ^ 1u, abort, p.err)) {
-                        ok = false;
-                        break;
-                    }
-                    const bool side_b = kc >= p.nk_in;
-                    const int d0 = (side_b ? kc - p.nk_in : kc) * kChunkK;
-                    mbar_arrive_tx(smem_u32(&full[s]), kTileBytes);
-                    tma_load_3d(smem_u32(sA + (size_t)s * kTileBytes), side_b ? &tmB : &tmA, d0, tt * kTileM,
-                                (int)n, smem_u32(&full[s]));
-                    issued[s] = true;
-                    last_par[s] = ph;
+        for (int ng; ok && (ng = it.take<G>(p, ncl, crank, gx, gt)) > 0;)
+            for (int kc = 0; kc < nk_tot; ++kc, ++ring) {
+                const int s = ring % C::kStages;
+                const uint32_t ph = (ring / C::kStages) & 1u;
+                if (!wait_bounded(smem_u32(&empty[s]), ph ^ 1u, abort, p.err)) {
+                    ok = false;
+                    break;
                 }
+                const bool side_b = kc >= p.nk_in;
+                const int d0 = (side_b ? kc - p.nk_in : kc) * kChunkK;
+                mbar_arrive_tx(smem_u32(&full[s]), (uint32_t)ng * kTileBytes);
+                for (int u = 0; u < ng; ++u) {
+                    // packed tiles: row x * pack * T of the [N*T][d] view; else tile tt of example x
+                    const int row = p.pack > 1 ? (int)(gx[u] * p.pack * p.T) : gt[u] * kTileM;
+                    const int ex = p.pack > 1 ? 0 : (int)gx[u];
+                    tma_load_3d(smem_u32(sA + (size_t)s * C::kStageBytes + (size_t)u * kTileBytes),
+                                side_b ? &tmB : &tmA, d0, row, ex, smem_u32(&full[s]));
+                }
+                issued[s] = true;
+                last_par[s] = ph;
+            }
         // drain: every issued copy must land before the CTA may exit
         for (int s = 0; s < C::kStages; ++s)
             if (issued[s]) {
@@ -179,39 +234,41 @@ project_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant
             }
     } else if (warp == 1 && lane == 0) {
         // ---------------- MMA issuer
-        uint32_t ring = 0, tile = 0;
+        uint32_t ring = 0, grp = 0;
         bool ok = true;
         const uint32_t idesc = idesc_bf16(kTileM, K);
-        for (int64_t n = cid; ok && n < p.N; n += ncl)
-            for (int tt = (int)crank; ok && tt < p.n_ttiles; tt += p.cs, ++tile) {
-                const uint32_t b = tile & 1u, use = tile >> 1;
-                if (!wait_bounded(smem_u32(&tempty[b]), (use & 1u) ^ 1u, abort, p.err)) {
+        for (int ng; ok && (ng = it.take<G>(p, ncl, crank, gx, gt)) > 0; ++grp) {
+            const uint32_t b = grp & 1u, use = grp >> 1;
+            if (!wait_bounded(smem_u32(&tempty[b]), (use & 1u) ^ 1u, abort, p.err)) {
+                ok = false;
+                break;
+            }
+            tc_fence_after();
+            for (int kc = 0; kc < nk_tot; ++kc, ++ring) {
+                const int s = ring % C::kStages;
+                const uint32_t ph = (ring / C::kStages) & 1u;
+                if (!wait_bounded(smem_u32(&full[s]), ph, abort, p.err) ||
+                    !wait_bounded(smem_u32(&sready[s]), ph, abort, p.err)) {
                     ok = false;
                     break;
                 }
                 tc_fence_after();
-                for (int kc = 0; kc < nk_tot; ++kc, ++ring) {
-                    const int s = ring % C::kStages;
-                    const uint32_t ph = (ring / C::kStages) & 1u;
-                    if (!wait_bounded(smem_u32(&full[s]), ph, abort, p.err) ||
-                        !wait_bounded(smem_u32(&sready[s]), ph, abort, p.err)) {
-                        ok = false;
-                        break;
-                    }
-                    tc_fence_after();
-                    const bool side_b = kc >= p.nk_in;
-                    const int kk = side_b ? kc - p.nk_in : kc;
-                    const uint32_t d_tmem = tmem + b * C::kAccCols + (side_b ? K : 0);
-                    const uint64_t ad = sw128_desc(smem_u32(sA + (size_t)s * kTileBytes));
-                    const uint64_t bd = sw128_desc(smem_u32(sS + (size_t)s * C::kSignBytes));
+                const bool side_b = kc >= p.nk_in;
+                const int kk = side_b ? kc - p.nk_in : kc;
+                uint8_t* stage = sA + (size_t)s * C::kStageBytes;
+                const uint64_t bd = sw128_desc(smem_u32(stage + (size_t)G * kTileBytes));
+                for (int u = 0; u < ng; ++u) {
+                    const uint32_t d_tmem = tmem + b * C::kBufCols + u * C::kAccCols + (side_b ? K : 0);
+                    const uint64_t ad = sw128_desc(smem_u32(stage + (size_t)u * kTileBytes));
 #pragma unroll
                     for (int k = 0; k < kChunkK / 16; ++k)
                         mma_bf16(d_tmem, ad + 2 * k, bd + 2 * k, idesc, (kk > 0 || k > 0) ? 1u : 0u);
-                    mma_commit(smem_u32(&empty[s]));
                 }
-                if (!ok) break;
-                mma_commit(smem_u32(&tfull[b]));
+                mma_commit(smem_u32(&empty[s]));
             }
+            if (!ok) break;
+            mma_commit(smem_u32(&tfull[b]));
+        }
         // all MMAs this thread issued have completed once mma_done fires
         mma_commit(smem_u32(mma_done));
         const uint64_t t0 = global_ns();
@@ -224,86 +281,49 @@ project_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant
         // ---------------- sign generators (two warps, one half-row each)
         uint32_t ring = 0;
         bool ok = true;
-        for (int64_t n = cid; ok && n < p.N; n += ncl)
-            for (int tt = (int)crank; ok && tt < p.n_ttiles; tt += p.cs)
-                for (int kc = 0; kc < nk_tot; ++kc, ++ring) {
-                    const int s = ring % C::kStages;
-                    const uint32_t ph = (ring / C::kStages) & 1u;
-                    bool got = true;
-                    if (lane == 0) got = wait_bounded(smem_u32(&empty[s]), ph ^ 1u, abort, p.err);
-                    got = __shfl_sync(0xffffffffu, got, 0);
-                    __syncwarp();
-                    if (!got) {
-                        ok = false;
-                        break;
-                    }
-                    const bool side_b = kc >= p.nk_in;
-                    const uint64_t key = side_b ? p.key_out : p.key_in;
-                    const uint64_t rb = (uint64_t)(side_b ? kc - p.nk_in : kc);
-                    uint8_t* tile = sS + (size_t)s * C::kSignBytes;
-                    for (int col = lane; col < K; col += 32)
-                        write_sign_half(tile, col, sign_word(key, (uint32_t)col, rb), warp - 2);
-                    fence_proxy_async();
-                    __syncwarp();
-                    if (lane == 0) mbar_arrive(smem_u32(&sready[s]));
+        for (int ng; ok && (ng = it.take<G>(p, ncl, crank, gx, gt)) > 0;)
+            for (int kc = 0; kc < nk_tot; ++kc, ++ring) {
+                const int s = ring % C::kStages;
+                const uint32_t ph = (ring / C::kStages) & 1u;
+                bool got = true;
+                if (lane == 0) got = wait_bounded(smem_u32(&empty[s]), ph ^ 1u, abort, p.err);
+                got = __shfl_sync(0xffffffffu, got, 0);
+                __syncwarp();
+                if (!got) {
+                    ok = false;
+                    break;
                 }
+                const bool side_b = kc >= p.nk_in;
+                const uint64_t key = side_b ? p.key_out : p.key_in;
+                const uint64_t rb = (uint64_t)(side_b ? kc - p.nk_in : kc);
+                uint8_t* tile = sA + (size_t)s * C::kStageBytes + (size_t)G * kTileBytes;
+                for (int col = lane; col < K; col += 32)
+                    write_sign_half(tile, col, sign_word(key, (uint32_t)col, rb), warp - 2);
+                fence_proxy_async();
+                __syncwarp();
+                if (lane == 0) mbar_arrive(smem_u32(&sready[s]));
+            }
     } else if (warp >= 4) {
         // ---------------- epilogue: TMEM -> shared -> Phi += Bt^T At
         const int q = warp & 3;          // TMEM lane quadrant of this warp
         const int et = threadIdx.x - 128;
-        const int row = q * 32 + lane;   // token within the tile
+        const int row = q * 32 + lane;   // token row within the tile
         const int rg = et >> 3, cg = et & 7;
-        uint32_t tile = 0, red_use = 0;
+        uint32_t grp = 0, red_use = 0;
         bool stop = false;
-        for (int64_t n = cid; !stop && n < p.N; n += ncl) {
-            float acc[C::RB][C::CB];
+        int64_t cur = -1;                // example whose Phi is accumulating (pack == 1)
+        float acc[C::RB][C::CB];
 #pragma unroll
-            for (int a = 0; a < C::RB; ++a)
+        for (int a = 0; a < C::RB; ++a)
 #pragma unroll
-                for (int c = 0; c < C::CB; ++c) acc[a][c] = 0.f;
-            for (int tt = (int)crank; tt < p.n_ttiles; tt += p.cs, ++tile) {
-                const uint32_t b = tile & 1u, use = tile >> 1;
-                bool got = true;
-                if (lane == 0) got = wait_bounded(smem_u32(&tfull[b]), use & 1u, abort, p.err);
-                got = __shfl_sync(0xffffffffu, got, 0);
-                if (epi_any(!got)) {
-                    stop = true;
-                    break;
-                }
-                tc_fence_after();
-                const uint32_t tbase = tmem + ((uint32_t)(q * 32) << 16) + b * C::kAccCols;
-#pragma unroll
-                for (int c0 = 0; c0 < 2 * K; c0 += 16) {
-                    float v[16];
-                    tmem_ld16(tbase + c0, v);
-                    float* dst = c0 < K ? stX + row * C::kStageLd + c0 : stY + row * C::kStageLd + (c0 - K);
-#pragma unroll
-                    for (int i = 0; i < 16; i += 4)
-                        *reinterpret_cast<float4*>(dst + i) = make_float4(v[i], v[i + 1], v[i + 2], v[i + 3]);
-                }
-                tc_fence_before();
-                __syncwarp();
-                if (lane == 0) mbar_arrive(smem_u32(&tempty[b]));
-                epi_sync();
-#pragma unroll 4
-                for (int t = 0; t < kTileM; ++t) {
-                    float y[C::RB], x[C::CB];
-#pragma unroll
-                    for (int a = 0; a < C::RB; ++a) y[a] = stY[t * C::kStageLd + rg * C::RB + a];
-#pragma unroll
-                    for (int c = 0; c < C::CB; ++c) x[c] = stX[t * C::kStageLd + cg * C::CB + c];
-#pragma unroll
-                    for (int a = 0; a < C::RB; ++a)
-#pragma unroll
-                        for (int c = 0; c < C::CB; ++c) acc[a][c] = fmaf(y[a], x[c], acc[a][c]);
-                }
-                epi_sync();
-            }
-            if (stop) break;
+            for (int c = 0; c < C::CB; ++c) acc[a][c] = 0.f;
+
+        // Phi of example `n` is complete in every cluster CTA: reduce the partial
+        // blocks into the leader (rank 0) over distributed shared memory and
+        // write it. The leader's staging buffer (free between tiles) receives
+        // member r's partial at offset (r-1)*K*K, thread-major.
+        auto flush = [&](int64_t n) -> bool {
             if (p.cs > 1) {
-                // Cluster reduction of the partial Phi blocks into the leader (rank
-                // 0). The leader's staging buffer (free between tiles) receives
-                // member r's partial at offset (r-1)*K*K, thread-major.
                 constexpr int kPer = C::RB * C::CB;
                 const uint32_t slot = smem_u32(stX) + (uint32_t)(et * kPer) * 4u;
                 bool got = true;
@@ -312,7 +332,7 @@ project_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant
                         for (int r = 1; r < p.cs; ++r) mbar_arrive_remote(smem_u32(red_go), (uint32_t)r);
                     if (lane == 0) got = wait_bounded_cluster(smem_u32(red_full), red_use & 1u, abort, p.err);
                     got = __shfl_sync(0xffffffffu, got, 0);
-                    if (epi_any(!got)) break;
+                    if (epi_any(!got)) return false;
                     for (int r = 1; r < p.cs; ++r) {
                         const float* part = stX + (r - 1) * K * K + et * kPer;
 #pragma unroll
@@ -324,26 +344,115 @@ project_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant
                 } else {
                     if (lane == 0) got = wait_bounded_cluster(smem_u32(red_go), red_use & 1u, abort, p.err);
                     got = __shfl_sync(0xffffffffu, got, 0);
-                    if (epi_any(!got)) break;
+                    if (epi_any(!got)) return false;
                     const uint32_t dst = map_rank(slot, 0) + (crank - 1) * (uint32_t)(K * K) * 4u;
 #pragma unroll
                     for (int a = 0; a < C::RB; ++a)
 #pragma unroll
-                        for (int c = 0; c < C::CB; ++c) st_cluster_f32(dst + (uint32_t)(a * C::CB + c) * 4u, acc[a][c]);
+                        for (int c = 0; c < C::CB; ++c)
+                            st_cluster_f32(dst + (uint32_t)(a * C::CB + c) * 4u, acc[a][c]);
                     fence_acq_rel_cluster();
                     epi_sync();
                     if (et == 0) mbar_arrive_remote(smem_u32(red_full), 0u);
                 }
                 ++red_use;
-                if (crank != 0) continue;
+                if (crank != 0) return true;
             }
             float* out = p.phi + n * p.ld_phi;
 #pragma unroll
             for (int a = 0; a < C::RB; ++a)
 #pragma unroll
-                for (int c = 0; c < C::CB; ++c)
-                    out[(rg * C::RB + a) * K + cg * C::CB + c] = acc[a][c] * p.scale;
+                for (int c = 0; c < C::CB; ++c) out[(rg * C::RB + a) * K + cg * C::CB + c] = acc[a][c] * p.scale;
+            return true;
+        };
+
+        for (int ng; !stop && (ng = it.take<G>(p, ncl, crank, gx, gt)) > 0; ++grp) {
+            const uint32_t b = grp & 1u, use = grp >> 1;
+            bool got = true;
+            if (lane == 0) got = wait_bounded(smem_u32(&tfull[b]), use & 1u, abort, p.err);
+            got = __shfl_sync(0xffffffffu, got, 0);
+            if (epi_any(!got)) {
+                stop = true;
+                break;
+            }
+            tc_fence_after();
+            for (int u = 0; u < ng; ++u) {
+                if (p.pack == 1 && gx[u] != cur) {
+                    if (cur >= 0 && !flush(cur)) {
+                        stop = true;
+                        break;
+                    }
+                    cur = gx[u];
+#pragma unroll
+                    for (int a = 0; a < C::RB; ++a)
+#pragma unroll
+                        for (int c = 0; c < C::CB; ++c) acc[a][c] = 0.f;
+                }
+                const uint32_t tbase =
+                    tmem + ((uint32_t)(q * 32) << 16) + b * C::kBufCols + (uint32_t)u * C::kAccCols;
+#pragma unroll
+                for (int c0 = 0; c0 < 2 * K; c0 += 16) {
+                    float v[16];
+                    tmem_ld16(tbase + c0, v);
+                    float* dst = c0 < K ? stX + row * C::kStageLd + c0 : stY + row * C::kStageLd + (c0 - K);
+#pragma unroll
+                    for (int i = 0; i < 16; i += 4)
+                        *reinterpret_cast<float4*>(dst + i) = make_float4(v[i], v[i + 1], v[i + 2], v[i + 3]);
+                }
+                if (u == ng - 1) {
+                    tc_fence_before();
+                    __syncwarp();
+                    if (lane == 0) mbar_arrive(smem_u32(&tempty[b]));
+                }
+                epi_sync();
+                if (p.pack == 1) {
+#pragma unroll 4
+                    for (int t = 0; t < kTileM; ++t) {
+                        float y[C::RB], x[C::CB];
+#pragma unroll
+                        for (int a = 0; a < C::RB; ++a) y[a] = stY[t * C::kStageLd + rg * C::RB + a];
+#pragma unroll
+                        for (int c = 0; c < C::CB; ++c) x[c] = stX[t * C::kStageLd + cg * C::CB + c];
+#pragma unroll
+                        for (int a = 0; a < C::RB; ++a)
+#pragma unroll
+                            for (int c = 0; c < C::CB; ++c) acc[a][c] = fmaf(y[a], x[c], acc[a][c]);
+                    }
+                } else {
+                    // packed tile: example x * pack + j owns rows j*T .. j*T + T - 1
+                    for (int j = 0; j < p.pack; ++j) {
+                        const int64_t e = gx[u] * p.pack + j;
+                        if (e >= p.N) break;
+                        float a2[C::RB][C::CB];
+#pragma unroll
+                        for (int a = 0; a < C::RB; ++a)
+#pragma unroll
+                            for (int c = 0; c < C::CB; ++c) a2[a][c] = 0.f;
+                        const int t1 = (j + 1) * (int)p.T;
+#pragma unroll 4
+                        for (int t = j * (int)p.T; t < t1; ++t) {
+                            float y[C::RB], x[C::CB];
+#pragma unroll
+                            for (int a = 0; a < C::RB; ++a) y[a] = stY[t * C::kStageLd + rg * C::RB + a];
+#pragma unroll
+                            for (int c = 0; c < C::CB; ++c) x[c] = stX[t * C::kStageLd + cg * C::CB + c];
+#pragma unroll
+                            for (int a = 0; a < C::RB; ++a)
+#pragma unroll
+                                for (int c = 0; c < C::CB; ++c) a2[a][c] = fmaf(y[a], x[c], a2[a][c]);
+                        }
+                        float* out = p.phi + e * p.ld_phi;
+#pragma unroll
+                        for (int a = 0; a < C::RB; ++a)
+#pragma unroll
+                            for (int c = 0; c < C::CB; ++c)
+                                out[(rg * C::RB + a) * K + cg * C::CB + c] = a2[a][c] * p.scale;
+                    }
+                }
+                epi_sync();
+            }
         }
+        if (!stop && p.pack == 1 && cur >= 0) flush(cur);
     }
 
     tc_fence_before();
@@ -375,7 +484,8 @@ EncodeTiledFn encode_fn() {
 }
 
 // 3-D map over X[N][T][d] (bf16): box 64 (d) x 128 (t) x 1 (example), 128B swizzle,
-// out-of-range elements read as zero.
+// out-of-range elements read as zero. For packed tiles the same memory is viewed
+// as [1][N*T][d], so one box spans several consecutive examples.
 bool make_map(CUtensorMap* tm, const void* X, int64_t N, int64_t T, int64_t d) {
     EncodeTiledFn enc = encode_fn();
     if (!enc) return false;
@@ -397,40 +507,52 @@ bool device_is_sm103() {
     return major == 10 && minor == 3;
 }
 
-template <int K>
-cudaError_t launch_k(const tda_layer_desc& L, const void* A, const void* B, int64_t N, float* phi,
-                     int64_t ld_phi, unsigned int* err, cudaStream_t s) {
-    using C = Cfg<K>;
+int sm_count() {
+    static int sms = 0;
+    if (!sms) {
+        int dev = 0, n = 0;
+        cudaGetDevice(&dev);
+        cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev);
+        sms = n > 0 ? n : 1;
+    }
+    return sms;
+}
+
+template <int K, int G>
+cudaError_t launch_kg(const tda_layer_desc& L, const void* A, const void* B, int64_t N, float* phi,
+                      int64_t ld_phi, unsigned int* err, cudaStream_t s, int pack) {
+    using C = Cfg<K, G>;
     CUtensorMap tmA, tmB;
-    if (!make_map(&tmA, A, N, L.T, L.d_in) || !make_map(&tmB, B, N, L.T, L.d_out)) return cudaErrorInvalidValue;
+    if (pack > 1) {
+        if (!make_map(&tmA, A, 1, N * L.T, L.d_in) || !make_map(&tmB, B, 1, N * L.T, L.d_out))
+            return cudaErrorInvalidValue;
+    } else if (!make_map(&tmA, A, N, L.T, L.d_in) || !make_map(&tmB, B, N, L.T, L.d_out)) {
+        return cudaErrorInvalidValue;
+    }
     Params p;
     p.N = N;
     p.T = L.T;
     p.d_in = L.d_in;
     p.d_out = L.d_out;
     p.ld_phi = ld_phi;
+    p.pack = pack;
+    p.n_slots = pack > 1 ? (N + pack - 1) / pack : N;
     p.key_in = side_key(L.seed, L.layer, 0);
     p.key_out = side_key(L.seed, L.layer, 1);
     p.scale = projection_scale(L);
     p.phi = phi;
     p.err = err;
-    p.n_ttiles = (int)((L.T + kTileM - 1) / kTileM);
+    p.n_ttiles = pack > 1 ? 1 : (int)((L.T + kTileM - 1) / kTileM);
     p.nk_in = (int)((L.d_in + kChunkK - 1) / kChunkK);
     p.nk_out = (int)((L.d_out + kChunkK - 1) / kChunkK);
-    static int sms = 0;
-    if (!sms) {
-        int dev = 0;
-        cudaGetDevice(&dev);
-        cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
-        if (sms <= 0) sms = 1;
-    }
-    cudaError_t e = cudaFuncSetAttribute(project_tc_kernel<K>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+    const int sms = sm_count();
+    cudaError_t e = cudaFuncSetAttribute(project_tc_kernel<K, G>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                          (int)C::kSmem);
     if (e != cudaSuccess) return e;
     // Fewer examples than SMs: a cluster of cs CTAs shares each example's token
     // tiles and reduces the partial features through distributed shared memory.
     int cs = 1;
-    if (N < sms) cs = (2 * N >= sms) ? 2 : 4;
+    if (pack == 1 && N < sms) cs = (2 * N >= sms) ? 2 : 4;
     while (cs > 1 && cs > p.n_ttiles) cs >>= 1;
     p.cs = cs;
     cudaLaunchConfig_t cfg = {};
@@ -444,17 +566,49 @@ cudaError_t launch_k(const tda_layer_desc& L, const void* A, const void* B, int6
     cfg.stream = s;
     cfg.attrs = attr;
     cfg.numAttrs = 1;
-    int64_t clusters = N;
     int max_clusters = 0;
     cfg.gridDim = dim3((unsigned)(cs * (sms / cs)));
-    if (cudaOccupancyMaxActiveClusters(&max_clusters, project_tc_kernel<K>, &cfg) != cudaSuccess || max_clusters < 1)
+    if (cudaOccupancyMaxActiveClusters(&max_clusters, project_tc_kernel<K, G>, &cfg) != cudaSuccess ||
+        max_clusters < 1)
         max_clusters = sms / cs;
+    int64_t clusters = p.n_slots;
     if (clusters > max_clusters) clusters = max_clusters;
     cfg.gridDim = dim3((unsigned)(clusters * cs));
     note_launches(1);
-    e = cudaLaunchKernelEx(&cfg, project_tc_kernel<K>, tmA, tmB, p);
+    e = cudaLaunchKernelEx(&cfg, project_tc_kernel<K, G>, tmA, tmB, p);
     if (e != cudaSuccess) return e;
     return cudaGetLastError();
+}
+
+// Two tiles per stage once every CTA has at least two groups of work; fewer
+// units run one tile per stage so that they spread over all SMs.
+template <int K>
+cudaError_t launch_k(const tda_layer_desc& L, const void* A, const void* B, int64_t N, float* phi,
+                     int64_t ld_phi, unsigned int* err, cudaStream_t s) {
+    int pack = L.T <= 64 ? (int)(kTileM / L.T) : 1;
+    if (pack > 1) {
+        // packed rows are addressed with 32-bit TMA coordinates and the [1][N*T][d]
+        // view's outer stride must stay below 2^40 bytes: split larger batches
+        const int64_t d_max = L.d_in > L.d_out ? L.d_in : L.d_out;
+        int64_t max_n = ((int64_t)1 << 30) / L.T;
+        const int64_t by_stride = (((int64_t)1 << 40) - 1) / (L.T * d_max * 2);
+        if (by_stride < max_n) max_n = by_stride;
+        max_n = max_n / pack * pack;
+        if (max_n < pack) pack = 1;  // one example per tile instead
+        else if (N > max_n) {
+            const size_t a_ex = (size_t)L.T * L.d_in * 2, b_ex = (size_t)L.T * L.d_out * 2;
+            for (int64_t e0 = 0; e0 < N; e0 += max_n) {
+                const int64_t n = N - e0 < max_n ? N - e0 : max_n;
+                cudaError_t e = launch_k<K>(L, (const char*)A + e0 * a_ex, (const char*)B + e0 * b_ex, n,
+                                            phi + e0 * ld_phi, ld_phi, err, s);
+                if (e != cudaSuccess) return e;
+            }
+            return cudaSuccess;
+        }
+    }
+    const int64_t units = pack > 1 ? (N + pack - 1) / pack : N * ((L.T + kTileM - 1) / kTileM);
+    if (units >= 4 * (int64_t)sm_count()) return launch_kg<K, 2>(L, A, B, N, phi, ld_phi, err, s, pack);
+    return launch_kg<K, 1>(L, A, B, N, phi, ld_phi, err, s, pack);
 }
 
 }  // namespace

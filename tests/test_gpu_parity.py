@@ -302,6 +302,14 @@ TC_CASES = [
     (50, 300, 128, 64, 16, "bf16"),     # 4-CTA clusters; more clusters than fit
     (64, 512, 512, 256, 64, "bf16"),    # 2-CTA clusters (the query batch shape)
     (1, 384, 64, 64, 32, "bf16"),       # one example over 2 CTAs, uneven tiles
+    # two token tiles per pipeline stage (many units): groups that straddle examples
+    (250, 300, 64, 72, 32, "bf16"),
+    (700, 256, 64, 128, 64, "bf16"),
+    # short sequences packed several examples to a tile, ragged last tile
+    (2001, 48, 64, 64, 16, "bf16"),     # 2 per tile, 32 rows unused, one tile per stage pair
+    (20001, 8, 64, 64, 16, "bf16"),     # 16 per tile
+    (300, 3, 128, 64, 32, "bf16"),      # 42 per tile
+    (1000, 64, 256, 128, 64, "bf16"),   # 2 per tile, K = 64
 ]
 
 
