@@ -102,6 +102,38 @@ def workload(args):
     }
 
 
+def _cpulist(text):
+    cpus = set()
+    for part in text.strip().split(","):
+        if part:
+            a, _, b = part.partition("-")
+            cpus.update(range(int(a), int(b or a) + 1))
+    return cpus
+
+
+def bind_to_gpu_numa(index):
+    """Pin this thread to the CPUs of the GPU's NUMA node (best effort).
+    Returns (previous affinity or None, node or None)."""
+    try:
+        out = subprocess.run(["nvidia-smi", "--query-gpu=pci.bus_id", "--format=csv,noheader", "-i", str(index)],
+                             capture_output=True, text=True, timeout=30).stdout.strip()
+        dom, rest = out.split(":", 1)
+        dev_path = "/sys/bus/pci/devices/%04x:%s/numa_node" % (int(dom, 16), rest.lower())
+        with open(dev_path) as f:
+            node = int(f.read().strip())
+        if node < 0:
+            return None, None
+        with open("/sys/devices/system/node/node%d/cpulist" % node) as f:
+            cpus = _cpulist(f.read()) & os.sched_getaffinity(0)
+        if not cpus:
+            return None, node
+        saved = os.sched_getaffinity(0)
+        os.sched_setaffinity(0, cpus)
+        return saved, node
+    except (OSError, ValueError, subprocess.SubprocessError):
+        return None, None
+
+
 # ---------------------------------------------------------------------------- clocks
 class ClockSampler:
     FIELDS = ("clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,clocks_event_reasons.hw_slowdown,"
@@ -263,7 +295,9 @@ def route_sweep_main(args):
     ops = [(tda.TDA_OP_PROJECT, "project", (0, 1)), (tda.TDA_OP_SIMILARITY_PROJECTED, "similarity_projected", (0, 1, 2)),
            (tda.TDA_OP_SIMILARITY_EXACT, "similarity_exact", (1, 2))]
     out = {"mode": "route-sweep", "linear": [d, d], "k": k, "n_query": nq, "dtype": "bf16",
-           "calibrated_rates_tflops": [r / 1e12 for r in rates[:3]], "calibrated_bw_gbs": rates[3] / 1e9,
+           "calibrated_rates_tflops": dict(zip(("factored", "materialize", "gram_bf16", "gram_fp32"),
+                                               [r / 1e12 for r in rates[:4]])),
+           "calibrated_bw_gbs": rates[4] / 1e9,
            "points": []}
     stream = torch.cuda.current_stream()
     for T in [int(x) for x in args.sweep_T.split(",")]:
@@ -310,13 +344,13 @@ def route_sweep_main(args):
             rec["calibrated_estimate_s"] = {names[r]: est[r] for r in routes}
             meas = {}
             for r in routes:
-                # pure pair-cost route (exact Gram): fewer queries when one train example is slow
                 n_q = nq
-                if op == tda.TDA_OP_SIMILARITY_EXACT and r == 2:
-                    per = 2.0 * T * T * 2 * d / 20e12  # seconds per pair at a conservative 20 TFLOP/s
-                    n_q = max(1, min(nq, int(0.5 / per)))
-                n1 = 1 if op != tda.TDA_OP_PROJECT else min(P, 8)
+                # start with enough train examples to fill the GPU (the fit below is in the train count)
+                n1 = min(P, 8)
                 wsb = max(tda.tda_workspace_size(op, L, tda.TDA_BF16, n_q, P, r), 256)
+                if op == tda.TDA_OP_SIMILARITY_EXACT and r == 1:
+                    # room for 128 materialised train gradients per chunk next to the queries'
+                    wsb = tda.tda_workspace_size(op, L, tda.TDA_BF16, n_q + 127, P, r)
                 if op == tda.TDA_OP_SIMILARITY_PROJECTED:
                     wsb = max(wsb, min(2 << 30, tda.tda_workspace_size(op, L, tda.TDA_BF16, n_q, P, r) * 16))
                 ws = torch.empty(wsb, dtype=torch.uint8, device=dev)
@@ -520,6 +554,9 @@ def main():
     # ---- e2e through tda_project_host with pinned host factors
     e2e = None
     if not args.no_e2e and not args.project_only:
+        # pinned pools on the host memory nearest the GPU: this thread runs on the
+        # GPU's NUMA node while the pools are allocated and first touched
+        saved_aff, numa = bind_to_gpu_numa(local)
         P = min(args.pool, N)
         pools = []
         for li, (_, di, do) in enumerate(LINEARS):
@@ -554,14 +591,17 @@ def main():
 
         e2e_step()
         # raw pinned-host -> device bandwidth on this machine, the ceiling of the e2e leg
+        # (best of five copies of one pool, CUDA events on the copying stream)
         hb = pools[0][0]
-        db = torch.empty_like(hb, device=dev)
-        torch.cuda.synchronize()
-        t0 = time.perf_counter()
-        for _ in range(3):
+        db = torch.empty(hb.shape, dtype=hb.dtype, device=dev)
+        h2d_gbs = 0.0
+        for _ in range(5):
+            c0, c1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            c0.record(stream)
             db.copy_(hb, non_blocking=True)
-        torch.cuda.synchronize()
-        h2d_gbs = 3 * hb.numel() * 2 / (time.perf_counter() - t0) / 1e9
+            c1.record(stream)
+            c1.synchronize()
+            h2d_gbs = max(h2d_gbs, hb.numel() * 2 / (c0.elapsed_time(c1) * 1e-3) / 1e9)
         del db
         if dist:
             dist.barrier()
@@ -578,7 +618,9 @@ def main():
         e2e = {"value": world * N / e2e_s, "unit": "examples/s", "h2d_bytes_per_step": h2d,
                "d2h_bytes_per_step": Nq * args.topk * 8, "ms_per_step": e2e_s * 1e3,
                "host_pool_examples": P, "h2d_gbs_measured": h2d_gbs,
-               "h2d_bound_examples_per_s": world * N / (h2d / (h2d_gbs * 1e9))}
+               "h2d_bound_examples_per_s": world * N / (h2d / (h2d_gbs * 1e9)), "host_numa_node": numa}
+        if saved_aff is not None:
+            os.sched_setaffinity(0, saved_aff)
 
     cpu = None
     if rank == 0 and world == 1 and not args.no_cpu_baseline and not args.project_only:

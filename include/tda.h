@@ -198,6 +198,14 @@ tda_status tda_similarity_exact(const tda_layer_desc* L, tda_dtype dtype,
                                 float* S, int64_t ld_S, float beta, tda_route_id route,
                                 void* ws, size_t ws_bytes, void* stream);
 
+/* Which kernel the GRAM route of tda_similarity_exact runs: 1 = the tcgen05
+ * kernel (bf16 factors, T a power of two, d_in and d_out multiples of 8,
+ * 16-byte aligned factors, sm_103), whose two token Grams (A_q A_i^T, B_q B_i^T)
+ * are tensor-core GEMMs with fp32 accumulation; 0 = the CUDA-core kernel.
+ * Host only. */
+int32_t tda_similarity_gram_engine(const tda_layer_desc* L, tda_dtype dtype, const void* Aq, const void* Bq,
+                                   const void* At, const void* Bt);
+
 /* ---------------------------------------------------------------------------
  * tda_similarity_projected -- inner products of PROJECTED gradients,
  *   S[q][i] = beta*S[q][i] + <Phi_q, Phi_i>,  Phi = P_g DW P_a^T (Eq. 2),
@@ -333,8 +341,10 @@ tda_status tda_route(const tda_layer_desc* L, tda_op op, int64_t n1, int64_t n2,
  * launches of the route kernels inside the caller's scratch `ws` (at least
  * TDA_CALIBRATE_WS_BYTES bytes, contents destroyed), synchronises `stream`,
  * then switches tda_route to the time model. rates_out (host, may be NULL)
- * receives 4 doubles: flop/s of the factored, materialise and Gram kernels
- * and the streaming bytes/s of the factored kernel. */
+ * receives 5 doubles: flop/s of the factored and materialise routes, of the
+ * Gram route on bf16 factors (exact similarity; tensor cores on sm_103), of
+ * the Gram route on fp32 factors (projected factors, fp32 layers, norms), and
+ * the streaming bytes/s of the factored kernel. */
 #define TDA_CALIBRATE_WS_BYTES ((size_t)768 << 20)
 tda_status tda_route_calibrate(void* ws, size_t ws_bytes, void* stream, double* rates_out);
 /* 0 = flop model (the paper's), 1 = calibrated time model. */

@@ -18,7 +18,7 @@ __all__ = [
     "tda_project_engine", "tda_project_host_ws_min", "tda_project_host", "tda_noalloc_scratch_bytes",
     "tda_project_materialized_noalloc",
     "tda_similarity_projected", "tda_similarity_exact", "tda_norms", "tda_cosine", "tda_precondition_state_bytes", "tda_precondition",
-    "tda_precondition_info", "tda_score", "tda_score_engine", "tda_topk", "tda_route", "tda_route_calibrate",
+    "tda_precondition_info", "tda_score", "tda_score_engine", "tda_similarity_gram_engine", "tda_topk", "tda_route", "tda_route_calibrate",
     "tda_route_set_model", "tda_device_status", "tda_selftest_bounded_wait", "tda_last_error", "tda_version", "tda_launch_count",
 ]
 
@@ -92,6 +92,7 @@ def load() -> ctypes.CDLL:
             "tda_score": (I32, [P, I32, I64, I64, P, I64, I64, I64, P, I64, F, P]),
             "tda_topk": (I32, [P, I64, I64, I64, I32, P, P, P]),
             "tda_score_engine": (I32, [P, I32, I64, I64, P, I64, I64, I64]),
+            "tda_similarity_gram_engine": (I32, [LP, I32, P, P, P, P]),
             "tda_route": (I32, [LP, I32, I64, I64, I32, ctypes.POINTER(I32), ctypes.POINTER(D)]),
             "tda_route_calibrate": (I32, [P, SZ, P, ctypes.POINTER(D)]),
             "tda_route_set_model": (I32, [I32]),
@@ -224,6 +225,10 @@ def tda_score(Qhat, q_dtype, n_q, ld_q, Phi, n_t, ld_phi, D, S, ld_S, beta=0.0, 
                             beta, _stream(stream)))
 
 
+def tda_similarity_gram_engine(L, dtype, Aq, Bq, At, Bt) -> int:
+    return int(load().tda_similarity_gram_engine(ctypes.byref(L), dtype, _ptr(Aq), _ptr(Bq), _ptr(At), _ptr(Bt)))
+
+
 def tda_score_engine(Qhat, q_dtype, n_q, ld_q, Phi, n_t, ld_phi, D) -> int:
     return int(load().tda_score_engine(_ptr(Qhat), q_dtype, n_q, ld_q, _ptr(Phi), n_t, ld_phi, D))
 
@@ -240,7 +245,7 @@ def tda_route(L, op, n1, n2, dtype) -> tuple[int, list[float]]:
 
 
 def tda_route_calibrate(ws, ws_bytes, stream=None) -> list[float]:
-    rates = (ctypes.c_double * 4)()
+    rates = (ctypes.c_double * 5)()
     _check(load().tda_route_calibrate(_ptr(ws), ws_bytes, _stream(stream), rates))
     return list(rates)
 

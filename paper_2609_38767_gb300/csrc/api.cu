@@ -53,17 +53,20 @@ unsigned int* device_error_word() {
 // ---------------------------------------------------------------------------
 static std::mutex g_route_mu;
 static int g_route_model = 0;
-static double g_rate[3] = {0, 0, 0};  // flop/s of the factored, materialise, Gram kernels
+// flop/s of the factored and materialise routes, of the Gram route on bf16
+// factors (tensor cores) and on fp32 factors (projected factors, CUDA cores)
+static double g_rate[4] = {0, 0, 0, 0};
 static double g_bw = 0;               // bytes/s
 
 struct RouteCounts {
     double flops[3];
     double bytes[3];
+    int gram_rate;  // which measured rate the Gram route runs at (2 or 3)
 };
 
-void set_route_rates(const double rate[3], double bw) {
+void set_route_rates(const double rate[4], double bw) {
     std::lock_guard<std::mutex> lock(g_route_mu);
-    for (int r = 0; r < 3; ++r) g_rate[r] = rate[r];
+    for (int r = 0; r < 4; ++r) g_rate[r] = rate[r];
     g_bw = bw;
     g_route_model = (rate[0] > 0 && bw > 0) ? 1 : 0;
 }
@@ -79,6 +82,11 @@ static RouteCounts route_counts(const tda_layer_desc& L, tda_op op, int64_t n1, 
     const double build = 2.0 * T * Ni * No;
     const double dense = 2.0 * No * Ni * ka + 2.0 * No * ka * kg;
     RouteCounts c;
+    // the unprojected Gram of bf16 factors runs on tensor cores when T is a power of two
+    c.gram_rate = (op == TDA_OP_SIMILARITY_EXACT && dt == TDA_BF16 && L.T > 0 && (L.T & (L.T - 1)) == 0 &&
+                   L.d_in % 8 == 0 && L.d_out % 8 == 0)
+                      ? 2
+                      : 3;
     if (op == TDA_OP_PROJECT) {
         c.flops[0] = B1 * (proj + contract);
         c.flops[1] = B1 * (build + dense);
@@ -157,8 +165,8 @@ static tda_route_id choose(const RouteCounts& c, double* cost_out) {
     for (int r = 0; r < 3; ++r) {
         if (c.flops[r] < 0) {
             cost[r] = -1;
-        } else if (g_route_model == 1 && g_rate[r] > 0 && g_bw > 0) {
-            cost[r] = std::fmax(c.flops[r] / g_rate[r], c.bytes[r] / g_bw);
+        } else if (g_route_model == 1 && g_rate[r == 2 ? c.gram_rate : r] > 0 && g_bw > 0) {
+            cost[r] = std::fmax(c.flops[r] / g_rate[r == 2 ? c.gram_rate : r], c.bytes[r] / g_bw);
         } else {
             cost[r] = c.flops[r];
         }
@@ -327,9 +335,16 @@ tda_status tda_similarity_exact(const tda_layer_desc* L, tda_dtype dtype, const 
         // DW = 0: the inner products are 0
         return cuda_check(launch_score(S, TDA_F32, n_q, 0, S, n_t, 0, 0, S, ld_S, beta, s), "zero S");
     }
-    if (route == TDA_ROUTE_GRAM)
+    if (route == TDA_ROUTE_GRAM) {
+        if (gram_tc_supported(*L, dtype, Aq, Bq, At, Bt)) {
+            unsigned int* err = device_error_word();
+            if (!err) return fail(TDA_ERR_CUDA, "device error word unavailable");
+            return cuda_check(launch_gram_tc(*L, Aq, Bq, n_q, At, Bt, n_t, S, ld_S, beta, 1.f, err, s),
+                              "similarity (gram, tensor cores)");
+        }
         return cuda_check(launch_similarity_gram(*L, dtype, Aq, Bq, n_q, At, Bt, n_t, S, ld_S, beta, s),
                           "similarity (gram)");
+    }
     if (route == TDA_ROUTE_MATERIALIZE) {
         const size_t need = similarity_materialize_ws_bytes(*L, n_q, 1);
         if (!ws || ws_bytes < need)
@@ -623,6 +638,12 @@ tda_status tda_score(const void* Qhat, tda_dtype q_dtype, int64_t n_q, int64_t l
     return cuda_check(launch_score(Qhat, q_dtype, n_q, ld_q, Phi, n_t, ld_phi, D, S, ld_S, beta,
                                    (cudaStream_t)stream),
                       "score");
+}
+
+int32_t tda_similarity_gram_engine(const tda_layer_desc* L, tda_dtype dtype, const void* Aq, const void* Bq,
+                                   const void* At, const void* Bt) {
+    if (!L || L->T < 1) return 0;
+    return gram_tc_supported(*L, dtype, Aq, Bq, At, Bt) ? 1 : 0;
 }
 
 int32_t tda_score_engine(const void* Qhat, tda_dtype q_dtype, int64_t n_q, int64_t ld_q, const float* Phi,

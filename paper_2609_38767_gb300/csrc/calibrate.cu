@@ -6,7 +6,7 @@
 #include "tda_internal.cuh"
 
 namespace tda {
-void set_route_rates(const double rate[3], double bw);
+void set_route_rates(const double rate[4], double bw);
 }
 
 using namespace tda;
@@ -56,19 +56,22 @@ extern "C" tda_status tda_route_calibrate(void* ws, size_t ws_bytes, void* strea
     float* S = (float*)(base + TDA_CALIBRATE_WS_BYTES - (1u << 20));
 
     EventTimer ev;
-    double secs[3] = {0, 0, 0};
-    double flops[3] = {0, 0, 0};
+    double secs[4] = {0, 0, 0, 0};
+    double flops[4] = {0, 0, 0, 0};
     double bytes_a = 0;
-    for (int route = 0; route < 3; ++route) {
+    for (int route = 0; route < 4; ++route) {
         for (int rep = 0; rep < 4; ++rep) {
             if (rep == 1) cudaEventRecord(ev.a, s);
             if (route == 0) {
                 st = tda_project(&L, TDA_BF16, A, B, Nf, phi, 1024, TDA_ROUTE_FACTORED, nullptr, 0, s);
             } else if (route == 1) {
                 st = tda_project(&L, TDA_BF16, A, B, 8, phi, 1024, TDA_ROUTE_MATERIALIZE, rest, rest_bytes, s);
-            } else {
-                st = tda_similarity_exact(&L, TDA_BF16, A, B, 2, A, B, 16, S, 16, 0.f, TDA_ROUTE_GRAM,
+            } else if (route == 2) {
+                st = tda_similarity_exact(&L, TDA_BF16, A, B, 8, A, B, 256, S, 256, 0.f, TDA_ROUTE_GRAM,
                                           nullptr, 0, s);
+            } else {  // Gram of projected (fp32) factors
+                st = tda_similarity_projected(&L, TDA_BF16, A, B, 8, A, B, 64, S, 64, 0.f, TDA_ROUTE_GRAM, rest,
+                                              rest_bytes, s);
             }
             if (st) return st;
         }
@@ -81,17 +84,19 @@ extern "C" tda_status tda_route_calibrate(void* ws, size_t ws_bytes, void* strea
     const double T = 128, d = 1024, k = 32;
     flops[0] = Nf * (2 * T * (d * k + d * k) + 2 * T * k * k);
     flops[1] = 8 * (2 * T * d * d + 2 * d * d * k + 2 * d * k * k);
-    flops[2] = 2 * 16 * 2 * T * T * (d + d);
+    flops[2] = 8 * 256 * 2 * T * T * (d + d);
+    flops[3] = (8 + 64) * 2 * T * (d * k + d * k) + 8 * 64 * 2 * T * T * (k + k);
     bytes_a = Nf * (T * (d + d) * 2 + 4 * k * k);
-    double rate[3];
-    for (int r = 0; r < 3; ++r) rate[r] = secs[r] > 0 ? flops[r] / secs[r] : 0;
+    double rate[4];
+    for (int r = 0; r < 4; ++r) rate[r] = secs[r] > 0 ? flops[r] / secs[r] : 0;
     const double bw = secs[0] > 0 ? bytes_a / secs[0] : 0;
     set_route_rates(rate, bw);
     if (rates_out) {
         rates_out[0] = rate[0];
         rates_out[1] = rate[1];
         rates_out[2] = rate[2];
-        rates_out[3] = bw;
+        rates_out[3] = rate[3];
+        rates_out[4] = bw;
     }
     return TDA_OK;
 }

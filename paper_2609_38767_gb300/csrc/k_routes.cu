@@ -320,6 +320,20 @@ cudaError_t launch_similarity_materialized(const tda_layer_desc& L, tda_dtype dt
     int64_t chunk = room < 65535 ? room : 65535;
     float* Gq = (float*)ws;
     float* Gt = Gq + n_q * gsz;
+    // The Frobenius dots have few rows and very long ones: split the feature
+    // axis over many CTAs when the chunk leaves one train gradient's room for
+    // the partial sums.
+    int splits = score_splitk_splits(n_q, chunk, gsz);
+    float* part = nullptr;
+    if (splits > 1) {
+        const size_t need = (size_t)splits * (size_t)n_q * (size_t)chunk;
+        if (chunk > 1 && need <= (size_t)gsz) {
+            --chunk;
+            part = Gt + chunk * gsz;
+        } else {
+            splits = 1;
+        }
+    }
     for (int64_t q0 = 0; q0 < n_q; q0 += 65535) {
         const int64_t cnt = (n_q - q0) < 65535 ? (n_q - q0) : 65535;
         if (dt == TDA_BF16)
@@ -333,7 +347,7 @@ cudaError_t launch_similarity_materialized(const tda_layer_desc& L, tda_dtype dt
             launch_materialize<__nv_bfloat16>(At, Bt, i0, cnt, L, Gt, s);
         else
             launch_materialize<float>(At, Bt, i0, cnt, L, Gt, s);
-        cudaError_t e = launch_score(Gq, TDA_F32, n_q, gsz, Gt, cnt, gsz, gsz, S + i0, ld_S, beta, s);
+        cudaError_t e = launch_score_splitk(Gq, n_q, gsz, Gt, cnt, gsz, gsz, S + i0, ld_S, beta, splits, part, s);
         if (e != cudaSuccess) return e;
     }
     return cudaGetLastError();

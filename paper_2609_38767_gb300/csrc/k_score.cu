@@ -32,10 +32,17 @@ template <typename TQ, typename TA>
 __global__ void __launch_bounds__(kSThreads)
 score_kernel(const TQ* __restrict__ Q, int64_t n_q, int64_t ld_q, const float* __restrict__ P,
              int64_t n_t, int64_t ld_p, int64_t D, float* __restrict__ S, int64_t ld_S,
-             float beta) {
+             float beta, int64_t kslice, int64_t slab) {
     __shared__ TA Qs[kSK][kTQ + 1];
     __shared__ TA Ps[kSK][kTT + 1];
     const int tid = threadIdx.x;
+    {   // split K: slice blockIdx.z of the features into its own slab of S
+        const int64_t k0 = (int64_t)blockIdx.z * kslice;
+        Q += k0;
+        P += k0;
+        D = D - k0 < kslice ? D - k0 : kslice;
+        S += (int64_t)blockIdx.z * slab;
+    }
     const int64_t q0 = (int64_t)blockIdx.y * kTQ, i0 = (int64_t)blockIdx.x * kTT;
     const int tq = tid >> 5, tt = tid & 31;
     const bool vq = (sizeof(TQ) == 4) && ((ld_q & 3) == 0) && (((uintptr_t)Q & 15) == 0);
@@ -205,10 +212,55 @@ cudaError_t launch_score(const void* Qhat, tda_dtype qdt, int64_t n_q, int64_t l
     note_launches(1);
     if (qdt == TDA_F64)
         score_kernel<double, double><<<grid, kSThreads, 0, s>>>(
-            (const double*)Qhat, n_q, ld_q, Phi, n_t, ld_phi, D, S, ld_S, beta);
+            (const double*)Qhat, n_q, ld_q, Phi, n_t, ld_phi, D, S, ld_S, beta, D, 0);
     else
         score_kernel<float, float><<<grid, kSThreads, 0, s>>>(
-            (const float*)Qhat, n_q, ld_q, Phi, n_t, ld_phi, D, S, ld_S, beta);
+            (const float*)Qhat, n_q, ld_q, Phi, n_t, ld_phi, D, S, ld_S, beta, D, 0);
+    return cudaGetLastError();
+}
+
+namespace {
+// S[q][i] = beta * S[q][i] + sum_z part[z][q][i] (slabs of n_q x n_t, fixed order)
+__global__ void sum_slabs_kernel(const float* __restrict__ part, int splits, int64_t n_q, int64_t n_t,
+                                 float* __restrict__ S, int64_t ld_S, float beta) {
+    const int64_t total = n_q * n_t;
+    for (int64_t e = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; e < total; e += (int64_t)gridDim.x * blockDim.x) {
+        float v = 0.f;
+        for (int z = 0; z < splits; ++z) v += part[z * total + e];
+        const int64_t q = e / n_t, i = e - q * n_t;
+        float* dst = S + q * ld_S + i;
+        *dst = beta == 0.f ? v : beta * (*dst) + v;
+    }
+}
+}  // namespace
+
+int score_splitk_splits(int64_t n_q, int64_t n_t, int64_t D) {
+    const int64_t tiles = ((n_t + kTT - 1) / kTT) * ((n_q + kTQ - 1) / kTQ);
+    int64_t z = 608 / (tiles > 0 ? tiles : 1);
+    const int64_t by_d = D / 4096;  // at least 4096 features per slice
+    if (z > by_d) z = by_d;
+    if (z > 256) z = 256;
+    return z < 2 ? 1 : (int)z;
+}
+
+// fp32 score with the feature axis split over `splits` CTAs per tile: for
+// few, very long rows (inner products of materialised gradients). part: device
+// scratch of splits * n_q * n_t floats.
+cudaError_t launch_score_splitk(const float* Q, int64_t n_q, int64_t ld_q, const float* Phi, int64_t n_t,
+                                int64_t ld_phi, int64_t D, float* S, int64_t ld_S, float beta, int splits,
+                                float* part, cudaStream_t s) {
+    if (n_q == 0 || n_t == 0) return cudaSuccess;
+    if (splits <= 1) return launch_score(Q, TDA_F32, n_q, ld_q, Phi, n_t, ld_phi, D, S, ld_S, beta, s);
+    int64_t kslice = (D + splits - 1) / splits;
+    kslice = (kslice + kSK - 1) / kSK * kSK;
+    const int z = (int)((D + kslice - 1) / kslice);
+    dim3 grid((unsigned)((n_t + kTT - 1) / kTT), (unsigned)((n_q + kTQ - 1) / kTQ), (unsigned)z);
+    note_launches(2);
+    score_kernel<float, float><<<grid, kSThreads, 0, s>>>(Q, n_q, ld_q, Phi, n_t, ld_phi, D, part, n_t, 0.f, kslice,
+                                                          n_q * n_t);
+    int64_t blocks = (n_q * n_t + 255) / 256;
+    if (blocks > 4096) blocks = 4096;
+    sum_slabs_kernel<<<(unsigned)blocks, 256, 0, s>>>(part, z, n_q, n_t, S, ld_S, beta);
     return cudaGetLastError();
 }
 

@@ -87,6 +87,12 @@ cudaError_t launch_similarity_materialized(const tda_layer_desc& L, tda_dtype dt
                                            const void* Bq, int64_t n_q, const void* At,
                                            const void* Bt, int64_t n_t, float* S, int64_t ld_S,
                                            float beta, void* ws, size_t ws_bytes, cudaStream_t s);
+// Route (c) on tcgen05 for bf16 factors with T a power of two (k_gram_tc.cu).
+bool gram_tc_supported(const tda_layer_desc& L, tda_dtype dt, const void* Aq, const void* Bq, const void* At,
+                       const void* Bt);
+cudaError_t launch_gram_tc(const tda_layer_desc& L, const void* Aq, const void* Bq, int64_t n_q, const void* At,
+                           const void* Bt, int64_t n_t, float* S, int64_t ld_S, float beta, float alpha,
+                           unsigned int* err, cudaStream_t s);
 cudaError_t launch_similarity_gram(const tda_layer_desc& L, tda_dtype dt, const void* Aq,
                                    const void* Bq, int64_t n_q, const void* At, const void* Bt,
                                    int64_t n_t, float* S, int64_t ld_S, float beta, cudaStream_t s);
@@ -132,6 +138,10 @@ bool score_tc_supported(tda_dtype qdt, const void* Qhat, int64_t n_q, int64_t ld
                         int64_t ld_phi, int64_t D);
 cudaError_t launch_score_tc(const float* Qhat, int64_t n_q, int64_t ld_q, const float* Phi, int64_t n_t, int64_t ld_phi,
                             int64_t D, float* S, int64_t ld_S, float beta, unsigned int* err, cudaStream_t s);
+int score_splitk_splits(int64_t n_q, int64_t n_t, int64_t D);
+cudaError_t launch_score_splitk(const float* Q, int64_t n_q, int64_t ld_q, const float* Phi, int64_t n_t,
+                                int64_t ld_phi, int64_t D, float* S, int64_t ld_S, float beta, int splits,
+                                float* part, cudaStream_t s);
 cudaError_t launch_topk(const float* S, int64_t n_q, int64_t n_t, int64_t ld_S, int32_t k,
                         int32_t* idx, float* val, cudaStream_t s);
 

@@ -132,8 +132,9 @@ def test_project_leading_dimension_and_edge_sizes(dev, orc):
 # ------------------------------------------------------------------ exact similarity
 @pytest.mark.parametrize("dtype", ["f32", "bf16"])
 @pytest.mark.parametrize("route", [tda.TDA_ROUTE_GRAM, tda.TDA_ROUTE_MATERIALIZE, tda.TDA_ROUTE_AUTO])
-def test_similarity_exact_matches_oracle(dev, orc, dtype, route):
-    nq, nt, T, di, do = 3, 5, 21, 40, 24
+@pytest.mark.parametrize("shape", [(3, 5, 21, 40, 24), (3, 5, 7, 256, 264)])  # 2nd: split-K Frobenius dots
+def test_similarity_exact_matches_oracle(dev, orc, dtype, route, shape):
+    nq, nt, T, di, do = shape
     Aq, Bq = make_factors(nq, T, di, do, dtype, stream=6, query=True)
     At, Bt = make_factors(nt, T, di, do, dtype, stream=6)
     L = tda.LayerDesc(di, do, T, 1, 1)
@@ -473,3 +474,31 @@ def test_norms_edge_cases(dev, orc):
                   tda.TDA_ROUTE_MATERIALIZE, ws, wsb)
     tda.tda_device_status()
     np.testing.assert_allclose(out.cpu().numpy(), orc.sq_norms(A, B, "gram"), rtol=1e-5)
+
+
+@pytest.mark.gpu
+@pytest.mark.parametrize("nq,nt,T,di,do,beta", [
+    (3, 37, 1, 64, 40, 0.0),      # 128 queries per tile row group of 1, 256 train per tile
+    (5, 70, 8, 128, 64, 1.0),     # ragged query and train tiles
+    (17, 33, 16, 64, 64, 0.0),    # three query tiles
+    (3, 9, 32, 64, 128, 0.5),
+    (4, 11, 64, 64, 64, 0.0),     # a query's rows span two epilogue warps
+    (2, 5, 128, 136, 64, 1.0),    # ragged K chunk (136 = 2 x 64 + 8)
+    (2, 3, 256, 64, 72, 0.0),     # one (query, train) pair per unit
+    (2, 2, 512, 64, 64, 1.0),     # 4 x 2 tile pairs per unit
+])
+def test_gram_tensor_core_matches_oracle(dev, orc, nq, nt, T, di, do, beta):
+    # route (c) of Eq. 4 on tcgen05: both token Grams as bf16 GEMMs, fp32 accumulation
+    Aq, Bq = make_factors(nq, T, di, do, "bf16", stream=31, query=True)
+    At, Bt = make_factors(nt, T, di, do, "bf16", stream=31)
+    L = tda.LayerDesc(di, do, T, 1, 1)
+    d = [to_dev(x, "bf16", dev) for x in (Aq, Bq, At, Bt)]
+    assert tda.tda_similarity_gram_engine(L, tda.TDA_BF16, *d) == 1
+    S0 = np.random.default_rng(T).standard_normal((nq, nt + 2)).astype(np.float32)
+    S = torch.from_numpy(S0).to(dev)
+    tda.tda_similarity_exact(L, tda.TDA_BF16, d[0], d[1], nq, d[2], d[3], nt, S, nt + 2, beta, tda.TDA_ROUTE_GRAM)
+    tda.tda_device_status()
+    ref = orc.similarity(*(synth.to_f64(x, "bf16") for x in (Aq, Bq, At, Bt))) + beta * S0[:, :nt]
+    got = S.cpu().numpy()
+    assert rel_fro(got[:, :nt], ref) <= 1e-5
+    np.testing.assert_array_equal(got[:, nt:], S0[:, nt:])
