@@ -295,6 +295,64 @@ tda_status tda_precondition_info(int32_t n_layers, int64_t D, tda_dtype state_dt
                                  double* info, void* stream);
 
 /* ---------------------------------------------------------------------------
+ * K-FAC and EK-FAC on the projected factors. The paper runs both
+ * Kronecker-factored curvature methods (Martens & Grosse 2015; George et al.
+ * 2018) on the projected pair (a~_t, g~_t) unchanged (App. A.2) and damps
+ * each layer by a multiple of its mean eigenvalue (App. B.2, 0.1 for EK-FAC).
+ * Per layer, with a~_t = P_a a_t (k_in) and g~_t = P_g g_t (k_out):
+ *   C_a = (1/M) sum a~_t a~_t^T,  C_g = (1/M) sum g~_t g~_t^T  (M = N*T token
+ *   positions of the N training examples seen),
+ *   C_a = U_a diag(alpha) U_a^T, C_g = U_g diag(gamma) U_g^T,
+ *   K-FAC eigenvalues  Lam[r][c] = gamma_r alpha_c,
+ *   EK-FAC eigenvalues Lam[r][c] = (1/N) sum_i ((U_g^T Phi_i U_a)[r][c])^2,
+ *   lambda = lambda_abs + lambda_rel * mean(Lam),
+ *   Qhat = U_g [(U_g^T Q U_a) / (Lam + lambda)] U_a^T  per query feature
+ *   (Q, Qhat, Phi: k_out x k_in row-major, index r*k_in + c, as tda_project).
+ *
+ * `state`: device buffer of tda_kfac_state_bytes(k_in, k_out) bytes, 16-byte
+ * aligned, fp64: an 8-double header (M, N, ...), the factor sums, the
+ * eigenbases and eigenvalues, the EK-FAC sums. Calls in order of use:
+ *   tda_kfac_reset                 zero the state.
+ *   tda_kfac_accumulate_factors    add the factor covariance sums of N training
+ *                                  examples (A, B as tda_project). ws >=
+ *                                  tda_kfac_workspace_size(L, dtype). Call once
+ *                                  per streamed chunk.
+ *   tda_project_kfac               tda_project (factored route) that also adds
+ *                                  the factor covariance sums, in one pass over
+ *                                  the factors (bf16, the tensor-core kernel's
+ *                                  shapes; TDA_ERR_UNSUPPORTED otherwise).
+ *   tda_kfac_eigen                 C = sums / M; both eigendecompositions
+ *                                  (parallel cyclic Jacobi in fp64, at most 60
+ *                                  sweeps; the sweep count, or -1 if it did not
+ *                                  converge, lands in header[2] (a) and [3] (g)).
+ *                                  Resets the EK-FAC sums.
+ *   tda_kfac_accumulate_eigenvalues  EK-FAC: add sum_i (U_g^T Phi_i U_a)^2 over n
+ *                                  training features (rows of stride ld_phi).
+ * ws (device scratch, 256-byte aligned) of tda_kfac_workspace_size(L, dtype)
+ * bytes serves every call that takes one; more lets accumulate_factors
+ * process more examples per pass.
+ *   tda_kfac_apply                 Qhat for n_q query rows; kind TDA_KFAC or
+ *                                  TDA_EKFAC.
+ * Supports 1 <= k_in, k_out <= 128. Errors: TDA_ERR_INVALID_ARG for bad sizes
+ * or pointers, TDA_ERR_WORKSPACE for a short ws.
+ * ------------------------------------------------------------------------- */
+#define TDA_KFAC 0
+#define TDA_EKFAC 1
+size_t tda_kfac_state_bytes(int32_t k_in, int32_t k_out);
+size_t tda_kfac_workspace_size(const tda_layer_desc* L, tda_dtype dtype);
+tda_status tda_kfac_reset(int32_t k_in, int32_t k_out, void* state, void* stream);
+tda_status tda_kfac_accumulate_factors(const tda_layer_desc* L, tda_dtype dtype, const void* A, const void* B,
+                                       int64_t N, void* state, void* ws, size_t ws_bytes, void* stream);
+tda_status tda_project_kfac(const tda_layer_desc* L, tda_dtype dtype, const void* A, const void* B, int64_t N,
+                            float* phi, int64_t ld_phi, void* state, void* ws, size_t ws_bytes, void* stream);
+tda_status tda_kfac_eigen(int32_t k_in, int32_t k_out, void* state, void* stream);
+tda_status tda_kfac_accumulate_eigenvalues(int32_t k_in, int32_t k_out, void* state, const float* phi,
+                                           int64_t n, int64_t ld_phi, void* ws, size_t ws_bytes, void* stream);
+tda_status tda_kfac_apply(int32_t kind, int32_t k_in, int32_t k_out, const void* state, double lambda_abs,
+                          double lambda_rel, const float* q, int64_t n_q, int64_t ld_q, float* qhat,
+                          int64_t ld_qhat, void* stream);
+
+/* ---------------------------------------------------------------------------
  * tda_score -- S[q][i] = beta*S[q][i] + sum_f Qhat[q][f] Phi[i][f]
  * (gradient inner products; GradDot when Qhat = Q, Sec. 3.2 / Eq. 4).
  *   Qhat  device, n_q rows of D, q_dtype TDA_F32 or TDA_F64, row stride ld_q.

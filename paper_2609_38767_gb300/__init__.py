@@ -17,7 +17,9 @@ __all__ = [
     "LayerDesc", "TdaError", "load", "tda_proj_entries", "tda_workspace_size", "tda_project",
     "tda_project_engine", "tda_project_host_ws_min", "tda_project_host", "tda_noalloc_scratch_bytes",
     "tda_project_materialized_noalloc",
-    "tda_similarity_projected", "tda_similarity_exact", "tda_norms", "tda_cosine", "tda_precondition_state_bytes", "tda_precondition",
+    "tda_similarity_projected", "tda_similarity_exact", "tda_norms", "tda_cosine", "tda_kfac_state_bytes", "tda_kfac_workspace_size",
+    "tda_kfac_reset", "tda_kfac_accumulate_factors", "tda_project_kfac", "tda_kfac_eigen",
+    "tda_kfac_accumulate_eigenvalues", "tda_kfac_apply", "tda_precondition_state_bytes", "tda_precondition",
     "tda_precondition_info", "tda_score", "tda_score_engine", "tda_similarity_gram_engine", "tda_topk", "tda_route", "tda_route_calibrate",
     "tda_route_set_model", "tda_device_status", "tda_selftest_bounded_wait", "tda_last_error", "tda_version", "tda_launch_count",
 ]
@@ -35,6 +37,7 @@ TDA_ROUTE_AUTO, TDA_ROUTE_FACTORED, TDA_ROUTE_MATERIALIZE, TDA_ROUTE_GRAM = -1, 
 TDA_OP_PROJECT, TDA_OP_SIMILARITY_PROJECTED, TDA_OP_SIMILARITY_EXACT = 0, 1, 2
 TDA_OP_NORM_PROJECTED, TDA_OP_NORM_EXACT = 3, 4
 TDA_PC_RESET, TDA_PC_FIT_ACCUM, TDA_PC_FACTOR, TDA_PC_APPLY = 0, 1, 2, 3
+TDA_KFAC, TDA_EKFAC = 0, 1
 TDA_CALIBRATE_WS_BYTES = 768 << 20
 _STATUS = {0: "TDA_OK", 1: "TDA_ERR_INVALID_ARG", 2: "TDA_ERR_UNSUPPORTED", 3: "TDA_ERR_WORKSPACE",
            4: "TDA_ERR_CUDA", 5: "TDA_ERR_NOT_SPD", 6: "TDA_ERR_TIMEOUT"}
@@ -87,6 +90,14 @@ def load() -> ctypes.CDLL:
             "tda_cosine": (I32, [P, I64, I64, I64, P, P, P]),
             "tda_similarity_exact": (I32, [LP, I32, P, P, I64, P, P, I64, P, I64, F, I32, P, SZ, P]),
             "tda_precondition_state_bytes": (SZ, [I64, I32]),
+            "tda_kfac_state_bytes": (SZ, [I32, I32]),
+            "tda_kfac_workspace_size": (SZ, [LP, I32]),
+            "tda_kfac_reset": (I32, [I32, I32, P, P]),
+            "tda_kfac_accumulate_factors": (I32, [LP, I32, P, P, I64, P, P, SZ, P]),
+            "tda_project_kfac": (I32, [LP, I32, P, P, I64, P, I64, P, P, SZ, P]),
+            "tda_kfac_eigen": (I32, [I32, I32, P, P]),
+            "tda_kfac_accumulate_eigenvalues": (I32, [I32, I32, P, P, I64, I64, P, SZ, P]),
+            "tda_kfac_apply": (I32, [I32, I32, I32, P, D, D, P, I64, I64, P, I64, P]),
             "tda_precondition": (I32, [I32, I32, I64, I32, P, P, I64, I64, I64, D, D, P, I64, I64, P, I64, P]),
             "tda_precondition_info": (I32, [I32, I64, I32, P, ctypes.POINTER(D), P]),
             "tda_score": (I32, [P, I32, I64, I64, P, I64, I64, I64, P, I64, F, P]),
@@ -201,6 +212,42 @@ def tda_similarity_exact(L, dtype, Aq, Bq, n_q, At, Bt, n_t, S, ld_S, beta=0.0, 
                          ws=None, ws_bytes=0, stream=None):
     _check(load().tda_similarity_exact(ctypes.byref(L), dtype, _ptr(Aq), _ptr(Bq), n_q, _ptr(At), _ptr(Bt),
                                        n_t, _ptr(S), ld_S, beta, route, _ptr(ws), ws_bytes, _stream(stream)))
+
+
+def tda_kfac_state_bytes(k_in, k_out) -> int:
+    return int(load().tda_kfac_state_bytes(k_in, k_out))
+
+
+def tda_kfac_workspace_size(L, dtype) -> int:
+    return int(load().tda_kfac_workspace_size(ctypes.byref(L), dtype))
+
+
+def tda_kfac_reset(k_in, k_out, state, stream=None):
+    _check(load().tda_kfac_reset(k_in, k_out, _ptr(state), _stream(stream)))
+
+
+def tda_kfac_accumulate_factors(L, dtype, A, B, N, state, ws, ws_bytes, stream=None):
+    _check(load().tda_kfac_accumulate_factors(ctypes.byref(L), dtype, _ptr(A), _ptr(B), N, _ptr(state), _ptr(ws),
+                                              ws_bytes, _stream(stream)))
+
+
+def tda_project_kfac(L, dtype, A, B, N, phi, ld_phi, state, ws, ws_bytes, stream=None):
+    _check(load().tda_project_kfac(ctypes.byref(L), dtype, _ptr(A), _ptr(B), N, _ptr(phi), ld_phi, _ptr(state),
+                                   _ptr(ws), ws_bytes, _stream(stream)))
+
+
+def tda_kfac_eigen(k_in, k_out, state, stream=None):
+    _check(load().tda_kfac_eigen(k_in, k_out, _ptr(state), _stream(stream)))
+
+
+def tda_kfac_accumulate_eigenvalues(k_in, k_out, state, phi, n, ld_phi, ws, ws_bytes, stream=None):
+    _check(load().tda_kfac_accumulate_eigenvalues(k_in, k_out, _ptr(state), _ptr(phi), n, ld_phi, _ptr(ws), ws_bytes,
+                                                  _stream(stream)))
+
+
+def tda_kfac_apply(kind, k_in, k_out, state, lambda_abs, lambda_rel, q, n_q, ld_q, qhat, ld_qhat, stream=None):
+    _check(load().tda_kfac_apply(kind, k_in, k_out, _ptr(state), float(lambda_abs), float(lambda_rel), _ptr(q), n_q,
+                                 ld_q, _ptr(qhat), ld_qhat, _stream(stream)))
 
 
 def tda_precondition_state_bytes(D, state_dtype) -> int:

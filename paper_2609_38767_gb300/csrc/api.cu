@@ -530,6 +530,162 @@ tda_status tda_cosine(float* S, int64_t n_q, int64_t n_t, int64_t ld_S, const fl
     return cuda_check(launch_cosine(S, n_q, n_t, ld_S, nq, nt, (cudaStream_t)stream), "cosine");
 }
 
+// ---------------------------------------------------------------- K-FAC / EK-FAC
+static bool kfac_dims_ok(int64_t ka, int64_t kg) { return ka >= 1 && kg >= 1 && ka <= 128 && kg <= 128; }
+
+size_t tda_kfac_state_bytes(int32_t k_in, int32_t k_out) {
+    if (!kfac_dims_ok(k_in, k_out)) return 0;
+    return kfac_state_bytes(k_in, k_out);
+}
+
+// scratch of the K-FAC calls: per-block partial sums (fixed-order reduction)
+// and, for tda_kfac_accumulate_factors, one example's projected factors
+static size_t kfac_partials_bytes(int64_t ka, int64_t kg) {
+    const int64_t kmax2 = (ka > kg ? ka : kg) * (ka > kg ? ka : kg);
+    size_t b = sizeof(float) * 304 * (size_t)kmax2;                                      // covariance / EK-FAC partials
+    const size_t fused = sizeof(float) * (size_t)project_tc_max_grid() * 2 * (size_t)kmax2;  // fused projection
+    if (fused > b) b = fused;
+    return (b + 255) & ~(size_t)255;
+}
+
+size_t tda_kfac_workspace_size(const tda_layer_desc* L, tda_dtype dtype) {
+    (void)dtype;
+    if (!L || !kfac_dims_ok(L->k_in, L->k_out) || L->T < 0) return 0;
+    return kfac_partials_bytes(L->k_in, L->k_out) + project_factors_bytes_per_example(*L);
+}
+
+static tda_status kfac_state_ok(int64_t ka, int64_t kg, const void* state) {
+    if (!kfac_dims_ok(ka, kg)) return fail(TDA_ERR_INVALID_ARG, "K-FAC needs 1 <= k_in, k_out <= 128");
+    if (!state || ((uintptr_t)state & 15)) return fail(TDA_ERR_INVALID_ARG, "state must be a 16-byte aligned pointer");
+    return TDA_OK;
+}
+
+tda_status tda_kfac_reset(int32_t k_in, int32_t k_out, void* state, void* stream) {
+    g_msg[0] = 0;
+    tda_status st = kfac_state_ok(k_in, k_out, state);
+    if (st) return st;
+    return cuda_check(cudaMemsetAsync(state, 0, kfac_state_bytes(k_in, k_out), (cudaStream_t)stream), "kfac reset");
+}
+
+tda_status tda_kfac_accumulate_factors(const tda_layer_desc* L, tda_dtype dtype, const void* A, const void* B,
+                                       int64_t N, void* state, void* ws, size_t ws_bytes, void* stream) {
+    g_msg[0] = 0;
+    tda_status st = validate_layer(L, true);
+    if (st) return st;
+    if ((st = validate_factors(L, dtype, A, B, N, "tda_kfac_accumulate_factors"))) return st;
+    if (L->kind != TDA_PROJ_RADEMACHER && L->kind != TDA_PROJ_IDENTITY) return fail(TDA_ERR_INVALID_ARG, "bad kind");
+    if ((st = kfac_state_ok(L->k_in, L->k_out, state))) return st;
+    const size_t need = tda_kfac_workspace_size(L, dtype);
+    if (!ws || ws_bytes < need)
+        return fail(TDA_ERR_WORKSPACE, "tda_kfac_accumulate_factors needs >= %zu bytes of ws, got %zu", need,
+                    ws_bytes);
+    if ((uintptr_t)ws & 255) return fail(TDA_ERR_INVALID_ARG, "ws must be 256-byte aligned");
+    cudaStream_t s = (cudaStream_t)stream;
+    double* sd = (double*)state;
+    const int64_t ka = L->k_in, kg = L->k_out;
+    double* Sa = sd + kfac_offset_sa(ka, kg);
+    double* Sg = sd + kfac_offset_sg(ka, kg);
+    // Rademacher factors come out of the projection with +-1 signs: 1/k restores P = S / sqrt(k)
+    const double sca = L->kind == TDA_PROJ_RADEMACHER ? 1.0 / (double)ka : 1.0;
+    const double scg = L->kind == TDA_PROJ_RADEMACHER ? 1.0 / (double)kg : 1.0;
+    const size_t pbytes = kfac_partials_bytes(ka, kg);
+    float* part = (float*)ws;
+    float* Y = (float*)((char*)ws + pbytes);
+    if (N == 0 || L->T == 0)
+        return cuda_check(launch_kfac_cov(Y, 0, (int)ka, Sa, sca, sd, (double)N * (double)L->T, part, s),
+                          "kfac token count");
+    const size_t per = project_factors_bytes_per_example(*L);
+    int64_t chunk = (int64_t)((ws_bytes - pbytes) / per);
+    if (chunk > N) chunk = N;
+    if (chunk > 65535) chunk = 65535;
+    for (int64_t e0 = 0; e0 < N; e0 += chunk) {
+        const int64_t c = N - e0 < chunk ? N - e0 : chunk;
+        if ((st = cuda_check(launch_project_factors(*L, dtype, A, B, e0, c, Y, s), "project factors"))) return st;
+        const int64_t rows = c * L->T;
+        if ((st = cuda_check(launch_kfac_cov(Y, rows, (int)ka, Sa, sca, sd, (double)rows, part, s), "cov a")))
+            return st;
+        if ((st = cuda_check(launch_kfac_cov(Y + rows * ka, rows, (int)kg, Sg, scg, nullptr, 0.0, part, s),
+                             "cov g")))
+            return st;
+    }
+    return TDA_OK;
+}
+
+tda_status tda_project_kfac(const tda_layer_desc* L, tda_dtype dtype, const void* A, const void* B, int64_t N,
+                            float* phi, int64_t ld_phi, void* state, void* ws, size_t ws_bytes, void* stream) {
+    g_msg[0] = 0;
+    tda_status st = validate_layer(L, true);
+    if (st) return st;
+    if ((st = validate_factors(L, dtype, A, B, N, "tda_project_kfac"))) return st;
+    if ((st = kfac_state_ok(L->k_in, L->k_out, state))) return st;
+    const int64_t D = (int64_t)L->k_in * L->k_out;
+    if (N > 0 && (!phi || ld_phi < D)) return fail(TDA_ERR_INVALID_ARG, "phi is NULL or ld_phi < k_in*k_out");
+    if (dtype != TDA_BF16 || N == 0 || L->T == 0 || !project_tc_supported(*L, A, B))
+        return fail(TDA_ERR_UNSUPPORTED, "tda_project_kfac runs the bf16 tensor-core projection only");
+    const size_t need = kfac_partials_bytes(L->k_in, L->k_out);
+    if (!ws || ws_bytes < need)
+        return fail(TDA_ERR_WORKSPACE, "tda_project_kfac needs >= %zu bytes of ws, got %zu", need, ws_bytes);
+    if ((uintptr_t)ws & 255) return fail(TDA_ERR_INVALID_ARG, "ws must be 256-byte aligned");
+    unsigned int* err = device_error_word();
+    if (!err) return fail(TDA_ERR_CUDA, "device error word unavailable");
+    cudaStream_t s = (cudaStream_t)stream;
+    float* part = (float*)ws;
+    int grid = 0;
+    if ((st = cuda_check(launch_project_tc_kfac(*L, A, B, N, phi, ld_phi, part, &grid, err, s), "project+kfac")))
+        return st;
+    const int64_t k = L->k_in, kk = k * k;
+    double* sd = (double*)state;
+    const double sc = 1.0 / (double)k;
+    if ((st = cuda_check(launch_kfac_sum_partials(part, grid, 2 * kk, kk, sd + kfac_offset_sa(k, k), sc, sd, 0,
+                                                  (double)N * (double)L->T, s),
+                         "kfac sums a")))
+        return st;
+    return cuda_check(launch_kfac_sum_partials(part + kk, grid, 2 * kk, kk, sd + kfac_offset_sg(k, k), sc, nullptr, 0,
+                                               0.0, s),
+                      "kfac sums g");
+}
+
+tda_status tda_kfac_eigen(int32_t k_in, int32_t k_out, void* state, void* stream) {
+    g_msg[0] = 0;
+    tda_status st = kfac_state_ok(k_in, k_out, state);
+    if (st) return st;
+    return cuda_check(launch_kfac_eigen((double*)state, k_in, k_out, (cudaStream_t)stream), "kfac eigen");
+}
+
+tda_status tda_kfac_accumulate_eigenvalues(int32_t k_in, int32_t k_out, void* state, const float* phi, int64_t n,
+                                           int64_t ld_phi, void* ws, size_t ws_bytes, void* stream) {
+    g_msg[0] = 0;
+    tda_status st = kfac_state_ok(k_in, k_out, state);
+    if (st) return st;
+    if (n < 0 || (n > 0 && (!phi || ld_phi < (int64_t)k_in * k_out)))
+        return fail(TDA_ERR_INVALID_ARG, "phi is NULL or ld_phi < k_in*k_out");
+    const size_t need = kfac_partials_bytes(k_in, k_out);
+    if (!ws || ws_bytes < need)
+        return fail(TDA_ERR_WORKSPACE, "tda_kfac_accumulate_eigenvalues needs >= %zu bytes of ws, got %zu", need,
+                    ws_bytes);
+    int nblk = (int)(n < 304 ? n : 304);
+    if (nblk < 1) nblk = 1;
+    return cuda_check(launch_kfac_ekfac_accum((double*)state, k_in, k_out, phi, n, ld_phi, (float*)ws, nblk,
+                                              (cudaStream_t)stream),
+                      "ekfac eigenvalues");
+}
+
+tda_status tda_kfac_apply(int32_t kind, int32_t k_in, int32_t k_out, const void* state, double lambda_abs,
+                          double lambda_rel, const float* q, int64_t n_q, int64_t ld_q, float* qhat, int64_t ld_qhat,
+                          void* stream) {
+    g_msg[0] = 0;
+    tda_status st = kfac_state_ok(k_in, k_out, state);
+    if (st) return st;
+    if (kind != TDA_KFAC && kind != TDA_EKFAC) return fail(TDA_ERR_INVALID_ARG, "kind must be TDA_KFAC or TDA_EKFAC");
+    const int64_t D = (int64_t)k_in * k_out;
+    if (n_q < 0 || n_q > 2147483647LL) return fail(TDA_ERR_INVALID_ARG, "bad n_q");
+    if (n_q > 0 && (!q || !qhat || ld_q < D || ld_qhat < D))
+        return fail(TDA_ERR_INVALID_ARG, "q/qhat NULL or leading dimension < k_in*k_out");
+    return cuda_check(launch_kfac_apply(kind, (const double*)state, k_in, k_out, lambda_abs, lambda_rel, q, n_q, ld_q,
+                                        qhat, ld_qhat, (cudaStream_t)stream),
+                      "kfac apply");
+}
+
 size_t tda_precondition_state_bytes(int64_t D, tda_dtype state_dtype) {
     if (D < 1 || (state_dtype != TDA_F32 && state_dtype != TDA_F64)) return 0;
     const size_t el = state_dtype == TDA_F64 ? 8 : 4;

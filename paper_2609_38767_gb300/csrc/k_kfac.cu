@@ -1,0 +1,385 @@
+// k_kfac.cu -- K-FAC and EK-FAC on projected factors (the paper applies both
+// Kronecker-factored curvature methods to the projected pair (a~, g~)
+// unchanged, App. A.2, and damps by a multiple of the mean eigenvalue,
+// App. B.2):
+//   factor covariances  C_a = (1/M) sum a~ a~^T, C_g = (1/M) sum g~ g~^T,
+//   eigenbases          C = U diag(w) U^T (parallel cyclic Jacobi, fp64),
+//   EK-FAC eigenvalues  Lam = (1/N) sum_i (U_g^T Phi_i U_a)^2,
+//   preconditioning     Qhat = U_g [(U_g^T Q U_a) / (Lam + lambda)] U_a^T.
+// Sums over examples go through per-CTA partials reduced in a fixed order, so
+// results do not depend on scheduling.
+#include "tda_internal.cuh"
+
+namespace tda {
+
+// fp64 state of one layer, offsets in doubles
+struct KfLayout {
+    int64_t ka, kg, Sa, Sg, Ua, wa, Ug, wg, Le, total;
+    __host__ __device__ explicit KfLayout(int64_t k_in, int64_t k_out) : ka(k_in), kg(k_out) {
+        Sa = 8;  // header: [0] M token positions, [1] N examples (EK-FAC), [2] Jacobi sweeps a, [3] sweeps g
+        Sg = Sa + ka * ka;
+        Ua = Sg + kg * kg;
+        wa = Ua + ka * ka;
+        Ug = wa + ka;
+        wg = Ug + kg * kg;
+        Le = wg + kg;
+        total = Le + ka * kg;
+    }
+};
+
+size_t kfac_state_bytes(int64_t k_in, int64_t k_out) {
+    const KfLayout l(k_in, k_out);
+    return ((size_t)l.total * 8 + 255) & ~(size_t)255;
+}
+
+namespace {
+
+constexpr int kKfThreads = 256;
+
+// part[b][i*k+j] = sum over the rows of block b of Y[r][i] * Y[r][j] (fp32)
+__global__ void __launch_bounds__(kKfThreads)
+cov_partial_kernel(const float* __restrict__ Y, int64_t rows, int k, int64_t rows_per_block, float* __restrict__ part) {
+    extern __shared__ float ys[];  // [64][k]
+    const int64_t r0 = (int64_t)blockIdx.x * rows_per_block;
+    int64_t r1 = r0 + rows_per_block;
+    if (r1 > rows) r1 = rows;
+    const int kk = k * k;
+    constexpr int kMaxPer = 64;  // k <= 128: k*k / 256 <= 64 entries per thread
+    float acc[kMaxPer];
+#pragma unroll
+    for (int m = 0; m < kMaxPer; ++m) acc[m] = 0.f;
+    for (int64_t b0 = r0; b0 < r1; b0 += 64) {
+        const int nr = (int)((r1 - b0) < 64 ? (r1 - b0) : 64);
+        __syncthreads();
+        for (int x = threadIdx.x; x < nr * k; x += blockDim.x) ys[x] = Y[b0 * k + x];
+        __syncthreads();
+#pragma unroll
+        for (int m = 0; m < kMaxPer; ++m) {
+            const int e = threadIdx.x + m * kKfThreads;
+            if (e < kk) {
+                const int i = e / k, j = e - (e / k) * k;
+                float a = acc[m];
+                for (int r = 0; r < nr; ++r) a = fmaf(ys[r * k + i], ys[r * k + j], a);
+                acc[m] = a;
+            }
+        }
+    }
+    float* out = part + (int64_t)blockIdx.x * kk;
+#pragma unroll
+    for (int m = 0; m < kMaxPer; ++m) {
+        const int e = threadIdx.x + m * kKfThreads;
+        if (e < kk) out[e] = acc[m];
+    }
+}
+
+// S[e] += scale * sum_b part[b * stride + e] in block order (fp64); header[slot] += add
+__global__ void sum_partials_kernel(const float* __restrict__ part, int nblk, int64_t stride, int64_t n,
+                                    double* __restrict__ S, double scale, double* __restrict__ header, int slot,
+                                    double add) {
+    for (int64_t e = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; e < n; e += (int64_t)gridDim.x * blockDim.x) {
+        double v = 0.0;
+        for (int b = 0; b < nblk; ++b) v += (double)part[(int64_t)b * stride + e];
+        S[e] += scale * v;
+    }
+    if (header && blockIdx.x == 0 && threadIdx.x == 0) header[slot] += add;
+}
+
+// Parallel cyclic Jacobi (round-robin pair ordering) on C = S / M for the
+// a side (blockIdx.x 0) and the g side (1). A lives in shared memory, the
+// eigenvectors accumulate in the state's U (V <- V J). Each round rotates
+// floor(m/2) disjoint pairs at once: angles from the round's starting matrix,
+// then all row updates, then all column updates, which is J^T A J for the
+// product J of the round's rotations.
+__global__ void __launch_bounds__(kKfThreads) jacobi_kernel(double* __restrict__ st, int64_t ka, int64_t kg) {
+    extern __shared__ double A[];  // [n][n], then c, s, p, q per pair
+    const KfLayout l(ka, kg);
+    const bool side_g = blockIdx.x == 1;
+    const int n = (int)(side_g ? kg : ka);
+    const double* S = st + (side_g ? l.Sg : l.Sa);
+    double* U = st + (side_g ? l.Ug : l.Ua);
+    double* w = st + (side_g ? l.wg : l.wa);
+    const int m = (n + 1) & ~1;  // even number of players; index n is a dummy when n is odd
+    double* cs = A + n * n;
+    double* sn = cs + m / 2;
+    int* P = (int*)(sn + m / 2);
+    int* Q = P + m / 2;
+    __shared__ double red[kKfThreads];
+    __shared__ int done;
+    const double Mtok = st[0];
+    const double inv = Mtok > 0 ? 1.0 / Mtok : 0.0;
+    for (int e = threadIdx.x; e < n * n; e += blockDim.x) {
+        A[e] = S[e] * inv;
+        U[e] = (e / n == e % n) ? 1.0 : 0.0;
+    }
+    __syncthreads();
+    // squared Frobenius norm
+    double f = 0.0;
+    for (int e = threadIdx.x; e < n * n; e += blockDim.x) f += A[e] * A[e];
+    red[threadIdx.x] = f;
+    __syncthreads();
+    for (int h = blockDim.x / 2; h > 0; h >>= 1) {
+        if (threadIdx.x < h) red[threadIdx.x] += red[threadIdx.x + h];
+        __syncthreads();
+    }
+    const double fro = red[0];
+    __syncthreads();
+    int sweep = 0;
+    for (; sweep < 60; ++sweep) {
+        double off = 0.0;
+        for (int e = threadIdx.x; e < n * n; e += blockDim.x)
+            if (e / n != e % n) off += A[e] * A[e];
+        red[threadIdx.x] = off;
+        __syncthreads();
+        for (int h = blockDim.x / 2; h > 0; h >>= 1) {
+            if (threadIdx.x < h) red[threadIdx.x] += red[threadIdx.x + h];
+            __syncthreads();
+        }
+        if (threadIdx.x == 0) done = (red[0] <= 1e-28 * fro) ? 1 : 0;
+        __syncthreads();
+        if (done) break;
+        for (int r = 0; r < m - 1; ++r) {
+            for (int i = threadIdx.x; i < m / 2; i += blockDim.x) {
+                int p = i == 0 ? r : (r + i) % (m - 1);
+                int q = i == 0 ? m - 1 : (r - i + m - 1) % (m - 1);
+                if (p > q) {
+                    const int t = p;
+                    p = q;
+                    q = t;
+                }
+                double c = 1.0, s = 0.0;
+                if (q < n) {
+                    const double apq = A[p * n + q];
+                    if (apq != 0.0) {
+                        const double tau = (A[q * n + q] - A[p * n + p]) / (2.0 * apq);
+                        const double t = (tau >= 0 ? 1.0 : -1.0) / (fabs(tau) + sqrt(1.0 + tau * tau));
+                        c = 1.0 / sqrt(1.0 + t * t);
+                        s = t * c;
+                    }
+                }
+                cs[i] = c;
+                sn[i] = s;
+                P[i] = p;
+                Q[i] = q < n ? q : -1;
+            }
+            __syncthreads();
+            const int half = m / 2;
+            for (int x = threadIdx.x; x < half * n; x += blockDim.x) {  // rows p, q: A <- J^T A
+                const int i = x / n, k = x - (x / n) * n;
+                if (Q[i] < 0 || sn[i] == 0.0) continue;
+                const int p = P[i], q = Q[i];
+                const double c = cs[i], s = sn[i], apk = A[p * n + k], aqk = A[q * n + k];
+                A[p * n + k] = c * apk - s * aqk;
+                A[q * n + k] = s * apk + c * aqk;
+            }
+            __syncthreads();
+            for (int x = threadIdx.x; x < half * n; x += blockDim.x) {  // columns p, q: A <- A J, V <- V J
+                const int i = x / n, k = x - (x / n) * n;
+                if (Q[i] < 0 || sn[i] == 0.0) continue;
+                const int p = P[i], q = Q[i];
+                const double c = cs[i], s = sn[i];
+                const double akp = A[k * n + p], akq = A[k * n + q];
+                A[k * n + p] = c * akp - s * akq;
+                A[k * n + q] = s * akp + c * akq;
+                const double vkp = U[k * n + p], vkq = U[k * n + q];
+                U[k * n + p] = c * vkp - s * vkq;
+                U[k * n + q] = s * vkp + c * vkq;
+            }
+            __syncthreads();
+        }
+    }
+    for (int i = threadIdx.x; i < n; i += blockDim.x) w[i] = A[i * n + i];
+    if (threadIdx.x == 0) st[2 + (side_g ? 1 : 0)] = done ? (double)sweep : -1.0;
+    if (blockIdx.x == 0) {  // a new eigenbasis invalidates the EK-FAC sums
+        for (int64_t e = threadIdx.x; e < ka * kg; e += blockDim.x) st[l.Le + e] = 0.0;
+        if (threadIdx.x == 0) st[1] = 0.0;
+    }
+}
+
+// part[b][r*ka+c] = sum over the examples of block b of ((U_g^T Phi_i U_a)[r][c])^2
+__global__ void __launch_bounds__(kKfThreads)
+ekfac_partial_kernel(const float* __restrict__ phi, int64_t n, int64_t ld, const double* __restrict__ st, int64_t ka,
+                     int64_t kg, float* __restrict__ part) {
+    extern __shared__ float sm[];  // Phi_i [kg][ka], Y [kg][ka]
+    const KfLayout l(ka, kg);
+    const double* Ua = st + l.Ua;
+    const double* Ug = st + l.Ug;
+    float* F = sm;
+    float* Y = sm + kg * ka;
+    const int64_t D = ka * kg;
+    constexpr int kMaxPer = 64;
+    float acc[kMaxPer];
+#pragma unroll
+    for (int m = 0; m < kMaxPer; ++m) acc[m] = 0.f;
+    for (int64_t i = blockIdx.x; i < n; i += gridDim.x) {
+        __syncthreads();
+        for (int64_t e = threadIdx.x; e < D; e += blockDim.x) F[e] = phi[i * ld + e];
+        __syncthreads();
+        for (int64_t e = threadIdx.x; e < D; e += blockDim.x) {  // Y = Phi U_a
+            const int64_t r = e / ka, c = e - (e / ka) * ka;
+            float s = 0.f;
+            for (int64_t j = 0; j < ka; ++j) s = fmaf(F[r * ka + j], (float)Ua[j * ka + c], s);
+            Y[e] = s;
+        }
+        __syncthreads();
+#pragma unroll
+        for (int m = 0; m < kMaxPer; ++m) {  // X = U_g^T Y, accumulate X^2
+            const int64_t e = threadIdx.x + (int64_t)m * kKfThreads;
+            if (e < D) {
+                const int64_t r = e / ka, c = e - (e / ka) * ka;
+                float s = 0.f;
+                for (int64_t j = 0; j < kg; ++j) s = fmaf((float)Ug[j * kg + r], Y[j * ka + c], s);
+                acc[m] = fmaf(s, s, acc[m]);
+            }
+        }
+    }
+    float* out = part + (int64_t)blockIdx.x * D;
+#pragma unroll
+    for (int m = 0; m < kMaxPer; ++m) {
+        const int64_t e = threadIdx.x + (int64_t)m * kKfThreads;
+        if (e < D) out[e] = acc[m];
+    }
+}
+
+// One CTA per query row: Qhat = U_g [(U_g^T Q U_a) / (Lam + lambda)] U_a^T,
+// fp64 accumulation, fp32 intermediates in shared memory.
+__global__ void __launch_bounds__(kKfThreads)
+kfac_apply_kernel(int kind, const double* __restrict__ st, int64_t ka, int64_t kg, double lambda_abs,
+                  double lambda_rel, const float* __restrict__ q, int64_t ld_q, float* __restrict__ qhat,
+                  int64_t ld_qhat) {
+    extern __shared__ float sm[];  // X [kg][ka], Y [kg][ka]
+    const KfLayout l(ka, kg);
+    const double* Ua = st + l.Ua;
+    const double* Ug = st + l.Ug;
+    const int64_t D = ka * kg;
+    float* X = sm;
+    float* Y = sm + D;
+    __shared__ double red[kKfThreads];
+    const double nex = st[1];
+    auto lam_of = [&](int64_t e) -> double {
+        const int64_t r = e / ka, c = e - (e / ka) * ka;
+        if (kind == 0) return st[l.wg + r] * st[l.wa + c];
+        return nex > 0 ? st[l.Le + e] / nex : 0.0;
+    };
+    double s = 0.0;
+    for (int64_t e = threadIdx.x; e < D; e += blockDim.x) s += lam_of(e);
+    red[threadIdx.x] = s;
+    __syncthreads();
+    for (int h = blockDim.x / 2; h > 0; h >>= 1) {
+        if (threadIdx.x < h) red[threadIdx.x] += red[threadIdx.x + h];
+        __syncthreads();
+    }
+    const double lambda = lambda_abs + lambda_rel * red[0] / (double)D;
+    const float* qi = q + (int64_t)blockIdx.x * ld_q;
+    for (int64_t e = threadIdx.x; e < D; e += blockDim.x) X[e] = qi[e];
+    __syncthreads();
+    for (int64_t e = threadIdx.x; e < D; e += blockDim.x) {  // Y = Q U_a
+        const int64_t r = e / ka, c = e - (e / ka) * ka;
+        double a = 0.0;
+        for (int64_t j = 0; j < ka; ++j) a += (double)X[r * ka + j] * Ua[j * ka + c];
+        Y[e] = (float)a;
+    }
+    __syncthreads();
+    for (int64_t e = threadIdx.x; e < D; e += blockDim.x) {  // X = (U_g^T Y) / (Lam + lambda)
+        const int64_t r = e / ka, c = e - (e / ka) * ka;
+        double a = 0.0;
+        for (int64_t j = 0; j < kg; ++j) a += Ug[j * kg + r] * (double)Y[j * ka + c];
+        X[e] = (float)(a / (lam_of(e) + lambda));
+    }
+    __syncthreads();
+    for (int64_t e = threadIdx.x; e < D; e += blockDim.x) {  // Y = X U_a^T
+        const int64_t r = e / ka, c = e - (e / ka) * ka;
+        double a = 0.0;
+        for (int64_t j = 0; j < ka; ++j) a += (double)X[r * ka + j] * Ua[c * ka + j];
+        Y[e] = (float)a;
+    }
+    __syncthreads();
+    float* out = qhat + (int64_t)blockIdx.x * ld_qhat;
+    for (int64_t e = threadIdx.x; e < D; e += blockDim.x) {  // Qhat = U_g Y
+        const int64_t r = e / ka, c = e - (e / ka) * ka;
+        double a = 0.0;
+        for (int64_t j = 0; j < kg; ++j) a += Ug[r * kg + j] * (double)Y[j * ka + c];
+        out[e] = (float)a;
+    }
+}
+
+}  // namespace
+
+int kfac_partial_blocks(int64_t rows) {
+    int64_t b = (rows + 255) / 256;
+    if (b > 304) b = 304;
+    return b < 1 ? 1 : (int)b;
+}
+
+// S += scale * Y^T Y for rows x k fp32 rows Y (deterministic), header M += add_m.
+cudaError_t launch_kfac_cov(const float* Y, int64_t rows, int k, double* S, double scale, double* header,
+                            double add_m, float* part, cudaStream_t s) {
+    if (rows == 0) {
+        if (header && add_m != 0) {
+            note_launches(1);
+            sum_partials_kernel<<<1, 32, 0, s>>>(part, 0, 0, 0, S, scale, header, 0, add_m);
+        }
+        return cudaGetLastError();
+    }
+    const int nb = kfac_partial_blocks(rows);
+    int64_t per = (rows + nb - 1) / nb;
+    per = (per + 63) / 64 * 64;
+    const int nblk = (int)((rows + per - 1) / per);
+    note_launches(2);
+    cov_partial_kernel<<<nblk, kKfThreads, (size_t)64 * k * 4, s>>>(Y, rows, k, per, part);
+    sum_partials_kernel<<<(unsigned)((k * k + 255) / 256), 256, 0, s>>>(part, nblk, (int64_t)k * k, (int64_t)k * k,
+                                                                       S, scale, header, 0, add_m);
+    return cudaGetLastError();
+}
+
+// Sums of per-CTA partials written by another kernel (the fused projection).
+cudaError_t launch_kfac_sum_partials(const float* part, int nblk, int64_t stride, int64_t n, double* S, double scale,
+                                     double* header, int slot, double add, cudaStream_t s) {
+    note_launches(1);
+    int64_t blocks = (n + 255) / 256;
+    if (blocks < 1) blocks = 1;
+    sum_partials_kernel<<<(unsigned)blocks, 256, 0, s>>>(part, nblk, stride, n, S, scale, header, slot, add);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_kfac_eigen(double* state, int64_t ka, int64_t kg, cudaStream_t s) {
+    const int64_t nmax = ka > kg ? ka : kg;
+    const int64_t mh = (nmax + 2) / 2;
+    const size_t smem = (size_t)nmax * nmax * 8 + (size_t)mh * (8 + 8 + 4 + 4);
+    cudaError_t e = cudaFuncSetAttribute(jacobi_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+    if (e != cudaSuccess) return e;
+    note_launches(1);
+    jacobi_kernel<<<2, kKfThreads, smem, s>>>(state, ka, kg);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_kfac_ekfac_accum(double* state, int64_t ka, int64_t kg, const float* phi, int64_t n, int64_t ld,
+                                    float* part, int nblk, cudaStream_t s) {
+    if (n == 0) return cudaSuccess;
+    const size_t smem = (size_t)2 * ka * kg * 4;
+    cudaError_t e = cudaFuncSetAttribute(ekfac_partial_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+    if (e != cudaSuccess) return e;
+    const KfLayout l(ka, kg);
+    note_launches(2);
+    ekfac_partial_kernel<<<nblk, kKfThreads, smem, s>>>(phi, n, ld, state, ka, kg, part);
+    sum_partials_kernel<<<(unsigned)((ka * kg + 255) / 256), 256, 0, s>>>(part, nblk, ka * kg, ka * kg, state + l.Le,
+                                                                        1.0, state, 1, (double)n);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_kfac_apply(int kind, const double* state, int64_t ka, int64_t kg, double lambda_abs,
+                              double lambda_rel, const float* q, int64_t n_q, int64_t ld_q, float* qhat,
+                              int64_t ld_qhat, cudaStream_t s) {
+    if (n_q == 0) return cudaSuccess;
+    const size_t smem = (size_t)2 * ka * kg * 4;
+    cudaError_t e = cudaFuncSetAttribute(kfac_apply_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+    if (e != cudaSuccess) return e;
+    note_launches(1);
+    kfac_apply_kernel<<<(unsigned)n_q, kKfThreads, smem, s>>>(kind, state, ka, kg, lambda_abs, lambda_rel, q, ld_q,
+                                                              qhat, ld_qhat);
+    return cudaGetLastError();
+}
+
+int64_t kfac_offset_sa(int64_t ka, int64_t kg) { return KfLayout(ka, kg).Sa; }
+int64_t kfac_offset_sg(int64_t ka, int64_t kg) { return KfLayout(ka, kg).Sg; }
+
+}  // namespace tda

@@ -85,6 +85,7 @@ struct Params {
     int pack;         // examples per token tile (T <= 64), else 1
     int nk_in, nk_out;
     int cs;           // CTAs per cluster sharing one example's token tiles (1, 2 or 4)
+    float* cov;       // K-FAC: per-CTA partial sums of At^T At and Bt^T Bt ([grid][2][K*K])
 };
 
 #include "tc_ptx.cuh"
@@ -139,7 +140,7 @@ __device__ __forceinline__ void write_sign_half(uint8_t* tile, int n, uint64_t w
     }
 }
 
-template <int K, int G>
+template <int K, int G, bool KF>
 __global__ void __launch_bounds__(kThreads, 1)
 project_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
                   const Params p) {
@@ -313,10 +314,18 @@ project_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant
         bool stop = false;
         int64_t cur = -1;                // example whose Phi is accumulating (pack == 1)
         float acc[C::RB][C::CB];
+        // K-FAC factor covariances (unscaled signs): ca += At^T At, cgm += Bt^T Bt over valid rows
+        float ca[KF ? C::RB : 1][KF ? C::CB : 1], cgm[KF ? C::RB : 1][KF ? C::CB : 1];
 #pragma unroll
         for (int a = 0; a < C::RB; ++a)
 #pragma unroll
             for (int c = 0; c < C::CB; ++c) acc[a][c] = 0.f;
+        if constexpr (KF) {
+#pragma unroll
+            for (int a = 0; a < C::RB; ++a)
+#pragma unroll
+                for (int c = 0; c < C::CB; ++c) ca[a][c] = cgm[a][c] = 0.f;
+        }
 
         // Phi of example `n` is complete in every cluster CTA: reduce the partial
         // blocks into the leader (rank 0) over distributed shared memory and
@@ -405,6 +414,31 @@ project_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant
                     if (lane == 0) mbar_arrive(smem_u32(&tempty[b]));
                 }
                 epi_sync();
+                if constexpr (KF) {
+                    // rows of packed tiles past pack * T belong to the next tile's examples
+                    const int rows = p.pack == 1 ? kTileM : p.pack * (int)p.T;
+#pragma unroll 2
+                    for (int t = 0; t < rows; ++t) {
+                        float xa[C::RB], xc[C::CB], ya[C::RB], yc[C::CB];
+#pragma unroll
+                        for (int a = 0; a < C::RB; ++a) {
+                            xa[a] = stX[t * C::kStageLd + rg * C::RB + a];
+                            ya[a] = stY[t * C::kStageLd + rg * C::RB + a];
+                        }
+#pragma unroll
+                        for (int c = 0; c < C::CB; ++c) {
+                            xc[c] = stX[t * C::kStageLd + cg * C::CB + c];
+                            yc[c] = stY[t * C::kStageLd + cg * C::CB + c];
+                        }
+#pragma unroll
+                        for (int a = 0; a < C::RB; ++a)
+#pragma unroll
+                            for (int c = 0; c < C::CB; ++c) {
+                                ca[a][c] = fmaf(xa[a], xc[c], ca[a][c]);
+                                cgm[a][c] = fmaf(ya[a], yc[c], cgm[a][c]);
+                            }
+                    }
+                }
                 if (p.pack == 1) {
 #pragma unroll 4
                     for (int t = 0; t < kTileM; ++t) {
@@ -453,6 +487,17 @@ project_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant
             }
         }
         if (!stop && p.pack == 1 && cur >= 0) flush(cur);
+        if constexpr (KF) {
+            float* out = p.cov + (size_t)blockIdx.x * 2 * K * K;
+#pragma unroll
+            for (int a = 0; a < C::RB; ++a)
+#pragma unroll
+                for (int c = 0; c < C::CB; ++c) {
+                    const int e = (rg * C::RB + a) * K + cg * C::CB + c;
+                    out[e] = ca[a][c];
+                    out[K * K + e] = cgm[a][c];
+                }
+        }
     }
 
     tc_fence_before();
@@ -518,9 +563,9 @@ int sm_count() {
     return sms;
 }
 
-template <int K, int G>
+template <int K, int G, bool KF>
 cudaError_t launch_kg(const tda_layer_desc& L, const void* A, const void* B, int64_t N, float* phi,
-                      int64_t ld_phi, unsigned int* err, cudaStream_t s, int pack) {
+                      int64_t ld_phi, unsigned int* err, cudaStream_t s, int pack, float* cov, int* grid_out) {
     using C = Cfg<K, G>;
     CUtensorMap tmA, tmB;
     if (pack > 1) {
@@ -545,8 +590,9 @@ cudaError_t launch_kg(const tda_layer_desc& L, const void* A, const void* B, int
     p.n_ttiles = pack > 1 ? 1 : (int)((L.T + kTileM - 1) / kTileM);
     p.nk_in = (int)((L.d_in + kChunkK - 1) / kChunkK);
     p.nk_out = (int)((L.d_out + kChunkK - 1) / kChunkK);
+    p.cov = cov;
     const int sms = sm_count();
-    cudaError_t e = cudaFuncSetAttribute(project_tc_kernel<K, G>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+    cudaError_t e = cudaFuncSetAttribute(project_tc_kernel<K, G, KF>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                          (int)C::kSmem);
     if (e != cudaSuccess) return e;
     // Fewer examples than SMs: a cluster of cs CTAs shares each example's token
@@ -568,23 +614,24 @@ cudaError_t launch_kg(const tda_layer_desc& L, const void* A, const void* B, int
     cfg.numAttrs = 1;
     int max_clusters = 0;
     cfg.gridDim = dim3((unsigned)(cs * (sms / cs)));
-    if (cudaOccupancyMaxActiveClusters(&max_clusters, project_tc_kernel<K, G>, &cfg) != cudaSuccess ||
+    if (cudaOccupancyMaxActiveClusters(&max_clusters, project_tc_kernel<K, G, KF>, &cfg) != cudaSuccess ||
         max_clusters < 1)
         max_clusters = sms / cs;
     int64_t clusters = p.n_slots;
     if (clusters > max_clusters) clusters = max_clusters;
     cfg.gridDim = dim3((unsigned)(clusters * cs));
+    if (grid_out) *grid_out = (int)(clusters * cs);
     note_launches(1);
-    e = cudaLaunchKernelEx(&cfg, project_tc_kernel<K, G>, tmA, tmB, p);
+    e = cudaLaunchKernelEx(&cfg, project_tc_kernel<K, G, KF>, tmA, tmB, p);
     if (e != cudaSuccess) return e;
     return cudaGetLastError();
 }
 
 // Two tiles per stage once every CTA has at least two groups of work; fewer
 // units run one tile per stage so that they spread over all SMs.
-template <int K>
+template <int K, bool KF>
 cudaError_t launch_k(const tda_layer_desc& L, const void* A, const void* B, int64_t N, float* phi,
-                     int64_t ld_phi, unsigned int* err, cudaStream_t s) {
+                     int64_t ld_phi, unsigned int* err, cudaStream_t s, float* cov, int* grid_out) {
     int pack = L.T <= 64 ? (int)(kTileM / L.T) : 1;
     if (pack > 1) {
         // packed rows are addressed with 32-bit TMA coordinates and the [1][N*T][d]
@@ -596,19 +643,21 @@ cudaError_t launch_k(const tda_layer_desc& L, const void* A, const void* B, int6
         max_n = max_n / pack * pack;
         if (max_n < pack) pack = 1;  // one example per tile instead
         else if (N > max_n) {
+            if (KF) return cudaErrorInvalidValue;  // one partial slab per CTA: one launch only
             const size_t a_ex = (size_t)L.T * L.d_in * 2, b_ex = (size_t)L.T * L.d_out * 2;
             for (int64_t e0 = 0; e0 < N; e0 += max_n) {
                 const int64_t n = N - e0 < max_n ? N - e0 : max_n;
-                cudaError_t e = launch_k<K>(L, (const char*)A + e0 * a_ex, (const char*)B + e0 * b_ex, n,
-                                            phi + e0 * ld_phi, ld_phi, err, s);
+                cudaError_t e = launch_k<K, KF>(L, (const char*)A + e0 * a_ex, (const char*)B + e0 * b_ex, n,
+                                                phi + e0 * ld_phi, ld_phi, err, s, nullptr, nullptr);
                 if (e != cudaSuccess) return e;
             }
             return cudaSuccess;
         }
     }
     const int64_t units = pack > 1 ? (N + pack - 1) / pack : N * ((L.T + kTileM - 1) / kTileM);
-    if (units >= 4 * (int64_t)sm_count()) return launch_kg<K, 2>(L, A, B, N, phi, ld_phi, err, s, pack);
-    return launch_kg<K, 1>(L, A, B, N, phi, ld_phi, err, s, pack);
+    if (units >= 4 * (int64_t)sm_count())
+        return launch_kg<K, 2, KF>(L, A, B, N, phi, ld_phi, err, s, pack, cov, grid_out);
+    return launch_kg<K, 1, KF>(L, A, B, N, phi, ld_phi, err, s, pack, cov, grid_out);
 }
 
 }  // namespace
@@ -629,11 +678,28 @@ cudaError_t launch_project_tc(const tda_layer_desc& L, const void* A, const void
                               int64_t ld_phi, unsigned int* err, cudaStream_t s) {
     if (N == 0) return cudaSuccess;
     switch (L.k_in) {
-        case 16: return launch_k<16>(L, A, B, N, phi, ld_phi, err, s);
-        case 32: return launch_k<32>(L, A, B, N, phi, ld_phi, err, s);
-        case 64: return launch_k<64>(L, A, B, N, phi, ld_phi, err, s);
+        case 16: return launch_k<16, false>(L, A, B, N, phi, ld_phi, err, s, nullptr, nullptr);
+        case 32: return launch_k<32, false>(L, A, B, N, phi, ld_phi, err, s, nullptr, nullptr);
+        case 64: return launch_k<64, false>(L, A, B, N, phi, ld_phi, err, s, nullptr, nullptr);
         default: return cudaErrorNotSupported;
     }
 }
+
+// Projection plus K-FAC factor covariance partials: cov receives one slab of
+// 2 * k * k floats per CTA (At^T At then Bt^T Bt, unscaled signs); *grid_out
+// is the number of slabs written.
+cudaError_t launch_project_tc_kfac(const tda_layer_desc& L, const void* A, const void* B, int64_t N, float* phi,
+                                   int64_t ld_phi, float* cov, int* grid_out, unsigned int* err, cudaStream_t s) {
+    *grid_out = 0;
+    if (N == 0) return cudaSuccess;
+    switch (L.k_in) {
+        case 16: return launch_k<16, true>(L, A, B, N, phi, ld_phi, err, s, cov, grid_out);
+        case 32: return launch_k<32, true>(L, A, B, N, phi, ld_phi, err, s, cov, grid_out);
+        case 64: return launch_k<64, true>(L, A, B, N, phi, ld_phi, err, s, cov, grid_out);
+        default: return cudaErrorNotSupported;
+    }
+}
+
+int project_tc_max_grid() { return sm_count(); }
 
 }  // namespace tda

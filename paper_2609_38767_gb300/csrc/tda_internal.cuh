@@ -72,6 +72,24 @@ cudaError_t launch_project_simt(const tda_layer_desc& L, tda_dtype dt, const voi
 // tcgen05 / TMA projection for bf16 inputs. Returns cudaErrorNotSupported if
 // the shape has no tensor-core instantiation (caller falls back to SIMT).
 bool project_tc_supported(const tda_layer_desc& L, const void* A, const void* B);
+cudaError_t launch_project_tc_kfac(const tda_layer_desc& L, const void* A, const void* B, int64_t N, float* phi,
+                                   int64_t ld_phi, float* cov, int* grid_out, unsigned int* err, cudaStream_t s);
+int project_tc_max_grid();
+// K-FAC / EK-FAC (k_kfac.cu)
+size_t kfac_state_bytes(int64_t k_in, int64_t k_out);
+int kfac_partial_blocks(int64_t rows);
+int64_t kfac_offset_sa(int64_t ka, int64_t kg);
+int64_t kfac_offset_sg(int64_t ka, int64_t kg);
+cudaError_t launch_kfac_cov(const float* Y, int64_t rows, int k, double* S, double scale, double* header,
+                            double add_m, float* part, cudaStream_t s);
+cudaError_t launch_kfac_sum_partials(const float* part, int nblk, int64_t stride, int64_t n, double* S, double scale,
+                                     double* header, int slot, double add, cudaStream_t s);
+cudaError_t launch_kfac_eigen(double* state, int64_t ka, int64_t kg, cudaStream_t s);
+cudaError_t launch_kfac_ekfac_accum(double* state, int64_t ka, int64_t kg, const float* phi, int64_t n, int64_t ld,
+                                    float* part, int nblk, cudaStream_t s);
+cudaError_t launch_kfac_apply(int kind, const double* state, int64_t ka, int64_t kg, double lambda_abs,
+                              double lambda_rel, const float* q, int64_t n_q, int64_t ld_q, float* qhat,
+                              int64_t ld_qhat, cudaStream_t s);
 cudaError_t launch_project_tc(const tda_layer_desc& L, const void* A, const void* B, int64_t N,
                               float* phi, int64_t ld_phi, unsigned int* err, cudaStream_t s);
 

@@ -147,3 +147,25 @@ def test_norm_entry_validation(libs):
     assert _err(tda.tda_norms, tda.TDA_OP_NORM_PROJECTED, L, tda.TDA_F32, 16, 16, 4, None, stream=s) \
         == tda.TDA_ERR_INVALID_ARG
     assert _err(tda.tda_cosine, 16, 2, 8, 4, 16, 16, stream=s) == tda.TDA_ERR_INVALID_ARG
+
+
+def test_kfac_state_and_validation(libs):
+    # state: 8-double header + Sa, Sg, Ua, wa, Ug, wg, EK-FAC sums (fp64), 256-byte multiple
+    for ka, kg in [(16, 16), (32, 64), (128, 128), (1, 3)]:
+        n = 8 + 2 * ka * ka + ka + 2 * kg * kg + kg + ka * kg
+        assert tda.tda_kfac_state_bytes(ka, kg) == (n * 8 + 255) // 256 * 256
+    assert tda.tda_kfac_state_bytes(0, 16) == 0 and tda.tda_kfac_state_bytes(16, 129) == 0
+    L = tda.LayerDesc(64, 64, 8, 16, 16)
+    s = 0
+    assert _err(tda.tda_kfac_reset, 16, 200, 256, stream=s) == tda.TDA_ERR_INVALID_ARG
+    assert _err(tda.tda_kfac_reset, 16, 16, 8, stream=s) == tda.TDA_ERR_INVALID_ARG  # misaligned state
+    assert _err(tda.tda_kfac_apply, 2, 16, 16, 256, 0.0, 0.1, 256, 1, 256, 256, 256, stream=s) \
+        == tda.TDA_ERR_INVALID_ARG
+    assert _err(tda.tda_kfac_apply, tda.TDA_KFAC, 16, 16, 256, 0.0, 0.1, 256, 1, 100, 256, 256, stream=s) \
+        == tda.TDA_ERR_INVALID_ARG  # ld_q < 256
+    assert _err(tda.tda_kfac_accumulate_factors, L, tda.TDA_BF16, 16, 16, 4, 256, 256, 100, stream=s) \
+        == tda.TDA_ERR_WORKSPACE
+    assert _err(tda.tda_kfac_accumulate_eigenvalues, 16, 16, 256, 16, 4, 256, 256, 100, stream=s) \
+        == tda.TDA_ERR_WORKSPACE
+    assert _err(tda.tda_project_kfac, L, tda.TDA_F32, 16, 16, 4, 16, 256, 256, 256, 1 << 24, stream=s) \
+        == tda.TDA_ERR_UNSUPPORTED

@@ -502,3 +502,86 @@ def test_gram_tensor_core_matches_oracle(dev, orc, nq, nt, T, di, do, beta):
     got = S.cpu().numpy()
     assert rel_fro(got[:, :nt], ref) <= 1e-5
     np.testing.assert_array_equal(got[:, nt:], S0[:, nt:])
+
+
+# ------------------------------------------------------------------ K-FAC / EK-FAC
+def _kfac_oracle(orc, A64, B64, k, seed, layer, kind, lam_abs, lam_rel, Q, phi64=None):
+    Ca, Cg = orc.kfac_covariances(A64, B64, k, k, seed, layer)
+    wa, Ua, _ = orc.sym_eig(Ca)
+    wg, Ug, _ = orc.sym_eig(Cg)
+    Lam = orc.kfac_eigenvalues(wa, wg) if kind == tda.TDA_KFAC else orc.ekfac_eigenvalues(phi64, Ua, Ug)
+    lam = orc.kfac_damping(Lam, lam_abs, lam_rel)
+    return Ca, Cg, wa, wg, orc.kfac_precondition(Ua, Ug, Lam, lam, Q)
+
+
+@pytest.mark.gpu
+@pytest.mark.parametrize("dtype,N,T,di,do,k,chunks", [("f32", 40, 13, 64, 48, 16, 3), ("bf16", 64, 32, 128, 64, 32, 2),
+                                                     ("bf16", 9, 5, 64, 64, 64, 1), ("f32", 12, 7, 40, 24, 8, 2)])
+@pytest.mark.parametrize("kind", [tda.TDA_KFAC, tda.TDA_EKFAC])
+def test_kfac_ekfac_match_oracle(dev, orc, dtype, N, T, di, do, k, chunks, kind):
+    # factor covariances streamed in chunks, Jacobi eigenbases, (EK-)FAC eigenvalues,
+    # damping 0.1 x mean eigenvalue, preconditioned queries: the whole chain vs the oracle
+    A, B = make_factors(N, T, di, do, dtype, stream=41, sigma_b=0.1, mask_p=0.02)
+    L = tda.LayerDesc(di, do, T, k, k, seed=8, layer=5)
+    Ad, Bd = to_dev(A, dtype, dev), to_dev(B, dtype, dev)
+    st = torch.empty(tda.tda_kfac_state_bytes(k, k) // 8, dtype=torch.float64, device=dev)
+    wsb = tda.tda_kfac_workspace_size(L, TD[dtype]) + 3 * 4 * T * 2 * k
+    ws = torch.empty(wsb, dtype=torch.uint8, device=dev)
+    tda.tda_kfac_reset(k, k, st)
+    assert Ad.shape == (N, T, di)
+    bounds = np.linspace(0, N, chunks + 1).astype(int)
+    for e0, e1 in zip(bounds[:-1], bounds[1:]):
+        tda.tda_kfac_accumulate_factors(L, TD[dtype], Ad[e0:], Bd[e0:], int(e1 - e0), st, ws, wsb)
+    tda.tda_kfac_eigen(k, k, st)
+    phi, _ = gpu_project(L, dtype, Ad, Bd, N, tda.TDA_ROUTE_FACTORED, dev)
+    phid = torch.from_numpy(phi.astype(np.float32)).to(dev)
+    if kind == tda.TDA_EKFAC:
+        tda.tda_kfac_accumulate_eigenvalues(k, k, st, phid[: N // 2], N // 2, k * k, ws, wsb)
+        tda.tda_kfac_accumulate_eigenvalues(k, k, st, phid[N // 2:], N - N // 2, k * k, ws, wsb)
+    nq = 5
+    Q = np.random.default_rng(k).standard_normal((nq, k * k)).astype(np.float32)
+    Qd = torch.from_numpy(Q).to(dev)
+    Qh = torch.full((nq, k * k + 3), float("nan"), device=dev)
+    tda.tda_kfac_apply(kind, k, k, st, 0.0, 0.1, Qd, nq, k * k, Qh, k * k + 3)
+    tda.tda_device_status()
+    A64, B64 = synth.to_f64(A, dtype), synth.to_f64(B, dtype)
+    phi64 = orc.project(A64, B64, k, k, 8, 5)
+    Ca, Cg, wa, wg, ref = _kfac_oracle(orc, A64, B64, k, 8, 5, kind, 0.0, 0.1, Q, phi64)
+    s = st.cpu().numpy()
+    M = s[0]
+    assert M == N * T
+    assert s[2] >= 0 and s[3] >= 0  # both Jacobi runs converged
+    np.testing.assert_allclose(s[8:8 + k * k].reshape(k, k) / M, Ca, rtol=2e-5, atol=1e-7 * np.abs(Ca).max())
+    o = 8 + k * k
+    np.testing.assert_allclose(s[o:o + k * k].reshape(k, k) / M, Cg, rtol=2e-5, atol=1e-7 * np.abs(Cg).max())
+    o += k * k
+    Ua = s[o:o + k * k].reshape(k, k)
+    np.testing.assert_allclose(Ua.T @ Ua, np.eye(k), atol=1e-12)
+    np.testing.assert_allclose(np.sort(s[o + k * k:o + k * k + k]), wa, rtol=1e-5, atol=1e-7 * wa.max())
+    got = Qh.cpu().numpy()
+    assert rel_fro(got[:, : k * k], ref) <= (1e-5 if dtype == "f32" else 1e-4)
+    assert np.isnan(got[:, k * k:]).all()
+
+
+@pytest.mark.gpu
+@pytest.mark.parametrize("N,T,di,do,k", [(700, 256, 64, 128, 64), (300, 16, 128, 64, 32), (20, 300, 64, 72, 16)])
+def test_project_kfac_fused_matches_oracle(dev, orc, N, T, di, do, k):
+    # covariances accumulated inside the tensor-core projection (one pass over the factors)
+    A, B = make_factors(N, T, di, do, "bf16", stream=43, sigma_b=0.05, mask_p=0.01)
+    L = tda.LayerDesc(di, do, T, k, k, seed=2, layer=1)
+    Ad, Bd = to_dev(A, "bf16", dev), to_dev(B, "bf16", dev)
+    st = torch.empty(tda.tda_kfac_state_bytes(k, k) // 8, dtype=torch.float64, device=dev)
+    wsb = tda.tda_kfac_workspace_size(L, tda.TDA_BF16)
+    ws = torch.empty(wsb, dtype=torch.uint8, device=dev)
+    phi = torch.full((N, k * k), float("nan"), device=dev)
+    tda.tda_kfac_reset(k, k, st)
+    tda.tda_project_kfac(L, tda.TDA_BF16, Ad, Bd, N, phi, k * k, st, ws, wsb)
+    tda.tda_device_status()
+    A64, B64 = synth.to_f64(A, "bf16"), synth.to_f64(B, "bf16")
+    ref_phi = orc.project(A64, B64, k, k, 2, 1)
+    assert rel_fro(phi.cpu().numpy().reshape(ref_phi.shape), ref_phi) <= 1e-5
+    Ca, Cg = orc.kfac_covariances(A64, B64, k, k, 2, 1)
+    s = st.cpu().numpy()
+    assert s[0] == N * T
+    assert rel_fro(s[8:8 + k * k].reshape(k, k) / s[0], Ca) <= 1e-5
+    assert rel_fro(s[8 + k * k:8 + 2 * k * k].reshape(k, k) / s[0], Cg) <= 1e-5
