@@ -71,6 +71,9 @@ def parse_args():
     p.add_argument("--k", type=int, default=32)
     p.add_argument("--topk", type=int, default=100)
     p.add_argument("--no-precondition", action="store_true")
+    p.add_argument("--curvature", default="fisher", choices=["fisher", "kfac", "ekfac"],
+                   help="preconditioner: full empirical Fisher of the projected features, or K-FAC / EK-FAC "
+                        "on the projected factors (damping 0.1 x mean eigenvalue)")
     p.add_argument("--e2e-steps", type=int, default=2)
     p.add_argument("--no-e2e", action="store_true")
     p.add_argument("--no-cpu-baseline", action="store_true")
@@ -96,7 +99,9 @@ def workload(args):
         "T": args.T, "n_train": args.n_train, "n_query": args.n_query,
         "k_in": args.k, "k_out": args.k, "features_per_example": len(LINEARS) * args.k * args.k,
         "factors": "A~N(0,1), B~N(0,1e-3), 1% tokens masked (seeded synthetic)",
-        "method": "GradDot" if args.no_precondition else "(F+lambda I)^-1-preconditioned, lambda=1e-2*mean eig",
+        "method": ("GradDot" if args.no_precondition else
+                   "(F+lambda I)^-1-preconditioned, lambda=1e-2*mean eig" if args.curvature == "fisher" else
+                   f"{args.curvature.upper()} on projected factors, lambda=0.1*mean eig"),
         "topk": args.topk, "l2": "inputs larger than L2 (no flush)",
         **({"mode": "project-only (kernel profiling)"} if args.project_only else {}),
     }
@@ -202,20 +207,39 @@ def oracle_sample(args, n_s, n_q_s, factors_of):
         t0 = time.perf_counter()
         qs.append(oracle.project(Aq, Bq, k, k, 0, li).reshape(n_q_s, D))
         t_query += time.perf_counter() - t0
-        if not args.no_precondition:
+        if not args.no_precondition and args.curvature == "fisher":
             t0 = time.perf_counter()
             F = oracle.fisher(phis[-1])
             t_fisher += time.perf_counter() - t0
             t0 = time.perf_counter()
             qs[-1] = oracle.precondition(F, oracle.damping(F, 0.0, 1e-2), qs[-1])
             t_factor += time.perf_counter() - t0
+        elif not args.no_precondition:
+            # K-FAC / EK-FAC: covariances and EK-FAC eigenvalues per train example,
+            # eigenbases once, the eigenbasis solve per query
+            t0 = time.perf_counter()
+            Ca, Cg = oracle.kfac_covariances(A, B, k, k, 0, li)
+            t_fisher += time.perf_counter() - t0
+            t0 = time.perf_counter()
+            wa, Ua, _ = oracle.sym_eig(Ca)
+            wg, Ug, _ = oracle.sym_eig(Cg)
+            t_factor += time.perf_counter() - t0
+            t0 = time.perf_counter()
+            Lam = (oracle.ekfac_eigenvalues(phis[-1].reshape(n_s, k, k), Ua, Ug) if args.curvature == "ekfac"
+                   else oracle.kfac_eigenvalues(wa, wg))
+            t_fisher += time.perf_counter() - t0
+            t0 = time.perf_counter()
+            qs[-1] = oracle.kfac_precondition(Ua, Ug, Lam, oracle.kfac_damping(Lam, 0.0, 0.1), qs[-1])
+            t_query += time.perf_counter() - t0
     t0 = time.perf_counter()
     S = oracle.score(np.concatenate(qs, 1), np.concatenate(phis, 1))
     oracle.topk(S, min(args.topk, n_s))
     t_score = time.perf_counter() - t0
     N, Nq = args.n_train, args.n_query
     total = (t_train + t_fisher + t_score * Nq / n_q_s) * N / n_s + t_query * Nq / n_q_s + t_factor
-    sample = (f"{n_s} train + {n_q_s} query examples (fp64, {threads} threads) through all 7 linears, Fisher/Cholesky/score on them; "
+    fit = {"fisher": "Fisher/Cholesky", "kfac": "K-FAC covariances/eigenbases",
+           "ekfac": "EK-FAC covariances/eigenbases/eigenvalues"}[args.curvature]
+    sample = (f"{n_s} train + {n_q_s} query examples (fp64, {threads} threads) through all 7 linears, {fit}/score on them; "
               f"per-train-example parts scaled by {N}/{n_s}, query parts by {Nq}/{n_q_s}, factorisation once")
     return N / total, threads, sample, t_train + t_query + t_fisher + t_factor + t_score
 
@@ -434,8 +458,10 @@ def main():
             store.append(x)
     from paper_2609_38767_gb300.block import BlockPipeline
 
+    kfac_mode = not args.no_precondition and args.curvature != "fisher"
     pipe = BlockPipeline([(di, do) for _, di, do in LINEARS], T, k, N, Nq, topk=args.topk,
-                         precondition=not args.no_precondition, lambda_rel=1e-2, device=dev)
+                         precondition=not args.no_precondition, lambda_rel=0.1 if kfac_mode else 1e-2, device=dev,
+                         curvature=args.curvature)
     layers, Phi, Q, idx, val = pipe.layers, pipe.Phi, pipe.Q, pipe.idx, pipe.val
     torch.cuda.synchronize()
 
@@ -476,7 +502,9 @@ def main():
         pipe.run(train, lambda li, L, route, phi, ld: project("query", li, L, route, phi, ld), after, mark)
 
     def project_dev(role, li, L, route, phi, ld):
-        if role == "train":
+        if role == "train" and kfac_mode:
+            pipe.project_train_kfac(li, At[li], Bt[li], phi, ld)
+        elif role == "train":
             tda.tda_project(L, tda.TDA_BF16, At[li], Bt[li], N, phi, ld, route)
         else:
             tda.tda_project(L, tda.TDA_BF16, Aq[li], Bq[li], Nq, phi, ld, route)
@@ -523,7 +551,7 @@ def main():
     roofline = {"bound": "hbm", "kernel": "factored projection (train, 7 linears)",
                 "engine": "tcgen05" if engines == [1] else ("cuda-core" if engines == [0] else "mixed"), "achieved": achieved,
                 "peak": hbm, "unit": "GB/s", "frac": achieved / hbm,
-                "traffic": TRAFFIC_RATIO * per_launch if (same_kernel and engines == [1]) else None,
+                "traffic": TRAFFIC_RATIO * per_launch if (same_kernel and engines == [1] and not kfac_mode) else None,
                 "algorithmic_bytes_per_launch": per_launch,
                 "peak_source": "MEASURED_PEAKS.json hbm_gbs" if peaks else "fallback 6.8 TB/s",
                 "share_of_step": proj_ms / (ms * args.steps)}
@@ -540,7 +568,9 @@ def main():
         "project_query": ("hbm", sum(Nq * (T * (L.d_in + L.d_out) * 2 + 4 * D) for L in layers), hbm, "GB/s"),
         "fisher_fit": ("alu", nl * N * Dn * (Dn + 1), alu, "TFLOP/s"),
         "factor": ("latency", nl * Dn ** 3 / 3, alu, "TFLOP/s"),
-        "apply": ("latency", nl * 2 * 2 * Dn * Dn * Nq, alu, "TFLOP/s"),
+        "apply": ("latency", (nl * 4 * 2 * Dn * k * Nq) if kfac_mode else (nl * 2 * 2 * Dn * Dn * Nq), alu, "TFLOP/s"),
+        "kfac_eigen": ("latency", nl * 2 * 10 * 4.0 * k ** 3, alu, "TFLOP/s"),
+        "ekfac_eigenvalues": ("alu", nl * N * 2 * 2 * Dn * k, alu, "TFLOP/s"),
         "score": ("alu", 2.0 * Nq * N * DT, alu, "TFLOP/s"),
         "topk": ("latency", 8.0 * Nq * N * 4, hbm, "GB/s"),
     }
@@ -553,7 +583,7 @@ def main():
 
     # ---- e2e through tda_project_host with pinned host factors
     e2e = None
-    if not args.no_e2e and not args.project_only:
+    if not args.no_e2e and not args.project_only and not kfac_mode:
         # pinned pools on the host memory nearest the GPU: this thread runs on the
         # GPU's NUMA node while the pools are allocated and first touched
         saved_aff, numa = bind_to_gpu_numa(local)

@@ -309,9 +309,14 @@ tda_status tda_precondition_info(int32_t n_layers, int64_t D, tda_dtype state_dt
  *   Qhat = U_g [(U_g^T Q U_a) / (Lam + lambda)] U_a^T  per query feature
  *   (Q, Qhat, Phi: k_out x k_in row-major, index r*k_in + c, as tda_project).
  *
- * `state`: device buffer of tda_kfac_state_bytes(k_in, k_out) bytes, 16-byte
- * aligned, fp64: an 8-double header (M, N, ...), the factor sums, the
- * eigenbases and eigenvalues, the EK-FAC sums. Calls in order of use:
+ * `state`: device buffer of n_layers * tda_kfac_state_bytes(k_in, k_out) bytes
+ * (layer l at byte l * tda_kfac_state_bytes), 16-byte aligned, fp64 per layer:
+ * an 8-double header (M, N, Jacobi sweeps), the factor sums, the eigenbases and
+ * eigenvalues, the EK-FAC sums. The n_layers calls (reset, eigen,
+ * accumulate_eigenvalues, apply) treat that many layers of equal k_in, k_out in
+ * one launch, their features side by side in each row (layer l at column
+ * l*k_in*k_out, as tda_precondition); accumulate_factors and project_kfac take
+ * one layer's factors and that layer's state. Calls in order of use:
  *   tda_kfac_reset                 zero the state.
  *   tda_kfac_accumulate_factors    add the factor covariance sums of N training
  *                                  examples (A, B as tda_project). ws >=
@@ -340,17 +345,18 @@ tda_status tda_precondition_info(int32_t n_layers, int64_t D, tda_dtype state_dt
 #define TDA_EKFAC 1
 size_t tda_kfac_state_bytes(int32_t k_in, int32_t k_out);
 size_t tda_kfac_workspace_size(const tda_layer_desc* L, tda_dtype dtype);
-tda_status tda_kfac_reset(int32_t k_in, int32_t k_out, void* state, void* stream);
+tda_status tda_kfac_reset(int32_t n_layers, int32_t k_in, int32_t k_out, void* state, void* stream);
 tda_status tda_kfac_accumulate_factors(const tda_layer_desc* L, tda_dtype dtype, const void* A, const void* B,
                                        int64_t N, void* state, void* ws, size_t ws_bytes, void* stream);
 tda_status tda_project_kfac(const tda_layer_desc* L, tda_dtype dtype, const void* A, const void* B, int64_t N,
                             float* phi, int64_t ld_phi, void* state, void* ws, size_t ws_bytes, void* stream);
-tda_status tda_kfac_eigen(int32_t k_in, int32_t k_out, void* state, void* stream);
-tda_status tda_kfac_accumulate_eigenvalues(int32_t k_in, int32_t k_out, void* state, const float* phi,
-                                           int64_t n, int64_t ld_phi, void* ws, size_t ws_bytes, void* stream);
-tda_status tda_kfac_apply(int32_t kind, int32_t k_in, int32_t k_out, const void* state, double lambda_abs,
-                          double lambda_rel, const float* q, int64_t n_q, int64_t ld_q, float* qhat,
-                          int64_t ld_qhat, void* stream);
+tda_status tda_kfac_eigen(int32_t n_layers, int32_t k_in, int32_t k_out, void* state, void* stream);
+tda_status tda_kfac_accumulate_eigenvalues(int32_t n_layers, int32_t k_in, int32_t k_out, void* state,
+                                           const float* phi, int64_t n, int64_t ld_phi, void* ws, size_t ws_bytes,
+                                           void* stream);
+tda_status tda_kfac_apply(int32_t kind, int32_t n_layers, int32_t k_in, int32_t k_out, const void* state,
+                          double lambda_abs, double lambda_rel, const float* q, int64_t n_q, int64_t ld_q,
+                          float* qhat, int64_t ld_qhat, void* stream);
 
 /* ---------------------------------------------------------------------------
  * tda_score -- S[q][i] = beta*S[q][i] + sum_f Qhat[q][f] Phi[i][f]

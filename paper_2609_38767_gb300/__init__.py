@@ -92,12 +92,12 @@ def load() -> ctypes.CDLL:
             "tda_precondition_state_bytes": (SZ, [I64, I32]),
             "tda_kfac_state_bytes": (SZ, [I32, I32]),
             "tda_kfac_workspace_size": (SZ, [LP, I32]),
-            "tda_kfac_reset": (I32, [I32, I32, P, P]),
+            "tda_kfac_reset": (I32, [I32, I32, I32, P, P]),
             "tda_kfac_accumulate_factors": (I32, [LP, I32, P, P, I64, P, P, SZ, P]),
             "tda_project_kfac": (I32, [LP, I32, P, P, I64, P, I64, P, P, SZ, P]),
-            "tda_kfac_eigen": (I32, [I32, I32, P, P]),
-            "tda_kfac_accumulate_eigenvalues": (I32, [I32, I32, P, P, I64, I64, P, SZ, P]),
-            "tda_kfac_apply": (I32, [I32, I32, I32, P, D, D, P, I64, I64, P, I64, P]),
+            "tda_kfac_eigen": (I32, [I32, I32, I32, P, P]),
+            "tda_kfac_accumulate_eigenvalues": (I32, [I32, I32, I32, P, P, I64, I64, P, SZ, P]),
+            "tda_kfac_apply": (I32, [I32, I32, I32, I32, P, D, D, P, I64, I64, P, I64, P]),
             "tda_precondition": (I32, [I32, I32, I64, I32, P, P, I64, I64, I64, D, D, P, I64, I64, P, I64, P]),
             "tda_precondition_info": (I32, [I32, I64, I32, P, ctypes.POINTER(D), P]),
             "tda_score": (I32, [P, I32, I64, I64, P, I64, I64, I64, P, I64, F, P]),
@@ -222,8 +222,8 @@ def tda_kfac_workspace_size(L, dtype) -> int:
     return int(load().tda_kfac_workspace_size(ctypes.byref(L), dtype))
 
 
-def tda_kfac_reset(k_in, k_out, state, stream=None):
-    _check(load().tda_kfac_reset(k_in, k_out, _ptr(state), _stream(stream)))
+def tda_kfac_reset(k_in, k_out, state, stream=None, n_layers=1):
+    _check(load().tda_kfac_reset(n_layers, k_in, k_out, _ptr(state), _stream(stream)))
 
 
 def tda_kfac_accumulate_factors(L, dtype, A, B, N, state, ws, ws_bytes, stream=None):
@@ -236,18 +236,19 @@ def tda_project_kfac(L, dtype, A, B, N, phi, ld_phi, state, ws, ws_bytes, stream
                                    _ptr(ws), ws_bytes, _stream(stream)))
 
 
-def tda_kfac_eigen(k_in, k_out, state, stream=None):
-    _check(load().tda_kfac_eigen(k_in, k_out, _ptr(state), _stream(stream)))
+def tda_kfac_eigen(k_in, k_out, state, stream=None, n_layers=1):
+    _check(load().tda_kfac_eigen(n_layers, k_in, k_out, _ptr(state), _stream(stream)))
 
 
-def tda_kfac_accumulate_eigenvalues(k_in, k_out, state, phi, n, ld_phi, ws, ws_bytes, stream=None):
-    _check(load().tda_kfac_accumulate_eigenvalues(k_in, k_out, _ptr(state), _ptr(phi), n, ld_phi, _ptr(ws), ws_bytes,
-                                                  _stream(stream)))
+def tda_kfac_accumulate_eigenvalues(k_in, k_out, state, phi, n, ld_phi, ws, ws_bytes, stream=None, n_layers=1):
+    _check(load().tda_kfac_accumulate_eigenvalues(n_layers, k_in, k_out, _ptr(state), _ptr(phi), n, ld_phi, _ptr(ws),
+                                                  ws_bytes, _stream(stream)))
 
 
-def tda_kfac_apply(kind, k_in, k_out, state, lambda_abs, lambda_rel, q, n_q, ld_q, qhat, ld_qhat, stream=None):
-    _check(load().tda_kfac_apply(kind, k_in, k_out, _ptr(state), float(lambda_abs), float(lambda_rel), _ptr(q), n_q,
-                                 ld_q, _ptr(qhat), ld_qhat, _stream(stream)))
+def tda_kfac_apply(kind, k_in, k_out, state, lambda_abs, lambda_rel, q, n_q, ld_q, qhat, ld_qhat, stream=None,
+                   n_layers=1):
+    _check(load().tda_kfac_apply(kind, n_layers, k_in, k_out, _ptr(state), float(lambda_abs), float(lambda_rel),
+                                 _ptr(q), n_q, ld_q, _ptr(qhat), ld_qhat, _stream(stream)))
 
 
 def tda_precondition_state_bytes(D, state_dtype) -> int:

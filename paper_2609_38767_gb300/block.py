@@ -4,7 +4,9 @@ A transformer block's linears (e.g. q, k, v, o, gate, up, down) share the token
 count T and the projection size k. For a batch of train and query examples the
 pass is: route choice per linear (Sec. 3.2 / App. A.4 cost model), factored
 projection of every example through every linear (Eq. 2), the per-linear Fisher
-fit and damped inverse applied to the queries (App. B.2, B.3), the query x train
+fit and damped inverse applied to the queries (App. B.2, B.3) -- the full empirical
+Fisher of the projected features, or K-FAC / EK-FAC on the projected factors with
+the covariances accumulated by the projection kernel itself -- the query x train
 score matrix summed over the linears (Eq. 4's left side) and the top-k train
 indices per query. Every step is a libtda.so call; this class only owns the
 device buffers and the order of the calls.
@@ -21,14 +23,17 @@ import paper_2609_38767_gb300 as tda
 
 
 class BlockPipeline:
+    CURVATURES = ("fisher", "kfac", "ekfac")
+
     def __init__(self, linears, T, k, n_train, n_query, *, topk=100, precondition=True,
-                 lambda_abs=0.0, lambda_rel=1e-2, seed=0, layer0=0, device="cuda"):
+                 lambda_abs=0.0, lambda_rel=1e-2, seed=0, layer0=0, device="cuda", curvature="fisher"):
+        assert curvature in self.CURVATURES
         self.layers = [tda.LayerDesc(di, do, T, k, k, seed=seed, layer=layer0 + i)
                        for i, (di, do) in enumerate(linears)]
         self.N, self.Nq, self.D = n_train, n_query, k * k
         self.nl = len(self.layers)
         self.DT = self.D * self.nl
-        self.topk, self.precondition = topk, precondition
+        self.topk, self.precondition, self.curvature = topk, precondition, curvature
         self.lambda_abs, self.lambda_rel = lambda_abs, lambda_rel
         dev = torch.device(device)
         self.Phi = torch.empty((n_train, self.DT), dtype=torch.float32, device=dev)
@@ -37,8 +42,21 @@ class BlockPipeline:
         self.S = torch.empty((n_query, n_train), dtype=torch.float32, device=dev)
         self.idx = torch.empty((n_query, topk), dtype=torch.int32, device=dev)
         self.val = torch.empty((n_query, topk), dtype=torch.float32, device=dev)
-        per = tda.tda_precondition_state_bytes(self.D, tda.TDA_F32)
-        self.state = torch.empty(self.nl * per, dtype=torch.uint8, device=dev)
+        self.k = k
+        if curvature == "fisher":
+            per = tda.tda_precondition_state_bytes(self.D, tda.TDA_F32)
+            self.state = torch.empty(self.nl * per, dtype=torch.uint8, device=dev)
+        else:
+            self.kf_per = tda.tda_kfac_state_bytes(k, k)
+            self.kf_states = torch.empty(self.nl * self.kf_per, dtype=torch.uint8, device=dev)
+            self.kf_state = [self.kf_states[i * self.kf_per:(i + 1) * self.kf_per] for i in range(self.nl)]
+            self.kf_wsb = max(tda.tda_kfac_workspace_size(L, tda.TDA_BF16) for L in self.layers)
+            self.kf_ws = torch.empty(self.kf_wsb, dtype=torch.uint8, device=dev)
+
+    def project_train_kfac(self, li, A, B, phi, ld):
+        """Train projection of linear li that also accumulates its K-FAC factor covariances."""
+        tda.tda_project_kfac(self.layers[li], tda.TDA_BF16, A, B, self.N, phi, ld, self.kf_state[li], self.kf_ws,
+                             self.kf_wsb)
 
     def routes(self):
         return [tda.tda_route(L, tda.TDA_OP_PROJECT, self.N, 0, tda.TDA_BF16)[0] for L in self.layers]
@@ -51,6 +69,9 @@ class BlockPipeline:
         mark = mark or (lambda name: None)
         routes = self.routes()
         D, DT = self.D, self.DT
+        kfac = self.precondition and self.curvature != "fisher"
+        if kfac:
+            tda.tda_kfac_reset(self.k, self.k, self.kf_states, n_layers=self.nl)
         mark("project_train")
         for li, L in enumerate(self.layers):
             project_train(li, L, routes[li], self.Phi[:, li * D:], DT)
@@ -60,7 +81,21 @@ class BlockPipeline:
         for li, L in enumerate(self.layers):
             project_query(li, L, routes[li], self.Q[:, li * D:], DT)
         target = self.Q
-        if self.precondition:
+        if kfac:
+            k = self.k
+            nl, sts = self.nl, self.kf_states
+            mark("kfac_eigen")
+            tda.tda_kfac_eigen(k, k, sts, n_layers=nl)
+            if self.curvature == "ekfac":
+                mark("ekfac_eigenvalues")
+                tda.tda_kfac_accumulate_eigenvalues(k, k, sts, self.Phi, self.N, DT, self.kf_ws, self.kf_wsb,
+                                                    n_layers=nl)
+            mark("apply")
+            kind = tda.TDA_EKFAC if self.curvature == "ekfac" else tda.TDA_KFAC
+            tda.tda_kfac_apply(kind, k, k, sts, self.lambda_abs, self.lambda_rel, self.Q, self.Nq, DT, self.Qh, DT,
+                               n_layers=nl)
+            target = self.Qh
+        elif self.precondition:
             nl, st, f32 = self.nl, self.state, tda.TDA_F32
             mark("fisher_fit")
             tda.tda_precondition(tda.TDA_PC_RESET, nl, D, f32, st)

@@ -560,11 +560,13 @@ static tda_status kfac_state_ok(int64_t ka, int64_t kg, const void* state) {
     return TDA_OK;
 }
 
-tda_status tda_kfac_reset(int32_t k_in, int32_t k_out, void* state, void* stream) {
+tda_status tda_kfac_reset(int32_t n_layers, int32_t k_in, int32_t k_out, void* state, void* stream) {
     g_msg[0] = 0;
     tda_status st = kfac_state_ok(k_in, k_out, state);
     if (st) return st;
-    return cuda_check(cudaMemsetAsync(state, 0, kfac_state_bytes(k_in, k_out), (cudaStream_t)stream), "kfac reset");
+    if (n_layers < 1 || n_layers > 65535) return fail(TDA_ERR_INVALID_ARG, "n_layers must be in [1, 65535]");
+    return cuda_check(cudaMemsetAsync(state, 0, (size_t)n_layers * kfac_state_bytes(k_in, k_out), (cudaStream_t)stream),
+                      "kfac reset");
 }
 
 tda_status tda_kfac_accumulate_factors(const tda_layer_desc* L, tda_dtype dtype, const void* A, const void* B,
@@ -645,44 +647,62 @@ tda_status tda_project_kfac(const tda_layer_desc* L, tda_dtype dtype, const void
                       "kfac sums g");
 }
 
-tda_status tda_kfac_eigen(int32_t k_in, int32_t k_out, void* state, void* stream) {
+tda_status tda_kfac_eigen(int32_t n_layers, int32_t k_in, int32_t k_out, void* state, void* stream) {
     g_msg[0] = 0;
     tda_status st = kfac_state_ok(k_in, k_out, state);
     if (st) return st;
-    return cuda_check(launch_kfac_eigen((double*)state, k_in, k_out, (cudaStream_t)stream), "kfac eigen");
+    if (n_layers < 1 || n_layers > 65535) return fail(TDA_ERR_INVALID_ARG, "n_layers must be in [1, 65535]");
+    return cuda_check(launch_kfac_eigen(n_layers, (double*)state, k_in, k_out, (cudaStream_t)stream), "kfac eigen");
 }
 
-tda_status tda_kfac_accumulate_eigenvalues(int32_t k_in, int32_t k_out, void* state, const float* phi, int64_t n,
-                                           int64_t ld_phi, void* ws, size_t ws_bytes, void* stream) {
+tda_status tda_kfac_accumulate_eigenvalues(int32_t n_layers, int32_t k_in, int32_t k_out, void* state,
+                                           const float* phi, int64_t n, int64_t ld_phi, void* ws, size_t ws_bytes,
+                                           void* stream) {
     g_msg[0] = 0;
     tda_status st = kfac_state_ok(k_in, k_out, state);
     if (st) return st;
-    if (n < 0 || (n > 0 && (!phi || ld_phi < (int64_t)k_in * k_out)))
-        return fail(TDA_ERR_INVALID_ARG, "phi is NULL or ld_phi < k_in*k_out");
+    if (n_layers < 1 || n_layers > 65535) return fail(TDA_ERR_INVALID_ARG, "n_layers must be in [1, 65535]");
+    const int64_t D = (int64_t)k_in * k_out;
+    if (n < 0 || (n > 0 && (!phi || ld_phi < (int64_t)n_layers * D)))
+        return fail(TDA_ERR_INVALID_ARG, "phi is NULL or ld_phi < n_layers*k_in*k_out");
     const size_t need = kfac_partials_bytes(k_in, k_out);
     if (!ws || ws_bytes < need)
         return fail(TDA_ERR_WORKSPACE, "tda_kfac_accumulate_eigenvalues needs >= %zu bytes of ws, got %zu", need,
                     ws_bytes);
-    int nblk = (int)(n < 304 ? n : 304);
-    if (nblk < 1) nblk = 1;
-    return cuda_check(launch_kfac_ekfac_accum((double*)state, k_in, k_out, phi, n, ld_phi, (float*)ws, nblk,
-                                              (cudaStream_t)stream),
-                      "ekfac eigenvalues");
+    // every (layer, block) pair writes one partial of D floats into ws
+    const int64_t slabs = (int64_t)(ws_bytes / (sizeof(float) * (size_t)D));
+    const size_t lbytes = kfac_state_bytes(k_in, k_out);
+    for (int32_t l0 = 0; l0 < n_layers;) {
+        int32_t nl = n_layers - l0;
+        if (nl > slabs) nl = (int32_t)slabs;
+        int64_t nblk = slabs / nl;
+        if (nblk > 304 / nl) nblk = 304 / nl;
+        if (nblk > n) nblk = n;
+        if (nblk < 1) nblk = 1;
+        if ((st = cuda_check(launch_kfac_ekfac_accum(nl, (double*)((char*)state + (size_t)l0 * lbytes), k_in, k_out,
+                                                     phi + (int64_t)l0 * D, n, ld_phi, (float*)ws, (int)nblk,
+                                                     (cudaStream_t)stream),
+                             "ekfac eigenvalues")))
+            return st;
+        l0 += nl;
+    }
+    return TDA_OK;
 }
 
-tda_status tda_kfac_apply(int32_t kind, int32_t k_in, int32_t k_out, const void* state, double lambda_abs,
-                          double lambda_rel, const float* q, int64_t n_q, int64_t ld_q, float* qhat, int64_t ld_qhat,
-                          void* stream) {
+tda_status tda_kfac_apply(int32_t kind, int32_t n_layers, int32_t k_in, int32_t k_out, const void* state,
+                          double lambda_abs, double lambda_rel, const float* q, int64_t n_q, int64_t ld_q, float* qhat,
+                          int64_t ld_qhat, void* stream) {
     g_msg[0] = 0;
     tda_status st = kfac_state_ok(k_in, k_out, state);
     if (st) return st;
     if (kind != TDA_KFAC && kind != TDA_EKFAC) return fail(TDA_ERR_INVALID_ARG, "kind must be TDA_KFAC or TDA_EKFAC");
+    if (n_layers < 1 || n_layers > 65535) return fail(TDA_ERR_INVALID_ARG, "n_layers must be in [1, 65535]");
     const int64_t D = (int64_t)k_in * k_out;
     if (n_q < 0 || n_q > 2147483647LL) return fail(TDA_ERR_INVALID_ARG, "bad n_q");
-    if (n_q > 0 && (!q || !qhat || ld_q < D || ld_qhat < D))
-        return fail(TDA_ERR_INVALID_ARG, "q/qhat NULL or leading dimension < k_in*k_out");
-    return cuda_check(launch_kfac_apply(kind, (const double*)state, k_in, k_out, lambda_abs, lambda_rel, q, n_q, ld_q,
-                                        qhat, ld_qhat, (cudaStream_t)stream),
+    if (n_q > 0 && (!q || !qhat || ld_q < n_layers * D || ld_qhat < n_layers * D))
+        return fail(TDA_ERR_INVALID_ARG, "q/qhat NULL or leading dimension < n_layers*k_in*k_out");
+    return cuda_check(launch_kfac_apply(kind, n_layers, (const double*)state, k_in, k_out, lambda_abs, lambda_rel, q,
+                                        n_q, ld_q, qhat, ld_qhat, (cudaStream_t)stream),
                       "kfac apply");
 }
 

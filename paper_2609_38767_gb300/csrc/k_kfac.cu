@@ -85,35 +85,39 @@ __global__ void sum_partials_kernel(const float* __restrict__ part, int nblk, in
 }
 
 // Parallel cyclic Jacobi (round-robin pair ordering) on C = S / M for the
-// a side (blockIdx.x 0) and the g side (1). A lives in shared memory, the
-// eigenvectors accumulate in the state's U (V <- V J). Each round rotates
-// floor(m/2) disjoint pairs at once: angles from the round's starting matrix,
-// then all row updates, then all column updates, which is J^T A J for the
-// product J of the round's rotations.
-__global__ void __launch_bounds__(kKfThreads) jacobi_kernel(double* __restrict__ st, int64_t ka, int64_t kg) {
-    extern __shared__ double A[];  // [n][n], then c, s, p, q per pair
+// a side (blockIdx.x 0) and the g side (1) of layer blockIdx.y. A lives in
+// shared memory, the eigenvectors V (V <- V J) too when n <= 64 (else in the
+// state's U). Each round rotates floor(m/2) disjoint pairs at once: angles from
+// the round's starting matrix, then all row updates, then all column updates,
+// which is J^T A J for the product J of the round's rotations.
+__global__ void __launch_bounds__(kKfThreads)
+jacobi_kernel(double* __restrict__ st0, int64_t stride, int64_t ka, int64_t kg) {
+    extern __shared__ double A[];  // [n][n], V [n][n] when n <= 64, then c, s, p, q per pair
+    double* st = st0 + (int64_t)blockIdx.y * stride;
     const KfLayout l(ka, kg);
     const bool side_g = blockIdx.x == 1;
     const int n = (int)(side_g ? kg : ka);
     const double* S = st + (side_g ? l.Sg : l.Sa);
     double* U = st + (side_g ? l.Ug : l.Ua);
     double* w = st + (side_g ? l.wg : l.wa);
+    const int nmax = (int)(ka > kg ? ka : kg);
+    const bool v_shared = nmax <= 64;
+    double* V = v_shared ? A + nmax * nmax : U;
     const int m = (n + 1) & ~1;  // even number of players; index n is a dummy when n is odd
-    double* cs = A + n * n;
-    double* sn = cs + m / 2;
-    int* P = (int*)(sn + m / 2);
-    int* Q = P + m / 2;
+    double* cs = A + (v_shared ? 2 : 1) * nmax * nmax;
+    double* sn = cs + (nmax + 2) / 2;
+    int* P = (int*)(sn + (nmax + 2) / 2);
+    int* Q = P + (nmax + 2) / 2;
     __shared__ double red[kKfThreads];
     __shared__ int done;
     const double Mtok = st[0];
     const double inv = Mtok > 0 ? 1.0 / Mtok : 0.0;
     for (int e = threadIdx.x; e < n * n; e += blockDim.x) {
         A[e] = S[e] * inv;
-        U[e] = (e / n == e % n) ? 1.0 : 0.0;
+        V[e] = (e / n == e % n) ? 1.0 : 0.0;
     }
     __syncthreads();
-    // squared Frobenius norm
-    double f = 0.0;
+    double f = 0.0;  // squared Frobenius norm
     for (int e = threadIdx.x; e < n * n; e += blockDim.x) f += A[e] * A[e];
     red[threadIdx.x] = f;
     __syncthreads();
@@ -146,18 +150,18 @@ __global__ void __launch_bounds__(kKfThreads) jacobi_kernel(double* __restrict__
                     p = q;
                     q = t;
                 }
-                double c = 1.0, s = 0.0;
+                double c = 1.0, sv = 0.0;
                 if (q < n) {
                     const double apq = A[p * n + q];
                     if (apq != 0.0) {
                         const double tau = (A[q * n + q] - A[p * n + p]) / (2.0 * apq);
                         const double t = (tau >= 0 ? 1.0 : -1.0) / (fabs(tau) + sqrt(1.0 + tau * tau));
                         c = 1.0 / sqrt(1.0 + t * t);
-                        s = t * c;
+                        sv = t * c;
                     }
                 }
                 cs[i] = c;
-                sn[i] = s;
+                sn[i] = sv;
                 P[i] = p;
                 Q[i] = q < n ? q : -1;
             }
@@ -167,27 +171,29 @@ __global__ void __launch_bounds__(kKfThreads) jacobi_kernel(double* __restrict__
                 const int i = x / n, k = x - (x / n) * n;
                 if (Q[i] < 0 || sn[i] == 0.0) continue;
                 const int p = P[i], q = Q[i];
-                const double c = cs[i], s = sn[i], apk = A[p * n + k], aqk = A[q * n + k];
-                A[p * n + k] = c * apk - s * aqk;
-                A[q * n + k] = s * apk + c * aqk;
+                const double c = cs[i], sv = sn[i], apk = A[p * n + k], aqk = A[q * n + k];
+                A[p * n + k] = c * apk - sv * aqk;
+                A[q * n + k] = sv * apk + c * aqk;
             }
             __syncthreads();
             for (int x = threadIdx.x; x < half * n; x += blockDim.x) {  // columns p, q: A <- A J, V <- V J
                 const int i = x / n, k = x - (x / n) * n;
                 if (Q[i] < 0 || sn[i] == 0.0) continue;
                 const int p = P[i], q = Q[i];
-                const double c = cs[i], s = sn[i];
+                const double c = cs[i], sv = sn[i];
                 const double akp = A[k * n + p], akq = A[k * n + q];
-                A[k * n + p] = c * akp - s * akq;
-                A[k * n + q] = s * akp + c * akq;
-                const double vkp = U[k * n + p], vkq = U[k * n + q];
-                U[k * n + p] = c * vkp - s * vkq;
-                U[k * n + q] = s * vkp + c * vkq;
+                A[k * n + p] = c * akp - sv * akq;
+                A[k * n + q] = sv * akp + c * akq;
+                const double vkp = V[k * n + p], vkq = V[k * n + q];
+                V[k * n + p] = c * vkp - sv * vkq;
+                V[k * n + q] = sv * vkp + c * vkq;
             }
             __syncthreads();
         }
     }
     for (int i = threadIdx.x; i < n; i += blockDim.x) w[i] = A[i * n + i];
+    if (v_shared)
+        for (int e = threadIdx.x; e < n * n; e += blockDim.x) U[e] = V[e];
     if (threadIdx.x == 0) st[2 + (side_g ? 1 : 0)] = done ? (double)sweep : -1.0;
     if (blockIdx.x == 0) {  // a new eigenbasis invalidates the EK-FAC sums
         for (int64_t e = threadIdx.x; e < ka * kg; e += blockDim.x) st[l.Le + e] = 0.0;
@@ -195,30 +201,49 @@ __global__ void __launch_bounds__(kKfThreads) jacobi_kernel(double* __restrict__
     }
 }
 
-// part[b][r*ka+c] = sum over the examples of block b of ((U_g^T Phi_i U_a)[r][c])^2
+// Eigenbases of one layer as fp32 in shared memory (SU) or read from the fp64
+// state (large k).
+template <bool SU>
+struct Bases {
+    const float* ua;
+    const float* ug;
+    const double* uad;
+    const double* ugd;
+    __device__ __forceinline__ float a(int64_t i) const { return SU ? ua[i] : (float)uad[i]; }
+    __device__ __forceinline__ float g(int64_t i) const { return SU ? ug[i] : (float)ugd[i]; }
+};
+
+// part[layer][b][r*ka+c] = sum over the examples of block b of ((U_g^T Phi_i U_a)[r][c])^2
+template <bool SU>
 __global__ void __launch_bounds__(kKfThreads)
-ekfac_partial_kernel(const float* __restrict__ phi, int64_t n, int64_t ld, const double* __restrict__ st, int64_t ka,
-                     int64_t kg, float* __restrict__ part) {
-    extern __shared__ float sm[];  // Phi_i [kg][ka], Y [kg][ka]
+ekfac_partial_kernel(const float* __restrict__ phi, int64_t n, int64_t ld, const double* __restrict__ st0,
+                     int64_t stride, int64_t ka, int64_t kg, float* __restrict__ part) {
+    extern __shared__ float sm[];  // [U_a, U_g if SU] Phi_i [kg][ka], Y [kg][ka]
+    const int layer = blockIdx.y;
+    const double* st = st0 + (int64_t)layer * stride;
     const KfLayout l(ka, kg);
-    const double* Ua = st + l.Ua;
-    const double* Ug = st + l.Ug;
-    float* F = sm;
-    float* Y = sm + kg * ka;
     const int64_t D = ka * kg;
+    float* F = sm + (SU ? ka * ka + kg * kg : 0);
+    float* Y = F + D;
+    Bases<SU> U{sm, sm + ka * ka, st + l.Ua, st + l.Ug};
+    if (SU) {
+        for (int64_t e = threadIdx.x; e < ka * ka; e += blockDim.x) sm[e] = (float)st[l.Ua + e];
+        for (int64_t e = threadIdx.x; e < kg * kg; e += blockDim.x) sm[ka * ka + e] = (float)st[l.Ug + e];
+    }
+    const float* ph = phi + (int64_t)layer * D;
     constexpr int kMaxPer = 64;
     float acc[kMaxPer];
 #pragma unroll
     for (int m = 0; m < kMaxPer; ++m) acc[m] = 0.f;
     for (int64_t i = blockIdx.x; i < n; i += gridDim.x) {
         __syncthreads();
-        for (int64_t e = threadIdx.x; e < D; e += blockDim.x) F[e] = phi[i * ld + e];
+        for (int64_t e = threadIdx.x; e < D; e += blockDim.x) F[e] = ph[i * ld + e];
         __syncthreads();
         for (int64_t e = threadIdx.x; e < D; e += blockDim.x) {  // Y = Phi U_a
             const int64_t r = e / ka, c = e - (e / ka) * ka;
-            float s = 0.f;
-            for (int64_t j = 0; j < ka; ++j) s = fmaf(F[r * ka + j], (float)Ua[j * ka + c], s);
-            Y[e] = s;
+            float sacc = 0.f;
+            for (int64_t j = 0; j < ka; ++j) sacc = fmaf(F[r * ka + j], U.a(j * ka + c), sacc);
+            Y[e] = sacc;
         }
         __syncthreads();
 #pragma unroll
@@ -226,13 +251,13 @@ ekfac_partial_kernel(const float* __restrict__ phi, int64_t n, int64_t ld, const
             const int64_t e = threadIdx.x + (int64_t)m * kKfThreads;
             if (e < D) {
                 const int64_t r = e / ka, c = e - (e / ka) * ka;
-                float s = 0.f;
-                for (int64_t j = 0; j < kg; ++j) s = fmaf((float)Ug[j * kg + r], Y[j * ka + c], s);
-                acc[m] = fmaf(s, s, acc[m]);
+                float sacc = 0.f;
+                for (int64_t j = 0; j < kg; ++j) sacc = fmaf(U.g(j * kg + r), Y[j * ka + c], sacc);
+                acc[m] = fmaf(sacc, sacc, acc[m]);
             }
         }
     }
-    float* out = part + (int64_t)blockIdx.x * D;
+    float* out = part + ((int64_t)layer * gridDim.x + blockIdx.x) * D;
 #pragma unroll
     for (int m = 0; m < kMaxPer; ++m) {
         const int64_t e = threadIdx.x + (int64_t)m * kKfThreads;
@@ -240,19 +265,40 @@ ekfac_partial_kernel(const float* __restrict__ phi, int64_t n, int64_t ld, const
     }
 }
 
-// One CTA per query row: Qhat = U_g [(U_g^T Q U_a) / (Lam + lambda)] U_a^T,
-// fp64 accumulation, fp32 intermediates in shared memory.
-__global__ void __launch_bounds__(kKfThreads)
-kfac_apply_kernel(int kind, const double* __restrict__ st, int64_t ka, int64_t kg, double lambda_abs,
-                  double lambda_rel, const float* __restrict__ q, int64_t ld_q, float* __restrict__ qhat,
-                  int64_t ld_qhat) {
-    extern __shared__ float sm[];  // X [kg][ka], Y [kg][ka]
+// Le of every layer += its block partials (fixed order); N += n
+__global__ void ekfac_reduce_kernel(const float* __restrict__ part, int nblk, double* __restrict__ st0, int64_t stride,
+                                    int64_t ka, int64_t kg, double n) {
+    const int layer = blockIdx.y;
+    double* st = st0 + (int64_t)layer * stride;
     const KfLayout l(ka, kg);
-    const double* Ua = st + l.Ua;
-    const double* Ug = st + l.Ug;
     const int64_t D = ka * kg;
-    float* X = sm;
-    float* Y = sm + D;
+    const float* pl = part + (int64_t)layer * nblk * D;
+    for (int64_t e = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; e < D; e += (int64_t)gridDim.x * blockDim.x) {
+        double v = 0.0;
+        for (int b = 0; b < nblk; ++b) v += (double)pl[(int64_t)b * D + e];
+        st[l.Le + e] += v;
+    }
+    if (blockIdx.x == 0 && threadIdx.x == 0) st[1] += n;
+}
+
+// One CTA per (query row, layer): Qhat = U_g [(U_g^T Q U_a) / (Lam + lambda)] U_a^T
+template <bool SU>
+__global__ void __launch_bounds__(kKfThreads)
+kfac_apply_kernel(int kind, const double* __restrict__ st0, int64_t stride, int64_t ka, int64_t kg,
+                  double lambda_abs, double lambda_rel, const float* __restrict__ q, int64_t ld_q,
+                  float* __restrict__ qhat, int64_t ld_qhat) {
+    extern __shared__ float sm[];  // [U_a, U_g if SU] X [kg][ka], Y [kg][ka]
+    const int layer = blockIdx.y;
+    const double* st = st0 + (int64_t)layer * stride;
+    const KfLayout l(ka, kg);
+    const int64_t D = ka * kg;
+    float* X = sm + (SU ? ka * ka + kg * kg : 0);
+    float* Y = X + D;
+    Bases<SU> U{sm, sm + ka * ka, st + l.Ua, st + l.Ug};
+    if (SU) {
+        for (int64_t e = threadIdx.x; e < ka * ka; e += blockDim.x) sm[e] = (float)st[l.Ua + e];
+        for (int64_t e = threadIdx.x; e < kg * kg; e += blockDim.x) sm[ka * ka + e] = (float)st[l.Ug + e];
+    }
     __shared__ double red[kKfThreads];
     const double nex = st[1];
     auto lam_of = [&](int64_t e) -> double {
@@ -260,45 +306,45 @@ kfac_apply_kernel(int kind, const double* __restrict__ st, int64_t ka, int64_t k
         if (kind == 0) return st[l.wg + r] * st[l.wa + c];
         return nex > 0 ? st[l.Le + e] / nex : 0.0;
     };
-    double s = 0.0;
-    for (int64_t e = threadIdx.x; e < D; e += blockDim.x) s += lam_of(e);
-    red[threadIdx.x] = s;
+    double sacc = 0.0;
+    for (int64_t e = threadIdx.x; e < D; e += blockDim.x) sacc += lam_of(e);
+    red[threadIdx.x] = sacc;
     __syncthreads();
     for (int h = blockDim.x / 2; h > 0; h >>= 1) {
         if (threadIdx.x < h) red[threadIdx.x] += red[threadIdx.x + h];
         __syncthreads();
     }
     const double lambda = lambda_abs + lambda_rel * red[0] / (double)D;
-    const float* qi = q + (int64_t)blockIdx.x * ld_q;
+    const float* qi = q + (int64_t)blockIdx.x * ld_q + (int64_t)layer * D;
     for (int64_t e = threadIdx.x; e < D; e += blockDim.x) X[e] = qi[e];
     __syncthreads();
     for (int64_t e = threadIdx.x; e < D; e += blockDim.x) {  // Y = Q U_a
         const int64_t r = e / ka, c = e - (e / ka) * ka;
-        double a = 0.0;
-        for (int64_t j = 0; j < ka; ++j) a += (double)X[r * ka + j] * Ua[j * ka + c];
-        Y[e] = (float)a;
+        float a = 0.f;
+        for (int64_t j = 0; j < ka; ++j) a = fmaf(X[r * ka + j], U.a(j * ka + c), a);
+        Y[e] = a;
     }
     __syncthreads();
     for (int64_t e = threadIdx.x; e < D; e += blockDim.x) {  // X = (U_g^T Y) / (Lam + lambda)
         const int64_t r = e / ka, c = e - (e / ka) * ka;
-        double a = 0.0;
-        for (int64_t j = 0; j < kg; ++j) a += Ug[j * kg + r] * (double)Y[j * ka + c];
-        X[e] = (float)(a / (lam_of(e) + lambda));
+        float a = 0.f;
+        for (int64_t j = 0; j < kg; ++j) a = fmaf(U.g(j * kg + r), Y[j * ka + c], a);
+        X[e] = (float)((double)a / (lam_of(e) + lambda));
     }
     __syncthreads();
     for (int64_t e = threadIdx.x; e < D; e += blockDim.x) {  // Y = X U_a^T
         const int64_t r = e / ka, c = e - (e / ka) * ka;
-        double a = 0.0;
-        for (int64_t j = 0; j < ka; ++j) a += (double)X[r * ka + j] * Ua[c * ka + j];
-        Y[e] = (float)a;
+        float a = 0.f;
+        for (int64_t j = 0; j < ka; ++j) a = fmaf(X[r * ka + j], U.a(c * ka + j), a);
+        Y[e] = a;
     }
     __syncthreads();
-    float* out = qhat + (int64_t)blockIdx.x * ld_qhat;
+    float* out = qhat + (int64_t)blockIdx.x * ld_qhat + (int64_t)layer * D;
     for (int64_t e = threadIdx.x; e < D; e += blockDim.x) {  // Qhat = U_g Y
         const int64_t r = e / ka, c = e - (e / ka) * ka;
-        double a = 0.0;
-        for (int64_t j = 0; j < kg; ++j) a += Ug[r * kg + j] * (double)Y[j * ka + c];
-        out[e] = (float)a;
+        float a = 0.f;
+        for (int64_t j = 0; j < kg; ++j) a = fmaf(U.g(r * kg + j), Y[j * ka + c], a);
+        out[e] = a;
     }
 }
 
@@ -341,41 +387,62 @@ cudaError_t launch_kfac_sum_partials(const float* part, int nblk, int64_t stride
     return cudaGetLastError();
 }
 
-cudaError_t launch_kfac_eigen(double* state, int64_t ka, int64_t kg, cudaStream_t s) {
+cudaError_t launch_kfac_eigen(int n_layers, double* state, int64_t ka, int64_t kg, cudaStream_t s) {
     const int64_t nmax = ka > kg ? ka : kg;
     const int64_t mh = (nmax + 2) / 2;
-    const size_t smem = (size_t)nmax * nmax * 8 + (size_t)mh * (8 + 8 + 4 + 4);
+    const size_t smem = (size_t)(nmax <= 64 ? 2 : 1) * nmax * nmax * 8 + (size_t)mh * (8 + 8 + 4 + 4);
     cudaError_t e = cudaFuncSetAttribute(jacobi_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
     if (e != cudaSuccess) return e;
     note_launches(1);
-    jacobi_kernel<<<2, kKfThreads, smem, s>>>(state, ka, kg);
+    jacobi_kernel<<<dim3(2, (unsigned)n_layers), kKfThreads, smem, s>>>(state, (int64_t)kfac_state_bytes(ka, kg) / 8,
+                                                                         ka, kg);
     return cudaGetLastError();
 }
 
-cudaError_t launch_kfac_ekfac_accum(double* state, int64_t ka, int64_t kg, const float* phi, int64_t n, int64_t ld,
-                                    float* part, int nblk, cudaStream_t s) {
+// EK-FAC sums of n_layers layers whose features sit side by side in phi
+// (layer l at column l*ka*kg); part holds n_layers * nblk * ka*kg floats.
+cudaError_t launch_kfac_ekfac_accum(int n_layers, double* state, int64_t ka, int64_t kg, const float* phi, int64_t n,
+                                    int64_t ld, float* part, int nblk, cudaStream_t s) {
     if (n == 0) return cudaSuccess;
-    const size_t smem = (size_t)2 * ka * kg * 4;
-    cudaError_t e = cudaFuncSetAttribute(ekfac_partial_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+    const bool su = ka <= 64 && kg <= 64;
+    const size_t smem = (size_t)(2 * ka * kg + (su ? ka * ka + kg * kg : 0)) * 4;
+    const int64_t stride = (int64_t)kfac_state_bytes(ka, kg) / 8;
+    cudaError_t e = su ? cudaFuncSetAttribute(ekfac_partial_kernel<true>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                              (int)smem)
+                       : cudaFuncSetAttribute(ekfac_partial_kernel<false>,
+                                              cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
     if (e != cudaSuccess) return e;
-    const KfLayout l(ka, kg);
     note_launches(2);
-    ekfac_partial_kernel<<<nblk, kKfThreads, smem, s>>>(phi, n, ld, state, ka, kg, part);
-    sum_partials_kernel<<<(unsigned)((ka * kg + 255) / 256), 256, 0, s>>>(part, nblk, ka * kg, ka * kg, state + l.Le,
-                                                                        1.0, state, 1, (double)n);
+    const dim3 grid((unsigned)nblk, (unsigned)n_layers);
+    if (su)
+        ekfac_partial_kernel<true><<<grid, kKfThreads, smem, s>>>(phi, n, ld, state, stride, ka, kg, part);
+    else
+        ekfac_partial_kernel<false><<<grid, kKfThreads, smem, s>>>(phi, n, ld, state, stride, ka, kg, part);
+    ekfac_reduce_kernel<<<dim3((unsigned)((ka * kg + 255) / 256), (unsigned)n_layers), 256, 0, s>>>(
+        part, nblk, state, stride, ka, kg, (double)n);
     return cudaGetLastError();
 }
 
-cudaError_t launch_kfac_apply(int kind, const double* state, int64_t ka, int64_t kg, double lambda_abs,
+cudaError_t launch_kfac_apply(int kind, int n_layers, const double* state, int64_t ka, int64_t kg, double lambda_abs,
                               double lambda_rel, const float* q, int64_t n_q, int64_t ld_q, float* qhat,
                               int64_t ld_qhat, cudaStream_t s) {
     if (n_q == 0) return cudaSuccess;
-    const size_t smem = (size_t)2 * ka * kg * 4;
-    cudaError_t e = cudaFuncSetAttribute(kfac_apply_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+    const bool su = ka <= 64 && kg <= 64;
+    const size_t smem = (size_t)(2 * ka * kg + (su ? ka * ka + kg * kg : 0)) * 4;
+    const int64_t stride = (int64_t)kfac_state_bytes(ka, kg) / 8;
+    cudaError_t e = su ? cudaFuncSetAttribute(kfac_apply_kernel<true>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                              (int)smem)
+                       : cudaFuncSetAttribute(kfac_apply_kernel<false>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                              (int)smem);
     if (e != cudaSuccess) return e;
     note_launches(1);
-    kfac_apply_kernel<<<(unsigned)n_q, kKfThreads, smem, s>>>(kind, state, ka, kg, lambda_abs, lambda_rel, q, ld_q,
-                                                              qhat, ld_qhat);
+    const dim3 grid((unsigned)n_q, (unsigned)n_layers);
+    if (su)
+        kfac_apply_kernel<true><<<grid, kKfThreads, smem, s>>>(kind, state, stride, ka, kg, lambda_abs, lambda_rel, q,
+                                                               ld_q, qhat, ld_qhat);
+    else
+        kfac_apply_kernel<false><<<grid, kKfThreads, smem, s>>>(kind, state, stride, ka, kg, lambda_abs, lambda_rel,
+                                                                q, ld_q, qhat, ld_qhat);
     return cudaGetLastError();
 }
 

@@ -84,10 +84,10 @@ cudaError_t launch_kfac_cov(const float* Y, int64_t rows, int k, double* S, doub
                             double add_m, float* part, cudaStream_t s);
 cudaError_t launch_kfac_sum_partials(const float* part, int nblk, int64_t stride, int64_t n, double* S, double scale,
                                      double* header, int slot, double add, cudaStream_t s);
-cudaError_t launch_kfac_eigen(double* state, int64_t ka, int64_t kg, cudaStream_t s);
-cudaError_t launch_kfac_ekfac_accum(double* state, int64_t ka, int64_t kg, const float* phi, int64_t n, int64_t ld,
-                                    float* part, int nblk, cudaStream_t s);
-cudaError_t launch_kfac_apply(int kind, const double* state, int64_t ka, int64_t kg, double lambda_abs,
+cudaError_t launch_kfac_eigen(int n_layers, double* state, int64_t ka, int64_t kg, cudaStream_t s);
+cudaError_t launch_kfac_ekfac_accum(int n_layers, double* state, int64_t ka, int64_t kg, const float* phi, int64_t n,
+                                    int64_t ld, float* part, int nblk, cudaStream_t s);
+cudaError_t launch_kfac_apply(int kind, int n_layers, const double* state, int64_t ka, int64_t kg, double lambda_abs,
                               double lambda_rel, const float* q, int64_t n_q, int64_t ld_q, float* qhat,
                               int64_t ld_qhat, cudaStream_t s);
 cudaError_t launch_project_tc(const tda_layer_desc& L, const void* A, const void* B, int64_t N,

@@ -585,3 +585,39 @@ def test_project_kfac_fused_matches_oracle(dev, orc, N, T, di, do, k):
     assert s[0] == N * T
     assert rel_fro(s[8:8 + k * k].reshape(k, k) / s[0], Ca) <= 1e-5
     assert rel_fro(s[8 + k * k:8 + 2 * k * k].reshape(k, k) / s[0], Cg) <= 1e-5
+
+
+@pytest.mark.gpu
+@pytest.mark.parametrize("kind", [tda.TDA_KFAC, tda.TDA_EKFAC])
+def test_kfac_batched_layers_match_oracle(dev, orc, kind):
+    # three linears of one block in one state buffer: fused projection per linear, then
+    # eigenbases, EK-FAC sums and the preconditioner for all linears in one launch each
+    N, T, k, nq = 160, 64, 32, 6
+    shapes = [(128, 128), (128, 256), (256, 128)]
+    D = k * k
+    per = tda.tda_kfac_state_bytes(k, k)
+    st = torch.empty(len(shapes) * per // 8, dtype=torch.float64, device=dev)
+    Ls = [tda.LayerDesc(di, do, T, k, k, seed=3, layer=i) for i, (di, do) in enumerate(shapes)]
+    wsb = max(tda.tda_kfac_workspace_size(L, tda.TDA_BF16) for L in Ls)
+    ws = torch.empty(wsb, dtype=torch.uint8, device=dev)
+    Phi = torch.empty((N, len(shapes) * D), device=dev)
+    tda.tda_kfac_reset(k, k, st, n_layers=len(shapes))
+    facts = []
+    for i, (L, (di, do)) in enumerate(zip(Ls, shapes)):
+        A, B = make_factors(N, T, di, do, "bf16", stream=50 + i, sigma_b=0.05)
+        facts.append((synth.to_f64(A, "bf16"), synth.to_f64(B, "bf16")))
+        tda.tda_project_kfac(L, tda.TDA_BF16, to_dev(A, "bf16", dev), to_dev(B, "bf16", dev), N, Phi[:, i * D:],
+                             len(shapes) * D, st[i * per // 8:], ws, wsb)
+    tda.tda_kfac_eigen(k, k, st, n_layers=len(shapes))
+    if kind == tda.TDA_EKFAC:
+        tda.tda_kfac_accumulate_eigenvalues(k, k, st, Phi, N, len(shapes) * D, ws, wsb, n_layers=len(shapes))
+    Q = np.random.default_rng(1).standard_normal((nq, len(shapes) * D)).astype(np.float32)
+    Qh = torch.empty((nq, len(shapes) * D), device=dev)
+    tda.tda_kfac_apply(kind, k, k, st, 0.0, 0.1, torch.from_numpy(Q).to(dev), nq, len(shapes) * D, Qh,
+                       len(shapes) * D, n_layers=len(shapes))
+    tda.tda_device_status()
+    got = Qh.cpu().numpy()
+    for i, (A64, B64) in enumerate(facts):
+        phi64 = orc.project(A64, B64, k, k, 3, i)
+        ref = _kfac_oracle(orc, A64, B64, k, 3, i, kind, 0.0, 0.1, Q[:, i * D:(i + 1) * D], phi64)[-1]
+        assert rel_fro(got[:, i * D:(i + 1) * D], ref) <= 1e-4, i
