@@ -72,6 +72,9 @@ def _load():
             "oracle_ekfac_eigenvalues": (None, [I64, I64, I64, D, D, D, D]),
             "oracle_kfac_damping": (ctypes.c_double, [I64, I64, D, ctypes.c_double, ctypes.c_double]),
             "oracle_kfac_precondition": (None, [I64, I64, D, D, D, ctypes.c_double, I64, D, D]),
+            "oracle_token_scores": (None, [I64, I64, I64, I64, I64, I64, U64, U32, I32, D, D, I64, D, D]),
+            "oracle_mask_gather": (None, [I64, I64, I64, I64, D, D, I64, ctypes.POINTER(I32), ctypes.POINTER(I32),
+                                          D]),
             "oracle_score": (None, [I64, I64, I64, D, D, D]),
             "oracle_topk": (None, [I64, I64, D, I32, ctypes.POINTER(I32), D]),
             "oracle_route_costs": (I32, [I32, I64, I64, I64, I64, I64, I64, I64, D]),
@@ -265,6 +268,33 @@ def kfac_precondition(Ua, Ug, Lam, lam: float, Q) -> np.ndarray:
     Q = Q.reshape(-1, k_out * k_in)
     out = np.empty_like(Q)
     _load().oracle_kfac_precondition(k_in, k_out, _p(Ua), _p(Ug), _p(Lam), lam, Q.shape[0], _p(Q), _p(out))
+    return out
+
+
+# ---------------------------------------------------------------- token scores / masks
+def token_scores(A, B, R, k_in: int, k_out: int, seed: int, layer: int, kind: int = 0) -> np.ndarray:
+    """A (N,T,d_in), B (N,T,d_out), R (n_q, k_out, k_in) -> s (n_q, N, T)."""
+    A, B, R = _f64(A), _f64(B), _f64(R)
+    N, T, d_in = A.shape
+    d_out = B.shape[2]
+    n_q = R.shape[0]
+    out = np.empty((n_q, N, T))
+    _load().oracle_token_scores(N, T, d_in, d_out, k_in, k_out, seed, layer, kind, _p(A), _p(B), n_q, _p(R),
+                                _p(out))
+    return out
+
+
+def mask_gather(A, B, rows, cols) -> np.ndarray:
+    """DW entries at (rows[m], cols[m]) for each example: (N, n_coords)."""
+    A, B = _f64(A), _f64(B)
+    N, T, d_in = A.shape
+    d_out = B.shape[2]
+    rows = np.ascontiguousarray(rows, dtype=np.int32)
+    cols = np.ascontiguousarray(cols, dtype=np.int32)
+    out = np.empty((N, rows.size))
+    ip = ctypes.POINTER(ctypes.c_int32)
+    _load().oracle_mask_gather(N, T, d_in, d_out, _p(A), _p(B), rows.size, rows.ctypes.data_as(ip),
+                               cols.ctypes.data_as(ip), _p(out))
     return out
 
 

@@ -557,6 +557,70 @@ void oracle_kfac_precondition(int64_t k_in, int64_t k_out, const double* Ua, con
 }
 
 /* ------------------------------------------------------------------------ */
+/* Token-level scores and random-mask reduction                             */
+/* ------------------------------------------------------------------------ */
+
+void oracle_token_scores(int64_t N, int64_t T, int64_t d_in, int64_t d_out, int64_t k_in,
+                         int64_t k_out, uint64_t seed, uint32_t layer, int32_t kind,
+                         const double* A, const double* B, int64_t n_q, const double* R,
+                         double* out) {
+    double* P_in = (double*)malloc(sizeof(double) * (size_t)(d_in * k_in));
+    double* P_out = (double*)malloc(sizeof(double) * (size_t)(d_out * k_out));
+    oracle_proj_matrix(seed, layer, 0, kind, d_in, k_in, P_in);
+    oracle_proj_matrix(seed, layer, 1, kind, d_out, k_out, P_out);
+#ifdef _OPENMP
+#pragma omp parallel for schedule(dynamic, 1) num_threads(g_threads)
+#endif
+    for (int64_t n = 0; n < N; ++n) {
+        double* at = (double*)malloc(sizeof(double) * (size_t)k_in);
+        double* gt = (double*)malloc(sizeof(double) * (size_t)k_out);
+        for (int64_t t = 0; t < T; ++t) {
+            const double* a = A + (n * T + t) * d_in;
+            const double* g = B + (n * T + t) * d_out;
+            for (int64_t c = 0; c < k_in; ++c) { /* a~_t = P_a a_t */
+                double s = 0.0;
+                for (int64_t x = 0; x < d_in; ++x) s += a[x] * P_in[x * k_in + c];
+                at[c] = s;
+            }
+            for (int64_t r = 0; r < k_out; ++r) { /* g~_t = P_g g_t */
+                double s = 0.0;
+                for (int64_t x = 0; x < d_out; ++x) s += g[x] * P_out[x * k_out + r];
+                gt[r] = s;
+            }
+            for (int64_t j = 0; j < n_q; ++j) { /* g~_t^T R_j a~_t */
+                const double* Rj = R + j * k_out * k_in;
+                double s = 0.0;
+                for (int64_t r = 0; r < k_out; ++r) {
+                    double u = 0.0;
+                    for (int64_t c = 0; c < k_in; ++c) u += Rj[r * k_in + c] * at[c];
+                    s += gt[r] * u;
+                }
+                out[(j * N + n) * T + t] = s;
+            }
+        }
+        free(at);
+        free(gt);
+    }
+    free(P_in);
+    free(P_out);
+}
+
+void oracle_mask_gather(int64_t N, int64_t T, int64_t d_in, int64_t d_out, const double* A,
+                        const double* B, int64_t n_coords, const int32_t* rows,
+                        const int32_t* cols, double* out) {
+#ifdef _OPENMP
+#pragma omp parallel for schedule(dynamic, 1) num_threads(g_threads)
+#endif
+    for (int64_t n = 0; n < N; ++n)
+        for (int64_t m = 0; m < n_coords; ++m) {
+            double s = 0.0;
+            for (int64_t t = 0; t < T; ++t)
+                s += B[(n * T + t) * d_out + rows[m]] * A[(n * T + t) * d_in + cols[m]];
+            out[n * n_coords + m] = s;
+        }
+}
+
+/* ------------------------------------------------------------------------ */
 /* Scores and top-k                                                         */
 /* ------------------------------------------------------------------------ */
 

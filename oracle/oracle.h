@@ -153,6 +153,24 @@ void oracle_kfac_precondition(int64_t k_in, int64_t k_out, const double* Ua, con
                               const double* Lam, double lambda, int64_t n_q, const double* Q,
                               double* Qhat);
 
+/* ---- token-level scores and random-mask reduction ---- */
+
+/* Token-level decomposition (appendix on token-level attribution): for train
+ * example i and query matrix R_j (k_out x k_in, row-major; e.g. a projected,
+ * possibly preconditioned query feature),
+ *   s[j][i][t] = g~_t^T R_j a~_t  with a~_t = P_a a_t, g~_t = P_g g_t,
+ * so that sum_t s[j][i][t] = <Phi_i, R_j>. out is n_q x N x T. */
+void oracle_token_scores(int64_t N, int64_t T, int64_t d_in, int64_t d_out, int64_t k_in,
+                         int64_t k_out, uint64_t seed, uint32_t layer, int32_t kind,
+                         const double* A, const double* B, int64_t n_q, const double* R,
+                         double* out);
+/* Random-mask reduction gathered from the factors: for each example and each
+ * mask coordinate (rows[m], cols[m]) of DW, the entry
+ *   out[n][m] = sum_t g_t[rows[m]] a_t[cols[m]]    (Eq. 1 at that entry). */
+void oracle_mask_gather(int64_t N, int64_t T, int64_t d_in, int64_t d_out, const double* A,
+                        const double* B, int64_t n_coords, const int32_t* rows,
+                        const int32_t* cols, double* out);
+
 /* ---- scores and ranking ---- */
 
 /* S[q][i] = sum_f Qhat[q][f] Phi[i][f]. */
