@@ -359,6 +359,44 @@ tda_status tda_kfac_apply(int32_t kind, int32_t n_layers, int32_t k_in, int32_t 
                           float* qhat, int64_t ld_qhat, void* stream);
 
 /* ---------------------------------------------------------------------------
+ * tda_token_scores -- token-level decomposition of the score (token-level
+ * attribution appendix): for query matrix R_j and train example i,
+ *   out[j*ld_q_out + i*T + t] = beta*out + g~_t^T R_j a~_t,
+ * with a~_t = P_a a_t, g~_t = P_g g_t the projected factors of token t of
+ * example i (identity kind: the raw factors, R_j then a full d_out x d_in
+ * matrix); sum_t of the result is <Phi_i, R_j>. Summing layers: call per
+ * layer with beta 1.
+ *   A, B   [N][T][d] (dtype as tda_project), device.
+ *   R      n_q rows of k_out*k_in fp32 (row-major [k_out][k_in], e.g. a
+ *          layer's columns of the preconditioned queries), row stride ld_R.
+ *   out    device fp32, ld_q_out >= N*T.
+ *   ws     >= tda_token_scores_workspace_size(L) bytes (one example's
+ *          projected factors; more lets a pass cover more examples).
+ * k_in, k_out <= 128.
+ * ------------------------------------------------------------------------- */
+size_t tda_token_scores_workspace_size(const tda_layer_desc* L);
+tda_status tda_token_scores(const tda_layer_desc* L, tda_dtype dtype, const void* A, const void* B, int64_t N,
+                            const float* R, int64_t n_q, int64_t ld_R, float* out, int64_t ld_q_out, float beta,
+                            void* ws, size_t ws_bytes, void* stream);
+
+/* ---------------------------------------------------------------------------
+ * tda_mask_gather -- random-mask reduction gathered from the factors (the
+ * reduced representation of App. B.4: a set of DW coordinates per layer,
+ * e.g. ten disjoint masks of 512 or 8192 entries):
+ *   out[n*ld_out + m] = sum_t g_t[rows[m]] a_t[cols[m]]  (Eq. 1 at that entry)
+ * for each of N examples and n_coords coordinates, without forming DW.
+ *   rows, cols  device int32 [n_coords] (the caller draws the masks); a
+ *               coordinate outside [0, d_out) x [0, d_in) yields NaN.
+ *   out         device fp32, ld_out >= n_coords.
+ * Scores of disjoint masks averaged = one tda_score over the concatenated
+ * coordinates divided by the mask count. Needs d_in, d_out <= 65536 and
+ * (d_in + d_out) * sizeof(dtype) <= 96 KiB.
+ * ------------------------------------------------------------------------- */
+tda_status tda_mask_gather(const tda_layer_desc* L, tda_dtype dtype, const void* A, const void* B, int64_t N,
+                           const int32_t* rows, const int32_t* cols, int64_t n_coords, float* out, int64_t ld_out,
+                           void* stream);
+
+/* ---------------------------------------------------------------------------
  * tda_score -- S[q][i] = beta*S[q][i] + sum_f Qhat[q][f] Phi[i][f]
  * (gradient inner products; GradDot when Qhat = Q, Sec. 3.2 / Eq. 4).
  *   Qhat  device, n_q rows of D, q_dtype TDA_F32 or TDA_F64, row stride ld_q.

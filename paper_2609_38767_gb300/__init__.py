@@ -19,7 +19,8 @@ __all__ = [
     "tda_project_materialized_noalloc",
     "tda_similarity_projected", "tda_similarity_exact", "tda_norms", "tda_cosine", "tda_kfac_state_bytes", "tda_kfac_workspace_size",
     "tda_kfac_reset", "tda_kfac_accumulate_factors", "tda_project_kfac", "tda_kfac_eigen",
-    "tda_kfac_accumulate_eigenvalues", "tda_kfac_apply", "tda_precondition_state_bytes", "tda_precondition",
+    "tda_kfac_accumulate_eigenvalues", "tda_kfac_apply",
+    "tda_token_scores_workspace_size", "tda_token_scores", "tda_mask_gather", "tda_precondition_state_bytes", "tda_precondition",
     "tda_precondition_info", "tda_score", "tda_score_engine", "tda_similarity_gram_engine", "tda_topk", "tda_route", "tda_route_calibrate",
     "tda_route_set_model", "tda_device_status", "tda_selftest_bounded_wait", "tda_last_error", "tda_version", "tda_launch_count",
 ]
@@ -91,6 +92,9 @@ def load() -> ctypes.CDLL:
             "tda_similarity_exact": (I32, [LP, I32, P, P, I64, P, P, I64, P, I64, F, I32, P, SZ, P]),
             "tda_precondition_state_bytes": (SZ, [I64, I32]),
             "tda_kfac_state_bytes": (SZ, [I32, I32]),
+            "tda_token_scores_workspace_size": (SZ, [LP]),
+            "tda_token_scores": (I32, [LP, I32, P, P, I64, P, I64, I64, P, I64, F, P, SZ, P]),
+            "tda_mask_gather": (I32, [LP, I32, P, P, I64, P, P, I64, P, I64, P]),
             "tda_kfac_workspace_size": (SZ, [LP, I32]),
             "tda_kfac_reset": (I32, [I32, I32, I32, P, P]),
             "tda_kfac_accumulate_factors": (I32, [LP, I32, P, P, I64, P, P, SZ, P]),
@@ -212,6 +216,20 @@ def tda_similarity_exact(L, dtype, Aq, Bq, n_q, At, Bt, n_t, S, ld_S, beta=0.0, 
                          ws=None, ws_bytes=0, stream=None):
     _check(load().tda_similarity_exact(ctypes.byref(L), dtype, _ptr(Aq), _ptr(Bq), n_q, _ptr(At), _ptr(Bt),
                                        n_t, _ptr(S), ld_S, beta, route, _ptr(ws), ws_bytes, _stream(stream)))
+
+
+def tda_token_scores_workspace_size(L) -> int:
+    return int(load().tda_token_scores_workspace_size(ctypes.byref(L)))
+
+
+def tda_token_scores(L, dtype, A, B, N, R, n_q, ld_R, out, ld_q_out, beta=0.0, ws=None, ws_bytes=0, stream=None):
+    _check(load().tda_token_scores(ctypes.byref(L), dtype, _ptr(A), _ptr(B), N, _ptr(R), n_q, ld_R, _ptr(out),
+                                   ld_q_out, beta, _ptr(ws), ws_bytes, _stream(stream)))
+
+
+def tda_mask_gather(L, dtype, A, B, N, rows, cols, n_coords, out, ld_out, stream=None):
+    _check(load().tda_mask_gather(ctypes.byref(L), dtype, _ptr(A), _ptr(B), N, _ptr(rows), _ptr(cols), n_coords,
+                                  _ptr(out), ld_out, _stream(stream)))
 
 
 def tda_kfac_state_bytes(k_in, k_out) -> int:

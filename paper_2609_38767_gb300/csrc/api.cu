@@ -530,6 +530,80 @@ tda_status tda_cosine(float* S, int64_t n_q, int64_t n_t, int64_t ld_S, const fl
     return cuda_check(launch_cosine(S, n_q, n_t, ld_S, nq, nt, (cudaStream_t)stream), "cosine");
 }
 
+// ---------------------------------------------------------------- token scores / masks
+size_t tda_token_scores_workspace_size(const tda_layer_desc* L) {
+    if (!L || L->k_in < 1 || L->k_out < 1 || L->T < 0) return 0;
+    return (project_factors_bytes_per_example(*L) + 255) & ~(size_t)255;
+}
+
+tda_status tda_token_scores(const tda_layer_desc* L, tda_dtype dtype, const void* A, const void* B, int64_t N,
+                            const float* R, int64_t n_q, int64_t ld_R, float* out, int64_t ld_q_out, float beta,
+                            void* ws, size_t ws_bytes, void* stream) {
+    g_msg[0] = 0;
+    tda_status st = validate_layer(L, true);
+    if (st) return st;
+    if ((st = validate_factors(L, dtype, A, B, N, "tda_token_scores"))) return st;
+    if (L->k_in > 128 || L->k_out > 128) return fail(TDA_ERR_UNSUPPORTED, "token scores need k_in, k_out <= 128");
+    const int64_t D = (int64_t)L->k_in * L->k_out;
+    if (n_q < 0) return fail(TDA_ERR_INVALID_ARG, "negative n_q");
+    if (N > 0 && n_q > 0 && L->T > 0) {
+        if (!R || ld_R < D) return fail(TDA_ERR_INVALID_ARG, "R is NULL or ld_R < k_in*k_out");
+        if (!out || ld_q_out < N * L->T) return fail(TDA_ERR_INVALID_ARG, "out is NULL or ld_q_out < N*T");
+    }
+    const size_t per = project_factors_bytes_per_example(*L);
+    if (N == 0 || n_q == 0 || L->T == 0) return TDA_OK;
+    if (!ws || ws_bytes < per)
+        return fail(TDA_ERR_WORKSPACE, "tda_token_scores needs >= %zu bytes of ws, got %zu", per, ws_bytes);
+    cudaStream_t s = (cudaStream_t)stream;
+    int64_t chunk = (int64_t)(ws_bytes / per);
+    if (chunk > N) chunk = N;
+    if (chunk > 65535) chunk = 65535;
+    const float scale = projection_scale(*L);
+    float* Y = (float*)ws;
+    for (int64_t e0 = 0; e0 < N; e0 += chunk) {
+        const int64_t c = N - e0 < chunk ? N - e0 : chunk;
+        if ((st = cuda_check(launch_project_factors(*L, dtype, A, B, e0, c, Y, s), "project factors"))) return st;
+        if ((st = cuda_check(launch_token_scores(Y, Y + c * L->T * L->k_in, c, L->T, L->k_in, L->k_out, R, n_q, ld_R,
+                                                 scale, out, ld_q_out, e0, beta, s),
+                             "token scores")))
+            return st;
+    }
+    return TDA_OK;
+}
+
+tda_status tda_mask_gather(const tda_layer_desc* L, tda_dtype dtype, const void* A, const void* B, int64_t N,
+                           const int32_t* rows, const int32_t* cols, int64_t n_coords, float* out, int64_t ld_out,
+                           void* stream) {
+    g_msg[0] = 0;
+    tda_status st = validate_layer(L, false);
+    if (st) return st;
+    if ((st = validate_factors(L, dtype, A, B, N, "tda_mask_gather"))) return st;
+    if (n_coords < 0) return fail(TDA_ERR_INVALID_ARG, "negative n_coords");
+    if (N > 0 && n_coords > 0 && (!rows || !cols || !out || ld_out < n_coords))
+        return fail(TDA_ERR_INVALID_ARG, "rows/cols/out NULL or ld_out < n_coords");
+    if (L->d_in > 65536 || L->d_out > 65536) return fail(TDA_ERR_UNSUPPORTED, "mask gather needs d <= 65536");
+    const size_t el = dtype == TDA_F32 ? 4 : 2;
+    if (mask_gather_tokens_per_pass(L->d_in, L->d_out, el) < 1)
+        return fail(TDA_ERR_UNSUPPORTED, "mask gather needs (d_in + d_out) * sizeof(dtype) <= 96 KiB");
+    if (N == 0 || n_coords == 0) return TDA_OK;
+    cudaStream_t s = (cudaStream_t)stream;
+    if (L->T == 0) {
+        for (int64_t n = 0; n < N; ++n)
+            if ((st = cuda_check(cudaMemsetAsync(out + n * ld_out, 0, sizeof(float) * (size_t)n_coords, s), "zero")))
+                return st;
+        return TDA_OK;
+    }
+    const size_t a_ex = (size_t)L->T * L->d_in * el, b_ex = (size_t)L->T * L->d_out * el;
+    for (int64_t e0 = 0; e0 < N; e0 += 65535) {
+        const int64_t c = N - e0 < 65535 ? N - e0 : 65535;
+        if ((st = cuda_check(launch_mask_gather(*L, dtype, (const char*)A + e0 * a_ex, (const char*)B + e0 * b_ex, c,
+                                                rows, cols, n_coords, out + e0 * ld_out, ld_out, s),
+                             "mask gather")))
+            return st;
+    }
+    return TDA_OK;
+}
+
 // ---------------------------------------------------------------- K-FAC / EK-FAC
 static bool kfac_dims_ok(int64_t ka, int64_t kg) { return ka >= 1 && kg >= 1 && ka <= 128 && kg <= 128; }
 

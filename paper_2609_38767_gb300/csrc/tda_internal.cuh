@@ -90,6 +90,14 @@ cudaError_t launch_kfac_ekfac_accum(int n_layers, double* state, int64_t ka, int
 cudaError_t launch_kfac_apply(int kind, int n_layers, const double* state, int64_t ka, int64_t kg, double lambda_abs,
                               double lambda_rel, const float* q, int64_t n_q, int64_t ld_q, float* qhat,
                               int64_t ld_qhat, cudaStream_t s);
+// Token-level scores and random-mask gather (k_tokens.cu)
+cudaError_t launch_token_scores(const float* Ya, const float* Yb, int64_t n, int64_t T, int ka, int kg,
+                                const float* R, int64_t n_q, int64_t ld_R, float scale, float* out, int64_t ld_q,
+                                int64_t i0, float beta, cudaStream_t s);
+int mask_gather_tokens_per_pass(int64_t d_in, int64_t d_out, size_t el);
+cudaError_t launch_mask_gather(const tda_layer_desc& L, tda_dtype dt, const void* A, const void* B, int64_t N,
+                               const int32_t* rows, const int32_t* cols, int64_t n_coords, float* out, int64_t ld_out,
+                               cudaStream_t s);
 cudaError_t launch_project_tc(const tda_layer_desc& L, const void* A, const void* B, int64_t N,
                               float* phi, int64_t ld_phi, unsigned int* err, cudaStream_t s);
 

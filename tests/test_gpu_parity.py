@@ -621,3 +621,56 @@ def test_kfac_batched_layers_match_oracle(dev, orc, kind):
         phi64 = orc.project(A64, B64, k, k, 3, i)
         ref = _kfac_oracle(orc, A64, B64, k, 3, i, kind, 0.0, 0.1, Q[:, i * D:(i + 1) * D], phi64)[-1]
         assert rel_fro(got[:, i * D:(i + 1) * D], ref) <= 1e-4, i
+
+
+# ------------------------------------------------------------------ token scores / masks
+@pytest.mark.gpu
+@pytest.mark.parametrize("dtype,N,T,di,do,k,kind", [("f32", 5, 70, 64, 48, 16, 0), ("bf16", 4, 130, 128, 64, 32, 0),
+                                                    ("f32", 3, 9, 24, 16, 24, 1)])
+def test_token_scores_match_oracle(dev, orc, dtype, N, T, di, do, k, kind):
+    # s_t = g~_t^T R a~_t per token; beta = 1 accumulates a second layer's share
+    ko = do if kind == 1 else k
+    ki = di if kind == 1 else k
+    A, B = make_factors(N, T, di, do, dtype, stream=61, sigma_b=0.1, mask_p=0.05)
+    L = tda.LayerDesc(di, do, T, ki, ko, seed=7, layer=4, kind=kind)
+    nq = 3
+    R = np.random.default_rng(T).standard_normal((nq, ko, ki)).astype(np.float32)
+    Rd = torch.from_numpy(R.reshape(nq, -1)).to(dev)
+    out0 = np.random.default_rng(1).standard_normal((nq, N * T + 5)).astype(np.float32)
+    out = torch.from_numpy(out0).to(dev)
+    wsb = tda.tda_token_scores_workspace_size(L) * 2
+    ws = torch.empty(wsb, dtype=torch.uint8, device=dev)
+    tda.tda_token_scores(L, TD[dtype], to_dev(A, dtype, dev), to_dev(B, dtype, dev), N, Rd, nq, ki * ko, out,
+                         N * T + 5, 1.0, ws, wsb)
+    tda.tda_device_status()
+    A64, B64 = synth.to_f64(A, dtype), synth.to_f64(B, dtype)
+    ref = orc.token_scores(A64, B64, R, ki, ko, 7, 4, kind)
+    got = out.cpu().numpy()
+    assert rel_fro(got[:, : N * T].reshape(nq, N, T) - out0[:, : N * T].reshape(nq, N, T), ref) <= 1e-5
+    np.testing.assert_array_equal(got[:, N * T:], out0[:, N * T:])
+    # the decomposition sums to the sequence-level score
+    phi = orc.project(A64, B64, ki, ko, 7, 4, kind)
+    np.testing.assert_allclose(ref.sum(2), orc.score(R, phi), rtol=1e-10)
+
+
+@pytest.mark.gpu
+@pytest.mark.parametrize("dtype,N,T,di,do,nc", [("bf16", 6, 37, 256, 128, 20000), ("f32", 3, 100, 64, 80, 700)])
+def test_mask_gather_matches_oracle(dev, orc, dtype, N, T, di, do, nc):
+    # entries of DW at random coordinates, gathered from the factors; invalid coordinates -> NaN
+    A, B = make_factors(N, T, di, do, dtype, stream=62, sigma_b=0.1)
+    rng = np.random.default_rng(nc)
+    rows = rng.integers(0, do, nc).astype(np.int32)
+    cols = rng.integers(0, di, nc).astype(np.int32)
+    rows[5], cols[7] = do, -1
+    L = tda.LayerDesc(di, do, T, 1, 1)
+    out = torch.full((N, nc + 2), 3.0, device=dev)
+    tda.tda_mask_gather(L, TD[dtype], to_dev(A, dtype, dev), to_dev(B, dtype, dev), N,
+                        torch.from_numpy(rows).to(dev), torch.from_numpy(cols).to(dev), nc, out, nc + 2)
+    tda.tda_device_status()
+    got = out.cpu().numpy()
+    ok = np.ones(nc, bool)
+    ok[[5, 7]] = False
+    ref = orc.mask_gather(synth.to_f64(A, dtype), synth.to_f64(B, dtype), np.where(ok, rows, 0), np.where(ok, cols, 0))
+    assert rel_fro(got[:, :nc][:, ok], ref[:, ok]) <= 1e-5
+    assert np.isnan(got[:, 5]).all() and np.isnan(got[:, 7]).all()
+    assert (got[:, nc:] == 3.0).all()
