@@ -82,6 +82,10 @@ def parse_args():
                    help="subset of the block's linears (profiling of a smaller case)")
     p.add_argument("--project-only", action="store_true",
                    help="time only the train projection (kernel profiling; not the metric's step)")
+    p.add_argument("--token-scores", action="store_true",
+                   help="time token-level scores of the block (every train token against every preconditioned query)")
+    p.add_argument("--masks", type=int, default=0,
+                   help="time the random-mask reduction: ten disjoint masks of this many DW coordinates per linear")
     p.add_argument("--route-sweep", action="store_true",
                    help="route cost-model sweep on one 8192x8192 bf16 linear (chosen vs measured fastest route)")
     p.add_argument("--sweep-T", default="8,32,128,512,2048,8192")
@@ -408,12 +412,126 @@ def route_sweep_main(args):
     print(json.dumps(out))
 
 
+def reuse_main(args):
+    """Two reuses of the block's factors, timed like the main step: token-level scores
+    (every train token against every preconditioned query, summed over the linears) or the
+    random-mask reduction (ten disjoint masks of --masks coordinates per linear, gathered
+    for train and query examples, then one score GEMM over the concatenated masks)."""
+    import numpy as np
+    import torch
+
+    import paper_2609_38767_gb300 as tda
+    from paper_2609_38767_gb300 import build as tbuild
+    from paper_2609_38767_gb300 import synth
+    from paper_2609_38767_gb300.block import BlockPipeline
+
+    tbuild.build()
+    tda.load()
+    dev = torch.device("cuda", 0)
+    torch.cuda.set_device(dev)
+    stream = torch.cuda.current_stream()
+    T, N, Nq, k = args.T, args.n_train, args.n_query, args.k
+    D, nl = k * k, len(LINEARS)
+    DT = D * nl
+    sb = math.sqrt(1e-3)
+    At, Bt, Aq, Bq = [], [], [], []
+    for li, (_, di, do) in enumerate(LINEARS):
+        for store, n, role, seed, d, sg in ((At, N, 0, synth.SEED_A, di, 1.0), (Aq, Nq, 1, synth.SEED_A, di, 1.0),
+                                            (Bt, N, 0, synth.SEED_B, do, sb), (Bq, Nq, 1, synth.SEED_B, do, sb)):
+            x = torch.empty((n, T, d), dtype=torch.bfloat16, device=dev)
+            synth.fill_device(x, seed, li + (synth.QUERY_STREAM_OFFSET if role else 0), n, T, d, sg, mask_p=0.01,
+                              mask_stream=1000 if role else 0)
+            store.append(x)
+    pipe = BlockPipeline([(di, do) for _, di, do in LINEARS], T, k, N, Nq, topk=args.topk, lambda_rel=1e-2,
+                         device=dev)
+    layers = pipe.layers
+
+    def proj(role, li, L, route, phi, ld):
+        X, Y, n = (At[li], Bt[li], N) if role == "train" else (Aq[li], Bq[li], Nq)
+        tda.tda_project(L, tda.TDA_BF16, X, Y, n, phi, ld, route)
+
+    pipe.run(lambda *a: proj("train", *a), lambda *a: proj("query", *a))  # preconditioned queries, untimed
+    torch.cuda.synchronize()
+    if args.token_scores:
+        out = torch.empty((Nq, N * T), dtype=torch.float32, device=dev)
+        wsb = max(tda.tda_token_scores_workspace_size(L) for L in layers) * 256
+        ws = torch.empty(wsb, dtype=torch.uint8, device=dev)
+
+        def step():
+            for li, L in enumerate(layers):
+                tda.tda_token_scores(L, tda.TDA_BF16, At[li], Bt[li], N, pipe.Qh[:, li * D:], Nq, DT, out, N * T,
+                                     0.0 if li == 0 else 1.0, ws, wsb)
+
+        flops = sum(N * 2.0 * T * (L.d_in + L.d_out) * k + 2.0 * Nq * N * T * D for L in layers)
+        mode = {"mode": "token-level scores", "n_query": Nq, "outputs_per_step": Nq * N * T}
+        roof_kernel, roof_bound = "factor projection + token contraction (CUDA cores)", "alu"
+    else:
+        K = args.masks
+        rng = np.random.default_rng(2026)
+        coords = []
+        for L in layers:
+            flat = rng.choice(L.d_in * L.d_out, size=10 * K, replace=False)
+            coords.append((torch.from_numpy((flat // L.d_in).astype(np.int32)).to(dev),
+                           torch.from_numpy((flat % L.d_in).astype(np.int32)).to(dev)))
+        nc = 10 * K
+        Gt = torch.empty((N, nl * nc), dtype=torch.float32, device=dev)
+        Gq = torch.empty((Nq, nl * nc), dtype=torch.float32, device=dev)
+
+        def step():
+            for li, L in enumerate(layers):
+                r, c = coords[li]
+                tda.tda_mask_gather(L, tda.TDA_BF16, At[li], Bt[li], N, r, c, nc, Gt[:, li * nc:], nl * nc)
+                tda.tda_mask_gather(L, tda.TDA_BF16, Aq[li], Bq[li], Nq, r, c, nc, Gq[:, li * nc:], nl * nc)
+            tda.tda_score(Gq, tda.TDA_F32, Nq, nl * nc, Gt, N, nl * nc, nl * nc, pipe.S, N, 0.0)
+            tda.tda_topk(pipe.S, Nq, N, N, args.topk, pipe.idx, pipe.val)
+
+        flops = sum(2.0 * (N + Nq) * T * nc for L in layers) + 2.0 * Nq * N * nl * nc
+        mode = {"mode": "random-mask reduction", "masks_per_linear": 10, "coordinates_per_mask": K}
+        roof_kernel, roof_bound = "mask gather + score", "alu"
+    for _ in range(max(args.warmup, 1)):
+        step()
+    tda.tda_device_status()
+    torch.cuda.synchronize()
+    clocks = ClockSampler(0)
+    clocks.start()
+    time.sleep(0.3)
+    l0 = tda.tda_launch_count()
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    e0.record(stream)
+    for _ in range(args.steps):
+        step()
+    e1.record(stream)
+    torch.cuda.synchronize()
+    launches = tda.tda_launch_count() - l0
+    ck = clocks.stop()
+    tda.tda_device_status()
+    ms = e0.elapsed_time(e1) / args.steps
+    peaks = {}
+    try:
+        with open(os.path.join(ROOT, "MEASURED_PEAKS.json")) as f:
+            peaks = json.load(f)
+    except OSError:
+        pass
+    alu = 152 * 128 * 2 * float(peaks.get("sm_max_mhz", 2070.0)) * 1e6 / 1e12
+    rate = flops / (ms * 1e-3) / 1e12
+    print(json.dumps({
+        "metric": METRIC, "value": N / (ms * 1e-3), "unit": "examples/s", "n_gpus": 1, "steps": args.steps,
+        "warmup": args.warmup, "ms_per_step": ms, "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
+        "dtype": "bf16", "data": "synthetic", "config": {**workload(args), **mode},
+        "roofline": {"bound": roof_bound, "kernel": roof_kernel, "achieved": rate, "peak": alu, "unit": "TFLOP/s",
+                     "frac": rate / alu, "traffic": None,
+                     "peak_source": "fp32 SIMT peak derived from 152 SMs x 128 lanes x 2 x max clock"},
+        "cpu_baseline": None, "e2e": None, "gpu_launches": launches, "clocks": ck}))
+
+
 def main():
     args = parse_args()
     if args.impl == "reference":
         return reference_main(args)
     if args.route_sweep:
         return route_sweep_main(args)
+    if args.token_scores or args.masks:
+        return reuse_main(args)
 
     import numpy as np
     import torch
