@@ -390,7 +390,7 @@ tda_status tda_token_scores(const tda_layer_desc* L, tda_dtype dtype, const void
  *   out         device fp32, ld_out >= n_coords.
  * Scores of disjoint masks averaged = one tda_score over the concatenated
  * coordinates divided by the mask count. Needs d_in, d_out <= 65536 and
- * (d_in + d_out) * sizeof(dtype) <= 96 KiB.
+ * (d_in + d_out) * sizeof(dtype) <= 48 KiB.
  * ------------------------------------------------------------------------- */
 tda_status tda_mask_gather(const tda_layer_desc* L, tda_dtype dtype, const void* A, const void* B, int64_t N,
                            const int32_t* rows, const int32_t* cols, int64_t n_coords, float* out, int64_t ld_out,

@@ -584,7 +584,7 @@ tda_status tda_mask_gather(const tda_layer_desc* L, tda_dtype dtype, const void*
     if (L->d_in > 65536 || L->d_out > 65536) return fail(TDA_ERR_UNSUPPORTED, "mask gather needs d <= 65536");
     const size_t el = dtype == TDA_F32 ? 4 : 2;
     if (mask_gather_tokens_per_pass(L->d_in, L->d_out, el) < 1)
-        return fail(TDA_ERR_UNSUPPORTED, "mask gather needs (d_in + d_out) * sizeof(dtype) <= 96 KiB");
+        return fail(TDA_ERR_UNSUPPORTED, "mask gather needs (d_in + d_out) * sizeof(dtype) <= 48 KiB");
     if (N == 0 || n_coords == 0) return TDA_OK;
     cudaStream_t s = (cudaStream_t)stream;
     if (L->T == 0) {

@@ -86,6 +86,7 @@ struct Params {
     int nk_in, nk_out;
     int cs;           // CTAs per cluster sharing one example's token tiles (1, 2 or 4)
     float* cov;       // K-FAC: per-CTA partial sums of At^T At and Bt^T Bt ([grid][2][K*K])
+    float* fout;      // factor output: At rows [N*T][K], then Bt rows [N*T][K] (unscaled signs)
 };
 
 #include "tc_ptx.cuh"
@@ -140,7 +141,9 @@ __device__ __forceinline__ void write_sign_half(uint8_t* tile, int n, uint64_t w
     }
 }
 
-template <int K, int G, bool KF>
+// KF: also accumulate the K-FAC factor covariances. FO: write the projected
+// factors At, Bt of every token instead of contracting them into Phi.
+template <int K, int G, bool KF, bool FO>
 __global__ void __launch_bounds__(kThreads, 1)
 project_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
                   const Params p) {
@@ -386,7 +389,7 @@ project_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant
             }
             tc_fence_after();
             for (int u = 0; u < ng; ++u) {
-                if (p.pack == 1 && gx[u] != cur) {
+                if (!FO && p.pack == 1 && gx[u] != cur) {
                     if (cur >= 0 && !flush(cur)) {
                         stop = true;
                         break;
@@ -414,6 +417,32 @@ project_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant
                     if (lane == 0) mbar_arrive(smem_u32(&tempty[b]));
                 }
                 epi_sync();
+                if constexpr (FO) {
+                    // token rows of this tile in the [N*T] row space: packed tiles hold pack*T
+                    // consecutive rows, a long tile rows tt*128 .. of example x
+                    int64_t g0;
+                    int nrows;
+                    if (p.pack > 1) {
+                        g0 = gx[u] * p.pack * p.T;
+                        nrows = p.pack * (int)p.T;
+                    } else {
+                        g0 = gx[u] * p.T + (int64_t)gt[u] * kTileM;
+                        nrows = (int)(p.T - (int64_t)gt[u] * kTileM < kTileM ? p.T - (int64_t)gt[u] * kTileM : kTileM);
+                    }
+                    const int64_t lim = p.N * p.T - g0;
+                    if (lim < nrows) nrows = (int)lim;
+                    float* oa = p.fout + g0 * K;
+                    float* ob = p.fout + p.N * p.T * K + g0 * K;
+                    for (int idx = et; idx < nrows * (K / 4); idx += 128) {
+                        const int r = idx / (K / 4), c4 = (idx - r * (K / 4)) * 4;
+                        *reinterpret_cast<float4*>(oa + (int64_t)r * K + c4) =
+                            *reinterpret_cast<const float4*>(stX + r * C::kStageLd + c4);
+                        *reinterpret_cast<float4*>(ob + (int64_t)r * K + c4) =
+                            *reinterpret_cast<const float4*>(stY + r * C::kStageLd + c4);
+                    }
+                    epi_sync();
+                    continue;
+                }
                 if constexpr (KF) {
                     // rows of packed tiles past pack * T belong to the next tile's examples
                     const int rows = p.pack == 1 ? kTileM : p.pack * (int)p.T;
@@ -486,7 +515,7 @@ project_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant
                 epi_sync();
             }
         }
-        if (!stop && p.pack == 1 && cur >= 0) flush(cur);
+        if (!FO && !stop && p.pack == 1 && cur >= 0) flush(cur);
         if constexpr (KF) {
             float* out = p.cov + (size_t)blockIdx.x * 2 * K * K;
 #pragma unroll
@@ -563,9 +592,10 @@ int sm_count() {
     return sms;
 }
 
-template <int K, int G, bool KF>
+template <int K, int G, bool KF, bool FO>
 cudaError_t launch_kg(const tda_layer_desc& L, const void* A, const void* B, int64_t N, float* phi,
-                      int64_t ld_phi, unsigned int* err, cudaStream_t s, int pack, float* cov, int* grid_out) {
+                      int64_t ld_phi, unsigned int* err, cudaStream_t s, int pack, float* cov, int* grid_out,
+                      float* fout) {
     using C = Cfg<K, G>;
     CUtensorMap tmA, tmB;
     if (pack > 1) {
@@ -591,14 +621,15 @@ cudaError_t launch_kg(const tda_layer_desc& L, const void* A, const void* B, int
     p.nk_in = (int)((L.d_in + kChunkK - 1) / kChunkK);
     p.nk_out = (int)((L.d_out + kChunkK - 1) / kChunkK);
     p.cov = cov;
+    p.fout = fout;
     const int sms = sm_count();
-    cudaError_t e = cudaFuncSetAttribute(project_tc_kernel<K, G, KF>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+    cudaError_t e = cudaFuncSetAttribute(project_tc_kernel<K, G, KF, FO>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                          (int)C::kSmem);
     if (e != cudaSuccess) return e;
     // Fewer examples than SMs: a cluster of cs CTAs shares each example's token
     // tiles and reduces the partial features through distributed shared memory.
     int cs = 1;
-    if (pack == 1 && N < sms) cs = (2 * N >= sms) ? 2 : 4;
+    if (pack == 1 && N < sms && !FO) cs = (2 * N >= sms) ? 2 : 4;
     while (cs > 1 && cs > p.n_ttiles) cs >>= 1;
     p.cs = cs;
     cudaLaunchConfig_t cfg = {};
@@ -614,24 +645,24 @@ cudaError_t launch_kg(const tda_layer_desc& L, const void* A, const void* B, int
     cfg.numAttrs = 1;
     int max_clusters = 0;
     cfg.gridDim = dim3((unsigned)(cs * (sms / cs)));
-    if (cudaOccupancyMaxActiveClusters(&max_clusters, project_tc_kernel<K, G, KF>, &cfg) != cudaSuccess ||
+    if (cudaOccupancyMaxActiveClusters(&max_clusters, project_tc_kernel<K, G, KF, FO>, &cfg) != cudaSuccess ||
         max_clusters < 1)
         max_clusters = sms / cs;
-    int64_t clusters = p.n_slots;
+    int64_t clusters = FO ? p.n_slots * p.n_ttiles : p.n_slots;
     if (clusters > max_clusters) clusters = max_clusters;
     cfg.gridDim = dim3((unsigned)(clusters * cs));
     if (grid_out) *grid_out = (int)(clusters * cs);
     note_launches(1);
-    e = cudaLaunchKernelEx(&cfg, project_tc_kernel<K, G, KF>, tmA, tmB, p);
+    e = cudaLaunchKernelEx(&cfg, project_tc_kernel<K, G, KF, FO>, tmA, tmB, p);
     if (e != cudaSuccess) return e;
     return cudaGetLastError();
 }
 
 // Two tiles per stage once every CTA has at least two groups of work; fewer
 // units run one tile per stage so that they spread over all SMs.
-template <int K, bool KF>
+template <int K, bool KF, bool FO>
 cudaError_t launch_k(const tda_layer_desc& L, const void* A, const void* B, int64_t N, float* phi,
-                     int64_t ld_phi, unsigned int* err, cudaStream_t s, float* cov, int* grid_out) {
+                     int64_t ld_phi, unsigned int* err, cudaStream_t s, float* cov, int* grid_out, float* fout) {
     int pack = L.T <= 64 ? (int)(kTileM / L.T) : 1;
     if (pack > 1) {
         // packed rows are addressed with 32-bit TMA coordinates and the [1][N*T][d]
@@ -643,12 +674,12 @@ cudaError_t launch_k(const tda_layer_desc& L, const void* A, const void* B, int6
         max_n = max_n / pack * pack;
         if (max_n < pack) pack = 1;  // one example per tile instead
         else if (N > max_n) {
-            if (KF) return cudaErrorInvalidValue;  // one partial slab per CTA: one launch only
+            if (KF || FO) return cudaErrorInvalidValue;  // one partial slab / one factor block per launch
             const size_t a_ex = (size_t)L.T * L.d_in * 2, b_ex = (size_t)L.T * L.d_out * 2;
             for (int64_t e0 = 0; e0 < N; e0 += max_n) {
                 const int64_t n = N - e0 < max_n ? N - e0 : max_n;
-                cudaError_t e = launch_k<K, KF>(L, (const char*)A + e0 * a_ex, (const char*)B + e0 * b_ex, n,
-                                                phi + e0 * ld_phi, ld_phi, err, s, nullptr, nullptr);
+                cudaError_t e = launch_k<K, KF, FO>(L, (const char*)A + e0 * a_ex, (const char*)B + e0 * b_ex, n,
+                                                    phi + e0 * ld_phi, ld_phi, err, s, nullptr, nullptr, nullptr);
                 if (e != cudaSuccess) return e;
             }
             return cudaSuccess;
@@ -656,8 +687,8 @@ cudaError_t launch_k(const tda_layer_desc& L, const void* A, const void* B, int6
     }
     const int64_t units = pack > 1 ? (N + pack - 1) / pack : N * ((L.T + kTileM - 1) / kTileM);
     if (units >= 4 * (int64_t)sm_count())
-        return launch_kg<K, 2, KF>(L, A, B, N, phi, ld_phi, err, s, pack, cov, grid_out);
-    return launch_kg<K, 1, KF>(L, A, B, N, phi, ld_phi, err, s, pack, cov, grid_out);
+        return launch_kg<K, 2, KF, FO>(L, A, B, N, phi, ld_phi, err, s, pack, cov, grid_out, fout);
+    return launch_kg<K, 1, KF, FO>(L, A, B, N, phi, ld_phi, err, s, pack, cov, grid_out, fout);
 }
 
 }  // namespace
@@ -678,9 +709,9 @@ cudaError_t launch_project_tc(const tda_layer_desc& L, const void* A, const void
                               int64_t ld_phi, unsigned int* err, cudaStream_t s) {
     if (N == 0) return cudaSuccess;
     switch (L.k_in) {
-        case 16: return launch_k<16, false>(L, A, B, N, phi, ld_phi, err, s, nullptr, nullptr);
-        case 32: return launch_k<32, false>(L, A, B, N, phi, ld_phi, err, s, nullptr, nullptr);
-        case 64: return launch_k<64, false>(L, A, B, N, phi, ld_phi, err, s, nullptr, nullptr);
+        case 16: return launch_k<16, false, false>(L, A, B, N, phi, ld_phi, err, s, nullptr, nullptr, nullptr);
+        case 32: return launch_k<32, false, false>(L, A, B, N, phi, ld_phi, err, s, nullptr, nullptr, nullptr);
+        case 64: return launch_k<64, false, false>(L, A, B, N, phi, ld_phi, err, s, nullptr, nullptr, nullptr);
         default: return cudaErrorNotSupported;
     }
 }
@@ -693,13 +724,26 @@ cudaError_t launch_project_tc_kfac(const tda_layer_desc& L, const void* A, const
     *grid_out = 0;
     if (N == 0) return cudaSuccess;
     switch (L.k_in) {
-        case 16: return launch_k<16, true>(L, A, B, N, phi, ld_phi, err, s, cov, grid_out);
-        case 32: return launch_k<32, true>(L, A, B, N, phi, ld_phi, err, s, cov, grid_out);
-        case 64: return launch_k<64, true>(L, A, B, N, phi, ld_phi, err, s, cov, grid_out);
+        case 16: return launch_k<16, true, false>(L, A, B, N, phi, ld_phi, err, s, cov, grid_out, nullptr);
+        case 32: return launch_k<32, true, false>(L, A, B, N, phi, ld_phi, err, s, cov, grid_out, nullptr);
+        case 64: return launch_k<64, true, false>(L, A, B, N, phi, ld_phi, err, s, cov, grid_out, nullptr);
         default: return cudaErrorNotSupported;
     }
 }
 
 int project_tc_max_grid() { return sm_count(); }
+
+// Projected factors of N examples (At rows then Bt rows, [N*T][k] each, fp32,
+// unscaled signs) by the tensor-core kernel.
+cudaError_t launch_project_factors_tc(const tda_layer_desc& L, const void* A, const void* B, int64_t N, float* Y,
+                                      unsigned int* err, cudaStream_t s) {
+    if (N == 0 || L.T == 0) return cudaSuccess;
+    switch (L.k_in) {
+        case 16: return launch_k<16, false, true>(L, A, B, N, nullptr, 0, err, s, nullptr, nullptr, Y);
+        case 32: return launch_k<32, false, true>(L, A, B, N, nullptr, 0, err, s, nullptr, nullptr, Y);
+        case 64: return launch_k<64, false, true>(L, A, B, N, nullptr, 0, err, s, nullptr, nullptr, Y);
+        default: return cudaErrorNotSupported;
+    }
+}
 
 }  // namespace tda

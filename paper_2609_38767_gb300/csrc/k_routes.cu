@@ -378,6 +378,16 @@ size_t project_factors_bytes_per_example(const tda_layer_desc& L) {
 cudaError_t launch_project_factors(const tda_layer_desc& L, tda_dtype dt, const void* A, const void* B, int64_t e0,
                                    int64_t n, float* Y, cudaStream_t s) {
     if (n == 0 || L.T == 0) return cudaSuccess;
+    if (dt == TDA_BF16) {
+        // bf16 factors in the tensor-core kernel's shapes: the same projection, at HBM speed
+        const void* Ae = (const char*)A + (size_t)e0 * L.T * L.d_in * 2;
+        const void* Be = (const char*)B + (size_t)e0 * L.T * L.d_out * 2;
+        unsigned int* err = device_error_word();
+        if (err && project_tc_supported(L, Ae, Be) && ((uintptr_t)Y & 15) == 0 && n * L.T < (1LL << 30)) {
+            cudaError_t e = launch_project_factors_tc(L, Ae, Be, n, Y, err, s);
+            if (e != cudaErrorInvalidValue) return e;
+        }
+    }
     const uint64_t key_in = side_key(L.seed, L.layer, 0), key_out = side_key(L.seed, L.layer, 1);
     float* Ya = Y;
     float* Yb = Y + n * L.T * L.k_in;

@@ -75,6 +75,8 @@ bool project_tc_supported(const tda_layer_desc& L, const void* A, const void* B)
 cudaError_t launch_project_tc_kfac(const tda_layer_desc& L, const void* A, const void* B, int64_t N, float* phi,
                                    int64_t ld_phi, float* cov, int* grid_out, unsigned int* err, cudaStream_t s);
 int project_tc_max_grid();
+cudaError_t launch_project_factors_tc(const tda_layer_desc& L, const void* A, const void* B, int64_t N, float* Y,
+                                      unsigned int* err, cudaStream_t s);
 // K-FAC / EK-FAC (k_kfac.cu)
 size_t kfac_state_bytes(int64_t k_in, int64_t k_out);
 int kfac_partial_blocks(int64_t rows);
