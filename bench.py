@@ -561,18 +561,22 @@ def main():
     DT = D * nl
     sb = math.sqrt(1e-3)
 
-    # ---- device-resident synthetic factors (untimed)
+    # ---- device-resident synthetic factors (untimed); rank r owns train examples
+    # [r*N, (r+1)*N) of the job, the queries are replicated
+    from paper_2609_38767_gb300 import shard
+
+    e0 = shard.shard_offset(rank, N)
     At, Bt, Aq, Bq = [], [], [], []
     for li, (_, di, do) in enumerate(LINEARS):
         for store, n, role in ((At, N, 0), (Aq, Nq, 1)):
             x = torch.empty(n * T * di, dtype=torch.bfloat16, device=dev)
             synth.fill_device(x, synth.SEED_A, li + (synth.QUERY_STREAM_OFFSET if role else 0), n, T, di, 1.0,
-                              mask_p=0.01, mask_stream=1000 if role else 0)
+                              e0=0 if role else e0, mask_p=0.01, mask_stream=1000 if role else 0)
             store.append(x)
         for store, n, role in ((Bt, N, 0), (Bq, Nq, 1)):
             x = torch.empty(n * T * do, dtype=torch.bfloat16, device=dev)
             synth.fill_device(x, synth.SEED_B, li + (synth.QUERY_STREAM_OFFSET if role else 0), n, T, do, sb,
-                              mask_p=0.01, mask_stream=1000 if role else 0)
+                              e0=0 if role else e0, mask_p=0.01, mask_stream=1000 if role else 0)
             store.append(x)
     from paper_2609_38767_gb300.block import BlockPipeline
 
@@ -581,6 +585,7 @@ def main():
                          precondition=not args.no_precondition, lambda_rel=0.1 if kfac_mode else 1e-2, device=dev,
                          curvature=args.curvature)
     layers, Phi, Q, idx, val = pipe.layers, pipe.Phi, pipe.Q, pipe.idx, pipe.val
+    select = shard.device_select(tda)
     torch.cuda.synchronize()
 
     ev = []  # (start, end, algorithmic bytes) per projection launch of the train set
@@ -618,6 +623,9 @@ def main():
                 after(li)
             return
         pipe.run(train, lambda li, L, route, phi, ld: project("query", li, L, route, phi, ld), after, mark)
+        if dist:
+            # the exchange step of a sharded job: the global top-k from every rank's top-k
+            shard.merge_topk(idx, val, e0, args.topk, dist, world, select)
 
     def project_dev(role, li, L, route, phi, ld):
         if role == "train" and kfac_mode:
@@ -787,7 +795,9 @@ def main():
         line = {
             "metric": METRIC, "value": value, "unit": "examples/s", "n_gpus": world, "steps": args.steps,
             "warmup": args.warmup, "ms_per_step": ms, "higher_is_better": True, "scaling": "weak",
-            "vs_baseline": None, "dtype": "bf16", "data": "synthetic", "config": workload(args),
+            "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
+            "config": {**workload(args), "parallelism": f"train examples sharded over {world} rank(s)"
+                       + (", global top-k merged by all-gather" if world > 1 else "")},
             "roofline": roofline, "phases": phases, "cpu_baseline": cpu, "e2e": e2e, "gpu_launches": launches,
             "clocks": ck,
         }
