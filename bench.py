@@ -46,8 +46,8 @@ METRIC = "train examples attributed/sec (project+score)"
 # one read of every factor byte, so it grows in proportion). Valid only for the
 # kernel source it was measured on (the kernel file and its PTX helper header);
 # any change makes the bench report null.
-TRAFFIC_RATIO = 1.0012345
-TRAFFIC_KERNEL_SHA256 = "b4c5b2d6bb40ec7aeb2aea603b9290c21580cf54be1bfba82bd146ca7d376969"
+TRAFFIC_RATIO = 1.0013011
+TRAFFIC_KERNEL_SHA256 = "d6671015213ecc7c281fa959fd3a87c213ad63238f248892b15b6ef9189c53fe"
 
 
 def projection_kernel_sha256():
@@ -89,6 +89,9 @@ def parse_args():
     p.add_argument("--route-sweep", action="store_true",
                    help="route cost-model sweep on one 8192x8192 bf16 linear (chosen vs measured fastest route)")
     p.add_argument("--sweep-T", default="8,32,128,512,2048,8192")
+    p.add_argument("--sweep-ops", default="project,similarity_projected,similarity_exact")
+    p.add_argument("--sweep-routes", default="factored,materialize,gram")
+    p.add_argument("--sweep-pool-gb", type=float, default=16.0, help="resident train factors per sweep point")
     a = p.parse_args()
     names = a.linears.split(",")
     global LINEARS
@@ -332,7 +335,7 @@ def route_sweep_main(args):
         N = 2 ** 24 // T
         L = tda.LayerDesc(d, d, T, k, k, seed=0, layer=0)
         ex_bytes = T * 2 * d * 2
-        P = max(1, min(N, int(16e9 // ex_bytes)))
+        P = max(1, min(N, int(args.sweep_pool_gb * 1e9 // ex_bytes)))
         A = torch.empty(P * T * d, dtype=torch.bfloat16, device=dev)
         B = torch.empty_like(A)
         Aq = torch.empty(nq * T * d, dtype=torch.bfloat16, device=dev)
@@ -364,6 +367,9 @@ def route_sweep_main(args):
 
         point = {"T": T, "n_train": N, "pool_examples": P, "ops": {}}
         for op, opname, routes in ops:
+            if opname not in args.sweep_ops.split(","):
+                continue
+            routes = tuple(r for r in routes if names[r] in args.sweep_routes.split(","))
             rec = {"flop_model_choice": names[tda.tda_route(L, op, nq, N, tda.TDA_BF16)[0]]}
             tda.tda_route_set_model(1)
             ch, est = tda.tda_route(L, op, nq, N, tda.TDA_BF16)
@@ -401,8 +407,9 @@ def route_sweep_main(args):
             fastest = min(meas, key=lambda x: meas[x]["seconds"])
             rec["measured"] = meas
             rec["measured_fastest"] = fastest
-            rec["calibrated_over_fastest"] = meas[rec["calibrated_choice"]]["seconds"] / meas[fastest]["seconds"]
-            rec["flop_model_over_fastest"] = meas[rec["flop_model_choice"]]["seconds"] / meas[fastest]["seconds"]
+            for key, choice in (("calibrated_over_fastest", rec["calibrated_choice"]),
+                                ("flop_model_over_fastest", rec["flop_model_choice"])):
+                rec[key] = meas[choice]["seconds"] / meas[fastest]["seconds"] if choice in meas else None
             point["ops"][opname] = rec
         tda.tda_device_status()
         out["points"].append(point)
