@@ -60,7 +60,12 @@ struct Cfg {
     static constexpr int kStageLd = K + 4;                                // padded fp32 staging row
     static constexpr int kAccCols = 2 * K;                                // At | Bt of one tile
     static constexpr int kBufCols = G * kAccCols;                         // one accumulator buffer
-    static constexpr uint32_t kTmemCols = 2 * kBufCols < 32 ? 32 : 2 * kBufCols;
+    // tcgen05.alloc takes a power of two from 32 to 512 columns
+    static constexpr uint32_t kTmemCols = 2 * kBufCols <= 32    ? 32
+                                          : 2 * kBufCols <= 64  ? 64
+                                          : 2 * kBufCols <= 128 ? 128
+                                          : 2 * kBufCols <= 256 ? 256
+                                                                : 512;
     static constexpr size_t kSmemStage = 2ull * kTileM * kStageLd * 4;
     static constexpr size_t kSmemBarsMax = 8 * (3 * kMaxStages + 7) + 16;
     static constexpr int kFit = (int)((kSmemMax - 1024 - kSmemStage - kSmemBarsMax) / kStageBytes);
@@ -71,7 +76,8 @@ struct Cfg {
     static constexpr int RB = K / 16 > 0 ? K / 16 : 1;
     static constexpr int CB = K / 8;
     static_assert(kStages >= 3 && kSmem <= kSmemMax, "shared memory per CTA");
-    static_assert(kStageBytes % 1024 == 0 && kTmemCols <= 512, "operand alignment / TMEM columns");
+    static_assert(kStageBytes % 1024 == 0 && 2 * kBufCols <= (int)kTmemCols && kTmemCols <= 512,
+                  "operand alignment / TMEM columns");
 };
 
 struct Params {
