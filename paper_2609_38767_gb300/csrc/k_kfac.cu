@@ -265,6 +265,74 @@ ekfac_partial_kernel(const float* __restrict__ phi, int64_t n, int64_t ld, const
     }
 }
 
+// Square k = 16, 32, 64: thread (column c, row group g) keeps U_a[:, c] and,
+// per example, column c of Y = Phi U_a in registers; Phi and U_g^T rows are
+// read from shared memory as warp broadcasts, so each multiply-add costs a
+// quarter of a (vector) shared load.
+template <int K>
+__global__ void __launch_bounds__(256)
+ekfac_reg_kernel(const float* __restrict__ phi, int64_t n, int64_t ld, const double* __restrict__ st0, int64_t stride,
+                 float* __restrict__ part) {
+    constexpr int RG = 256 / K;  // row groups
+    constexpr int RPT = K / RG;  // rows per thread
+    __shared__ __align__(16) float F[K * K];    // Phi_i [r][j]
+    __shared__ __align__(16) float Y[K * K];    // Phi_i U_a [r][c]
+    __shared__ __align__(16) float UgT[K * K];  // U_g^T [r][j]
+    const int layer = blockIdx.y;
+    const double* st = st0 + (int64_t)layer * stride;
+    const KfLayout l(K, K);
+    const int c = threadIdx.x % K, g = threadIdx.x / K;
+    float ua[K];
+#pragma unroll
+    for (int j = 0; j < K; ++j) ua[j] = (float)st[l.Ua + j * K + c];
+    for (int e = threadIdx.x; e < K * K; e += 256) UgT[e] = (float)st[l.Ug + (e % K) * K + e / K];
+    float acc[RPT];
+#pragma unroll
+    for (int m = 0; m < RPT; ++m) acc[m] = 0.f;
+    const float* ph = phi + (int64_t)layer * K * K;
+    for (int64_t i = blockIdx.x; i < n; i += gridDim.x) {
+        __syncthreads();
+        for (int e = threadIdx.x; e < K * K / 4; e += 256)
+            reinterpret_cast<float4*>(F)[e] = reinterpret_cast<const float4*>(ph + i * ld)[e];
+        __syncthreads();
+#pragma unroll
+        for (int m = 0; m < RPT; ++m) {  // Y[r][c] = sum_j Phi[r][j] U_a[j][c]
+            const int r = g + RG * m;
+            float sacc = 0.f;
+#pragma unroll
+            for (int j = 0; j < K; j += 4) {
+                const float4 f = *reinterpret_cast<const float4*>(F + r * K + j);
+                sacc = fmaf(f.x, ua[j], sacc);
+                sacc = fmaf(f.y, ua[j + 1], sacc);
+                sacc = fmaf(f.z, ua[j + 2], sacc);
+                sacc = fmaf(f.w, ua[j + 3], sacc);
+            }
+            Y[r * K + c] = sacc;
+        }
+        __syncthreads();
+        float yc[K];
+#pragma unroll
+        for (int j = 0; j < K; ++j) yc[j] = Y[j * K + c];
+#pragma unroll
+        for (int m = 0; m < RPT; ++m) {  // X[r][c] = sum_j U_g[j][r] Y[j][c]; accumulate X^2
+            const int r = g + RG * m;
+            float sacc = 0.f;
+#pragma unroll
+            for (int j = 0; j < K; j += 4) {
+                const float4 u = *reinterpret_cast<const float4*>(UgT + r * K + j);
+                sacc = fmaf(u.x, yc[j], sacc);
+                sacc = fmaf(u.y, yc[j + 1], sacc);
+                sacc = fmaf(u.z, yc[j + 2], sacc);
+                sacc = fmaf(u.w, yc[j + 3], sacc);
+            }
+            acc[m] = fmaf(sacc, sacc, acc[m]);
+        }
+    }
+    float* out = part + ((int64_t)layer * gridDim.x + blockIdx.x) * K * K;
+#pragma unroll
+    for (int m = 0; m < RPT; ++m) out[(g + RG * m) * K + c] = acc[m];
+}
+
 // Le of every layer += its block partials (fixed order); N += n
 __global__ void ekfac_reduce_kernel(const float* __restrict__ part, int nblk, double* __restrict__ st0, int64_t stride,
                                     int64_t ka, int64_t kg, double n) {
@@ -407,13 +475,26 @@ cudaError_t launch_kfac_ekfac_accum(int n_layers, double* state, int64_t ka, int
     const bool su = ka <= 64 && kg <= 64;
     const size_t smem = (size_t)(2 * ka * kg + (su ? ka * ka + kg * kg : 0)) * 4;
     const int64_t stride = (int64_t)kfac_state_bytes(ka, kg) / 8;
+    const dim3 grid((unsigned)nblk, (unsigned)n_layers);
+    const bool aligned = ((uintptr_t)phi & 15) == 0 && (ld & 3) == 0;
+    if (ka == kg && aligned && (ka == 16 || ka == 32 || ka == 64)) {
+        note_launches(2);
+        if (ka == 16)
+            ekfac_reg_kernel<16><<<grid, 256, 0, s>>>(phi, n, ld, state, stride, part);
+        else if (ka == 32)
+            ekfac_reg_kernel<32><<<grid, 256, 0, s>>>(phi, n, ld, state, stride, part);
+        else
+            ekfac_reg_kernel<64><<<grid, 256, 0, s>>>(phi, n, ld, state, stride, part);
+        ekfac_reduce_kernel<<<dim3((unsigned)((ka * kg + 255) / 256), (unsigned)n_layers), 256, 0, s>>>(
+            part, nblk, state, stride, ka, kg, (double)n);
+        return cudaGetLastError();
+    }
     cudaError_t e = su ? cudaFuncSetAttribute(ekfac_partial_kernel<true>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                               (int)smem)
                        : cudaFuncSetAttribute(ekfac_partial_kernel<false>,
                                               cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
     if (e != cudaSuccess) return e;
     note_launches(2);
-    const dim3 grid((unsigned)nblk, (unsigned)n_layers);
     if (su)
         ekfac_partial_kernel<true><<<grid, kKfThreads, smem, s>>>(phi, n, ld, state, stride, ka, kg, part);
     else

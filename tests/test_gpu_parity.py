@@ -674,3 +674,21 @@ def test_mask_gather_matches_oracle(dev, orc, dtype, N, T, di, do, nc):
     assert rel_fro(got[:, :nc][:, ok], ref[:, ok]) <= 1e-5
     assert np.isnan(got[:, 5]).all() and np.isnan(got[:, 7]).all()
     assert (got[:, nc:] == 3.0).all()
+
+
+@pytest.mark.gpu
+@pytest.mark.parametrize("kind", [tda.TDA_KFAC, tda.TDA_EKFAC])
+def test_kfac_without_curvature_is_damping_only(dev, kind):
+    # degenerate case: no training tokens seen (M = 0): C_a = C_g = 0, every eigenvalue is 0,
+    # so the preconditioner is lambda_abs^-1 I and Qhat = Q / lambda_abs
+    k = 16
+    st = torch.empty(tda.tda_kfac_state_bytes(k, k) // 8, dtype=torch.float64, device=dev)
+    tda.tda_kfac_reset(k, k, st)
+    tda.tda_kfac_eigen(k, k, st)
+    Q = torch.randn(3, k * k, device=dev)
+    Qh = torch.empty_like(Q)
+    tda.tda_kfac_apply(kind, k, k, st, 0.5, 0.1, Q, 3, k * k, Qh, k * k)
+    tda.tda_device_status()
+    s = st.cpu().numpy()
+    assert s[2] == 0 and s[3] == 0  # Jacobi: already diagonal, zero sweeps
+    torch.testing.assert_close(Qh, Q / 0.5, rtol=1e-6, atol=1e-7)
