@@ -326,9 +326,9 @@ def route_sweep_main(args):
     ops = [(tda.TDA_OP_PROJECT, "project", (0, 1)), (tda.TDA_OP_SIMILARITY_PROJECTED, "similarity_projected", (0, 1, 2)),
            (tda.TDA_OP_SIMILARITY_EXACT, "similarity_exact", (1, 2))]
     out = {"mode": "route-sweep", "linear": [d, d], "k": k, "n_query": nq, "dtype": "bf16",
-           "calibrated_rates_tflops": dict(zip(("factored", "materialize", "gram_bf16", "gram_fp32"),
-                                               [r / 1e12 for r in rates[:4]])),
-           "calibrated_bw_gbs": rates[4] / 1e9,
+           "calibrated_rates_tflops": dict(zip(("factored", "materialize_build", "gram_bf16", "gram_fp32",
+                                                "dw_sign_projection", "dw_dots"), [r / 1e12 for r in rates[:6]])),
+           "calibrated_bw_gbs": rates[6] / 1e9,
            "points": []}
     stream = torch.cuda.current_stream()
     for T in [int(x) for x in args.sweep_T.split(",")]:
@@ -383,14 +383,17 @@ def route_sweep_main(args):
                 n1 = min(P, 8)
                 wsb = max(tda.tda_workspace_size(op, L, tda.TDA_BF16, n_q, P, r), 256)
                 if op == tda.TDA_OP_SIMILARITY_EXACT and r == 1:
-                    # room for 128 materialised train gradients per chunk next to the queries'
-                    wsb = tda.tda_workspace_size(op, L, tda.TDA_BF16, n_q + 127, P, r)
+                    # materialised train gradients go through in chunks, each chunk re-reading the
+                    # queries' DW: time whole chunks (one and two per call) so that cost lands in the slope
+                    chunk = max(1, min(128, P // 2))
+                    wsb = tda.tda_workspace_size(op, L, tda.TDA_BF16, n_q + chunk - 1, P, r)
+                    n1 = chunk
                 if op == tda.TDA_OP_SIMILARITY_PROJECTED:
                     wsb = max(wsb, min(2 << 30, tda.tda_workspace_size(op, L, tda.TDA_BF16, n_q, P, r) * 16))
                 ws = torch.empty(wsb, dtype=torch.uint8, device=dev)
                 timed(op, r, n_q, n1, ws, wsb)  # warm-up
                 t1 = timed(op, r, n_q, n1, ws, wsb)
-                while t1 < 0.05 and n1 < N:
+                while t1 < 0.05 and n1 < N and not (op == tda.TDA_OP_SIMILARITY_EXACT and r == 1):
                     n1 = min(N, n1 * max(2, int(0.1 / max(t1, 1e-6))))
                     t1 = timed(op, r, n_q, n1, ws, wsb)
                 if 2 * n1 <= N:

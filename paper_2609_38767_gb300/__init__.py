@@ -311,7 +311,7 @@ def tda_route(L, op, n1, n2, dtype) -> tuple[int, list[float]]:
 
 
 def tda_route_calibrate(ws, ws_bytes, stream=None) -> list[float]:
-    rates = (ctypes.c_double * 5)()
+    rates = (ctypes.c_double * 7)()
     _check(load().tda_route_calibrate(_ptr(ws), ws_bytes, _stream(stream), rates))
     return list(rates)
 

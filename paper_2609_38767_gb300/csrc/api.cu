@@ -53,20 +53,25 @@ unsigned int* device_error_word() {
 // ---------------------------------------------------------------------------
 static std::mutex g_route_mu;
 static int g_route_model = 0;
-// flop/s of the factored and materialise routes, of the Gram route on bf16
-// factors (tensor cores) and on fp32 factors (projected factors, CUDA cores)
-static double g_rate[4] = {0, 0, 0, 0};
+// measured flop/s: [0] factored projection, [1] materialising DW, [2] Gram
+// route on bf16 factors (tensor cores), [3] Gram route on fp32 factors
+// (projected factors, CUDA cores), [4] projecting a materialised DW with the
+// signs, [5] Frobenius inner products of materialised DW
+constexpr int kNumRates = 6;
+static double g_rate[kNumRates] = {0, 0, 0, 0, 0, 0};
 static double g_bw = 0;               // bytes/s
 
 struct RouteCounts {
     double flops[3];
     double bytes[3];
-    int gram_rate;  // which measured rate the Gram route runs at (2 or 3)
+    int gram_rate;   // which measured rate the Gram route runs at (2 or 3)
+    double build;    // the materialise route's DW construction flops (the rest of flops[1] runs at post_rate)
+    int post_rate;   // 4 (sign projection of DW) or 5 (Frobenius inner products)
 };
 
-void set_route_rates(const double rate[4], double bw) {
+void set_route_rates(const double* rate, double bw) {
     std::lock_guard<std::mutex> lock(g_route_mu);
-    for (int r = 0; r < 4; ++r) g_rate[r] = rate[r];
+    for (int r = 0; r < kNumRates; ++r) g_rate[r] = rate[r];
     g_bw = bw;
     g_route_model = (rate[0] > 0 && bw > 0) ? 1 : 0;
 }
@@ -87,6 +92,8 @@ static RouteCounts route_counts(const tda_layer_desc& L, tda_op op, int64_t n1, 
                    L.d_in % 8 == 0 && L.d_out % 8 == 0)
                       ? 2
                       : 3;
+    c.build = (op == TDA_OP_PROJECT || op == TDA_OP_NORM_PROJECTED || op == TDA_OP_NORM_EXACT ? B1 : B1 + B2) * build;
+    c.post_rate = (op == TDA_OP_SIMILARITY_EXACT || op == TDA_OP_NORM_EXACT) ? 5 : 4;
     if (op == TDA_OP_PROJECT) {
         c.flops[0] = B1 * (proj + contract);
         c.flops[1] = B1 * (build + dense);
@@ -165,6 +172,9 @@ static tda_route_id choose(const RouteCounts& c, double* cost_out) {
     for (int r = 0; r < 3; ++r) {
         if (c.flops[r] < 0) {
             cost[r] = -1;
+        } else if (g_route_model == 1 && r == 1 && g_rate[1] > 0 && g_rate[c.post_rate] > 0 && g_bw > 0) {
+            // materialise: DW construction and its use run on different kernels
+            cost[r] = std::fmax(c.build / g_rate[1] + (c.flops[1] - c.build) / g_rate[c.post_rate], c.bytes[r] / g_bw);
         } else if (g_route_model == 1 && g_rate[r == 2 ? c.gram_rate : r] > 0 && g_bw > 0) {
             cost[r] = std::fmax(c.flops[r] / g_rate[r == 2 ? c.gram_rate : r], c.bytes[r] / g_bw);
         } else {

@@ -3,10 +3,12 @@
 // different rates, so the estimate becomes seconds = max(flops / rate_route,
 // bytes / bandwidth) with rates measured here by short launches of the route
 // kernels themselves).
+#include <cmath>
+
 #include "tda_internal.cuh"
 
 namespace tda {
-void set_route_rates(const double rate[4], double bw);
+void set_route_rates(const double* rate, double bw);
 }
 
 using namespace tda;
@@ -56,22 +58,50 @@ extern "C" tda_status tda_route_calibrate(void* ws, size_t ws_bytes, void* strea
     float* S = (float*)(base + TDA_CALIBRATE_WS_BYTES - (1u << 20));
 
     EventTimer ev;
-    double secs[4] = {0, 0, 0, 0};
-    double flops[4] = {0, 0, 0, 0};
-    double bytes_a = 0;
-    for (int route = 0; route < 4; ++route) {
+    // kinds: 0 factored projection, 1 DW construction, 2 Gram (bf16), 3 Gram (projected factors),
+    // 4 materialise route of the projection (construction + sign projection), 5 Frobenius dots
+    constexpr int kKinds = 6;
+    double secs[kKinds] = {0, 0, 0, 0, 0, 0};
+    const double T = 128, d = 1024, k = 32;
+    const int64_t nG = 16;                      // materialised DW for kinds 1, 5 (16 x 4 MiB)
+    float* G = (float*)rest;
+    float* part = G + (size_t)nG * 1024 * 1024;  // split-K partial sums for kind 5 (2 Mi floats)
+    char* rest2 = (char*)(part + (2 << 20));
+    const size_t rest2_bytes = TDA_CALIBRATE_WS_BYTES - (size_t)(rest2 - base) - (1u << 20);
+    // DW construction of a 2048 x 2048 layer at T = 512 (the same factor bytes viewed as 32
+    // examples of 512 tokens): 4 DWs of 16 MiB
+    tda_layer_desc L512 = L;
+    L512.T = 512;
+    L512.d_in = L512.d_out = 2048;
+    const int64_t nB = 4;
+    // Gram route on a 4096 x 4096 layer (the factor bytes viewed as 128 examples of 128 tokens)
+    tda_layer_desc L4k = L;
+    L4k.d_in = L4k.d_out = 4096;
+    // Frobenius dots of 32 query and 64 train DWs of a 1024 x 1024 layer (4 MiB each)
+    const int64_t d5 = 1024 * 1024;
+    float* G5 = (float*)rest2;
+    const int splits = score_splitk_splits(32, 64, d5);
+    if ((size_t)splits * 32 * 64 > ((size_t)2 << 20) || rest2_bytes < (size_t)96 * d5 * 4)
+        return fail(TDA_ERR_WORKSPACE, "calibration scratch layout");
+    for (int kind = 0; kind < kKinds; ++kind) {
         for (int rep = 0; rep < 4; ++rep) {
             if (rep == 1) cudaEventRecord(ev.a, s);
-            if (route == 0) {
+            if (kind == 0) {
                 st = tda_project(&L, TDA_BF16, A, B, Nf, phi, 1024, TDA_ROUTE_FACTORED, nullptr, 0, s);
-            } else if (route == 1) {
-                st = tda_project(&L, TDA_BF16, A, B, 8, phi, 1024, TDA_ROUTE_MATERIALIZE, rest, rest_bytes, s);
-            } else if (route == 2) {
-                st = tda_similarity_exact(&L, TDA_BF16, A, B, 8, A, B, 256, S, 256, 0.f, TDA_ROUTE_GRAM,
+            } else if (kind == 1) {
+                st = cuda_check(launch_materialize_G(L512, TDA_BF16, A, B, 0, nB, G, s), "calibrate DW");
+            } else if (kind == 2) {
+                st = tda_similarity_exact(&L4k, TDA_BF16, A, B, 8, A, B, 112, S, 112, 0.f, TDA_ROUTE_GRAM,
                                           nullptr, 0, s);
-            } else {  // Gram of projected (fp32) factors
-                st = tda_similarity_projected(&L, TDA_BF16, A, B, 8, A, B, 64, S, 64, 0.f, TDA_ROUTE_GRAM, rest,
-                                              rest_bytes, s);
+            } else if (kind == 3) {
+                st = tda_similarity_projected(&L, TDA_BF16, A, B, 8, A, B, 64, S, 64, 0.f, TDA_ROUTE_GRAM, rest2,
+                                              rest2_bytes, s);
+            } else if (kind == 4) {
+                st = tda_project(&L, TDA_BF16, A, B, 8, phi, 1024, TDA_ROUTE_MATERIALIZE, rest2, rest2_bytes, s);
+            } else {
+                st = cuda_check(
+                    launch_score_splitk(G5, 32, d5, G5 + 32 * d5, 64, d5, d5, S, 64, 0.f, splits, part, s),
+                    "calibrate dots");
             }
             if (st) return st;
         }
@@ -79,24 +109,25 @@ extern "C" tda_status tda_route_calibrate(void* ws, size_t ws_bytes, void* strea
         if ((st = cuda_check(cudaEventSynchronize(ev.b), "calibration sync"))) return st;
         float ms = 0;
         cudaEventElapsedTime(&ms, ev.a, ev.b);
-        secs[route] = ms * 1e-3 / 3.0;
+        secs[kind] = ms * 1e-3 / 3.0;
     }
-    const double T = 128, d = 1024, k = 32;
-    flops[0] = Nf * (2 * T * (d * k + d * k) + 2 * T * k * k);
-    flops[1] = 8 * (2 * T * d * d + 2 * d * d * k + 2 * d * k * k);
-    flops[2] = 8 * 256 * 2 * T * T * (d + d);
-    flops[3] = (8 + 64) * 2 * T * (d * k + d * k) + 8 * 64 * 2 * T * T * (k + k);
-    bytes_a = Nf * (T * (d + d) * 2 + 4 * k * k);
-    double rate[4];
-    for (int r = 0; r < 4; ++r) rate[r] = secs[r] > 0 ? flops[r] / secs[r] : 0;
-    const double bw = secs[0] > 0 ? bytes_a / secs[0] : 0;
+    const double build = 2 * T * d * d;
+    double rate[kKinds];
+    rate[0] = Nf * (2 * T * (d * k + d * k) + 2 * T * k * k) / secs[0];
+    rate[1] = nB * 2 * 512.0 * 2048.0 * 2048.0 / secs[1];
+    rate[2] = 8 * 112 * 2 * T * T * (4096.0 + 4096.0) / secs[2];
+    rate[3] = ((8 + 64) * 2 * T * (d * k + d * k) + 8 * 64 * 2 * T * T * (k + k)) / secs[3];
+    // the projection's materialise route minus its construction (at T = 128): the sign projection alone
+    const double sign_secs = secs[4] - 8 * build / rate[1];
+    rate[4] = 8 * (2 * d * d * k + 2 * d * k * k) / (sign_secs > secs[4] * 0.05 ? sign_secs : secs[4] * 0.05);
+    rate[5] = 32.0 * 64 * 2 * d5 / secs[5];
+    for (int r = 0; r < kKinds; ++r)
+        if (!(rate[r] > 0) || !std::isfinite(rate[r])) rate[r] = 0;
+    const double bw = secs[0] > 0 ? Nf * (T * (d + d) * 2 + 4 * k * k) / secs[0] : 0;
     set_route_rates(rate, bw);
     if (rates_out) {
-        rates_out[0] = rate[0];
-        rates_out[1] = rate[1];
-        rates_out[2] = rate[2];
-        rates_out[3] = rate[3];
-        rates_out[4] = bw;
+        for (int r = 0; r < kKinds; ++r) rates_out[r] = rate[r];
+        rates_out[kKinds] = bw;
     }
     return TDA_OK;
 }

@@ -8,6 +8,8 @@
 //   never forming DW.
 #include <cuda_bf16.h>
 
+#include <type_traits>
+
 #include "tda_internal.cuh"
 
 namespace tda {
@@ -265,6 +267,14 @@ project_factors_kernel(const T* __restrict__ X, int64_t e0, int64_t Tn, int64_t 
 template <typename T>
 void launch_materialize(const void* A, const void* B, int64_t e0, int64_t nb,
                         const tda_layer_desc& L, float* G, cudaStream_t s) {
+    if constexpr (std::is_same<T, __nv_bfloat16>::value) {
+        // bf16 factors: the tensor-core kernel (fp32 accumulation, same result up to summation order)
+        unsigned int* err = device_error_word();
+        if (err && materialize_tc_supported(L, TDA_BF16, A, B, G)) {
+            launch_materialize_tc(L, A, B, e0, nb, G, err, s);
+            return;
+        }
+    }
     dim3 grid((unsigned)((L.d_in + kT - 1) / kT), (unsigned)((L.d_out + kT - 1) / kT), (unsigned)nb);
     note_launches(1);
     materialize_kernel<T><<<grid, kTh, 0, s>>>((const T*)A, (const T*)B, e0, L.T, L.d_in, L.d_out, G);

@@ -237,7 +237,7 @@ __global__ void sum_slabs_kernel(const float* __restrict__ part, int splits, int
 int score_splitk_splits(int64_t n_q, int64_t n_t, int64_t D) {
     const int64_t tiles = ((n_t + kTT - 1) / kTT) * ((n_q + kTQ - 1) / kTQ);
     int64_t z = 608 / (tiles > 0 ? tiles : 1);
-    const int64_t by_d = D / 4096;  // at least 4096 features per slice
+    const int64_t by_d = D / 1024;  // at least 1024 features per slice
     if (z > by_d) z = by_d;
     if (z > 256) z = 256;
     return z < 2 ? 1 : (int)z;

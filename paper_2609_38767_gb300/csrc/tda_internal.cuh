@@ -100,6 +100,10 @@ int mask_gather_tokens_per_pass(int64_t d_in, int64_t d_out, size_t el);
 cudaError_t launch_mask_gather(const tda_layer_desc& L, tda_dtype dt, const void* A, const void* B, int64_t N,
                                const int32_t* rows, const int32_t* cols, int64_t n_coords, float* out, int64_t ld_out,
                                cudaStream_t s);
+// Route (b)'s materialisation on tcgen05 for bf16 factors (k_materialize_tc.cu)
+bool materialize_tc_supported(const tda_layer_desc& L, tda_dtype dt, const void* A, const void* B, const float* G);
+cudaError_t launch_materialize_tc(const tda_layer_desc& L, const void* A, const void* B, int64_t e0, int64_t n,
+                                  float* G, unsigned int* err, cudaStream_t s);
 cudaError_t launch_project_tc(const tda_layer_desc& L, const void* A, const void* B, int64_t N,
                               float* phi, int64_t ld_phi, unsigned int* err, cudaStream_t s);
 

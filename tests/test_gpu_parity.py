@@ -692,3 +692,22 @@ def test_kfac_without_curvature_is_damping_only(dev, kind):
     s = st.cpu().numpy()
     assert s[2] == 0 and s[3] == 0  # Jacobi: already diagonal, zero sweeps
     torch.testing.assert_close(Qh, Q / 0.5, rtol=1e-6, atol=1e-7)
+
+
+@pytest.mark.gpu
+@pytest.mark.parametrize("N,T,di,do,k", [(3, 70, 264, 136, 16), (2, 37, 512, 200, 32), (5, 130, 256, 128, 8)])
+def test_materialize_route_tensor_core_matches_oracle(dev, orc, N, T, di, do, k):
+    # route (b) for bf16: DW built by the tensor-core kernel (ragged rows, columns and token chunks),
+    # then projected; also the exact norms and similarities that materialise DW
+    A, B = make_factors(N, T, di, do, "bf16", stream=71, sigma_b=0.1, mask_p=0.02)
+    L = tda.LayerDesc(di, do, T, k, k, seed=9, layer=6)
+    Ad, Bd = to_dev(A, "bf16", dev), to_dev(B, "bf16", dev)
+    got, _ = gpu_project(L, "bf16", Ad, Bd, N, tda.TDA_ROUTE_MATERIALIZE, dev)
+    A64, B64 = synth.to_f64(A, "bf16"), synth.to_f64(B, "bf16")
+    assert rel_fro(got, orc.project(A64, B64, k, k, 9, 6)) <= 1e-5
+    wsb = tda.tda_workspace_size(tda.TDA_OP_NORM_EXACT, L, tda.TDA_BF16, N, 0, tda.TDA_ROUTE_MATERIALIZE) * 2
+    ws = torch.empty(wsb, dtype=torch.uint8, device=dev)
+    nrm = torch.empty(N, device=dev)
+    tda.tda_norms(tda.TDA_OP_NORM_EXACT, L, tda.TDA_BF16, Ad, Bd, N, nrm, tda.TDA_ROUTE_MATERIALIZE, ws, wsb)
+    tda.tda_device_status()
+    np.testing.assert_allclose(nrm.cpu().numpy(), orc.sq_norms(A64, B64, "materialized"), rtol=1e-5)
