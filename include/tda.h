@@ -3,8 +3,12 @@
  *
  * The library turns per-example weight gradients of linear layers, given in
  * factored form, into seeded Kronecker-projected features, preconditions the
- * queries with a damped Fisher inverse and scores queries against training
- * examples (dattri-LLM paper, Sec. 3.2 and App. A.2, A.4, B.2, B.3).
+ * queries with a damped Fisher inverse (or K-FAC / EK-FAC on the projected
+ * factors) and scores queries against training examples, routing each layer
+ * and operation between factored, materialised and Gram forms (dattri-LLM
+ * paper, Sec. 3.2 and App. A.2, A.4, B.2, B.3). It also computes routed
+ * per-example gradient norms and cosine scores, token-level score
+ * decompositions and random-mask reductions from the same factors.
  *
  * Notation. A linear layer z = W a has W in R^{N_o x N_i}. For one example with
  * T token positions the paper's factors are a in R^{N_i x T} and g = Dz in
@@ -110,7 +114,8 @@ tda_status tda_proj_entries(uint64_t seed, uint32_t layer, int32_t side, int32_t
 /* ---------------------------------------------------------------------------
  * tda_workspace_size -- bytes of scratch `ws` that the matching call needs
  * (op PROJECT -> tda_project; SIMILARITY_PROJECTED -> tda_similarity_projected;
- * SIMILARITY_EXACT -> tda_similarity_exact), for one train example per chunk.
+ * SIMILARITY_EXACT -> tda_similarity_exact; NORM_* -> tda_norms), for one
+ * train example per chunk.
  * n1 = examples (or queries), n2 = train examples (similarity only).
  * route AUTO resolves through tda_route() first. Host only; no device work.
  * ------------------------------------------------------------------------- */
@@ -443,10 +448,14 @@ tda_status tda_route(const tda_layer_desc* L, tda_op op, int64_t n1, int64_t n2,
  * launches of the route kernels inside the caller's scratch `ws` (at least
  * TDA_CALIBRATE_WS_BYTES bytes, contents destroyed), synchronises `stream`,
  * then switches tda_route to the time model. rates_out (host, may be NULL)
- * receives 5 doubles: flop/s of the factored and materialise routes, of the
- * Gram route on bf16 factors (exact similarity; tensor cores on sm_103), of
- * the Gram route on fp32 factors (projected factors, fp32 layers, norms), and
- * the streaming bytes/s of the factored kernel. */
+ * receives 7 doubles: flop/s of [0] the factored projection, [1] building DW
+ * (materialise route; tensor cores for bf16 on sm_103), [2] the Gram route on
+ * bf16 factors (exact similarity; tensor cores), [3] the Gram route on fp32
+ * factors (projected factors, fp32 layers, norms), [4] projecting a built DW
+ * with the signs, [5] Frobenius inner products of built DWs; [6] the streaming
+ * bytes/s of the factored kernel. The materialise route's time is its DW
+ * construction at [1] plus the rest at [4] or [5]. Rates are measured on bf16
+ * factors. */
 #define TDA_CALIBRATE_WS_BYTES ((size_t)768 << 20)
 tda_status tda_route_calibrate(void* ws, size_t ws_bytes, void* stream, double* rates_out);
 /* 0 = flop model (the paper's), 1 = calibrated time model. */
