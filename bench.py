@@ -807,7 +807,9 @@ def main():
             "warmup": args.warmup, "ms_per_step": ms, "higher_is_better": True, "scaling": "weak",
             "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
             "config": {**workload(args), "parallelism": f"train examples sharded over {world} rank(s)"
-                       + (", global top-k merged by all-gather" if world > 1 else "")},
+                       + (", global top-k merged by all-gather" if world > 1 else ""),
+                       "routes": {name: {0: "factored", 1: "materialize", 2: "gram"}[r] for (name, _, _), r
+                                  in zip(LINEARS, pipe.routes())}},
             "roofline": roofline, "phases": phases, "cpu_baseline": cpu, "e2e": e2e, "gpu_launches": launches,
             "clocks": ck,
         }
