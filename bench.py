@@ -92,6 +92,8 @@ def parse_args():
     p.add_argument("--sweep-ops", default="project,similarity_projected,similarity_exact")
     p.add_argument("--sweep-routes", default="factored,materialize,gram")
     p.add_argument("--sweep-pool-gb", type=float, default=16.0, help="resident train factors per sweep point")
+    p.add_argument("--sweep-d", type=int, default=8192, help="square linear d x d of the sweep")
+    p.add_argument("--sweep-nq", type=int, default=128, help="queries of the sweep")
     a = p.parse_args()
     names = a.linears.split(",")
     global LINEARS
@@ -303,7 +305,8 @@ def reference_main(args):
 
 # ---------------------------------------------------------------------------- GPU arm
 def route_sweep_main(args):
-    """One 8192x8192 bf16 linear, A, B ~ N(0,1), k = 64, 128 queries, N_train = 2^24 / T for each T:
+    """One 8192x8192 bf16 linear (--sweep-d), A, B ~ N(0,1), k = 64, 128 queries (--sweep-nq),
+    N_train = 2^24 / T for each T:
     every route of every op is timed on the device and extrapolated to the full N_train by a
     two-point linear fit in the train count (t = a + b n); the route the Table 2 flop model
     picks and the one the calibrated model picks are reported beside the measured fastest."""
@@ -317,7 +320,7 @@ def route_sweep_main(args):
     tda.load()
     dev = torch.device("cuda", 0)
     torch.cuda.set_device(dev)
-    d, k, nq = 8192, 64, 128
+    d, k, nq = args.sweep_d, 64, args.sweep_nq
     D = k * k
     cal_ws = torch.empty(tda.TDA_CALIBRATE_WS_BYTES, dtype=torch.uint8, device=dev)
     rates = tda.tda_route_calibrate(cal_ws, tda.TDA_CALIBRATE_WS_BYTES)
@@ -464,7 +467,8 @@ def reuse_main(args):
     torch.cuda.synchronize()
     if args.token_scores:
         out = torch.empty((Nq, N * T), dtype=torch.float32, device=dev)
-        wsb = max(tda.tda_token_scores_workspace_size(L) for L in layers) * 256
+        # 1024 examples per chunk, plus room for the query matrices' hi/lo halves (tensor-core contraction)
+        wsb = max(tda.tda_token_scores_workspace_size(L) for L in layers) * 1024 + (4 << 20)
         ws = torch.empty(wsb, dtype=torch.uint8, device=dev)
 
         def step():
@@ -473,8 +477,12 @@ def reuse_main(args):
                                      0.0 if li == 0 else 1.0, ws, wsb)
 
         flops = sum(N * 2.0 * T * (L.d_in + L.d_out) * k + 2.0 * Nq * N * T * D for L in layers)
-        mode = {"mode": "token-level scores", "n_query": Nq, "outputs_per_step": Nq * N * T}
-        roof_kernel, roof_bound = "factor projection + token contraction (CUDA cores)", "alu"
+        # the step reads every factor once (projection, HBM-bound) and then contracts the projected
+        # factors on the tensor cores; the roofline is the whole step against reading the factors
+        fbytes = sum(2.0 * N * T * (L.d_in + L.d_out) for L in layers)
+        mode = {"mode": "token-level scores", "n_query": Nq, "outputs_per_step": Nq * N * T,
+                "contraction_tflop_per_step": 2.0 * Nq * N * T * D * nl / 1e12}
+        roof_kernel, roof_bound = "factor projection (tcgen05) + token contraction (tcgen05, 3xTF32), whole step", "hbm"
     else:
         K = args.masks
         rng = np.random.default_rng(2026)
@@ -524,13 +532,20 @@ def reuse_main(args):
         pass
     alu = 152 * 128 * 2 * float(peaks.get("sm_max_mhz", 2070.0)) * 1e6 / 1e12
     rate = flops / (ms * 1e-3) / 1e12
+    if roof_bound == "hbm":
+        hbm = float(peaks.get("hbm_gbs", 6794.1))
+        roof = {"bound": "hbm", "kernel": roof_kernel, "achieved": fbytes / (ms * 1e-3) / 1e9, "peak": hbm,
+                "unit": "GB/s", "frac": fbytes / (ms * 1e-3) / 1e9 / hbm, "traffic": None,
+                "peak_source": "MEASURED_PEAKS.json hbm_gbs (copy)"}
+    else:
+        roof = {"bound": roof_bound, "kernel": roof_kernel, "achieved": rate, "peak": alu, "unit": "TFLOP/s",
+                "frac": rate / alu, "traffic": None,
+                "peak_source": "fp32 SIMT peak derived from 152 SMs x 128 lanes x 2 x max clock"}
     print(json.dumps({
         "metric": METRIC, "value": N / (ms * 1e-3), "unit": "examples/s", "n_gpus": 1, "steps": args.steps,
         "warmup": args.warmup, "ms_per_step": ms, "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
         "dtype": "bf16", "data": "synthetic", "config": {**workload(args), **mode},
-        "roofline": {"bound": roof_bound, "kernel": roof_kernel, "achieved": rate, "peak": alu, "unit": "TFLOP/s",
-                     "frac": rate / alu, "traffic": None,
-                     "peak_source": "fp32 SIMT peak derived from 152 SMs x 128 lanes x 2 x max clock"},
+        "roofline": roof,
         "cpu_baseline": None, "e2e": None, "gpu_launches": launches, "clocks": ck}))
 
 

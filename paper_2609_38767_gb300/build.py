@@ -25,7 +25,7 @@ FLAGS = ["-O3", "-std=c++17", "-lineinfo", "-Xcompiler", "-fPIC", "--expt-relaxe
 
 LIBS = {
     "libtda.so": ["api.cu", "calibrate.cu", "k_project_simt.cu", "k_project_tc.cu", "k_routes.cu",
-                  "k_precond.cu", "k_score.cu", "stream_host.cu", "noalloc.cu", "selftest.cu", "k_gemm_tc.cu", "k_gram_tc.cu", "k_kfac.cu", "k_tokens.cu", "k_materialize_tc.cu"],
+                  "k_precond.cu", "k_score.cu", "stream_host.cu", "noalloc.cu", "selftest.cu", "k_gemm_tc.cu", "k_gram_tc.cu", "k_kfac.cu", "k_tokens.cu", "k_tokens_tc.cu", "k_materialize_tc.cu"],
     "libtda_synth.so": ["synth.cu"],
 }
 

@@ -565,18 +565,30 @@ tda_status tda_token_scores(const tda_layer_desc* L, tda_dtype dtype, const void
     if (!ws || ws_bytes < per)
         return fail(TDA_ERR_WORKSPACE, "tda_token_scores needs >= %zu bytes of ws, got %zu", per, ws_bytes);
     cudaStream_t s = (cudaStream_t)stream;
-    int64_t chunk = (int64_t)(ws_bytes / per);
+    // The tensor-core contraction (k_in = 32) keeps R's hi and lo halves at the
+    // front of the workspace when it has room for them and one example.
+    const size_t rsplit = token_tc_split_bytes(L->k_in, L->k_out, n_q);
+    const bool tc = token_tc_supported(L->k_in, L->k_out, n_q) && ((uintptr_t)ws & 255) == 0 && ws_bytes >= rsplit + per &&
+                    ((uintptr_t)R & 3) == 0;
+    const size_t off = tc ? rsplit : 0;
+    int64_t chunk = (int64_t)((ws_bytes - off) / per);
     if (chunk > N) chunk = N;
     if (chunk > 65535) chunk = 65535;
     const float scale = projection_scale(*L);
-    float* Y = (float*)ws;
+    float* Y = (float*)((char*)ws + off);
     for (int64_t e0 = 0; e0 < N; e0 += chunk) {
         const int64_t c = N - e0 < chunk ? N - e0 : chunk;
         if ((st = cuda_check(launch_project_factors(*L, dtype, A, B, e0, c, Y, s), "project factors"))) return st;
-        if ((st = cuda_check(launch_token_scores(Y, Y + c * L->T * L->k_in, c, L->T, L->k_in, L->k_out, R, n_q, ld_R,
-                                                 scale, out, ld_q_out, e0, beta, s),
-                             "token scores")))
-            return st;
+        const float* Yb = Y + c * L->T * L->k_in;
+        if (tc)
+            st = cuda_check(launch_token_scores_tc(Y, Yb, c, L->T, L->k_in, L->k_out, R, n_q, ld_R, scale, out,
+                                                   ld_q_out, e0, beta, (float*)ws, s),
+                            "token scores (tensor cores)");
+        else
+            st = cuda_check(launch_token_scores(Y, Yb, c, L->T, L->k_in, L->k_out, R, n_q, ld_R, scale, out, ld_q_out,
+                                                e0, beta, s),
+                            "token scores");
+        if (st) return st;
     }
     return TDA_OK;
 }

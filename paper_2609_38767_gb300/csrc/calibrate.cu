@@ -77,11 +77,13 @@ extern "C" tda_status tda_route_calibrate(void* ws, size_t ws_bytes, void* strea
     // Gram route on a 4096 x 4096 layer (the factor bytes viewed as 128 examples of 128 tokens)
     tda_layer_desc L4k = L;
     L4k.d_in = L4k.d_out = 4096;
-    // Frobenius dots of 32 query and 64 train DWs of a 1024 x 1024 layer (4 MiB each)
-    const int64_t d5 = 1024 * 1024;
+    // Frobenius dots of 128 query and 128 train DWs of a 512 x 512 layer (1 MiB each): one
+    // full query batch against one chunk of materialised train gradients
+    const int64_t d5 = 512 * 512, nq5 = 128, nt5 = 128;
     float* G5 = (float*)rest2;
-    const int splits = score_splitk_splits(32, 64, d5);
-    if ((size_t)splits * 32 * 64 > ((size_t)2 << 20) || rest2_bytes < (size_t)96 * d5 * 4)
+    const bool dots_tc = score_dots_tc(G5, nq5, d5, G5 + nq5 * d5, nt5, d5, d5);
+    const int splits = score_splitk_splits(nq5, nt5, d5, dots_tc);
+    if ((size_t)splits * nq5 * nt5 > ((size_t)2 << 20) || rest2_bytes < (size_t)(nq5 + nt5) * d5 * 4)
         return fail(TDA_ERR_WORKSPACE, "calibration scratch layout");
     for (int kind = 0; kind < kKinds; ++kind) {
         for (int rep = 0; rep < 4; ++rep) {
@@ -100,7 +102,7 @@ extern "C" tda_status tda_route_calibrate(void* ws, size_t ws_bytes, void* strea
                 st = tda_project(&L, TDA_BF16, A, B, 8, phi, 1024, TDA_ROUTE_MATERIALIZE, rest2, rest2_bytes, s);
             } else {
                 st = cuda_check(
-                    launch_score_splitk(G5, 32, d5, G5 + 32 * d5, 64, d5, d5, S, 64, 0.f, splits, part, s),
+                    launch_score_splitk(G5, nq5, d5, G5 + nq5 * d5, nt5, d5, d5, S, nt5, 0.f, splits, part, dots_tc, s),
                     "calibrate dots");
             }
             if (st) return st;
@@ -120,7 +122,7 @@ extern "C" tda_status tda_route_calibrate(void* ws, size_t ws_bytes, void* strea
     // the projection's materialise route minus its construction (at T = 128): the sign projection alone
     const double sign_secs = secs[4] - 8 * build / rate[1];
     rate[4] = 8 * (2 * d * d * k + 2 * d * k * k) / (sign_secs > secs[4] * 0.05 ? sign_secs : secs[4] * 0.05);
-    rate[5] = 32.0 * 64 * 2 * d5 / secs[5];
+    rate[5] = (double)nq5 * nt5 * 2 * d5 / secs[5];
     for (int r = 0; r < kKinds; ++r)
         if (!(rate[r] > 0) || !std::isfinite(rate[r])) rate[r] = 0;
     const double bw = secs[0] > 0 ? Nf * (T * (d + d) * 2 + 4 * k * k) / secs[0] : 0;

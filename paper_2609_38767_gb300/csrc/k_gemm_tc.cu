@@ -9,14 +9,17 @@
 // size ~2^-22). Each K=8 step therefore issues three tcgen05.mma.kind::tf32.
 //
 // CTA tile: 128 rows of Phi (MMA M, one TMEM lane each) x BN query columns
-// (MMA N). Warps 0-3 load 128-byte row chunks with coalesced 16-byte loads,
-// split them and store hi and lo in the 128B-swizzled K-major operand layout
-// of a stage; lane 0 of warp 4 issues the MMAs; warps 4-7 read the fp32
-// accumulator tile from TMEM. A thread-block cluster of cs CTAs splits K; the
+// (MMA N). Lane 0 of warp 5 copies the fp32 chunks of both operands with TMA
+// (32 features = one 128-byte row per operand row, 128B swizzle: already the
+// K-major operand layout) into the hi tiles of a stage; warps 0-3 split them in
+// place (hi stays, lo goes to the lo tile at the same offset); lane 0 of warp 4
+// issues the MMAs; warps 4-7 read the fp32 accumulator tile from TMEM. A thread-block cluster of cs CTAs splits K; the
 // members' partial tiles are summed into the leader CTA over distributed shared
 // memory (deterministic, no workspace) before the leader writes S. All waits
 // are bounded (see tc_ptx.cuh).
 #include <cuda.h>
+
+#include <mutex>
 
 #include "tda_internal.cuh"
 
@@ -41,7 +44,7 @@ struct GCfg {
     // error; the epilogue sums them on CUDA cores with round-to-nearest.
     static constexpr int kAcc = 512 / BN < 8 ? 512 / BN : 8;
     static constexpr uint32_t kTmemCols = 512;
-    static constexpr size_t kSmem = 1024 + (size_t)kStages * kStageBytes + 8 * (2 * kStages + 4) + 16;  // + barriers, TMEM slot, abort flag
+    static constexpr size_t kSmem = 1024 + (size_t)kStages * kStageBytes + 8 * (3 * kStages + 4) + 16;  // + barriers, TMEM slot, abort flag
 };
 
 struct GParams {
@@ -51,6 +54,8 @@ struct GParams {
     int64_t n_t, n_q, K, lda, ldb, ld_S;
     float beta;
     int cs, tiles_n;
+    int64_t kslice, slab;  // split-K over gridDim.y: K slice per CTA row, S stride per slice (0: no split)
+    int splits;            // gridDim.y
     unsigned int* err;
 };
 
@@ -71,52 +76,34 @@ __device__ __forceinline__ void split_tf32(float x, float& hi, float& lo) {
     lo = x - hi;
 }
 
-// Rows [r0, r0+rows) of a row-major fp32 matrix, K chunk kc, into the hi and lo
-// tiles (row r at r*128 bytes, 16-byte chunk c at (c ^ (r & 7)) * 16). The 128
-// producer threads cover 4 rows x 8 chunks per pass; out-of-range is zero.
-// ROWS is a compile-time multiple of 16 so that all of a thread's loads issue
-// before the first one is consumed.
-template <int ROWS>
-__device__ __forceinline__ void load_split(const float* __restrict__ X, int64_t ld, int64_t nrows, int64_t K,
-                                           int64_t r0, int64_t k0, uint8_t* hi, uint8_t* lo, int pt) {
-    constexpr int kPer = ROWS / 16;
-    const int c = pt & 7;
-    const int64_t kk = k0 + c * 4;
-    float4 vals[kPer];
-#pragma unroll
-    for (int u = 0; u < kPer; ++u) {
-        const int64_t r = r0 + (pt >> 3) + 16 * u;
-        float4 v = make_float4(0.f, 0.f, 0.f, 0.f);
-        if (r < nrows) {
-            const float* p = X + r * ld + kk;
-            if (kk + 3 < K) {
-                v = __ldg(reinterpret_cast<const float4*>(p));
-            } else {
-                v.x = kk < K ? p[0] : 0.f;
-                v.y = kk + 1 < K ? p[1] : 0.f;
-                v.z = kk + 2 < K ? p[2] : 0.f;
-                v.w = 0.f;
-            }
-        }
-        vals[u] = v;
-    }
-#pragma unroll
-    for (int u = 0; u < kPer; ++u) {
-        const int rr = (pt >> 3) + 16 * u;
-        const float4 v = vals[u];
+// Split a TMA-written fp32 tile in place: hi = x truncated to TF32 stays, lo =
+// x - hi goes to the lo tile at the same byte offset (the swizzle is the same
+// for both). 128 threads, one 16-byte group each per pass (conflict-free).
+template <uint32_t BYTES>
+__device__ __forceinline__ void split_tile(uint8_t* hi, uint8_t* lo, int pt) {
+#pragma unroll 4
+    for (uint32_t off = (uint32_t)pt * 16u; off < BYTES; off += 128u * 16u) {
+        const float4 v = *reinterpret_cast<const float4*>(hi + off);
         float4 h, l;
         split_tf32(v.x, h.x, l.x);
         split_tf32(v.y, h.y, l.y);
         split_tf32(v.z, h.z, l.z);
         split_tf32(v.w, h.w, l.w);
-        const uint32_t off = (uint32_t)rr * kRowBytes + (uint32_t)((c ^ (rr & 7)) << 4);
         *reinterpret_cast<float4*>(hi + off) = h;
         *reinterpret_cast<float4*>(lo + off) = l;
     }
 }
+__device__ __forceinline__ void tma_load_2d(uint32_t dst, const CUtensorMap* tm, int c0, int c1, uint32_t bar) {
+    asm volatile(
+        "cp.async.bulk.tensor.2d.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1, {%2, %3}], [%4];" ::"r"(
+            dst),
+        "l"((uint64_t)tm), "r"(c0), "r"(c1), "r"(bar)
+        : "memory");
+}
 
 template <int BN>
-__global__ void __launch_bounds__(kThreads, 1) score3x_kernel(const GParams p) {
+__global__ void __launch_bounds__(kThreads, 1)
+score3x_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB, const GParams p) {
     using C = GCfg<BN>;
     extern __shared__ uint8_t smem_raw[];
     uint8_t* smem = (uint8_t*)(((uintptr_t)smem_raw + 1023) & ~(uintptr_t)1023);
@@ -127,7 +114,8 @@ __global__ void __launch_bounds__(kThreads, 1) score3x_kernel(const GParams p) {
     uint64_t* red_go = tfull + 1;            // count 1 (leader's remote arrive)
     uint64_t* red_full = red_go + 1;         // count cs-1
     uint64_t* mma_done = red_full + 1;       // count 1
-    uint32_t* tmem_slot = (uint32_t*)(mma_done + 1);
+    uint64_t* raw_full = mma_done + 1;       // [kStages] TMA bytes landed (count 1 + tx)
+    uint32_t* tmem_slot = (uint32_t*)(raw_full + C::kStages);
     volatile int* abort = (volatile int*)(tmem_slot + 1);
 
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
@@ -135,6 +123,7 @@ __global__ void __launch_bounds__(kThreads, 1) score3x_kernel(const GParams p) {
         for (int s = 0; s < C::kStages; ++s) {
             mbar_init(smem_u32(&full[s]), 4);
             mbar_init(smem_u32(&empty[s]), 1);
+            mbar_init(smem_u32(&raw_full[s]), 1);
         }
         mbar_init(smem_u32(tfull), 1);
         mbar_init(smem_u32(red_go), 1);
@@ -156,31 +145,64 @@ __global__ void __launch_bounds__(kThreads, 1) score3x_kernel(const GParams p) {
     const uint32_t crank = cluster_rank();
     const int64_t tile = blockIdx.x / p.cs;
     const int64_t m0 = (tile / p.tiles_n) * kBM, n0 = (tile % p.tiles_n) * BN;
-    const int64_t nkc = (p.K + kKC - 1) / kKC;
+    // split-K slice z covers features [z*kslice, z*kslice + Kz) and writes its own slab of S
+    const int64_t kbase = (int64_t)blockIdx.y * p.kslice;
+    const int64_t Kz = p.kslice ? ((p.K - kbase) < p.kslice ? (p.K - kbase) : p.kslice) : p.K;
+    float* Sz = p.S + (int64_t)blockIdx.y * p.slab;
+    const int64_t nkc = (Kz + kKC - 1) / kKC;
     const int64_t per = (nkc + p.cs - 1) / p.cs;
     const int64_t kc0 = crank * per, kc1 = (kc0 + per) < nkc ? (kc0 + per) : nkc;
 
     if (warp < 4) {
-        // ---------------- producers: global fp32 -> split -> swizzled smem
+        // ---------------- split warps: raw fp32 (TMA) -> hi in place + lo
         const int pt = threadIdx.x;
         uint32_t it = 0;
         for (int64_t kc = kc0; kc < kc1; ++kc, ++it) {
             const int s = it % C::kStages;
             const uint32_t ph = (it / C::kStages) & 1u;
             bool got = true;
-            if (lane == 0) got = wait_bounded(smem_u32(&empty[s]), ph ^ 1u, abort, p.err);
+            if (lane == 0) got = wait_bounded(smem_u32(&raw_full[s]), ph, abort, p.err);
             got = __shfl_sync(0xffffffffu, got, 0);
             __syncwarp();
             if (!got) break;
             uint8_t* st = smem + (size_t)s * C::kStageBytes;
-            load_split<kBM>(p.A, p.lda, p.n_t, p.K, m0, kc * kKC, st, st + C::kABytes, pt);
-            load_split<BN>(p.B, p.ldb, p.n_q, p.K, n0, kc * kKC, st + 2 * C::kABytes,
-                           st + 2 * C::kABytes + C::kBBytes, pt);
+            split_tile<C::kABytes>(st, st + C::kABytes, pt);
+            split_tile<C::kBBytes>(st + 2 * C::kABytes, st + 2 * C::kABytes + C::kBBytes, pt);
             fence_proxy_async();
             __syncwarp();
             if (lane == 0) mbar_arrive(smem_u32(&full[s]));
         }
     } else {
+        if (warp == 5 && lane == 0) {
+            // ---------------- TMA producer: fp32 chunks of Phi rows m0.. and Qhat rows n0..
+            // (features past the slice end belong to the next slice only when the slice
+            // is not the last; slices are multiples of 32 features, so no chunk crosses one)
+            uint32_t it = 0, last_par[C::kStages];
+            bool issued[C::kStages];
+            for (int s = 0; s < C::kStages; ++s) issued[s] = false;
+            for (int64_t kc = kc0; kc < kc1; ++kc, ++it) {
+                const int s = it % C::kStages;
+                const uint32_t ph = (it / C::kStages) & 1u;
+                if (!wait_bounded(smem_u32(&empty[s]), ph ^ 1u, abort, p.err)) break;
+                const uint32_t st = smem_u32(smem + (size_t)s * C::kStageBytes), bar = smem_u32(&raw_full[s]);
+                const int k = (int)(kbase + kc * kKC);
+                mbar_arrive_tx(bar, C::kABytes + C::kBBytes);
+                tma_load_2d(st, &tmA, k, (int)m0, bar);
+                tma_load_2d(st + 2 * C::kABytes, &tmB, k, (int)n0, bar);
+                issued[s] = true;
+                last_par[s] = ph;
+            }
+            // copies still in flight when the consumers stopped early land before the CTA exits
+            for (int s = 0; s < C::kStages; ++s)
+                if (issued[s]) {
+                    const uint64_t t0 = global_ns();
+                    while (!mbar_try_wait(smem_u32(&raw_full[s]), last_par[s]))
+                        if (global_ns() - t0 > kTimeoutNs) {
+                            atomicOr(p.err, kErrTimeout);
+                            break;
+                        }
+                }
+        }
         if (warp == 4 && lane == 0) {
             // ---------------- MMA issuer
             const uint32_t idesc = idesc_tf32(kBM, BN);
@@ -290,7 +312,7 @@ __global__ void __launch_bounds__(kThreads, 1) score3x_kernel(const GParams p) {
                     for (int c = 0; c < BN; ++c) {
                         const int64_t n = n0 + c;
                         if (n < p.n_q) {
-                            float* dst = p.S + n * p.ld_S + m;
+                            float* dst = Sz + n * p.ld_S + m;
                             *dst = (p.beta == 0.f) ? acc[c] : p.beta * (*dst) + acc[c];
                         }
                     }
@@ -499,9 +521,44 @@ __global__ void __launch_bounds__(kThreads, 1) fit3x_kernel(const FParams p) {
     }
 }
 
+typedef CUresult (*EncodeTiledFn)(CUtensorMap*, CUtensorMapDataType, cuuint32_t, void*, const cuuint64_t*,
+                                  const cuuint64_t*, const cuuint32_t*, const cuuint32_t*, CUtensorMapInterleave,
+                                  CUtensorMapSwizzle, CUtensorMapL2promotion, CUtensorMapFloatOOBfill);
+
+EncodeTiledFn encode_fn() {
+    static EncodeTiledFn fn = nullptr;
+    static std::once_flag once;
+    std::call_once(once, [] {
+        void* f = nullptr;
+        cudaDriverEntryPointQueryResult q;
+        if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &f, 12000, cudaEnableDefault, &q) ==
+                cudaSuccess &&
+            q == cudaDriverEntryPointSuccess)
+            fn = (EncodeTiledFn)f;
+    });
+    return fn;
+}
+
+// 2-D map over fp32 X[rows][ld] (features 0..K-1 used): box 32 features x box_rows rows,
+// 128-byte swizzle, zero fill past K and past the last row.
+bool make_map_f32(CUtensorMap* tm, const float* X, int64_t rows, int64_t K, int64_t ld, int box_rows) {
+    EncodeTiledFn enc = encode_fn();
+    if (!enc) return false;
+    cuuint64_t dims[2] = {(cuuint64_t)K, (cuuint64_t)rows};
+    cuuint64_t strides[1] = {(cuuint64_t)(ld * 4)};
+    cuuint32_t box[2] = {(cuuint32_t)kKC, (cuuint32_t)box_rows};
+    cuuint32_t estr[2] = {1, 1};
+    return enc(tm, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, 2, const_cast<float*>(X), dims, strides, box, estr,
+               CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+               CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
 template <int BN>
 cudaError_t launch_bn(GParams p, cudaStream_t s) {
     using C = GCfg<BN>;
+    CUtensorMap tmA, tmB;
+    if (!make_map_f32(&tmA, p.A, p.n_t, p.K, p.lda, kBM) || !make_map_f32(&tmB, p.B, p.n_q, p.K, p.ldb, BN))
+        return cudaErrorInvalidValue;
     static int sms = 0;
     if (!sms) {
         int dev = 0;
@@ -511,9 +568,9 @@ cudaError_t launch_bn(GParams p, cudaStream_t s) {
     }
     const int64_t tiles_m = (p.n_t + kBM - 1) / kBM, tiles_n = (p.n_q + BN - 1) / BN;
     const int64_t tiles = tiles_m * tiles_n;
-    const int64_t nkc = (p.K + kKC - 1) / kKC;
+    const int64_t nkc = ((p.kslice ? p.kslice : p.K) + kKC - 1) / kKC;
     int cs = 1;
-    while (cs < 4 && tiles * cs * 2 <= sms && nkc >= 8 * cs * 2) cs *= 2;
+    while (cs < 4 && tiles * p.splits * cs * 2 <= sms && nkc >= 8 * cs * 2) cs *= 2;
     // the leader's stage buffers must hold the members' partial tiles
     while (cs > 1 && (size_t)(cs - 1) * kBM * BN * 4 > (size_t)C::kStages * C::kStageBytes) cs >>= 1;
     p.cs = cs;
@@ -526,14 +583,14 @@ cudaError_t launch_bn(GParams p, cudaStream_t s) {
     attr[0].val.clusterDim.x = (unsigned)cs;
     attr[0].val.clusterDim.y = 1;
     attr[0].val.clusterDim.z = 1;
-    cfg.gridDim = dim3((unsigned)(tiles * cs));
+    cfg.gridDim = dim3((unsigned)(tiles * cs), (unsigned)p.splits);
     cfg.blockDim = dim3(kThreads);
     cfg.dynamicSmemBytes = C::kSmem;
     cfg.stream = s;
     cfg.attrs = attr;
     cfg.numAttrs = 1;
     note_launches(1);
-    e = cudaLaunchKernelEx(&cfg, score3x_kernel<BN>, p);
+    e = cudaLaunchKernelEx(&cfg, score3x_kernel<BN>, tmA, tmB, p);
     if (e != cudaSuccess) return e;
     return cudaGetLastError();
 }
@@ -550,8 +607,11 @@ bool score_tc_supported(tda_dtype qdt, const void* Qhat, int64_t n_q, int64_t ld
         cudaDeviceGetAttribute(&minor, cudaDevAttrComputeCapabilityMinor, dev);
         sm103 = (major == 10 && minor == 3) ? 1 : 0;
     }
-    if (!sm103 || qdt != TDA_F32) return false;
-    if (n_q < 1 || n_t < 1 || D < 64 || n_q > (1LL << 24) || n_t > (1LL << 31) / kBM * kBM) return false;
+    if (!sm103 || qdt != TDA_F32 || !encode_fn()) return false;
+    // TMA: 32-bit coordinates, row strides of whole 16-byte groups below 2^40 bytes
+    if (n_q < 1 || n_t < 1 || D < 64 || D >= (1LL << 31) || n_q > (1LL << 24) || n_t > (1LL << 31) / kBM * kBM)
+        return false;
+    if (ld_q * 4 >= (1LL << 40) || ld_phi * 4 >= (1LL << 40)) return false;
     if ((ld_q & 3) || (ld_phi & 3)) return false;
     if (((uintptr_t)Qhat & 15) || ((uintptr_t)Phi & 15)) return false;
     return true;
@@ -570,7 +630,44 @@ cudaError_t launch_score_tc(const float* Qhat, int64_t n_q, int64_t ld_q, const 
     p.ldb = ld_q;
     p.ld_S = ld_S;
     p.beta = beta;
+    p.kslice = 0;
+    p.slab = 0;
+    p.splits = 1;
     p.err = err;
+    if (n_q <= 64) return launch_bn<64>(p, s);
+    return launch_bn<128>(p, s);
+}
+
+int score_tc_tiles(int64_t n_q, int64_t n_t) {
+    const int64_t bn = n_q <= 64 ? 64 : 128;
+    const int64_t t = ((n_t + kBM - 1) / kBM) * ((n_q + bn - 1) / bn);
+    return t > (1 << 30) ? (1 << 30) : (int)t;
+}
+
+// Partial scores of `splits` feature slices: part[z][q][i] = sum over slice z of
+// Phi[i][f] Qhat[q][f] (slices of a multiple of 32 features; part holds
+// splits * n_q * n_t floats). The caller sums the slabs.
+cudaError_t launch_score_tc_slices(const float* Qhat, int64_t n_q, int64_t ld_q, const float* Phi, int64_t n_t,
+                                   int64_t ld_phi, int64_t D, int splits, float* part, unsigned int* err,
+                                   cudaStream_t s) {
+    GParams p{};
+    p.A = Phi;
+    p.B = Qhat;
+    p.n_t = n_t;
+    p.n_q = n_q;
+    p.K = D;
+    p.lda = ld_phi;
+    p.ldb = ld_q;
+    int64_t kslice = (D + splits - 1) / splits;
+    kslice = (kslice + kKC - 1) / kKC * kKC;
+    p.kslice = kslice;
+    p.splits = (int)((D + kslice - 1) / kslice);
+    p.slab = n_q * n_t;
+    p.S = part;
+    p.ld_S = n_t;
+    p.beta = 0.f;
+    p.err = err;
+    if (p.splits > 65535) return cudaErrorInvalidValue;
     if (n_q <= 64) return launch_bn<64>(p, s);
     return launch_bn<128>(p, s);
 }

@@ -333,7 +333,10 @@ cudaError_t launch_similarity_materialized(const tda_layer_desc& L, tda_dtype dt
     // The Frobenius dots have few rows and very long ones: split the feature
     // axis over many CTAs when the chunk leaves one train gradient's room for
     // the partial sums.
-    int splits = score_splitk_splits(n_q, chunk, gsz);
+    // (3xTF32 tensor cores when the operands allow, decided once for every chunk:
+    // Gq and Gt share base alignment and row length)
+    const bool tc = score_dots_tc(Gq, n_q, gsz, Gt, chunk, gsz, gsz);
+    int splits = score_splitk_splits(n_q, chunk, gsz, tc);
     float* part = nullptr;
     if (splits > 1) {
         const size_t need = (size_t)splits * (size_t)n_q * (size_t)chunk;
@@ -357,7 +360,7 @@ cudaError_t launch_similarity_materialized(const tda_layer_desc& L, tda_dtype dt
             launch_materialize<__nv_bfloat16>(At, Bt, i0, cnt, L, Gt, s);
         else
             launch_materialize<float>(At, Bt, i0, cnt, L, Gt, s);
-        cudaError_t e = launch_score_splitk(Gq, n_q, gsz, Gt, cnt, gsz, gsz, S + i0, ld_S, beta, splits, part, s);
+        cudaError_t e = launch_score_splitk(Gq, n_q, gsz, Gt, cnt, gsz, gsz, S + i0, ld_S, beta, splits, part, tc, s);
         if (e != cudaSuccess) return e;
     }
     return cudaGetLastError();

@@ -234,22 +234,56 @@ __global__ void sum_slabs_kernel(const float* __restrict__ part, int splits, int
 }
 }  // namespace
 
-int score_splitk_splits(int64_t n_q, int64_t n_t, int64_t D) {
-    const int64_t tiles = ((n_t + kTT - 1) / kTT) * ((n_q + kTQ - 1) / kTQ);
-    int64_t z = 608 / (tiles > 0 ? tiles : 1);
-    const int64_t by_d = D / 1024;  // at least 1024 features per slice
-    if (z > by_d) z = by_d;
+bool score_dots_tc(const float* Q, int64_t n_q, int64_t ld_q, const float* Phi, int64_t n_t, int64_t ld_phi,
+                   int64_t D) {
+    return device_error_word() != nullptr && score_tc_supported(TDA_F32, Q, n_q, ld_q, Phi, n_t, ld_phi, D);
+}
+
+int score_splitk_splits(int64_t n_q, int64_t n_t, int64_t D, bool tc) {
+    int64_t z;
+    if (tc) {
+        // one 3xTF32 CTA per SM (about 200 KiB of shared memory each), slices of >= 4096 features
+        static int sms = 0;
+        if (!sms) {
+            int dev = 0;
+            cudaGetDevice(&dev);
+            cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+            if (sms <= 0) sms = 1;
+        }
+        const int64_t tiles = score_tc_tiles(n_q, n_t);
+        z = sms / (tiles > 0 ? tiles : 1);
+        if (z > D / 4096) z = D / 4096;
+    } else {
+        const int64_t tiles = ((n_t + kTT - 1) / kTT) * ((n_q + kTQ - 1) / kTQ);
+        z = 608 / (tiles > 0 ? tiles : 1);
+        if (z > D / 1024) z = D / 1024;  // at least 1024 features per slice
+    }
     if (z > 256) z = 256;
     return z < 2 ? 1 : (int)z;
 }
 
 // fp32 score with the feature axis split over `splits` CTAs per tile: for
 // few, very long rows (inner products of materialised gradients). part: device
-// scratch of splits * n_q * n_t floats.
+// scratch of splits * n_q * n_t floats. tc: the 3xTF32 tensor-core kernel
+// (score_dots_tc said yes), else the CUDA-core one.
 cudaError_t launch_score_splitk(const float* Q, int64_t n_q, int64_t ld_q, const float* Phi, int64_t n_t,
                                 int64_t ld_phi, int64_t D, float* S, int64_t ld_S, float beta, int splits,
-                                float* part, cudaStream_t s) {
+                                float* part, bool tc, cudaStream_t s) {
     if (n_q == 0 || n_t == 0) return cudaSuccess;
+    if (tc) {
+        unsigned int* err = device_error_word();
+        if (splits <= 1) return launch_score_tc(Q, n_q, ld_q, Phi, n_t, ld_phi, D, S, ld_S, beta, err, s);
+        int64_t kslice = (D + splits - 1) / splits;
+        kslice = (kslice + 31) / 32 * 32;
+        const int z = (int)((D + kslice - 1) / kslice);
+        cudaError_t e = launch_score_tc_slices(Q, n_q, ld_q, Phi, n_t, ld_phi, D, splits, part, err, s);
+        if (e != cudaSuccess) return e;
+        int64_t blocks = (n_q * n_t + 255) / 256;
+        if (blocks > 4096) blocks = 4096;
+        note_launches(1);
+        sum_slabs_kernel<<<(unsigned)blocks, 256, 0, s>>>(part, z, n_q, n_t, S, ld_S, beta);
+        return cudaGetLastError();
+    }
     if (splits <= 1) return launch_score(Q, TDA_F32, n_q, ld_q, Phi, n_t, ld_phi, D, S, ld_S, beta, s);
     int64_t kslice = (D + splits - 1) / splits;
     kslice = (kslice + kSK - 1) / kSK * kSK;

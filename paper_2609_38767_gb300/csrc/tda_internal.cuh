@@ -97,6 +97,13 @@ cudaError_t launch_token_scores(const float* Ya, const float* Yb, int64_t n, int
                                 const float* R, int64_t n_q, int64_t ld_R, float scale, float* out, int64_t ld_q,
                                 int64_t i0, float beta, cudaStream_t s);
 int mask_gather_tokens_per_pass(int64_t d_in, int64_t d_out, size_t el);
+// Token-level scores on tcgen05, 3xTF32 (k_tokens_tc.cu): k_in = 32, k_out in {16, 32, 64};
+// Rs is token_tc_split_bytes of scratch for R's hi and lo halves.
+size_t token_tc_split_bytes(int ka, int kg, int64_t n_q);
+bool token_tc_supported(int ka, int kg, int64_t n_q);
+cudaError_t launch_token_scores_tc(const float* Ya, const float* Yb, int64_t n, int64_t T, int ka, int kg,
+                                   const float* R, int64_t n_q, int64_t ld_R, float scale, float* out, int64_t ld_q,
+                                   int64_t i0, float beta, float* Rs, cudaStream_t s);
 cudaError_t launch_mask_gather(const tda_layer_desc& L, tda_dtype dt, const void* A, const void* B, int64_t N,
                                const int32_t* rows, const int32_t* cols, int64_t n_coords, float* out, int64_t ld_out,
                                cudaStream_t s);
@@ -170,10 +177,20 @@ bool score_tc_supported(tda_dtype qdt, const void* Qhat, int64_t n_q, int64_t ld
                         int64_t ld_phi, int64_t D);
 cudaError_t launch_score_tc(const float* Qhat, int64_t n_q, int64_t ld_q, const float* Phi, int64_t n_t, int64_t ld_phi,
                             int64_t D, float* S, int64_t ld_S, float beta, unsigned int* err, cudaStream_t s);
-int score_splitk_splits(int64_t n_q, int64_t n_t, int64_t D);
+int score_tc_tiles(int64_t n_q, int64_t n_t);
+cudaError_t launch_score_tc_slices(const float* Qhat, int64_t n_q, int64_t ld_q, const float* Phi, int64_t n_t,
+                                   int64_t ld_phi, int64_t D, int splits, float* part, unsigned int* err,
+                                   cudaStream_t s);
+// Split-K score for few, very long rows (Frobenius dots of materialised DW):
+// score_dots_tc says whether the tensor-core kernel takes these operands;
+// score_splitk_splits plans the feature slices for that kernel (tc) or the
+// CUDA-core one; launch_score_splitk runs the plan (part: splits * n_q * n_t floats).
+bool score_dots_tc(const float* Q, int64_t n_q, int64_t ld_q, const float* Phi, int64_t n_t, int64_t ld_phi,
+                   int64_t D);
+int score_splitk_splits(int64_t n_q, int64_t n_t, int64_t D, bool tc);
 cudaError_t launch_score_splitk(const float* Q, int64_t n_q, int64_t ld_q, const float* Phi, int64_t n_t,
                                 int64_t ld_phi, int64_t D, float* S, int64_t ld_S, float beta, int splits,
-                                float* part, cudaStream_t s);
+                                float* part, bool tc, cudaStream_t s);
 cudaError_t launch_topk(const float* S, int64_t n_q, int64_t n_t, int64_t ld_S, int32_t k,
                         int32_t* idx, float* val, cudaStream_t s);
 

@@ -132,7 +132,8 @@ def test_project_leading_dimension_and_edge_sizes(dev, orc):
 # ------------------------------------------------------------------ exact similarity
 @pytest.mark.parametrize("dtype", ["f32", "bf16"])
 @pytest.mark.parametrize("route", [tda.TDA_ROUTE_GRAM, tda.TDA_ROUTE_MATERIALIZE, tda.TDA_ROUTE_AUTO])
-@pytest.mark.parametrize("shape", [(3, 5, 21, 40, 24), (3, 5, 7, 256, 264)])  # 2nd: split-K Frobenius dots
+# 2nd, 3rd: split-K Frobenius dots (3rd: a ragged last feature slice)
+@pytest.mark.parametrize("shape", [(3, 5, 21, 40, 24), (3, 5, 7, 256, 264), (2, 11, 5, 264, 136)])
 def test_similarity_exact_matches_oracle(dev, orc, dtype, route, shape):
     nq, nt, T, di, do = shape
     Aq, Bq = make_factors(nq, T, di, do, dtype, stream=6, query=True)
@@ -651,6 +652,30 @@ def test_token_scores_match_oracle(dev, orc, dtype, N, T, di, do, k, kind):
     # the decomposition sums to the sequence-level score
     phi = orc.project(A64, B64, ki, ko, 7, 4, kind)
     np.testing.assert_allclose(ref.sum(2), orc.score(R, phi), rtol=1e-10)
+
+
+@pytest.mark.gpu
+@pytest.mark.parametrize("dtype,N,T,di,do,ki,ko,nq", [("bf16", 64, 512, 128, 64, 32, 32, 9),
+                                                      ("f32", 7, 45, 96, 80, 32, 16, 11),
+                                                      ("bf16", 5, 77, 64, 128, 32, 64, 5)])
+def test_token_scores_tensor_core_shapes(dev, orc, dtype, N, T, di, do, ki, ko, nq):
+    # k_in = 32 runs on the tensor cores: several token tiles per CTA (first case), several query
+    # stages of 256 (q, r) rows, k_out = 16 / 32 / 64, ragged token and query tails; beta = 0.5
+    A, B = make_factors(N, T, di, do, dtype, stream=63, sigma_b=0.1, mask_p=0.05)
+    L = tda.LayerDesc(di, do, T, ki, ko, seed=11, layer=2)
+    R = np.random.default_rng(N + T).standard_normal((nq, ko, ki)).astype(np.float32)
+    Rd = torch.from_numpy(R.reshape(nq, -1)).to(dev)
+    out0 = np.random.default_rng(2).standard_normal((nq, N * T + 3)).astype(np.float32)
+    out = torch.from_numpy(out0).to(dev)
+    wsb = tda.tda_token_scores_workspace_size(L) * N + (1 << 20)
+    ws = torch.empty(wsb, dtype=torch.uint8, device=dev)
+    tda.tda_token_scores(L, TD[dtype], to_dev(A, dtype, dev), to_dev(B, dtype, dev), N, Rd, nq, ki * ko, out,
+                         N * T + 3, 0.5, ws, wsb)
+    tda.tda_device_status()
+    ref = orc.token_scores(synth.to_f64(A, dtype), synth.to_f64(B, dtype), R, ki, ko, 11, 2, 0)
+    got = out.cpu().numpy()
+    assert rel_fro(got[:, : N * T].reshape(nq, N, T) - 0.5 * out0[:, : N * T].reshape(nq, N, T), ref) <= 1e-5
+    np.testing.assert_array_equal(got[:, N * T:], out0[:, N * T:])
 
 
 @pytest.mark.gpu
