@@ -74,6 +74,8 @@ def parse_args():
     p.add_argument("--curvature", default="fisher", choices=["fisher", "kfac", "ekfac"],
                    help="preconditioner: full empirical Fisher of the projected features, or K-FAC / EK-FAC "
                         "on the projected factors (damping 0.1 x mean eigenvalue)")
+    p.add_argument("--overlap-sms", type=int, default=0,
+                   help="Fisher query side on a second stream; the train projection leaves this many SMs free")
     p.add_argument("--e2e-steps", type=int, default=2)
     p.add_argument("--no-e2e", action="store_true")
     p.add_argument("--no-cpu-baseline", action="store_true")
@@ -113,6 +115,9 @@ def workload(args):
                    f"{args.curvature.upper()} on projected factors, lambda=0.1*mean eig"),
         "topk": args.topk, "l2": "inputs larger than L2 (no flush)",
         **({"mode": "project-only (kernel profiling)"} if args.project_only else {}),
+        **({"query_side": f"second stream beside the train projection, which leaves {args.overlap_sms} SMs free"}
+           if getattr(args, "overlap_sms", 0) > 0 and not args.no_precondition and args.curvature == "fisher"
+           and not args.project_only else {}),
     }
 
 
@@ -647,7 +652,8 @@ def main():
                 train(li, L, route, Phi[:, li * D:], DT)
                 after(li)
             return
-        pipe.run(train, lambda li, L, route, phi, ld: project("query", li, L, route, phi, ld), after, mark)
+        pipe.run(train, lambda li, L, route, phi, ld: project("query", li, L, route, phi, ld), after, mark,
+                 overlap_sms=args.overlap_sms)
         if dist:
             # the exchange step of a sharded job: the global top-k from every rank's top-k
             shard.merge_topk(idx, val, e0, args.topk, dist, world, select)
@@ -724,7 +730,12 @@ def main():
         "ekfac_eigenvalues": ("alu", nl * N * 2 * 2 * Dn * k, alu, "TFLOP/s"),
         "score": ("alu", 2.0 * Nq * N * DT, alu, "TFLOP/s"),
         "topk": ("latency", 8.0 * Nq * N * 4, hbm, "GB/s"),
+        # overlapped query side: what is left of it after the last train projection
+        "query_side_tail": ("latency", nl * 2 * 2 * Dn * Dn * Nq / nl, alu, "TFLOP/s"),
     }
+    if args.overlap_sms > 0 and "project_train" in ph:
+        # the train phase also carries the query projection, fit, factorisation and preconditioning
+        per_unit["project_train"] = ("hbm", per_unit["project_train"][1] + per_unit["project_query"][1], hbm, "GB/s")
     phases = {}
     for name, ms_ in ph.items():
         bound, work, peak, unit = per_unit[name]

@@ -483,6 +483,16 @@ int32_t tda_version(void);
  * devices, all threads). Host only; for counting launches in a timed region. */
 uint64_t tda_launch_count(void);
 
+/* SM budget of the tensor-core factored projection (no counterpart in the
+ * paper, which runs PyTorch ops on one stream). That kernel is persistent,
+ * one CTA per SM; with n_sms > 0 its later launches use at most n_sms CTAs so
+ * that kernels queued on another stream (the query side of a step: the query
+ * projection, the curvature fit, its factorisation and the preconditioning)
+ * find SMs free and run beside it. 0 (the default) = every SM. Process-wide,
+ * host only; results do not depend on it. n_sms < 0 -> TDA_ERR_INVALID_ARG. */
+tda_status tda_set_sm_budget(int32_t n_sms);
+int32_t tda_get_sm_budget(void);
+
 #ifdef __cplusplus
 }
 #endif

@@ -23,6 +23,7 @@ __all__ = [
     "tda_token_scores_workspace_size", "tda_token_scores", "tda_mask_gather", "tda_precondition_state_bytes", "tda_precondition",
     "tda_precondition_info", "tda_score", "tda_score_engine", "tda_similarity_gram_engine", "tda_topk", "tda_route", "tda_route_calibrate",
     "tda_route_set_model", "tda_device_status", "tda_selftest_bounded_wait", "tda_last_error", "tda_version", "tda_launch_count",
+    "tda_set_sm_budget", "tda_get_sm_budget",
 ]
 
 _HERE = os.path.dirname(os.path.abspath(__file__))
@@ -116,6 +117,8 @@ def load() -> ctypes.CDLL:
             "tda_last_error": (ctypes.c_char_p, []),
             "tda_version": (I32, []),
             "tda_launch_count": (U64, []),
+            "tda_set_sm_budget": (I32, [I32]),
+            "tda_get_sm_budget": (I32, []),
         }
         for name, (res, args) in sig.items():
             fn = getattr(lib, name)
@@ -158,6 +161,14 @@ def tda_version() -> int:
 
 def tda_launch_count() -> int:
     return int(load().tda_launch_count())
+
+
+def tda_set_sm_budget(n_sms: int) -> None:
+    _check(load().tda_set_sm_budget(n_sms))
+
+
+def tda_get_sm_budget() -> int:
+    return int(load().tda_get_sm_budget())
 
 
 def tda_proj_entries(seed, layer, side, kind, rows, cols, out, stream=None):

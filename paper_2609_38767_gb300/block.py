@@ -61,12 +61,20 @@ class BlockPipeline:
     def routes(self):
         return [tda.tda_route(L, tda.TDA_OP_PROJECT, self.N, 0, tda.TDA_BF16)[0] for L in self.layers]
 
-    def run(self, project_train, project_query, after_train_linear=None, mark=None):
+    def run(self, project_train, project_query, after_train_linear=None, mark=None, overlap_sms=0):
         """project_train(li, L, route, phi_view, ld) fills train features of linear li;
         project_query likewise for the queries. after_train_linear(li) is called after
         each train projection; mark(name) before each phase and mark(None) at the end
-        (e.g. to record timing events on the stream)."""
+        (e.g. to record timing events on the stream).
+
+        overlap_sms > 0 (Fisher curvature): the query side runs on a second stream
+        beside the train projections, which leave that many SMs free
+        (tda_set_sm_budget): the query projections first, then, as soon as linear
+        l's train features exist, its Fisher fit, factorisation and preconditioning.
+        The arithmetic of every call is unchanged, so are the results."""
         mark = mark or (lambda name: None)
+        if overlap_sms > 0 and self.precondition and self.curvature == "fisher":
+            return self._run_overlapped(project_train, project_query, after_train_linear, mark, overlap_sms)
         routes = self.routes()
         D, DT = self.D, self.DT
         kfac = self.precondition and self.curvature != "fisher"
@@ -107,8 +115,51 @@ class BlockPipeline:
             tda.tda_precondition(tda.TDA_PC_APPLY, nl, D, f32, st, q=self.Q, n_q=self.Nq, ld_q=DT,
                                  qhat=self.Qh, ld_qhat=DT)
             target = self.Qh
+        self._score(target, mark)
+
+    def _score(self, target, mark):
+        DT = self.DT
         mark("score")
         tda.tda_score(target, tda.TDA_F32, self.Nq, DT, self.Phi, self.N, DT, DT, self.S, self.N, 0.0)
         mark("topk")
         tda.tda_topk(self.S, self.Nq, self.N, self.N, self.topk, self.idx, self.val)
         mark(None)
+
+    def _run_overlapped(self, project_train, project_query, after_train_linear, mark, overlap_sms):
+        routes = self.routes()
+        D, DT, f32 = self.D, self.DT, tda.TDA_F32
+        per = tda.tda_precondition_state_bytes(D, f32)
+        main = torch.cuda.current_stream()
+        if getattr(self, "_side", None) is None:
+            self._side = torch.cuda.Stream(device=main.device)
+        side = self._side
+        sms = torch.cuda.get_device_properties(main.device).multi_processor_count
+        side.wait_stream(main)  # inputs written on the main stream
+        with torch.cuda.stream(side):
+            for li, L in enumerate(self.layers):
+                project_query(li, L, routes[li], self.Q[:, li * D:], DT)
+        budget = tda.tda_get_sm_budget()
+        tda.tda_set_sm_budget(max(1, sms - overlap_sms))
+        try:
+            mark("project_train")
+            for li, L in enumerate(self.layers):
+                project_train(li, L, routes[li], self.Phi[:, li * D:], DT)
+                if after_train_linear:
+                    after_train_linear(li)
+                done = torch.cuda.Event()
+                done.record(main)
+                side.wait_event(done)
+                with torch.cuda.stream(side):
+                    st = self.state[li * per:(li + 1) * per]
+                    tda.tda_precondition(tda.TDA_PC_RESET, 1, D, f32, st)
+                    tda.tda_precondition(tda.TDA_PC_FIT_ACCUM, 1, D, f32, st, phi=self.Phi[:, li * D:], n=self.N,
+                                         ld_phi=DT)
+                    tda.tda_precondition(tda.TDA_PC_FACTOR, 1, D, f32, st, n_total=self.N,
+                                         lambda_abs=self.lambda_abs, lambda_rel_mean_eig=self.lambda_rel)
+                    tda.tda_precondition(tda.TDA_PC_APPLY, 1, D, f32, st, q=self.Q[:, li * D:], n_q=self.Nq,
+                                         ld_q=DT, qhat=self.Qh[:, li * D:], ld_qhat=DT)
+        finally:
+            tda.tda_set_sm_budget(budget)
+        mark("query_side_tail")
+        main.wait_stream(side)
+        self._score(self.Qh, mark)

@@ -30,6 +30,9 @@ tda_status cuda_check(cudaError_t e, const char* what) {
 static std::atomic<uint64_t> g_launches{0};
 void note_launches(uint64_t n) { g_launches.fetch_add(n, std::memory_order_relaxed); }
 
+static std::atomic<int> g_sm_budget{0};
+int sm_budget() { return g_sm_budget.load(std::memory_order_relaxed); }
+
 // The device error word: bounded waits that expire OR bits into it.
 __device__ unsigned int g_error_word;
 
@@ -204,6 +207,15 @@ const char* tda_last_error(void) { return g_msg; }
 int32_t tda_version(void) { return 100; }
 
 uint64_t tda_launch_count(void) { return g_launches.load(std::memory_order_relaxed); }
+
+tda_status tda_set_sm_budget(int32_t n_sms) {
+    g_msg[0] = 0;
+    if (n_sms < 0) return fail(TDA_ERR_INVALID_ARG, "tda_set_sm_budget: negative n_sms");
+    g_sm_budget.store(n_sms, std::memory_order_relaxed);
+    return TDA_OK;
+}
+
+int32_t tda_get_sm_budget(void) { return g_sm_budget.load(std::memory_order_relaxed); }
 
 tda_status tda_proj_entries(uint64_t seed, uint32_t layer, int32_t side, int32_t kind, int64_t rows,
                             int32_t cols, int8_t* out, void* stream) {

@@ -438,9 +438,293 @@ apply_kernel(St<TS> st, const float* __restrict__ q, int64_t n_q, int64_t ld_q, 
         for (int64_t i = tid; i < D; i += blockDim.x) out[(g0 + g) * ld_out + (int64_t)l * D + i] = y[g * D + i];
 }
 
+// ---------------------------------------------------------------- FACTOR in one launch (fp32)
+// The same right-looking Cholesky in 32-column steps, with one thread-block
+// cluster of CS CTAs per layer instead of two launches per step: every CTA
+// factors the diagonal block, the CTAs share the panel rows and the trailing
+// 64 x 64 tiles, and cluster barriers separate the phases. M is read through
+// L2 (ld.global.cg): other CTAs of the cluster wrote it. Each step does the
+// arithmetic of prepare/scale/panel/update_kernel in the same order; the
+// factored diagonal blocks are kept in M's diagonal blocks and inverted into
+// Dinv after the last step, one warp per block.
+__device__ __forceinline__ uint32_t cluster_ctarank() {
+    uint32_t r;
+    asm volatile("mov.u32 %0, %%cluster_ctarank;" : "=r"(r));
+    return r;
+}
+__device__ __forceinline__ void cluster_barrier() {
+    __threadfence();
+    asm volatile("barrier.cluster.arrive.release.aligned;\n barrier.cluster.wait.acquire.aligned;" ::: "memory");
+}
+
+// Cholesky of a 32 x 32 block by one warp. Lane i holds row i of the block
+// in registers, shifted so that r[0] is always the column being eliminated:
+// the step loop stays rolled (compact code; every array index is static).
+// Column j of L goes to row j of LkT (LkT[j][i] = L[i][j], zero above the
+// diagonal), 1 / L_jj to dinv[j]. Returns the first non-positive pivot's
+// column or -1.
+__device__ __forceinline__ int warp_cholesky32(const float (*A)[kNB + 1], float (*LkT)[2 * kNB + 1],
+                                               float* dinv, int lane) {
+    float r[kNB];
+#pragma unroll
+    for (int c = 0; c < kNB; ++c) r[c] = A[lane][c];
+    int bad = -1;
+#pragma unroll 1
+    for (int j = 0; j < kNB; ++j) {
+        const float p = __shfl_sync(0xffffffffu, r[0], j);
+        const bool ok = p > 0.f;
+        if (!ok && bad < 0) bad = j;
+        // L_jj = p * rsqrt(p) and 1 / L_jj = rsqrt(p): one special-function op on the
+        // serial path instead of a rounded square root and a division
+        const float inv = ok ? rsqrtf(p) : NAN;
+        const float piv = p * inv;
+        if (lane == j) r[0] = piv;
+        else if (lane > j) r[0] *= inv;
+        LkT[j][lane] = (lane >= j) ? r[0] : 0.f;
+        if (lane == 0) dinv[j] = inv;
+        // A[i][j + idx] -= L[i][j] L[j + idx][j] below the diagonal
+#pragma unroll
+        for (int idx = 1; idx < kNB; ++idx) {
+            const float v = __shfl_sync(0xffffffffu, r[0], (j + idx) & (kNB - 1));
+            if (lane >= j + idx) r[idx] -= r[0] * v;
+        }
+#pragma unroll
+        for (int idx = 0; idx < kNB - 1; ++idx) r[idx] = r[idx + 1];
+        r[kNB - 1] = 0.f;
+    }
+    return bad;
+}
+
+template <int CS>
+__global__ void __launch_bounds__(256, 1) factor_cluster_kernel(St<float> st, int64_t n_total, double lambda_abs,
+                                                              double lambda_rel) {
+    __shared__ float Lk[kNB][kNB + 1];        // the diagonal block before factoring
+    __shared__ float LkT[kNB][2 * kNB + 1];   // L transposed; columns 32..63 stay zero
+    __shared__ float dinv[kNB];               // 1 / L_jj of the current block
+    __shared__ double part[256];
+    constexpr int T = 64;
+    __shared__ __align__(16) float Pi[kNB][T + 4];  // 16-byte rows: the products read float4
+    __shared__ __align__(16) float Pj[kNB][T + 4];
+    const int rank = (int)cluster_ctarank();
+    const int l = blockIdx.x / CS;
+    const int64_t D = st.D;
+    float* M = st.M(l);
+    double* h = st.header(l);
+    const int tid = threadIdx.x, lane = tid & 31, ty = tid / 16, tx = tid % 16;
+    for (int e = tid; e < kNB * (2 * kNB + 1); e += blockDim.x) (&LkT[0][0])[e] = 0.f;
+    // damping from the mean eigenvalue tr(M)/(n_total D), summed like prepare_kernel
+    double s = 0.0;
+    for (int64_t a = tid; a < D; a += blockDim.x) s += (double)__ldcg(M + a * D + a);
+    part[tid] = s;
+    __syncthreads();
+    for (int w = blockDim.x / 2; w > 0; w >>= 1) {
+        if (tid < w) part[tid] += part[tid + w];
+        __syncthreads();
+    }
+    const double mean_eig = part[0] / (double)n_total / (double)D;
+    const double lambda = lambda_abs + lambda_rel * mean_eig;
+    if (rank == 0 && tid == 0) {
+        h[kPcLambda] = lambda;
+        h[kPcMeanEig] = mean_eig;
+        h[kPcFailedPivot] = 0.0;
+        h[kPcNTotal] = (double)n_total;
+    }
+    cluster_barrier();  // every CTA has read the diagonal before it is scaled
+    {
+        const float inv_n = (float)(1.0 / (double)n_total), lam = (float)lambda;
+        for (int64_t i = rank; i < D; i += CS)
+            for (int64_t j = tid; j <= i; j += blockDim.x) {
+                float v = __ldcg(M + i * D + j) * inv_n;
+                if (i == j) v += lam;
+                M[i * D + j] = v;
+            }
+    }
+    cluster_barrier();
+    for (int64_t k0 = 0; k0 < D; k0 += kNB) {
+        // ---- diagonal block: factored in registers by warp 0 of every CTA
+        for (int e = tid; e < kNB * kNB; e += blockDim.x) {
+            const int i = e / kNB, j = e % kNB;
+            Lk[i][j] = (j <= i) ? __ldcg(M + (k0 + i) * D + k0 + j) : 0.f;
+        }
+        __syncthreads();
+        if (tid < 32) {
+            const int bad = warp_cholesky32(Lk, LkT, dinv, lane);
+            if (rank == 0 && lane == 0 && bad >= 0 && h[kPcFailedPivot] == 0.0) h[kPcFailedPivot] = (double)(k0 + bad + 1);
+        }
+        __syncthreads();
+        // ---- panel rows below the block: x L_kk^T = a, every CS-th row to each CTA of the
+        // cluster. Column order with the same register shift: once x_j is known it leaves
+        // every later entry
+        for (int64_t i = k0 + kNB + (int64_t)tid * CS + rank; i < D; i += (int64_t)CS * blockDim.x) {
+            float x[kNB];
+#pragma unroll
+            for (int j = 0; j < kNB; ++j) x[j] = __ldcg(M + i * D + k0 + j);
+            float* out = M + i * D + k0;
+#pragma unroll 1
+            for (int j = 0; j < kNB; ++j) {
+                const float xj = x[0] * dinv[j];
+                out[j] = xj;
+#pragma unroll
+                for (int idx = 1; idx < kNB; ++idx) x[idx] -= xj * LkT[j][j + idx];
+#pragma unroll
+                for (int idx = 0; idx < kNB - 1; ++idx) x[idx] = x[idx + 1];
+                x[kNB - 1] = 0.f;
+            }
+        }
+        cluster_barrier();
+        // the factored block goes back into M's diagonal block once every CTA has read the
+        // unfactored one (no later step reads that block); the inverses of all diagonal
+        // blocks are formed after the last step
+        if (rank == 0)
+            for (int e = tid; e < kNB * kNB; e += blockDim.x) {
+                const int i = e / kNB, j = e % kNB;
+                if (j <= i) M[(k0 + i) * D + k0 + j] = LkT[j][i];
+            }
+        // ---- trailing update of the lower triangle, 64 x 64 tiles shared by the cluster
+        const int64_t s0 = k0 + kNB;
+        const int64_t rest = D - s0;
+        if (rest > 0) {
+            const int64_t t = (rest + T - 1) / T, tiles = t * (t + 1) / 2;
+            // tile u -> (bi, bj), bj <= bi, row-major over the lower triangle of tiles
+            auto tile_of = [&](int64_t u, int64_t& i0, int64_t& j0) {
+                // fp32 estimate (fp64 is a slow pipe here), corrected in integers
+                int64_t bi = (int64_t)((sqrtf(8.f * (float)u + 1.f) - 1.f) * 0.5f);
+                while (bi * (bi + 1) / 2 > u) --bi;
+                while ((bi + 1) * (bi + 2) / 2 <= u) ++bi;
+                i0 = s0 + bi * T;
+                j0 = s0 + (u - bi * (bi + 1) / 2) * T;
+            };
+            // software pipeline: while tile u is multiplied, the panel rows and the current
+            // values of this CTA's next tile are on their way (each thread: 8 + 8 panel values,
+            // row e/32, column e%32, and its 4 x 4 outputs)
+            float ra[8], rb[8], mv[4][4];
+            auto load_tile = [&](int64_t u) {
+                int64_t i0, j0;
+                tile_of(u, i0, j0);
+#pragma unroll
+                for (int h = 0; h < 8; ++h) {
+                    const int e = tid + h * 256, r = e / kNB, m = e % kNB;
+                    ra[h] = (i0 + r < D) ? __ldcg(M + (i0 + r) * D + k0 + m) : 0.f;
+                    rb[h] = (j0 + r < D) ? __ldcg(M + (j0 + r) * D + k0 + m) : 0.f;
+                }
+#pragma unroll
+                for (int q = 0; q < 4; ++q)
+#pragma unroll
+                    for (int v = 0; v < 4; ++v) {
+                        const int64_t i = i0 + ty * 4 + q, j = j0 + tx * 4 + v;
+                        mv[q][v] = (i < D && j < D && j <= i) ? __ldcg(M + i * D + j) : 0.f;
+                    }
+            };
+            int64_t u = rank;
+            if (u < tiles) load_tile(u);
+            for (; u < tiles; u += CS) {
+                int64_t i0, j0;
+                tile_of(u, i0, j0);
+#pragma unroll
+                for (int h = 0; h < 8; ++h) {
+                    const int e = tid + h * 256, r = e / kNB, m = e % kNB;
+                    Pi[m][r] = ra[h];
+                    Pj[m][r] = rb[h];
+                }
+                float acc[4][4];
+#pragma unroll
+                for (int a = 0; a < 4; ++a)
+#pragma unroll
+                    for (int b = 0; b < 4; ++b) acc[a][b] = mv[a][b];
+                __syncthreads();
+                if (u + CS < tiles) load_tile(u + CS);
+#pragma unroll 8
+                for (int m = 0; m < kNB; ++m) {
+                    const float4 a4 = *reinterpret_cast<const float4*>(&Pi[m][ty * 4]);
+                    const float4 b4 = *reinterpret_cast<const float4*>(&Pj[m][tx * 4]);
+                    const float a[4] = {a4.x, a4.y, a4.z, a4.w}, b[4] = {b4.x, b4.y, b4.z, b4.w};
+#pragma unroll
+                    for (int q = 0; q < 4; ++q)
+#pragma unroll
+                        for (int v = 0; v < 4; ++v) acc[q][v] -= a[q] * b[v];
+                }
+#pragma unroll
+                for (int q = 0; q < 4; ++q)
+#pragma unroll
+                    for (int v = 0; v < 4; ++v) {
+                        const int64_t i = i0 + ty * 4 + q, j = j0 + tx * 4 + v;
+                        if (i < D && j < D && j <= i) M[i * D + j] = acc[q][v];
+                    }
+                __syncthreads();
+            }
+        }
+        cluster_barrier();
+    }
+    // inverses of the factored diagonal blocks: a CTA stages a block in shared
+    // memory and lane c of warp 0 solves L X[:, c] = e_c in column order
+    const int nblk = (int)(D / kNB);
+    for (int b = rank; b < nblk; b += CS) {
+        const float* Lb = M + (int64_t)b * kNB * D + (int64_t)b * kNB;
+        for (int e = tid; e < kNB * kNB; e += blockDim.x) {
+            const int i = e / kNB, j = e % kNB;
+            Lk[i][j] = (j <= i) ? __ldcg(Lb + (int64_t)i * D + j) : 0.f;
+        }
+        __syncthreads();
+        if (tid < kNB) {
+            const int c = lane;
+            float x[kNB];
+#pragma unroll
+            for (int i = 0; i < kNB; ++i) x[i] = (i == c) ? 1.f : 0.f;
+#pragma unroll
+            for (int j = 0; j < kNB; ++j) {
+                x[j] = (j < c) ? 0.f : x[j] / Lk[j][j];
+#pragma unroll
+                for (int i = j + 1; i < kNB; ++i) x[i] -= Lk[i][j] * x[j];
+            }
+            float* Di = st.Dinv(l) + (int64_t)b * (kNB * kNB);
+#pragma unroll
+            for (int i = 0; i < kNB; ++i) Di[i * kNB + c] = x[i];
+        }
+        __syncthreads();
+    }
+}
+
+template <int CS>
+cudaError_t factor_cluster(int n_layers, int64_t D, void* state, int64_t n_total, double la, double lr,
+                           cudaStream_t s) {
+    cudaError_t e = cudaSuccess;
+    if (CS > 8) e = cudaFuncSetAttribute(factor_cluster_kernel<CS>, cudaFuncAttributeNonPortableClusterSizeAllowed, 1);
+    if (e != cudaSuccess) return e;
+    cudaLaunchConfig_t cfg = {};
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeClusterDimension;
+    attr[0].val.clusterDim.x = CS;
+    attr[0].val.clusterDim.y = 1;
+    attr[0].val.clusterDim.z = 1;
+    cfg.gridDim = dim3((unsigned)(n_layers * CS));
+    cfg.blockDim = dim3(256);
+    cfg.dynamicSmemBytes = 0;
+    cfg.stream = s;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    int max_clusters = 0;
+    if (cudaOccupancyMaxActiveClusters(&max_clusters, factor_cluster_kernel<CS>, &cfg) != cudaSuccess ||
+        max_clusters < 1) {
+        cudaGetLastError();
+        return cudaErrorNotSupported;
+    }
+    note_launches(1);
+    e = cudaLaunchKernelEx(&cfg, factor_cluster_kernel<CS>, state_of<float>(state, D), n_total, la, lr);
+    if (e != cudaSuccess) return e;
+    return cudaGetLastError();
+}
+
 template <typename TS>
 cudaError_t factor_impl(int n_layers, int64_t D, void* state, int64_t n_total, double la, double lr,
                         cudaStream_t s) {
+    if constexpr (sizeof(TS) == 4) {
+        // fp32 state, whole 32-column blocks: one launch, a cluster of 16 (else 8) CTAs per layer
+        if (D % kNB == 0 && D >= 2 * kNB) {
+            cudaError_t e = factor_cluster<16>(n_layers, D, state, n_total, la, lr, s);
+            if (e == cudaErrorNotSupported) e = factor_cluster<8>(n_layers, D, state, n_total, la, lr, s);
+            if (e != cudaErrorNotSupported) return e;
+        }
+    }
     St<TS> st = state_of<TS>(state, D);
     note_launches(2);
     prepare_kernel<TS><<<n_layers, 256, 0, s>>>(st, n_total, la, lr);

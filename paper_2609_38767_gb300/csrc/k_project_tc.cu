@@ -587,7 +587,7 @@ bool device_is_sm103() {
     return major == 10 && minor == 3;
 }
 
-int sm_count() {
+int device_sms() {
     static int sms = 0;
     if (!sms) {
         int dev = 0, n = 0;
@@ -596,6 +596,12 @@ int sm_count() {
         sms = n > 0 ? n : 1;
     }
     return sms;
+}
+
+// SMs this launch may fill: all of them, or the tda_set_sm_budget cap
+int sm_count() {
+    const int sms = device_sms(), b = sm_budget();
+    return (b > 0 && b < sms) ? b : sms;
 }
 
 template <int K, int G, bool KF, bool FO>
@@ -654,6 +660,7 @@ cudaError_t launch_kg(const tda_layer_desc& L, const void* A, const void* B, int
     if (cudaOccupancyMaxActiveClusters(&max_clusters, project_tc_kernel<K, G, KF, FO>, &cfg) != cudaSuccess ||
         max_clusters < 1)
         max_clusters = sms / cs;
+    if (max_clusters > sms / cs) max_clusters = sms / cs;  // the SM budget (the occupancy query sees every SM)
     int64_t clusters = FO ? p.n_slots * p.n_ttiles : p.n_slots;
     if (clusters > max_clusters) clusters = max_clusters;
     cfg.gridDim = dim3((unsigned)(clusters * cs));
@@ -737,7 +744,7 @@ cudaError_t launch_project_tc_kfac(const tda_layer_desc& L, const void* A, const
     }
 }
 
-int project_tc_max_grid() { return sm_count(); }
+int project_tc_max_grid() { return device_sms(); }
 
 // Projected factors of N examples (At rows then Bt rows, [N*T][k] each, fp32,
 // unscaled signs) by the tensor-core kernel.

@@ -49,6 +49,8 @@ float projection_scale(const tda_layer_desc& L);
 
 // Host-side count of kernels this library has launched (tda_launch_count).
 void note_launches(uint64_t n);
+// tda_set_sm_budget's cap on the persistent projection grid (0 = none).
+int sm_budget();
 
 // Device address of the library's error word on the current device.
 unsigned int* device_error_word();

@@ -169,3 +169,14 @@ def test_kfac_state_and_validation(libs):
         == tda.TDA_ERR_WORKSPACE
     assert _err(tda.tda_project_kfac, L, tda.TDA_F32, 16, 16, 4, 16, 256, 256, 256, 1 << 24, stream=s) \
         == tda.TDA_ERR_UNSUPPORTED
+
+
+def test_sm_budget_is_host_state(libs):
+    # the projection's SM cap is plain host state: set, read back, reset; negative rejected
+    assert tda.tda_get_sm_budget() == 0
+    tda.tda_set_sm_budget(100)
+    assert tda.tda_get_sm_budget() == 100
+    assert _err(tda.tda_set_sm_budget, -1) == tda.TDA_ERR_INVALID_ARG
+    assert tda.tda_get_sm_budget() == 100
+    tda.tda_set_sm_budget(0)
+    assert tda.tda_get_sm_budget() == 0

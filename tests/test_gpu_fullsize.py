@@ -183,3 +183,27 @@ def test_route_sweep_linear_exact_similarity(dev, orc, T):
         tda.tda_similarity_exact(L, tda.TDA_BF16, to(Aq), to(Bq), nq, to(At), to(Bt), nt, S, nt, 0.0, route, ws, wsb)
         tda.tda_device_status()
         assert rel_fro(S.cpu().numpy(), ref) <= TOL, route
+
+
+def test_overlapped_query_side_matches_serial(dev):
+    # the query side on a second stream beside an SM-capped train projection: same calls,
+    # same arithmetic, so the features, preconditioned queries, scores and top-k are bit-identical
+    linears, T, k, N, Nq = LLAMA1B, 256, 32, 1024, 16
+    sb = math.sqrt(1e-3)
+    At, Bt, Aq, Bq = [], [], [], []
+    for li, (di, do) in enumerate(linears):
+        At.append(fill(N, T, di, synth.SEED_A, li, 1.0, 0, 0.01, 0, dev))
+        Bt.append(fill(N, T, do, synth.SEED_B, li, sb, 0, 0.01, 0, dev))
+        Aq.append(fill(Nq, T, di, synth.SEED_A, li + synth.QUERY_STREAM_OFFSET, 1.0, 0, 0.01, 1000, dev))
+        Bq.append(fill(Nq, T, do, synth.SEED_B, li + synth.QUERY_STREAM_OFFSET, sb, 0, 0.01, 1000, dev))
+    out = []
+    for overlap in (0, 24):
+        pipe = BlockPipeline(linears, T, k, N, Nq, topk=50, precondition=True, lambda_rel=1e-2, device=dev)
+        pipe.run(lambda li, L, r, phi, ld: tda.tda_project(L, tda.TDA_BF16, At[li], Bt[li], N, phi, ld, r),
+                 lambda li, L, r, phi, ld: tda.tda_project(L, tda.TDA_BF16, Aq[li], Bq[li], Nq, phi, ld, r),
+                 overlap_sms=overlap)
+        tda.tda_device_status()
+        out.append([x.cpu().numpy() for x in (pipe.Phi, pipe.Q, pipe.Qh, pipe.S, pipe.idx, pipe.val)])
+        assert tda.tda_get_sm_budget() == 0
+    for a, b in zip(*out):
+        np.testing.assert_array_equal(a, b)

@@ -196,8 +196,8 @@ def test_preconditioned_scores_bf16_fp32_state_relative_damping(dev, orc):
     assert rel_fro(S, Sref) <= 2e-2
 
 
-def test_precondition_not_spd_is_reported(dev):
-    D = 8
+@pytest.mark.parametrize("D", [8, 64, 96])  # 64, 96: the one-launch cluster factorisation
+def test_precondition_not_spd_is_reported(dev, D):
     state = torch.empty(tda.tda_precondition_state_bytes(D, tda.TDA_F32), dtype=torch.uint8, device=dev)
     tda.tda_precondition(tda.TDA_PC_RESET, 1, D, tda.TDA_F32, state)
     phi = torch.ones((2, D), device=dev)
@@ -331,7 +331,8 @@ def test_tc_projection_matches_oracle(dev, orc, case):
 
 @pytest.mark.parametrize("sdt,D,lam_abs,lam_rel,tol", [(tda.TDA_F64, 70, 1e-3, 0.0, 1e-9),
                                                        (tda.TDA_F32, 96, 0.0, 1e-2, 1e-4),
-                                                       (tda.TDA_F32, 1000, 0.0, 1e-2, 1e-3)])
+                                                       (tda.TDA_F32, 1000, 0.0, 1e-2, 1e-3),
+                                                       (tda.TDA_F32, 1024, 0.0, 1e-2, 1e-3)])
 def test_precondition_batched_layers_match_oracle(dev, orc, sdt, D, lam_abs, lam_rel, tol):
     # three layers side by side in each feature row, ragged D, streamed in two chunks
     rng = np.random.default_rng(D)
