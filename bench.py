@@ -653,7 +653,7 @@ def main():
                 after(li)
             return
         pipe.run(train, lambda li, L, route, phi, ld: project("query", li, L, route, phi, ld), after, mark,
-                 overlap_sms=args.overlap_sms)
+                 overlap_sms=args.overlap_sms, dist=dist)
         if dist:
             # the exchange step of a sharded job: the global top-k from every rank's top-k
             shard.merge_topk(idx, val, e0, args.topk, dist, world, select)
@@ -730,6 +730,8 @@ def main():
         "ekfac_eigenvalues": ("alu", nl * N * 2 * 2 * Dn * k, alu, "TFLOP/s"),
         "score": ("alu", 2.0 * Nq * N * DT, alu, "TFLOP/s"),
         "topk": ("latency", 8.0 * Nq * N * 4, hbm, "GB/s"),
+        # sharded job: the curvature sums added over the ranks (NCCL all-reduce)
+        "curvature_allreduce": ("latency", (nl * D * D * 4) if not kfac_mode else (nl * 2 * k * k * 8), hbm, "GB/s"),
         # overlapped query side: what is left of it after the last train projection
         "query_side_tail": ("latency", nl * 2 * 2 * Dn * Dn * Nq / nl, alu, "TFLOP/s"),
     }
@@ -833,7 +835,7 @@ def main():
             "warmup": args.warmup, "ms_per_step": ms, "higher_is_better": True, "scaling": "weak",
             "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
             "config": {**workload(args), "parallelism": f"train examples sharded over {world} rank(s)"
-                       + (", global top-k merged by all-gather" if world > 1 else ""),
+                       + (", curvature sums all-reduced, global top-k merged by all-gather" if world > 1 else ""),
                        "routes": {name: {0: "factored", 1: "materialize", 2: "gram"}[r] for (name, _, _), r
                                   in zip(LINEARS, pipe.routes())}},
             "roofline": roofline, "phases": phases, "cpu_baseline": cpu, "e2e": e2e, "gpu_launches": launches,

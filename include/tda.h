@@ -263,7 +263,10 @@ tda_status tda_cosine(float* S, int64_t n_q, int64_t n_t, int64_t ld_S, const fl
  * `state` is a device buffer of n_layers * tda_precondition_state_bytes(D,
  * state_dtype) bytes, 16-byte aligned: per layer a 64-byte header, the D x D
  * matrix M and the inverses of M's 32 x 32 diagonal blocks, all in
- * state_dtype (TDA_F32 or TDA_F64). The ops, in order of use:
+ * state_dtype (TDA_F32 or TDA_F64). A job whose training features are sharded
+ * over ranks adds the layers' M (bytes [64, 64 + D*D*sizeof) of each layer's
+ * state) over the ranks (an all-reduce) between FIT_ACCUM and FACTOR, and
+ * passes the global n_total to FACTOR. The ops, in order of use:
  *   TDA_PC_RESET      zero the state.
  *   TDA_PC_FIT_ACCUM  M_l += Phi_l^T Phi_l over n feature rows. Call once per
  *                     streamed chunk of training features.
@@ -317,7 +320,12 @@ tda_status tda_precondition_info(int32_t n_layers, int64_t D, tda_dtype state_dt
  * `state`: device buffer of n_layers * tda_kfac_state_bytes(k_in, k_out) bytes
  * (layer l at byte l * tda_kfac_state_bytes), 16-byte aligned, fp64 per layer:
  * an 8-double header (M, N, Jacobi sweeps), the factor sums, the eigenbases and
- * eigenvalues, the EK-FAC sums. The n_layers calls (reset, eigen,
+ * eigenvalues, the EK-FAC sums. The sums, in doubles from the layer's start
+ * (ka = k_in, kg = k_out): [0] M; [8, 8 + ka^2) sum a~a~^T; [8 + ka^2,
+ * 8 + ka^2 + kg^2) sum g~g~^T; [1] N and [Le, Le + ka*kg) the EK-FAC sums, with
+ * Le = 8 + 2 ka^2 + 2 kg^2 + ka + kg. A job whose training examples are
+ * sharded over ranks adds these ranges over the ranks (an all-reduce) before
+ * tda_kfac_eigen, respectively before tda_kfac_apply for EK-FAC. The n_layers calls (reset, eigen,
  * accumulate_eigenvalues, apply) treat that many layers of equal k_in, k_out in
  * one launch, their features side by side in each row (layer l at column
  * l*k_in*k_out, as tda_precondition); accumulate_factors and project_kfac take

@@ -20,6 +20,7 @@ from __future__ import annotations
 import torch
 
 import paper_2609_38767_gb300 as tda
+from paper_2609_38767_gb300 import shard
 
 
 class BlockPipeline:
@@ -61,7 +62,7 @@ class BlockPipeline:
     def routes(self):
         return [tda.tda_route(L, tda.TDA_OP_PROJECT, self.N, 0, tda.TDA_BF16)[0] for L in self.layers]
 
-    def run(self, project_train, project_query, after_train_linear=None, mark=None, overlap_sms=0):
+    def run(self, project_train, project_query, after_train_linear=None, mark=None, overlap_sms=0, dist=None):
         """project_train(li, L, route, phi_view, ld) fills train features of linear li;
         project_query likewise for the queries. after_train_linear(li) is called after
         each train projection; mark(name) before each phase and mark(None) at the end
@@ -71,9 +72,14 @@ class BlockPipeline:
         beside the train projections, which leave that many SMs free
         (tda_set_sm_budget): the query projections first, then, as soon as linear
         l's train features exist, its Fisher fit, factorisation and preconditioning.
-        The arithmetic of every call is unchanged, so are the results."""
+        The arithmetic of every call is unchanged, so are the results.
+
+        dist (torch.distributed, train examples sharded over its ranks): the curvature is
+        fitted over all shards -- the sums are all-reduced before the factorisation and
+        every rank preconditions its queries with the same global curvature."""
         mark = mark or (lambda name: None)
-        if overlap_sms > 0 and self.precondition and self.curvature == "fisher":
+        world = dist.get_world_size() if dist is not None else 1
+        if overlap_sms > 0 and self.precondition and self.curvature == "fisher" and world == 1:
             return self._run_overlapped(project_train, project_query, after_train_linear, mark, overlap_sms)
         routes = self.routes()
         D, DT = self.D, self.DT
@@ -92,12 +98,17 @@ class BlockPipeline:
         if kfac:
             k = self.k
             nl, sts = self.nl, self.kf_states
+            if world > 1:
+                mark("curvature_allreduce")
+                shard.allreduce_kfac(sts, nl, k, k, self.kf_per, dist, world)
             mark("kfac_eigen")
             tda.tda_kfac_eigen(k, k, sts, n_layers=nl)
             if self.curvature == "ekfac":
                 mark("ekfac_eigenvalues")
                 tda.tda_kfac_accumulate_eigenvalues(k, k, sts, self.Phi, self.N, DT, self.kf_ws, self.kf_wsb,
                                                     n_layers=nl)
+                if world > 1:
+                    shard.allreduce_kfac(sts, nl, k, k, self.kf_per, dist, world, eigenvalue_sums=True)
             mark("apply")
             kind = tda.TDA_EKFAC if self.curvature == "ekfac" else tda.TDA_KFAC
             tda.tda_kfac_apply(kind, k, k, sts, self.lambda_abs, self.lambda_rel, self.Q, self.Nq, DT, self.Qh, DT,
@@ -108,9 +119,12 @@ class BlockPipeline:
             mark("fisher_fit")
             tda.tda_precondition(tda.TDA_PC_RESET, nl, D, f32, st)
             tda.tda_precondition(tda.TDA_PC_FIT_ACCUM, nl, D, f32, st, phi=self.Phi, n=self.N, ld_phi=DT)
+            if world > 1:
+                mark("curvature_allreduce")
+                shard.allreduce_fisher(st, nl, D, tda.tda_precondition_state_bytes(D, f32), 4, dist, world)
             mark("factor")
-            tda.tda_precondition(tda.TDA_PC_FACTOR, nl, D, f32, st, n_total=self.N, lambda_abs=self.lambda_abs,
-                                 lambda_rel_mean_eig=self.lambda_rel)
+            tda.tda_precondition(tda.TDA_PC_FACTOR, nl, D, f32, st, n_total=self.N * world,
+                                 lambda_abs=self.lambda_abs, lambda_rel_mean_eig=self.lambda_rel)
             mark("apply")
             tda.tda_precondition(tda.TDA_PC_APPLY, nl, D, f32, st, q=self.Q, n_q=self.Nq, ld_q=DT,
                                  qhat=self.Qh, ld_qhat=DT)

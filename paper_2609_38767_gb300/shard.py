@@ -3,9 +3,11 @@
 Train examples are independent in every step of the path, so a job splits them
 into contiguous shards, one per rank: rank r owns global examples
 [r * n_local, (r + 1) * n_local). The queries (and, once solved, the
-preconditioned queries) are replicated. Scores and top-k are computed per shard;
-the one exchange step is the merge of the per-rank top-k candidates into the
-global top-k: an all-gather of n_q x k (index, score) pairs per rank, then a
+preconditioned queries) are replicated. Scores and top-k are computed per shard.
+Two steps exchange data: the curvature fit over the training set (each rank's
+sums are all-reduced before the factorisation, so every rank preconditions with
+the same global curvature), and the merge of the per-rank top-k candidates into
+the global top-k: an all-gather of n_q x k (index, score) pairs per rank, then a
 top-k over the n_q x (world * k) candidates.
 
 Ties: candidates are laid out rank-major and, within a rank, in the local
@@ -59,3 +61,39 @@ def device_select(tda):
         tda.tda_topk(cand_val, n_q, n_c, n_c, k, pos, top)
         return pos, top
     return select
+
+
+# ---------------------------------------------------------------- curvature fit over all shards
+# The fit over the training set is the path's other exchange step: every rank
+# accumulates its shard's sums, an all-reduce adds them, and every rank then
+# factorises the same global curvature (the layouts are those tda.h documents).
+
+def allreduce_fisher(state, n_layers: int, D: int, state_bytes: int, itemsize: int, dist, world: int) -> None:
+    """Add the Fisher sums M of every layer over the ranks (between FIT_ACCUM and FACTOR).
+    state: uint8 tensor of n_layers * state_bytes; itemsize 4 (F32 state) or 8 (F64)."""
+    if world == 1:
+        return
+    dt = {4: torch.float32, 8: torch.float64}[itemsize]
+    for l in range(n_layers):
+        m = state[l * state_bytes + 64:l * state_bytes + 64 + D * D * itemsize].view(dt)
+        dist.all_reduce(m)
+
+
+def kfac_sum_ranges(k_in: int, k_out: int):
+    """Double-index ranges of one layer's K-FAC state that hold sums: (factor sums, EK-FAC sums)."""
+    ka, kg = k_in, k_out
+    le = 8 + 2 * ka * ka + 2 * kg * kg + ka + kg
+    return [(0, 1), (8, 8 + ka * ka + kg * kg)], [(1, 2), (le, le + ka * kg)]
+
+
+def allreduce_kfac(states, n_layers: int, k_in: int, k_out: int, state_bytes: int, dist, world: int,
+                   eigenvalue_sums: bool = False) -> None:
+    """Add the K-FAC factor sums (before tda_kfac_eigen) or, with eigenvalue_sums, the EK-FAC
+    eigenvalue sums (before tda_kfac_apply) of every layer over the ranks."""
+    if world == 1:
+        return
+    factor, ekfac = kfac_sum_ranges(k_in, k_out)
+    for l in range(n_layers):
+        st = states[l * state_bytes:(l + 1) * state_bytes].view(torch.float64)
+        for a, b in (ekfac if eigenvalue_sums else factor):
+            dist.all_reduce(st[a:b])
