@@ -726,6 +726,7 @@ def main():
         "fisher_fit": ("alu", nl * N * Dn * (Dn + 1), alu, "TFLOP/s"),
         "factor": ("latency", nl * Dn ** 3 / 3, alu, "TFLOP/s"),
         "apply": ("latency", (nl * 4 * 2 * Dn * k * Nq) if kfac_mode else (nl * 2 * 2 * Dn * Dn * Nq), alu, "TFLOP/s"),
+        "factor_apply": ("latency", nl * (Dn ** 3 / 3 + 2 * 2 * Dn * Dn * Nq), alu, "TFLOP/s"),
         "kfac_eigen": ("latency", nl * 2 * 10 * 4.0 * k ** 3, alu, "TFLOP/s"),
         "ekfac_eigenvalues": ("alu", nl * N * 2 * 2 * Dn * k, alu, "TFLOP/s"),
         "score": ("alu", 2.0 * Nq * N * DT, alu, "TFLOP/s"),

@@ -279,12 +279,19 @@ tda_status tda_cosine(float* S, int64_t n_q, int64_t n_t, int64_t ld_S, const fl
  *                     (q fp32; qhat in state_dtype, i.e. fp64 rows for an F64
  *                     state). Layers whose FACTOR failed get NaN rows.
  *                     Needs D <= 40960 (F32) or 20480 (F64).
+ *   TDA_PC_FACTOR_APPLY  FACTOR, then APPLY, in one call (same arguments and
+ *                     results as the two; a failed layer's rows are NaN). For an
+ *                     F32 state with D a multiple of 32 and n_q <= 256 both run
+ *                     in one launch: the query rows are solved alongside the
+ *                     factorisation (forward substitution as extra rows of each
+ *                     step) and then backward. qhat may not alias q.
  * Arguments not used by an op are ignored (may be 0/NULL).
  * ------------------------------------------------------------------------- */
 #define TDA_PC_RESET 0
 #define TDA_PC_FIT_ACCUM 1
 #define TDA_PC_FACTOR 2
 #define TDA_PC_APPLY 3
+#define TDA_PC_FACTOR_APPLY 4
 
 /* Bytes of ONE layer's state (a multiple of 256). */
 size_t tda_precondition_state_bytes(int64_t D, tda_dtype state_dtype);

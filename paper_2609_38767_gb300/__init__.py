@@ -38,7 +38,7 @@ TDA_PROJ_RADEMACHER, TDA_PROJ_IDENTITY = 0, 1
 TDA_ROUTE_AUTO, TDA_ROUTE_FACTORED, TDA_ROUTE_MATERIALIZE, TDA_ROUTE_GRAM = -1, 0, 1, 2
 TDA_OP_PROJECT, TDA_OP_SIMILARITY_PROJECTED, TDA_OP_SIMILARITY_EXACT = 0, 1, 2
 TDA_OP_NORM_PROJECTED, TDA_OP_NORM_EXACT = 3, 4
-TDA_PC_RESET, TDA_PC_FIT_ACCUM, TDA_PC_FACTOR, TDA_PC_APPLY = 0, 1, 2, 3
+TDA_PC_RESET, TDA_PC_FIT_ACCUM, TDA_PC_FACTOR, TDA_PC_APPLY, TDA_PC_FACTOR_APPLY = 0, 1, 2, 3, 4
 TDA_KFAC, TDA_EKFAC = 0, 1
 TDA_CALIBRATE_WS_BYTES = 768 << 20
 _STATUS = {0: "TDA_OK", 1: "TDA_ERR_INVALID_ARG", 2: "TDA_ERR_UNSUPPORTED", 3: "TDA_ERR_WORKSPACE",

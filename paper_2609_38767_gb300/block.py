@@ -122,12 +122,10 @@ class BlockPipeline:
             if world > 1:
                 mark("curvature_allreduce")
                 shard.allreduce_fisher(st, nl, D, tda.tda_precondition_state_bytes(D, f32), 4, dist, world)
-            mark("factor")
-            tda.tda_precondition(tda.TDA_PC_FACTOR, nl, D, f32, st, n_total=self.N * world,
-                                 lambda_abs=self.lambda_abs, lambda_rel_mean_eig=self.lambda_rel)
-            mark("apply")
-            tda.tda_precondition(tda.TDA_PC_APPLY, nl, D, f32, st, q=self.Q, n_q=self.Nq, ld_q=DT,
-                                 qhat=self.Qh, ld_qhat=DT)
+            mark("factor_apply")
+            tda.tda_precondition(tda.TDA_PC_FACTOR_APPLY, nl, D, f32, st, n_total=self.N * world,
+                                 lambda_abs=self.lambda_abs, lambda_rel_mean_eig=self.lambda_rel,
+                                 q=self.Q, n_q=self.Nq, ld_q=DT, qhat=self.Qh, ld_qhat=DT)
             target = self.Qh
         self._score(target, mark)
 
@@ -168,10 +166,10 @@ class BlockPipeline:
                     tda.tda_precondition(tda.TDA_PC_RESET, 1, D, f32, st)
                     tda.tda_precondition(tda.TDA_PC_FIT_ACCUM, 1, D, f32, st, phi=self.Phi[:, li * D:], n=self.N,
                                          ld_phi=DT)
-                    tda.tda_precondition(tda.TDA_PC_FACTOR, 1, D, f32, st, n_total=self.N,
-                                         lambda_abs=self.lambda_abs, lambda_rel_mean_eig=self.lambda_rel)
-                    tda.tda_precondition(tda.TDA_PC_APPLY, 1, D, f32, st, q=self.Q[:, li * D:], n_q=self.Nq,
-                                         ld_q=DT, qhat=self.Qh[:, li * D:], ld_qhat=DT)
+                    tda.tda_precondition(tda.TDA_PC_FACTOR_APPLY, 1, D, f32, st, n_total=self.N,
+                                         lambda_abs=self.lambda_abs, lambda_rel_mean_eig=self.lambda_rel,
+                                         q=self.Q[:, li * D:], n_q=self.Nq, ld_q=DT, qhat=self.Qh[:, li * D:],
+                                         ld_qhat=DT)
         finally:
             tda.tda_set_sm_budget(budget)
         mark("query_side_tail")

@@ -852,6 +852,25 @@ tda_status tda_precondition(int32_t op, int32_t n_layers, int64_t D, tda_dtype s
             return cuda_check(launch_pc_factor(n_layers, D, state_dtype, state, n_total, lambda_abs,
                                                lambda_rel_mean_eig, s),
                               "factor");
+        case TDA_PC_FACTOR_APPLY: {
+            if (n_total < 1) return fail(TDA_ERR_INVALID_ARG, "n_total must be >= 1");
+            if (!(lambda_abs >= 0) || !(lambda_rel_mean_eig >= 0) ||
+                !(lambda_abs > 0 || lambda_rel_mean_eig > 0))
+                return fail(TDA_ERR_INVALID_ARG, "damping must be >= 0 and not both zero");
+            if (n_q < 0) return fail(TDA_ERR_INVALID_ARG, "negative n_q");
+            if (n_q > 0 && (!q || !qhat)) return fail(TDA_ERR_INVALID_ARG, "q/qhat is NULL");
+            if (ld_q < width || ld_qhat < width) return fail(TDA_ERR_INVALID_ARG, "ld_q/ld_qhat < n_layers*D");
+            if (D > precondition_apply_max_d(state_dtype))
+                return fail(TDA_ERR_UNSUPPORTED, "APPLY keeps a query row in shared memory: D > %lld",
+                            (long long)precondition_apply_max_d(state_dtype));
+            if (n_q == 0)
+                return cuda_check(launch_pc_factor(n_layers, D, state_dtype, state, n_total, lambda_abs,
+                                                   lambda_rel_mean_eig, s),
+                                  "factor");
+            return cuda_check(launch_pc_factor_apply(n_layers, D, state_dtype, state, n_total, lambda_abs,
+                                                     lambda_rel_mean_eig, q, n_q, ld_q, qhat, ld_qhat, s),
+                              "factor + apply");
+        }
         case TDA_PC_APPLY: {
             if (n_q < 0) return fail(TDA_ERR_INVALID_ARG, "negative n_q");
             if (n_q > 0 && (!q || !qhat)) return fail(TDA_ERR_INVALID_ARG, "q/qhat is NULL");

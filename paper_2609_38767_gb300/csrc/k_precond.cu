@@ -495,9 +495,57 @@ __device__ __forceinline__ int warp_cholesky32(const float (*A)[kNB + 1], float 
     return bad;
 }
 
-template <int CS>
+// Queries solved inside the factorisation (FACTOR_APPLY): the query rows ride
+// along as extra rows below M -- solved against each diagonal block and updated
+// by each panel, which is the forward substitution L y = q -- and a second sweep
+// from the last block to the first does the backward substitution L^T x = y.
+// CTA r of the cluster keeps the query columns of the 64-wide tiles t with
+// t % CS == r in shared memory for the whole call; the owner of a block's
+// columns solves that block for all queries and the others read the result
+// through distributed shared memory (two buffers, alternating by step).
+constexpr int kQT = 64, kQP = kQT + 4;  // query column tile and its padded row
+constexpr int kXS = kNB + 4;            // row stride of a solved block: 16-byte rows
+// 16 bytes of CTA `rank`'s shared memory at the address of p in this CTA
+__device__ __forceinline__ float4 ld_peer4(const float* p, uint32_t rank) {
+    uint32_t a = (uint32_t)__cvta_generic_to_shared(p), r;
+    asm volatile("mapa.shared::cluster.u32 %0, %1, %2;" : "=r"(r) : "r"(a), "r"(rank));
+    float4 v;
+    asm volatile("ld.shared::cluster.v4.f32 {%0, %1, %2, %3}, [%4];" : "=f"(v.x), "=f"(v.y), "=f"(v.z), "=f"(v.w)
+                 : "r"(r));
+    return v;
+}
+// this CTA's copy of the solved block [n_q][kNB] (stride kXS) that CTA `rank` holds at Xo
+__device__ __forceinline__ void copy_peer_block(float* XL, const float* Xo, int64_t n_q, uint32_t rank, int tid) {
+    const int64_t n4 = n_q * (kNB / 4);
+    for (int64_t e0 = tid; e0 < n4; e0 += 4 * 256) {
+        float4 v[4];
+#pragma unroll
+        for (int u = 0; u < 4; ++u) {  // four loads in flight before the first store
+            const int64_t e = e0 + u * 256;
+            if (e < n4) v[u] = ld_peer4(Xo + (e / (kNB / 4)) * kXS + (e % (kNB / 4)) * 4, rank);
+        }
+#pragma unroll
+        for (int u = 0; u < 4; ++u) {
+            const int64_t e = e0 + u * 256;
+            if (e < n4) *reinterpret_cast<float4*>(XL + (e / (kNB / 4)) * kXS + (e % (kNB / 4)) * 4) = v[u];
+        }
+    }
+}
+__host__ __device__ inline int64_t query_tiles_per_cta(int64_t D, int cs) {
+    return ((D + kQT - 1) / kQT + cs - 1) / cs;
+}
+__host__ __device__ inline size_t solve_smem_bytes(int64_t D, int64_t n_q, int cs) {
+    return sizeof(float) * ((size_t)query_tiles_per_cta(D, cs) * n_q * kQP + 3 * (size_t)n_q * kXS);
+}
+struct QArgs {
+    const float* q;   // layer 0's column 0 of query row 0
+    float* qhat;
+    int64_t n_q, ld_q, ld_qhat;
+};
+
+template <int CS, bool SOLVE>
 __global__ void __launch_bounds__(256, 1) factor_cluster_kernel(St<float> st, int64_t n_total, double lambda_abs,
-                                                              double lambda_rel) {
+                                                              double lambda_rel, QArgs qa) {
     __shared__ float Lk[kNB][kNB + 1];        // the diagonal block before factoring
     __shared__ float LkT[kNB][2 * kNB + 1];   // L transposed; columns 32..63 stay zero
     __shared__ float dinv[kNB];               // 1 / L_jj of the current block
@@ -511,6 +559,12 @@ __global__ void __launch_bounds__(256, 1) factor_cluster_kernel(St<float> st, in
     float* M = st.M(l);
     double* h = st.header(l);
     const int tid = threadIdx.x, lane = tid & 31, ty = tid / 16, tx = tid % 16;
+    const int64_t n_q = SOLVE ? qa.n_q : 0;
+    extern __shared__ __align__(16) float qsm[];
+    const int64_t nown = SOLVE ? query_tiles_per_cta(D, CS) : 0;
+    float* Qs = qsm;                                 // [nown][n_q][kQP]: owned query column tiles
+    float* XB = Qs + nown * n_q * kQP;               // [2][n_q][kXS]: a solved block, for the others
+    float* XL = XB + 2 * n_q * kXS;                  // [n_q][kXS]: the owner's block, copied here
     for (int e = tid; e < kNB * (2 * kNB + 1); e += blockDim.x) (&LkT[0][0])[e] = 0.f;
     // damping from the mean eigenvalue tr(M)/(n_total D), summed like prepare_kernel
     double s = 0.0;
@@ -538,6 +592,14 @@ __global__ void __launch_bounds__(256, 1) factor_cluster_kernel(St<float> st, in
                 if (i == j) v += lam;
                 M[i * D + j] = v;
             }
+        if (SOLVE)
+            for (int64_t o = 0; o < nown; ++o) {
+                const int64_t c0 = (rank + o * CS) * kQT;
+                for (int64_t e = tid; e < n_q * kQT; e += blockDim.x) {
+                    const int64_t qi = e / kQT, c = c0 + e % kQT;
+                    Qs[(o * n_q + qi) * kQP + e % kQT] = c < D ? qa.q[qi * qa.ld_q + (int64_t)l * D + c] : 0.f;
+                }
+            }
     }
     cluster_barrier();
     for (int64_t k0 = 0; k0 < D; k0 += kNB) {
@@ -552,18 +614,18 @@ __global__ void __launch_bounds__(256, 1) factor_cluster_kernel(St<float> st, in
             if (rank == 0 && lane == 0 && bad >= 0 && h[kPcFailedPivot] == 0.0) h[kPcFailedPivot] = (double)(k0 + bad + 1);
         }
         __syncthreads();
-        // ---- panel rows below the block: x L_kk^T = a, every CS-th row to each CTA of the
-        // cluster. Column order with the same register shift: once x_j is known it leaves
-        // every later entry
+        // ---- panel rows below the block (and the query rows): x L_kk^T = a, every CS-th row
+        // to each CTA of the cluster. Column order with the same register shift: once x_j is
+        // known it leaves every later entry
         for (int64_t i = k0 + kNB + (int64_t)tid * CS + rank; i < D; i += (int64_t)CS * blockDim.x) {
+            float* row = M + i * D + k0;
             float x[kNB];
 #pragma unroll
-            for (int j = 0; j < kNB; ++j) x[j] = __ldcg(M + i * D + k0 + j);
-            float* out = M + i * D + k0;
+            for (int j = 0; j < kNB; ++j) x[j] = __ldcg(row + j);
 #pragma unroll 1
             for (int j = 0; j < kNB; ++j) {
                 const float xj = x[0] * dinv[j];
-                out[j] = xj;
+                row[j] = xj;
 #pragma unroll
                 for (int idx = 1; idx < kNB; ++idx) x[idx] -= xj * LkT[j][j + idx];
 #pragma unroll
@@ -571,7 +633,66 @@ __global__ void __launch_bounds__(256, 1) factor_cluster_kernel(St<float> st, in
                 x[kNB - 1] = 0.f;
             }
         }
+        const int blk = (int)(k0 / kNB), own = (blk / 2) % CS;  // the block's columns: tile blk / 2
+        if (SOLVE && rank == own) {
+            // y_b = q~_b L_bb^-T for every query, the same column-order solve as a panel row
+            float* Qb = Qs + ((blk / 2) / CS) * n_q * kQP + (blk % 2) * kNB;
+            float* Xo = XB + (blk & 1) * n_q * kXS;
+            // query rows start at thread 128: the panel rows above keep at most the first
+            // ceil((D - 32) / CS) threads busy, so both chains run side by side
+            for (int64_t qi = (tid + blockDim.x / 2) % blockDim.x; qi < n_q; qi += blockDim.x) {
+                float* row = Qb + qi * kQP;
+                float x[kNB];
+#pragma unroll
+                for (int j = 0; j < kNB; ++j) x[j] = row[j];
+#pragma unroll 1
+                for (int j = 0; j < kNB; ++j) {
+                    const float xj = x[0] * dinv[j];
+                    row[j] = xj;
+                    Xo[qi * kXS + j] = xj;
+#pragma unroll
+                    for (int idx = 1; idx < kNB; ++idx) x[idx] -= xj * LkT[j][j + idx];
+#pragma unroll
+                    for (int idx = 0; idx < kNB - 1; ++idx) x[idx] = x[idx + 1];
+                    x[kNB - 1] = 0.f;
+                }
+            }
+        }
         cluster_barrier();
+        if (SOLVE && k0 + kNB < D) {
+            // q~[:, c] -= y_b L[c][k0..k0+31]^T for the owned columns c >= k0 + 32
+            copy_peer_block(XL, XB + (blk & 1) * n_q * kXS, n_q, (uint32_t)own, tid);
+            __syncthreads();
+            for (int64_t o = 0; o < nown; ++o) {
+                const int64_t c0 = (rank + o * CS) * kQT;
+                if (c0 + kQT <= k0 + kNB || c0 >= D) continue;
+                for (int e = tid; e < kNB * kQT; e += blockDim.x) {
+                    const int cc = e / kNB, m = e % kNB;
+                    const int64_t c = c0 + cc;
+                    Pj[m][cc] = (c >= k0 + kNB && c < D) ? __ldcg(M + c * D + k0 + m) : 0.f;
+                }
+                __syncthreads();
+                for (int64_t q0 = 0; q0 < n_q; q0 += kQT) {
+#pragma unroll
+                    for (int r = 0; r < 4; ++r) {
+                        const int64_t qi = q0 + ty * 4 + r;
+                        if (qi >= n_q) break;
+                        float acc[4] = {0.f, 0.f, 0.f, 0.f};
+#pragma unroll 8
+                        for (int m = 0; m < kNB; ++m) {
+                            const float xv = XL[qi * kXS + m];
+                            const float4 b4 = *reinterpret_cast<const float4*>(&Pj[m][tx * 4]);
+                            acc[0] += xv * b4.x, acc[1] += xv * b4.y, acc[2] += xv * b4.z, acc[3] += xv * b4.w;
+                        }
+                        float4* dst = reinterpret_cast<float4*>(Qs + (o * n_q + qi) * kQP + tx * 4);
+                        float4 v = *dst;
+                        v.x -= acc[0], v.y -= acc[1], v.z -= acc[2], v.w -= acc[3];
+                        *dst = v;
+                    }
+                }
+                __syncthreads();
+            }
+        }
         // the factored block goes back into M's diagonal block once every CTA has read the
         // unfactored one (no later step reads that block); the inverses of all diagonal
         // blocks are formed after the last step
@@ -580,51 +701,62 @@ __global__ void __launch_bounds__(256, 1) factor_cluster_kernel(St<float> st, in
                 const int i = e / kNB, j = e % kNB;
                 if (j <= i) M[(k0 + i) * D + k0 + j] = LkT[j][i];
             }
-        // ---- trailing update of the lower triangle, 64 x 64 tiles shared by the cluster
+        // ---- trailing update of the lower triangle (and of the query rows' remaining
+        // columns), 64 x 64 tiles shared by the cluster
         const int64_t s0 = k0 + kNB;
         const int64_t rest = D - s0;
         if (rest > 0) {
-            const int64_t t = (rest + T - 1) / T, tiles = t * (t + 1) / 2;
-            // tile u -> (bi, bj), bj <= bi, row-major over the lower triangle of tiles
-            auto tile_of = [&](int64_t u, int64_t& i0, int64_t& j0) {
-                // fp32 estimate (fp64 is a slow pipe here), corrected in integers
-                int64_t bi = (int64_t)((sqrtf(8.f * (float)u + 1.f) - 1.f) * 0.5f);
-                while (bi * (bi + 1) / 2 > u) --bi;
-                while ((bi + 1) * (bi + 2) / 2 <= u) ++bi;
-                i0 = s0 + bi * T;
-                j0 = s0 + (u - bi * (bi + 1) / 2) * T;
+            const int64_t t = (rest + T - 1) / T, lower = t * (t + 1) / 2;
+            const int64_t tiles = lower;
+            // tile u: lower-triangle tile (bi, bj), bj <= bi, row-major; then query tiles (qb, bj)
+            struct Tile {
+                float* rows;  // M or the query rows
+                int64_t ld, lim, i0, j0;
+                bool tri;     // lower triangle of M: only j <= i
+            };
+            auto tile_of = [&](int64_t u) {
+                Tile tl;
+                {
+                    // fp32 estimate (fp64 is a slow pipe here), corrected in integers
+                    int64_t bi = (int64_t)((sqrtf(8.f * (float)u + 1.f) - 1.f) * 0.5f);
+                    while (bi * (bi + 1) / 2 > u) --bi;
+                    while ((bi + 1) * (bi + 2) / 2 <= u) ++bi;
+                    tl.rows = M, tl.ld = D, tl.lim = D, tl.tri = true;
+                    tl.i0 = s0 + bi * T;
+                    tl.j0 = s0 + (u - bi * (bi + 1) / 2) * T;
+                }
+                return tl;
             };
             // software pipeline: while tile u is multiplied, the panel rows and the current
             // values of this CTA's next tile are on their way (each thread: 8 + 8 panel values,
             // row e/32, column e%32, and its 4 x 4 outputs)
             float ra[8], rb[8], mv[4][4];
             auto load_tile = [&](int64_t u) {
-                int64_t i0, j0;
-                tile_of(u, i0, j0);
+                const Tile tl = tile_of(u);
 #pragma unroll
-                for (int h = 0; h < 8; ++h) {
-                    const int e = tid + h * 256, r = e / kNB, m = e % kNB;
-                    ra[h] = (i0 + r < D) ? __ldcg(M + (i0 + r) * D + k0 + m) : 0.f;
-                    rb[h] = (j0 + r < D) ? __ldcg(M + (j0 + r) * D + k0 + m) : 0.f;
+                for (int hh = 0; hh < 8; ++hh) {
+                    const int e = tid + hh * 256, r = e / kNB, m = e % kNB;
+                    ra[hh] = (tl.i0 + r < tl.lim) ? __ldcg(tl.rows + (tl.i0 + r) * tl.ld + k0 + m) : 0.f;
+                    rb[hh] = (tl.j0 + r < D) ? __ldcg(M + (tl.j0 + r) * D + k0 + m) : 0.f;
                 }
 #pragma unroll
                 for (int q = 0; q < 4; ++q)
 #pragma unroll
                     for (int v = 0; v < 4; ++v) {
-                        const int64_t i = i0 + ty * 4 + q, j = j0 + tx * 4 + v;
-                        mv[q][v] = (i < D && j < D && j <= i) ? __ldcg(M + i * D + j) : 0.f;
+                        const int64_t i = tl.i0 + ty * 4 + q, j = tl.j0 + tx * 4 + v;
+                        mv[q][v] = (i < tl.lim && j < D && (!tl.tri || j <= i)) ? __ldcg(tl.rows + i * tl.ld + j)
+                                                                                 : 0.f;
                     }
             };
             int64_t u = rank;
             if (u < tiles) load_tile(u);
             for (; u < tiles; u += CS) {
-                int64_t i0, j0;
-                tile_of(u, i0, j0);
+                const Tile tl = tile_of(u);
 #pragma unroll
-                for (int h = 0; h < 8; ++h) {
-                    const int e = tid + h * 256, r = e / kNB, m = e % kNB;
-                    Pi[m][r] = ra[h];
-                    Pj[m][r] = rb[h];
+                for (int hh = 0; hh < 8; ++hh) {
+                    const int e = tid + hh * 256, r = e / kNB, m = e % kNB;
+                    Pi[m][r] = ra[hh];
+                    Pj[m][r] = rb[hh];
                 }
                 float acc[4][4];
 #pragma unroll
@@ -647,8 +779,8 @@ __global__ void __launch_bounds__(256, 1) factor_cluster_kernel(St<float> st, in
                 for (int q = 0; q < 4; ++q)
 #pragma unroll
                     for (int v = 0; v < 4; ++v) {
-                        const int64_t i = i0 + ty * 4 + q, j = j0 + tx * 4 + v;
-                        if (i < D && j < D && j <= i) M[i * D + j] = acc[q][v];
+                        const int64_t i = tl.i0 + ty * 4 + q, j = tl.j0 + tx * 4 + v;
+                        if (i < tl.lim && j < D && (!tl.tri || j <= i)) tl.rows[i * tl.ld + j] = acc[q][v];
                     }
                 __syncthreads();
             }
@@ -682,14 +814,109 @@ __global__ void __launch_bounds__(256, 1) factor_cluster_kernel(St<float> st, in
         }
         __syncthreads();
     }
+    if constexpr (SOLVE) {
+        // ---- backward substitution L^T x = y from the last block: the owner of block b forms
+        // x_b = Dinv_b^T y~_b for every query; then each CTA removes x_b L[b0..b0+31][c] from
+        // its owned columns c < b0
+        cluster_barrier();  // Dinv complete
+        const int64_t ldh = qa.ld_qhat;
+        float* Qh = qa.qhat + (int64_t)l * D;
+        if (__ldcg(&h[kPcFailedPivot]) != 0.0) {
+            for (int64_t o = 0; o < nown; ++o) {
+                const int64_t c0 = (rank + o * CS) * kQT;
+                for (int64_t e = tid; e < n_q * kQT; e += blockDim.x)
+                    if (c0 + e % kQT < D) Qh[(e / kQT) * ldh + c0 + e % kQT] = NAN;
+            }
+            return;
+        }
+        for (int b = nblk - 1; b >= 0; --b) {
+            const int64_t b0 = (int64_t)b * kNB;
+            const int own = (b / 2) % CS;
+            // L[b0..b0+31][c] of this CTA's first owned tile left of the block does not depend
+            // on x_b: staged while the owner solves
+            const bool pre = nown > 0 && (int64_t)rank * kQT < b0;
+            if (pre)
+                for (int e = tid; e < kNB * kQT; e += blockDim.x) {
+                    const int m = e / kQT, cc = e % kQT;
+                    const int64_t c = (int64_t)rank * kQT + cc;
+                    Pj[m][cc] = (c < b0) ? __ldcg(M + (b0 + m) * D + c) : 0.f;
+                }
+            if (rank == own) {
+                const float* Di = st.Dinv(l) + (int64_t)b * (kNB * kNB);
+                for (int e = tid; e < kNB * kNB; e += blockDim.x) Lk[e / kNB][e % kNB] = __ldcg(Di + e);
+                __syncthreads();
+                float* Qb = Qs + ((b / 2) / CS) * n_q * kQP + (b % 2) * kNB;
+                float* Xo = XB + (b & 1) * n_q * kXS;
+                for (int64_t e = tid; e < n_q * kNB; e += blockDim.x) {
+                    const int64_t qi = e / kNB;
+                    const int c = (int)(e % kNB);
+                    float acc = 0.f;  // Dinv_b is lower triangular: entries above the diagonal are 0
+#pragma unroll
+                    for (int i = 0; i < kNB; ++i) acc += Lk[i][c] * Qb[qi * kQP + i];
+                    Xo[qi * kXS + c] = acc;
+                }
+                __syncthreads();
+                for (int64_t e = tid; e < n_q * kNB; e += blockDim.x)
+                    Qb[(e / kNB) * kQP + e % kNB] = Xo[(e / kNB) * kXS + e % kNB];
+            }
+            cluster_barrier();
+            if (b0 == 0) break;
+            copy_peer_block(XL, XB + (b & 1) * n_q * kXS, n_q, (uint32_t)own, tid);
+            __syncthreads();
+            for (int64_t o = 0; o < nown; ++o) {
+                const int64_t c0 = (rank + o * CS) * kQT;
+                if (c0 >= b0) continue;
+                if (o > 0) {
+                    for (int e = tid; e < kNB * kQT; e += blockDim.x) {
+                        const int m = e / kQT, cc = e % kQT;
+                        Pj[m][cc] = (c0 + cc < b0) ? __ldcg(M + (b0 + m) * D + c0 + cc) : 0.f;
+                    }
+                }
+                __syncthreads();
+                for (int64_t q0 = 0; q0 < n_q; q0 += kQT) {
+#pragma unroll
+                    for (int r = 0; r < 4; ++r) {
+                        const int64_t qi = q0 + ty * 4 + r;
+                        if (qi >= n_q) break;
+                        float acc[4] = {0.f, 0.f, 0.f, 0.f};
+#pragma unroll 8
+                        for (int m = 0; m < kNB; ++m) {
+                            const float xv = XL[qi * kXS + m];
+                            const float4 b4 = *reinterpret_cast<const float4*>(&Pj[m][tx * 4]);
+                            acc[0] += xv * b4.x, acc[1] += xv * b4.y, acc[2] += xv * b4.z, acc[3] += xv * b4.w;
+                        }
+                        float4* dst = reinterpret_cast<float4*>(Qs + (o * n_q + qi) * kQP + tx * 4);
+                        float4 v = *dst;
+                        v.x -= acc[0], v.y -= acc[1], v.z -= acc[2], v.w -= acc[3];
+                        *dst = v;
+                    }
+                }
+                __syncthreads();
+            }
+        }
+        // the owned columns now hold x: out to qhat
+        for (int64_t o = 0; o < nown; ++o) {
+            const int64_t c0 = (rank + o * CS) * kQT;
+            for (int64_t e = tid; e < n_q * kQT; e += blockDim.x)
+                if (c0 + e % kQT < D) Qh[(e / kQT) * ldh + c0 + e % kQT] = Qs[(o * n_q + e / kQT) * kQP + e % kQT];
+        }
+        cluster_barrier();  // peers may still read this CTA's exchange buffer
+    }
 }
 
-template <int CS>
+template <int CS, bool SOLVE>
 cudaError_t factor_cluster(int n_layers, int64_t D, void* state, int64_t n_total, double la, double lr,
-                           cudaStream_t s) {
+                           const QArgs& qa, cudaStream_t s) {
     cudaError_t e = cudaSuccess;
-    if (CS > 8) e = cudaFuncSetAttribute(factor_cluster_kernel<CS>, cudaFuncAttributeNonPortableClusterSizeAllowed, 1);
+    if (CS > 8)
+        e = cudaFuncSetAttribute(factor_cluster_kernel<CS, SOLVE>, cudaFuncAttributeNonPortableClusterSizeAllowed, 1);
     if (e != cudaSuccess) return e;
+    const size_t smem = SOLVE ? solve_smem_bytes(D, qa.n_q, CS) : 0;
+    if (smem > 190 * 1024) return cudaErrorNotSupported;
+    if (SOLVE &&
+        (e = cudaFuncSetAttribute(factor_cluster_kernel<CS, SOLVE>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                  (int)smem)) != cudaSuccess)
+        return e;
     cudaLaunchConfig_t cfg = {};
     cudaLaunchAttribute attr[1];
     attr[0].id = cudaLaunchAttributeClusterDimension;
@@ -698,18 +925,18 @@ cudaError_t factor_cluster(int n_layers, int64_t D, void* state, int64_t n_total
     attr[0].val.clusterDim.z = 1;
     cfg.gridDim = dim3((unsigned)(n_layers * CS));
     cfg.blockDim = dim3(256);
-    cfg.dynamicSmemBytes = 0;
+    cfg.dynamicSmemBytes = smem;
     cfg.stream = s;
     cfg.attrs = attr;
     cfg.numAttrs = 1;
     int max_clusters = 0;
-    if (cudaOccupancyMaxActiveClusters(&max_clusters, factor_cluster_kernel<CS>, &cfg) != cudaSuccess ||
+    if (cudaOccupancyMaxActiveClusters(&max_clusters, factor_cluster_kernel<CS, SOLVE>, &cfg) != cudaSuccess ||
         max_clusters < 1) {
         cudaGetLastError();
         return cudaErrorNotSupported;
     }
     note_launches(1);
-    e = cudaLaunchKernelEx(&cfg, factor_cluster_kernel<CS>, state_of<float>(state, D), n_total, la, lr);
+    e = cudaLaunchKernelEx(&cfg, factor_cluster_kernel<CS, SOLVE>, state_of<float>(state, D), n_total, la, lr, qa);
     if (e != cudaSuccess) return e;
     return cudaGetLastError();
 }
@@ -720,8 +947,9 @@ cudaError_t factor_impl(int n_layers, int64_t D, void* state, int64_t n_total, d
     if constexpr (sizeof(TS) == 4) {
         // fp32 state, whole 32-column blocks: one launch, a cluster of 16 (else 8) CTAs per layer
         if (D % kNB == 0 && D >= 2 * kNB) {
-            cudaError_t e = factor_cluster<16>(n_layers, D, state, n_total, la, lr, s);
-            if (e == cudaErrorNotSupported) e = factor_cluster<8>(n_layers, D, state, n_total, la, lr, s);
+            const QArgs none{nullptr, nullptr, 0, 0, 0};
+            cudaError_t e = factor_cluster<16, false>(n_layers, D, state, n_total, la, lr, none, s);
+            if (e == cudaErrorNotSupported) e = factor_cluster<8, false>(n_layers, D, state, n_total, la, lr, none, s);
             if (e != cudaErrorNotSupported) return e;
         }
     }
@@ -789,6 +1017,23 @@ cudaError_t launch_pc_factor(int n_layers, int64_t D, tda_dtype sdt, void* state
                              double lambda_abs, double lambda_rel, cudaStream_t s) {
     if (sdt == TDA_F64) return factor_impl<double>(n_layers, D, state, n_total, lambda_abs, lambda_rel, s);
     return factor_impl<float>(n_layers, D, state, n_total, lambda_abs, lambda_rel, s);
+}
+
+cudaError_t launch_pc_factor_apply(int n_layers, int64_t D, tda_dtype sdt, void* state, int64_t n_total,
+                                   double lambda_abs, double lambda_rel, const float* q, int64_t n_q, int64_t ld_q,
+                                   void* qhat, int64_t ld_qhat, cudaStream_t s) {
+    // fp32 state, whole 32-column blocks, up to 256 queries: factorisation and both
+    // substitutions in one cluster launch per call; otherwise FACTOR, then APPLY
+    if (sdt == TDA_F32 && D % kNB == 0 && D >= 2 * kNB && n_q >= 1 && n_q <= 256) {
+        const QArgs qa{q, (float*)qhat, n_q, ld_q, ld_qhat};
+        cudaError_t e = factor_cluster<16, true>(n_layers, D, state, n_total, lambda_abs, lambda_rel, qa, s);
+        if (e == cudaErrorNotSupported)
+            e = factor_cluster<8, true>(n_layers, D, state, n_total, lambda_abs, lambda_rel, qa, s);
+        if (e != cudaErrorNotSupported) return e;
+    }
+    cudaError_t e = launch_pc_factor(n_layers, D, sdt, state, n_total, lambda_abs, lambda_rel, s);
+    if (e != cudaSuccess) return e;
+    return launch_pc_apply(n_layers, D, sdt, state, q, n_q, ld_q, qhat, ld_qhat, s);
 }
 
 cudaError_t launch_pc_apply(int n_layers, int64_t D, tda_dtype sdt, const void* state, const float* q,

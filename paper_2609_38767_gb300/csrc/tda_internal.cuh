@@ -162,6 +162,9 @@ cudaError_t launch_pc_fit(int n_layers, int64_t D, tda_dtype sdt, void* state, c
                           int64_t ld, cudaStream_t s);
 cudaError_t launch_pc_factor(int n_layers, int64_t D, tda_dtype sdt, void* state, int64_t n_total,
                              double lambda_abs, double lambda_rel, cudaStream_t s);
+cudaError_t launch_pc_factor_apply(int n_layers, int64_t D, tda_dtype sdt, void* state, int64_t n_total,
+                                   double lambda_abs, double lambda_rel, const float* q, int64_t n_q, int64_t ld_q,
+                                   void* qhat, int64_t ld_qhat, cudaStream_t s);
 cudaError_t launch_pc_apply(int n_layers, int64_t D, tda_dtype sdt, const void* state, const float* q,
                             int64_t n_q, int64_t ld_q, void* qhat, int64_t ld_qhat, cudaStream_t s);
 

@@ -360,6 +360,58 @@ def test_precondition_batched_layers_match_oracle(dev, orc, sdt, D, lam_abs, lam
         assert rel_fro(got[:, l * D:(l + 1) * D], ref) <= tol
 
 
+@pytest.mark.parametrize("D,Nq,nl", [(64, 11, 1), (96, 70, 3), (1024, 64, 2), (1000, 9, 1), (128, 300, 1)])
+def test_precondition_factor_apply_matches_oracle(dev, orc, D, Nq, nl):
+    # FACTOR_APPLY: one launch for an fp32 state with D a multiple of 32 and <= 256 queries (the
+    # queries solved alongside the factorisation), FACTOR then APPLY otherwise (D = 1000, 300 queries)
+    rng = np.random.default_rng(D + Nq)
+    N = 150
+    phi = (rng.standard_normal((N, nl * D)) * rng.uniform(0.5, 2.0, nl * D)).astype(np.float32)
+    q = rng.standard_normal((Nq, nl * D + 3)).astype(np.float32)
+    sdt = tda.TDA_F32
+    per = tda.tda_precondition_state_bytes(D, sdt)
+    state = torch.empty(nl * per, dtype=torch.uint8, device=dev)
+    phid, qd = torch.from_numpy(phi).to(dev), torch.from_numpy(q).to(dev)
+    tda.tda_precondition(tda.TDA_PC_RESET, nl, D, sdt, state)
+    tda.tda_precondition(tda.TDA_PC_FIT_ACCUM, nl, D, sdt, state, phi=phid, n=N, ld_phi=nl * D)
+    qh = torch.full((Nq, nl * D + 5), 7.0, device=dev)
+    tda.tda_precondition(tda.TDA_PC_FACTOR_APPLY, nl, D, sdt, state, n_total=N, lambda_abs=0.0,
+                         lambda_rel_mean_eig=1e-2, q=qd, n_q=Nq, ld_q=nl * D + 3, qhat=qh, ld_qhat=nl * D + 5)
+    info = tda.tda_precondition_info(nl, D, sdt, state)
+    tda.tda_device_status()
+    got = qh.cpu().numpy().astype(np.float64)
+    assert (got[:, nl * D:] == 7.0).all()
+    for l in range(nl):
+        F = orc.fisher(phi[:, l * D:(l + 1) * D].astype(np.float64))
+        lam = orc.damping(F, 0.0, 1e-2)
+        assert abs(info[4 * l] - lam) <= 1e-5 * lam and info[4 * l + 2] == 0
+        ref = orc.precondition(F, lam, q[:, l * D:(l + 1) * D].astype(np.float64))
+        assert rel_fro(got[:, l * D:(l + 1) * D], ref) <= 1e-3
+    # the same state applied again through APPLY gives the same rows (up to summation order)
+    qh2 = torch.empty((Nq, nl * D), device=dev)
+    tda.tda_precondition(tda.TDA_PC_APPLY, nl, D, sdt, state, q=qd, n_q=Nq, ld_q=nl * D + 3, qhat=qh2, ld_qhat=nl * D)
+    tda.tda_device_status()
+    assert rel_fro(qh2.cpu().numpy(), got[:, :nl * D]) <= 1e-5
+
+
+@pytest.mark.parametrize("D", [64, 8])
+def test_precondition_factor_apply_not_spd_gives_nan(dev, D):
+    state = torch.empty(tda.tda_precondition_state_bytes(D, tda.TDA_F32), dtype=torch.uint8, device=dev)
+    tda.tda_precondition(tda.TDA_PC_RESET, 1, D, tda.TDA_F32, state)
+    phi = torch.ones((2, D), device=dev)
+    tda.tda_precondition(tda.TDA_PC_FIT_ACCUM, 1, D, tda.TDA_F32, state, phi=phi, n=2, ld_phi=D)
+    m = state[64:64 + 4 * D * D].view(torch.float32).view(D, D)
+    m[3, 3] = -100.0
+    q = torch.ones((2, D), device=dev)
+    qh = torch.zeros((2, D), device=dev)
+    tda.tda_precondition(tda.TDA_PC_FACTOR_APPLY, 1, D, tda.TDA_F32, state, n_total=2, lambda_abs=1e-3,
+                         q=q, n_q=2, ld_q=D, qhat=qh, ld_qhat=D)
+    with pytest.raises(tda.TdaError) as e:
+        tda.tda_precondition_info(1, D, tda.TDA_F32, state)
+    assert e.value.status == tda.TDA_ERR_NOT_SPD
+    assert torch.isnan(qh).all()
+
+
 def test_bounded_wait_times_out_and_context_survives(dev, orc):
     # a wait on a barrier nothing arrives on runs out after 50 ms; the error word reports it
     tda.tda_device_status()
