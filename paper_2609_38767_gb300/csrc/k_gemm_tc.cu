@@ -338,12 +338,11 @@ score3x_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
 // writes the four features transposed into the swizzled layout (conflict-free:
 // the 32 lanes hit 32 distinct banks).
 template <int ROWS>
-__device__ __forceinline__ void load_split_t(const float* __restrict__ X, int64_t ld, int64_t nrows, int64_t D,
-                                             int64_t f0, int64_t e0, uint8_t* hi, uint8_t* lo, int pt) {
+__device__ __forceinline__ void load_t(const float* __restrict__ X, int64_t ld, int64_t nrows, int64_t D, int64_t f0,
+                                       int64_t e0, float4 (&vals)[ROWS / 16], int pt) {
     constexpr int kPer = ROWS / 16;  // float4 groups per thread: 4 warps x 4 features x kPer
     const int lane = pt & 31, w = pt >> 5;
     const int64_t e = e0 + lane;
-    float4 vals[kPer];
 #pragma unroll
     for (int j = 0; j < kPer; ++j) {
         const int64_t f = f0 + (ROWS / 4) * w + 4 * j;
@@ -361,6 +360,11 @@ __device__ __forceinline__ void load_split_t(const float* __restrict__ X, int64_
         }
         vals[j] = v;
     }
+}
+template <int ROWS>
+__device__ __forceinline__ void store_split_t(const float4 (&vals)[ROWS / 16], uint8_t* hi, uint8_t* lo, int pt) {
+    constexpr int kPer = ROWS / 16;
+    const int lane = pt & 31, w = pt >> 5;
 #pragma unroll
     for (int j = 0; j < kPer; ++j) {
         const float in[4] = {vals[j].x, vals[j].y, vals[j].z, vals[j].w};
@@ -428,22 +432,42 @@ __global__ void __launch_bounds__(kThreads, 1) fit3x_kernel(const FParams p) {
     const int64_t nkc = (p.n + kKC - 1) / kKC;
 
     if (warp < 4) {
+        // producers, software-pipelined: chunk kc + 1 is loaded into registers while chunk kc
+        // is split and written to its stage (two register sets, swapped by unrolling by two)
+        float4 va[2][kBM / 16], vb[2][BN / 16];
+        if (nkc > 0) {
+            load_t<kBM>(ph, p.ld, p.n, p.D, a0, 0, va[0], threadIdx.x);
+            load_t<BN>(ph, p.ld, p.n, p.D, b0, 0, vb[0], threadIdx.x);
+        }
         uint32_t it = 0;
-        for (int64_t kc = 0; kc < nkc; ++kc, ++it) {
+        bool ok = true;
+        auto step = [&](int64_t kc, float4 (&ca)[kBM / 16], float4 (&cb)[BN / 16], float4 (&na)[kBM / 16],
+                        float4 (&nb)[BN / 16]) {
             const int s = it % C::kStages;
             const uint32_t phz = (it / C::kStages) & 1u;
+            if (kc + 1 < nkc) {
+                load_t<kBM>(ph, p.ld, p.n, p.D, a0, (kc + 1) * kKC, na, threadIdx.x);
+                load_t<BN>(ph, p.ld, p.n, p.D, b0, (kc + 1) * kKC, nb, threadIdx.x);
+            }
             bool got = true;
             if (lane == 0) got = wait_bounded(smem_u32(&empty[s]), phz ^ 1u, abort, p.err);
             got = __shfl_sync(0xffffffffu, got, 0);
             __syncwarp();
-            if (!got) break;
+            if (!got) {
+                ok = false;
+                return;
+            }
             uint8_t* st = smem + (size_t)s * C::kStageBytes;
-            load_split_t<kBM>(ph, p.ld, p.n, p.D, a0, kc * kKC, st, st + C::kABytes, threadIdx.x);
-            load_split_t<BN>(ph, p.ld, p.n, p.D, b0, kc * kKC, st + 2 * C::kABytes, st + 2 * C::kABytes + C::kBBytes,
-                             threadIdx.x);
+            store_split_t<kBM>(ca, st, st + C::kABytes, threadIdx.x);
+            store_split_t<BN>(cb, st + 2 * C::kABytes, st + 2 * C::kABytes + C::kBBytes, threadIdx.x);
             fence_proxy_async();
             __syncwarp();
             if (lane == 0) mbar_arrive(smem_u32(&full[s]));
+            ++it;
+        };
+        for (int64_t kc = 0; ok && kc < nkc; kc += 2) {
+            step(kc, va[0], vb[0], va[1], vb[1]);
+            if (ok && kc + 1 < nkc) step(kc + 1, va[1], vb[1], va[0], vb[0]);
         }
     } else {
         if (warp == 4 && lane == 0) {
