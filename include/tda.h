@@ -347,10 +347,13 @@ tda_status tda_precondition_info(int32_t n_layers, int64_t D, tda_dtype state_dt
  *                                  the factors (bf16, the tensor-core kernel's
  *                                  shapes; TDA_ERR_UNSUPPORTED otherwise).
  *   tda_kfac_eigen                 C = sums / M; both eigendecompositions
- *                                  (parallel cyclic Jacobi in fp64, at most 60
- *                                  sweeps; the sweep count, or -1 if it did not
- *                                  converge, lands in header[2] (a) and [3] (g)).
- *                                  Resets the EK-FAC sums.
+ *                                  (parallel cyclic Jacobi: for k <= 64 fp32
+ *                                  sweeps, then the fp32 eigenvectors made
+ *                                  orthonormal in fp64 and fp64 sweeps on
+ *                                  V^T C V; fp64 sweeps throughout for larger k;
+ *                                  at most 60 fp64 sweeps, their count, or -1 if
+ *                                  they did not converge, lands in header[2] (a)
+ *                                  and [3] (g)). Resets the EK-FAC sums.
  *   tda_kfac_accumulate_eigenvalues  EK-FAC: add sum_i (U_g^T Phi_i U_a)^2 over n
  *                                  training features (rows of stride ld_phi).
  * ws (device scratch, 256-byte aligned) of tda_kfac_workspace_size(L, dtype)

@@ -84,41 +84,29 @@ __global__ void sum_partials_kernel(const float* __restrict__ part, int nblk, in
     if (header && blockIdx.x == 0 && threadIdx.x == 0) header[slot] += add;
 }
 
-// Parallel cyclic Jacobi (round-robin pair ordering) on C = S / M for the
-// a side (blockIdx.x 0) and the g side (1) of layer blockIdx.y. A lives in
-// shared memory, the eigenvectors V (V <- V J) too when n <= 64 (else in the
-// state's U). Each round rotates floor(m/2) disjoint pairs at once: angles from
-// the round's starting matrix, then all row updates, then all column updates,
-// which is J^T A J for the product J of the round's rotations.
-__global__ void __launch_bounds__(kKfThreads)
-jacobi_kernel(double* __restrict__ st0, int64_t stride, int64_t ka, int64_t kg) {
-    extern __shared__ double A[];  // [n][n], V [n][n] when n <= 64, then c, s, p, q per pair
-    double* st = st0 + (int64_t)blockIdx.y * stride;
-    const KfLayout l(ka, kg);
-    const bool side_g = blockIdx.x == 1;
-    const int n = (int)(side_g ? kg : ka);
-    const double* S = st + (side_g ? l.Sg : l.Sa);
-    double* U = st + (side_g ? l.Ug : l.Ua);
-    double* w = st + (side_g ? l.wg : l.wa);
-    const int nmax = (int)(ka > kg ? ka : kg);
-    const bool v_shared = nmax <= 64;
-    double* V = v_shared ? A + nmax * nmax : U;
+__device__ __forceinline__ float j_sqrt(float x) { return sqrtf(x); }
+__device__ __forceinline__ double j_sqrt(double x) { return sqrt(x); }
+__device__ __forceinline__ float j_abs(float x) { return fabsf(x); }
+__device__ __forceinline__ double j_abs(double x) { return fabs(x); }
+
+// Parallel cyclic Jacobi (round-robin pair ordering) by one CTA on the
+// symmetric n x n matrix A in shared memory (row stride lda), accumulating
+// V <- V J (row stride ldv). Each round rotates floor(m/2) disjoint pairs at
+// once: angles from the round's starting matrix, then all row updates, then
+// all column updates, which is J^T A J for the product J of the round's
+// rotations. Stops when the off-diagonal squared norm is <= tol * fro (fro =
+// squared norm of A at entry); returns the sweep count, or -1 after
+// max_sweeps. Shared matrices use an odd row stride (n + 1) so that the column
+// updates, whose threads walk down a column, hit distinct banks.
+template <typename T>
+__device__ int jacobi_sweeps(T* A, int lda, T* V, int ldv, int n, T* cs, T* sn, int* P, int* Q, double* red, int* done,
+                             double tol, int max_sweeps) {
     const int m = (n + 1) & ~1;  // even number of players; index n is a dummy when n is odd
-    double* cs = A + (v_shared ? 2 : 1) * nmax * nmax;
-    double* sn = cs + (nmax + 2) / 2;
-    int* P = (int*)(sn + (nmax + 2) / 2);
-    int* Q = P + (nmax + 2) / 2;
-    __shared__ double red[kKfThreads];
-    __shared__ int done;
-    const double Mtok = st[0];
-    const double inv = Mtok > 0 ? 1.0 / Mtok : 0.0;
+    double f = 0.0;
     for (int e = threadIdx.x; e < n * n; e += blockDim.x) {
-        A[e] = S[e] * inv;
-        V[e] = (e / n == e % n) ? 1.0 : 0.0;
+        const double a = (double)A[(e / n) * lda + e % n];
+        f += a * a;
     }
-    __syncthreads();
-    double f = 0.0;  // squared Frobenius norm
-    for (int e = threadIdx.x; e < n * n; e += blockDim.x) f += A[e] * A[e];
     red[threadIdx.x] = f;
     __syncthreads();
     for (int h = blockDim.x / 2; h > 0; h >>= 1) {
@@ -128,19 +116,22 @@ jacobi_kernel(double* __restrict__ st0, int64_t stride, int64_t ka, int64_t kg) 
     const double fro = red[0];
     __syncthreads();
     int sweep = 0;
-    for (; sweep < 60; ++sweep) {
+    for (; sweep < max_sweeps; ++sweep) {
         double off = 0.0;
         for (int e = threadIdx.x; e < n * n; e += blockDim.x)
-            if (e / n != e % n) off += A[e] * A[e];
+            if (e / n != e % n) {
+                const double a = (double)A[(e / n) * lda + e % n];
+                off += a * a;
+            }
         red[threadIdx.x] = off;
         __syncthreads();
         for (int h = blockDim.x / 2; h > 0; h >>= 1) {
             if (threadIdx.x < h) red[threadIdx.x] += red[threadIdx.x + h];
             __syncthreads();
         }
-        if (threadIdx.x == 0) done = (red[0] <= 1e-28 * fro) ? 1 : 0;
+        if (threadIdx.x == 0) *done = (red[0] <= tol * fro) ? 1 : 0;
         __syncthreads();
-        if (done) break;
+        if (*done) return sweep;
         for (int r = 0; r < m - 1; ++r) {
             for (int i = threadIdx.x; i < m / 2; i += blockDim.x) {
                 int p = i == 0 ? r : (r + i) % (m - 1);
@@ -150,13 +141,13 @@ jacobi_kernel(double* __restrict__ st0, int64_t stride, int64_t ka, int64_t kg) 
                     p = q;
                     q = t;
                 }
-                double c = 1.0, sv = 0.0;
+                T c = 1, sv = 0;
                 if (q < n) {
-                    const double apq = A[p * n + q];
-                    if (apq != 0.0) {
-                        const double tau = (A[q * n + q] - A[p * n + p]) / (2.0 * apq);
-                        const double t = (tau >= 0 ? 1.0 : -1.0) / (fabs(tau) + sqrt(1.0 + tau * tau));
-                        c = 1.0 / sqrt(1.0 + t * t);
+                    const T apq = A[p * lda + q];
+                    if (apq != T(0)) {
+                        const T tau = (A[q * lda + q] - A[p * lda + p]) / (T(2) * apq);
+                        const T t = (tau >= T(0) ? T(1) : T(-1)) / (j_abs(tau) + j_sqrt(T(1) + tau * tau));
+                        c = T(1) / j_sqrt(T(1) + t * t);
                         sv = t * c;
                     }
                 }
@@ -169,32 +160,131 @@ jacobi_kernel(double* __restrict__ st0, int64_t stride, int64_t ka, int64_t kg) 
             const int half = m / 2;
             for (int x = threadIdx.x; x < half * n; x += blockDim.x) {  // rows p, q: A <- J^T A
                 const int i = x / n, k = x - (x / n) * n;
-                if (Q[i] < 0 || sn[i] == 0.0) continue;
+                if (Q[i] < 0 || sn[i] == T(0)) continue;
                 const int p = P[i], q = Q[i];
-                const double c = cs[i], sv = sn[i], apk = A[p * n + k], aqk = A[q * n + k];
-                A[p * n + k] = c * apk - sv * aqk;
-                A[q * n + k] = sv * apk + c * aqk;
+                const T c = cs[i], sv = sn[i], apk = A[p * lda + k], aqk = A[q * lda + k];
+                A[p * lda + k] = c * apk - sv * aqk;
+                A[q * lda + k] = sv * apk + c * aqk;
             }
             __syncthreads();
             for (int x = threadIdx.x; x < half * n; x += blockDim.x) {  // columns p, q: A <- A J, V <- V J
                 const int i = x / n, k = x - (x / n) * n;
-                if (Q[i] < 0 || sn[i] == 0.0) continue;
+                if (Q[i] < 0 || sn[i] == T(0)) continue;
                 const int p = P[i], q = Q[i];
-                const double c = cs[i], sv = sn[i];
-                const double akp = A[k * n + p], akq = A[k * n + q];
-                A[k * n + p] = c * akp - sv * akq;
-                A[k * n + q] = sv * akp + c * akq;
-                const double vkp = V[k * n + p], vkq = V[k * n + q];
-                V[k * n + p] = c * vkp - sv * vkq;
-                V[k * n + q] = sv * vkp + c * vkq;
+                const T c = cs[i], sv = sn[i];
+                const T akp = A[k * lda + p], akq = A[k * lda + q];
+                A[k * lda + p] = c * akp - sv * akq;
+                A[k * lda + q] = sv * akp + c * akq;
+                const T vkp = V[k * ldv + p], vkq = V[k * ldv + q];
+                V[k * ldv + p] = c * vkp - sv * vkq;
+                V[k * ldv + q] = sv * vkp + c * vkq;
             }
             __syncthreads();
         }
     }
-    for (int i = threadIdx.x; i < n; i += blockDim.x) w[i] = A[i * n + i];
-    if (v_shared)
-        for (int e = threadIdx.x; e < n * n; e += blockDim.x) U[e] = V[e];
-    if (threadIdx.x == 0) st[2 + (side_g ? 1 : 0)] = done ? (double)sweep : -1.0;
+    return -1;
+}
+
+// out = X^T Y (tx) or X Y, n x n fp64 in shared memory, row stride ld (one CTA)
+__device__ void gemm_nn(double* out, const double* X, const double* Y, int n, int ld, bool tx) {
+    for (int e = threadIdx.x; e < n * n; e += blockDim.x) {
+        const int i = e / n, j = e - (e / n) * n;
+        double acc = 0.0;
+        for (int k = 0; k < n; ++k) acc += (tx ? X[k * ld + i] : X[i * ld + k]) * Y[k * ld + j];
+        out[i * ld + j] = acc;
+    }
+    __syncthreads();
+}
+
+// Eigenbases of C = S / M for the a side (blockIdx.x 0) and the g side (1) of
+// layer blockIdx.y, C = U diag(w) U^T.
+//   n <= 64 (MIXED): the sweeps run in fp32 (the fp64 pipe is a small fraction
+//   of the fp32 one here) until the off-diagonal part is near fp32 rounding;
+//   then, in fp64, two Newton-Schulz steps V <- V (3I - V^T V) / 2 make the
+//   fp32 eigenvectors orthonormal to fp64 precision, A = V^T C V is formed
+//   afresh, and fp64 sweeps finish (typically two). The header gets the fp64
+//   sweep count.
+//   n > 64: fp64 sweeps from the start, V in the state's U.
+template <bool MIXED>
+__global__ void __launch_bounds__(kKfThreads)
+jacobi_kernel(double* __restrict__ st0, int64_t stride, int64_t ka, int64_t kg) {
+    extern __shared__ double smd[];
+    double* st = st0 + (int64_t)blockIdx.y * stride;
+    const KfLayout l(ka, kg);
+    const bool side_g = blockIdx.x == 1;
+    const int n = (int)(side_g ? kg : ka);
+    const double* S = st + (side_g ? l.Sg : l.Sa);
+    double* U = st + (side_g ? l.Ug : l.Ua);
+    double* w = st + (side_g ? l.wg : l.wa);
+    const int nmax = (int)(ka > kg ? ka : kg), mh = (nmax + 2) / 2, ld = n + 1, sq = nmax * (nmax + 1);
+    __shared__ double red[kKfThreads];
+    __shared__ int done;
+    const double Mtok = st[0];
+    const double inv = Mtok > 0 ? 1.0 / Mtok : 0.0;
+    double* A = smd;  // [n][ld]
+    int sweeps;
+    if constexpr (MIXED) {
+        double* V = A + sq;
+        double* Tm = V + sq;  // fp64 scratch
+        double* cs = Tm + sq;
+        double* sn = cs + mh;
+        float* A32 = (float*)(sn + mh);
+        float* V32 = A32 + sq;
+        float* cs32 = V32 + sq;
+        float* sn32 = cs32 + mh;
+        int* P = (int*)(sn32 + mh);
+        int* Q = P + mh;
+        for (int e = threadIdx.x; e < n * n; e += blockDim.x) {
+            const int i = e / n, j = e % n;
+            A32[i * ld + j] = (float)(S[e] * inv);
+            V32[i * ld + j] = (i == j) ? 1.f : 0.f;
+        }
+        __syncthreads();
+        // fp32: the off-diagonal part down to about 1e-6 of ||C|| (near fp32 rounding; at most
+        // 20 sweeps, since fp32 cannot go much further)
+        jacobi_sweeps<float>(A32, ld, V32, ld, n, cs32, sn32, P, Q, red, &done, 1e-12, 20);
+        for (int e = threadIdx.x; e < n * n; e += blockDim.x) {
+            const int i = e / n, j = e % n;
+            V[i * ld + j] = (double)V32[i * ld + j];
+        }
+        __syncthreads();
+        for (int it = 0; it < 2; ++it) {  // Newton-Schulz: V <- V (3I - V^T V) / 2
+            gemm_nn(Tm, V, V, n, ld, true);
+            for (int e = threadIdx.x; e < n * n; e += blockDim.x) {
+                const int i = e / n, j = e % n;
+                Tm[i * ld + j] = ((i == j) ? 1.5 : 0.0) - 0.5 * Tm[i * ld + j];
+            }
+            __syncthreads();
+            gemm_nn(A, V, Tm, n, ld, false);
+            for (int e = threadIdx.x; e < n * n; e += blockDim.x) V[(e / n) * ld + e % n] = A[(e / n) * ld + e % n];
+            __syncthreads();
+        }
+        for (int e = threadIdx.x; e < n * n; e += blockDim.x) A[(e / n) * ld + e % n] = S[e] * inv;  // C
+        __syncthreads();
+        gemm_nn(Tm, A, V, n, ld, false);  // C V
+        gemm_nn(A, V, Tm, n, ld, true);   // V^T C V
+        sweeps = jacobi_sweeps<double>(A, ld, V, ld, n, cs, sn, P, Q, red, &done, 1e-28, 60);
+        for (int e = threadIdx.x; e < n * n; e += blockDim.x) U[e] = V[(e / n) * ld + e % n];
+    } else {
+        const bool v_shared = nmax <= 64;
+        double* V = v_shared ? A + sq : U;
+        const int ldv = v_shared ? ld : n;
+        double* cs = A + (v_shared ? 2 : 1) * sq;
+        double* sn = cs + mh;
+        int* P = (int*)(sn + mh);
+        int* Q = P + mh;
+        for (int e = threadIdx.x; e < n * n; e += blockDim.x) {
+            const int i = e / n, j = e % n;
+            A[i * ld + j] = S[e] * inv;
+            V[i * ldv + j] = (i == j) ? 1.0 : 0.0;
+        }
+        __syncthreads();
+        sweeps = jacobi_sweeps<double>(A, ld, V, ldv, n, cs, sn, P, Q, red, &done, 1e-28, 60);
+        if (v_shared)
+            for (int e = threadIdx.x; e < n * n; e += blockDim.x) U[e] = V[(e / n) * ld + e % n];
+    }
+    for (int i = threadIdx.x; i < n; i += blockDim.x) w[i] = A[i * ld + i];
+    if (threadIdx.x == 0) st[2 + (side_g ? 1 : 0)] = (double)sweeps;
     if (blockIdx.x == 0) {  // a new eigenbasis invalidates the EK-FAC sums
         for (int64_t e = threadIdx.x; e < ka * kg; e += blockDim.x) st[l.Le + e] = 0.0;
         if (threadIdx.x == 0) st[1] = 0.0;
@@ -457,13 +547,21 @@ cudaError_t launch_kfac_sum_partials(const float* part, int nblk, int64_t stride
 
 cudaError_t launch_kfac_eigen(int n_layers, double* state, int64_t ka, int64_t kg, cudaStream_t s) {
     const int64_t nmax = ka > kg ? ka : kg;
-    const int64_t mh = (nmax + 2) / 2;
-    const size_t smem = (size_t)(nmax <= 64 ? 2 : 1) * nmax * nmax * 8 + (size_t)mh * (8 + 8 + 4 + 4);
-    cudaError_t e = cudaFuncSetAttribute(jacobi_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
-    if (e != cudaSuccess) return e;
+    const int64_t mh = (nmax + 2) / 2, sq = nmax * (nmax + 1);
+    const int64_t stride = (int64_t)kfac_state_bytes(ka, kg) / 8;
+    cudaError_t e;
     note_launches(1);
-    jacobi_kernel<<<dim3(2, (unsigned)n_layers), kKfThreads, smem, s>>>(state, (int64_t)kfac_state_bytes(ka, kg) / 8,
-                                                                         ka, kg);
+    if (nmax <= 64) {
+        const size_t smem = (size_t)3 * sq * 8 + (size_t)mh * (8 + 8) + (size_t)2 * sq * 4 + (size_t)mh * (4 + 4 + 4 + 4);
+        if ((e = cudaFuncSetAttribute(jacobi_kernel<true>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem)))
+            return e;
+        jacobi_kernel<true><<<dim3(2, (unsigned)n_layers), kKfThreads, smem, s>>>(state, stride, ka, kg);
+        return cudaGetLastError();
+    }
+    const size_t smem = (size_t)sq * 8 + (size_t)mh * (8 + 8 + 4 + 4);
+    if ((e = cudaFuncSetAttribute(jacobi_kernel<false>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem)))
+        return e;
+    jacobi_kernel<false><<<dim3(2, (unsigned)n_layers), kKfThreads, smem, s>>>(state, stride, ka, kg);
     return cudaGetLastError();
 }
 
