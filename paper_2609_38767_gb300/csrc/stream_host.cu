@@ -1,9 +1,11 @@
 // stream_host.cu -- tda_project_host: the factored projection of factors that
 // live in host memory. App. A.2 applies the projection as the factors arrive,
 // so raw factors are never buffered whole; here they stream through two
-// device staging halves of the caller's scratch: the copy of chunk c+1 (on a
-// library-owned copy stream) overlaps the projection of chunk c (on the
-// caller's stream).
+// device staging halves of the caller's scratch: the copies of chunk c+1
+// overlap the projection of chunk c (on the caller's stream). Each chunk's
+// bytes are split evenly over kCopyStreams library-owned copy streams: on the
+// GB300 machines measured, one stream moved 106-135 GB/s host to device and
+// three concurrent ones up to 183 GB/s.
 #include <mutex>
 
 #include "tda_internal.cuh"
@@ -11,11 +13,14 @@
 namespace tda {
 namespace {
 
+constexpr int kCopyStreams = 4;
+
 struct HostPipe {
     bool ready = false;
-    cudaStream_t copy = nullptr;
-    cudaEvent_t copied[2] = {nullptr, nullptr};
+    cudaStream_t copy[kCopyStreams] = {};
+    cudaEvent_t copied[2][kCopyStreams] = {};  // [half][stream]
     cudaEvent_t done[2] = {nullptr, nullptr};
+    uint64_t next = 0;  // staging half of the next chunk: alternates across calls too
     std::mutex mu;
 };
 
@@ -29,9 +34,11 @@ cudaError_t pipe_for_device(HostPipe** out) {
     HostPipe& p = g_pipes[dev];
     *out = &p;
     if (p.ready) return cudaSuccess;
-    if ((e = cudaStreamCreateWithFlags(&p.copy, cudaStreamNonBlocking)) != cudaSuccess) return e;
+    for (int i = 0; i < kCopyStreams; ++i)
+        if ((e = cudaStreamCreateWithFlags(&p.copy[i], cudaStreamNonBlocking)) != cudaSuccess) return e;
     for (int b = 0; b < 2; ++b) {
-        if ((e = cudaEventCreateWithFlags(&p.copied[b], cudaEventDisableTiming)) != cudaSuccess) return e;
+        for (int i = 0; i < kCopyStreams; ++i)
+            if ((e = cudaEventCreateWithFlags(&p.copied[b][i], cudaEventDisableTiming)) != cudaSuccess) return e;
         if ((e = cudaEventCreateWithFlags(&p.done[b], cudaEventDisableTiming)) != cudaSuccess) return e;
     }
     p.ready = true;
@@ -75,20 +82,36 @@ extern "C" tda_status tda_project_host(const tda_layer_desc* L, tda_dtype dtype,
     int64_t chunk = (int64_t)(half / (a_ex + b_ex));
     if (chunk > N) chunk = N;
     cudaStream_t s = (cudaStream_t)stream;
-    for (int64_t c0 = 0, c = 0; c0 < N; c0 += chunk, ++c) {
-        const int b = (int)(c & 1);
+    for (int64_t c0 = 0; c0 < N; c0 += chunk) {
+        // consecutive chunks, also of consecutive calls, use alternate halves: the copy of the
+        // next one overlaps the projection of this one (done[] orders reuse of a half)
+        const int b = (int)(p->next++ & 1);
         const int64_t cnt = (N - c0) < chunk ? (N - c0) : chunk;
         char* dA = (char*)ws + (size_t)b * half;
         char* dB = dA + (size_t)chunk * a_ex;
-        if ((st = cuda_check(cudaStreamWaitEvent(p->copy, p->done[b], 0), "wait buffer"))) return st;
-        if ((st = cuda_check(cudaMemcpyAsync(dA, (const char*)A_h + (size_t)c0 * a_ex, (size_t)cnt * a_ex,
-                                             cudaMemcpyHostToDevice, p->copy), "copy A")))
-            return st;
-        if ((st = cuda_check(cudaMemcpyAsync(dB, (const char*)B_h + (size_t)c0 * b_ex, (size_t)cnt * b_ex,
-                                             cudaMemcpyHostToDevice, p->copy), "copy B")))
-            return st;
-        if ((st = cuda_check(cudaEventRecord(p->copied[b], p->copy), "record copy"))) return st;
-        if ((st = cuda_check(cudaStreamWaitEvent(s, p->copied[b], 0), "wait copy"))) return st;
+        const char* srcA = (const char*)A_h + (size_t)c0 * a_ex;
+        const char* srcB = (const char*)B_h + (size_t)c0 * b_ex;
+        const size_t nA = (size_t)cnt * a_ex, nB = (size_t)cnt * b_ex;
+        for (int i = 0; i < kCopyStreams; ++i) {
+            // part i of each factor: bytes [i n / kCopyStreams, (i + 1) n / kCopyStreams), 256-byte cuts
+            auto cut = [](size_t n, int k) {
+                const size_t c = ((n * (size_t)k / kCopyStreams) + 255) & ~(size_t)255;
+                return c < n ? c : n;
+            };
+            const size_t a0 = i == 0 ? 0 : cut(nA, i), a1 = i + 1 == kCopyStreams ? nA : cut(nA, i + 1);
+            const size_t b0 = i == 0 ? 0 : cut(nB, i), b1 = i + 1 == kCopyStreams ? nB : cut(nB, i + 1);
+            if ((st = cuda_check(cudaStreamWaitEvent(p->copy[i], p->done[b], 0), "wait buffer"))) return st;
+            if (a1 > a0 && (st = cuda_check(cudaMemcpyAsync(dA + a0, srcA + a0, a1 - a0, cudaMemcpyHostToDevice,
+                                                            p->copy[i]),
+                                            "copy A")))
+                return st;
+            if (b1 > b0 && (st = cuda_check(cudaMemcpyAsync(dB + b0, srcB + b0, b1 - b0, cudaMemcpyHostToDevice,
+                                                            p->copy[i]),
+                                            "copy B")))
+                return st;
+            if ((st = cuda_check(cudaEventRecord(p->copied[b][i], p->copy[i]), "record copy"))) return st;
+            if ((st = cuda_check(cudaStreamWaitEvent(s, p->copied[b][i], 0), "wait copy"))) return st;
+        }
         if ((st = tda_project(L, dtype, dA, dB, cnt, phi + c0 * ld_phi, ld_phi, TDA_ROUTE_FACTORED, nullptr, 0,
                               stream)))
             return st;
