@@ -333,34 +333,14 @@ score3x_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
 // ---------------------------------------------------------------------------
 // Fisher fit on the tensor cores: M_l += Phi_l^T Phi_l for the lower 128 x 128
 // tiles of every layer l (layer l's features at column l*D of each row of Phi).
-// The operand tiles are features x examples, K-major: 32 examples per chunk.
-// Lane l of a producer warp loads example row e0+l, 16 bytes at a time, and
-// writes the four features transposed into the swizzled layout (conflict-free:
-// the 32 lanes hit 32 distinct banks).
-template <int ROWS>
-__device__ __forceinline__ void load_t(const float* __restrict__ X, int64_t ld, int64_t nrows, int64_t D, int64_t f0,
-                                       int64_t e0, float4 (&vals)[ROWS / 16], int pt) {
-    constexpr int kPer = ROWS / 16;  // float4 groups per thread: 4 warps x 4 features x kPer
-    const int lane = pt & 31, w = pt >> 5;
-    const int64_t e = e0 + lane;
-#pragma unroll
-    for (int j = 0; j < kPer; ++j) {
-        const int64_t f = f0 + (ROWS / 4) * w + 4 * j;
-        float4 v = make_float4(0.f, 0.f, 0.f, 0.f);
-        if (e < nrows) {
-            const float* p = X + e * ld + f;
-            if (f + 3 < D) {
-                v = __ldg(reinterpret_cast<const float4*>(p));
-            } else {
-                v.x = f < D ? p[0] : 0.f;
-                v.y = f + 1 < D ? p[1] : 0.f;
-                v.z = f + 2 < D ? p[2] : 0.f;
-                v.w = 0.f;
-            }
-        }
-        vals[j] = v;
-    }
-}
+// The MMA operand tiles are features x examples, K-major (32 examples per
+// chunk), but Phi holds examples x features. Lane 0 of warp 5 copies each chunk
+// raw with TMA (32 examples x 32 features per box, 128-byte swizzle, 4 boxes
+// per operand) into a ring of raw stages; warps 0-3 read it back transposed
+// (lane = example, 16 bytes of features per load: conflict-free thanks to the
+// swizzle), split every value to hi/lo and write both into the K-major swizzled
+// operand layout (conflict-free: the 32 lanes hit 32 distinct banks). A tile on
+// the diagonal has A = B and loads and splits one operand.
 template <int ROWS>
 __device__ __forceinline__ void store_split_t(const float4 (&vals)[ROWS / 16], uint8_t* hi, uint8_t* lo, int pt) {
     constexpr int kPer = ROWS / 16;
@@ -379,27 +359,59 @@ __device__ __forceinline__ void store_split_t(const float4 (&vals)[ROWS / 16], u
         }
     }
 }
+// Warp w's 32 features of one raw operand (box w: row = example, 128 bytes of
+// features, 16-byte groups swizzled by the row's low three bits).
+__device__ __forceinline__ void load_raw_t(const uint8_t* raw, float4 (&vals)[8], int pt) {
+    const int lane = pt & 31, w = pt >> 5;
+    const uint8_t* row = raw + (uint32_t)w * 4096u + (uint32_t)lane * kRowBytes;
+#pragma unroll
+    for (int j = 0; j < 8; ++j) vals[j] = *reinterpret_cast<const float4*>(row + ((j ^ (lane & 7)) << 4));
+}
+
+struct FCfg {
+    static constexpr int kStages = 2;       // hi/lo operand stages
+    static constexpr int kRawStages = 3;    // raw TMA chunks
+    static constexpr uint32_t kABytes = kBM * kRowBytes;    // 16 KiB: one operand, hi or lo or raw
+    static constexpr uint32_t kStageBytes = 4 * kABytes;    // hi and lo of both operands
+    static constexpr uint32_t kRawBytes = 2 * kABytes;      // raw chunk of both operands
+    // The tensor pipe's fp32 accumulation rounds toward zero, so a long same-sign sum
+    // (a diagonal entry of M) drifts low by ~1 ulp per accumulate. Each accumulator
+    // therefore takes a group of kGroup consecutive chunks (48 accumulates) and the
+    // epilogue warps drain it into round-to-nearest fp32 registers while the MMAs
+    // move on to the next of the kAcc accumulators.
+    static constexpr int kAcc = 4;                          // 4 x 128 TMEM columns
+    static constexpr int kGroup = 4;                        // chunks per accumulator group
+    static constexpr uint32_t kTmemCols = 512;
+    static constexpr size_t kBarOff = (size_t)kStages * kStageBytes + (size_t)kRawStages * kRawBytes;
+    static constexpr size_t kSmem = 1024 + kBarOff + 8 * (2 * kStages + 2 * kRawStages + 2 * kAcc + 1) + 16;
+};
+static_assert(FCfg::kSmem <= 232448, "fit3x shared memory");
+static_assert(128 * 129 * 4 <= FCfg::kStages * FCfg::kStageBytes, "fit3x staging tile");
 
 struct FParams {
-    const float* phi;
     char* state;       // layer states, `bytes` apart; M at +64
     size_t bytes;
-    int64_t D, n, ld;
+    int64_t D, n;
     int tiles;         // lower tiles per layer
     unsigned int* err;
 };
 
-__global__ void __launch_bounds__(kThreads, 1) fit3x_kernel(const FParams p) {
+constexpr int kFitThreads = 320;  // warps 0-3 split, 4-7 epilogue, 8 MMA, 9 TMA
+__global__ void __launch_bounds__(kFitThreads, 1) fit3x_kernel(const __grid_constant__ CUtensorMap tm, const FParams p) {
     constexpr int BN = 128;
-    using C = GCfg<BN>;
+    using C = FCfg;
     extern __shared__ uint8_t smem_raw[];
     uint8_t* smem = (uint8_t*)(((uintptr_t)smem_raw + 1023) & ~(uintptr_t)1023);
-    uint64_t* bars = (uint64_t*)(smem + (size_t)C::kStages * C::kStageBytes);
-    uint64_t* full = bars;
-    uint64_t* empty = bars + C::kStages;
-    uint64_t* tfull = empty + C::kStages;
-    uint64_t* mma_done = tfull + 1;
-    uint32_t* tmem_slot = (uint32_t*)(mma_done + 3);
+    uint8_t* raw0 = smem + (size_t)C::kStages * C::kStageBytes;
+    uint64_t* bars = (uint64_t*)(smem + C::kBarOff);
+    uint64_t* full = bars;                          // count 4 (producer warps)
+    uint64_t* empty = bars + C::kStages;            // count 1 (MMA commit)
+    uint64_t* raw_full = empty + C::kStages;        // count 1 + TMA bytes
+    uint64_t* raw_empty = raw_full + C::kRawStages; // count 4 (producer warps)
+    uint64_t* acc_full = raw_empty + C::kRawStages; // count 1 (MMA commit): a group is in accumulator a
+    uint64_t* acc_empty = acc_full + C::kAcc;       // count 4 (epilogue warps): accumulator a drained
+    uint64_t* mma_done = acc_empty + C::kAcc;
+    uint32_t* tmem_slot = (uint32_t*)(mma_done + 1);
     volatile int* abort = (volatile int*)(tmem_slot + 1);
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     if (threadIdx.x == 0) {
@@ -407,7 +419,14 @@ __global__ void __launch_bounds__(kThreads, 1) fit3x_kernel(const FParams p) {
             mbar_init(smem_u32(&full[s]), 4);
             mbar_init(smem_u32(&empty[s]), 1);
         }
-        mbar_init(smem_u32(tfull), 1);
+        for (int r = 0; r < C::kRawStages; ++r) {
+            mbar_init(smem_u32(&raw_full[r]), 1);
+            mbar_init(smem_u32(&raw_empty[r]), 4);
+        }
+        for (int a = 0; a < C::kAcc; ++a) {
+            mbar_init(smem_u32(&acc_full[a]), 1);
+            mbar_init(smem_u32(&acc_empty[a]), 4);
+        }
         mbar_init(smem_u32(mma_done), 1);
         *abort = 0;
         fence_mbar_init();
@@ -427,75 +446,102 @@ __global__ void __launch_bounds__(kThreads, 1) fit3x_kernel(const FParams p) {
     while ((by + 1) * (by + 2) / 2 <= t) ++by;
     while (by * (by + 1) / 2 > t) --by;
     const int bx = t - by * (by + 1) / 2;
+    const bool diag = bx == by;
     const int64_t a0 = (int64_t)by * kBM, b0 = (int64_t)bx * BN;
-    const float* ph = p.phi + (int64_t)layer * p.D;
     const int64_t nkc = (p.n + kKC - 1) / kKC;
 
     if (warp < 4) {
-        // producers, software-pipelined: chunk kc + 1 is loaded into registers while chunk kc
-        // is split and written to its stage (two register sets, swapped by unrolling by two)
-        float4 va[2][kBM / 16], vb[2][BN / 16];
-        if (nkc > 0) {
-            load_t<kBM>(ph, p.ld, p.n, p.D, a0, 0, va[0], threadIdx.x);
-            load_t<BN>(ph, p.ld, p.n, p.D, b0, 0, vb[0], threadIdx.x);
-        }
-        uint32_t it = 0;
-        bool ok = true;
-        auto step = [&](int64_t kc, float4 (&ca)[kBM / 16], float4 (&cb)[BN / 16], float4 (&na)[kBM / 16],
-                        float4 (&nb)[BN / 16]) {
-            const int s = it % C::kStages;
-            const uint32_t phz = (it / C::kStages) & 1u;
-            if (kc + 1 < nkc) {
-                load_t<kBM>(ph, p.ld, p.n, p.D, a0, (kc + 1) * kKC, na, threadIdx.x);
-                load_t<BN>(ph, p.ld, p.n, p.D, b0, (kc + 1) * kKC, nb, threadIdx.x);
-            }
+        // ---------------- split warps: raw chunk (transposed reads) -> hi/lo operand stage
+        const int pt = threadIdx.x;
+        float4 va[8], vb[8];
+        for (int64_t kc = 0; kc < nkc; ++kc) {
+            const int r = (int)(kc % C::kRawStages), s = (int)(kc % C::kStages);
+            const uint32_t rph = (uint32_t)(kc / C::kRawStages) & 1u, ph = (uint32_t)(kc / C::kStages) & 1u;
             bool got = true;
-            if (lane == 0) got = wait_bounded(smem_u32(&empty[s]), phz ^ 1u, abort, p.err);
+            if (lane == 0) got = wait_bounded(smem_u32(&raw_full[r]), rph, abort, p.err);
             got = __shfl_sync(0xffffffffu, got, 0);
             __syncwarp();
-            if (!got) {
-                ok = false;
-                return;
-            }
+            if (!got) break;
+            const uint8_t* raw = raw0 + (size_t)r * C::kRawBytes;
+            load_raw_t(raw, va, pt);
+            if (!diag) load_raw_t(raw + C::kABytes, vb, pt);
+            __syncwarp();
+            if (lane == 0) mbar_arrive(smem_u32(&raw_empty[r]));
+            if (lane == 0) got = wait_bounded(smem_u32(&empty[s]), ph ^ 1u, abort, p.err);
+            got = __shfl_sync(0xffffffffu, got, 0);
+            __syncwarp();
+            if (!got) break;
             uint8_t* st = smem + (size_t)s * C::kStageBytes;
-            store_split_t<kBM>(ca, st, st + C::kABytes, threadIdx.x);
-            store_split_t<BN>(cb, st + 2 * C::kABytes, st + 2 * C::kABytes + C::kBBytes, threadIdx.x);
+            store_split_t<kBM>(va, st, st + C::kABytes, pt);
+            if (!diag) store_split_t<BN>(vb, st + 2 * C::kABytes, st + 3 * C::kABytes, pt);
             fence_proxy_async();
             __syncwarp();
             if (lane == 0) mbar_arrive(smem_u32(&full[s]));
-            ++it;
-        };
-        for (int64_t kc = 0; ok && kc < nkc; kc += 2) {
-            step(kc, va[0], vb[0], va[1], vb[1]);
-            if (ok && kc + 1 < nkc) step(kc + 1, va[1], vb[1], va[0], vb[0]);
         }
-    } else {
-        if (warp == 4 && lane == 0) {
-            const uint32_t idesc = idesc_tf32(kBM, BN);
-            uint32_t it = 0;
-            bool ok = true;
-            for (int64_t kc = 0; kc < nkc; ++kc, ++it) {
-                const int s = it % C::kStages;
-                const uint32_t phz = (it / C::kStages) & 1u;
-                if (!wait_bounded(smem_u32(&full[s]), phz, abort, p.err)) {
-                    ok = false;
-                    break;
+    } else if (warp == 9) {
+        if (lane == 0) {
+            // ---------------- TMA producer: raw chunks of 32 examples, features a0.. (and b0..)
+            const int xa = (int)(layer * p.D + a0), xb = (int)(layer * p.D + b0);
+            const uint32_t bytes = diag ? C::kABytes : C::kRawBytes;
+            uint32_t last_par[C::kRawStages];
+            bool issued[C::kRawStages];
+            for (int r = 0; r < C::kRawStages; ++r) issued[r] = false;
+            for (int64_t kc = 0; kc < nkc; ++kc) {
+                const int r = (int)(kc % C::kRawStages);
+                const uint32_t rph = (uint32_t)(kc / C::kRawStages) & 1u;
+                if (!wait_bounded(smem_u32(&raw_empty[r]), rph ^ 1u, abort, p.err)) break;
+                const uint32_t dst = smem_u32(raw0 + (size_t)r * C::kRawBytes), bar = smem_u32(&raw_full[r]);
+                const int y = (int)(kc * kKC);
+                mbar_arrive_tx(bar, bytes);
+#pragma unroll
+                for (int b = 0; b < 4; ++b) tma_load_2d(dst + (uint32_t)b * 4096u, &tm, xa + 32 * b, y, bar);
+                if (!diag)
+#pragma unroll
+                    for (int b = 0; b < 4; ++b)
+                        tma_load_2d(dst + C::kABytes + (uint32_t)b * 4096u, &tm, xb + 32 * b, y, bar);
+                issued[r] = true;
+                last_par[r] = rph;
+            }
+            // copies still in flight when the consumers stopped early land before the CTA exits
+            for (int r = 0; r < C::kRawStages; ++r)
+                if (issued[r]) {
+                    const uint64_t t0 = global_ns();
+                    while (!mbar_try_wait(smem_u32(&raw_full[r]), last_par[r]))
+                        if (global_ns() - t0 > kTimeoutNs) {
+                            atomicOr(p.err, kErrTimeout);
+                            break;
+                        }
                 }
+        }
+    } else if (warp == 8) {
+        if (lane == 0) {
+            // ---------------- MMA issuer
+            const uint32_t idesc = idesc_tf32(kBM, BN);
+            for (int64_t kc = 0; kc < nkc; ++kc) {
+                const int s = (int)(kc % C::kStages);
+                const uint32_t ph = (uint32_t)(kc / C::kStages) & 1u;
+                const int64_t g = kc / C::kGroup;  // group g goes to accumulator g % kAcc, its use g / kAcc
+                const int a = (int)(g % C::kAcc);
+                const bool start = kc % C::kGroup == 0;
+                if (start && g >= C::kAcc &&
+                    !wait_bounded(smem_u32(&acc_empty[a]), (uint32_t)((g / C::kAcc) - 1) & 1u, abort, p.err))
+                    break;
+                if (!wait_bounded(smem_u32(&full[s]), ph, abort, p.err)) break;
                 tc_fence_after();
                 const uint32_t st = smem_u32(smem + (size_t)s * C::kStageBytes);
                 const uint64_t ahi = sw128_desc(st), alo = sw128_desc(st + C::kABytes);
-                const uint64_t bhi = sw128_desc(st + 2 * C::kABytes), blo = sw128_desc(st + 2 * C::kABytes + C::kBBytes);
+                const uint64_t bhi = diag ? ahi : sw128_desc(st + 2 * C::kABytes);
+                const uint64_t blo = diag ? alo : sw128_desc(st + 3 * C::kABytes);
+                const uint32_t d = tmem + (uint32_t)a * BN;
 #pragma unroll
                 for (int k = 0; k < kKC / 8; ++k) {
-                    const uint32_t d = tmem + (it % C::kAcc) * BN;
-                    const uint32_t first = (it < (uint32_t)C::kAcc && k == 0) ? 0u : 1u;
-                    mma_tf32(d, ahi + 2 * k, bhi + 2 * k, idesc, first);
+                    mma_tf32(d, ahi + 2 * k, bhi + 2 * k, idesc, (start && k == 0) ? 0u : 1u);
                     mma_tf32(d, ahi + 2 * k, blo + 2 * k, idesc, 1u);
                     mma_tf32(d, alo + 2 * k, bhi + 2 * k, idesc, 1u);
                 }
                 mma_commit(smem_u32(&empty[s]));
+                if (kc % C::kGroup == C::kGroup - 1 || kc == nkc - 1) mma_commit(smem_u32(&acc_full[a]));
             }
-            if (ok) mma_commit(smem_u32(tfull));
             mma_commit(smem_u32(mma_done));
             const uint64_t t0 = global_ns();
             while (!mbar_try_wait(smem_u32(mma_done), 0))
@@ -504,41 +550,71 @@ __global__ void __launch_bounds__(kThreads, 1) fit3x_kernel(const FParams p) {
                     break;
                 }
         }
-        __syncwarp();
+    } else {
+        // ---------------- epilogue (warps 4-7): drain each group's accumulator into fp32
+        // registers (one row of the tile per thread), then M += the sum
         const int q = warp & 3;
         const int row = q * 32 + lane;
-        bool got = true;
-        if (lane == 0) got = wait_bounded(smem_u32(tfull), 0, abort, p.err);
-        got = __shfl_sync(0xffffffffu, got, 0);
-        if (!epi_any(!got)) {
+        const uint32_t tbase = tmem + ((uint32_t)(q * 32) << 16);
+        const int64_t ngroups = (nkc + C::kGroup - 1) / C::kGroup;
+        float acc[BN];
+#pragma unroll
+        for (int c = 0; c < BN; ++c) acc[c] = 0.f;
+        bool ok = true;
+        for (int64_t g = 0; g < ngroups; ++g) {
+            const int a = (int)(g % C::kAcc);
+            bool got = true;
+            if (lane == 0) got = wait_bounded(smem_u32(&acc_full[a]), (uint32_t)(g / C::kAcc) & 1u, abort, p.err);
+            got = __shfl_sync(0xffffffffu, got, 0);
+            if (!got) {
+                ok = false;
+                break;
+            }
             tc_fence_after();
-            const uint32_t tbase = tmem + ((uint32_t)(q * 32) << 16);
-            const int used = (int)(nkc < C::kAcc ? nkc : C::kAcc);
-            const int64_t a = a0 + row;
-            float* M = (float*)(p.state + (size_t)layer * p.bytes + 64);
 #pragma unroll
             for (int c0 = 0; c0 < BN; c0 += 16) {
-                float acc[16];
+                float v[16];
+                tmem_ld16(tbase + (uint32_t)(a * BN + c0), v);
 #pragma unroll
-                for (int i = 0; i < 16; ++i) acc[i] = 0.f;
-                for (int u = 0; u < used; ++u) {
-                    float v[16];
-                    tmem_ld16(tbase + u * BN + c0, v);
-#pragma unroll
-                    for (int i = 0; i < 16; ++i) acc[i] += v[i];
-                }
-                if (a < p.D)
-#pragma unroll
-                    for (int i = 0; i < 16; ++i) {
-                        const int64_t b = b0 + c0 + i;
-                        if (b < p.D) M[a * p.D + b] += acc[i];
-                    }
+                for (int i = 0; i < 16; ++i) acc[c0 + i] += v[i];
             }
             tc_fence_before();
+            __syncwarp();
+            if (lane == 0) mbar_arrive(smem_u32(&acc_empty[a]));
+        }
+        // the tile's sums to shared memory (the operand stages are free once the last group
+        // has landed: every stage was consumed by its MMAs), row stride 129: conflict-free
+        if (ok) {
+            float* stg = (float*)smem;
+#pragma unroll
+            for (int c = 0; c < BN; ++c) stg[row * (BN + 1) + c] = acc[c];
         }
     }
     tc_fence_before();
     __syncthreads();
+    if (!*abort) {
+        // M += tile, coalesced: warp w takes rows 4j..4j+3 for j = w, w + 10, ..., lane the
+        // columns lane + 32i; all 16 old values of a batch are loaded before any store
+        const float* stg = (const float*)smem;
+        float* M = (float*)(p.state + (size_t)layer * p.bytes + 64);
+        for (int j = warp; j < kBM / 4; j += kFitThreads / 32) {
+            float old[4][BN / 32];
+#pragma unroll
+            for (int r = 0; r < 4; ++r)
+#pragma unroll
+                for (int i = 0; i < BN / 32; ++i) {
+                    const int64_t a = a0 + 4 * j + r, b = b0 + lane + 32 * i;
+                    old[r][i] = (a < p.D && b < p.D) ? M[a * p.D + b] : 0.f;
+                }
+#pragma unroll
+            for (int r = 0; r < 4; ++r)
+#pragma unroll
+                for (int i = 0; i < BN / 32; ++i) {
+                    const int64_t a = a0 + 4 * j + r, b = b0 + lane + 32 * i;
+                    if (a < p.D && b < p.D) M[a * p.D + b] = old[r][i] + stg[(4 * j + r) * (BN + 1) + lane + 32 * i];
+                }
+        }
+    }
     if (warp == 4) {
         tc_fence_after();
         tmem_dealloc(tmem, C::kTmemCols);
@@ -696,32 +772,37 @@ cudaError_t launch_score_tc_slices(const float* Qhat, int64_t n_q, int64_t ld_q,
     return launch_bn<128>(p, s);
 }
 
-bool fit_tc_supported(int64_t D, const float* phi, int64_t ld) {
+bool fit_tc_supported(int n_layers, int64_t D, const float* phi, int64_t n, int64_t ld) {
     int dev = 0, major = 0, minor = 0;
     cudaGetDevice(&dev);
     cudaDeviceGetAttribute(&major, cudaDevAttrComputeCapabilityMajor, dev);
     cudaDeviceGetAttribute(&minor, cudaDevAttrComputeCapabilityMinor, dev);
-    if (!(major == 10 && minor == 3)) return false;
-    return D >= 128 && (D & 3) == 0 && (ld & 3) == 0 && ((uintptr_t)phi & 15) == 0;
+    if (!(major == 10 && minor == 3) || !encode_fn()) return false;
+    // TMA: 32-bit coordinates, 16-byte aligned base and row stride below 2^40 bytes, feature
+    // coordinates a multiple of 4 (every tile starts at l*D + 128*j)
+    if (D < 128 || (D & 3) || (ld & 3) || ((uintptr_t)phi & 15)) return false;
+    if ((int64_t)n_layers * D >= (1LL << 31) || n >= (1LL << 31) - kKC || ld * 4 >= (1LL << 40)) return false;
+    return true;
 }
 
 cudaError_t launch_fit_tc(int n_layers, int64_t D, void* state, size_t state_bytes, const float* phi, int64_t n,
                           int64_t ld, unsigned int* err, cudaStream_t s) {
-    using C = GCfg<128>;
+    using C = FCfg;
     const int64_t nt = (D + kBM - 1) / kBM;
+    // features of all layers, examples as rows; zero fill past the last layer's features and the last example
+    CUtensorMap tm;
+    if (!make_map_f32(&tm, phi, n, (int64_t)n_layers * D, ld, kKC)) return cudaErrorInvalidValue;
     FParams p{};
-    p.phi = phi;
     p.state = (char*)state;
     p.bytes = state_bytes;
     p.D = D;
     p.n = n;
-    p.ld = ld;
     p.tiles = (int)(nt * (nt + 1) / 2);
     p.err = err;
     cudaError_t e = cudaFuncSetAttribute(fit3x_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)C::kSmem);
     if (e != cudaSuccess) return e;
     note_launches(1);
-    fit3x_kernel<<<(unsigned)(p.tiles * n_layers), kThreads, C::kSmem, s>>>(p);
+    fit3x_kernel<<<(unsigned)(p.tiles * n_layers), kFitThreads, C::kSmem, s>>>(tm, p);
     return cudaGetLastError();
 }
 

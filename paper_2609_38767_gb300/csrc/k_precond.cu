@@ -602,16 +602,28 @@ __global__ void __launch_bounds__(256, 1) factor_cluster_kernel(St<float> st, in
             }
     }
     cluster_barrier();
+    static_assert(CS >= 2, "rank 0 factors the next diagonal block while the others update");
     for (int64_t k0 = 0; k0 < D; k0 += kNB) {
-        // ---- diagonal block: factored in registers by warp 0 of every CTA
-        for (int e = tid; e < kNB * kNB; e += blockDim.x) {
-            const int i = e / kNB, j = e % kNB;
-            Lk[i][j] = (j <= i) ? __ldcg(M + (k0 + i) * D + k0 + j) : 0.f;
-        }
-        __syncthreads();
-        if (tid < 32) {
-            const int bad = warp_cholesky32(Lk, LkT, dinv, lane);
-            if (rank == 0 && lane == 0 && bad >= 0 && h[kPcFailedPivot] == 0.0) h[kPcFailedPivot] = (double)(k0 + bad + 1);
+        // ---- diagonal block. The first is factored in registers by warp 0 of every CTA; each
+        // later one was factored by rank 0 during the previous step's trailing update (look-
+        // ahead: it lies in that update's first tile), which rank 0 keeps in LkT / dinv and the
+        // others read back from M's diagonal block and the block's slot of Dinv
+        if (k0 == 0) {
+            for (int e = tid; e < kNB * kNB; e += blockDim.x) {
+                const int i = e / kNB, j = e % kNB;
+                Lk[i][j] = (j <= i) ? __ldcg(M + (k0 + i) * D + k0 + j) : 0.f;
+            }
+            __syncthreads();
+            if (tid < 32) {
+                const int bad = warp_cholesky32(Lk, LkT, dinv, lane);
+                if (rank == 0 && lane == 0 && bad >= 0 && h[kPcFailedPivot] == 0.0) h[kPcFailedPivot] = (double)(k0 + bad + 1);
+            }
+        } else if (rank != 0) {
+            for (int e = tid; e < kNB * kNB; e += blockDim.x) {
+                const int i = e / kNB, j = e % kNB;
+                LkT[j][i] = (j <= i) ? __ldcg(M + (k0 + i) * D + k0 + j) : 0.f;
+            }
+            if (tid < kNB) dinv[tid] = __ldcg(st.Dinv(l) + (k0 / kNB) * (kNB * kNB) + tid);
         }
         __syncthreads();
         // ---- panel rows below the block (and the query rows): x L_kk^T = a, every CS-th row
@@ -696,7 +708,7 @@ __global__ void __launch_bounds__(256, 1) factor_cluster_kernel(St<float> st, in
         // the factored block goes back into M's diagonal block once every CTA has read the
         // unfactored one (no later step reads that block); the inverses of all diagonal
         // blocks are formed after the last step
-        if (rank == 0)
+        if (k0 == 0 && rank == 0)
             for (int e = tid; e < kNB * kNB; e += blockDim.x) {
                 const int i = e / kNB, j = e % kNB;
                 if (j <= i) M[(k0 + i) * D + k0 + j] = LkT[j][i];
@@ -748,9 +760,12 @@ __global__ void __launch_bounds__(256, 1) factor_cluster_kernel(St<float> st, in
                                                                                  : 0.f;
                     }
             };
+            // rank 0 takes tile 0 alone (it holds the next diagonal block, factored right after);
+            // ranks 1 .. CS-1 share the others
+            const int64_t ustep = rank == 0 ? tiles : CS - 1;
             int64_t u = rank;
             if (u < tiles) load_tile(u);
-            for (; u < tiles; u += CS) {
+            for (; u < tiles; u += ustep) {
                 const Tile tl = tile_of(u);
 #pragma unroll
                 for (int hh = 0; hh < 8; ++hh) {
@@ -764,7 +779,7 @@ __global__ void __launch_bounds__(256, 1) factor_cluster_kernel(St<float> st, in
 #pragma unroll
                     for (int b = 0; b < 4; ++b) acc[a][b] = mv[a][b];
                 __syncthreads();
-                if (u + CS < tiles) load_tile(u + CS);
+                if (u + ustep < tiles) load_tile(u + ustep);
 #pragma unroll 8
                 for (int m = 0; m < kNB; ++m) {
                     const float4 a4 = *reinterpret_cast<const float4*>(&Pi[m][ty * 4]);
@@ -781,8 +796,24 @@ __global__ void __launch_bounds__(256, 1) factor_cluster_kernel(St<float> st, in
                     for (int v = 0; v < 4; ++v) {
                         const int64_t i = tl.i0 + ty * 4 + q, j = tl.j0 + tx * 4 + v;
                         if (i < tl.lim && j < D && (!tl.tri || j <= i)) tl.rows[i * tl.ld + j] = acc[q][v];
+                        // tile 0's top-left 32 x 32: the next diagonal block, updated (D - s0 >= 32)
+                        if (u == 0 && ty * 4 + q < kNB && tx * 4 + v < kNB)
+                            Lk[ty * 4 + q][tx * 4 + v] = (tx * 4 + v <= ty * 4 + q) ? acc[q][v] : 0.f;
                     }
                 __syncthreads();
+            }
+            if (rank == 0) {
+                // look-ahead: factor the next diagonal block now; the others read it after the barrier
+                if (tid < 32) {
+                    const int bad = warp_cholesky32(Lk, LkT, dinv, lane);
+                    if (lane == 0 && bad >= 0 && h[kPcFailedPivot] == 0.0) h[kPcFailedPivot] = (double)(s0 + bad + 1);
+                }
+                __syncthreads();
+                for (int e = tid; e < kNB * kNB; e += blockDim.x) {
+                    const int i = e / kNB, j = e % kNB;
+                    if (j <= i) M[(s0 + i) * D + s0 + j] = LkT[j][i];
+                }
+                if (tid < kNB) st.Dinv(l)[(s0 / kNB) * (kNB * kNB) + tid] = dinv[tid];
             }
         }
         cluster_barrier();
@@ -997,7 +1028,7 @@ int64_t precondition_apply_max_d(tda_dtype sdt) {
 cudaError_t launch_pc_fit(int n_layers, int64_t D, tda_dtype sdt, void* state, const float* phi, int64_t n,
                           int64_t ld, cudaStream_t s) {
     if (n == 0) return cudaSuccess;
-    if (sdt == TDA_F32 && fit_tc_supported(D, phi, ld)) {
+    if (sdt == TDA_F32 && fit_tc_supported(n_layers, D, phi, n, ld)) {
         unsigned int* err = device_error_word();
         if (err)
             return launch_fit_tc(n_layers, D, state, tda_precondition_state_bytes(D, TDA_F32), phi, n, ld, err, s);

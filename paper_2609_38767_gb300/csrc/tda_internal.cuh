@@ -173,7 +173,7 @@ cudaError_t launch_score(const void* Qhat, tda_dtype qdt, int64_t n_q, int64_t l
                          const float* Phi, int64_t n_t, int64_t ld_phi, int64_t D, float* S,
                          int64_t ld_S, float beta, cudaStream_t s);
 // Fisher fit on tcgen05 (3xTF32) for an fp32 state: M_l += Phi_l^T Phi_l.
-bool fit_tc_supported(int64_t D, const float* phi, int64_t ld);
+bool fit_tc_supported(int n_layers, int64_t D, const float* phi, int64_t n, int64_t ld);
 cudaError_t launch_fit_tc(int n_layers, int64_t D, void* state, size_t state_bytes, const float* phi, int64_t n,
                           int64_t ld, unsigned int* err, cudaStream_t s);
 

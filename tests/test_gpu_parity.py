@@ -360,6 +360,39 @@ def test_precondition_batched_layers_match_oracle(dev, orc, sdt, D, lam_abs, lam
         assert rel_fro(got[:, l * D:(l + 1) * D], ref) <= tol
 
 
+@pytest.mark.parametrize("D,nl,chunks,pad", [(128, 1, (5, 40), 0), (1000, 3, (70, 80, 31), 4),
+                                             (1024, 2, (4096,), 0), (256, 2, (1, 33, 64), 8)])
+def test_fisher_fit_accumulates_phi_t_phi(dev, orc, D, nl, chunks, pad):
+    # FIT_ACCUM on an fp32 state (the tensor-core fit for D >= 128): M_l = sum over the streamed
+    # chunks of Phi_l^T Phi_l, compared on the lower triangle with the oracle's Fisher times N.
+    # Ragged D makes a layer's last tile read the next layer's features (rows past D, discarded);
+    # chunks of 1, 5, 31, 33 examples end inside a 32-example operand chunk; 4096 examples wrap
+    # every pipeline ring many times.
+    rng = np.random.default_rng(D + nl)
+    N = sum(chunks)
+    W = nl * D + pad
+    phi = (rng.standard_normal((N, W)) * rng.uniform(0.5, 2.0, W)).astype(np.float32)
+    sdt = tda.TDA_F32
+    per = tda.tda_precondition_state_bytes(D, sdt)
+    state = torch.empty(nl * per, dtype=torch.uint8, device=dev)
+    phid = torch.from_numpy(phi).to(dev)
+    tda.tda_precondition(tda.TDA_PC_RESET, nl, D, sdt, state)
+    e0 = 0
+    for c in chunks:
+        tda.tda_precondition(tda.TDA_PC_FIT_ACCUM, nl, D, sdt, state, phi=phid[e0:], n=c, ld_phi=W)
+        e0 += c
+    tda.tda_device_status()
+    low = np.tril_indices(D)
+    for l in range(nl):
+        M = state[l * per + 64:l * per + 64 + 4 * D * D].view(torch.float32).view(D, D).cpu().numpy()
+        ref = N * orc.fisher(phi[:, l * D:(l + 1) * D].astype(np.float64))
+        assert np.isfinite(M[low]).all()
+        assert rel_fro(M[low], ref[low]) <= 1e-5
+        # element by element against the Cauchy-Schwarz scale of each entry
+        scale = np.sqrt(np.outer(np.diag(ref), np.diag(ref)))
+        assert (np.abs(M - ref)[low] <= 1e-5 * scale[low]).all()
+
+
 @pytest.mark.parametrize("D,Nq,nl", [(64, 11, 1), (96, 70, 3), (1024, 64, 2), (1000, 9, 1), (128, 300, 1)])
 def test_precondition_factor_apply_matches_oracle(dev, orc, D, Nq, nl):
     # FACTOR_APPLY: one launch for an fp32 state with D a multiple of 32 and <= 256 queries (the
