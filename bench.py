@@ -76,6 +76,8 @@ def parse_args():
                         "on the projected factors (damping 0.1 x mean eigenvalue)")
     p.add_argument("--overlap-sms", type=int, default=0,
                    help="Fisher query side on a second stream; the train projection leaves this many SMs free")
+    p.add_argument("--query-streams", type=int, default=8,
+                   help="streams the query projections of the linears are spread over (device-resident leg)")
     p.add_argument("--e2e-steps", type=int, default=2)
     p.add_argument("--no-e2e", action="store_true")
     p.add_argument("--no-cpu-baseline", action="store_true")
@@ -613,7 +615,7 @@ def main():
     kfac_mode = not args.no_precondition and args.curvature != "fisher"
     pipe = BlockPipeline([(di, do) for _, di, do in LINEARS], T, k, N, Nq, topk=args.topk,
                          precondition=not args.no_precondition, lambda_rel=0.1 if kfac_mode else 1e-2, device=dev,
-                         curvature=args.curvature)
+                         curvature=args.curvature, query_streams=args.query_streams)
     layers, Phi, Q, idx, val = pipe.layers, pipe.Phi, pipe.Q, pipe.idx, pipe.val
     select = shard.device_select(tda)
     torch.cuda.synchronize()
@@ -777,6 +779,9 @@ def main():
                     tda.tda_project_host(L, tda.TDA_BF16, a, b, n, phi[e0:], ld, ws, wsb)
             else:
                 tda.tda_project_host(L, tda.TDA_BF16, qa, qb, Nq, phi, ld, ws, wsb)
+
+        # host-streamed projections share the staging workspace: one query stream
+        pipe.query_streams = 1
 
         def e2e_step():
             attribute(project_host)

@@ -27,8 +27,10 @@ class BlockPipeline:
     CURVATURES = ("fisher", "kfac", "ekfac")
 
     def __init__(self, linears, T, k, n_train, n_query, *, topk=100, precondition=True,
-                 lambda_abs=0.0, lambda_rel=1e-2, seed=0, layer0=0, device="cuda", curvature="fisher"):
+                 lambda_abs=0.0, lambda_rel=1e-2, seed=0, layer0=0, device="cuda", curvature="fisher",
+                 query_streams=8):
         assert curvature in self.CURVATURES
+        self.query_streams = query_streams
         self.layers = [tda.LayerDesc(di, do, T, k, k, seed=seed, layer=layer0 + i)
                        for i, (di, do) in enumerate(linears)]
         self.N, self.Nq, self.D = n_train, n_query, k * k
@@ -92,8 +94,7 @@ class BlockPipeline:
             if after_train_linear:
                 after_train_linear(li)
         mark("project_query")
-        for li, L in enumerate(self.layers):
-            project_query(li, L, routes[li], self.Q[:, li * D:], DT)
+        self._project_queries(project_query, routes)
         target = self.Q
         if kfac:
             k = self.k
@@ -128,6 +129,29 @@ class BlockPipeline:
                                  q=self.Q, n_q=self.Nq, ld_q=DT, qhat=self.Qh, ld_qhat=DT)
             target = self.Qh
         self._score(target, mark)
+
+    def _project_queries(self, project_query, routes):
+        """The query projections of all linears. A query batch is smaller than the GPU (64
+        examples fill 128 of 152 SMs), so the linears go out on query_streams streams at once
+        and the later launches fill the SMs the earlier ones leave idle; every launch writes
+        its own feature columns, so the results do not depend on the order."""
+        D, DT = self.D, self.DT
+        n = min(self.query_streams, self.nl)
+        if n <= 1 or not torch.cuda.is_available():
+            for li, L in enumerate(self.layers):
+                project_query(li, L, routes[li], self.Q[:, li * D:], DT)
+            return
+        main = torch.cuda.current_stream()
+        if len(getattr(self, "_qstreams", ())) < n:
+            self._qstreams = [torch.cuda.Stream(device=main.device) for _ in range(n)]
+        streams = self._qstreams[:n]
+        for s in streams:
+            s.wait_stream(main)
+        for li, L in enumerate(self.layers):
+            with torch.cuda.stream(streams[li % n]):
+                project_query(li, L, routes[li], self.Q[:, li * D:], DT)
+        for s in streams:
+            main.wait_stream(s)
 
     def _score(self, target, mark):
         DT = self.DT
