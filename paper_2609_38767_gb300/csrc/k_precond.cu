@@ -452,8 +452,10 @@ __device__ __forceinline__ uint32_t cluster_ctarank() {
     asm volatile("mov.u32 %0, %%cluster_ctarank;" : "=r"(r));
     return r;
 }
+// release / acquire at cluster scope order every earlier global and shared access of
+// the arriving threads before every later access of the waiting ones: the data the CTAs
+// exchange through M (read back with ld.global.cg) needs no separate device-wide fence
 __device__ __forceinline__ void cluster_barrier() {
-    __threadfence();
     asm volatile("barrier.cluster.arrive.release.aligned;\n barrier.cluster.wait.acquire.aligned;" ::: "memory");
 }
 
