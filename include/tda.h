@@ -269,7 +269,10 @@ tda_status tda_cosine(float* S, int64_t n_q, int64_t n_t, int64_t ld_S, const fl
  * passes the global n_total to FACTOR. The ops, in order of use:
  *   TDA_PC_RESET      zero the state.
  *   TDA_PC_FIT_ACCUM  M_l += Phi_l^T Phi_l over n feature rows. Call once per
- *                     streamed chunk of training features.
+ *                     streamed chunk of training features. Only the lower
+ *                     triangle (column <= row) of M_l is guaranteed (FACTOR
+ *                     reads nothing else); an F32 state accumulates in fp32
+ *                     from 3xTF32 tensor-core products for D >= 128.
  *   TDA_PC_FACTOR     F_l = M_l / n_total; lambda_l = lambda_abs +
  *                     lambda_rel_mean_eig * tr(F_l)/D; factor F_l + lambda_l I
  *                     = L L^T (Cholesky) into the state. A non-positive pivot
