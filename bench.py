@@ -717,6 +717,9 @@ def main():
 
     # ---- every phase of the step against its own ceiling
     alu = 152 * 128 * 2 * float(peaks.get("sm_max_mhz", 2070.0)) * 1e6 / 1e12  # fp32 FMA TFLOP/s
+    # 3xTF32 on the tensor cores: the sustained bf16 peak x the nominal tf32/bf16 ratio (1/2), three
+    # MMAs per fp32 product: the ceiling in useful fp32 flops of the fit and the score
+    tf32x3 = float(peaks.get("bf16_tflops_sustained", 1700.0)) * 0.5 / 3.0
     ph = {}
     for (name, e0), (_, e1) in zip(phase_ev, phase_ev[1:]):
         if name is not None:
@@ -725,13 +728,13 @@ def main():
     per_unit = {
         "project_train": ("hbm", sum(N * (T * (L.d_in + L.d_out) * 2 + 4 * D) for L in layers), hbm, "GB/s"),
         "project_query": ("hbm", sum(Nq * (T * (L.d_in + L.d_out) * 2 + 4 * D) for L in layers), hbm, "GB/s"),
-        "fisher_fit": ("alu", nl * N * Dn * (Dn + 1), alu, "TFLOP/s"),
+        "fisher_fit": ("tensor", nl * N * Dn * (Dn + 1), tf32x3, "TFLOP/s"),
         "factor": ("latency", nl * Dn ** 3 / 3, alu, "TFLOP/s"),
         "apply": ("latency", (nl * 4 * 2 * Dn * k * Nq) if kfac_mode else (nl * 2 * 2 * Dn * Dn * Nq), alu, "TFLOP/s"),
         "factor_apply": ("latency", nl * (Dn ** 3 / 3 + 2 * 2 * Dn * Dn * Nq), alu, "TFLOP/s"),
         "kfac_eigen": ("latency", nl * 2 * 10 * 4.0 * k ** 3, alu, "TFLOP/s"),
         "ekfac_eigenvalues": ("alu", nl * N * 2 * 2 * Dn * k, alu, "TFLOP/s"),
-        "score": ("alu", 2.0 * Nq * N * DT, alu, "TFLOP/s"),
+        "score": ("tensor", 2.0 * Nq * N * DT, tf32x3, "TFLOP/s"),
         "topk": ("latency", 8.0 * Nq * N * 4, hbm, "GB/s"),
         # sharded job: the curvature sums added over the ranks (NCCL all-reduce)
         "curvature_allreduce": ("latency", (nl * D * D * 4) if not kfac_mode else (nl * 2 * k * k * 8), hbm, "GB/s"),
