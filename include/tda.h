@@ -140,7 +140,7 @@ tda_status tda_project(const tda_layer_desc* L, tda_dtype dtype, const void* A, 
 
 /* Which kernel tda_project (route FACTORED) would run for these arguments on
  * the current device: 1 = the tcgen05/TMA tensor-core kernel (bf16, k_in ==
- * k_out in {16, 32, 64}, sm_103), 0 = the CUDA-core kernel, negative = the
+ * k_out in {16, 32, 64, 128}, sm_103), 0 = the CUDA-core kernel, negative = the
  * arguments are invalid. Host only; for tests and benchmark reports. */
 int32_t tda_project_engine(const tda_layer_desc* L, tda_dtype dtype, const void* A, const void* B);
 

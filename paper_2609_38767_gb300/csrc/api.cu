@@ -310,7 +310,7 @@ tda_status tda_project(const tda_layer_desc* L, tda_dtype dtype, const void* A, 
     if (N == 0) return TDA_OK;
     if (L->T == 0) return cuda_check(cudaMemset2DAsync(phi, ld_phi * 4, 0, D * 4, N, s), "zero phi");
     if (route == TDA_ROUTE_FACTORED) {
-        if (dtype == TDA_BF16 && project_tc_supported(*L, A, B)) {
+        if (dtype == TDA_BF16 && project_tc_plain_supported(*L, A, B)) {
             unsigned int* err = device_error_word();
             if (!err) return fail(TDA_ERR_CUDA, "cannot resolve the device error word");
             return cuda_check(launch_project_tc(*L, A, B, N, phi, ld_phi, err, s), "project (tcgen05)");
@@ -331,7 +331,7 @@ tda_status tda_project(const tda_layer_desc* L, tda_dtype dtype, const void* A, 
 int32_t tda_project_engine(const tda_layer_desc* L, tda_dtype dtype, const void* A, const void* B) {
     g_msg[0] = 0;
     if (validate_layer(L, true) || validate_factors(L, dtype, A, B, 1, "tda_project_engine")) return -1;
-    return (dtype == TDA_BF16 && project_tc_supported(*L, A, B)) ? 1 : 0;
+    return (dtype == TDA_BF16 && project_tc_plain_supported(*L, A, B)) ? 1 : 0;
 }
 
 tda_status tda_similarity_exact(const tda_layer_desc* L, tda_dtype dtype, const void* Aq,

@@ -22,9 +22,16 @@
 // generating them once for G tiles halves the generators' work and the MMA
 // commits per byte streamed.
 //
-// The kernel streams every factor byte once from HBM; at k <= 64 its
-// arithmetic intensity (~k flop/B) is far below the tensor-core ridge, so it
-// is HBM-bound and the pipeline is sized for bytes in flight.
+// The kernel streams every factor byte once from HBM; its arithmetic
+// intensity (~k flop/B, k <= 128) is below the tensor-core ridge, so it is
+// HBM-bound and the pipeline is sized for bytes in flight.
+//
+// k = 128 (K = 128): At | Bt of one tile fill 256 TMEM columns, so the two
+// accumulator buffers take all 512 and a stage holds one token tile; the
+// epilogue stages and contracts the tile's tokens in two 64-row halves (the
+// fp32 rows of a whole tile would leave too little shared memory for the
+// stage ring), and at most 2-CTA clusters share an example (their partial
+// K x K blocks are reduced inside the leader's staging rows).
 //
 // Warp roles (256 threads, one persistent CTA per SM):
 //   warp 0  TMA producer: 128x64 bf16 factor tiles into the stage ring
@@ -55,9 +62,14 @@ constexpr int kMaxStages = 12;
 
 template <int K, int G>
 struct Cfg {
+    static constexpr int kK = K;
     static constexpr uint32_t kSignBytes = K * 128;                       // K rows x 128 bytes
     static constexpr uint32_t kStageBytes = G * kTileBytes + kSignBytes;  // G factor tiles, then signs
     static constexpr int kStageLd = K + 4;                                // padded fp32 staging row
+    // K = 128: the fp32 rows of a whole tile (2 x 128 x 132 floats) would crowd out the
+    // stage ring, so the epilogue stages and contracts 64 token rows at a time
+    static constexpr bool kHalf = K > 64;
+    static constexpr int kStageRows = kHalf ? kTileM / 2 : kTileM;
     static constexpr int kAccCols = 2 * K;                                // At | Bt of one tile
     static constexpr int kBufCols = G * kAccCols;                         // one accumulator buffer
     // tcgen05.alloc takes a power of two from 32 to 512 columns
@@ -66,16 +78,20 @@ struct Cfg {
                                           : 2 * kBufCols <= 128 ? 128
                                           : 2 * kBufCols <= 256 ? 256
                                                                 : 512;
-    static constexpr size_t kSmemStage = 2ull * kTileM * kStageLd * 4;
+    static constexpr size_t kSmemStage = 2ull * kStageRows * kStageLd * 4;
+    // a cluster of cs CTAs reduces cs - 1 partial K x K blocks inside the leader's staging rows
+    static constexpr int kMaxCs = (int)(2 * kStageRows * kStageLd / (K * K)) + 1;
     static constexpr size_t kSmemBarsMax = 8 * (3 * kMaxStages + 7) + 16;
     static constexpr int kFit = (int)((kSmemMax - 1024 - kSmemStage - kSmemBarsMax) / kStageBytes);
     static constexpr int kStages = kFit > kMaxStages ? kMaxStages : kFit;
     static constexpr size_t kSmemBars = 8 * (3 * kStages + 7) + 16;
-    static constexpr size_t kSmem = 1024 + (size_t)kStages * kStageBytes + kSmemStage + kSmemBars;
+    static constexpr size_t kBarsOff = (size_t)kStages * kStageBytes + kSmemStage;  // after ring and staging
+    static constexpr size_t kSmem = 1024 + kBarsOff + kSmemBars;
     // contraction blocking: 16 row groups x 8 column groups of threads
     static constexpr int RB = K / 16 > 0 ? K / 16 : 1;
     static constexpr int CB = K / 8;
     static_assert(kStages >= 3 && kSmem <= kSmemMax, "shared memory per CTA");
+    static_assert(!kHalf || G == 1, "K = 128 fills TMEM with one double-buffered tile");
     static_assert(kStageBytes % 1024 == 0 && 2 * kBufCols <= (int)kTmemCols && kTmemCols <= 512,
                   "operand alignment / TMEM columns");
 };
@@ -147,6 +163,59 @@ __device__ __forceinline__ void write_sign_half(uint8_t* tile, int n, uint64_t w
     }
 }
 
+// Phi of example n (K x K partial sums in acc, thread et holding rows
+// rg*RB.. and columns cg*CB..) is complete in every CTA of the cluster: reduce
+// the members' blocks into the leader (rank 0) over distributed shared memory
+// and write it, scaled. The leader's staging rows (free between tiles) receive
+// member r's block at offset (r-1)*K*K floats, thread-major.
+template <class C>
+__device__ __forceinline__ bool store_phi(float (&acc)[C::RB][C::CB], int64_t n, const Params& p, uint32_t crank,
+                                          float* stage, uint64_t* red_go, uint64_t* red_full, uint32_t& red_use,
+                                          volatile int* abort, int et, int lane) {
+    constexpr int K = C::kK;
+    const int rg = et >> 3, cg = et & 7;
+    if (p.cs > 1) {
+        constexpr int kPer = C::RB * C::CB;
+        const uint32_t slot = smem_u32(stage) + (uint32_t)(et * kPer) * 4u;
+        bool got = true;
+        if (crank == 0) {
+            if (et == 0)
+                for (int r = 1; r < p.cs; ++r) mbar_arrive_remote(smem_u32(red_go), (uint32_t)r);
+            if (lane == 0) got = wait_bounded_cluster(smem_u32(red_full), red_use & 1u, abort, p.err);
+            got = __shfl_sync(0xffffffffu, got, 0);
+            if (epi_any(!got)) return false;
+            for (int r = 1; r < p.cs; ++r) {
+                const float* part = stage + (r - 1) * K * K + et * kPer;
+#pragma unroll
+                for (int a = 0; a < C::RB; ++a)
+#pragma unroll
+                    for (int c = 0; c < C::CB; ++c) acc[a][c] += part[a * C::CB + c];
+            }
+            epi_sync();  // partials consumed; staging free for the next tile
+        } else {
+            if (lane == 0) got = wait_bounded_cluster(smem_u32(red_go), red_use & 1u, abort, p.err);
+            got = __shfl_sync(0xffffffffu, got, 0);
+            if (epi_any(!got)) return false;
+            const uint32_t dst = map_rank(slot, 0) + (crank - 1) * (uint32_t)(K * K) * 4u;
+#pragma unroll
+            for (int a = 0; a < C::RB; ++a)
+#pragma unroll
+                for (int c = 0; c < C::CB; ++c) st_cluster_f32(dst + (uint32_t)(a * C::CB + c) * 4u, acc[a][c]);
+            fence_acq_rel_cluster();
+            epi_sync();
+            if (et == 0) mbar_arrive_remote(smem_u32(red_full), 0u);
+        }
+        ++red_use;
+        if (crank != 0) return true;
+    }
+    float* out = p.phi + n * p.ld_phi;
+#pragma unroll
+    for (int a = 0; a < C::RB; ++a)
+#pragma unroll
+        for (int c = 0; c < C::CB; ++c) out[(rg * C::RB + a) * K + cg * C::CB + c] = acc[a][c] * p.scale;
+    return true;
+}
+
 // KF: also accumulate the K-FAC factor covariances. FO: write the projected
 // factors At, Bt of every token instead of contracting them into Phi.
 template <int K, int G, bool KF, bool FO>
@@ -157,9 +226,9 @@ project_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant
     extern __shared__ uint8_t smem_raw[];
     uint8_t* smem = (uint8_t*)(((uintptr_t)smem_raw + 1023) & ~(uintptr_t)1023);
     uint8_t* sA = smem;                           // kStages x [G factor tiles | sign tile]
-    float* stX = (float*)(sA + (size_t)C::kStages * C::kStageBytes);  // [128][K+4] At rows
-    float* stY = stX + kTileM * C::kStageLd;      // [128][K+4] Bt rows
-    uint64_t* bars = (uint64_t*)(stY + kTileM * C::kStageLd);
+    float* stX = (float*)(sA + (size_t)C::kStages * C::kStageBytes);  // [128 or 64][K+4] At rows
+    float* stY = stX + C::kStageRows * C::kStageLd;  // [128 or 64][K+4] Bt rows
+    uint64_t* bars = (uint64_t*)(smem + C::kBarsOff);
     uint64_t* full = bars;                        // TMA landed        (count 1 + tx)
     uint64_t* sready = bars + C::kStages;         // signs written     (count 2)
     uint64_t* empty = bars + 2 * C::kStages;      // MMAs done reading (count 1)
@@ -313,6 +382,72 @@ project_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant
                 __syncwarp();
                 if (lane == 0) mbar_arrive(smem_u32(&sready[s]));
             }
+    } else if (C::kHalf && warp >= 4) {
+        // ---------------- epilogue for K = 128 (one example per tile, one tile per group):
+        // token rows 0-63 (TMEM lane quadrants 0, 1), then rows 64-127 (quadrants 2, 3),
+        // each staged in shared memory and contracted, Phi += Bt^T At, in fp32. The
+        // accumulators live for one example (the loop nest keeps them within the
+        // register budget: 128 per thread).
+        const int q = warp & 3;
+        const int et = threadIdx.x - 128;
+        const int rg = et >> 3, cg = et & 7;
+        uint32_t grp = 0, red_use = 0;
+        bool ok = true;
+        int ng = it.take<G>(p, ncl, crank, gx, gt);
+        while (ok && ng > 0) {
+            const int64_t cur = gx[0];
+            float acc[C::RB][C::CB];
+#pragma unroll
+            for (int a = 0; a < C::RB; ++a)
+#pragma unroll
+                for (int c = 0; c < C::CB; ++c) acc[a][c] = 0.f;
+            do {
+                const uint32_t b = grp & 1u, use = grp >> 1;
+                bool got = true;
+                if (lane == 0) got = wait_bounded(smem_u32(&tfull[b]), use & 1u, abort, p.err);
+                got = __shfl_sync(0xffffffffu, got, 0);
+                if (epi_any(!got)) {
+                    ok = false;
+                    break;
+                }
+                tc_fence_after();
+                const uint32_t tbase = tmem + ((uint32_t)(q * 32) << 16) + b * C::kBufCols;
+                for (int h = 0; h < 2; ++h) {
+                    if ((q >> 1) == h) {
+                        const int srow = (q & 1) * 32 + lane;
+#pragma unroll 4
+                        for (int c0 = 0; c0 < 2 * K; c0 += 16) {
+                            float v[16];
+                            tmem_ld16(tbase + c0, v);
+                            float* dst = c0 < K ? stX + srow * C::kStageLd + c0 : stY + srow * C::kStageLd + (c0 - K);
+#pragma unroll
+                            for (int i = 0; i < 16; i += 4)
+                                *reinterpret_cast<float4*>(dst + i) = make_float4(v[i], v[i + 1], v[i + 2], v[i + 3]);
+                        }
+                        tc_fence_before();
+                        __syncwarp();
+                        if (lane == 0) mbar_arrive(smem_u32(&tempty[b]));
+                    }
+                    epi_sync();
+#pragma unroll 1
+                    for (int t = 0; t < C::kStageRows; ++t) {
+                        float y[C::RB], x[C::CB];
+#pragma unroll
+                        for (int a = 0; a < C::RB; ++a) y[a] = stY[t * C::kStageLd + rg * C::RB + a];
+#pragma unroll
+                        for (int c = 0; c < C::CB; ++c) x[c] = stX[t * C::kStageLd + cg * C::CB + c];
+#pragma unroll
+                        for (int a = 0; a < C::RB; ++a)
+#pragma unroll
+                            for (int c = 0; c < C::CB; ++c) acc[a][c] = fmaf(y[a], x[c], acc[a][c]);
+                    }
+                    epi_sync();
+                }
+                ++grp;
+                ng = it.take<G>(p, ncl, crank, gx, gt);
+            } while (ng > 0 && gx[0] == cur);
+            if (ok && !store_phi<C>(acc, cur, p, crank, stX, red_go, red_full, red_use, abort, et, lane)) ok = false;
+        }
     } else if (warp >= 4) {
         // ---------------- epilogue: TMEM -> shared -> Phi += Bt^T At
         const int q = warp & 3;          // TMEM lane quadrant of this warp
@@ -642,7 +777,7 @@ cudaError_t launch_kg(const tda_layer_desc& L, const void* A, const void* B, int
     // tiles and reduces the partial features through distributed shared memory.
     int cs = 1;
     if (pack == 1 && N < sms && !FO) cs = (2 * N >= sms) ? 2 : 4;
-    while (cs > 1 && cs > p.n_ttiles) cs >>= 1;
+    while (cs > 1 && (cs > p.n_ttiles || cs > C::kMaxCs)) cs >>= 1;
     p.cs = cs;
     cudaLaunchConfig_t cfg = {};
     cudaLaunchAttribute attr[1];
@@ -676,7 +811,8 @@ cudaError_t launch_kg(const tda_layer_desc& L, const void* A, const void* B, int
 template <int K, bool KF, bool FO>
 cudaError_t launch_k(const tda_layer_desc& L, const void* A, const void* B, int64_t N, float* phi,
                      int64_t ld_phi, unsigned int* err, cudaStream_t s, float* cov, int* grid_out, float* fout) {
-    int pack = L.T <= 64 ? (int)(kTileM / L.T) : 1;
+    // K = 128 keeps one example per tile (its epilogue contracts 64-row halves)
+    int pack = (K <= 64 && L.T <= 64) ? (int)(kTileM / L.T) : 1;
     if (pack > 1) {
         // packed rows are addressed with 32-bit TMA coordinates and the [1][N*T][d]
         // view's outer stride must stay below 2^40 bytes: split larger batches
@@ -698,10 +834,14 @@ cudaError_t launch_k(const tda_layer_desc& L, const void* A, const void* B, int6
             return cudaSuccess;
         }
     }
-    const int64_t units = pack > 1 ? (N + pack - 1) / pack : N * ((L.T + kTileM - 1) / kTileM);
-    if (units >= 4 * (int64_t)sm_count())
-        return launch_kg<K, 2, KF, FO>(L, A, B, N, phi, ld_phi, err, s, pack, cov, grid_out, fout);
-    return launch_kg<K, 1, KF, FO>(L, A, B, N, phi, ld_phi, err, s, pack, cov, grid_out, fout);
+    if constexpr (K > 64) {
+        return launch_kg<K, 1, KF, FO>(L, A, B, N, phi, ld_phi, err, s, pack, cov, grid_out, fout);
+    } else {
+        const int64_t units = pack > 1 ? (N + pack - 1) / pack : N * ((L.T + kTileM - 1) / kTileM);
+        if (units >= 4 * (int64_t)sm_count())
+            return launch_kg<K, 2, KF, FO>(L, A, B, N, phi, ld_phi, err, s, pack, cov, grid_out, fout);
+        return launch_kg<K, 1, KF, FO>(L, A, B, N, phi, ld_phi, err, s, pack, cov, grid_out, fout);
+    }
 }
 
 }  // namespace
@@ -718,6 +858,17 @@ bool project_tc_supported(const tda_layer_desc& L, const void* A, const void* B)
     return true;
 }
 
+// The plain projection also runs k = 128 on the tensor cores (the fused K-FAC
+// covariances and the factor output stay at k <= 64).
+bool project_tc_plain_supported(const tda_layer_desc& L, const void* A, const void* B) {
+    if (L.k_in == 128 && L.k_out == 128) {
+        tda_layer_desc L64 = L;
+        L64.k_in = L64.k_out = 64;
+        return project_tc_supported(L64, A, B);
+    }
+    return project_tc_supported(L, A, B);
+}
+
 cudaError_t launch_project_tc(const tda_layer_desc& L, const void* A, const void* B, int64_t N, float* phi,
                               int64_t ld_phi, unsigned int* err, cudaStream_t s) {
     if (N == 0) return cudaSuccess;
@@ -725,6 +876,7 @@ cudaError_t launch_project_tc(const tda_layer_desc& L, const void* A, const void
         case 16: return launch_k<16, false, false>(L, A, B, N, phi, ld_phi, err, s, nullptr, nullptr, nullptr);
         case 32: return launch_k<32, false, false>(L, A, B, N, phi, ld_phi, err, s, nullptr, nullptr, nullptr);
         case 64: return launch_k<64, false, false>(L, A, B, N, phi, ld_phi, err, s, nullptr, nullptr, nullptr);
+        case 128: return launch_k<128, false, false>(L, A, B, N, phi, ld_phi, err, s, nullptr, nullptr, nullptr);
         default: return cudaErrorNotSupported;
     }
 }

@@ -74,6 +74,7 @@ cudaError_t launch_project_simt(const tda_layer_desc& L, tda_dtype dt, const voi
 // tcgen05 / TMA projection for bf16 inputs. Returns cudaErrorNotSupported if
 // the shape has no tensor-core instantiation (caller falls back to SIMT).
 bool project_tc_supported(const tda_layer_desc& L, const void* A, const void* B);
+bool project_tc_plain_supported(const tda_layer_desc& L, const void* A, const void* B);  // also k = 128
 cudaError_t launch_project_tc_kfac(const tda_layer_desc& L, const void* A, const void* B, int64_t N, float* phi,
                                    int64_t ld_phi, float* cov, int* grid_out, unsigned int* err, cudaStream_t s);
 int project_tc_max_grid();

@@ -270,11 +270,12 @@ def test_route_auto_and_calibration(dev, orc):
 
 
 # ------------------------------------------------------------------ tensor-core projection specifics
-def test_tc_projection_signs_bit_exact(dev, orc):
+@pytest.mark.parametrize("k", [32, 128])
+def test_tc_projection_signs_bit_exact(dev, orc, k):
     # One-hot factors: A_n = I (T = d_in tokens), B_n = e_r at token t only, so
     # Phi_n / scale = outer(S_out[r, :], S_in[t, :]) exactly -- the signs the
     # tensor-core kernel generated on chip, compared bit for bit with the oracle's.
-    d, k, N = 128, 32, 4
+    d, N = 128, 4
     picks = [(0, 5), (77, 127), (127, 64), (31, 0)]  # (t, r) per example
     A = np.zeros((N, d, d), dtype=np.float32)
     B = np.zeros((N, d, d), dtype=np.float32)
@@ -312,6 +313,12 @@ TC_CASES = [
     (20001, 8, 64, 64, 16, "bf16"),     # 16 per tile
     (300, 3, 128, 64, 32, "bf16"),      # 42 per tile
     (1000, 64, 256, 128, 64, "bf16"),   # 2 per tile, K = 64
+    # k = 128: one tile per stage, the epilogue contracts 64-token halves
+    (200, 200, 136, 200, 128, "bf16"),  # persistent loop, ragged K chunks and last tile
+    (5, 384, 256, 128, 128, "bf16"),    # fewer examples than SMs: 2-CTA clusters
+    (1, 200, 64, 64, 128, "bf16"),      # one example over 2 CTAs, ragged second tile
+    (40, 48, 64, 64, 128, "bf16"),      # short sequences stay one example per tile
+    (3, 1, 72, 64, 128, "bf16"),        # T = 1
 ]
 
 
