@@ -82,16 +82,21 @@ struct Cfg {
     // a cluster of cs CTAs reduces cs - 1 partial K x K blocks inside the leader's staging rows
     static constexpr int kMaxCs = (int)(2 * kStageRows * kStageLd / (K * K)) + 1;
     static constexpr size_t kSmemBarsMax = 8 * (3 * kMaxStages + 7) + 16;
-    static constexpr int kFit = (int)((kSmemMax - 1024 - kSmemStage - kSmemBarsMax) / kStageBytes);
+    // K = 128: a 256-entry table expands a byte of sign bits into eight bf16 signs
+    static constexpr size_t kLutBytes = kHalf ? 256 * 16 : 0;
+    static constexpr size_t kLutMax = kHalf ? kLutBytes + 8 : 0;
+    static constexpr int kFit = (int)((kSmemMax - 1024 - kSmemStage - kSmemBarsMax - kLutMax) / kStageBytes);
     static constexpr int kStages = kFit > kMaxStages ? kMaxStages : kFit;
     static constexpr size_t kSmemBars = 8 * (3 * kStages + 7) + 16;
     static constexpr size_t kBarsOff = (size_t)kStages * kStageBytes + kSmemStage;  // after ring and staging
-    static constexpr size_t kSmem = 1024 + kBarsOff + kSmemBars;
+    static constexpr size_t kLutOff = (kBarsOff + kSmemBars + 15) / 16 * 16;
+    static constexpr size_t kSmem = 1024 + (kHalf ? kLutOff + kLutBytes : kBarsOff + kSmemBars);
     // contraction blocking: 16 row groups x 8 column groups of threads
     static constexpr int RB = K / 16 > 0 ? K / 16 : 1;
     static constexpr int CB = K / 8;
     static_assert(kStages >= 3 && kSmem <= kSmemMax, "shared memory per CTA");
     static_assert(!kHalf || G == 1, "K = 128 fills TMEM with one double-buffered tile");
+    static_assert(!kHalf || kThreads == 256, "one thread per sign-table entry");
     static_assert(kStageBytes % 1024 == 0 && 2 * kBufCols <= (int)kTmemCols && kTmemCols <= 512,
                   "operand alignment / TMEM columns");
 };
@@ -216,6 +221,33 @@ __device__ __forceinline__ bool store_phi(float (&acc)[C::RB][C::CB], int64_t n,
     return true;
 }
 
+__device__ __forceinline__ uint4 lds128(uint32_t a) {
+    uint4 v;
+    asm volatile("ld.shared.v4.u32 {%0, %1, %2, %3}, [%4];" : "=r"(v.x), "=r"(v.y), "=r"(v.z), "=r"(v.w) : "r"(a));
+    return v;
+}
+
+// Entry e of the sign expansion table: bit j of e as the bf16 sign of element j
+// (+1 = 0x3F80, -1 = 0xBF80), the layout write_sign_half produces.
+__device__ __forceinline__ void init_sign_lut(uint8_t* lut, uint32_t e) {
+    uint32_t q[4];
+#pragma unroll
+    for (int p = 0; p < 4; ++p)
+        q[p] = (0x3F80u | (((e >> (2 * p)) & 1u) << 15)) | ((0x3F80u | (((e >> (2 * p + 1)) & 1u) << 15)) << 16);
+    *reinterpret_cast<uint4*>(lut + e * 16) = make_uint4(q[0], q[1], q[2], q[3]);
+}
+
+// All eight 16-byte chunks of row n of a K-major 128B-swizzled sign tile from
+// the expansion table at shared address lut: one table read per byte of w.
+__device__ __forceinline__ void write_sign_row(uint8_t* tile, int n, uint64_t w, uint32_t lut) {
+    uint8_t* row = tile + (n >> 3) * 1024 + (n & 7) * 128;
+    uint4 q[8];
+#pragma unroll
+    for (int c = 0; c < 8; ++c) q[c] = lds128(lut + ((((uint32_t)(w >> (8 * c))) & 0xFFu) << 4));
+#pragma unroll
+    for (int c = 0; c < 8; ++c) *reinterpret_cast<uint4*>(row + ((c ^ (n & 7)) << 4)) = q[c];
+}
+
 // KF: also accumulate the K-FAC factor covariances. FO: write the projected
 // factors At, Bt of every token instead of contracting them into Phi.
 template <int K, int G, bool KF, bool FO>
@@ -257,6 +289,7 @@ project_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant
         *abort = 0;
         fence_mbar_init();
     }
+    if constexpr (C::kHalf) init_sign_lut(smem + C::kLutOff, threadIdx.x);  // kThreads == 256 entries
     if (warp == 1) {
         tmem_alloc(smem_u32(tmem_slot), C::kTmemCols);
         tmem_relinquish();
@@ -376,16 +409,24 @@ project_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant
                 const uint64_t key = side_b ? p.key_out : p.key_in;
                 const uint64_t rb = (uint64_t)(side_b ? kc - p.nk_in : kc);
                 uint8_t* tile = sA + (size_t)s * C::kStageBytes + (size_t)G * kTileBytes;
-                for (int col = lane; col < K; col += 32)
-                    write_sign_half(tile, col, sign_word(key, (uint32_t)col, rb), warp - 2);
+                if constexpr (C::kHalf) {
+                    // each warp the whole rows of one half of the K columns
+                    const uint32_t lut = smem_u32(smem + C::kLutOff);
+                    for (int col = (warp - 2) * (K / 2) + lane; col < (warp - 1) * (K / 2); col += 32)
+                        write_sign_row(tile, col, sign_word(key, (uint32_t)col, rb), lut);
+                } else {
+                    for (int col = lane; col < K; col += 32)
+                        write_sign_half(tile, col, sign_word(key, (uint32_t)col, rb), warp - 2);
+                }
                 fence_proxy_async();
                 __syncwarp();
                 if (lane == 0) mbar_arrive(smem_u32(&sready[s]));
             }
     } else if (C::kHalf && warp >= 4) {
         // ---------------- epilogue for K = 128 (one example per tile, one tile per group):
-        // token rows 0-63 (TMEM lane quadrants 0, 1), then rows 64-127 (quadrants 2, 3),
-        // each staged in shared memory and contracted, Phi += Bt^T At, in fp32. The
+        // the tile's token rows in parts of kStageRows (rows 0-63 from TMEM lane
+        // quadrants 0, 1, then rows 64-127 from quadrants 2, 3), each part staged in
+        // shared memory and contracted, Phi += Bt^T At, in fp32. The
         // accumulators live for one example (the loop nest keeps them within the
         // register budget: 128 per thread).
         const int q = warp & 3;
@@ -412,9 +453,10 @@ project_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant
                 }
                 tc_fence_after();
                 const uint32_t tbase = tmem + ((uint32_t)(q * 32) << 16) + b * C::kBufCols;
-                for (int h = 0; h < 2; ++h) {
-                    if ((q >> 1) == h) {
-                        const int srow = (q & 1) * 32 + lane;
+                constexpr int kParts = kTileM / C::kStageRows, kWarpsPer = 4 / kParts;
+                for (int h = 0; h < kParts; ++h) {
+                    if (q / kWarpsPer == h) {
+                        const int srow = (q % kWarpsPer) * 32 + lane;
 #pragma unroll 4
                         for (int c0 = 0; c0 < 2 * K; c0 += 16) {
                             float v[16];
