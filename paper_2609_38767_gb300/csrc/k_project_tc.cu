@@ -96,7 +96,7 @@ struct Cfg {
     static constexpr int CB = K / 8;
     static_assert(kStages >= 3 && kSmem <= kSmemMax, "shared memory per CTA");
     static_assert(!kHalf || G == 1, "K = 128 fills TMEM with one double-buffered tile");
-    static_assert(!kHalf || kThreads == 256, "one thread per sign-table entry");
+    static_assert(!kHalf || (kThreads == 256 && K == 128), "one thread per sign-table entry; two columns per lane");
     static_assert(kStageBytes % 1024 == 0 && 2 * kBufCols <= (int)kTmemCols && kTmemCols <= 512,
                   "operand alignment / TMEM columns");
 };
@@ -237,13 +237,16 @@ __device__ __forceinline__ void init_sign_lut(uint8_t* lut, uint32_t e) {
     *reinterpret_cast<uint4*>(lut + e * 16) = make_uint4(q[0], q[1], q[2], q[3]);
 }
 
-// All eight 16-byte chunks of row n of a K-major 128B-swizzled sign tile from
-// the expansion table at shared address lut: one table read per byte of w.
-__device__ __forceinline__ void write_sign_row(uint8_t* tile, int n, uint64_t w, uint32_t lut) {
-    uint8_t* row = tile + (n >> 3) * 1024 + (n & 7) * 128;
-    uint4 q[8];
+// The eight 16-byte chunks of one sign-tile row (the 64 signs of sign word w)
+// from the expansion table at shared address lut: one table read per byte.
+__device__ __forceinline__ void expand_signs(uint4 (&q)[8], uint64_t w, uint32_t lut) {
 #pragma unroll
     for (int c = 0; c < 8; ++c) q[c] = lds128(lut + ((((uint32_t)(w >> (8 * c))) & 0xFFu) << 4));
+}
+
+// Row n of a K-major 128B-swizzled sign tile from its eight expanded chunks.
+__device__ __forceinline__ void store_sign_row(uint8_t* tile, int n, const uint4 (&q)[8]) {
+    uint8_t* row = tile + (n >> 3) * 1024 + (n & 7) * 128;
 #pragma unroll
     for (int c = 0; c < 8; ++c) *reinterpret_cast<uint4*>(row + ((c ^ (n & 7)) << 4)) = q[c];
 }
@@ -397,6 +400,19 @@ project_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant
             for (int kc = 0; kc < nk_tot; ++kc, ++ring) {
                 const int s = ring % C::kStages;
                 const uint32_t ph = (ring / C::kStages) & 1u;
+                const bool side_b = kc >= p.nk_in;
+                const uint64_t key = side_b ? p.key_out : p.key_in;
+                const uint64_t rb = (uint64_t)(side_b ? kc - p.nk_in : kc);
+                // K = 128: each warp writes whole rows of one half of the K columns (columns
+                // col0 and col0 + 32 per lane); their sign words and table expansion do not
+                // depend on the stage's memory, so they are formed before the wait below
+                const int col0 = (warp - 2) * (K / 2) + lane;
+                uint4 q[C::kHalf ? 2 : 1][8];
+                if constexpr (C::kHalf) {
+                    const uint32_t lut = smem_u32(smem + C::kLutOff);
+#pragma unroll
+                    for (int j = 0; j < 2; ++j) expand_signs(q[j], sign_word(key, (uint32_t)(col0 + 32 * j), rb), lut);
+                }
                 bool got = true;
                 if (lane == 0) got = wait_bounded(smem_u32(&empty[s]), ph ^ 1u, abort, p.err);
                 got = __shfl_sync(0xffffffffu, got, 0);
@@ -405,15 +421,10 @@ project_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant
                     ok = false;
                     break;
                 }
-                const bool side_b = kc >= p.nk_in;
-                const uint64_t key = side_b ? p.key_out : p.key_in;
-                const uint64_t rb = (uint64_t)(side_b ? kc - p.nk_in : kc);
                 uint8_t* tile = sA + (size_t)s * C::kStageBytes + (size_t)G * kTileBytes;
                 if constexpr (C::kHalf) {
-                    // each warp the whole rows of one half of the K columns
-                    const uint32_t lut = smem_u32(smem + C::kLutOff);
-                    for (int col = (warp - 2) * (K / 2) + lane; col < (warp - 1) * (K / 2); col += 32)
-                        write_sign_row(tile, col, sign_word(key, (uint32_t)col, rb), lut);
+#pragma unroll
+                    for (int j = 0; j < 2; ++j) store_sign_row(tile, col0 + 32 * j, q[j]);
                 } else {
                     for (int col = lane; col < K; col += 32)
                         write_sign_half(tile, col, sign_word(key, (uint32_t)col, rb), warp - 2);
