@@ -66,6 +66,8 @@ def _load():
             "oracle_damping": (ctypes.c_double, [I64, D, ctypes.c_double, ctypes.c_double]),
             "oracle_cholesky": (I32, [I64, D]),
             "oracle_precondition": (I32, [I64, D, ctypes.c_double, I64, D, D]),
+            "oracle_damping_features": (ctypes.c_double, [I64, I64, D, ctypes.c_double, ctypes.c_double]),
+            "oracle_precondition_lowrank": (I32, [I64, I64, D, ctypes.c_double, I64, D, D]),
             "oracle_kfac_covariances": (None, [I64, I64, I64, I64, I64, I64, U64, U32, I32, D, D, D, D]),
             "oracle_sym_eig": (I32, [I64, D, D, D]),
             "oracle_kfac_eigenvalues": (None, [I64, I64, D, D, D]),
@@ -217,6 +219,27 @@ def precondition(F, lam: float, Q) -> np.ndarray:
     st = int(_load().oracle_precondition(D, _p(F), lam, Q.shape[0], _p(Q), _p(out)))
     if st != 0:
         raise np.linalg.LinAlgError(f"F + lambda I not positive definite (minor {st})")
+    return out
+
+
+def damping_features(phi, lambda_abs: float, lambda_rel: float) -> float:
+    """lambda from the features (N, D) without forming F."""
+    phi = _f64(phi)
+    phi = phi.reshape(phi.shape[0], -1)
+    return float(_load().oracle_damping_features(phi.shape[1], phi.shape[0], _p(phi), lambda_abs, lambda_rel))
+
+
+def precondition_lowrank(phi, lam: float, Q) -> np.ndarray:
+    """(F + lam I)^{-1} Q with F = Phi^T Phi / N given by Phi (N, D): Woodbury, an N x N solve."""
+    phi, Q = _f64(phi), _f64(Q)
+    N = phi.shape[0]
+    phi = phi.reshape(N, -1)
+    D = phi.shape[1]
+    Q = Q.reshape(-1, D)
+    out = np.empty_like(Q)
+    st = int(_load().oracle_precondition_lowrank(D, N, _p(phi), lam, Q.shape[0], _p(Q), _p(out)))
+    if st != 0:
+        raise np.linalg.LinAlgError(f"N lambda I + Phi Phi^T not positive definite (minor {st})")
     return out
 
 

@@ -278,17 +278,23 @@ void oracle_cosine(int64_t n_q, int64_t n_t, const double* S, const double* nq,
 /* ------------------------------------------------------------------------ */
 
 /* Empirical Fisher of the projected training gradients, the mean of the
- * outer products phi_i phi_i^T over the N training examples. */
+ * outer products phi_i phi_i^T over the N training examples. Entry (a, b) is
+ * the sum over n = 0..N-1, in that order, of phi_na phi_nb, divided by N; the
+ * loop over n sits outside the loop over b only so that the rows of phi are
+ * read contiguously (each entry's additions happen in the same order). */
 void oracle_fisher(int64_t D, int64_t N, const double* phi, double* F) {
 #ifdef _OPENMP
 #pragma omp parallel for schedule(dynamic, 1) num_threads(g_threads)
 #endif
-    for (int64_t a = 0; a < D; ++a)
-        for (int64_t b = 0; b < D; ++b) {
-            double s = 0.0;
-            for (int64_t n = 0; n < N; ++n) s += phi[n * D + a] * phi[n * D + b];
-            F[a * D + b] = s / (double)N;
+    for (int64_t a = 0; a < D; ++a) {
+        double* row = F + a * D;
+        for (int64_t b = 0; b < D; ++b) row[b] = 0.0;
+        for (int64_t n = 0; n < N; ++n) {
+            const double pa = phi[n * D + a];
+            for (int64_t b = 0; b < D; ++b) row[b] += pa * phi[n * D + b];
         }
+        for (int64_t b = 0; b < D; ++b) row[b] = row[b] / (double)N;
+    }
 }
 
 /* Damping in units of the mean eigenvalue (App. B.2); the mean eigenvalue of a
@@ -296,6 +302,20 @@ void oracle_fisher(int64_t D, int64_t N, const double* phi, double* F) {
 double oracle_damping(int64_t D, const double* F, double lambda_abs, double lambda_rel) {
     double tr = 0.0;
     for (int64_t a = 0; a < D; ++a) tr += F[a * D + a];
+    return lambda_abs + lambda_rel * tr / (double)D;
+}
+
+/* The same damping from the features themselves, without forming F: the
+ * diagonal entry F_aa is (sum over n of phi_na^2) / N, summed over a in order
+ * (the same additions as oracle_fisher followed by oracle_damping). */
+double oracle_damping_features(int64_t D, int64_t N, const double* phi, double lambda_abs,
+                               double lambda_rel) {
+    double tr = 0.0;
+    for (int64_t a = 0; a < D; ++a) {
+        double s = 0.0;
+        for (int64_t n = 0; n < N; ++n) s += phi[n * D + a] * phi[n * D + a];
+        tr += s / (double)N;
+    }
     return lambda_abs + lambda_rel * tr / (double)D;
 }
 
@@ -308,6 +328,10 @@ int32_t oracle_cholesky(int64_t D, double* M) {
         if (!(s > 0.0)) return (int32_t)(j + 1);
         double ljj = sqrt(s);
         M[j * D + j] = ljj;
+        /* for a fixed column j the rows i > j are independent of each other */
+#ifdef _OPENMP
+#pragma omp parallel for schedule(static) num_threads(g_threads) if (D - j > 256)
+#endif
         for (int64_t i = j + 1; i < D; ++i) {
             double t = M[i * D + j];
             for (int64_t k = 0; k < j; ++k) t -= M[i * D + k] * M[j * D + k];
@@ -321,7 +345,7 @@ int32_t oracle_cholesky(int64_t D, double* M) {
 
 /* Per-layer preconditioning of the queries (App. B.3): with
  * F + lambda I = L L^T, solve L y = q by forward and L^T x = y by backward
- * substitution, so x = (F + lambda I)^{-1} q. */
+ * substitution, so x = (F + lambda I)^{-1} q. Query rows are independent. */
 int32_t oracle_precondition(int64_t D, const double* F, double lambda,
                             int64_t n_q, const double* Q, double* Qhat) {
     double* L = (double*)malloc(sizeof(double) * (size_t)(D * D));
@@ -332,8 +356,11 @@ int32_t oracle_precondition(int64_t D, const double* F, double lambda,
         free(L);
         return st;
     }
-    double* y = (double*)malloc(sizeof(double) * (size_t)D);
+#ifdef _OPENMP
+#pragma omp parallel for schedule(dynamic, 1) num_threads(g_threads)
+#endif
     for (int64_t q = 0; q < n_q; ++q) {
+        double* y = (double*)malloc(sizeof(double) * (size_t)D);
         const double* b = Q + q * D;
         double* x = Qhat + q * D;
         for (int64_t i = 0; i < D; ++i) {
@@ -346,9 +373,68 @@ int32_t oracle_precondition(int64_t D, const double* F, double lambda,
             for (int64_t k = i + 1; k < D; ++k) s -= L[k * D + i] * x[k];
             x[i] = s / L[i * D + i];
         }
+        free(y);
     }
-    free(y);
     free(L);
+    return 0;
+}
+
+/* The same damped inverse when the Fisher has fewer examples than features
+ * (N < D), without the D x D matrix. F + lambda I = lambda I + Phi^T Phi / N,
+ * and the Woodbury identity gives
+ *   (F + lambda I)^{-1} q = (q - Phi^T z) / lambda,
+ *   (N lambda I + Phi Phi^T) z = Phi q,
+ * an N x N system (Cholesky as above). Exact for any N; cheaper when N < D. */
+int32_t oracle_precondition_lowrank(int64_t D, int64_t N, const double* phi, double lambda,
+                                    int64_t n_q, const double* Q, double* Qhat) {
+    double* K = (double*)malloc(sizeof(double) * (size_t)(N * N));
+#ifdef _OPENMP
+#pragma omp parallel for schedule(dynamic, 1) num_threads(g_threads)
+#endif
+    for (int64_t i = 0; i < N; ++i)
+        for (int64_t j = 0; j < N; ++j) {
+            double s = 0.0;
+            for (int64_t a = 0; a < D; ++a) s += phi[i * D + a] * phi[j * D + a];
+            K[i * N + j] = s;
+        }
+    for (int64_t i = 0; i < N; ++i) K[i * N + i] += (double)N * lambda;
+    int32_t st = oracle_cholesky(N, K);
+    if (st != 0) {
+        free(K);
+        return st;
+    }
+#ifdef _OPENMP
+#pragma omp parallel for schedule(dynamic, 1) num_threads(g_threads)
+#endif
+    for (int64_t q = 0; q < n_q; ++q) {
+        double* u = (double*)malloc(sizeof(double) * (size_t)N);
+        double* z = (double*)malloc(sizeof(double) * (size_t)N);
+        const double* b = Q + q * D;
+        double* x = Qhat + q * D;
+        for (int64_t i = 0; i < N; ++i) {
+            double s = 0.0;
+            for (int64_t a = 0; a < D; ++a) s += phi[i * D + a] * b[a];
+            u[i] = s;
+        }
+        for (int64_t i = 0; i < N; ++i) {
+            double s = u[i];
+            for (int64_t k = 0; k < i; ++k) s -= K[i * N + k] * z[k];
+            z[i] = s / K[i * N + i];
+        }
+        for (int64_t i = N - 1; i >= 0; --i) {
+            double s = z[i];
+            for (int64_t k = i + 1; k < N; ++k) s -= K[k * N + i] * z[k];
+            z[i] = s / K[i * N + i];
+        }
+        for (int64_t a = 0; a < D; ++a) {
+            double s = b[a];
+            for (int64_t i = 0; i < N; ++i) s -= phi[i * D + a] * z[i];
+            x[a] = s / lambda;
+        }
+        free(u);
+        free(z);
+    }
+    free(K);
     return 0;
 }
 
@@ -644,13 +730,18 @@ typedef struct {
     int32_t i;
 } oracle_pair;
 
-/* Descending value, then ascending index: a total order, so qsort's result
- * is the unique sorted sequence. */
+/* Descending value, then ascending index, with NaN above every number (NaNs
+ * ordered by index among themselves) and -0 equal to +0 (IEEE comparison):
+ * a total order, so qsort's result is the unique sorted sequence. */
 static int oracle_pair_cmp(const void* x, const void* y) {
     const oracle_pair* a = (const oracle_pair*)x;
     const oracle_pair* b = (const oracle_pair*)y;
-    if (a->v > b->v) return -1;
-    if (a->v < b->v) return 1;
+    const int na = a->v != a->v, nb = b->v != b->v;
+    if (na != nb) return na ? -1 : 1;
+    if (!na) {
+        if (a->v > b->v) return -1;
+        if (a->v < b->v) return 1;
+    }
     return (a->i > b->i) - (a->i < b->i);
 }
 

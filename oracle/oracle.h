@@ -109,12 +109,19 @@ void oracle_cosine(int64_t n_q, int64_t n_t, const double* S, const double* nq,
 void oracle_fisher(int64_t D, int64_t N, const double* phi, double* F);
 /* lambda = lambda_abs + lambda_rel * tr(F)/D (tr(F)/D is the mean eigenvalue). */
 double oracle_damping(int64_t D, const double* F, double lambda_abs, double lambda_rel);
+/* The same lambda from the N x D features directly (tr(F) = sum_a (1/N) sum_n phi_na^2). */
+double oracle_damping_features(int64_t D, int64_t N, const double* phi, double lambda_abs,
+                               double lambda_rel);
 /* In-place lower Cholesky factor of the D x D SPD matrix M (upper part zeroed).
  * Returns 0, or j+1 if the leading minor of order j+1 is not positive. */
 int32_t oracle_cholesky(int64_t D, double* M);
 /* Qhat = (F + lambda I)^{-1} Q for n_q row vectors Q[q][:] (D each). */
 int32_t oracle_precondition(int64_t D, const double* F, double lambda,
                             int64_t n_q, const double* Q, double* Qhat);
+/* The same Qhat = (F + lambda I)^{-1} Q with F = (1/N) Phi^T Phi given by its
+ * N x D features, through the Woodbury identity (an N x N solve). */
+int32_t oracle_precondition_lowrank(int64_t D, int64_t N, const double* phi, double lambda,
+                                    int64_t n_q, const double* Q, double* Qhat);
 
 /* ---- Kronecker-factored curvature on the projected factors (K-FAC of
  *      Martens & Grosse 2015, EK-FAC of George et al. 2018; the paper applies
@@ -177,7 +184,7 @@ void oracle_mask_gather(int64_t N, int64_t T, int64_t d_in, int64_t d_out, const
 void oracle_score(int64_t n_q, int64_t n_t, int64_t D,
                   const double* Qhat, const double* phi, double* S);
 /* Per row of S (n_q x n_t), the k largest entries, descending, ties broken
- * by the smaller train index. */
+ * by the smaller train index; NaN ranks above every number, -0 equals +0. */
 void oracle_topk(int64_t n_q, int64_t n_t, const double* S, int32_t k,
                  int32_t* idx, double* val);
 

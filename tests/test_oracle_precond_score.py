@@ -91,3 +91,46 @@ def test_topk_full_row_when_k_equals_n(orc, k):
     S = np.linspace(-1, 1, k)[None, :]
     idx, _ = orc.topk(S, k)
     assert list(idx[0]) == list(range(k - 1, -1, -1))
+
+
+def test_fisher_entry_is_the_ordered_sum_over_examples(orc):
+    # F[a][b] = (sum over n in order of phi_na phi_nb) / N, bit for bit
+    rng = np.random.default_rng(7)
+    N, D = 11, 5
+    phi = rng.standard_normal((N, D))
+    F = orc.fisher(phi)
+    for a in range(D):
+        for b in range(D):
+            s = 0.0
+            for n in range(N):
+                s += phi[n, a] * phi[n, b]
+            assert F[a, b] == s / N
+
+
+def test_damping_from_features_equals_damping_of_fisher(orc):
+    rng = np.random.default_rng(8)
+    phi = rng.standard_normal((13, 9))
+    assert orc.damping_features(phi, 1e-3, 1e-2) == orc.damping(orc.fisher(phi), 1e-3, 1e-2)
+
+
+@pytest.mark.parametrize("N,D", [(6, 40), (40, 12), (1, 7)])
+def test_lowrank_precondition_agrees_with_cholesky_route(orc, N, D):
+    # Woodbury (N x N solve) and the D x D Cholesky solve of the same (F + lambda I)
+    rng = np.random.default_rng(N * 100 + D)
+    phi = rng.standard_normal((N, D)) * rng.uniform(0.5, 2.0, D)
+    Q = rng.standard_normal((4, D))
+    F = orc.fisher(phi)
+    lam = orc.damping(F, 0.0, 1e-2)
+    a = orc.precondition_lowrank(phi, lam, Q)
+    b = orc.precondition(F, lam, Q)
+    np.testing.assert_allclose(a, b, rtol=1e-9, atol=1e-12 * np.abs(b).max())
+    c = np.linalg.solve(phi.T @ phi / N + lam * np.eye(D), Q.T).T
+    np.testing.assert_allclose(a, c, rtol=1e-9, atol=1e-12 * np.abs(c).max())
+
+
+def test_topk_nan_ranks_first_and_signed_zeros_tie(orc):
+    # NaN is ranked above +inf (NaNs among themselves by index); -0 and +0 are equal
+    S = np.array([[0.0, np.nan, -0.0, 1.0, np.inf, np.nan, -np.inf, 0.0, -1.0]])
+    idx, val = orc.topk(S, 9)
+    assert list(idx[0]) == [1, 5, 4, 3, 0, 2, 7, 8, 6]
+    assert np.isnan(val[0, :2]).all() and list(val[0, 2:4]) == [np.inf, 1.0]
