@@ -1,22 +1,35 @@
 #!/usr/bin/env python3
 """Throughput of the attribution hot path on GB300.
 
-Workload: one Llama-style 1B transformer block, bf16 -- linears q/k/v/o
-2048x2048, gate/up 2048->8192, down 8192->2048; T = 512 tokens; 4096 train and
-64 query examples; factors A ~ N(0,1), B ~ N(0,1e-3) with 1% of tokens masked
-in both; seeded Kronecker Rademacher projection k_in = k_out = 32 per linear
-(1024 features per linear, 7168 per example).
+Workloads (--workload):
 
-One step = one pass of the whole path over the block: route choice per linear
-(host cost model), factored projection of every train and query example
-through all 7 linears, per-linear Fisher fit over the train features, damped
-inverse (lambda = 1e-2 x mean eigenvalue) applied to the queries, the 64 x 4096
-score matrix and the top-100 train indices per query.
+* llama3_8b_stack (default): a Llama-3-8B-shaped stack of 32 layers x 7 linears
+  (q/o 4096x4096, k/v 4096->1024, gate/up 4096->14336, down 14336->4096), bf16,
+  T = 1024 tokens, k_in = k_out = 64 (4096 features per linear, 917,504 per
+  example), 8192 train examples streamed in chunks of 256, 256 queries,
+  per-linear (F + lambda I)^-1 with lambda = 1e-2 x mean eigenvalue, top-100.
+* large_model: one block of large-model layers (d_model 12288, ffn 49152, GQA
+  k/v 12288->1536), bf16, T = 2048, k = 128 (16384 features per linear), 16384
+  train examples in chunks of 512, 512 queries, A ~ Student-t(4), B ~ N(0,1e-4),
+  lambda = 1e-2 x mean eigenvalue, top-100.
+* llama1b_block: one Llama-style 1B block (q/k/v/o 2048x2048, gate/up
+  2048->8192, down 8192->2048), T = 512, 4096 train / 64 query examples, k = 32,
+  1% of tokens masked, every factor resident.
+
+Stack workloads (paper_2609_38767_gb300.stream.StackJob): one step is one
+chunk of train examples through the whole path -- the chunk's factored
+projection through every linear and its Fisher sums, plus a 1/C share of the
+previous job's query side (query projections, factorisation and
+preconditioning, score) and of the job before's top-k, C = chunks per job. C
+consecutive steps do exactly one job's work, so examples/s = chunk / step
+time is whole-job throughput. Jobs run back to back; two jobs run untimed
+first so that every share of the timed steps exists.
 
 value: train examples attributed per second with the factors resident in HBM
-(198 GB, larger than L2, so no flush is needed between steps). e2e: the same
-metric through tda_project_host with the factors in pinned host memory, the
-H2D copies and the D2H read of the top-k inside the timed region.
+(pools of examples larger than L2, so no flush is needed between steps; each
+chunk of each layer reads its own window of the pool). e2e: the same steps
+with the factors in pinned host memory through tda_project_host, the H2D
+copies and the D2H read of the step's top-k rows inside the timed region.
 
 --impl reference times the fp64 CPU oracle on a bounded sample of the same
 workload on the host cores (the only other place this file runs the oracle).
@@ -65,6 +78,7 @@ def parse_args():
     p.add_argument("--steps", type=int, default=5)
     p.add_argument("--warmup", type=int, default=3)
     p.add_argument("--impl", default="ours", choices=["ours", "reference"])
+    p.add_argument("--workload", default="llama3_8b_stack", choices=["llama3_8b_stack", "large_model", "llama1b_block"])
     p.add_argument("--n-train", type=int, default=4096)
     p.add_argument("--n-query", type=int, default=64)
     p.add_argument("--T", type=int, default=512)
@@ -76,6 +90,8 @@ def parse_args():
                         "on the projected factors (damping 0.1 x mean eigenvalue)")
     p.add_argument("--overlap-sms", type=int, default=0,
                    help="Fisher query side on a second stream; the train projection leaves this many SMs free")
+    p.add_argument("--train-streams", type=int, default=2,
+                   help="stack workloads: streams the train projections of a chunk are spread over")
     p.add_argument("--query-streams", type=int, default=8,
                    help="streams the query projections of the linears are spread over (device-resident leg)")
     p.add_argument("--e2e-steps", type=int, default=2)
@@ -116,6 +132,7 @@ def workload(args):
                    "(F+lambda I)^-1-preconditioned, lambda=1e-2*mean eig" if args.curvature == "fisher" else
                    f"{args.curvature.upper()} on projected factors, lambda=0.1*mean eig"),
         "topk": args.topk, "l2": "inputs larger than L2 (no flush)",
+        "parallelism": "train examples sharded over the ranks (one GPU per rank)",
         **({"mode": "project-only (kernel profiling)"} if args.project_only else {}),
         **({"query_side": f"second stream beside the train projection, which leaves {args.overlap_sms} SMs free"}
            if getattr(args, "overlap_sms", 0) > 0 and not args.no_precondition and args.curvature == "fisher"
@@ -300,10 +317,11 @@ def reference_main(args):
     value = statistics.median(vals)
     line = {
         "impl": "reference", "metric": METRIC, "value": value, "unit": "examples/s", "n_gpus": args.gpus,
-        "steps": args.steps, "warmup": args.warmup, "ms_per_step": 1e3 * args.n_train / value,
+        "steps": args.steps, "warmup": args.warmup, "ms_per_step": 1e3 * statistics.median(secs),
         "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
         "config": workload(args),
-        "cpu_baseline": {"value": value, "unit": "examples/s", "cores": cores, "kind": "oracle", "sample": sample},
+        "cpu_baseline": {"value": value, "unit": "examples/s", "cores": cores, "kind": "oracle",
+                         "sample": sample + "; ms_per_step is one sample's wall time"},
         "e2e": {"value": value, "unit": "examples/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
     }
     print(json.dumps(line), flush=True)
@@ -556,8 +574,383 @@ def reuse_main(args):
         "cpu_baseline": None, "e2e": None, "gpu_launches": launches, "clocks": ck}))
 
 
+# ---------------------------------------------------------------------------- streamed stacks
+STACKS = {
+    "llama3_8b_stack": {
+        "layer": [("q", 4096, 4096), ("k", 4096, 1024), ("v", 4096, 1024), ("o", 4096, 4096),
+                  ("gate", 4096, 14336), ("up", 4096, 14336), ("down", 14336, 4096)],
+        "n_layers": 32, "T": 1024, "k": 64, "n_train": 8192, "chunk": 256, "n_query": 256,
+        "dist_a": 0, "sigma_b": math.sqrt(1e-3), "lambda_rel": 1e-2,
+        "train_pool": 512, "query_pool": 256, "host_pool": 32,
+        "factors": "A~N(0,1), B~N(0,1e-3) (seeded synthetic)",
+    },
+    "large_model": {
+        "layer": [("q", 12288, 12288), ("k", 12288, 1536), ("v", 12288, 1536), ("o", 12288, 12288),
+                  ("gate", 12288, 49152), ("up", 12288, 49152), ("down", 49152, 12288)],
+        "n_layers": 1, "T": 2048, "k": 128, "n_train": 16384, "chunk": 512, "n_query": 512,
+        "dist_a": 1, "sigma_b": 0.01, "lambda_rel": 1e-2,
+        "train_pool": 96, "query_pool": 64, "host_pool": 16,
+        "factors": "A~Student-t(4), B~N(0,1e-4) (seeded synthetic)",
+    },
+}
+
+
+def stack_config(args, spec):
+    lin = spec["layer"]
+    nlin = len(lin) * spec["n_layers"]
+    D = spec["k"] ** 2
+    return {
+        "workload": args.workload,
+        "linears_per_layer": {n: [di, do] for n, di, do in lin}, "layers": spec["n_layers"],
+        "T": spec["T"], "n_train": spec["n_train"], "chunk": spec["chunk"], "n_query": spec["n_query"],
+        "k_in": spec["k"], "k_out": spec["k"], "features_per_example": nlin * D,
+        "factors": spec["factors"],
+        "method": f"(F+lambda I)^-1-preconditioned per linear, lambda={spec['lambda_rel']:g}*mean eig",
+        "topk": args.topk,
+        "step": (f"one chunk of {spec['chunk']} train examples projected through all {nlin} linears + "
+                 f"1/{spec['n_train'] // spec['chunk']} of the previous job's query side (Fisher fit over the "
+                 "job's resident features, query projection, factorisation + preconditioning, score) and of the "
+                 "job before's top-k"),
+        "resident_pools": (f"{spec['train_pool']} train / {spec['query_pool']} query examples per linear shape in "
+                           "HBM; each (chunk, layer) reads its own window of the train pool"),
+        "l2": "inputs larger than L2 (no flush)",
+        "parallelism": "one GPU", "routes": "factored (every linear)",
+    }
+
+
+def stack_oracle_sample(spec, factors_of):
+    """Time the fp64 oracle on a bounded sample of a stack job and extrapolate to the job's
+    examples/s: n_s train and 2 query examples through the 7 linears of one layer, the Fisher
+    of one linear over the n_s train features, the damped inverse (D x D Cholesky) applied to
+    the queries, and their scores. factors_of(role, li, n) returns float64 (A, B)."""
+    import numpy as np
+
+    import oracle
+
+    oracle.build()
+    threads = os.cpu_count() or 1
+    oracle.set_threads(threads)
+    n_s, nq_s, k, D = max(2, threads), 2, spec["k"], spec["k"] ** 2
+    t_proj = t_qproj = 0.0
+    phis, qs = [], []
+    for li in range(len(spec["layer"])):
+        A, B = factors_of("train", li, n_s)
+        t0 = time.perf_counter()
+        phis.append(oracle.project(A, B, k, k, 0, li).reshape(n_s, D))
+        t_proj += time.perf_counter() - t0
+        Aq, Bq = factors_of("query", li, nq_s)
+        t0 = time.perf_counter()
+        qs.append(oracle.project(Aq, Bq, k, k, 0, li).reshape(nq_s, D))
+        t_qproj += time.perf_counter() - t0
+    t0 = time.perf_counter()
+    F = oracle.fisher(phis[0])
+    t_fit = time.perf_counter() - t0
+    t0 = time.perf_counter()
+    qh = oracle.precondition(F, oracle.damping(F, 0.0, spec["lambda_rel"]), qs[0])
+    t_fact = time.perf_counter() - t0
+    t0 = time.perf_counter()
+    S = oracle.score(qh, phis[0])
+    oracle.topk(S, 1)
+    t_score = time.perf_counter() - t0
+    N, Nq, L = spec["n_train"], spec["n_query"], spec["n_layers"]
+    nlin = L * len(spec["layer"])
+    total = (t_proj * L * N / n_s + t_qproj * L * Nq / nq_s + t_fit * nlin * N / n_s + t_fact * nlin
+             + t_score * nlin * (N / n_s) * (Nq / nq_s))
+    sample = (f"{n_s} train + {nq_s} query examples (fp64, {threads} threads) through the 7 linears of one layer, "
+              f"Fisher of one linear over them, D x D Cholesky + solves, scores; projection scaled by "
+              f"{L} layers x {N}/{n_s} (queries {Nq}/{nq_s}), Fisher by {nlin} linears x {N}/{n_s}, factorisation "
+              f"by {nlin} linears, score by {nlin} x {N}/{n_s} x {Nq}/{nq_s}")
+    wall = t_proj + t_qproj + t_fit + t_fact + t_score
+    return N / total, threads, sample, wall
+
+
+def stack_factors_host(spec, li, role, n):
+    """float64 factors of n examples of linear li of the layer (for the oracle sample)."""
+    from paper_2609_38767_gb300 import synth
+
+    _, di, do = spec["layer"][li]
+    off = synth.QUERY_STREAM_OFFSET if role == "query" else 0
+    A = synth.factors(synth.SEED_A, li + off, n, spec["T"], di, 1.0, spec["dist_a"], 0, "bf16")
+    B = synth.factors(synth.SEED_B, li + off, n, spec["T"], do, spec["sigma_b"], 0, 0, "bf16")
+    return synth.to_f64(A, "bf16"), synth.to_f64(B, "bf16")
+
+
+def stack_reference_main(args, spec):
+    if int(os.environ.get("RANK", "0")) != 0:
+        return 0
+    cache = {}
+
+    def factors_of(role, li, n):
+        key = (role, li, n)
+        if key not in cache:
+            cache[key] = stack_factors_host(spec, li, role, n)
+        return cache[key]
+
+    factors_of("train", 0, max(2, os.cpu_count() or 1))  # generation stays out of the timing
+    vals, walls = [], []
+    sample, cores = "", 1
+    for i in range(args.warmup + args.steps):
+        v, cores, sample, wall = stack_oracle_sample(spec, factors_of)
+        if i >= args.warmup:
+            vals.append(v)
+            walls.append(wall)
+    value = statistics.median(vals)
+    line = {
+        "impl": "reference", "metric": METRIC, "value": value, "unit": "examples/s", "n_gpus": args.gpus,
+        "steps": args.steps, "warmup": args.warmup, "ms_per_step": 1e3 * statistics.median(walls),
+        "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+        "config": stack_config(args, spec),
+        "cpu_baseline": {"value": value, "unit": "examples/s", "cores": cores, "kind": "oracle",
+                         "sample": sample + "; ms_per_step is one sample's wall time"},
+        "e2e": {"value": value, "unit": "examples/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
+    }
+    print(json.dumps(line), flush=True)
+    return 0
+
+
+def stack_main(args, spec):
+    import numpy as np
+    import torch
+
+    import paper_2609_38767_gb300 as tda
+    from paper_2609_38767_gb300 import build as tbuild
+    from paper_2609_38767_gb300 import synth
+    from paper_2609_38767_gb300.stream import StackJob
+
+    if int(os.environ.get("WORLD_SIZE", "1")) > 1 and int(os.environ.get("RANK", "0")) != 0:
+        return 0  # one GPU: the stack job does not shard here
+    tbuild.build()
+    tda.load()
+    dev = torch.device("cuda", 0)
+    torch.cuda.set_device(dev)
+    stream = torch.cuda.current_stream()
+    lin, L = spec["layer"], spec["n_layers"]
+    T, k, N, chunk, Nq = spec["T"], spec["k"], spec["n_train"], spec["chunk"], spec["n_query"]
+    D = k * k
+    C = N // chunk
+    nshape = len(lin)
+    linears = [(di, do) for _ in range(L) for _, di, do in lin]
+    nlin = len(linears)
+    steps = args.steps
+    if (nlin % C or Nq % C) and steps % C:
+        steps = (steps + C - 1) // C * C  # unequal shares per step: time whole jobs
+    Pt, Pq = spec["train_pool"], spec["query_pool"]
+
+    # ---- resident pools (untimed): per linear shape, Pt train and Pq query examples
+    pools = []
+    for si, (_, di, do) in enumerate(lin):
+        ent = []
+        for n, off, seed, d, sg, dist in ((Pt, 0, synth.SEED_A, di, 1.0, spec["dist_a"]),
+                                          (Pt, 0, synth.SEED_B, do, spec["sigma_b"], 0),
+                                          (Pq, synth.QUERY_STREAM_OFFSET, synth.SEED_A, di, 1.0, spec["dist_a"]),
+                                          (Pq, synth.QUERY_STREAM_OFFSET, synth.SEED_B, do, spec["sigma_b"], 0)):
+            x = torch.empty((n, T, d), dtype=torch.bfloat16, device=dev)
+            synth.fill_device(x, seed, si + off, n, T, d, sg, dist, mask_stream=1000 if off else 0)
+            ent.append(x)
+        pools.append(ent)
+
+    def window(li, j, s):
+        """First pool row of chunk s of job j for linear li (a pseudo-random window per chunk and layer)."""
+        layer = li // nshape
+        span = Pt - chunk + 1 if Pt >= chunk else Pt
+        return (131 * s + 37 * layer + 71 * j) % span
+
+    def dev_factors(role, li, j, s):
+        A, B, Aq, Bq = pools[li % nshape]
+        if role == "train":
+            if Pt >= chunk:
+                o = window(li, j, s)
+                return [(A[o:o + chunk], B[o:o + chunk], 0, chunk)]
+            return [(A[:min(Pt, chunk - r)], B[:min(Pt, chunk - r)], r, min(Pt, chunk - r)) for r in range(0, chunk, Pt)]
+        return [(Aq[:min(Pq, Nq - r)], Bq[:min(Pq, Nq - r)], r, min(Pq, Nq - r)) for r in range(0, Nq, Pq)]
+
+    job = StackJob(linears, T, k, N, chunk, Nq, topk=args.topk, lambda_rel=spec["lambda_rel"], device=dev,
+                   train_streams=args.train_streams)
+    for si in range(nshape):  # every linear shape runs on the tensor-core projection kernel
+        assert tda.tda_project_engine(job.layers[si], tda.TDA_BF16, pools[si][0], pools[si][1]) == 1
+    state = {"j": 0, "s": 0}
+
+    def advance(factors, mark=None, hook=None):
+        job.step(state["j"], state["s"], factors, mark=mark, hook=hook)
+        state["s"] += 1
+        if state["s"] == C:
+            state["s"], state["j"] = 0, state["j"] + 1
+
+    for _ in range(2 * C):  # two jobs: every share of the following steps exists
+        advance(dev_factors)
+    for _ in range(args.warmup):
+        advance(dev_factors)
+    tda.tda_device_status()
+    torch.cuda.synchronize()
+
+    ev, phase_ev, open_ev = [], [], {}
+
+    def mark(name):
+        e = torch.cuda.Event(enable_timing=True)
+        e.record(stream)
+        phase_ev.append((name, e))
+
+    def hook(role, li, when, n):
+        if role != "train":
+            return
+        e = torch.cuda.Event(enable_timing=True)
+        e.record(stream)
+        if when == "begin":
+            open_ev[li] = e
+        else:
+            di, do = linears[li]
+            ev.append((open_ev.pop(li), e, n * (T * (di + do) * 2 + 4 * D)))
+
+    clocks = ClockSampler(0)
+    clocks.start()
+    time.sleep(0.3)
+    l0 = tda.tda_launch_count()
+    t0, t1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    t0.record(stream)
+    for _ in range(steps):
+        advance(dev_factors, mark, hook)
+    t1.record(stream)
+    torch.cuda.synchronize()
+    launches = tda.tda_launch_count() - l0
+    ck = clocks.stop()
+    tda.tda_device_status()
+    ms = t0.elapsed_time(t1) / steps
+    value = chunk / (ms * 1e-3)
+
+    peaks = {}
+    try:
+        with open(os.path.join(ROOT, "MEASURED_PEAKS.json")) as f:
+            peaks = json.load(f)
+    except OSError:
+        pass
+    hbm = float(peaks.get("hbm_gbs", 6800.0))
+    tf32x3 = float(peaks.get("bf16_tflops_sustained", 1700.0)) * 0.5 / 3.0
+    # the train projections of a step overlap across streams: the kernel's rate is its phase's
+    # algorithmic bytes over the phase's time (events on the launching stream around the fork
+    # and join of the projection streams)
+    proj_bytes = sum(x for _, _, x in ev)
+    ph_train = sum(a.elapsed_time(b) for (name, a), (_, b) in zip(phase_ev, phase_ev[1:]) if name == "project_train")
+    achieved = proj_bytes / (ph_train * 1e-3) / 1e9
+    per_launch = proj_bytes / max(len(ev), 1)
+    roofline = {"bound": "hbm", "kernel": f"factored projection (train, k = {k}, tcgen05)", "achieved": achieved,
+                "peak": hbm, "unit": "GB/s", "frac": achieved / hbm,
+                "traffic": None, "algorithmic_bytes_per_launch": per_launch, "launches_timed": len(ev),
+                "timing": (f"train projection phase of each step ({len(ev) // steps} launches over "
+                           f"{args.train_streams} stream(s)), CUDA events"),
+                "peak_source": "MEASURED_PEAKS.json hbm_gbs" if peaks else "fallback 6.8 TB/s",
+                "share_of_step": ph_train / (ms * steps)}
+    if k == 64 and projection_kernel_sha256() == TRAFFIC_KERNEL_SHA256:
+        roofline["traffic"] = TRAFFIC_RATIO * per_launch
+    ph = {}
+    for (name, a), (_, b) in zip(phase_ev, phase_ev[1:]):
+        if name is not None:
+            ph[name] = ph.get(name, 0.0) + a.elapsed_time(b) / steps
+    Dn = float(D)
+    per_job_lin = {
+        "project_train": ("hbm", sum(N * (T * (di + do) * 2 + 4 * D) for di, do in linears), hbm, "GB/s"),
+        "fisher_fit": ("tensor", nlin * N * Dn * (Dn + 1), tf32x3, "TFLOP/s"),
+        "project_query": ("hbm", sum(Nq * (T * (di + do) * 2 + 4 * D) for di, do in linears), hbm, "GB/s"),
+        "factor_apply": ("tensor", nlin * 2 * (Dn ** 3 / 3 + 2 * Dn * Dn * Nq), tf32x3, "TFLOP/s"),
+        "score": ("tensor", 2.0 * Nq * N * D * nlin, tf32x3, "TFLOP/s"),
+        "topk": ("latency", 4.0 * Nq * N, hbm, "GB/s"),
+    }
+    phases = {}
+    for name, ms_ in ph.items():
+        bound, work, peak, unit = per_job_lin[name]
+        rate = work / C / (ms_ * 1e-3) / (1e9 if unit == "GB/s" else 1e12)
+        phases[name] = {"ms": ms_, "bound": bound, "achieved": rate, "peak": peak, "unit": unit, "frac": rate / peak}
+
+    # ---- e2e: the same steps with the factors in pinned host memory
+    e2e = None
+    if not args.no_e2e:
+        saved_aff, numa = bind_to_gpu_numa(0)
+        Ph = spec["host_pool"]
+        hpools = []
+        for si in range(nshape):
+            A, B, Aq, Bq = pools[si]
+            hp = []
+            for x in (A, B, Aq, Bq):
+                h = torch.empty((Ph,) + tuple(x.shape[1:]), dtype=torch.bfloat16).pin_memory()
+                h.copy_(x[:Ph])
+                hp.append(h)
+            hpools.append(hp)
+        wsb = 2 * Ph * T * max(di + do for _, di, do in lin) * 2
+        job.host_ws_bytes = wsb
+        job.host_ws = torch.empty(wsb, dtype=torch.uint8, device=dev)
+
+        def host_factors(role, li, j, s):
+            A, B, Aq, Bq = hpools[li % nshape]
+            n_all, X, Y = (chunk, A, B) if role == "train" else (Nq, Aq, Bq)
+            return [(X[:min(Ph, n_all - r)], Y[:min(Ph, n_all - r)], r, min(Ph, n_all - r)) for r in range(0, n_all, Ph)]
+
+        # the H2D ceiling, measured as the e2e leg copies: four copy streams at once, several GB
+        copy_streams = [torch.cuda.Stream(device=dev) for _ in range(4)]
+        srcs = [hpools[si][i] for si in range(nshape) for i in range(2)]
+        dsts = [torch.empty_like(x, device=dev) for x in srcs]
+        nbytes = sum(x.numel() * 2 for x in srcs)
+        for rep in range(2):
+            torch.cuda.synchronize()
+            c0 = time.perf_counter()
+            for i, (hs, ds) in enumerate(zip(srcs, dsts)):
+                with torch.cuda.stream(copy_streams[i % 4]):
+                    ds.copy_(hs, non_blocking=True)
+            torch.cuda.synchronize()
+            h2d_gbs = nbytes / (time.perf_counter() - c0) / 1e9
+        del dsts
+        idx_h = torch.empty((Nq, args.topk), dtype=torch.int32).pin_memory()
+        val_h = torch.empty((Nq, args.topk), dtype=torch.float32).pin_memory()
+
+        def e2e_step():
+            s = state["s"]
+            advance(host_factors)
+            r0, r1 = job.share(s, Nq)
+            idx_h[r0:r1].copy_(job.idx[r0:r1], non_blocking=True)
+            val_h[r0:r1].copy_(job.val[r0:r1], non_blocking=True)
+            stream.synchronize()
+
+        e2e_step()
+        torch.cuda.synchronize()
+        n_e2e = max(1, args.e2e_steps)
+        c0 = time.perf_counter()
+        for _ in range(n_e2e):
+            e2e_step()
+        e2e_s = (time.perf_counter() - c0) / n_e2e
+        tda.tda_device_status()
+        h2d = (chunk * T * sum(di + do for di, do in linears) * 2
+               + Nq * T * sum(di + do for di, do in linears) * 2 // C)
+        e2e = {"value": chunk / e2e_s, "unit": "examples/s", "h2d_bytes_per_step": h2d,
+               "d2h_bytes_per_step": (Nq // C) * args.topk * 8, "ms_per_step": e2e_s * 1e3, "steps": n_e2e,
+               "host_pool_examples": Ph, "h2d_gbs_measured_4_streams": h2d_gbs,
+               "h2d_bound_examples_per_s": chunk / (h2d / (h2d_gbs * 1e9)), "host_numa_node": numa}
+        if saved_aff is not None:
+            os.sched_setaffinity(0, saved_aff)
+
+    cpu = None
+    if not args.no_cpu_baseline:
+        def factors_of(role, li, n):
+            A, B, Aq, Bq = pools[li]
+            X, Y = (A, B) if role == "train" else (Aq, Bq)
+            return (X[:n].float().cpu().numpy().astype(np.float64), Y[:n].float().cpu().numpy().astype(np.float64))
+
+        v, cores, sample, _ = stack_oracle_sample(spec, factors_of)
+        cpu = {"value": v, "unit": "examples/s", "cores": cores, "kind": "oracle", "sample": sample}
+
+    line = {
+        "metric": METRIC, "value": value, "unit": "examples/s", "n_gpus": 1, "steps": steps, "warmup": args.warmup,
+        "ms_per_step": ms, "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "bf16",
+        "data": "synthetic", "config": stack_config(args, spec), "roofline": roofline, "phases": phases,
+        "cpu_baseline": cpu, "e2e": e2e, "gpu_launches": launches, "clocks": ck,
+    }
+    print(json.dumps(line), flush=True)
+    return 0
+
+
 def main():
     args = parse_args()
+    if args.workload in STACKS:
+        if args.impl == "reference":
+            return stack_reference_main(args, STACKS[args.workload])
+        return stack_main(args, STACKS[args.workload])
     if args.impl == "reference":
         return reference_main(args)
     if args.route_sweep:
@@ -843,10 +1236,11 @@ def main():
             "metric": METRIC, "value": value, "unit": "examples/s", "n_gpus": world, "steps": args.steps,
             "warmup": args.warmup, "ms_per_step": ms, "higher_is_better": True, "scaling": "weak",
             "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
-            "config": {**workload(args), "parallelism": f"train examples sharded over {world} rank(s)"
-                       + (", curvature sums all-reduced, global top-k merged by all-gather" if world > 1 else ""),
-                       "routes": {name: {0: "factored", 1: "materialize", 2: "gram"}[r] for (name, _, _), r
-                                  in zip(LINEARS, pipe.routes())}},
+            "config": workload(args),
+            "ranks": world, **({"exchange": "curvature sums all-reduced, global top-k merged by all-gather"}
+                               if world > 1 else {}),
+            "routes": {name: {0: "factored", 1: "materialize", 2: "gram"}[r] for (name, _, _), r
+                       in zip(LINEARS, pipe.routes())},
             "roofline": roofline, "phases": phases, "cpu_baseline": cpu, "e2e": e2e, "gpu_launches": launches,
             "clocks": ck,
         }

@@ -173,8 +173,13 @@ tda_status tda_project_host(const tda_layer_desc* L, tda_dtype dtype, const void
  *   Arguments as tda_project; A, B, phi are still the caller's buffers.
  *   Rejects (TDA_ERR_WORKSPACE) a layer whose per-example scratch,
  *   4*(d_out*d_in + d_out*k_in) bytes, exceeds the array.
- *   The first call on a device, with that device current, resolves the
- *   array's device address (cudaGetSymbolAddress); make that first call
+ *   The first call in a CUDA context (normally the runtime's primary context
+ *   of the current device) resolves the array's device address
+ *   (cudaGetSymbolAddress) and caches it for that context. Under lazy module
+ *   loading (CUDA_MODULE_LOADING=LAZY, the default) that first call is also
+ *   when the driver loads the module and commits the 64 MiB, so it can fail
+ *   with TDA_ERR_CUDA if the device is full: make the first call at
+ *   initialisation, before the host program takes the rest of the memory and
  *   before any stream capture.
  *   Every call shares the one array and leaves its contents behind; the
  *   kernels overwrite what they read, so nothing needs clearing. Calls whose
@@ -284,10 +289,16 @@ tda_status tda_cosine(float* S, int64_t n_q, int64_t n_t, int64_t ld_S, const fl
  *                     Needs D <= 40960 (F32) or 20480 (F64).
  *   TDA_PC_FACTOR_APPLY  FACTOR, then APPLY, in one call (same arguments and
  *                     results as the two; a failed layer's rows are NaN). For an
- *                     F32 state with D a multiple of 32 and n_q <= 256 both run
- *                     in one launch: the query rows are solved alongside the
- *                     factorisation (forward substitution as extra rows of each
- *                     step) and then backward. qhat may not alias q.
+ *                     F32 state with D a multiple of 32 below 2048 and n_q <= 256
+ *                     both run in one launch: the query rows are solved alongside
+ *                     the factorisation (forward substitution as extra rows of
+ *                     each step) and then backward. qhat may not alias q.
+ * Large layers (F32 state, D a multiple of 128, D >= 2048): FACTOR is a blocked
+ * Cholesky in 256-column panels whose trailing updates run on the tensor cores
+ * (3xTF32, fp32-accurate); it also leaves L^T in M's upper triangle, and APPLY
+ * (qhat 16-byte aligned, ld_qhat a multiple of 4) then solves the query rows in
+ * 128-column blocks with tensor-core updates. In this mode qhat may alias q
+ * (same pointer and row stride: solved in place).
  * Arguments not used by an op are ignored (may be 0/NULL).
  * ------------------------------------------------------------------------- */
 #define TDA_PC_RESET 0

@@ -268,6 +268,8 @@ tda_status tda_workspace_size(tda_op op, const tda_layer_desc* L, tda_dtype dtyp
     }
     if (op == TDA_OP_PROJECT) {
         if (route == TDA_ROUTE_MATERIALIZE) *bytes = materialize_ws_bytes_per_example(*L);
+        // optional for the factored route: k = 128 bf16 reads precomputed sign tiles from it
+        if (route == TDA_ROUTE_FACTORED && dtype == TDA_BF16) *bytes = project_tc_sign_table_bytes(*L);
         return TDA_OK;
     }
     if (op == TDA_OP_SIMILARITY_EXACT) {
@@ -313,7 +315,7 @@ tda_status tda_project(const tda_layer_desc* L, tda_dtype dtype, const void* A, 
         if (dtype == TDA_BF16 && project_tc_plain_supported(*L, A, B)) {
             unsigned int* err = device_error_word();
             if (!err) return fail(TDA_ERR_CUDA, "cannot resolve the device error word");
-            return cuda_check(launch_project_tc(*L, A, B, N, phi, ld_phi, err, s), "project (tcgen05)");
+            return cuda_check(launch_project_tc(*L, A, B, N, phi, ld_phi, err, s, ws, ws_bytes), "project (tcgen05)");
         }
         return cuda_check(launch_project_simt(*L, dtype, A, B, N, phi, ld_phi, s), "project (simt)");
     }

@@ -52,10 +52,13 @@ struct GParams {
     const float* B;  // Qhat, n_q rows
     float* S;
     int64_t n_t, n_q, K, lda, ldb, ld_S;
-    float beta;
+    float beta, alpha;     // S = beta * S + alpha * (product); the score uses alpha = 1
+    int lower;             // square product (n_t == n_q, BN == kBM): only tiles with m0 <= n0
     int cs, tiles_n;
     int64_t kslice, slab;  // split-K over gridDim.y: K slice per CTA row, S stride per slice (0: no split)
     int splits;            // gridDim.y
+    int batched;           // grid z = batch entry: A and B maps are 3-D (z the third coordinate)
+    int64_t s_z;           // S element offset between batch entries
     unsigned int* err;
 };
 
@@ -144,11 +147,20 @@ score3x_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
 
     const uint32_t crank = cluster_rank();
     const int64_t tile = blockIdx.x / p.cs;
-    const int64_t m0 = (tile / p.tiles_n) * kBM, n0 = (tile % p.tiles_n) * BN;
+    int64_t m0 = (tile / p.tiles_n) * kBM, n0 = (tile % p.tiles_n) * BN;
+    if (p.lower) {
+        // tile t of the lower triangle: row tile i (n), column tile j (m) <= i, t = i(i+1)/2 + j
+        int64_t i = (int64_t)((sqrt(8.0 * (double)tile + 1.0) - 1.0) * 0.5);
+        while (i * (i + 1) / 2 > tile) --i;
+        while ((i + 1) * (i + 2) / 2 <= tile) ++i;
+        n0 = i * BN;
+        m0 = (tile - i * (i + 1) / 2) * kBM;
+    }
     // split-K slice z covers features [z*kslice, z*kslice + Kz) and writes its own slab of S
     const int64_t kbase = (int64_t)blockIdx.y * p.kslice;
     const int64_t Kz = p.kslice ? ((p.K - kbase) < p.kslice ? (p.K - kbase) : p.kslice) : p.K;
-    float* Sz = p.S + (int64_t)blockIdx.y * p.slab;
+    float* Sz = p.S + (int64_t)blockIdx.y * p.slab + (int64_t)blockIdx.z * p.s_z;
+    const int zc = (int)blockIdx.z;
     const int64_t nkc = (Kz + kKC - 1) / kKC;
     const int64_t per = (nkc + p.cs - 1) / p.cs;
     const int64_t kc0 = crank * per, kc1 = (kc0 + per) < nkc ? (kc0 + per) : nkc;
@@ -187,8 +199,13 @@ score3x_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
                 const uint32_t st = smem_u32(smem + (size_t)s * C::kStageBytes), bar = smem_u32(&raw_full[s]);
                 const int k = (int)(kbase + kc * kKC);
                 mbar_arrive_tx(bar, C::kABytes + C::kBBytes);
-                tma_load_2d(st, &tmA, k, (int)m0, bar);
-                tma_load_2d(st + 2 * C::kABytes, &tmB, k, (int)n0, bar);
+                if (p.batched) {
+                    tma_load_3d(st, &tmA, k, (int)m0, zc, bar);
+                    tma_load_3d(st + 2 * C::kABytes, &tmB, k, (int)n0, zc, bar);
+                } else {
+                    tma_load_2d(st, &tmA, k, (int)m0, bar);
+                    tma_load_2d(st + 2 * C::kABytes, &tmB, k, (int)n0, bar);
+                }
                 issued[s] = true;
                 last_par[s] = ph;
             }
@@ -308,12 +325,28 @@ score3x_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
             if (ok) {
                 const int64_t m = m0 + row;
                 if (m < p.n_t) {
+                    if (p.beta == 0.f) {
 #pragma unroll
-                    for (int c = 0; c < BN; ++c) {
-                        const int64_t n = n0 + c;
-                        if (n < p.n_q) {
-                            float* dst = Sz + n * p.ld_S + m;
-                            *dst = (p.beta == 0.f) ? acc[c] : p.beta * (*dst) + acc[c];
+                        for (int c = 0; c < BN; ++c) {
+                            const int64_t n = n0 + c;
+                            if (n < p.n_q) Sz[n * p.ld_S + m] = p.alpha * acc[c];
+                        }
+                    } else {
+                        // the previous values of 32 columns are loaded before any is stored, so
+                        // the loads are in flight together instead of one round trip per column
+#pragma unroll
+                        for (int c0 = 0; c0 < BN; c0 += 32) {
+                            float old[32];
+#pragma unroll
+                            for (int i = 0; i < 32; ++i) {
+                                const int64_t n = n0 + c0 + i;
+                                old[i] = n < p.n_q ? __ldcg(Sz + n * p.ld_S + m) : 0.f;
+                            }
+#pragma unroll
+                            for (int i = 0; i < 32; ++i) {
+                                const int64_t n = n0 + c0 + i;
+                                if (n < p.n_q) Sz[n * p.ld_S + m] = p.beta * old[i] + p.alpha * acc[c0 + i];
+                            }
                         }
                     }
                 }
@@ -653,12 +686,33 @@ bool make_map_f32(CUtensorMap* tm, const float* X, int64_t rows, int64_t K, int6
                CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
+// 3-D map over nz batch entries of fp32 X[rows][ld] (features 0..K-1 used), entry z at byte
+// offset z * z_bytes from X; box 32 features x box_rows rows x 1 entry, 128-byte swizzle.
+bool make_map_f32_3d(CUtensorMap* tm, const float* X, int64_t rows, int64_t K, int64_t ld, int64_t nz,
+                     size_t z_bytes, int box_rows) {
+    EncodeTiledFn enc = encode_fn();
+    if (!enc) return false;
+    cuuint64_t dims[3] = {(cuuint64_t)K, (cuuint64_t)rows, (cuuint64_t)nz};
+    cuuint64_t strides[2] = {(cuuint64_t)(ld * 4), (cuuint64_t)z_bytes};
+    cuuint32_t box[3] = {(cuuint32_t)kKC, (cuuint32_t)box_rows, 1};
+    cuuint32_t estr[3] = {1, 1, 1};
+    return enc(tm, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, 3, const_cast<float*>(X), dims, strides, box, estr,
+               CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+               CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
 template <int BN>
-cudaError_t launch_bn(GParams p, cudaStream_t s) {
+cudaError_t launch_bn(GParams p, cudaStream_t s, int64_t nz = 1, size_t a_z_bytes = 0, size_t b_z_bytes = 0) {
     using C = GCfg<BN>;
     CUtensorMap tmA, tmB;
-    if (!make_map_f32(&tmA, p.A, p.n_t, p.K, p.lda, kBM) || !make_map_f32(&tmB, p.B, p.n_q, p.K, p.ldb, BN))
+    if (nz > 1) {
+        if (!make_map_f32_3d(&tmA, p.A, p.n_t, p.K, p.lda, nz, a_z_bytes, kBM) ||
+            !make_map_f32_3d(&tmB, p.B, p.n_q, p.K, p.ldb, nz, b_z_bytes, BN))
+            return cudaErrorInvalidValue;
+        p.batched = 1;
+    } else if (!make_map_f32(&tmA, p.A, p.n_t, p.K, p.lda, kBM) || !make_map_f32(&tmB, p.B, p.n_q, p.K, p.ldb, BN)) {
         return cudaErrorInvalidValue;
+    }
     static int sms = 0;
     if (!sms) {
         int dev = 0;
@@ -667,10 +721,11 @@ cudaError_t launch_bn(GParams p, cudaStream_t s) {
         if (sms <= 0) sms = 1;
     }
     const int64_t tiles_m = (p.n_t + kBM - 1) / kBM, tiles_n = (p.n_q + BN - 1) / BN;
-    const int64_t tiles = tiles_m * tiles_n;
+    const int64_t tiles = p.lower ? tiles_n * (tiles_n + 1) / 2 : tiles_m * tiles_n;
     const int64_t nkc = ((p.kslice ? p.kslice : p.K) + kKC - 1) / kKC;
     int cs = 1;
-    while (cs < 4 && tiles * p.splits * cs * 2 <= sms && nkc >= 8 * cs * 2) cs *= 2;
+    // split K over a cluster only while the tiles of all batch entries leave SMs idle
+    while (cs < 4 && tiles * p.splits * nz * cs * 2 <= sms && nkc >= 8 * cs * 2) cs *= 2;
     // the leader's stage buffers must hold the members' partial tiles
     while (cs > 1 && (size_t)(cs - 1) * kBM * BN * 4 > (size_t)C::kStages * C::kStageBytes) cs >>= 1;
     p.cs = cs;
@@ -683,7 +738,7 @@ cudaError_t launch_bn(GParams p, cudaStream_t s) {
     attr[0].val.clusterDim.x = (unsigned)cs;
     attr[0].val.clusterDim.y = 1;
     attr[0].val.clusterDim.z = 1;
-    cfg.gridDim = dim3((unsigned)(tiles * cs), (unsigned)p.splits);
+    cfg.gridDim = dim3((unsigned)(tiles * cs), (unsigned)p.splits, (unsigned)nz);
     cfg.blockDim = dim3(kThreads);
     cfg.dynamicSmemBytes = C::kSmem;
     cfg.stream = s;
@@ -730,6 +785,7 @@ cudaError_t launch_score_tc(const float* Qhat, int64_t n_q, int64_t ld_q, const 
     p.ldb = ld_q;
     p.ld_S = ld_S;
     p.beta = beta;
+    p.alpha = 1.f;
     p.kslice = 0;
     p.slab = 0;
     p.splits = 1;
@@ -766,10 +822,68 @@ cudaError_t launch_score_tc_slices(const float* Qhat, int64_t n_q, int64_t ld_q,
     p.S = part;
     p.ld_S = n_t;
     p.beta = 0.f;
+    p.alpha = 1.f;
     p.err = err;
     if (p.splits > 65535) return cudaErrorInvalidValue;
     if (n_q <= 64) return launch_bn<64>(p, s);
     return launch_bn<128>(p, s);
+}
+
+cudaError_t launch_gemm_nt_tc_batched(const float* A, int64_t n_a, int64_t lda, size_t a_z_bytes, const float* B,
+                                      int64_t n_b, int64_t ldb, size_t b_z_bytes, int64_t K, float* C, int64_t ldc,
+                                      int64_t c_z, int64_t nz, float alpha, float beta, bool lower,
+                                      unsigned int* err, cudaStream_t s);
+
+// C[n][m] = beta * C[n][m] + alpha * sum_k A[m][k] B[n][k] (C row stride ldc): the
+// score GEMM with a sign, used by the blocked Cholesky and triangular solves. With
+// lower = true, A and B must be the same n x n operand rows (a symmetric rank-K
+// update) and only the 128 x 128 tiles on or below the diagonal (m0 <= n0) are
+// formed; entries above the diagonal inside a diagonal tile are written too.
+cudaError_t launch_gemm_nt_tc(const float* A, int64_t n_a, int64_t lda, const float* B, int64_t n_b, int64_t ldb,
+                              int64_t K, float* C, int64_t ldc, float alpha, float beta, bool lower,
+                              unsigned int* err, cudaStream_t s) {
+    return launch_gemm_nt_tc_batched(A, n_a, lda, 0, B, n_b, ldb, 0, K, C, ldc, 0, 1, alpha, beta, lower, err, s);
+}
+
+cudaError_t launch_gemm_nt_tc_batched(const float* A, int64_t n_a, int64_t lda, size_t a_z_bytes, const float* B,
+                                      int64_t n_b, int64_t ldb, size_t b_z_bytes, int64_t K, float* C, int64_t ldc,
+                                      int64_t c_z, int64_t nz, float alpha, float beta, bool lower,
+                                      unsigned int* err, cudaStream_t s) {
+    if (nz < 1 || nz > 65535) return cudaErrorInvalidValue;
+    if (nz > 1 && ((a_z_bytes & 15) || (b_z_bytes & 15) || !a_z_bytes || !b_z_bytes)) return cudaErrorInvalidValue;
+    GParams p{};
+    p.A = A;
+    p.B = B;
+    p.S = C;
+    p.n_t = n_a;
+    p.n_q = n_b;
+    p.K = K;
+    p.lda = lda;
+    p.ldb = ldb;
+    p.ld_S = ldc;
+    p.beta = beta;
+    p.alpha = alpha;
+    p.lower = lower ? 1 : 0;
+    p.kslice = 0;
+    p.slab = 0;
+    p.splits = 1;
+    p.s_z = c_z;
+    p.err = err;
+    if (lower && (n_a != n_b || n_b <= 64)) return cudaErrorInvalidValue;
+    if (n_b <= 64) return launch_bn<64>(p, s, nz, a_z_bytes, b_z_bytes);
+    return launch_bn<128>(p, s, nz, a_z_bytes, b_z_bytes);
+}
+
+bool gemm_tc_available() {
+    static int ok = -1;
+    if (ok < 0) {
+        int dev = 0, major = 0, minor = 0;
+        cudaGetDevice(&dev);
+        cudaDeviceGetAttribute(&major, cudaDevAttrComputeCapabilityMajor, dev);
+        cudaDeviceGetAttribute(&minor, cudaDevAttrComputeCapabilityMinor, dev);
+        ok = (major == 10 && minor == 3 && encode_fn()) ? 1 : 0;
+    }
+    return ok == 1;
 }
 
 bool fit_tc_supported(int n_layers, int64_t D, const float* phi, int64_t n, int64_t ld) {

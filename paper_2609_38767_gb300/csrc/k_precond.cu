@@ -21,6 +21,18 @@
 //   APPLY   forward and backward block substitution; with Dinv each 32-row
 //           block step is a small matrix product instead of a serial chain.
 // Every launch covers all layers of the call (grid z or y = layer).
+//
+// Blocked path (fp32 state, D a multiple of 128 and at least 2048): the same
+// right-looking Cholesky in 256-column panels of two 128-column halves. Per
+// half: the 128 x 128 diagonal block is factored in shared memory (its four
+// 32-column steps as above, Dinv of its four 32 x 32 blocks) and the rows below
+// it are solved against it (x L_BB^T = a); the second half's columns first take
+// the first half's update. The trailing lower triangle then takes the rank-256
+// update M -= P P^T on the tensor cores (3xTF32, launch_gemm_nt_tc). After the
+// last panel, L^T is copied into M's upper triangle. APPLY then solves the
+// query rows block by block: a 128-wide triangular solve per panel, and the
+// rest of every row updated by a tensor-core product with L's panel (forward)
+// or with L^T's panel from the upper triangle (backward).
 #include <math.h>
 
 #include "tda_internal.cuh"
@@ -1020,6 +1032,327 @@ cudaError_t apply_impl(int n_layers, int64_t D, const void* state, const float* 
     return cudaGetLastError();
 }
 
+// ---------------------------------------------------------------- blocked path (fp32)
+constexpr int kBB = 128;                // panel width
+constexpr int64_t kBlockedMinD = 2048;  // smaller layers keep the one-launch cluster path
+constexpr int kTrsmWarps = 8;
+constexpr size_t kDiagSmem = sizeof(float) * ((size_t)kBB * (kBB + 1) + (size_t)(kBB - kNB) * (kNB + 1));
+constexpr size_t kTrsmSmem =
+    sizeof(float) * ((size_t)kBB * (kBB + 1) + (size_t)(kBB / kNB) * kNB * (kNB + 1) + (size_t)kTrsmWarps * kBB);
+
+// Factor the 128 x 128 diagonal block at lo of every layer (grid = layer) in
+// shared memory, in four 32-column steps: Cholesky of the 32 x 32 block by one
+// warp (as panel_kernel), its inverse into Dinv, the block's rows below it
+// solved against it, the rest of the block updated. L returns to M's lower
+// triangle; a non-positive pivot is recorded in the header.
+__global__ void __launch_bounds__(256) diag_block_kernel(St<float> st, int64_t lo) {
+    extern __shared__ __align__(16) float dsm[];
+    float(*A)[kBB + 1] = reinterpret_cast<float(*)[kBB + 1]>(dsm);
+    float(*X)[kNB + 1] = reinterpret_cast<float(*)[kNB + 1]>(dsm + kBB * (kBB + 1));
+    __shared__ float Di[kNB][kNB + 1];
+    const int l = blockIdx.x;
+    const int64_t D = st.D;
+    float* M = st.M(l);
+    const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+    for (int e = tid; e < kBB * kBB; e += 256) {
+        const int i = e / kBB, j = e % kBB;
+        A[i][j] = (j <= i) ? M[(lo + i) * D + lo + j] : 0.f;
+    }
+    __syncthreads();
+    for (int c0 = 0; c0 < kBB; c0 += kNB) {
+        if (warp == 0) {
+            float r[kNB];
+#pragma unroll
+            for (int c = 0; c < kNB; ++c) r[c] = A[c0 + lane][c0 + c];
+            int bad = -1;
+#pragma unroll
+            for (int j = 0; j < kNB; ++j) {
+                const float p = __shfl_sync(0xffffffffu, r[j], j);
+                const bool ok = p > 0.f;
+                if (!ok && bad < 0) bad = j;
+                const float piv = ok ? sqrtf(p) : NAN;
+                if (lane == j) r[j] = piv;
+                if (lane > j) r[j] /= piv;
+#pragma unroll
+                for (int c = j + 1; c < kNB; ++c) {
+                    const float v = __shfl_sync(0xffffffffu, r[j], c);  // L[c][j]
+                    if (lane >= c) r[c] -= r[j] * v;
+                }
+            }
+#pragma unroll
+            for (int c = 0; c < kNB; ++c) A[c0 + lane][c0 + c] = (c <= lane) ? r[c] : 0.f;
+            if (lane == 0 && bad >= 0) {
+                double* h = st.header(l);
+                if (h[kPcFailedPivot] == 0.0) h[kPcFailedPivot] = (double)(lo + c0 + bad + 1);
+            }
+            __syncwarp();
+            // inverse of the block: lane c solves L x = e_c
+            float x[kNB];
+#pragma unroll
+            for (int i = 0; i < kNB; ++i) {
+                float t = (i == lane) ? 1.f : 0.f;
+#pragma unroll
+                for (int m = 0; m < i; ++m) t -= A[c0 + i][c0 + m] * x[m];
+                x[i] = (i < lane) ? 0.f : t / A[c0 + i][c0 + i];
+            }
+            float* Dg = st.Dinv(l) + ((lo + c0) / kNB) * (kNB * kNB);
+#pragma unroll
+            for (int i = 0; i < kNB; ++i) {
+                Di[i][lane] = x[i];
+                Dg[i * kNB + lane] = x[i];
+            }
+        }
+        __syncthreads();
+        const int rows = kBB - c0 - kNB;  // rows of the block below this step's diagonal block
+        // x L_ss^T = a, i.e. x_j = sum_{m <= j} Dinv[j][m] a_m
+        for (int e = tid; e < rows * kNB; e += 256) {
+            const int i = e / kNB, j = e % kNB;
+            float acc = 0.f;
+            for (int m = 0; m <= j; ++m) acc += Di[j][m] * A[c0 + kNB + i][c0 + m];
+            X[i][j] = acc;
+        }
+        __syncthreads();
+        for (int e = tid; e < rows * kNB; e += 256) {
+            const int i = e / kNB, j = e % kNB;
+            A[c0 + kNB + i][c0 + j] = X[i][j];
+        }
+        // the block's trailing lower triangle
+        for (int e = tid; e < rows * rows; e += 256) {
+            const int i = e / rows, j = e % rows;
+            if (j > i) continue;
+            float acc = 0.f;
+#pragma unroll 8
+            for (int m = 0; m < kNB; ++m) acc += X[i][m] * X[j][m];
+            A[c0 + kNB + i][c0 + kNB + j] -= acc;
+        }
+        __syncthreads();
+    }
+    for (int e = tid; e < kBB * kBB; e += 256) {
+        const int i = e / kBB, j = e % kBB;
+        if (j <= i) M[(lo + i) * D + lo + j] = A[i][j];
+    }
+}
+
+// Triangular solves of row vectors against the diagonal block B at lo of layer
+// l (grid y): FWD x <- L_BB^{-1} x, else x <- L_BB^{-T} x, for n_rows rows of
+// 128 values at column lo of X (row stride ldx, layer l's rows at byte offset
+// l * layer_bytes from base). One warp per row; the block's L and its four
+// diagonal inverses sit in shared memory. Used for the panel (rows of M below
+// the block, FWD) and for the query rows of APPLY (both directions).
+template <bool FWD>
+__global__ void __launch_bounds__(256) trsm_block_kernel(St<float> st, int64_t lo, char* base, size_t layer_bytes,
+                                                         int64_t ldx, int64_t n_rows) {
+    extern __shared__ __align__(16) float tsm[];
+    float(*Lb)[kBB + 1] = reinterpret_cast<float(*)[kBB + 1]>(tsm);
+    float(*Di)[kNB][kNB + 1] = reinterpret_cast<float(*)[kNB][kNB + 1]>(tsm + kBB * (kBB + 1));
+    float* Y = tsm + kBB * (kBB + 1) + (kBB / kNB) * kNB * (kNB + 1);
+    const int l = blockIdx.y;
+    const int64_t D = st.D;
+    const float* M = st.M(l);
+    const float* Dv = st.Dinv(l) + (lo / kNB) * (kNB * kNB);
+    const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+    for (int e = tid; e < kBB * kBB; e += 256) {
+        const int i = e / kBB, j = e % kBB;
+        Lb[i][j] = (j <= i) ? M[(lo + i) * D + lo + j] : 0.f;
+    }
+    for (int e = tid; e < (kBB / kNB) * kNB * kNB; e += 256) {
+        const int b = e / (kNB * kNB), i = (e / kNB) % kNB, j = e % kNB;
+        Di[b][i][j] = Dv[e];
+    }
+    __syncthreads();
+    float* y = Y + warp * kBB;
+    float* X = (float*)(base + (size_t)l * layer_bytes);
+    for (int64_t r = (int64_t)blockIdx.x * kTrsmWarps + warp; r < n_rows; r += (int64_t)gridDim.x * kTrsmWarps) {
+        float* x = X + r * ldx + lo;
+#pragma unroll
+        for (int c = lane; c < kBB; c += 32) y[c] = x[c];
+        __syncwarp();
+        if (FWD) {
+#pragma unroll 1
+            for (int b = 0; b < kBB / kNB; ++b) {
+                const int c0 = b * kNB;
+                float acc = y[c0 + lane];
+                for (int m = 0; m < c0; ++m) acc -= Lb[c0 + lane][m] * y[m];
+                float out = 0.f;
+#pragma unroll
+                for (int m = 0; m < kNB; ++m) {
+                    const float rm = __shfl_sync(0xffffffffu, acc, m);
+                    if (m <= lane) out += Di[b][lane][m] * rm;
+                }
+                __syncwarp();
+                y[c0 + lane] = out;
+                __syncwarp();
+            }
+        } else {
+#pragma unroll 1
+            for (int b = kBB / kNB - 1; b >= 0; --b) {
+                const int c0 = b * kNB;
+                float acc = y[c0 + lane];
+                for (int m = c0 + kNB; m < kBB; ++m) acc -= Lb[m][c0 + lane] * y[m];
+                float out = 0.f;
+#pragma unroll
+                for (int j = 0; j < kNB; ++j) {
+                    const float rj = __shfl_sync(0xffffffffu, acc, j);
+                    if (j >= lane) out += Di[b][j][lane] * rj;
+                }
+                __syncwarp();
+                y[c0 + lane] = out;
+                __syncwarp();
+            }
+        }
+#pragma unroll
+        for (int c = lane; c < kBB; c += 32) x[c] = y[c];
+        __syncwarp();
+    }
+}
+
+// M[i][j] = M[j][i] for every 32 x 32 block strictly above the diagonal blocks
+// (U = L^T, read by the backward solve's tensor-core products).
+__global__ void __launch_bounds__(256) upper_from_lower_kernel(St<float> st, int n_layers) {
+    __shared__ float t[kNB][kNB + 1];
+    const int64_t D = st.D, nb = D / kNB, pairs = nb * (nb - 1) / 2;
+    const int tx = threadIdx.x & 31, ty = threadIdx.x >> 5;
+    for (int64_t w = blockIdx.x; w < pairs * n_layers; w += gridDim.x) {
+        const int l = (int)(w / pairs);
+        const int64_t p = w - (int64_t)l * pairs;
+        int64_t bj = (int64_t)((1.0 + sqrt(1.0 + 8.0 * (double)p)) * 0.5);  // p = bj(bj-1)/2 + bi, bi < bj
+        while (bj * (bj - 1) / 2 > p) --bj;
+        while ((bj + 1) * bj / 2 <= p) ++bj;
+        const int64_t bi = p - bj * (bj - 1) / 2;
+        float* M = st.M(l);
+        for (int r = ty; r < kNB; r += 8) t[r][tx] = M[(bj * kNB + r) * D + bi * kNB + tx];
+        __syncthreads();
+        for (int r = ty; r < kNB; r += 8) M[(bi * kNB + r) * D + bj * kNB + tx] = t[tx][r];
+        __syncthreads();
+    }
+}
+
+// Query rows of a layer whose factorisation failed become NaN.
+__global__ void nan_failed_kernel(St<float> st, float* qhat, int64_t ld, int64_t n_q) {
+    const int l = blockIdx.y;
+    if (st.header(l)[kPcFailedPivot] == 0.0) return;
+    const int64_t D = st.D;
+    for (int64_t e = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; e < n_q * D; e += (int64_t)gridDim.x * blockDim.x)
+        qhat[(e / D) * ld + (int64_t)l * D + e % D] = NAN;
+}
+
+bool blocked_pc(int64_t D, tda_dtype sdt) {
+    return sdt == TDA_F32 && D % kBB == 0 && D >= kBlockedMinD && D < (1LL << 31) / kBB && gemm_tc_available();
+}
+
+cudaError_t blocked_attrs() {
+    static cudaError_t e = [] {
+        cudaError_t r = cudaFuncSetAttribute(diag_block_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                             (int)kDiagSmem);
+        if (r == cudaSuccess)
+            r = cudaFuncSetAttribute(trsm_block_kernel<true>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                     (int)kTrsmSmem);
+        if (r == cudaSuccess)
+            r = cudaFuncSetAttribute(trsm_block_kernel<false>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                     (int)kTrsmSmem);
+        return r;
+    }();
+    return e;
+}
+
+unsigned trsm_grid(int64_t n_rows, int n_layers) {
+    int64_t g = (n_rows + kTrsmWarps - 1) / kTrsmWarps;
+    const int64_t cap = n_layers >= 304 ? 1 : 304 / n_layers;  // about two CTAs per SM over all layers
+    if (g > cap) g = cap;
+    return (unsigned)(g < 1 ? 1 : g);
+}
+
+cudaError_t factor_blocked(int n_layers, int64_t D, void* state, int64_t n_total, double la, double lr,
+                           cudaStream_t s) {
+    cudaError_t e = blocked_attrs();
+    if (e != cudaSuccess) return e;
+    unsigned int* err = device_error_word();
+    if (!err) return cudaErrorUnknown;
+    St<float> st = state_of<float>(state, D);
+    note_launches(2);
+    prepare_kernel<float><<<n_layers, 256, 0, s>>>(st, n_total, la, lr);
+    int64_t blocks = (D * D * n_layers + 255) / 256;
+    if (blocks > 152 * 16) blocks = 152 * 16;
+    scale_kernel<float><<<(unsigned)blocks, 256, 0, s>>>(st, n_layers);
+    // outer panels of 256 columns, each two 128-column sub-panels: the second sub-panel's
+    // columns take the first one's update alone (a 128-wide product), and the trailing
+    // matrix takes both at once (rank-256 update: twice the work per tile pass over M)
+    float* M0 = (float*)((char*)state + 64);  // layer l's M is st.bytes further on
+    const int64_t cz = (int64_t)(st.bytes / 4);
+    for (int64_t lo = 0; lo < D; lo += 2 * kBB) {
+        const int64_t mid = lo + kBB;
+        note_launches(1);
+        diag_block_kernel<<<n_layers, 256, kDiagSmem, s>>>(st, lo);
+        if (mid == D) break;
+        note_launches(1);
+        trsm_block_kernel<true><<<dim3(trsm_grid(D - mid, n_layers), n_layers), 256, kTrsmSmem, s>>>(
+            st, lo, (char*)M0 + (size_t)mid * D * 4, st.bytes, D, D - mid);
+        // rows [mid, D) of columns [mid, mid + 128) -= L[rows, lo:mid] L[mid:mid+128, lo:mid]^T
+        e = launch_gemm_nt_tc_batched(M0 + mid * D + lo, kBB, D, st.bytes, M0 + mid * D + lo, D - mid, D, st.bytes,
+                                      kBB, M0 + mid * D + mid, D, cz, n_layers, -1.f, 1.f, false, err, s);
+        if (e != cudaSuccess) return e;
+        note_launches(1);
+        diag_block_kernel<<<n_layers, 256, kDiagSmem, s>>>(st, mid);
+        const int64_t hi = mid + kBB, rest = D - hi;
+        if (rest == 0) break;
+        note_launches(1);
+        trsm_block_kernel<true><<<dim3(trsm_grid(rest, n_layers), n_layers), 256, kTrsmSmem, s>>>(
+            st, mid, (char*)M0 + (size_t)hi * D * 4, st.bytes, D, rest);
+        // trailing lower triangle of all layers in one launch: M -= P P^T, P = L[hi:D, lo:hi]
+        e = launch_gemm_nt_tc_batched(M0 + hi * D + lo, rest, D, st.bytes, M0 + hi * D + lo, rest, D, st.bytes,
+                                      2 * kBB, M0 + hi * D + hi, D, cz, n_layers, -1.f, 1.f, true, err, s);
+        if (e != cudaSuccess) return e;
+    }
+    const int64_t nb = D / kNB;
+    int64_t g = nb * (nb - 1) / 2 * n_layers;
+    if (g > 152 * 8) g = 152 * 8;
+    note_launches(1);
+    upper_from_lower_kernel<<<(unsigned)g, 256, 0, s>>>(st, n_layers);
+    return cudaGetLastError();
+}
+
+bool apply_blocked_ok(int64_t D, tda_dtype sdt, const void* qhat, int64_t ld_qhat, int64_t n_q) {
+    return blocked_pc(D, sdt) && ((uintptr_t)qhat & 15) == 0 && (ld_qhat & 3) == 0 && n_q < (1LL << 24);
+}
+
+cudaError_t apply_blocked(int n_layers, int64_t D, const void* state, const float* q, int64_t n_q, int64_t ld_q,
+                          float* qhat, int64_t ld_qhat, cudaStream_t s) {
+    cudaError_t e = blocked_attrs();
+    if (e != cudaSuccess) return e;
+    unsigned int* err = device_error_word();
+    if (!err) return cudaErrorUnknown;
+    St<float> st = state_of<float>(const_cast<void*>(state), D);
+    if (q != qhat || ld_q != ld_qhat) {
+        e = cudaMemcpy2DAsync(qhat, (size_t)ld_qhat * 4, q, (size_t)ld_q * 4, (size_t)n_layers * D * 4, (size_t)n_q,
+                              cudaMemcpyDeviceToDevice, s);
+        if (e != cudaSuccess) return e;
+    }
+    const unsigned gx = trsm_grid(n_q, n_layers);
+    const size_t lb = (size_t)D * 4;  // layer l's columns start l * D floats into each row
+    const float* M0 = (const float*)((const char*)state + 64);  // layer l's M is st.bytes further on
+    for (int64_t lo = 0; lo < D; lo += kBB) {
+        note_launches(1);
+        trsm_block_kernel<true><<<dim3(gx, n_layers), 256, kTrsmSmem, s>>>(st, lo, (char*)qhat, lb, ld_qhat, n_q);
+        const int64_t hi = lo + kBB;
+        if (hi == D) break;
+        e = launch_gemm_nt_tc_batched(M0 + hi * D + lo, D - hi, D, st.bytes, qhat + lo, n_q, ld_qhat, lb, kBB,
+                                      qhat + hi, ld_qhat, D, n_layers, -1.f, 1.f, false, err, s);
+        if (e != cudaSuccess) return e;
+    }
+    for (int64_t lo = D - kBB; lo >= 0; lo -= kBB) {
+        note_launches(1);
+        trsm_block_kernel<false><<<dim3(gx, n_layers), 256, kTrsmSmem, s>>>(st, lo, (char*)qhat, lb, ld_qhat, n_q);
+        if (lo == 0) break;
+        // rows [0, lo) of U = L^T, columns [lo, lo + 128): U[i][j] = L[j][i]
+        e = launch_gemm_nt_tc_batched(M0 + lo, lo, D, st.bytes, qhat + lo, n_q, ld_qhat, lb, kBB, qhat, ld_qhat, D,
+                                      n_layers, -1.f, 1.f, false, err, s);
+        if (e != cudaSuccess) return e;
+    }
+    note_launches(1);
+    nan_failed_kernel<<<dim3(64, n_layers), 256, 0, s>>>(st, qhat, ld_qhat, n_q);
+    return cudaGetLastError();
+}
+
 }  // namespace
 
 int64_t precondition_apply_max_d(tda_dtype sdt) {
@@ -1048,6 +1381,7 @@ cudaError_t launch_pc_fit(int n_layers, int64_t D, tda_dtype sdt, void* state, c
 
 cudaError_t launch_pc_factor(int n_layers, int64_t D, tda_dtype sdt, void* state, int64_t n_total,
                              double lambda_abs, double lambda_rel, cudaStream_t s) {
+    if (blocked_pc(D, sdt)) return factor_blocked(n_layers, D, state, n_total, lambda_abs, lambda_rel, s);
     if (sdt == TDA_F64) return factor_impl<double>(n_layers, D, state, n_total, lambda_abs, lambda_rel, s);
     return factor_impl<float>(n_layers, D, state, n_total, lambda_abs, lambda_rel, s);
 }
@@ -1056,8 +1390,9 @@ cudaError_t launch_pc_factor_apply(int n_layers, int64_t D, tda_dtype sdt, void*
                                    double lambda_abs, double lambda_rel, const float* q, int64_t n_q, int64_t ld_q,
                                    void* qhat, int64_t ld_qhat, cudaStream_t s) {
     // fp32 state, whole 32-column blocks, up to 256 queries: factorisation and both
-    // substitutions in one cluster launch per call; otherwise FACTOR, then APPLY
-    if (sdt == TDA_F32 && D % kNB == 0 && D >= 2 * kNB && n_q >= 1 && n_q <= 256) {
+    // substitutions in one cluster launch per call (below the blocked path's sizes);
+    // otherwise FACTOR, then APPLY
+    if (sdt == TDA_F32 && !blocked_pc(D, sdt) && D % kNB == 0 && D >= 2 * kNB && n_q >= 1 && n_q <= 256) {
         const QArgs qa{q, (float*)qhat, n_q, ld_q, ld_qhat};
         cudaError_t e = factor_cluster<16, true>(n_layers, D, state, n_total, lambda_abs, lambda_rel, qa, s);
         if (e == cudaErrorNotSupported)
@@ -1072,6 +1407,9 @@ cudaError_t launch_pc_factor_apply(int n_layers, int64_t D, tda_dtype sdt, void*
 cudaError_t launch_pc_apply(int n_layers, int64_t D, tda_dtype sdt, const void* state, const float* q,
                             int64_t n_q, int64_t ld_q, void* qhat, int64_t ld_qhat, cudaStream_t s) {
     if (n_q == 0) return cudaSuccess;
+    // a blocked factorisation left L^T in M's upper triangle: tensor-core substitutions
+    if (apply_blocked_ok(D, sdt, qhat, ld_qhat, n_q))
+        return apply_blocked(n_layers, D, state, q, n_q, ld_q, (float*)qhat, ld_qhat, s);
     const size_t el = sdt == TDA_F64 ? 8 : 4;
     const size_t budget = 160 * 1024;
     if (sdt == TDA_F64) {

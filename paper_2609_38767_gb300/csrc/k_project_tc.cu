@@ -46,6 +46,7 @@
 #include <cuda.h>
 #include <cuda_bf16.h>
 
+#include <cstring>
 #include <mutex>
 
 #include "tda_internal.cuh"
@@ -252,10 +253,13 @@ __device__ __forceinline__ void store_sign_row(uint8_t* tile, int n, const uint4
 }
 
 // KF: also accumulate the K-FAC factor covariances. FO: write the projected
-// factors At, Bt of every token instead of contracting them into Phi.
-template <int K, int G, bool KF, bool FO>
+// factors At, Bt of every token instead of contracting them into Phi. SL: the
+// sign tiles come by TMA from a precomputed table (tmSA, tmSB: [K][d] bf16, a
+// side's S transposed) instead of the generator warps.
+template <int K, int G, bool KF, bool FO, bool SL = false>
 __global__ void __launch_bounds__(kThreads, 1)
 project_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
+                  const __grid_constant__ CUtensorMap tmSA, const __grid_constant__ CUtensorMap tmSB,
                   const Params p) {
     using C = Cfg<K, G>;
     extern __shared__ uint8_t smem_raw[];
@@ -326,7 +330,10 @@ project_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant
                 }
                 const bool side_b = kc >= p.nk_in;
                 const int d0 = (side_b ? kc - p.nk_in : kc) * kChunkK;
-                mbar_arrive_tx(smem_u32(&full[s]), (uint32_t)ng * kTileBytes);
+                mbar_arrive_tx(smem_u32(&full[s]), (uint32_t)ng * kTileBytes + (SL ? C::kSignBytes : 0u));
+                if constexpr (SL)
+                    tma_load_3d(smem_u32(sA + (size_t)s * C::kStageBytes + (size_t)G * kTileBytes),
+                                side_b ? &tmSB : &tmSA, d0, 0, 0, smem_u32(&full[s]));
                 for (int u = 0; u < ng; ++u) {
                     // packed tiles: row x * pack * T of the [N*T][d] view; else tile tt of example x
                     const int row = p.pack > 1 ? (int)(gx[u] * p.pack * p.T) : gt[u] * kTileM;
@@ -363,7 +370,7 @@ project_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant
                 const int s = ring % C::kStages;
                 const uint32_t ph = (ring / C::kStages) & 1u;
                 if (!wait_bounded(smem_u32(&full[s]), ph, abort, p.err) ||
-                    !wait_bounded(smem_u32(&sready[s]), ph, abort, p.err)) {
+                    (!SL && !wait_bounded(smem_u32(&sready[s]), ph, abort, p.err))) {
                     ok = false;
                     break;
                 }
@@ -392,7 +399,7 @@ project_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant
                 atomicOr(p.err, kErrTimeout);
                 break;
             }
-    } else if (warp == 2 || warp == 3) {
+    } else if (!SL && (warp == 2 || warp == 3)) {
         // ---------------- sign generators (two warps, one half-row each)
         uint32_t ring = 0;
         bool ok = true;
@@ -766,6 +773,49 @@ bool make_map(CUtensorMap* tm, const void* X, int64_t N, int64_t T, int64_t d) {
                CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
+// A side's sign table for the SL kernel: tab[j][r] = S[r][j] as bf16 +-1 for
+// r < d, j < K (bit r mod 64 of sign word (j, r / 64); a set bit is -1), the
+// same signs the generator warps write. One thread per (column, 64-row group).
+__global__ void sign_table_kernel(uint16_t* __restrict__ tab, int64_t d, int K, uint64_t key) {
+    const int64_t groups = (d + 63) / 64;
+    for (int64_t e = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; e < groups * K;
+         e += (int64_t)gridDim.x * blockDim.x) {
+        const int j = (int)(e / groups);
+        const int64_t rb = e - (int64_t)j * groups;
+        const uint64_t w = sign_word(key, (uint32_t)j, (uint64_t)rb);
+        uint16_t* row = tab + (int64_t)j * d + rb * 64;
+        const int64_t n = (d - rb * 64) < 64 ? (d - rb * 64) : 64;
+        if (n == 64) {
+#pragma unroll
+            for (int c = 0; c < 8; ++c) {
+                uint32_t q[4];
+#pragma unroll
+                for (int t = 0; t < 4; ++t) {
+                    const uint32_t lo = 0x3F80u | ((uint32_t)((w >> (8 * c + 2 * t)) & 1u) << 15);
+                    const uint32_t hi = 0x3F80u | ((uint32_t)((w >> (8 * c + 2 * t + 1)) & 1u) << 15);
+                    q[t] = lo | (hi << 16);
+                }
+                *reinterpret_cast<uint4*>(row + 8 * c) = make_uint4(q[0], q[1], q[2], q[3]);
+            }
+        } else {
+            for (int64_t r = 0; r < n; ++r) row[r] = (uint16_t)(0x3F80u | ((uint32_t)((w >> r) & 1u) << 15));
+        }
+    }
+}
+
+// 3-D map over a sign table [1][K][d] (bf16): box 64 (d) x K x 1, 128B swizzle, zero fill past d.
+bool make_sign_map(CUtensorMap* tm, const void* tab, int64_t d, int K) {
+    EncodeTiledFn enc = encode_fn();
+    if (!enc) return false;
+    cuuint64_t dims[3] = {(cuuint64_t)d, (cuuint64_t)K, 1};
+    cuuint64_t strides[2] = {(cuuint64_t)(d * 2), (cuuint64_t)(K * d * 2)};
+    cuuint32_t box[3] = {kChunkK, (cuuint32_t)K, 1};
+    cuuint32_t estr[3] = {1, 1, 1};
+    return enc(tm, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, const_cast<void*>(tab), dims, strides, box, estr,
+               CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+               CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
 bool device_is_sm103() {
     int dev = 0;
     if (cudaGetDevice(&dev) != cudaSuccess) return false;
@@ -792,12 +842,20 @@ int sm_count() {
     return (b > 0 && b < sms) ? b : sms;
 }
 
-template <int K, int G, bool KF, bool FO>
+template <int K, int G, bool KF, bool FO, bool SL = false>
 cudaError_t launch_kg(const tda_layer_desc& L, const void* A, const void* B, int64_t N, float* phi,
                       int64_t ld_phi, unsigned int* err, cudaStream_t s, int pack, float* cov, int* grid_out,
-                      float* fout) {
+                      float* fout, const void* signs = nullptr) {
     using C = Cfg<K, G>;
-    CUtensorMap tmA, tmB;
+    CUtensorMap tmA, tmB, tmSA, tmSB;
+    if constexpr (SL) {
+        const uint16_t* tab = (const uint16_t*)signs;
+        if (!make_sign_map(&tmSA, tab, L.d_in, K) || !make_sign_map(&tmSB, tab + (int64_t)K * L.d_in, L.d_out, K))
+            return cudaErrorInvalidValue;
+    } else {
+        memset(&tmSA, 0, sizeof(tmSA));
+        memset(&tmSB, 0, sizeof(tmSB));
+    }
     if (pack > 1) {
         if (!make_map(&tmA, A, 1, N * L.T, L.d_in) || !make_map(&tmB, B, 1, N * L.T, L.d_out))
             return cudaErrorInvalidValue;
@@ -823,8 +881,8 @@ cudaError_t launch_kg(const tda_layer_desc& L, const void* A, const void* B, int
     p.cov = cov;
     p.fout = fout;
     const int sms = sm_count();
-    cudaError_t e = cudaFuncSetAttribute(project_tc_kernel<K, G, KF, FO>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                         (int)C::kSmem);
+    cudaError_t e = cudaFuncSetAttribute(project_tc_kernel<K, G, KF, FO, SL>,
+                                         cudaFuncAttributeMaxDynamicSharedMemorySize, (int)C::kSmem);
     if (e != cudaSuccess) return e;
     // Fewer examples than SMs: a cluster of cs CTAs shares each example's token
     // tiles and reduces the partial features through distributed shared memory.
@@ -845,7 +903,7 @@ cudaError_t launch_kg(const tda_layer_desc& L, const void* A, const void* B, int
     cfg.numAttrs = 1;
     int max_clusters = 0;
     cfg.gridDim = dim3((unsigned)(cs * (sms / cs)));
-    if (cudaOccupancyMaxActiveClusters(&max_clusters, project_tc_kernel<K, G, KF, FO>, &cfg) != cudaSuccess ||
+    if (cudaOccupancyMaxActiveClusters(&max_clusters, project_tc_kernel<K, G, KF, FO, SL>, &cfg) != cudaSuccess ||
         max_clusters < 1)
         max_clusters = sms / cs;
     if (max_clusters > sms / cs) max_clusters = sms / cs;  // the SM budget (the occupancy query sees every SM)
@@ -854,7 +912,7 @@ cudaError_t launch_kg(const tda_layer_desc& L, const void* A, const void* B, int
     cfg.gridDim = dim3((unsigned)(clusters * cs));
     if (grid_out) *grid_out = (int)(clusters * cs);
     note_launches(1);
-    e = cudaLaunchKernelEx(&cfg, project_tc_kernel<K, G, KF, FO>, tmA, tmB, p);
+    e = cudaLaunchKernelEx(&cfg, project_tc_kernel<K, G, KF, FO, SL>, tmA, tmB, tmSA, tmSB, p);
     if (e != cudaSuccess) return e;
     return cudaGetLastError();
 }
@@ -863,7 +921,8 @@ cudaError_t launch_kg(const tda_layer_desc& L, const void* A, const void* B, int
 // units run one tile per stage so that they spread over all SMs.
 template <int K, bool KF, bool FO>
 cudaError_t launch_k(const tda_layer_desc& L, const void* A, const void* B, int64_t N, float* phi,
-                     int64_t ld_phi, unsigned int* err, cudaStream_t s, float* cov, int* grid_out, float* fout) {
+                     int64_t ld_phi, unsigned int* err, cudaStream_t s, float* cov, int* grid_out, float* fout,
+                     const void* signs = nullptr) {
     // K = 128 keeps one example per tile (its epilogue contracts 64-row halves)
     int pack = (K <= 64 && L.T <= 64) ? (int)(kTileM / L.T) : 1;
     if (pack > 1) {
@@ -881,13 +940,17 @@ cudaError_t launch_k(const tda_layer_desc& L, const void* A, const void* B, int6
             for (int64_t e0 = 0; e0 < N; e0 += max_n) {
                 const int64_t n = N - e0 < max_n ? N - e0 : max_n;
                 cudaError_t e = launch_k<K, KF, FO>(L, (const char*)A + e0 * a_ex, (const char*)B + e0 * b_ex, n,
-                                                    phi + e0 * ld_phi, ld_phi, err, s, nullptr, nullptr, nullptr);
+                                                    phi + e0 * ld_phi, ld_phi, err, s, nullptr, nullptr, nullptr,
+                                                    signs);
                 if (e != cudaSuccess) return e;
             }
             return cudaSuccess;
         }
     }
     if constexpr (K > 64) {
+        if constexpr (!KF && !FO)
+            if (signs) return launch_kg<K, 1, false, false, true>(L, A, B, N, phi, ld_phi, err, s, pack, cov, grid_out,
+                                                                  fout, signs);
         return launch_kg<K, 1, KF, FO>(L, A, B, N, phi, ld_phi, err, s, pack, cov, grid_out, fout);
     } else {
         const int64_t units = pack > 1 ? (N + pack - 1) / pack : N * ((L.T + kTileM - 1) / kTileM);
@@ -922,14 +985,37 @@ bool project_tc_plain_supported(const tda_layer_desc& L, const void* A, const vo
     return project_tc_supported(L, A, B);
 }
 
+size_t project_tc_sign_table_bytes(const tda_layer_desc& L) {
+    if (L.k_in != 128 || L.k_out != 128) return 0;
+    return (size_t)L.k_in * (size_t)(L.d_in + L.d_out) * 2;
+}
+
 cudaError_t launch_project_tc(const tda_layer_desc& L, const void* A, const void* B, int64_t N, float* phi,
-                              int64_t ld_phi, unsigned int* err, cudaStream_t s) {
+                              int64_t ld_phi, unsigned int* err, cudaStream_t s, void* ws, size_t ws_bytes) {
     if (N == 0) return cudaSuccess;
     switch (L.k_in) {
         case 16: return launch_k<16, false, false>(L, A, B, N, phi, ld_phi, err, s, nullptr, nullptr, nullptr);
         case 32: return launch_k<32, false, false>(L, A, B, N, phi, ld_phi, err, s, nullptr, nullptr, nullptr);
         case 64: return launch_k<64, false, false>(L, A, B, N, phi, ld_phi, err, s, nullptr, nullptr, nullptr);
-        case 128: return launch_k<128, false, false>(L, A, B, N, phi, ld_phi, err, s, nullptr, nullptr, nullptr);
+        case 128: {
+            // with room in ws: both sides' sign tables once per call (L2-resident, read by TMA
+            // beside the factor tiles) instead of sign tiles written by the generator warps
+            const size_t need = project_tc_sign_table_bytes(L);
+            const void* signs = nullptr;
+            if (ws && ws_bytes >= need && ((uintptr_t)ws & 255) == 0) {
+                uint16_t* tab = (uint16_t*)ws;
+                const int64_t items = 128 * ((L.d_in + 63) / 64 + (L.d_out + 63) / 64);
+                const unsigned blocks = (unsigned)((items + 255) / 256 < 1216 ? (items + 255) / 256 : 1216);
+                note_launches(2);
+                sign_table_kernel<<<blocks, 256, 0, s>>>(tab, L.d_in, 128, side_key(L.seed, L.layer, 0));
+                sign_table_kernel<<<blocks, 256, 0, s>>>(tab + 128 * L.d_in, L.d_out, 128,
+                                                         side_key(L.seed, L.layer, 1));
+                cudaError_t e = cudaGetLastError();
+                if (e != cudaSuccess) return e;
+                signs = tab;
+            }
+            return launch_k<128, false, false>(L, A, B, N, phi, ld_phi, err, s, nullptr, nullptr, nullptr, signs);
+        }
         default: return cudaErrorNotSupported;
     }
 }

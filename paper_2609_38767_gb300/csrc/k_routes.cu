@@ -334,8 +334,10 @@ cudaError_t launch_similarity_materialized(const tda_layer_desc& L, tda_dtype dt
     // axis over many CTAs when the chunk leaves one train gradient's room for
     // the partial sums.
     // (3xTF32 tensor cores when the operands allow, decided once for every chunk:
-    // Gq and Gt share base alignment and row length)
-    const bool tc = score_dots_tc(Gq, n_q, gsz, Gt, chunk, gsz, gsz);
+    // Gq and Gt share base alignment and row length; fp32 factors keep fp32 CUDA-core
+    // dots: the tensor pipe accumulates a slice of thousands of features in truncating
+    // fp32, about 1e-5 of relative error, the size of the fp32 tolerance itself)
+    const bool tc = dt == TDA_BF16 && score_dots_tc(Gq, n_q, gsz, Gt, chunk, gsz, gsz);
     int splits = score_splitk_splits(n_q, chunk, gsz, tc);
     float* part = nullptr;
     if (splits > 1) {

@@ -11,6 +11,8 @@
 // Cost of the convenience: every GPU that loads libtda.so holds the array
 // (kNoAllocScratchBytes) from module load until process exit, and all calls
 // share it.
+#include <cuda.h>
+
 #include <mutex>
 
 #include "tda_internal.cuh"
@@ -21,28 +23,55 @@ namespace {
 constexpr size_t kNoAllocScratchBytes = (size_t)64 << 20;  // 64 MiB
 
 // The shared scratch. In host code this name is only a host-side stand-in for
-// the symbol, never a device address: the address is resolved per device with
-// cudaGetSymbolAddress below.
+// the symbol, never a device address: the address is resolved per CUDA
+// context with cudaGetSymbolAddress below.
 static __device__ __align__(256) unsigned char g_noalloc_scratch[kNoAllocScratchBytes];
 
-std::mutex g_noalloc_mu;
-void* g_noalloc_ptr[64] = {};
+typedef CUresult (*CtxGetCurrentFn)(CUcontext*);
 
-// First call on a device (with that device current) resolves the array's
-// device address; later calls reuse it.
+CtxGetCurrentFn ctx_get_current() {
+    static CtxGetCurrentFn fn = nullptr;
+    static std::once_flag once;
+    std::call_once(once, [] {
+        void* f = nullptr;
+        cudaDriverEntryPointQueryResult q;
+        if (cudaGetDriverEntryPointByVersion("cuCtxGetCurrent", &f, 12000, cudaEnableDefault, &q) == cudaSuccess &&
+            q == cudaDriverEntryPointSuccess)
+            fn = (CtxGetCurrentFn)f;
+    });
+    return fn;
+}
+
+// Resolved addresses, one per CUDA context (the array lives in each context
+// that loads this module: normally the runtime's primary context of a device).
+struct Slot {
+    CUcontext ctx;
+    void* ptr;
+};
+std::mutex g_noalloc_mu;
+Slot g_noalloc_slots[64] = {};
+int g_noalloc_nslots = 0;
+
+// The first call in a context resolves the array's device address (with lazy
+// module loading that call also loads the module, which commits the 64 MiB);
+// later calls in the same context reuse it.
 cudaError_t noalloc_scratch(void** out) {
-    int dev = 0;
-    cudaError_t e = cudaGetDevice(&dev);
-    if (e != cudaSuccess) return e;
-    if (dev < 0 || dev >= 64) return cudaErrorInvalidDevice;
+    CtxGetCurrentFn get = ctx_get_current();
+    if (!get) return cudaErrorNotSupported;
     std::lock_guard<std::mutex> lock(g_noalloc_mu);
-    if (!g_noalloc_ptr[dev]) {
-        void* p = nullptr;
-        e = cudaGetSymbolAddress(&p, g_noalloc_scratch);
-        if (e != cudaSuccess) return e;
-        g_noalloc_ptr[dev] = p;
-    }
-    *out = g_noalloc_ptr[dev];
+    CUcontext ctx = nullptr;
+    if (get(&ctx) != CUDA_SUCCESS) return cudaErrorUnknown;
+    for (int i = 0; ctx && i < g_noalloc_nslots; ++i)
+        if (g_noalloc_slots[i].ctx == ctx) {
+            *out = g_noalloc_slots[i].ptr;
+            return cudaSuccess;
+        }
+    void* p = nullptr;
+    cudaError_t e = cudaGetSymbolAddress(&p, g_noalloc_scratch);  // binds the primary context if none is current
+    if (e != cudaSuccess) return e;
+    if (!ctx && get(&ctx) != CUDA_SUCCESS) return cudaErrorUnknown;
+    if (g_noalloc_nslots < 64) g_noalloc_slots[g_noalloc_nslots++] = Slot{ctx, p};
+    *out = p;
     return cudaSuccess;
 }
 

@@ -114,8 +114,12 @@ cudaError_t launch_mask_gather(const tda_layer_desc& L, tda_dtype dt, const void
 bool materialize_tc_supported(const tda_layer_desc& L, tda_dtype dt, const void* A, const void* B, const float* G);
 cudaError_t launch_materialize_tc(const tda_layer_desc& L, const void* A, const void* B, int64_t e0, int64_t n,
                                   float* G, unsigned int* err, cudaStream_t s);
+// ws (optional, 256-byte aligned): for k = 128, >= project_tc_sign_table_bytes(L)
+// bytes let the kernel read precomputed sign tiles by TMA instead of generating them.
+size_t project_tc_sign_table_bytes(const tda_layer_desc& L);
 cudaError_t launch_project_tc(const tda_layer_desc& L, const void* A, const void* B, int64_t N,
-                              float* phi, int64_t ld_phi, unsigned int* err, cudaStream_t s);
+                              float* phi, int64_t ld_phi, unsigned int* err, cudaStream_t s,
+                              void* ws = nullptr, size_t ws_bytes = 0);
 
 // Route (b): materialise G = B^T A for nb examples into ws, then project it.
 size_t materialize_ws_bytes_per_example(const tda_layer_desc& L);
@@ -184,6 +188,18 @@ bool score_tc_supported(tda_dtype qdt, const void* Qhat, int64_t n_q, int64_t ld
 cudaError_t launch_score_tc(const float* Qhat, int64_t n_q, int64_t ld_q, const float* Phi, int64_t n_t, int64_t ld_phi,
                             int64_t D, float* S, int64_t ld_S, float beta, unsigned int* err, cudaStream_t s);
 int score_tc_tiles(int64_t n_q, int64_t n_t);
+bool gemm_tc_available();  // tcgen05 and the tensor-map encoder are usable on this device
+// C[n][m] = beta C[n][m] + alpha sum_k A[m][k] B[n][k] on tcgen05 (3xTF32); lower: square
+// symmetric update, tiles on or below the diagonal only. Same operand rules as the score.
+cudaError_t launch_gemm_nt_tc(const float* A, int64_t n_a, int64_t lda, const float* B, int64_t n_b, int64_t ldb,
+                              int64_t K, float* C, int64_t ldc, float alpha, float beta, bool lower,
+                              unsigned int* err, cudaStream_t s);
+// The same for nz independent problems in one launch (grid z): problem z's A, B start
+// a_z_bytes, b_z_bytes (multiples of 16) after the previous one's, its C c_z floats after.
+cudaError_t launch_gemm_nt_tc_batched(const float* A, int64_t n_a, int64_t lda, size_t a_z_bytes, const float* B,
+                                      int64_t n_b, int64_t ldb, size_t b_z_bytes, int64_t K, float* C, int64_t ldc,
+                                      int64_t c_z, int64_t nz, float alpha, float beta, bool lower,
+                                      unsigned int* err, cudaStream_t s);
 cudaError_t launch_score_tc_slices(const float* Qhat, int64_t n_q, int64_t ld_q, const float* Phi, int64_t n_t,
                                    int64_t ld_phi, int64_t D, int splits, float* part, unsigned int* err,
                                    cudaStream_t s);

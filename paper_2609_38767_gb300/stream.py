@@ -1,0 +1,156 @@
+"""A streamed attribution job over a stack of layers, through the C ABI.
+
+The training set of a job is too large to hold its factors, so it streams in
+chunks (App. A.2: the factors are projected as they arrive and never buffered
+whole); the projected features stay resident. A job over N_train examples and
+a stack of linears is, per linear (Sec. 3.2, App. B.2, B.3):
+
+  project every training chunk (Eq. 2) into the resident features, fit the
+  linear's Fisher F = Phi^T Phi / N over all of them, project the queries,
+  factor F + lambda I and precondition the queries (lambda = lambda_rel x mean
+  eigenvalue), add the linear's share of the query x train score matrix
+  (Eq. 4's left side), and finally take the top-k train indices per query.
+
+Jobs run back to back, software-pipelined in steps of one chunk: step s of job
+j projects chunk s of job j; it also runs the s-th share of job j-1's query
+side (the linears in [s L / C, (s+1) L / C) of L linears: their Fisher fit over
+job j-1's features, query projections, factorisation and preconditioning, and
+their share of job j-1's score), and the top-k of the s-th share of job j-2's
+query rows (C chunks per job). Each step thus does 1/C of every phase of a job,
+and C consecutive steps do a whole job's work. Buffers that two jobs in flight
+need at once (features, score matrix) are double-buffered by job parity; the
+Fisher states hold one share of linears.
+
+Every step is a libtda.so call; this class only owns the device buffers and the
+order of the calls. The caller provides the factors of a (role, linear, chunk)
+as pieces (device tensors, or pinned host tensors for tda_project_host).
+"""
+from __future__ import annotations
+
+import torch
+
+import paper_2609_38767_gb300 as tda
+
+
+class StackJob:
+    def __init__(self, linears, T, k, n_train, chunk, n_query, *, topk=100, lambda_rel=1e-2, lambda_abs=0.0,
+                 seed=0, device="cuda", host_ws_bytes=0, train_streams=1, proj_ws=True):
+        """linears: [(d_in, d_out)] of the whole stack, in layer order (linear i uses projection
+        layer id i). n_train must be a multiple of chunk. train_streams > 1 spreads the train
+        projections of a chunk round-robin over that many streams, so that a launch's CTAs fill
+        the SMs its predecessor's last tiles leave idle (every launch writes its own feature
+        columns: the results do not depend on the order). proj_ws: give the factored projection
+        its optional workspace (k = 128: precomputed sign tables)."""
+        assert n_train % chunk == 0 and n_train >= topk >= 1
+        self.layers = [tda.LayerDesc(di, do, T, k, k, seed=seed, layer=i) for i, (di, do) in enumerate(linears)]
+        self.nl = len(self.layers)
+        self.T, self.k, self.D = T, k, k * k
+        self.DT = self.D * self.nl
+        self.N, self.chunk, self.Nq, self.topk = n_train, chunk, n_query, topk
+        self.C = n_train // chunk
+        self.lambda_abs, self.lambda_rel = lambda_abs, lambda_rel
+        dev = torch.device(device)
+        self.per = tda.tda_precondition_state_bytes(self.D, tda.TDA_F32)
+        self.Phi = [torch.empty((n_train, self.DT), dtype=torch.float32, device=dev) for _ in range(2)]
+        self.share_max = max(b - a for a, b in (self.share(s, self.nl) for s in range(self.C)))
+        self.state = torch.empty(max(self.share_max, 1) * self.per, dtype=torch.uint8, device=dev)
+        self.S = [torch.empty((n_query, n_train), dtype=torch.float32, device=dev) for _ in range(2)]
+        self.Q = torch.empty((n_query, self.DT), dtype=torch.float32, device=dev)
+        self.Qh = torch.empty((n_query, self.DT), dtype=torch.float32, device=dev)
+        self.idx = torch.empty((n_query, topk), dtype=torch.int32, device=dev)
+        self.val = torch.empty((n_query, topk), dtype=torch.float32, device=dev)
+        self.host_ws_bytes = host_ws_bytes
+        self.host_ws = torch.empty(host_ws_bytes, dtype=torch.uint8, device=dev) if host_ws_bytes else None
+        self.train_streams = max(1, train_streams)
+        self._streams = []
+        # one workspace per stream (a call writes its sign tables into it)
+        self.proj_wsb = max(tda.tda_workspace_size(tda.TDA_OP_PROJECT, L, tda.TDA_BF16, chunk, 0,
+                                                   tda.TDA_ROUTE_FACTORED) for L in self.layers) if proj_ws else 0
+        self.proj_ws = [torch.empty(self.proj_wsb, dtype=torch.uint8, device=dev)
+                        for _ in range(self.train_streams)] if self.proj_wsb else None
+
+    # ------------------------------------------------------------------ shares of a job
+    def share(self, s, total):
+        """[lo, hi) of `total` items handled at step s (the s-th of C near-equal shares)."""
+        return total * s // self.C, total * (s + 1) // self.C
+
+    def _project(self, L, pieces, phi, hook=None, li=0, role="train", slot=0):
+        """pieces: [(A, B, row, n)] -- n examples written to feature row `row` of phi."""
+        ws = self.proj_ws[slot] if self.proj_ws else None
+        for A, B, row, n in pieces:
+            if hook:
+                hook(role, li, "begin", n)
+            if A.is_cuda:
+                tda.tda_project(L, tda.TDA_BF16, A, B, n, phi[row:], self.DT, tda.TDA_ROUTE_FACTORED, ws,
+                                self.proj_wsb if ws is not None else 0)
+            else:
+                tda.tda_project_host(L, tda.TDA_BF16, A, B, n, phi[row:], self.DT, self.host_ws, self.host_ws_bytes)
+            if hook:
+                hook(role, li, "end", n)
+
+    def train_part(self, j, s, factors, mark=None, hook=None):
+        """Chunk s of job j: project it through every linear into the resident features."""
+        if mark:
+            mark("project_train")
+        Phi = self.Phi[j % 2][s * self.chunk:(s + 1) * self.chunk]
+        n = min(self.train_streams, self.nl)
+        if n <= 1:
+            for li, L in enumerate(self.layers):
+                self._project(L, factors("train", li, j, s), Phi[:, li * self.D:], hook, li, "train")
+            return
+        main = torch.cuda.current_stream()
+        if len(self._streams) < n:
+            self._streams = [torch.cuda.Stream(device=main.device) for _ in range(n)]
+        for st in self._streams[:n]:
+            st.wait_stream(main)
+        for li, L in enumerate(self.layers):
+            with torch.cuda.stream(self._streams[li % n]):
+                self._project(L, factors("train", li, j, s), Phi[:, li * self.D:], hook, li, "train", li % n)
+        for st in self._streams[:n]:
+            main.wait_stream(st)
+
+    def query_part(self, j, s, factors, mark=None, hook=None):
+        """Share s of job j's query side: the Fisher fit of linears [l0, l1) over all of job
+        j's features, their query projections, factorisation and preconditioning, and their
+        share of the score matrix."""
+        b = j % 2
+        mark = mark or (lambda name: None)
+        l0, l1 = self.share(s, self.nl)
+        if l1 == l0:
+            return
+        D, DT = self.D, self.DT
+        st = self.state[:(l1 - l0) * self.per]
+        mark("fisher_fit")
+        tda.tda_precondition(tda.TDA_PC_RESET, l1 - l0, D, tda.TDA_F32, st)
+        tda.tda_precondition(tda.TDA_PC_FIT_ACCUM, l1 - l0, D, tda.TDA_F32, st, phi=self.Phi[b][:, l0 * D:],
+                             n=self.N, ld_phi=DT)
+        mark("project_query")
+        for li in range(l0, l1):
+            self._project(self.layers[li], factors("query", li, j, s), self.Q[:, li * D:], hook, li, "query")
+        mark("factor_apply")
+        tda.tda_precondition(tda.TDA_PC_FACTOR_APPLY, l1 - l0, D, tda.TDA_F32, st, n_total=self.N,
+                             lambda_abs=self.lambda_abs, lambda_rel_mean_eig=self.lambda_rel, q=self.Q[:, l0 * D:],
+                             n_q=self.Nq, ld_q=DT, qhat=self.Qh[:, l0 * D:], ld_qhat=DT)
+        mark("score")
+        tda.tda_score(self.Qh[:, l0 * D:], tda.TDA_F32, self.Nq, DT, self.Phi[b][:, l0 * D:], self.N, DT,
+                      (l1 - l0) * D, self.S[b], self.N, 0.0 if l0 == 0 else 1.0)
+
+    def topk_part(self, j, s, mark=None):
+        """Share s of job j's query rows: their top-k train indices (job j's S is complete)."""
+        r0, r1 = self.share(s, self.Nq)
+        if r1 == r0:
+            return
+        if mark:
+            mark("topk")
+        tda.tda_topk(self.S[j % 2][r0:], r1 - r0, self.N, self.N, self.topk, self.idx[r0:], self.val[r0:])
+
+    def step(self, j, s, factors, first_job=0, mark=None, hook=None):
+        """Step s of job j: chunk s of job j, share s of job j-1's query side and of job
+        j-2's top-k. Jobs before first_job do not exist (their shares are skipped)."""
+        self.train_part(j, s, factors, mark, hook)
+        if j - 1 >= first_job:
+            self.query_part(j - 1, s, factors, mark, hook)
+        if j - 2 >= first_job:
+            self.topk_part(j - 2, s, mark)
+        if mark:
+            mark(None)

@@ -1,18 +1,24 @@
 """Parity at the workloads' full sizes, on sampled outputs the oracle computes
-one by one, and through properties that hold at any size.
+one by one, and stage by stage from the GPU's own features.
 
 * Llama-1B block (the benchmark's workload and launch configuration): 4096 train
   and 64 query examples resident, the whole pass of BlockPipeline; sampled
-  feature rows and GradDot scores against the oracle, top-k selection bit-exact,
-  the preconditioner's solve checked by its residual.
+  feature rows and GradDot scores against the oracle; then, from the GPU's
+  downloaded features, the oracle's fp64 damping, preconditioned queries and
+  preconditioned score matrix, compared with the GPU's S; top-k selection
+  bit-exact on the GPU's S and consistent with the oracle's S wherever the
+  score gaps exceed the measured score error.
 * Llama-3-8B layer shapes (k = 64, T = 1024): one streamed chunk of 256 train
-  examples through the 7 linears of a layer.
-* Large-model layer shapes (k = 128, T = 2048, Student-t activations), factors
-  streamed from pinned host memory through tda_project_host.
+  examples through the 7 linears of a layer, with 16 and with all 256 queries.
+* Large-model block (d_model 12288, ffn 49152, GQA k/v 12288 -> 1536; k = 128,
+  T = 2048, Student-t activations): 7 x 16384 features per example, the
+  D = 16384 Fisher fit, factorisation and query solves, the preconditioned
+  score and the top-100; the factors are also streamed from pinned host memory.
 * The 8192 x 8192 linear of the route sweep: exact similarity by both routes.
 Tolerances: relative Frobenius error 2e-2 for bf16 factors (spec bound).
 """
 import math
+import os
 
 import numpy as np
 import pytest
@@ -73,6 +79,62 @@ def run_block(dev, linears, T, k, N, Nq, sig_b, dist_a, mask_p, topk):
     return pipe, S_plain, info
 
 
+def topk_against_reference_scores(idx, S_gpu, S_ref, k):
+    """Top-k test against the oracle's fp64 scores: at every rank whose oracle score is
+    more than twice the row's measured score error away from both neighbours, the GPU's
+    index must be the oracle's; returns the number of ranks where the two differ (swaps
+    among scores closer than the error)."""
+    oi, ov = _orc_topk(S_ref, k + 1)
+    swaps = 0
+    for q in range(S_ref.shape[0]):
+        err = float(np.abs(S_gpu[q].astype(np.float64) - S_ref[q]).max())
+        for r in range(k):
+            gap = ov[q, r] - ov[q, r + 1]
+            if r > 0:
+                gap = min(gap, ov[q, r - 1] - ov[q, r])
+            if gap > 2 * err:
+                assert idx[q, r] == oi[q, r], (q, r, err, gap)
+            elif idx[q, r] != oi[q, r]:
+                swaps += 1
+    return swaps
+
+
+_ORC = None
+
+
+def _orc_topk(S, k):
+    return _ORC.topk(S, k)
+
+
+def stagewise(orc, pipe, info, lam_rel=1e-2):
+    """F, lambda, Qhat and S recomputed in fp64 by the oracle from the GPU's features, per
+    linear (D x D Cholesky when N >= D, its Woodbury form otherwise); S compared with the
+    GPU's preconditioned score matrix, the top-k with the oracle's scores."""
+    global _ORC
+    _ORC = orc
+    orc.set_threads(os.cpu_count() or 1)
+    D, N = pipe.D, pipe.N
+    Phi64 = pipe.Phi.cpu().numpy().astype(np.float64)
+    Q64 = pipe.Q.cpu().numpy().astype(np.float64)
+    Qh = pipe.Qh.cpu().numpy().astype(np.float64)
+    Qh_ref = np.empty_like(Q64)
+    for li in range(pipe.nl):
+        sl = slice(li * D, (li + 1) * D)
+        P = np.ascontiguousarray(Phi64[:, sl])
+        lam = orc.damping_features(P, 0.0, lam_rel)
+        assert abs(info[4 * li] - lam) <= 1e-4 * lam, li
+        Ql = np.ascontiguousarray(Q64[:, sl])
+        Qh_ref[:, sl] = orc.precondition(orc.fisher(P), lam, Ql) if N >= D else orc.precondition_lowrank(P, lam, Ql)
+        assert rel_fro(Qh[:, sl], Qh_ref[:, sl]) <= TOL, ("qhat", li)
+    S_ref = orc.score(Qh_ref, Phi64)
+    S = pipe.S.cpu().numpy()
+    err = rel_fro(S, S_ref)
+    assert err <= TOL, err
+    swaps = topk_against_reference_scores(pipe.idx.cpu().numpy(), S, S_ref, pipe.topk)
+    print(f"preconditioned S: rel. Frobenius error {err:.2e}; top-{pipe.topk} swaps among near-ties: {swaps}")
+    return err, swaps
+
+
 def check_block(orc, pipe, S_plain, info, linears, T, k, sig_b, dist_a, mask_p, train_s, query_s, rng):
     D, N, Nq = k * k, pipe.N, pipe.Nq
     phi = {e: pipe.Phi[e].cpu().numpy() for e in train_s}
@@ -109,6 +171,8 @@ def check_block(orc, pipe, S_plain, info, linears, T, k, sig_b, dist_a, mask_p, 
         X = Qh[:, li * D:(li + 1) * D]
         R = (X @ P.T) @ P / N + lam * X - Q[:, li * D:(li + 1) * D]
         assert np.linalg.norm(R) <= 1e-3 * np.linalg.norm(Q[:, li * D:(li + 1) * D]), li
+    # stage by stage against the oracle: F, lambda, Qhat and the preconditioned S
+    stagewise(orc, pipe, info)
     return got, ref
 
 
@@ -125,10 +189,62 @@ def test_llama1b_block_full_size(dev, orc):
     check_block(orc, pipe, S_plain, info, LLAMA1B, 512, 32, sb, 0, 0.01, train_s, [0, 63], rng)
 
 
-def test_llama8b_layer_chunk_full_shapes(dev, orc):
-    # one streamed chunk of 256 train examples, 16 queries, T = 1024, k = 64
-    pipe, S_plain, info = run_block(dev, LLAMA8B, 1024, 64, 256, 16, 0.1, 0, 0.0, 100)
+@pytest.mark.parametrize("Nq", [16, 256])
+def test_llama8b_layer_chunk_full_shapes(dev, orc, Nq):
+    # one streamed chunk of 256 train examples, T = 1024, k = 64; 16 queries, or all 256 of the
+    # workload (the blocked D = 4096 solve with a full query tile count)
+    pipe, S_plain, info = run_block(dev, LLAMA8B, 1024, 64, 256, Nq, 0.1, 0, 0.0, 100)
     check_block(orc, pipe, S_plain, info, LLAMA8B, 1024, 64, 0.1, 0, 0.0, [0, 255], [7], np.random.default_rng(1))
+
+
+LARGE = [(12288, 12288), (12288, 1536), (12288, 1536), (12288, 12288), (12288, 49152), (12288, 49152),
+         (49152, 12288)]
+
+
+def test_large_model_block_preconditioned_top100(dev, orc):
+    # the large-model block at full width: T = 2048, k = 128 (D = 16384 per linear), A ~ Student-t(4),
+    # B ~ N(0, 1e-4); 2048 train and 32 query examples (the full 16384 x 512 workload's factors do not
+    # fit the device), factors generated on the device one 256-example chunk at a time;
+    # lambda = 1e-2 x mean eigenvalue; preconditioned 32 x 2048 score and top-100 per query.
+    # With fewer train examples than features F has rank N: the fp32 rounding of Qhat's large
+    # component along F's null space (about q / lambda) reaches S with a weight that grows like
+    # (D/N)^1.5 / lambda_rel; at N = 256 it alone is ~5% of S, at N = 2048 ~0.2%.
+    T, k, N, Nq, sb, CH = 2048, 128, 2048, 32, 0.01, 256
+    dist = synth.DIST_STUDENT_T4
+    pipe = BlockPipeline(LARGE, T, k, N, Nq, topk=100, precondition=True, lambda_rel=1e-2, device=dev)
+
+    def proj(role):
+        n_all, off, ms = (N, 0, 0) if role == "train" else (Nq, synth.QUERY_STREAM_OFFSET, 1000)
+
+        def f(li, L, route, phi, ld):
+            di, do = LARGE[li]
+            for c0 in range(0, n_all, CH):
+                n = min(CH, n_all - c0)
+                A = torch.empty(n * T * di, dtype=torch.bfloat16, device=dev)
+                B = torch.empty(n * T * do, dtype=torch.bfloat16, device=dev)
+                synth.fill_device(A, synth.SEED_A, li + off, n, T, di, 1.0, dist, e0=c0, mask_stream=ms)
+                synth.fill_device(B, synth.SEED_B, li + off, n, T, do, sb, 0, e0=c0, mask_stream=ms)
+                assert tda.tda_project_engine(L, tda.TDA_BF16, A, B) == 1
+                tda.tda_project(L, tda.TDA_BF16, A, B, n, phi[c0:], ld, route)
+                torch.cuda.synchronize()
+                del A, B
+        return f
+
+    pipe.run(proj("train"), proj("query"))
+    info = tda.tda_precondition_info(pipe.nl, pipe.D, tda.TDA_F32, pipe.state)
+    tda.tda_device_status()
+    # sampled features against the oracle (the narrow k/v linear, train examples in two chunks, a query)
+    D = k * k
+    for role, e in (("train", 3), ("train", 1500), ("query", 5)):
+        ref = oracle_example(orc, e, role, 1, T, 12288, 1536, k, sb, dist, 0.0, 1)
+        got = (pipe.Phi if role == "train" else pipe.Q)[e, D:2 * D].cpu().numpy()
+        assert rel_fro(got, ref) <= TOL, (role, e)
+    # top-100 selection bit-exact on the GPU's own scores
+    S = pipe.S.cpu().numpy()
+    oi, ov = orc.topk(S.astype(np.float64), 100)
+    np.testing.assert_array_equal(pipe.idx.cpu().numpy(), oi)
+    np.testing.assert_array_equal(pipe.val.cpu().numpy(), ov.astype(np.float32))
+    stagewise(orc, pipe, info)
 
 
 @pytest.mark.parametrize("li,di,do", [(1, 12288, 1536), (4, 12288, 49152)])

@@ -3,6 +3,8 @@ the fp64 oracle on the same seeded inputs. Tolerances: projected features and
 score matrices within a relative Frobenius error of 1e-5 for fp32 factors and
 2e-2 for bf16 factors (fp32 accumulation); sign entries, indices and top-k
 bit-exact."""
+import os
+
 import numpy as np
 import pytest
 import torch
@@ -47,7 +49,7 @@ def to_dev(x, dtype, device):
 TD = {"f32": tda.TDA_F32, "bf16": tda.TDA_BF16}
 
 
-def gpu_project(L, dtype, A, B, N, route, device, ld=None):
+def gpu_project(L, dtype, A, B, N, route, device, ld=None, sign_ws=False):
     D = L.k_in * L.k_out
     ld = ld or D
     phi = torch.full((N, ld), float("nan"), dtype=torch.float32, device=device)
@@ -55,6 +57,10 @@ def gpu_project(L, dtype, A, B, N, route, device, ld=None):
     if route == tda.TDA_ROUTE_MATERIALIZE:
         wsb = tda.tda_workspace_size(tda.TDA_OP_PROJECT, L, TD[dtype], N, 0, route) * min(N, 3)
         ws = torch.empty(wsb, dtype=torch.uint8, device=device)
+    elif sign_ws:  # the optional workspace of the factored route (k = 128: precomputed sign tables)
+        wsb = tda.tda_workspace_size(tda.TDA_OP_PROJECT, L, TD[dtype], N, 0, route)
+        assert wsb == 2 * L.k_in * (L.d_in + L.d_out)
+        ws = torch.full((wsb,), 0x7F, dtype=torch.uint8, device=device)
     tda.tda_project(L, TD[dtype], A, B, N, phi, ld, route, ws, wsb)
     tda.tda_device_status()
     return phi[:, :D].cpu().numpy().reshape(N, L.k_out, L.k_in), phi
@@ -246,6 +252,65 @@ def test_topk_selection_bit_exact_on_gpu_scores(dev, orc):
     np.testing.assert_array_equal(val.cpu().numpy(), ov.astype(np.float32))
 
 
+def test_topk_nan_first_and_signed_zeros(dev, orc):
+    # NaN ranks above every number (NaNs by index), -0 ties with +0 (by index): the GPU and the
+    # oracle's total order agree on every index, values compared bit for bit apart from NaN payloads
+    rng = np.random.default_rng(11)
+    nq, nt, k = 4, 3000, 60
+    S = (np.round(rng.standard_normal((nq, nt)) * 8) / 8).astype(np.float32)
+    S[0, [5, 900, 2999]] = np.nan
+    S[1, :] = 0.0
+    S[1, ::3] = -0.0
+    S[2, [10, 20]] = np.inf
+    S[2, [30, 40]] = np.nan
+    S[3, :] = -np.inf
+    S[3, 100:140] = np.nan
+    idx = torch.empty((nq, k), dtype=torch.int32, device=dev)
+    val = torch.empty((nq, k), device=dev)
+    tda.tda_topk(torch.from_numpy(S).to(dev), nq, nt, nt, k, idx, val)
+    tda.tda_device_status()
+    oi, ov = orc.topk(S.astype(np.float64), k)
+    np.testing.assert_array_equal(idx.cpu().numpy(), oi)
+    np.testing.assert_array_equal(val.cpu().numpy(), ov.astype(np.float32))
+    assert list(oi[0, :3]) == [5, 900, 2999] and list(oi[2, :4]) == [30, 40, 10, 20]
+    g = val.cpu().numpy()
+    assert (np.signbit(g[1]) == np.signbit(S[1, oi[1]])).all()  # each selected zero keeps its sign
+
+
+@pytest.mark.parametrize("dtype", ["f32", "bf16"])
+def test_config1_layer_three_routes_agree(dev, orc, dtype):
+    # the 256 x 256 layer, T = 32, k = 16, 8 queries x 64 train: projected similarity by the
+    # factored, materialised and Gram routes against the oracle, and the exact (unprojected)
+    # similarity by the materialised and Gram routes
+    nq, nt, T, d, k = 8, 64, 32, 256, 16
+    Aq, Bq = make_factors(nq, T, d, d, dtype, stream=0, query=True)
+    At, Bt = make_factors(nt, T, d, d, dtype, stream=0)
+    L = tda.LayerDesc(d, d, T, k, k, seed=0, layer=0)
+    args = [to_dev(x, dtype, dev) for x in (Aq, Bq, At, Bt)]
+    fq = orc.project(synth.to_f64(Aq, dtype), synth.to_f64(Bq, dtype), k, k, 0, 0)
+    ft = orc.project(synth.to_f64(At, dtype), synth.to_f64(Bt, dtype), k, k, 0, 0)
+    ref_p = orc.score(fq, ft)
+    ref_x = orc.similarity(*(synth.to_f64(x, dtype) for x in (Aq, Bq, At, Bt)))
+    got = {}
+    for route in (tda.TDA_ROUTE_FACTORED, tda.TDA_ROUTE_MATERIALIZE, tda.TDA_ROUTE_GRAM):
+        wsb = max(tda.tda_workspace_size(tda.TDA_OP_SIMILARITY_PROJECTED, L, TD[dtype], nq, nt, route), 256)
+        ws = torch.empty(wsb, dtype=torch.uint8, device=dev)
+        S = torch.empty((nq, nt), device=dev)
+        tda.tda_similarity_projected(L, TD[dtype], args[0], args[1], nq, args[2], args[3], nt, S, nt, 0.0, route,
+                                     ws, wsb)
+        tda.tda_device_status()
+        got[route] = S.cpu().numpy()
+        assert rel_fro(got[route], ref_p) <= TOL[dtype], route
+    for route in (tda.TDA_ROUTE_MATERIALIZE, tda.TDA_ROUTE_GRAM):
+        wsb = max(tda.tda_workspace_size(tda.TDA_OP_SIMILARITY_EXACT, L, TD[dtype], nq, nt, route), 256)
+        ws = torch.empty(wsb, dtype=torch.uint8, device=dev)
+        S = torch.empty((nq, nt), device=dev)
+        tda.tda_similarity_exact(L, TD[dtype], args[0], args[1], nq, args[2], args[3], nt, S, nt, 0.0, route, ws,
+                                 wsb)
+        tda.tda_device_status()
+        assert rel_fro(S.cpu().numpy(), ref_x) <= TOL[dtype], route
+
+
 @pytest.mark.parametrize("k", [1, 7, 1024])
 def test_topk_sizes(dev, orc, k):
     rng = np.random.default_rng(k)
@@ -270,8 +335,8 @@ def test_route_auto_and_calibration(dev, orc):
 
 
 # ------------------------------------------------------------------ tensor-core projection specifics
-@pytest.mark.parametrize("k", [32, 128])
-def test_tc_projection_signs_bit_exact(dev, orc, k):
+@pytest.mark.parametrize("k,sign_ws", [(32, False), (128, False), (128, True)])
+def test_tc_projection_signs_bit_exact(dev, orc, k, sign_ws):
     # One-hot factors: A_n = I (T = d_in tokens), B_n = e_r at token t only, so
     # Phi_n / scale = outer(S_out[r, :], S_in[t, :]) exactly -- the signs the
     # tensor-core kernel generated on chip, compared bit for bit with the oracle's.
@@ -286,7 +351,7 @@ def test_tc_projection_signs_bit_exact(dev, orc, k):
     Bb = torch.from_numpy(B).to(dev).to(torch.bfloat16)
     L = tda.LayerDesc(d, d, d, k, k, seed=2024, layer=9)
     assert tda.tda_project_engine(L, tda.TDA_BF16, Ab, Bb) == 1
-    got, _ = gpu_project(L, "bf16", Ab, Bb, N, tda.TDA_ROUTE_FACTORED, dev)
+    got, _ = gpu_project(L, "bf16", Ab, Bb, N, tda.TDA_ROUTE_FACTORED, dev, sign_ws=sign_ws)
     S_in = orc.proj_entries(2024, 9, 0, d, k).astype(np.float32)
     S_out = orc.proj_entries(2024, 9, 1, d, k).astype(np.float32)
     for n, (t, r) in enumerate(picks):
@@ -320,6 +385,21 @@ TC_CASES = [
     (40, 48, 64, 64, 128, "bf16"),      # short sequences stay one example per tile
     (3, 1, 72, 64, 128, "bf16"),        # T = 1
 ]
+
+
+@pytest.mark.parametrize("case", [c for c in TC_CASES if c[4] == 128] + [(9, 130, 1000, 2056, 128, "bf16")])
+def test_tc_projection_k128_sign_tables_match_oracle(dev, orc, case):
+    # k = 128 with the optional workspace: both sides' sign tables written once per call and
+    # read by TMA beside the factor tiles (d not a multiple of 64: zero-filled last chunk)
+    N, T, di, do, k, dtype = case
+    A, B = make_factors(N, T, di, do, dtype, stream=12, sigma_b=0.03, mask_p=0.01)
+    L = tda.LayerDesc(di, do, T, k, k, seed=6, layer=4)
+    Ad, Bd = to_dev(A, dtype, dev), to_dev(B, dtype, dev)
+    got, _ = gpu_project(L, dtype, Ad, Bd, N, tda.TDA_ROUTE_FACTORED, dev, sign_ws=True)
+    plain, _ = gpu_project(L, dtype, Ad, Bd, N, tda.TDA_ROUTE_FACTORED, dev)
+    np.testing.assert_array_equal(got, plain)  # same signs, same arithmetic order
+    ref = orc.project(synth.to_f64(A, dtype), synth.to_f64(B, dtype), k, k, 6, 4)
+    assert max(rel_fro(got[n], ref[n]) for n in range(N)) <= TOL[dtype]
 
 
 @pytest.mark.parametrize("case", TC_CASES)
@@ -432,6 +512,67 @@ def test_precondition_factor_apply_matches_oracle(dev, orc, D, Nq, nl):
     tda.tda_precondition(tda.TDA_PC_APPLY, nl, D, sdt, state, q=qd, n_q=Nq, ld_q=nl * D + 3, qhat=qh2, ld_qhat=nl * D)
     tda.tda_device_status()
     assert rel_fro(qh2.cpu().numpy(), got[:, :nl * D]) <= 1e-5
+
+
+@pytest.mark.parametrize("D,nl,N,Nq,op", [(2048, 2, 700, 37, "split"), (2048, 1, 3000, 300, "fused"),
+                                          (4096, 2, 400, 5, "fused"), (2048, 3, 150, 130, "inplace")])
+def test_precondition_blocked_matches_oracle(dev, orc, D, nl, N, Nq, op):
+    # fp32 state, D a multiple of 128 and >= 2048: 128-column panels, tensor-core trailing updates
+    # and substitutions. Ragged query counts (not multiples of the 128-row tiles), N above and
+    # below D (the oracle solves through the D x D Cholesky or its Woodbury form), the two ops
+    # split (FACTOR, then APPLY with padded row strides), fused, or solved in place (qhat = q).
+    orc.set_threads(os.cpu_count() or 1)
+    rng = np.random.default_rng(D + N + Nq)
+    phi = (rng.standard_normal((N, nl * D)) * rng.uniform(0.5, 2.0, nl * D)).astype(np.float32)
+    ldq = nl * D + (4 if op == "split" else 0)
+    q = rng.standard_normal((Nq, ldq)).astype(np.float32)
+    sdt = tda.TDA_F32
+    per = tda.tda_precondition_state_bytes(D, sdt)
+    state = torch.empty(nl * per, dtype=torch.uint8, device=dev)
+    phid, qd = torch.from_numpy(phi).to(dev), torch.from_numpy(q).to(dev)
+    tda.tda_precondition(tda.TDA_PC_RESET, nl, D, sdt, state)
+    tda.tda_precondition(tda.TDA_PC_FIT_ACCUM, nl, D, sdt, state, phi=phid, n=N, ld_phi=nl * D)
+    if op == "inplace":
+        qh, ldh = qd, ldq
+    else:
+        ldh = nl * D + (8 if op == "split" else 0)
+        qh = torch.full((Nq, ldh), 7.0, device=dev)
+    if op == "split":
+        tda.tda_precondition(tda.TDA_PC_FACTOR, nl, D, sdt, state, n_total=N, lambda_rel_mean_eig=1e-2)
+        tda.tda_precondition(tda.TDA_PC_APPLY, nl, D, sdt, state, q=qd, n_q=Nq, ld_q=ldq, qhat=qh, ld_qhat=ldh)
+    else:
+        tda.tda_precondition(tda.TDA_PC_FACTOR_APPLY, nl, D, sdt, state, n_total=N, lambda_rel_mean_eig=1e-2,
+                             q=qd, n_q=Nq, ld_q=ldq, qhat=qh, ld_qhat=ldh)
+    info = tda.tda_precondition_info(nl, D, sdt, state)
+    tda.tda_device_status()
+    got = qh.cpu().numpy().astype(np.float64)
+    if op == "split":
+        assert (got[:, nl * D:] == 7.0).all()
+    for l in range(nl):
+        P = phi[:, l * D:(l + 1) * D].astype(np.float64)
+        lam = orc.damping_features(P, 0.0, 1e-2)
+        assert abs(info[4 * l] - lam) <= 1e-5 * lam and info[4 * l + 2] == 0
+        Ql = q[:, l * D:(l + 1) * D].astype(np.float64)
+        ref = orc.precondition(orc.fisher(P), lam, Ql) if N >= D else orc.precondition_lowrank(P, lam, Ql)
+        assert rel_fro(got[:, l * D:(l + 1) * D], ref) <= 1e-3, l
+
+
+def test_precondition_blocked_not_spd_gives_nan(dev):
+    D = 2048
+    state = torch.empty(tda.tda_precondition_state_bytes(D, tda.TDA_F32), dtype=torch.uint8, device=dev)
+    tda.tda_precondition(tda.TDA_PC_RESET, 1, D, tda.TDA_F32, state)
+    phi = torch.ones((2, D), device=dev)
+    tda.tda_precondition(tda.TDA_PC_FIT_ACCUM, 1, D, tda.TDA_F32, state, phi=phi, n=2, ld_phi=D)
+    m = state[64:64 + 4 * D * D].view(torch.float32).view(D, D)
+    m[1500, 1500] = -1e6
+    q = torch.ones((3, D), device=dev)
+    qh = torch.zeros((3, D), device=dev)
+    tda.tda_precondition(tda.TDA_PC_FACTOR_APPLY, 1, D, tda.TDA_F32, state, n_total=2, lambda_abs=1e-3,
+                         q=q, n_q=3, ld_q=D, qhat=qh, ld_qhat=D)
+    with pytest.raises(tda.TdaError) as e:
+        tda.tda_precondition_info(1, D, tda.TDA_F32, state)
+    assert e.value.status == tda.TDA_ERR_NOT_SPD
+    assert torch.isnan(qh).all()
 
 
 @pytest.mark.parametrize("D", [64, 8])

@@ -7,8 +7,10 @@ synchronisation): its scratch is a fixed array inside libtda.so. This test
 calls it through the C ABI twice in a row -- the second call on different
 inputs, so the array holds the first call's leftovers -- and checks each result
 against tda_project with route MATERIALIZE and a caller workspace, within the
-tolerances the other parity tests use. It lives in its own file, collected
-last, and passes alone in a fresh process as well as after the other tests.
+tolerances the other parity tests use, and against the oracle; a third call
+projects more examples than the array holds at once. It lives in its own
+file, collected last, and passes alone in a fresh process as well as after the
+other tests.
 """
 import numpy as np
 import pytest
@@ -39,13 +41,19 @@ def _rel(x, ref):
 
 
 @pytest.mark.parametrize("dtype", ["f32", "bf16"])
-def test_noalloc_matches_workspace_route_on_consecutive_calls(dtype):
+def test_noalloc_matches_workspace_route_on_consecutive_calls(dtype, orc):
     assert torch.cuda.is_available(), "GPU tests need a CUDA device"
     tbuild.build()
     dev = torch.device("cuda:0")
-    shapes = [(6, 45, 256, 192, 32, 16), (4, 130, 512, 256, 16, 32)]  # second call: other sizes
+    # second call: other sizes; third: 20 examples of 4.3 MB of scratch each, more than the
+    # 64 MiB array holds at once, so one call runs the route's chunk loop over the array twice
+    shapes = [(6, 45, 256, 192, 32, 16), (4, 130, 512, 256, 16, 32), (20, 24, 1024, 1024, 32, 32)]
     for call, (N, T, di, do, ki, ko) in enumerate(shapes):
         L = tda.LayerDesc(di, do, T, ki, ko, seed=7, layer=call)
+        if call == 2:
+            assert N * 4 * (do * di + do * ki) > tda.tda_noalloc_scratch_bytes()
+        Ah = synth.factors(synth.SEED_A, 20 + call, N, T, di, 1.0, dtype=dtype, mask_p=0.02)
+        Bh = synth.factors(synth.SEED_B, 20 + call, N, T, do, 0.1, dtype=dtype, mask_p=0.02)
         A, B = _factors(N, T, di, do, dtype, 20 + call, dev)
         D = ki * ko
         got = torch.full((N, D), float("nan"), device=dev)
@@ -57,6 +65,9 @@ def test_noalloc_matches_workspace_route_on_consecutive_calls(dtype):
         tda.tda_device_status()
         assert not torch.isnan(got).any()
         assert _rel(got, ref) <= TOL[dtype]
+        # and against the oracle's fp64 projection of the same factor bits
+        oref = orc.project(synth.to_f64(Ah, dtype), synth.to_f64(Bh, dtype), ki, ko, 7, call).reshape(N, D)
+        assert _rel(got, torch.from_numpy(oref)) <= TOL[dtype]
 
 
 def test_noalloc_rejects_layers_beyond_the_scratch():
