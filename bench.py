@@ -92,6 +92,10 @@ def parse_args():
                    help="Fisher query side on a second stream; the train projection leaves this many SMs free")
     p.add_argument("--train-streams", type=int, default=2,
                    help="stack workloads: streams the train projections of a chunk are spread over")
+    p.add_argument("--query-side-stream", type=int, default=1,
+                   help="stack workloads: 1 = the query side and top-k on a stream of their own beside the "
+                        "next chunks' projections, 0 = in line after each chunk")
+    p.add_argument("--query-priority", type=int, default=0, help="priority of that stream (lower = higher)")
     p.add_argument("--query-streams", type=int, default=8,
                    help="streams the query projections of the linears are spread over (device-resident leg)")
     p.add_argument("--e2e-steps", type=int, default=2)
@@ -106,6 +110,13 @@ def parse_args():
                    help="time token-level scores of the block (every train token against every preconditioned query)")
     p.add_argument("--masks", type=int, default=0,
                    help="time the random-mask reduction: ten disjoint masks of this many DW coordinates per linear")
+    p.add_argument("--profile-project", default="",
+                   help="stack workloads: time only the factored projection of this linear of a layer "
+                        "(e.g. gate) over --profile-n examples, --steps launches (kernel profiling)")
+    p.add_argument("--profile-precond", action="store_true",
+                   help="stack workloads: time only one share's Fisher fit and factorisation with query solves "
+                        "(one layer's linears, --profile-n train features) (kernel profiling)")
+    p.add_argument("--profile-n", type=int, default=64)
     p.add_argument("--route-sweep", action="store_true",
                    help="route cost-model sweep on one 8192x8192 bf16 linear (chosen vs measured fastest route)")
     p.add_argument("--sweep-T", default="8,32,128,512,2048,8192")
@@ -581,7 +592,7 @@ STACKS = {
                   ("gate", 4096, 14336), ("up", 4096, 14336), ("down", 14336, 4096)],
         "n_layers": 32, "T": 1024, "k": 64, "n_train": 8192, "chunk": 256, "n_query": 256,
         "dist_a": 0, "sigma_b": math.sqrt(1e-3), "lambda_rel": 1e-2,
-        "train_pool": 512, "query_pool": 256, "host_pool": 32,
+        "train_pool": 512, "query_pool": 256, "host_pool": 128,
         "factors": "A~N(0,1), B~N(0,1e-3) (seeded synthetic)",
     },
     "large_model": {
@@ -589,7 +600,7 @@ STACKS = {
                   ("gate", 12288, 49152), ("up", 12288, 49152), ("down", 49152, 12288)],
         "n_layers": 1, "T": 2048, "k": 128, "n_train": 16384, "chunk": 512, "n_query": 512,
         "dist_a": 1, "sigma_b": 0.01, "lambda_rel": 1e-2,
-        "train_pool": 96, "query_pool": 64, "host_pool": 16,
+        "train_pool": 128, "query_pool": 64, "host_pool": 16,
         "factors": "A~Student-t(4), B~N(0,1e-4) (seeded synthetic)",
     },
 }
@@ -708,6 +719,74 @@ def stack_reference_main(args, spec):
     return 0
 
 
+def stack_profile_main(args, spec):
+    """Small cases of the stack workloads' dominant kernels for ncu: one linear's factored
+    projection, or one share's Fisher fit + factorisation with the query solves."""
+    import torch
+
+    import paper_2609_38767_gb300 as tda
+    from paper_2609_38767_gb300 import build as tbuild
+    from paper_2609_38767_gb300 import synth
+
+    tbuild.build()
+    tda.load()
+    dev = torch.device("cuda", 0)
+    torch.cuda.set_device(dev)
+    stream = torch.cuda.current_stream()
+    T, k, n = spec["T"], spec["k"], args.profile_n
+    D = k * k
+    ev0, ev1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    if args.profile_project:
+        li = [x[0] for x in spec["layer"]].index(args.profile_project)
+        _, di, do = spec["layer"][li]
+        A = torch.empty((n, T, di), dtype=torch.bfloat16, device=dev)
+        B = torch.empty((n, T, do), dtype=torch.bfloat16, device=dev)
+        synth.fill_device(A, synth.SEED_A, li, n, T, di, 1.0, spec["dist_a"])
+        synth.fill_device(B, synth.SEED_B, li, n, T, do, spec["sigma_b"])
+        L = tda.LayerDesc(di, do, T, k, k, seed=0, layer=li)
+        assert tda.tda_project_engine(L, tda.TDA_BF16, A, B) == 1
+        wsb = tda.tda_workspace_size(tda.TDA_OP_PROJECT, L, tda.TDA_BF16, n, 0, tda.TDA_ROUTE_FACTORED)
+        ws = torch.empty(max(wsb, 256), dtype=torch.uint8, device=dev)
+        phi = torch.empty((n, D), device=dev)
+        run = lambda: tda.tda_project(L, tda.TDA_BF16, A, B, n, phi, D, tda.TDA_ROUTE_FACTORED, ws, wsb)
+        work = ("GB/s", n * (T * (di + do) * 2 + 4 * D) / 1e9)
+        what = {"kernel": "factored projection", "linear": [di, do], "n": n, "T": T, "k": k,
+                "sign_tables": bool(wsb)}
+    else:
+        nl = len(spec["layer"])
+        per = tda.tda_precondition_state_bytes(D, tda.TDA_F32)
+        st = torch.empty(nl * per, dtype=torch.uint8, device=dev)
+        phi = torch.empty(n * nl * D, dtype=torch.float32, device=dev)
+        synth.fill_device(phi, 5, 0, n, 1, nl * D, 1.0)
+        q = torch.empty(spec["n_query"] * nl * D, dtype=torch.float32, device=dev)
+        synth.fill_device(q, 6, 0, spec["n_query"], 1, nl * D, 1.0)
+        qh = torch.empty_like(q)
+        Nq = spec["n_query"]
+
+        def run():
+            tda.tda_precondition(tda.TDA_PC_RESET, nl, D, tda.TDA_F32, st)
+            tda.tda_precondition(tda.TDA_PC_FIT_ACCUM, nl, D, tda.TDA_F32, st, phi=phi, n=n, ld_phi=nl * D)
+            tda.tda_precondition(tda.TDA_PC_FACTOR_APPLY, nl, D, tda.TDA_F32, st, n_total=n,
+                                 lambda_rel_mean_eig=spec["lambda_rel"], q=q, n_q=Nq, ld_q=nl * D, qhat=qh,
+                                 ld_qhat=nl * D)
+        work = ("TFLOP/s", nl * (n * D * (D + 1) + 2 * (D ** 3 / 3 + 2 * D * D * Nq)) / 1e12)
+        what = {"kernel": "Fisher fit + factorisation + query solves", "linears": nl, "D": D, "n_train": n,
+                "n_query": Nq}
+    for _ in range(max(args.warmup, 1)):
+        run()
+    torch.cuda.synchronize()
+    ev0.record(stream)
+    for _ in range(args.steps):
+        run()
+    ev1.record(stream)
+    torch.cuda.synchronize()
+    tda.tda_device_status()
+    ms = ev0.elapsed_time(ev1) / args.steps
+    print(json.dumps({"mode": "profile", **what, "ms_per_call": ms,
+                      "rate": work[1] / (ms * 1e-3), "unit": work[0]}))
+    return 0
+
+
 def stack_main(args, spec):
     import numpy as np
     import torch
@@ -765,7 +844,8 @@ def stack_main(args, spec):
         return [(Aq[:min(Pq, Nq - r)], Bq[:min(Pq, Nq - r)], r, min(Pq, Nq - r)) for r in range(0, Nq, Pq)]
 
     job = StackJob(linears, T, k, N, chunk, Nq, topk=args.topk, lambda_rel=spec["lambda_rel"], device=dev,
-                   train_streams=args.train_streams)
+                   train_streams=args.train_streams, query_stream=bool(args.query_side_stream),
+                   query_priority=args.query_priority)
     for si in range(nshape):  # every linear shape runs on the tensor-core projection kernel
         assert tda.tda_project_engine(job.layers[si], tda.TDA_BF16, pools[si][0], pools[si][1]) == 1
     state = {"j": 0, "s": 0}
@@ -780,21 +860,23 @@ def stack_main(args, spec):
         advance(dev_factors)
     for _ in range(args.warmup):
         advance(dev_factors)
+    job.join()
     tda.tda_device_status()
     torch.cuda.synchronize()
 
     ev, phase_ev, open_ev = [], [], {}
 
     def mark(name):
+        st = torch.cuda.current_stream()  # phases are timed on the stream they run on
         e = torch.cuda.Event(enable_timing=True)
-        e.record(stream)
-        phase_ev.append((name, e))
+        e.record(st)
+        phase_ev.append((name, e, st.cuda_stream))
 
     def hook(role, li, when, n):
         if role != "train":
             return
         e = torch.cuda.Event(enable_timing=True)
-        e.record(stream)
+        e.record(torch.cuda.current_stream())
         if when == "begin":
             open_ev[li] = e
         else:
@@ -809,6 +891,7 @@ def stack_main(args, spec):
     t0.record(stream)
     for _ in range(steps):
         advance(dev_factors, mark, hook)
+    job.join()  # the query side queued in the timed steps is inside the timed region
     t1.record(stream)
     torch.cuda.synchronize()
     launches = tda.tda_launch_count() - l0
@@ -829,7 +912,15 @@ def stack_main(args, spec):
     # algorithmic bytes over the phase's time (events on the launching stream around the fork
     # and join of the projection streams)
     proj_bytes = sum(x for _, _, x in ev)
-    ph_train = sum(a.elapsed_time(b) for (name, a), (_, b) in zip(phase_ev, phase_ev[1:]) if name == "project_train")
+    seqs = {}
+    for name, e, sid in phase_ev:
+        seqs.setdefault(sid, []).append((name, e))
+    ph = {}
+    for seq in seqs.values():
+        for (name, a), (_, b) in zip(seq, seq[1:]):
+            if name is not None:
+                ph[name] = ph.get(name, 0.0) + a.elapsed_time(b) / steps
+    ph_train = ph.get("project_train", 0.0) * steps
     achieved = proj_bytes / (ph_train * 1e-3) / 1e9
     per_launch = proj_bytes / max(len(ev), 1)
     roofline = {"bound": "hbm", "kernel": f"factored projection (train, k = {k}, tcgen05)", "achieved": achieved,
@@ -841,10 +932,6 @@ def stack_main(args, spec):
                 "share_of_step": ph_train / (ms * steps)}
     if k == 64 and projection_kernel_sha256() == TRAFFIC_KERNEL_SHA256:
         roofline["traffic"] = TRAFFIC_RATIO * per_launch
-    ph = {}
-    for (name, a), (_, b) in zip(phase_ev, phase_ev[1:]):
-        if name is not None:
-            ph[name] = ph.get(name, 0.0) + a.elapsed_time(b) / steps
     Dn = float(D)
     per_job_lin = {
         "project_train": ("hbm", sum(N * (T * (di + do) * 2 + 4 * D) for di, do in linears), hbm, "GB/s"),
@@ -886,6 +973,8 @@ def stack_main(args, spec):
         # the H2D ceiling, measured as the e2e leg copies: four copy streams at once, several GB
         copy_streams = [torch.cuda.Stream(device=dev) for _ in range(4)]
         srcs = [hpools[si][i] for si in range(nshape) for i in range(2)]
+        while len(srcs) > 2 and sum(x.numel() * 2 for x in srcs) > 12e9:
+            srcs = srcs[:-1]
         dsts = [torch.empty_like(x, device=dev) for x in srcs]
         nbytes = sum(x.numel() * 2 for x in srcs)
         for rep in range(2):
@@ -903,6 +992,7 @@ def stack_main(args, spec):
         def e2e_step():
             s = state["s"]
             advance(host_factors)
+            job.join()
             r0, r1 = job.share(s, Nq)
             idx_h[r0:r1].copy_(job.idx[r0:r1], non_blocking=True)
             val_h[r0:r1].copy_(job.val[r0:r1], non_blocking=True)
@@ -950,6 +1040,8 @@ def main():
     if args.workload in STACKS:
         if args.impl == "reference":
             return stack_reference_main(args, STACKS[args.workload])
+        if args.profile_project or args.profile_precond:
+            return stack_profile_main(args, STACKS[args.workload])
         return stack_main(args, STACKS[args.workload])
     if args.impl == "reference":
         return reference_main(args)

@@ -1036,20 +1036,23 @@ cudaError_t apply_impl(int n_layers, int64_t D, const void* state, const float* 
 constexpr int kBB = 128;                // panel width
 constexpr int64_t kBlockedMinD = 2048;  // smaller layers keep the one-launch cluster path
 constexpr int kTrsmWarps = 8;
-constexpr size_t kDiagSmem = sizeof(float) * ((size_t)kBB * (kBB + 1) + (size_t)(kBB - kNB) * (kNB + 1));
+constexpr size_t kDiagSmem = sizeof(float) * (size_t)kBB * (kBB + 1);
 constexpr size_t kTrsmSmem =
     sizeof(float) * ((size_t)kBB * (kBB + 1) + (size_t)(kBB / kNB) * kNB * (kNB + 1) + (size_t)kTrsmWarps * kBB);
 
 // Factor the 128 x 128 diagonal block at lo of every layer (grid = layer) in
 // shared memory, in four 32-column steps: Cholesky of the 32 x 32 block by one
-// warp (as panel_kernel), its inverse into Dinv, the block's rows below it
-// solved against it, the rest of the block updated. L returns to M's lower
-// triangle; a non-positive pivot is recorded in the header.
+// warp (warp_cholesky32: rolled steps, the pivot column in register 0), the
+// block's rows below it solved against it by forward substitution (one thread
+// per row, rolled loops), the rest of the block updated. L returns to M's lower
+// triangle; the inverses of the four 32 x 32 diagonal blocks go to Dinv (one
+// warp each, after the last step); a non-positive pivot is recorded in the header.
 __global__ void __launch_bounds__(256) diag_block_kernel(St<float> st, int64_t lo) {
     extern __shared__ __align__(16) float dsm[];
     float(*A)[kBB + 1] = reinterpret_cast<float(*)[kBB + 1]>(dsm);
-    float(*X)[kNB + 1] = reinterpret_cast<float(*)[kNB + 1]>(dsm + kBB * (kBB + 1));
-    __shared__ float Di[kNB][kNB + 1];
+    __shared__ float Bk[kNB][kNB + 1];        // the step's diagonal block before factoring
+    __shared__ float LkT[kNB][2 * kNB + 1];   // its factor, transposed
+    __shared__ float dinv[kNB];
     const int l = blockIdx.x;
     const int64_t D = st.D;
     float* M = st.M(l);
@@ -1060,72 +1063,61 @@ __global__ void __launch_bounds__(256) diag_block_kernel(St<float> st, int64_t l
     }
     __syncthreads();
     for (int c0 = 0; c0 < kBB; c0 += kNB) {
+        for (int e = tid; e < kNB * kNB; e += 256) Bk[e / kNB][e % kNB] = A[c0 + e / kNB][c0 + e % kNB];
+        __syncthreads();
         if (warp == 0) {
-            float r[kNB];
-#pragma unroll
-            for (int c = 0; c < kNB; ++c) r[c] = A[c0 + lane][c0 + c];
-            int bad = -1;
-#pragma unroll
-            for (int j = 0; j < kNB; ++j) {
-                const float p = __shfl_sync(0xffffffffu, r[j], j);
-                const bool ok = p > 0.f;
-                if (!ok && bad < 0) bad = j;
-                const float piv = ok ? sqrtf(p) : NAN;
-                if (lane == j) r[j] = piv;
-                if (lane > j) r[j] /= piv;
-#pragma unroll
-                for (int c = j + 1; c < kNB; ++c) {
-                    const float v = __shfl_sync(0xffffffffu, r[j], c);  // L[c][j]
-                    if (lane >= c) r[c] -= r[j] * v;
-                }
-            }
-#pragma unroll
-            for (int c = 0; c < kNB; ++c) A[c0 + lane][c0 + c] = (c <= lane) ? r[c] : 0.f;
+            const int bad = warp_cholesky32(Bk, LkT, dinv, lane);
             if (lane == 0 && bad >= 0) {
                 double* h = st.header(l);
                 if (h[kPcFailedPivot] == 0.0) h[kPcFailedPivot] = (double)(lo + c0 + bad + 1);
             }
-            __syncwarp();
-            // inverse of the block: lane c solves L x = e_c
-            float x[kNB];
-#pragma unroll
-            for (int i = 0; i < kNB; ++i) {
-                float t = (i == lane) ? 1.f : 0.f;
-#pragma unroll
-                for (int m = 0; m < i; ++m) t -= A[c0 + i][c0 + m] * x[m];
-                x[i] = (i < lane) ? 0.f : t / A[c0 + i][c0 + i];
-            }
-            float* Dg = st.Dinv(l) + ((lo + c0) / kNB) * (kNB * kNB);
-#pragma unroll
-            for (int i = 0; i < kNB; ++i) {
-                Di[i][lane] = x[i];
-                Dg[i * kNB + lane] = x[i];
-            }
         }
         __syncthreads();
+        for (int e = tid; e < kNB * kNB; e += 256) {
+            const int i = e / kNB, j = e % kNB;  // L of the step's block back into A
+            A[c0 + i][c0 + j] = (j <= i) ? LkT[j][i] : 0.f;
+        }
         const int rows = kBB - c0 - kNB;  // rows of the block below this step's diagonal block
-        // x L_ss^T = a, i.e. x_j = sum_{m <= j} Dinv[j][m] a_m
-        for (int e = tid; e < rows * kNB; e += 256) {
-            const int i = e / kNB, j = e % kNB;
-            float acc = 0.f;
-            for (int m = 0; m <= j; ++m) acc += Di[j][m] * A[c0 + kNB + i][c0 + m];
-            X[i][j] = acc;
+        // x L_ss^T = a, one row per thread: x_j = (a_j - sum_{m<j} x_m L_jm) / L_jj, in place
+        if (tid < rows) {
+            float* a = A[c0 + kNB + tid] + c0;
+#pragma unroll 1
+            for (int jj = 0; jj < kNB; ++jj) {
+                float t = a[jj];
+#pragma unroll 4
+                for (int m = 0; m < jj; ++m) t -= a[m] * LkT[m][jj];
+                a[jj] = t * dinv[jj];
+            }
         }
         __syncthreads();
-        for (int e = tid; e < rows * kNB; e += 256) {
-            const int i = e / kNB, j = e % kNB;
-            A[c0 + kNB + i][c0 + j] = X[i][j];
-        }
         // the block's trailing lower triangle
         for (int e = tid; e < rows * rows; e += 256) {
             const int i = e / rows, j = e % rows;
             if (j > i) continue;
+            const float* xi = A[c0 + kNB + i] + c0;
+            const float* xj = A[c0 + kNB + j] + c0;
             float acc = 0.f;
 #pragma unroll 8
-            for (int m = 0; m < kNB; ++m) acc += X[i][m] * X[j][m];
+            for (int m = 0; m < kNB; ++m) acc += xi[m] * xj[m];
             A[c0 + kNB + i][c0 + kNB + j] -= acc;
         }
         __syncthreads();
+    }
+    // inverses of the four diagonal blocks: warp w, lane c solves L X[:, c] = e_c
+    if (warp < kBB / kNB) {
+        const int b0 = warp * kNB, c = lane;
+        float x[kNB];
+#pragma unroll
+        for (int i = 0; i < kNB; ++i) x[i] = (i == c) ? 1.f : 0.f;
+#pragma unroll
+        for (int jj = 0; jj < kNB; ++jj) {
+            x[jj] = (jj < c) ? 0.f : x[jj] / A[b0 + jj][b0 + jj];
+#pragma unroll
+            for (int i = jj + 1; i < kNB; ++i) x[i] -= A[b0 + i][b0 + jj] * x[jj];
+        }
+        float* Dg = st.Dinv(l) + ((lo + b0) / kNB) * (kNB * kNB);
+#pragma unroll
+        for (int i = 0; i < kNB; ++i) Dg[i * kNB + c] = x[i];
     }
     for (int e = tid; e < kBB * kBB; e += 256) {
         const int i = e / kBB, j = e % kBB;
@@ -1206,6 +1198,25 @@ __global__ void __launch_bounds__(256) trsm_block_kernel(St<float> st, int64_t l
     }
 }
 
+// Lower triangle of M <- M / n_total + lambda I for the blocked path: one row per
+// loop step of a CTA, the row's columns across the threads (coalesced, no per-element
+// index division). grid (row groups, layer).
+__global__ void __launch_bounds__(256) scale_lower_kernel(St<float> st) {
+    const int l = blockIdx.y;
+    const int64_t D = st.D;
+    const double* h = st.header(l);
+    const float inv_n = (float)(1.0 / h[kPcNTotal]), lam = (float)h[kPcLambda];
+    float* M = st.M(l);
+    for (int64_t a = blockIdx.x; a < D; a += gridDim.x) {
+        float* row = M + a * D;
+        for (int64_t b = threadIdx.x; b <= a; b += 256) {
+            float v = row[b] * inv_n;
+            if (b == a) v += lam;
+            row[b] = v;
+        }
+    }
+}
+
 // M[i][j] = M[j][i] for every 32 x 32 block strictly above the diagonal blocks
 // (U = L^T, read by the backward solve's tensor-core products).
 __global__ void __launch_bounds__(256) upper_from_lower_kernel(St<float> st, int n_layers) {
@@ -1271,9 +1282,8 @@ cudaError_t factor_blocked(int n_layers, int64_t D, void* state, int64_t n_total
     St<float> st = state_of<float>(state, D);
     note_launches(2);
     prepare_kernel<float><<<n_layers, 256, 0, s>>>(st, n_total, la, lr);
-    int64_t blocks = (D * D * n_layers + 255) / 256;
-    if (blocks > 152 * 16) blocks = 152 * 16;
-    scale_kernel<float><<<(unsigned)blocks, 256, 0, s>>>(st, n_layers);
+    const unsigned rows_per = (unsigned)((D < 1024 ? D : 1024) * (n_layers < 8 ? 8 / n_layers : 1));
+    scale_lower_kernel<<<dim3(rows_per < (unsigned)D ? rows_per : (unsigned)D, n_layers), 256, 0, s>>>(st);
     // outer panels of 256 columns, each two 128-column sub-panels: the second sub-panel's
     // columns take the first one's update alone (a 128-wide product), and the trailing
     // matrix takes both at once (rank-256 update: twice the work per tile pass over M)

@@ -34,13 +34,18 @@ import paper_2609_38767_gb300 as tda
 
 class StackJob:
     def __init__(self, linears, T, k, n_train, chunk, n_query, *, topk=100, lambda_rel=1e-2, lambda_abs=0.0,
-                 seed=0, device="cuda", host_ws_bytes=0, train_streams=1, proj_ws=True):
+                 seed=0, device="cuda", host_ws_bytes=0, train_streams=1, proj_ws=True, query_stream=False,
+                 query_priority=0):
         """linears: [(d_in, d_out)] of the whole stack, in layer order (linear i uses projection
         layer id i). n_train must be a multiple of chunk. train_streams > 1 spreads the train
         projections of a chunk round-robin over that many streams, so that a launch's CTAs fill
         the SMs its predecessor's last tiles leave idle (every launch writes its own feature
         columns: the results do not depend on the order). proj_ws: give the factored projection
-        its optional workspace (k = 128: precomputed sign tables)."""
+        its optional workspace (k = 128: precomputed sign tables). query_stream: run the query
+        side and the top-k on a stream of their own (priority query_priority), beside the
+        next chunks' projections; events order the two job-boundary dependencies (a job's
+        query side starts after its last chunk is projected; a job's features are overwritten
+        two jobs later only after that query side has read them)."""
         assert n_train % chunk == 0 and n_train >= topk >= 1
         self.layers = [tda.LayerDesc(di, do, T, k, k, seed=seed, layer=i) for i, (di, do) in enumerate(linears)]
         self.nl = len(self.layers)
@@ -67,7 +72,10 @@ class StackJob:
         self.proj_wsb = max(tda.tda_workspace_size(tda.TDA_OP_PROJECT, L, tda.TDA_BF16, chunk, 0,
                                                    tda.TDA_ROUTE_FACTORED) for L in self.layers) if proj_ws else 0
         self.proj_ws = [torch.empty(self.proj_wsb, dtype=torch.uint8, device=dev)
-                        for _ in range(self.train_streams)] if self.proj_wsb else None
+                        for _ in range(self.train_streams + 1)] if self.proj_wsb else None
+        self.side = torch.cuda.Stream(device=dev, priority=query_priority) if query_stream else None
+        self._train_done = {}  # job -> event after its last chunk's projections (train stream)
+        self._query_done = {}  # job -> event after its last query share (query stream)
 
     # ------------------------------------------------------------------ shares of a job
     def share(self, s, total):
@@ -120,13 +128,14 @@ class StackJob:
             return
         D, DT = self.D, self.DT
         st = self.state[:(l1 - l0) * self.per]
+        slot = self.train_streams  # the query side's own projection workspace
         mark("fisher_fit")
         tda.tda_precondition(tda.TDA_PC_RESET, l1 - l0, D, tda.TDA_F32, st)
         tda.tda_precondition(tda.TDA_PC_FIT_ACCUM, l1 - l0, D, tda.TDA_F32, st, phi=self.Phi[b][:, l0 * D:],
                              n=self.N, ld_phi=DT)
         mark("project_query")
         for li in range(l0, l1):
-            self._project(self.layers[li], factors("query", li, j, s), self.Q[:, li * D:], hook, li, "query")
+            self._project(self.layers[li], factors("query", li, j, s), self.Q[:, li * D:], hook, li, "query", slot)
         mark("factor_apply")
         tda.tda_precondition(tda.TDA_PC_FACTOR_APPLY, l1 - l0, D, tda.TDA_F32, st, n_total=self.N,
                              lambda_abs=self.lambda_abs, lambda_rel_mean_eig=self.lambda_rel, q=self.Q[:, l0 * D:],
@@ -147,10 +156,40 @@ class StackJob:
     def step(self, j, s, factors, first_job=0, mark=None, hook=None):
         """Step s of job j: chunk s of job j, share s of job j-1's query side and of job
         j-2's top-k. Jobs before first_job do not exist (their shares are skipped)."""
+        if self.side is None:
+            self.train_part(j, s, factors, mark, hook)
+            if j - 1 >= first_job:
+                self.query_part(j - 1, s, factors, mark, hook)
+            if j - 2 >= first_job:
+                self.topk_part(j - 2, s, mark)
+            if mark:
+                mark(None)
+            return
+        main = torch.cuda.current_stream()
+        if s == 0 and (j - 2) in self._query_done:
+            main.wait_event(self._query_done.pop(j - 2))  # job j overwrites job j-2's features
         self.train_part(j, s, factors, mark, hook)
-        if j - 1 >= first_job:
-            self.query_part(j - 1, s, factors, mark, hook)
-        if j - 2 >= first_job:
-            self.topk_part(j - 2, s, mark)
         if mark:
             mark(None)
+        if s == self.C - 1:
+            e = torch.cuda.Event()
+            e.record(main)
+            self._train_done[j] = e
+        with torch.cuda.stream(self.side):
+            if j - 1 >= first_job:
+                if s == 0 and (j - 1) in self._train_done:
+                    self.side.wait_event(self._train_done.pop(j - 1))
+                self.query_part(j - 1, s, factors, mark, hook)
+                if s == self.C - 1:
+                    e = torch.cuda.Event()
+                    e.record(self.side)
+                    self._query_done[j - 1] = e
+            if j - 2 >= first_job:
+                self.topk_part(j - 2, s, mark)
+            if mark:
+                mark(None)
+
+    def join(self):
+        """Make the current stream wait for the query side's work queued so far."""
+        if self.side is not None:
+            torch.cuda.current_stream().wait_stream(self.side)

@@ -8,7 +8,7 @@ Fisher, damped inverse (Woodbury form: fewer examples than features), score
 matrix and top-k over the same factors. The shares of the query side differ in
 size (six linears over four steps), D = 4096 takes the blocked tensor-core
 preconditioner, and the train projections of a chunk run on one or on three
-streams.
+streams, the query side in line or on a stream of its own.
 """
 import os
 
@@ -51,8 +51,8 @@ def window(role, li, j, s):
     return [(2 * j + li + r) % PQ for r in range(NQ)]
 
 
-@pytest.mark.parametrize("train_streams", [1, 3])
-def test_stack_job_matches_oracle(orc, train_streams):
+@pytest.mark.parametrize("train_streams,query_stream", [(1, False), (3, True)])
+def test_stack_job_matches_oracle(orc, train_streams, query_stream):
     assert torch.cuda.is_available(), "GPU tests need a CUDA device"
     tbuild.build()
     tda.load()
@@ -73,11 +73,14 @@ def test_stack_job_matches_oracle(orc, train_streams):
             r = e + 1
         return pieces
 
-    job = StackJob(LIN, T, K, N, CHUNK, NQ, topk=TOPK, lambda_rel=1e-2, device=dev, train_streams=train_streams)
+    job = StackJob(LIN, T, K, N, CHUNK, NQ, topk=TOPK, lambda_rel=1e-2, device=dev, train_streams=train_streams,
+                   query_stream=query_stream)
     marks = []
     for j in range(3):
         for s in range(job.C):
             job.step(j, s, factors, mark=marks.append)
+    job.join()
+    torch.cuda.synchronize()
     tda.tda_device_status()
     assert {"project_train", "fisher_fit", "project_query", "factor_apply", "score", "topk"} <= set(marks)
 
