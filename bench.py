@@ -117,6 +117,10 @@ def parse_args():
                    help="stack workloads: time only one share's Fisher fit and factorisation with query solves "
                         "(one layer's linears, --profile-n train features) (kernel profiling)")
     p.add_argument("--profile-n", type=int, default=64)
+    p.add_argument("--sm-budget", type=int, default=0,
+                   help="cap the persistent projection grid at this many CTAs (tda_set_sm_budget; 0 = every SM)")
+    p.add_argument("--nvtx", action="store_true",
+                   help="stack workloads: push an NVTX range 'timed' around the timed steps (for ncu --nvtx)")
     p.add_argument("--route-sweep", action="store_true",
                    help="route cost-model sweep on one 8192x8192 bf16 linear (chosen vs measured fastest route)")
     p.add_argument("--sweep-T", default="8,32,128,512,2048,8192")
@@ -730,6 +734,7 @@ def stack_profile_main(args, spec):
 
     tbuild.build()
     tda.load()
+    tda.tda_set_sm_budget(args.sm_budget)
     dev = torch.device("cuda", 0)
     torch.cuda.set_device(dev)
     stream = torch.cuda.current_stream()
@@ -782,7 +787,7 @@ def stack_profile_main(args, spec):
     torch.cuda.synchronize()
     tda.tda_device_status()
     ms = ev0.elapsed_time(ev1) / args.steps
-    print(json.dumps({"mode": "profile", **what, "ms_per_call": ms,
+    print(json.dumps({"mode": "profile", **what, "sm_budget": args.sm_budget, "ms_per_call": ms,
                       "rate": work[1] / (ms * 1e-3), "unit": work[0]}))
     return 0
 
@@ -800,6 +805,7 @@ def stack_main(args, spec):
         return 0  # one GPU: the stack job does not shard here
     tbuild.build()
     tda.load()
+    tda.tda_set_sm_budget(args.sm_budget)
     dev = torch.device("cuda", 0)
     torch.cuda.set_device(dev)
     stream = torch.cuda.current_stream()
@@ -888,11 +894,15 @@ def stack_main(args, spec):
     time.sleep(0.3)
     l0 = tda.tda_launch_count()
     t0, t1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    if args.nvtx:
+        torch.cuda.nvtx.range_push("timed")
     t0.record(stream)
     for _ in range(steps):
         advance(dev_factors, mark, hook)
     job.join()  # the query side queued in the timed steps is inside the timed region
     t1.record(stream)
+    if args.nvtx:
+        torch.cuda.nvtx.range_pop()
     torch.cuda.synchronize()
     launches = tda.tda_launch_count() - l0
     ck = clocks.stop()

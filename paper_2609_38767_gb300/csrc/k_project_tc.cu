@@ -61,16 +61,23 @@ constexpr uint32_t kTileBytes = kTileM * kChunkK * 2;  // 16 KiB per factor tile
 constexpr size_t kSmemMax = 232448;    // 227 KiB of dynamic shared memory per CTA
 constexpr int kMaxStages = 12;
 
-template <int K, int G>
+// SR: token rows the epilogue stages in shared memory at a time (32, 64 or 128).
+// Fewer rows leave room for more stages in the ring, i.e. more factor bytes in
+// flight per SM, which is what an HBM-bound stream needs; a whole tile (128)
+// is staged where the epilogue needs every row at once (packed short
+// sequences, the K-FAC covariances, the factor output).
+template <int K, int G, int SR = (K > 64 ? kTileM / 2 : kTileM)>
 struct Cfg {
     static constexpr int kK = K;
     static constexpr uint32_t kSignBytes = K * 128;                       // K rows x 128 bytes
     static constexpr uint32_t kStageBytes = G * kTileBytes + kSignBytes;  // G factor tiles, then signs
     static constexpr int kStageLd = K + 4;                                // padded fp32 staging row
-    // K = 128: the fp32 rows of a whole tile (2 x 128 x 132 floats) would crowd out the
-    // stage ring, so the epilogue stages and contracts 64 token rows at a time
+    // K = 128: signs are expanded through a byte table, two columns per generator lane
     static constexpr bool kHalf = K > 64;
-    static constexpr int kStageRows = kHalf ? kTileM / 2 : kTileM;
+    // the epilogue stages and contracts a tile's token rows in parts of SR rows
+    static constexpr bool kParted = SR < kTileM;
+    static constexpr int kStageRows = SR;
+    static_assert(SR == 32 || SR == 64 || SR == 128, "whole TMEM lane quadrants per part");
     static constexpr int kAccCols = 2 * K;                                // At | Bt of one tile
     static constexpr int kBufCols = G * kAccCols;                         // one accumulator buffer
     // tcgen05.alloc takes a power of two from 32 to 512 columns
@@ -97,6 +104,7 @@ struct Cfg {
     static constexpr int CB = K / 8;
     static_assert(kStages >= 3 && kSmem <= kSmemMax, "shared memory per CTA");
     static_assert(!kHalf || G == 1, "K = 128 fills TMEM with one double-buffered tile");
+    static_assert(!kHalf || kParted, "K = 128 stages at most half a tile");
     static_assert(!kHalf || (kThreads == 256 && K == 128), "one thread per sign-table entry; two columns per lane");
     static_assert(kStageBytes % 1024 == 0 && 2 * kBufCols <= (int)kTmemCols && kTmemCols <= 512,
                   "operand alignment / TMEM columns");
@@ -256,12 +264,13 @@ __device__ __forceinline__ void store_sign_row(uint8_t* tile, int n, const uint4
 // factors At, Bt of every token instead of contracting them into Phi. SL: the
 // sign tiles come by TMA from a precomputed table (tmSA, tmSB: [K][d] bf16, a
 // side's S transposed) instead of the generator warps.
-template <int K, int G, bool KF, bool FO, bool SL = false>
+template <int K, int G, bool KF, bool FO, bool SL = false, int SR = Cfg<K, G>::kStageRows>
 __global__ void __launch_bounds__(kThreads, 1)
 project_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
                   const __grid_constant__ CUtensorMap tmSA, const __grid_constant__ CUtensorMap tmSB,
                   const Params p) {
-    using C = Cfg<K, G>;
+    using C = Cfg<K, G, SR>;
+    static_assert(!C::kParted || (!KF && !FO), "the K-FAC and factor-output epilogues stage whole tiles");
     extern __shared__ uint8_t smem_raw[];
     uint8_t* smem = (uint8_t*)(((uintptr_t)smem_raw + 1023) & ~(uintptr_t)1023);
     uint8_t* sA = smem;                           // kStages x [G factor tiles | sign tile]
@@ -440,21 +449,22 @@ project_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant
                 __syncwarp();
                 if (lane == 0) mbar_arrive(smem_u32(&sready[s]));
             }
-    } else if (C::kHalf && warp >= 4) {
-        // ---------------- epilogue for K = 128 (one example per tile, one tile per group):
-        // the tile's token rows in parts of kStageRows (rows 0-63 from TMEM lane
-        // quadrants 0, 1, then rows 64-127 from quadrants 2, 3), each part staged in
-        // shared memory and contracted, Phi += Bt^T At, in fp32. The
-        // accumulators live for one example (the loop nest keeps them within the
-        // register budget: 128 per thread).
+    } else if (C::kParted && warp >= 4) {
+        // ---------------- epilogue, one example per tile (no packing): each tile's token
+        // rows in parts of kStageRows (part h holds the TMEM lane quadrants of warps
+        // h * kWarpsPer ..), each part staged in shared memory and contracted,
+        // Phi += Bt^T At, in fp32. A warp releases the accumulator buffer once it has
+        // read its quadrant of the group's last tile. The accumulators live for one
+        // example (K = 128: the loop nest keeps them within 255 registers a thread).
         const int q = warp & 3;
         const int et = threadIdx.x - 128;
         const int rg = et >> 3, cg = et & 7;
+        constexpr int kParts = kTileM / C::kStageRows, kWarpsPer = 4 / kParts;
         uint32_t grp = 0, red_use = 0;
         bool ok = true;
-        int ng = it.take<G>(p, ncl, crank, gx, gt);
+        int ng = it.take<G>(p, ncl, crank, gx, gt), u = 0;  // u: next tile of the current group
         while (ok && ng > 0) {
-            const int64_t cur = gx[0];
+            const int64_t cur = gx[u];
             float acc[C::RB][C::CB];
 #pragma unroll
             for (int a = 0; a < C::RB; ++a)
@@ -462,16 +472,18 @@ project_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant
                 for (int c = 0; c < C::CB; ++c) acc[a][c] = 0.f;
             do {
                 const uint32_t b = grp & 1u, use = grp >> 1;
-                bool got = true;
-                if (lane == 0) got = wait_bounded(smem_u32(&tfull[b]), use & 1u, abort, p.err);
-                got = __shfl_sync(0xffffffffu, got, 0);
-                if (epi_any(!got)) {
-                    ok = false;
-                    break;
+                if (u == 0) {
+                    bool got = true;
+                    if (lane == 0) got = wait_bounded(smem_u32(&tfull[b]), use & 1u, abort, p.err);
+                    got = __shfl_sync(0xffffffffu, got, 0);
+                    if (epi_any(!got)) {
+                        ok = false;
+                        break;
+                    }
+                    tc_fence_after();
                 }
-                tc_fence_after();
-                const uint32_t tbase = tmem + ((uint32_t)(q * 32) << 16) + b * C::kBufCols;
-                constexpr int kParts = kTileM / C::kStageRows, kWarpsPer = 4 / kParts;
+                const uint32_t tbase =
+                    tmem + ((uint32_t)(q * 32) << 16) + b * C::kBufCols + (uint32_t)u * C::kAccCols;
                 for (int h = 0; h < kParts; ++h) {
                     if (q / kWarpsPer == h) {
                         const int srow = (q % kWarpsPer) * 32 + lane;
@@ -484,12 +496,14 @@ project_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant
                             for (int i = 0; i < 16; i += 4)
                                 *reinterpret_cast<float4*>(dst + i) = make_float4(v[i], v[i + 1], v[i + 2], v[i + 3]);
                         }
-                        tc_fence_before();
-                        __syncwarp();
-                        if (lane == 0) mbar_arrive(smem_u32(&tempty[b]));
+                        if (u == ng - 1) {
+                            tc_fence_before();
+                            __syncwarp();
+                            if (lane == 0) mbar_arrive(smem_u32(&tempty[b]));
+                        }
                     }
                     epi_sync();
-#pragma unroll 1
+#pragma unroll(K > 64 ? 1 : 4)
                     for (int t = 0; t < C::kStageRows; ++t) {
                         float y[C::RB], x[C::CB];
 #pragma unroll
@@ -503,9 +517,12 @@ project_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant
                     }
                     epi_sync();
                 }
-                ++grp;
-                ng = it.take<G>(p, ncl, crank, gx, gt);
-            } while (ng > 0 && gx[0] == cur);
+                if (++u == ng) {
+                    ++grp;
+                    ng = it.take<G>(p, ncl, crank, gx, gt);
+                    u = 0;
+                }
+            } while (ng > 0 && gx[u] == cur);
             if (ok && !store_phi<C>(acc, cur, p, crank, stX, red_go, red_full, red_use, abort, et, lane)) ok = false;
         }
     } else if (warp >= 4) {
@@ -842,11 +859,12 @@ int sm_count() {
     return (b > 0 && b < sms) ? b : sms;
 }
 
-template <int K, int G, bool KF, bool FO, bool SL = false>
+template <int K, int G, bool KF, bool FO, bool SL = false, int SR = Cfg<K, G>::kStageRows>
 cudaError_t launch_kg(const tda_layer_desc& L, const void* A, const void* B, int64_t N, float* phi,
                       int64_t ld_phi, unsigned int* err, cudaStream_t s, int pack, float* cov, int* grid_out,
                       float* fout, const void* signs = nullptr) {
-    using C = Cfg<K, G>;
+    using C = Cfg<K, G, SR>;
+    if (C::kParted && pack > 1) return cudaErrorInvalidValue;  // packed tiles are staged whole
     CUtensorMap tmA, tmB, tmSA, tmSB;
     if constexpr (SL) {
         const uint16_t* tab = (const uint16_t*)signs;
@@ -881,7 +899,7 @@ cudaError_t launch_kg(const tda_layer_desc& L, const void* A, const void* B, int
     p.cov = cov;
     p.fout = fout;
     const int sms = sm_count();
-    cudaError_t e = cudaFuncSetAttribute(project_tc_kernel<K, G, KF, FO, SL>,
+    cudaError_t e = cudaFuncSetAttribute(project_tc_kernel<K, G, KF, FO, SL, SR>,
                                          cudaFuncAttributeMaxDynamicSharedMemorySize, (int)C::kSmem);
     if (e != cudaSuccess) return e;
     // Fewer examples than SMs: a cluster of cs CTAs shares each example's token
@@ -903,7 +921,7 @@ cudaError_t launch_kg(const tda_layer_desc& L, const void* A, const void* B, int
     cfg.numAttrs = 1;
     int max_clusters = 0;
     cfg.gridDim = dim3((unsigned)(cs * (sms / cs)));
-    if (cudaOccupancyMaxActiveClusters(&max_clusters, project_tc_kernel<K, G, KF, FO, SL>, &cfg) != cudaSuccess ||
+    if (cudaOccupancyMaxActiveClusters(&max_clusters, project_tc_kernel<K, G, KF, FO, SL, SR>, &cfg) != cudaSuccess ||
         max_clusters < 1)
         max_clusters = sms / cs;
     if (max_clusters > sms / cs) max_clusters = sms / cs;  // the SM budget (the occupancy query sees every SM)
@@ -912,7 +930,7 @@ cudaError_t launch_kg(const tda_layer_desc& L, const void* A, const void* B, int
     cfg.gridDim = dim3((unsigned)(clusters * cs));
     if (grid_out) *grid_out = (int)(clusters * cs);
     note_launches(1);
-    e = cudaLaunchKernelEx(&cfg, project_tc_kernel<K, G, KF, FO, SL>, tmA, tmB, tmSA, tmSB, p);
+    e = cudaLaunchKernelEx(&cfg, project_tc_kernel<K, G, KF, FO, SL, SR>, tmA, tmB, tmSA, tmSB, p);
     if (e != cudaSuccess) return e;
     return cudaGetLastError();
 }
@@ -947,15 +965,31 @@ cudaError_t launch_k(const tda_layer_desc& L, const void* A, const void* B, int6
             return cudaSuccess;
         }
     }
+    // At least one example per SM (no cluster shares an example): stage 32 token rows at a
+    // time, which leaves room for one or two more stages in the ring; fewer examples keep the
+    // larger staging rows, which also hold the cluster's partial blocks.
+    const bool narrow = pack == 1 && N >= (int64_t)sm_count();
     if constexpr (K > 64) {
-        if constexpr (!KF && !FO)
-            if (signs) return launch_kg<K, 1, false, false, true>(L, A, B, N, phi, ld_phi, err, s, pack, cov, grid_out,
-                                                                  fout, signs);
+        if constexpr (!KF && !FO) {
+            if (signs)
+                return narrow ? launch_kg<K, 1, false, false, true, 32>(L, A, B, N, phi, ld_phi, err, s, pack, cov,
+                                                                         grid_out, fout, signs)
+                              : launch_kg<K, 1, false, false, true>(L, A, B, N, phi, ld_phi, err, s, pack, cov,
+                                                                    grid_out, fout, signs);
+            if (narrow)
+                return launch_kg<K, 1, false, false, false, 32>(L, A, B, N, phi, ld_phi, err, s, pack, cov, grid_out,
+                                                                fout);
+        }
         return launch_kg<K, 1, KF, FO>(L, A, B, N, phi, ld_phi, err, s, pack, cov, grid_out, fout);
     } else {
         const int64_t units = pack > 1 ? (N + pack - 1) / pack : N * ((L.T + kTileM - 1) / kTileM);
-        if (units >= 4 * (int64_t)sm_count())
+        if (units >= 4 * (int64_t)sm_count()) {
+            if constexpr (!KF && !FO)
+                if (narrow)
+                    return launch_kg<K, 2, false, false, false, 32>(L, A, B, N, phi, ld_phi, err, s, pack, cov,
+                                                                    grid_out, fout);
             return launch_kg<K, 2, KF, FO>(L, A, B, N, phi, ld_phi, err, s, pack, cov, grid_out, fout);
+        }
         return launch_kg<K, 1, KF, FO>(L, A, B, N, phi, ld_phi, err, s, pack, cov, grid_out, fout);
     }
 }

@@ -373,6 +373,9 @@ TC_CASES = [
     # two token tiles per pipeline stage (many units): groups that straddle examples
     (250, 300, 64, 72, 32, "bf16"),
     (700, 256, 64, 128, 64, "bf16"),
+    # at least one example per SM: 32 token rows staged at a time, groups straddling examples
+    (300, 300, 200, 136, 64, "bf16"),
+    (160, 48, 64, 64, 128, "bf16"),
     # short sequences packed several examples to a tile, ragged last tile
     (2001, 48, 64, 64, 16, "bf16"),     # 2 per tile, 32 rows unused, one tile per stage pair
     (20001, 8, 64, 64, 16, "bf16"),     # 16 per tile
