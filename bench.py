@@ -972,6 +972,10 @@ def stack_main(args, spec):
                 hp.append(h)
             hpools.append(hp)
         wsb = 2 * Ph * T * max(di + do for _, di, do in lin) * 2
+        # room for the projection's own workspace beside each staging half (balanced tile ranges)
+        pws = max(tda.tda_workspace_size(tda.TDA_OP_PROJECT, Lr, tda.TDA_BF16, 1, 0, tda.TDA_ROUTE_FACTORED)
+                  for Lr in job.layers[:nshape])
+        wsb += 2 * ((pws + 255) // 256 * 256)
         job.host_ws_bytes = wsb
         job.host_ws = torch.empty(wsb, dtype=torch.uint8, device=dev)
 

@@ -133,6 +133,13 @@ tda_status tda_workspace_size(tda_op op, const tda_layer_desc* L, tda_dtype dtyp
  *          (tda_route's choice for TDA_OP_PROJECT).
  * Both routes give the same result up to rounding (App. A.4).
  * bf16 requires d_in % 8 == 0 and d_out % 8 == 0; fp32 requires % 4.
+ *   ws     MATERIALIZE: required (tda_workspace_size bytes per example in a
+ *          chunk). FACTORED on the tensor cores: optional, 256-byte aligned;
+ *          with tda_workspace_size bytes the kernel gives every SM an equal
+ *          run of 128-token tiles (an example split between SMs is summed in
+ *          a fixed order, so results do not depend on timing) and, for
+ *          k = 128, reads sign tables written once per call; without it each
+ *          SM takes whole examples. Calls that share a ws must not overlap.
  * ------------------------------------------------------------------------- */
 tda_status tda_project(const tda_layer_desc* L, tda_dtype dtype, const void* A, const void* B,
                        int64_t N, float* phi, int64_t ld_phi, tda_route_id route,
@@ -153,8 +160,10 @@ int32_t tda_project_engine(const tda_layer_desc* L, tda_dtype dtype, const void*
  * (cudaHostAlloc / cudaHostRegister) lets copies overlap compute; pageable
  * memory works but serialises. The host buffers must stay unchanged until
  * `stream` has completed. ws: >= tda_project_host_ws_min() bytes (one example
- * per half), 256-byte aligned; larger ws means larger chunks. Calls on one
- * device serialise their enqueueing on a library mutex.
+ * per half), 256-byte aligned; larger ws means larger chunks. With at least
+ * 2 x tda_workspace_size(TDA_OP_PROJECT, FACTORED) bytes beyond the minimum, the
+ * end of ws also serves as the projection's optional workspace (one per half).
+ * Calls on one device serialise their enqueueing on a library mutex.
  * ------------------------------------------------------------------------- */
 size_t tda_project_host_ws_min(const tda_layer_desc* L, tda_dtype dtype);
 tda_status tda_project_host(const tda_layer_desc* L, tda_dtype dtype, const void* A_h, const void* B_h,

@@ -268,8 +268,11 @@ tda_status tda_workspace_size(tda_op op, const tda_layer_desc* L, tda_dtype dtyp
     }
     if (op == TDA_OP_PROJECT) {
         if (route == TDA_ROUTE_MATERIALIZE) *bytes = materialize_ws_bytes_per_example(*L);
-        // optional for the factored route: k = 128 bf16 reads precomputed sign tiles from it
-        if (route == TDA_ROUTE_FACTORED && dtype == TDA_BF16) *bytes = project_tc_sign_table_bytes(*L);
+        // optional for the factored route on the tensor cores: balanced token-tile ranges
+        // (and for k = 128 precomputed sign tiles)
+        if (route == TDA_ROUTE_FACTORED && dtype == TDA_BF16 && L->k_in == L->k_out && L->kind == TDA_PROJ_RADEMACHER &&
+            (L->k_in == 16 || L->k_in == 32 || L->k_in == 64 || L->k_in == 128))
+            *bytes = project_tc_ws_bytes(*L);
         return TDA_OK;
     }
     if (op == TDA_OP_SIMILARITY_EXACT) {

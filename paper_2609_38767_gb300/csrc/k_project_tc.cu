@@ -48,6 +48,7 @@
 
 #include <cstring>
 #include <mutex>
+#include <type_traits>
 
 #include "tda_internal.cuh"
 
@@ -123,6 +124,13 @@ struct Params {
     int cs;           // CTAs per cluster sharing one example's token tiles (1, 2 or 4)
     float* cov;       // K-FAC: per-CTA partial sums of At^T At and Bt^T Bt ([grid][2][K*K])
     float* fout;      // factor output: At rows [N*T][K], then Bt rows [N*T][K] (unscaled signs)
+    // balanced ranges (BAL): CTA c owns token tiles [n_units*c/grid, n_units*(c+1)/grid) of the
+    // flattened (example, tile) sequence; an example split across CTAs leaves an unscaled partial
+    // block per CTA in part ([grid][2][K*K]: slot 0 = the CTA's first example, 1 = its last) and
+    // the last of them to finish (counter cnt[first CTA of the example]) sums them in CTA order
+    int64_t n_units;
+    float* part;
+    unsigned int* cnt;
 };
 
 #include "tc_ptx.cuh"
@@ -133,7 +141,7 @@ struct Params {
 struct Units {
     int64_t x;
     int tt;
-    __device__ __forceinline__ void first(uint32_t cid, uint32_t crank) {
+    __device__ __forceinline__ void first(const Params&, uint32_t cid, uint32_t crank) {
         x = cid;
         tt = (int)crank;
     }
@@ -152,6 +160,28 @@ struct Units {
                     tt = (int)crank;
                     x += ncl;
                 }
+            }
+        return n;
+    }
+};
+
+// Balanced ranges: the same contiguous run of token tiles for every warp role.
+struct TileRange {
+    int64_t t, t1;
+    __device__ __forceinline__ void first(const Params& p, uint32_t, uint32_t) {
+        t = p.n_units * (int64_t)blockIdx.x / gridDim.x;
+        t1 = p.n_units * ((int64_t)blockIdx.x + 1) / gridDim.x;
+    }
+    template <int G>
+    __device__ __forceinline__ int take(const Params& p, uint32_t, uint32_t, int64_t* gx, int* gt) {
+        int n = 0;
+#pragma unroll
+        for (int u = 0; u < G; ++u)
+            if (t < t1) {
+                gx[u] = t / p.n_ttiles;
+                gt[u] = (int)(t - gx[u] * p.n_ttiles);
+                ++t;
+                ++n;
             }
         return n;
     }
@@ -230,6 +260,67 @@ __device__ __forceinline__ bool store_phi(float (&acc)[C::RB][C::CB], int64_t n,
     return true;
 }
 
+// Balanced ranges: Phi of example n (K x K partial sums in acc, layout as in
+// store_phi) after this CTA's last tile of it. An example wholly inside the
+// CTA's range is written directly; otherwise the partial goes to the CTA's
+// slot in p.part, and the last of the example's CTAs to arrive at its counter
+// adds all partials in CTA order (the same sum whichever CTA finishes last),
+// scales, writes Phi and clears the counter. Nothing waits on another CTA.
+template <class C>
+__device__ __forceinline__ void store_phi_bal(float (&acc)[C::RB][C::CB], int64_t n, const Params& p, int et,
+                                              volatile int* flag) {
+    constexpr int K = C::kK;
+    const int rg = et >> 3, cg = et & 7;
+    const int64_t nt = p.n_ttiles, U = p.n_units, g = gridDim.x, c = blockIdx.x;
+    const int64_t u0 = n * nt, u1 = u0 + nt;               // the example's tiles
+    const int64_t r0 = U * c / g, r1 = U * (c + 1) / g;     // this CTA's tiles
+    float* out = p.phi + n * p.ld_phi;
+    if (u0 >= r0 && u1 <= r1) {
+#pragma unroll
+        for (int a = 0; a < C::RB; ++a)
+#pragma unroll
+            for (int b = 0; b < C::CB; ++b) out[(rg * C::RB + a) * K + cg * C::CB + b] = acc[a][b] * p.scale;
+        return;
+    }
+    float* mine = p.part + ((size_t)c * 2 + (n == r0 / nt ? 0 : 1)) * K * K;
+#pragma unroll
+    for (int a = 0; a < C::RB; ++a)
+#pragma unroll
+        for (int b = 0; b < C::CB; ++b) mine[(rg * C::RB + a) * K + cg * C::CB + b] = acc[a][b];
+    __threadfence();
+    epi_sync();
+    // CTAs holding the example's first and last tiles (every CTA's range is non-empty)
+    const int64_t cf = ((u0 + 1) * g - 1) / U, cl = (u1 * g - 1) / U;
+    if (et == 0) {
+        const unsigned int prev = atomicAdd(p.cnt + cf, 1u);
+        const bool last = prev == (unsigned int)(cl - cf);
+        if (last) p.cnt[cf] = 0u;  // ready for the next call
+        *flag = last ? 1 : 0;
+    }
+    epi_sync();
+    const bool last = *flag != 0;
+    epi_sync();  // every thread has read the flag before the next example may set it
+    if (!last) return;
+    __threadfence();
+    float sum[C::RB][C::CB];
+#pragma unroll
+    for (int a = 0; a < C::RB; ++a)
+#pragma unroll
+        for (int b = 0; b < C::CB; ++b) sum[a][b] = 0.f;
+    for (int64_t c2 = cf; c2 <= cl; ++c2) {
+        const int64_t first_ex = (U * c2 / g) / nt;
+        const float* part = p.part + ((size_t)c2 * 2 + (n == first_ex ? 0 : 1)) * K * K;
+#pragma unroll
+        for (int a = 0; a < C::RB; ++a)
+#pragma unroll
+            for (int b = 0; b < C::CB; ++b) sum[a][b] += __ldcg(part + (rg * C::RB + a) * K + cg * C::CB + b);
+    }
+#pragma unroll
+    for (int a = 0; a < C::RB; ++a)
+#pragma unroll
+        for (int b = 0; b < C::CB; ++b) out[(rg * C::RB + a) * K + cg * C::CB + b] = sum[a][b] * p.scale;
+}
+
 __device__ __forceinline__ uint4 lds128(uint32_t a) {
     uint4 v;
     asm volatile("ld.shared.v4.u32 {%0, %1, %2, %3}, [%4];" : "=r"(v.x), "=r"(v.y), "=r"(v.z), "=r"(v.w) : "r"(a));
@@ -264,13 +355,14 @@ __device__ __forceinline__ void store_sign_row(uint8_t* tile, int n, const uint4
 // factors At, Bt of every token instead of contracting them into Phi. SL: the
 // sign tiles come by TMA from a precomputed table (tmSA, tmSB: [K][d] bf16, a
 // side's S transposed) instead of the generator warps.
-template <int K, int G, bool KF, bool FO, bool SL = false, int SR = Cfg<K, G>::kStageRows>
+template <int K, int G, bool KF, bool FO, bool SL = false, int SR = Cfg<K, G>::kStageRows, bool BAL = false>
 __global__ void __launch_bounds__(kThreads, 1)
 project_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
                   const __grid_constant__ CUtensorMap tmSA, const __grid_constant__ CUtensorMap tmSB,
                   const Params p) {
     using C = Cfg<K, G, SR>;
     static_assert(!C::kParted || (!KF && !FO), "the K-FAC and factor-output epilogues stage whole tiles");
+    static_assert(!BAL || C::kParted, "balanced ranges use the parted epilogue");
     extern __shared__ uint8_t smem_raw[];
     uint8_t* smem = (uint8_t*)(((uintptr_t)smem_raw + 1023) & ~(uintptr_t)1023);
     uint8_t* sA = smem;                           // kStages x [G factor tiles | sign tile]
@@ -319,8 +411,8 @@ project_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant
     const int nk_tot = p.nk_in + p.nk_out;
     int64_t gx[G];
     int gt[G];
-    Units it;
-    it.first(cid, crank);
+    typename std::conditional<BAL, TileRange, Units>::type it;
+    it.first(p, cid, crank);
 
     if (warp == 0 && lane == 0) {
         // ---------------- TMA producer
@@ -523,7 +615,11 @@ project_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant
                     u = 0;
                 }
             } while (ng > 0 && gx[u] == cur);
-            if (ok && !store_phi<C>(acc, cur, p, crank, stX, red_go, red_full, red_use, abort, et, lane)) ok = false;
+            if constexpr (BAL) {
+                if (ok) store_phi_bal<C>(acc, cur, p, et, abort + 1);
+            } else if (ok && !store_phi<C>(acc, cur, p, crank, stX, red_go, red_full, red_use, abort, et, lane)) {
+                ok = false;
+            }
         }
     } else if (warp >= 4) {
         // ---------------- epilogue: TMEM -> shared -> Phi += Bt^T At
@@ -859,12 +955,13 @@ int sm_count() {
     return (b > 0 && b < sms) ? b : sms;
 }
 
-template <int K, int G, bool KF, bool FO, bool SL = false, int SR = Cfg<K, G>::kStageRows>
+template <int K, int G, bool KF, bool FO, bool SL = false, int SR = Cfg<K, G>::kStageRows, bool BAL = false>
 cudaError_t launch_kg(const tda_layer_desc& L, const void* A, const void* B, int64_t N, float* phi,
                       int64_t ld_phi, unsigned int* err, cudaStream_t s, int pack, float* cov, int* grid_out,
-                      float* fout, const void* signs = nullptr) {
+                      float* fout, const void* signs = nullptr, void* bal_ws = nullptr) {
     using C = Cfg<K, G, SR>;
     if (C::kParted && pack > 1) return cudaErrorInvalidValue;  // packed tiles are staged whole
+    if (BAL && !bal_ws) return cudaErrorInvalidValue;
     CUtensorMap tmA, tmB, tmSA, tmSB;
     if constexpr (SL) {
         const uint16_t* tab = (const uint16_t*)signs;
@@ -898,14 +995,17 @@ cudaError_t launch_kg(const tda_layer_desc& L, const void* A, const void* B, int
     p.nk_out = (int)((L.d_out + kChunkK - 1) / kChunkK);
     p.cov = cov;
     p.fout = fout;
+    p.n_units = p.n_slots * p.n_ttiles;
+    p.part = nullptr;
+    p.cnt = nullptr;
     const int sms = sm_count();
-    cudaError_t e = cudaFuncSetAttribute(project_tc_kernel<K, G, KF, FO, SL, SR>,
+    cudaError_t e = cudaFuncSetAttribute(project_tc_kernel<K, G, KF, FO, SL, SR, BAL>,
                                          cudaFuncAttributeMaxDynamicSharedMemorySize, (int)C::kSmem);
     if (e != cudaSuccess) return e;
     // Fewer examples than SMs: a cluster of cs CTAs shares each example's token
     // tiles and reduces the partial features through distributed shared memory.
     int cs = 1;
-    if (pack == 1 && N < sms && !FO) cs = (2 * N >= sms) ? 2 : 4;
+    if (!BAL && pack == 1 && N < sms && !FO) cs = (2 * N >= sms) ? 2 : 4;
     while (cs > 1 && (cs > p.n_ttiles || cs > C::kMaxCs)) cs >>= 1;
     p.cs = cs;
     cudaLaunchConfig_t cfg = {};
@@ -921,16 +1021,23 @@ cudaError_t launch_kg(const tda_layer_desc& L, const void* A, const void* B, int
     cfg.numAttrs = 1;
     int max_clusters = 0;
     cfg.gridDim = dim3((unsigned)(cs * (sms / cs)));
-    if (cudaOccupancyMaxActiveClusters(&max_clusters, project_tc_kernel<K, G, KF, FO, SL, SR>, &cfg) != cudaSuccess ||
+    if (cudaOccupancyMaxActiveClusters(&max_clusters, project_tc_kernel<K, G, KF, FO, SL, SR, BAL>, &cfg) != cudaSuccess ||
         max_clusters < 1)
         max_clusters = sms / cs;
     if (max_clusters > sms / cs) max_clusters = sms / cs;  // the SM budget (the occupancy query sees every SM)
-    int64_t clusters = FO ? p.n_slots * p.n_ttiles : p.n_slots;
+    int64_t clusters = (FO || BAL) ? p.n_units : p.n_slots;
     if (clusters > max_clusters) clusters = max_clusters;
     cfg.gridDim = dim3((unsigned)(clusters * cs));
     if (grid_out) *grid_out = (int)(clusters * cs);
+    if constexpr (BAL) {
+        // partial slots, then one counter per CTA (cleared here; each call leaves them clear)
+        p.part = (float*)bal_ws;
+        p.cnt = (unsigned int*)((char*)bal_ws + (size_t)2 * device_sms() * K * K * sizeof(float));
+        e = cudaMemsetAsync(p.cnt, 0, (size_t)clusters * sizeof(unsigned int), s);
+        if (e != cudaSuccess) return e;
+    }
     note_launches(1);
-    e = cudaLaunchKernelEx(&cfg, project_tc_kernel<K, G, KF, FO, SL, SR>, tmA, tmB, tmSA, tmSB, p);
+    e = cudaLaunchKernelEx(&cfg, project_tc_kernel<K, G, KF, FO, SL, SR, BAL>, tmA, tmB, tmSA, tmSB, p);
     if (e != cudaSuccess) return e;
     return cudaGetLastError();
 }
@@ -940,7 +1047,7 @@ cudaError_t launch_kg(const tda_layer_desc& L, const void* A, const void* B, int
 template <int K, bool KF, bool FO>
 cudaError_t launch_k(const tda_layer_desc& L, const void* A, const void* B, int64_t N, float* phi,
                      int64_t ld_phi, unsigned int* err, cudaStream_t s, float* cov, int* grid_out, float* fout,
-                     const void* signs = nullptr) {
+                     const void* signs = nullptr, void* bal_ws = nullptr) {
     // K = 128 keeps one example per tile (its epilogue contracts 64-row halves)
     int pack = (K <= 64 && L.T <= 64) ? (int)(kTileM / L.T) : 1;
     if (pack > 1) {
@@ -959,23 +1066,32 @@ cudaError_t launch_k(const tda_layer_desc& L, const void* A, const void* B, int6
                 const int64_t n = N - e0 < max_n ? N - e0 : max_n;
                 cudaError_t e = launch_k<K, KF, FO>(L, (const char*)A + e0 * a_ex, (const char*)B + e0 * b_ex, n,
                                                     phi + e0 * ld_phi, ld_phi, err, s, nullptr, nullptr, nullptr,
-                                                    signs);
+                                                    signs, bal_ws);
                 if (e != cudaSuccess) return e;
             }
             return cudaSuccess;
         }
     }
-    // At least one example per SM (no cluster shares an example): stage 32 token rows at a
-    // time, which leaves room for one or two more stages in the ring; fewer examples keep the
-    // larger staging rows, which also hold the cluster's partial blocks.
+    // With the balanced-range workspace (one example per tile): contiguous runs of token tiles
+    // per CTA, 32 token rows staged at a time (room for one or two more stages in the ring).
+    // Without it, at least one example per SM (no cluster shares an example) stages 32 rows as
+    // well; fewer examples keep the larger staging rows, which hold the cluster's partial blocks.
+    const bool bal = bal_ws && pack == 1;
     const bool narrow = pack == 1 && N >= (int64_t)sm_count();
     if constexpr (K > 64) {
         if constexpr (!KF && !FO) {
-            if (signs)
+            if (signs) {
+                if (bal)
+                    return launch_kg<K, 1, false, false, true, 32, true>(L, A, B, N, phi, ld_phi, err, s, pack, cov,
+                                                                         grid_out, fout, signs, bal_ws);
                 return narrow ? launch_kg<K, 1, false, false, true, 32>(L, A, B, N, phi, ld_phi, err, s, pack, cov,
                                                                          grid_out, fout, signs)
                               : launch_kg<K, 1, false, false, true>(L, A, B, N, phi, ld_phi, err, s, pack, cov,
                                                                     grid_out, fout, signs);
+            }
+            if (bal)
+                return launch_kg<K, 1, false, false, false, 32, true>(L, A, B, N, phi, ld_phi, err, s, pack, cov,
+                                                                      grid_out, fout, nullptr, bal_ws);
             if (narrow)
                 return launch_kg<K, 1, false, false, false, 32>(L, A, B, N, phi, ld_phi, err, s, pack, cov, grid_out,
                                                                 fout);
@@ -984,12 +1100,20 @@ cudaError_t launch_k(const tda_layer_desc& L, const void* A, const void* B, int6
     } else {
         const int64_t units = pack > 1 ? (N + pack - 1) / pack : N * ((L.T + kTileM - 1) / kTileM);
         if (units >= 4 * (int64_t)sm_count()) {
-            if constexpr (!KF && !FO)
+            if constexpr (!KF && !FO) {
+                if (bal)
+                    return launch_kg<K, 2, false, false, false, 32, true>(L, A, B, N, phi, ld_phi, err, s, pack, cov,
+                                                                          grid_out, fout, nullptr, bal_ws);
                 if (narrow)
                     return launch_kg<K, 2, false, false, false, 32>(L, A, B, N, phi, ld_phi, err, s, pack, cov,
                                                                     grid_out, fout);
+            }
             return launch_kg<K, 2, KF, FO>(L, A, B, N, phi, ld_phi, err, s, pack, cov, grid_out, fout);
         }
+        if constexpr (!KF && !FO)
+            if (bal)
+                return launch_kg<K, 1, false, false, false, 32, true>(L, A, B, N, phi, ld_phi, err, s, pack, cov,
+                                                                      grid_out, fout, nullptr, bal_ws);
         return launch_kg<K, 1, KF, FO>(L, A, B, N, phi, ld_phi, err, s, pack, cov, grid_out, fout);
     }
 }
@@ -1024,19 +1148,34 @@ size_t project_tc_sign_table_bytes(const tda_layer_desc& L) {
     return (size_t)L.k_in * (size_t)(L.d_in + L.d_out) * 2;
 }
 
+// Balanced token-tile ranges: two K x K partial blocks and one counter per SM.
+size_t project_tc_balance_bytes(const tda_layer_desc& L) {
+    const size_t sms = (size_t)device_sms();
+    return sms * (2 * (size_t)L.k_in * L.k_out * sizeof(float) + sizeof(unsigned int));
+}
+
+size_t project_tc_ws_bytes(const tda_layer_desc& L) {
+    return (project_tc_sign_table_bytes(L) + 255) / 256 * 256 + project_tc_balance_bytes(L);
+}
+
 cudaError_t launch_project_tc(const tda_layer_desc& L, const void* A, const void* B, int64_t N, float* phi,
                               int64_t ld_phi, unsigned int* err, cudaStream_t s, void* ws, size_t ws_bytes) {
     if (N == 0) return cudaSuccess;
+    // ws (256-byte aligned): [k = 128: both sides' sign tables, rounded up to 256 bytes]
+    // [balanced-range partials and counters]; either part is used when ws has room for it
+    if (ws && ((uintptr_t)ws & 255)) ws = nullptr;
+    const size_t sign_b = (project_tc_sign_table_bytes(L) + 255) / 256 * 256;
+    void* bal_ws = (ws && ws_bytes >= project_tc_ws_bytes(L)) ? (char*)ws + sign_b : nullptr;
     switch (L.k_in) {
-        case 16: return launch_k<16, false, false>(L, A, B, N, phi, ld_phi, err, s, nullptr, nullptr, nullptr);
-        case 32: return launch_k<32, false, false>(L, A, B, N, phi, ld_phi, err, s, nullptr, nullptr, nullptr);
-        case 64: return launch_k<64, false, false>(L, A, B, N, phi, ld_phi, err, s, nullptr, nullptr, nullptr);
+        case 16: return launch_k<16, false, false>(L, A, B, N, phi, ld_phi, err, s, nullptr, nullptr, nullptr, nullptr, bal_ws);
+        case 32: return launch_k<32, false, false>(L, A, B, N, phi, ld_phi, err, s, nullptr, nullptr, nullptr, nullptr, bal_ws);
+        case 64: return launch_k<64, false, false>(L, A, B, N, phi, ld_phi, err, s, nullptr, nullptr, nullptr, nullptr, bal_ws);
         case 128: {
             // with room in ws: both sides' sign tables once per call (L2-resident, read by TMA
             // beside the factor tiles) instead of sign tiles written by the generator warps
             const size_t need = project_tc_sign_table_bytes(L);
             const void* signs = nullptr;
-            if (ws && ws_bytes >= need && ((uintptr_t)ws & 255) == 0) {
+            if (ws && ws_bytes >= need) {
                 uint16_t* tab = (uint16_t*)ws;
                 const int64_t items = 128 * ((L.d_in + 63) / 64 + (L.d_out + 63) / 64);
                 const unsigned blocks = (unsigned)((items + 255) / 256 < 1216 ? (items + 255) / 256 : 1216);
@@ -1048,7 +1187,8 @@ cudaError_t launch_project_tc(const tda_layer_desc& L, const void* A, const void
                 if (e != cudaSuccess) return e;
                 signs = tab;
             }
-            return launch_k<128, false, false>(L, A, B, N, phi, ld_phi, err, s, nullptr, nullptr, nullptr, signs);
+            return launch_k<128, false, false>(L, A, B, N, phi, ld_phi, err, s, nullptr, nullptr, nullptr, signs,
+                                               bal_ws);
         }
         default: return cudaErrorNotSupported;
     }

@@ -78,7 +78,13 @@ extern "C" tda_status tda_project_host(const tda_layer_desc* L, tda_dtype dtype,
     std::lock_guard<std::mutex> lock(p->mu);
     const size_t el = dtype == TDA_F32 ? 4 : 2;
     const size_t a_ex = (size_t)L->T * L->d_in * el, b_ex = (size_t)L->T * L->d_out * el;
-    const size_t half = (ws_bytes / 2) & ~(size_t)255;
+    // Room beyond the minimum: the projection's own optional workspace, one per staging half
+    // (its uses are ordered by the same events as the half's), taken from the end of ws.
+    size_t pws = 0;
+    if (tda_workspace_size(TDA_OP_PROJECT, L, dtype, 1, 0, TDA_ROUTE_FACTORED, &pws) != TDA_OK) pws = 0;
+    pws = (pws + 255) & ~(size_t)255;
+    if (pws && ws_bytes < need + 2 * pws) pws = 0;
+    const size_t half = ((ws_bytes - 2 * pws) / 2) & ~(size_t)255;
     int64_t chunk = (int64_t)(half / (a_ex + b_ex));
     if (chunk > N) chunk = N;
     cudaStream_t s = (cudaStream_t)stream;
@@ -112,7 +118,8 @@ extern "C" tda_status tda_project_host(const tda_layer_desc* L, tda_dtype dtype,
             if ((st = cuda_check(cudaEventRecord(p->copied[b][i], p->copy[i]), "record copy"))) return st;
             if ((st = cuda_check(cudaStreamWaitEvent(s, p->copied[b][i], 0), "wait copy"))) return st;
         }
-        if ((st = tda_project(L, dtype, dA, dB, cnt, phi + c0 * ld_phi, ld_phi, TDA_ROUTE_FACTORED, nullptr, 0,
+        void* pw = pws ? (char*)ws + 2 * half + (size_t)b * pws : nullptr;
+        if ((st = tda_project(L, dtype, dA, dB, cnt, phi + c0 * ld_phi, ld_phi, TDA_ROUTE_FACTORED, pw, pws,
                               stream)))
             return st;
         if ((st = cuda_check(cudaEventRecord(p->done[b], s), "record done"))) return st;

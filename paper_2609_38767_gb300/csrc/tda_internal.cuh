@@ -115,8 +115,11 @@ bool materialize_tc_supported(const tda_layer_desc& L, tda_dtype dt, const void*
 cudaError_t launch_materialize_tc(const tda_layer_desc& L, const void* A, const void* B, int64_t e0, int64_t n,
                                   float* G, unsigned int* err, cudaStream_t s);
 // ws (optional, 256-byte aligned): for k = 128, >= project_tc_sign_table_bytes(L)
-// bytes let the kernel read precomputed sign tiles by TMA instead of generating them.
+// bytes let the kernel read precomputed sign tiles by TMA instead of generating them;
+// >= project_tc_ws_bytes(L) bytes also balance token tiles across the SMs (partial
+// blocks of examples split between CTAs after the sign tables).
 size_t project_tc_sign_table_bytes(const tda_layer_desc& L);
+size_t project_tc_ws_bytes(const tda_layer_desc& L);
 cudaError_t launch_project_tc(const tda_layer_desc& L, const void* A, const void* B, int64_t N,
                               float* phi, int64_t ld_phi, unsigned int* err, cudaStream_t s,
                               void* ws = nullptr, size_t ws_bytes = 0);

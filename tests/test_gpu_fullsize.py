@@ -247,9 +247,12 @@ def test_large_model_block_preconditioned_top100(dev, orc):
     stagewise(orc, pipe, info)
 
 
-@pytest.mark.parametrize("li,di,do", [(1, 12288, 1536), (4, 12288, 49152)])
-def test_large_model_layer_from_pinned_host(dev, orc, li, di, do):
-    # T = 2048, k = 128, A ~ Student-t(4), B ~ N(0, 1e-4); factors in pinned host memory
+@pytest.mark.parametrize("li,di,do,pws", [(1, 12288, 1536, False), (4, 12288, 49152, False),
+                                          (1, 12288, 1536, True)])
+def test_large_model_layer_from_pinned_host(dev, orc, li, di, do, pws):
+    # T = 2048, k = 128, A ~ Student-t(4), B ~ N(0, 1e-4); factors in pinned host memory.
+    # pws: room for the projection's own workspace beside the staging halves (sign tables,
+    # balanced token-tile ranges: 2 examples' 32 tiles over 32 SMs)
     T, k, n, sb = 2048, 128, 2, 0.01
     A = synth.factors(synth.SEED_A, li, n, T, di, 1.0, synth.DIST_STUDENT_T4, 0, "bf16")
     B = synth.factors(synth.SEED_B, li, n, T, do, sb, 0, 0, "bf16")
@@ -257,6 +260,9 @@ def test_large_model_layer_from_pinned_host(dev, orc, li, di, do):
     Bh = torch.from_numpy(B.view(np.int16)).view(torch.bfloat16).pin_memory()
     L = tda.LayerDesc(di, do, T, k, k, seed=0, layer=li)
     wsb = 2 * tda.tda_project_host_ws_min(L, tda.TDA_BF16)
+    if pws:
+        p = tda.tda_workspace_size(tda.TDA_OP_PROJECT, L, tda.TDA_BF16, n, 0, tda.TDA_ROUTE_FACTORED)
+        wsb += 2 * ((p + 255) // 256 * 256)
     ws = torch.empty(wsb, dtype=torch.uint8, device=dev)
     phi = torch.empty((n, k * k), device=dev)
     tda.tda_project_host(L, tda.TDA_BF16, Ah, Bh, n, phi, k * k, ws, wsb)

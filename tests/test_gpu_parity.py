@@ -57,9 +57,12 @@ def gpu_project(L, dtype, A, B, N, route, device, ld=None, sign_ws=False):
     if route == tda.TDA_ROUTE_MATERIALIZE:
         wsb = tda.tda_workspace_size(tda.TDA_OP_PROJECT, L, TD[dtype], N, 0, route) * min(N, 3)
         ws = torch.empty(wsb, dtype=torch.uint8, device=device)
-    elif sign_ws:  # the optional workspace of the factored route (k = 128: precomputed sign tables)
+    elif sign_ws:  # the optional workspace of the factored route
         wsb = tda.tda_workspace_size(tda.TDA_OP_PROJECT, L, TD[dtype], N, 0, route)
-        assert wsb == 2 * L.k_in * (L.d_in + L.d_out)
+        signs = 2 * L.k_in * (L.d_in + L.d_out) if L.k_in == 128 else 0
+        assert wsb >= (signs + 255) // 256 * 256 + 2 * L.k_in * L.k_out * 4
+        if sign_ws == "signs":  # room for the k = 128 sign tables only: whole examples per SM
+            wsb = signs
         ws = torch.full((wsb,), 0x7F, dtype=torch.uint8, device=device)
     tda.tda_project(L, TD[dtype], A, B, N, phi, ld, route, ws, wsb)
     tda.tda_device_status()
@@ -335,7 +338,7 @@ def test_route_auto_and_calibration(dev, orc):
 
 
 # ------------------------------------------------------------------ tensor-core projection specifics
-@pytest.mark.parametrize("k,sign_ws", [(32, False), (128, False), (128, True)])
+@pytest.mark.parametrize("k,sign_ws", [(32, False), (32, True), (128, False), (128, "signs"), (128, True)])
 def test_tc_projection_signs_bit_exact(dev, orc, k, sign_ws):
     # One-hot factors: A_n = I (T = d_in tokens), B_n = e_r at token t only, so
     # Phi_n / scale = outer(S_out[r, :], S_in[t, :]) exactly -- the signs the
@@ -398,25 +401,65 @@ def test_tc_projection_k128_sign_tables_match_oracle(dev, orc, case):
     A, B = make_factors(N, T, di, do, dtype, stream=12, sigma_b=0.03, mask_p=0.01)
     L = tda.LayerDesc(di, do, T, k, k, seed=6, layer=4)
     Ad, Bd = to_dev(A, dtype, dev), to_dev(B, dtype, dev)
-    got, _ = gpu_project(L, dtype, Ad, Bd, N, tda.TDA_ROUTE_FACTORED, dev, sign_ws=True)
+    got, _ = gpu_project(L, dtype, Ad, Bd, N, tda.TDA_ROUTE_FACTORED, dev, sign_ws="signs")
     plain, _ = gpu_project(L, dtype, Ad, Bd, N, tda.TDA_ROUTE_FACTORED, dev)
     np.testing.assert_array_equal(got, plain)  # same signs, same arithmetic order
     ref = orc.project(synth.to_f64(A, dtype), synth.to_f64(B, dtype), k, k, 6, 4)
     assert max(rel_fro(got[n], ref[n]) for n in range(N)) <= TOL[dtype]
+    # the whole workspace: sign tables and balanced token-tile ranges
+    bal, _ = gpu_project(L, dtype, Ad, Bd, N, tda.TDA_ROUTE_FACTORED, dev, sign_ws=True)
+    assert max(rel_fro(bal[n], ref[n]) for n in range(N)) <= TOL[dtype]
 
 
+@pytest.mark.parametrize("ws", [False, True])
 @pytest.mark.parametrize("case", TC_CASES)
-def test_tc_projection_matches_oracle(dev, orc, case):
+def test_tc_projection_matches_oracle(dev, orc, case, ws):
+    # ws: with the optional workspace every SM takes an equal run of token tiles (examples split
+    # between SMs are summed from partial blocks); without it, whole examples or clusters
     N, T, di, do, k, dtype = case
     A, B = make_factors(N, T, di, do, dtype, stream=11, sigma_b=0.03, mask_p=0.01)
     L = tda.LayerDesc(di, do, T, k, k, seed=5, layer=3)
     Ad, Bd = to_dev(A, dtype, dev), to_dev(B, dtype, dev)
     assert tda.tda_project_engine(L, TD[dtype], Ad, Bd) == 1  # the tensor-core kernel runs
-    got, _ = gpu_project(L, dtype, Ad, Bd, N, tda.TDA_ROUTE_FACTORED, dev)
+    got, _ = gpu_project(L, dtype, Ad, Bd, N, tda.TDA_ROUTE_FACTORED, dev, sign_ws=ws)
     ref = orc.project(synth.to_f64(A, dtype), synth.to_f64(B, dtype), k, k, 5, 3)
     assert rel_fro(got, ref) <= TOL[dtype]
     worst = max(rel_fro(got[n], ref[n]) for n in range(N))
     assert worst <= TOL[dtype], worst
+
+
+BAL_CASES = [
+    # (N, T, d_in, d_out, k): examples split over several SMs, few examples, one tile per example
+    (1, 2048, 128, 64, 128),    # one example over 16 SMs
+    (5, 2048, 136, 200, 64),    # 80 tiles: some SMs idle (grid = tiles)
+    (16, 2048, 256, 128, 128),  # 256 tiles over every SM, split examples at most boundaries
+    (153, 1024, 64, 72, 32),    # 1224 tiles: ranges of 8 or 9 tiles, G = 2 groups across examples
+    (200, 100, 64, 64, 16),     # one tile per example: nothing split
+    (7, 300, 64, 64, 64),       # 21 tiles, ragged last tile of every example
+]
+
+
+@pytest.mark.parametrize("case", BAL_CASES)
+def test_tc_projection_balanced_ranges(dev, orc, case):
+    # Balanced ranges are deterministic (the split examples' partial blocks are added in SM
+    # order whichever SM finishes last) and leave the workspace's counters clear: a second call
+    # on the same workspace reproduces the first bit for bit; both match the oracle.
+    N, T, di, do, k = case
+    A, B = make_factors(N, T, di, do, "bf16", stream=13, sigma_b=0.03, mask_p=0.01)
+    L = tda.LayerDesc(di, do, T, k, k, seed=8, layer=2)
+    Ad, Bd = to_dev(A, "bf16", dev), to_dev(B, "bf16", dev)
+    wsb = tda.tda_workspace_size(tda.TDA_OP_PROJECT, L, tda.TDA_BF16, N, 0, tda.TDA_ROUTE_FACTORED)
+    ws = torch.full((wsb,), 0x5A, dtype=torch.uint8, device=dev)
+    outs = []
+    for _ in range(2):
+        phi = torch.full((N, k * k), float("nan"), device=dev)
+        tda.tda_project(L, tda.TDA_BF16, Ad, Bd, N, phi, k * k, tda.TDA_ROUTE_FACTORED, ws, wsb)
+        tda.tda_device_status()
+        outs.append(phi.cpu().numpy().reshape(N, k, k))
+    np.testing.assert_array_equal(outs[0], outs[1])
+    ref = orc.project(synth.to_f64(A, "bf16"), synth.to_f64(B, "bf16"), k, k, 8, 2)
+    worst = max(rel_fro(outs[0][n], ref[n]) for n in range(N))
+    assert worst <= TOL["bf16"], worst
 
 
 @pytest.mark.parametrize("sdt,D,lam_abs,lam_rel,tol", [(tda.TDA_F64, 70, 1e-3, 0.0, 1e-9),
