@@ -52,15 +52,17 @@ LINEARS = [("q", 2048, 2048), ("k", 2048, 2048), ("v", 2048, 2048), ("o", 2048, 
            ("gate", 2048, 8192), ("up", 2048, 8192), ("down", 8192, 2048)]
 METRIC = "train examples attributed/sec (project+score)"
 
-# DRAM traffic of the tensor-core projection kernel, from one ncu capture
-# (dram__bytes_read.sum + dram__bytes_write.sum) of 608 examples of the 2048x2048
-# linear (profiles/tc_projection_q608.md): measured bytes over algorithmic bytes.
-# Launches of other linears are scaled by their algorithmic bytes (traffic is
-# one read of every factor byte, so it grows in proportion). Valid only for the
-# kernel source it was measured on (the kernel file and its PTX helper header);
-# any change makes the bench report null.
-TRAFFIC_RATIO = 1.0009831
-TRAFFIC_KERNEL_SHA256 = "ccf2d47e90fde7485863190648a37305d4e282e45265a58eb2d4ce2ffda0757e"
+# DRAM traffic of the tensor-core projection kernel, from one ncu capture per k
+# (dram__bytes_read.sum + dram__bytes_write.sum over the algorithmic bytes of the
+# launch): k = 64, 160 examples of the 4096x4096 linear at T = 1024
+# (profiles/tc_projection_k64_llama3_q160.md); k = 128, 32 examples of the
+# 12288 -> 1536 linear at T = 2048 (profiles/tc_projection_k128_large_k32.md).
+# Launches of other linears are scaled by their algorithmic bytes (every factor
+# byte is read once, so traffic grows in proportion). Valid only for the kernel
+# source it was measured on (the kernel file and its PTX helper header); any
+# change makes the bench report null.
+TRAFFIC_RATIO = {64: 1.0030041, 128: 1.0161786}
+TRAFFIC_KERNEL_SHA256 = "5e334442b0a93a40d94f1506bb2bc1776c1cb6a7702f4eb0eaf8e7beef7d17a7"
 
 
 def projection_kernel_sha256():
@@ -95,7 +97,8 @@ def parse_args():
     p.add_argument("--query-side-stream", type=int, default=1,
                    help="stack workloads: 1 = the query side and top-k on a stream of their own beside the "
                         "next chunks' projections, 0 = in line after each chunk")
-    p.add_argument("--query-priority", type=int, default=0, help="priority of that stream (lower = higher)")
+    p.add_argument("--query-priority", type=int, default=None,
+                   help="priority of that stream (lower = higher; default: the workload's)")
     p.add_argument("--query-streams", type=int, default=8,
                    help="streams the query projections of the linears are spread over (device-resident leg)")
     p.add_argument("--e2e-steps", type=int, default=2)
@@ -117,8 +120,13 @@ def parse_args():
                    help="stack workloads: time only one share's Fisher fit and factorisation with query solves "
                         "(one layer's linears, --profile-n train features) (kernel profiling)")
     p.add_argument("--profile-n", type=int, default=64)
+    p.add_argument("--profile-linears", type=int, default=0,
+                   help="--profile-precond: linears per call (0 = every linear of a layer)")
     p.add_argument("--sm-budget", type=int, default=0,
                    help="cap the persistent projection grid at this many CTAs (tda_set_sm_budget; 0 = every SM)")
+    p.add_argument("--balance", type=int, default=-1,
+                   help="stack workloads: 1 = balanced token-tile ranges in the train projections, 0 = whole "
+                        "examples per SM, -1 = the workload's default")
     p.add_argument("--nvtx", action="store_true",
                    help="stack workloads: push an NVTX range 'timed' around the timed steps (for ncu --nvtx)")
     p.add_argument("--route-sweep", action="store_true",
@@ -596,7 +604,7 @@ STACKS = {
                   ("gate", 4096, 14336), ("up", 4096, 14336), ("down", 14336, 4096)],
         "n_layers": 32, "T": 1024, "k": 64, "n_train": 8192, "chunk": 256, "n_query": 256,
         "dist_a": 0, "sigma_b": math.sqrt(1e-3), "lambda_rel": 1e-2,
-        "train_pool": 512, "query_pool": 256, "host_pool": 128,
+        "train_pool": 512, "query_pool": 256, "host_pool": 128, "balance": False, "query_priority": 0,
         "factors": "A~N(0,1), B~N(0,1e-3) (seeded synthetic)",
     },
     "large_model": {
@@ -604,7 +612,7 @@ STACKS = {
                   ("gate", 12288, 49152), ("up", 12288, 49152), ("down", 49152, 12288)],
         "n_layers": 1, "T": 2048, "k": 128, "n_train": 16384, "chunk": 512, "n_query": 512,
         "dist_a": 1, "sigma_b": 0.01, "lambda_rel": 1e-2,
-        "train_pool": 128, "query_pool": 64, "host_pool": 16,
+        "train_pool": 128, "query_pool": 64, "host_pool": 16, "balance": True, "query_priority": -1,
         "factors": "A~Student-t(4), B~N(0,1e-4) (seeded synthetic)",
     },
 }
@@ -630,6 +638,9 @@ def stack_config(args, spec):
                            "HBM; each (chunk, layer) reads its own window of the train pool"),
         "l2": "inputs larger than L2 (no flush)",
         "parallelism": "one GPU", "routes": "factored (every linear)",
+        "train_schedule": ("balanced token-tile ranges per launch"
+                           if (spec["balance"] if args.balance < 0 else bool(args.balance))
+                           else "whole examples per SM") + f", {args.train_streams} train streams",
     }
 
 
@@ -758,7 +769,7 @@ def stack_profile_main(args, spec):
         what = {"kernel": "factored projection", "linear": [di, do], "n": n, "T": T, "k": k,
                 "sign_tables": bool(wsb)}
     else:
-        nl = len(spec["layer"])
+        nl = args.profile_linears or len(spec["layer"])
         per = tda.tda_precondition_state_bytes(D, tda.TDA_F32)
         st = torch.empty(nl * per, dtype=torch.uint8, device=dev)
         phi = torch.empty(n * nl * D, dtype=torch.float32, device=dev)
@@ -774,7 +785,7 @@ def stack_profile_main(args, spec):
             tda.tda_precondition(tda.TDA_PC_FACTOR_APPLY, nl, D, tda.TDA_F32, st, n_total=n,
                                  lambda_rel_mean_eig=spec["lambda_rel"], q=q, n_q=Nq, ld_q=nl * D, qhat=qh,
                                  ld_qhat=nl * D)
-        work = ("TFLOP/s", nl * (n * D * (D + 1) + 2 * (D ** 3 / 3 + 2 * D * D * Nq)) / 1e12)
+        work = ("TFLOP/s", nl * (n * D * (D + 1) + D ** 3 / 3 + 2 * D * D * Nq) / 1e12)
         what = {"kernel": "Fisher fit + factorisation + query solves", "linears": nl, "D": D, "n_train": n,
                 "n_query": Nq}
     for _ in range(max(args.warmup, 1)):
@@ -849,9 +860,11 @@ def stack_main(args, spec):
             return [(A[:min(Pt, chunk - r)], B[:min(Pt, chunk - r)], r, min(Pt, chunk - r)) for r in range(0, chunk, Pt)]
         return [(Aq[:min(Pq, Nq - r)], Bq[:min(Pq, Nq - r)], r, min(Pq, Nq - r)) for r in range(0, Nq, Pq)]
 
+    balance = spec["balance"] if args.balance < 0 else bool(args.balance)
     job = StackJob(linears, T, k, N, chunk, Nq, topk=args.topk, lambda_rel=spec["lambda_rel"], device=dev,
                    train_streams=args.train_streams, query_stream=bool(args.query_side_stream),
-                   query_priority=args.query_priority)
+                   query_priority=spec["query_priority"] if args.query_priority is None else args.query_priority,
+                   balance=balance)
     for si in range(nshape):  # every linear shape runs on the tensor-core projection kernel
         assert tda.tda_project_engine(job.layers[si], tda.TDA_BF16, pools[si][0], pools[si][1]) == 1
     state = {"j": 0, "s": 0}
@@ -940,14 +953,16 @@ def stack_main(args, spec):
                            f"{args.train_streams} stream(s)), CUDA events"),
                 "peak_source": "MEASURED_PEAKS.json hbm_gbs" if peaks else "fallback 6.8 TB/s",
                 "share_of_step": ph_train / (ms * steps)}
-    if k == 64 and projection_kernel_sha256() == TRAFFIC_KERNEL_SHA256:
-        roofline["traffic"] = TRAFFIC_RATIO * per_launch
+    if k in TRAFFIC_RATIO and projection_kernel_sha256() == TRAFFIC_KERNEL_SHA256:
+        roofline["traffic"] = TRAFFIC_RATIO[k] * per_launch
+        roofline["traffic_source"] = f"ncu dram bytes / algorithmic bytes of one k = {k} launch, scaled per launch"
     Dn = float(D)
     per_job_lin = {
         "project_train": ("hbm", sum(N * (T * (di + do) * 2 + 4 * D) for di, do in linears), hbm, "GB/s"),
         "fisher_fit": ("tensor", nlin * N * Dn * (Dn + 1), tf32x3, "TFLOP/s"),
         "project_query": ("hbm", sum(Nq * (T * (di + do) * 2 + 4 * D) for di, do in linears), hbm, "GB/s"),
-        "factor_apply": ("tensor", nlin * 2 * (Dn ** 3 / 3 + 2 * Dn * Dn * Nq), tf32x3, "TFLOP/s"),
+        # Cholesky D^3/3 flops, the two triangular solves 2 D^2 flops per query
+        "factor_apply": ("tensor", nlin * (Dn ** 3 / 3 + 2 * Dn * Dn * Nq), tf32x3, "TFLOP/s"),
         "score": ("tensor", 2.0 * Nq * N * D * nlin, tf32x3, "TFLOP/s"),
         "topk": ("latency", 4.0 * Nq * N, hbm, "GB/s"),
     }
@@ -1209,7 +1224,8 @@ def main():
     roofline = {"bound": "hbm", "kernel": "factored projection (train, 7 linears)",
                 "engine": "tcgen05" if engines == [1] else ("cuda-core" if engines == [0] else "mixed"), "achieved": achieved,
                 "peak": hbm, "unit": "GB/s", "frac": achieved / hbm,
-                "traffic": TRAFFIC_RATIO * per_launch if (same_kernel and engines == [1] and not kfac_mode) else None,
+                "traffic": (TRAFFIC_RATIO[k] * per_launch
+                            if (same_kernel and engines == [1] and not kfac_mode and k in TRAFFIC_RATIO) else None),
                 "algorithmic_bytes_per_launch": per_launch,
                 "peak_source": "MEASURED_PEAKS.json hbm_gbs" if peaks else "fallback 6.8 TB/s",
                 "share_of_step": proj_ms / (ms * args.steps)}
@@ -1230,7 +1246,7 @@ def main():
         "fisher_fit": ("tensor", nl * N * Dn * (Dn + 1), tf32x3, "TFLOP/s"),
         "factor": ("latency", nl * Dn ** 3 / 3, alu, "TFLOP/s"),
         "apply": ("latency", (nl * 4 * 2 * Dn * k * Nq) if kfac_mode else (nl * 2 * 2 * Dn * Dn * Nq), alu, "TFLOP/s"),
-        "factor_apply": ("latency", nl * (Dn ** 3 / 3 + 2 * 2 * Dn * Dn * Nq), alu, "TFLOP/s"),
+        "factor_apply": ("latency", nl * (Dn ** 3 / 3 + 2 * Dn * Dn * Nq), alu, "TFLOP/s"),
         "kfac_eigen": ("latency", nl * 2 * 10 * 4.0 * k ** 3, alu, "TFLOP/s"),
         "ekfac_eigenvalues": ("alu", nl * N * 2 * 2 * Dn * k, alu, "TFLOP/s"),
         "score": ("tensor", 2.0 * Nq * N * DT, tf32x3, "TFLOP/s"),

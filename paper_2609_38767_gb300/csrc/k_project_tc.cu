@@ -67,7 +67,9 @@ constexpr int kMaxStages = 12;
 // flight per SM, which is what an HBM-bound stream needs; a whole tile (128)
 // is staged where the epilogue needs every row at once (packed short
 // sequences, the K-FAC covariances, the factor output).
-template <int K, int G, int SR = (K > 64 ? kTileM / 2 : kTileM)>
+// LUT: shared memory for the sign-expansion table (K = 128 with generator warps;
+// sign tiles that arrive by TMA need none, which leaves room for one more stage).
+template <int K, int G, int SR = (K > 64 ? kTileM / 2 : kTileM), bool LUT = (K > 64)>
 struct Cfg {
     static constexpr int kK = K;
     static constexpr uint32_t kSignBytes = K * 128;                       // K rows x 128 bytes
@@ -92,14 +94,15 @@ struct Cfg {
     static constexpr int kMaxCs = (int)(2 * kStageRows * kStageLd / (K * K)) + 1;
     static constexpr size_t kSmemBarsMax = 8 * (3 * kMaxStages + 7) + 16;
     // K = 128: a 256-entry table expands a byte of sign bits into eight bf16 signs
-    static constexpr size_t kLutBytes = kHalf ? 256 * 16 : 0;
-    static constexpr size_t kLutMax = kHalf ? kLutBytes + 8 : 0;
+    static constexpr bool kLut = LUT;
+    static constexpr size_t kLutBytes = kLut ? 256 * 16 : 0;
+    static constexpr size_t kLutMax = kLut ? kLutBytes + 8 : 0;
     static constexpr int kFit = (int)((kSmemMax - 1024 - kSmemStage - kSmemBarsMax - kLutMax) / kStageBytes);
     static constexpr int kStages = kFit > kMaxStages ? kMaxStages : kFit;
     static constexpr size_t kSmemBars = 8 * (3 * kStages + 7) + 16;
     static constexpr size_t kBarsOff = (size_t)kStages * kStageBytes + kSmemStage;  // after ring and staging
     static constexpr size_t kLutOff = (kBarsOff + kSmemBars + 15) / 16 * 16;
-    static constexpr size_t kSmem = 1024 + (kHalf ? kLutOff + kLutBytes : kBarsOff + kSmemBars);
+    static constexpr size_t kSmem = 1024 + (kLut ? kLutOff + kLutBytes : kBarsOff + kSmemBars);
     // contraction blocking: 16 row groups x 8 column groups of threads
     static constexpr int RB = K / 16 > 0 ? K / 16 : 1;
     static constexpr int CB = K / 8;
@@ -360,7 +363,7 @@ __global__ void __launch_bounds__(kThreads, 1)
 project_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
                   const __grid_constant__ CUtensorMap tmSA, const __grid_constant__ CUtensorMap tmSB,
                   const Params p) {
-    using C = Cfg<K, G, SR>;
+    using C = Cfg<K, G, SR, (K > 64) && !SL>;
     static_assert(!C::kParted || (!KF && !FO), "the K-FAC and factor-output epilogues stage whole tiles");
     static_assert(!BAL || C::kParted, "balanced ranges use the parted epilogue");
     extern __shared__ uint8_t smem_raw[];
@@ -397,7 +400,7 @@ project_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant
         *abort = 0;
         fence_mbar_init();
     }
-    if constexpr (C::kHalf) init_sign_lut(smem + C::kLutOff, threadIdx.x);  // kThreads == 256 entries
+    if constexpr (C::kLut) init_sign_lut(smem + C::kLutOff, threadIdx.x);  // kThreads == 256 entries
     if (warp == 1) {
         tmem_alloc(smem_u32(tmem_slot), C::kTmemCols);
         tmem_relinquish();
@@ -515,8 +518,8 @@ project_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant
                 // col0 and col0 + 32 per lane); their sign words and table expansion do not
                 // depend on the stage's memory, so they are formed before the wait below
                 const int col0 = (warp - 2) * (K / 2) + lane;
-                uint4 q[C::kHalf ? 2 : 1][8];
-                if constexpr (C::kHalf) {
+                uint4 q[C::kLut ? 2 : 1][8];
+                if constexpr (C::kLut) {
                     const uint32_t lut = smem_u32(smem + C::kLutOff);
 #pragma unroll
                     for (int j = 0; j < 2; ++j) expand_signs(q[j], sign_word(key, (uint32_t)(col0 + 32 * j), rb), lut);
@@ -530,7 +533,7 @@ project_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant
                     break;
                 }
                 uint8_t* tile = sA + (size_t)s * C::kStageBytes + (size_t)G * kTileBytes;
-                if constexpr (C::kHalf) {
+                if constexpr (C::kLut) {
 #pragma unroll
                     for (int j = 0; j < 2; ++j) store_sign_row(tile, col0 + 32 * j, q[j]);
                 } else {
@@ -959,7 +962,7 @@ template <int K, int G, bool KF, bool FO, bool SL = false, int SR = Cfg<K, G>::k
 cudaError_t launch_kg(const tda_layer_desc& L, const void* A, const void* B, int64_t N, float* phi,
                       int64_t ld_phi, unsigned int* err, cudaStream_t s, int pack, float* cov, int* grid_out,
                       float* fout, const void* signs = nullptr, void* bal_ws = nullptr) {
-    using C = Cfg<K, G, SR>;
+    using C = Cfg<K, G, SR, (K > 64) && !SL>;
     if (C::kParted && pack > 1) return cudaErrorInvalidValue;  // packed tiles are staged whole
     if (BAL && !bal_ws) return cudaErrorInvalidValue;
     CUtensorMap tmA, tmB, tmSA, tmSB;

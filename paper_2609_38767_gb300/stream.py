@@ -35,13 +35,15 @@ import paper_2609_38767_gb300 as tda
 class StackJob:
     def __init__(self, linears, T, k, n_train, chunk, n_query, *, topk=100, lambda_rel=1e-2, lambda_abs=0.0,
                  seed=0, device="cuda", host_ws_bytes=0, train_streams=1, proj_ws=True, query_stream=False,
-                 query_priority=0):
+                 query_priority=0, balance=True):
         """linears: [(d_in, d_out)] of the whole stack, in layer order (linear i uses projection
         layer id i). n_train must be a multiple of chunk. train_streams > 1 spreads the train
         projections of a chunk round-robin over that many streams, so that a launch's CTAs fill
         the SMs its predecessor's last tiles leave idle (every launch writes its own feature
         columns: the results do not depend on the order). proj_ws: give the factored projection
-        its optional workspace (k = 128: precomputed sign tables). query_stream: run the query
+        its optional workspace (k = 128: precomputed sign tables). balance: let it use that
+        workspace for balanced token-tile ranges too (otherwise every SM takes whole examples,
+        whose staggered ends the next launch on another stream fills). query_stream: run the query
         side and the top-k on a stream of their own (priority query_priority), beside the
         next chunks' projections; events order the two job-boundary dependencies (a job's
         query side starts after its last chunk is projected; a job's features are overwritten
@@ -71,6 +73,8 @@ class StackJob:
         # one workspace per stream (a call writes its sign tables into it)
         self.proj_wsb = max(tda.tda_workspace_size(tda.TDA_OP_PROJECT, L, tda.TDA_BF16, chunk, 0,
                                                    tda.TDA_ROUTE_FACTORED) for L in self.layers) if proj_ws else 0
+        if proj_ws and not balance:  # room for the k = 128 sign tables only
+            self.proj_wsb = 2 * k * max(di + do for di, do in linears) if k == 128 else 0
         self.proj_ws = [torch.empty(self.proj_wsb, dtype=torch.uint8, device=dev)
                         for _ in range(self.train_streams + 1)] if self.proj_wsb else None
         self.side = torch.cuda.Stream(device=dev, priority=query_priority) if query_stream else None
