@@ -122,8 +122,9 @@ def parse_args():
     p.add_argument("--profile-n", type=int, default=64)
     p.add_argument("--profile-linears", type=int, default=0,
                    help="--profile-precond: linears per call (0 = every linear of a layer)")
-    p.add_argument("--sm-budget", type=int, default=0,
-                   help="cap the persistent projection grid at this many CTAs (tda_set_sm_budget; 0 = every SM)")
+    p.add_argument("--sm-budget", type=int, default=None,
+                   help="cap the persistent projection grid at this many CTAs (tda_set_sm_budget; 0 = every SM; "
+                        "default: the workload's)")
     p.add_argument("--balance", type=int, default=-1,
                    help="stack workloads: 1 = balanced token-tile ranges in the train projections, 0 = whole "
                         "examples per SM, -1 = the workload's default")
@@ -604,7 +605,7 @@ STACKS = {
                   ("gate", 4096, 14336), ("up", 4096, 14336), ("down", 14336, 4096)],
         "n_layers": 32, "T": 1024, "k": 64, "n_train": 8192, "chunk": 256, "n_query": 256,
         "dist_a": 0, "sigma_b": math.sqrt(1e-3), "lambda_rel": 1e-2,
-        "train_pool": 512, "query_pool": 256, "host_pool": 128, "balance": False, "query_priority": 0,
+        "train_pool": 512, "query_pool": 256, "host_pool": 128, "balance": False, "query_priority": 0, "sm_budget": 0,
         "factors": "A~N(0,1), B~N(0,1e-3) (seeded synthetic)",
     },
     "large_model": {
@@ -612,7 +613,7 @@ STACKS = {
                   ("gate", 12288, 49152), ("up", 12288, 49152), ("down", 49152, 12288)],
         "n_layers": 1, "T": 2048, "k": 128, "n_train": 16384, "chunk": 512, "n_query": 512,
         "dist_a": 1, "sigma_b": 0.01, "lambda_rel": 1e-2,
-        "train_pool": 128, "query_pool": 64, "host_pool": 16, "balance": True, "query_priority": -1,
+        "train_pool": 128, "query_pool": 64, "host_pool": 16, "balance": True, "query_priority": -1, "sm_budget": 128,
         "factors": "A~Student-t(4), B~N(0,1e-4) (seeded synthetic)",
     },
 }
@@ -640,7 +641,9 @@ def stack_config(args, spec):
         "parallelism": "one GPU", "routes": "factored (every linear)",
         "train_schedule": ("balanced token-tile ranges per launch"
                            if (spec["balance"] if args.balance < 0 else bool(args.balance))
-                           else "whole examples per SM") + f", {args.train_streams} train streams",
+                           else "whole examples per SM") + f", {args.train_streams} train streams"
+                          + (lambda b: f", projection grids capped at {b} CTAs" if b else "")(
+                              spec["sm_budget"] if args.sm_budget is None else args.sm_budget),
     }
 
 
@@ -745,7 +748,7 @@ def stack_profile_main(args, spec):
 
     tbuild.build()
     tda.load()
-    tda.tda_set_sm_budget(args.sm_budget)
+    tda.tda_set_sm_budget(args.sm_budget or 0)
     dev = torch.device("cuda", 0)
     torch.cuda.set_device(dev)
     stream = torch.cuda.current_stream()
@@ -798,7 +801,7 @@ def stack_profile_main(args, spec):
     torch.cuda.synchronize()
     tda.tda_device_status()
     ms = ev0.elapsed_time(ev1) / args.steps
-    print(json.dumps({"mode": "profile", **what, "sm_budget": args.sm_budget, "ms_per_call": ms,
+    print(json.dumps({"mode": "profile", **what, "sm_budget": args.sm_budget or 0, "ms_per_call": ms,
                       "rate": work[1] / (ms * 1e-3), "unit": work[0]}))
     return 0
 
@@ -816,7 +819,8 @@ def stack_main(args, spec):
         return 0  # one GPU: the stack job does not shard here
     tbuild.build()
     tda.load()
-    tda.tda_set_sm_budget(args.sm_budget)
+    sm_budget = spec["sm_budget"] if args.sm_budget is None else args.sm_budget
+    tda.tda_set_sm_budget(sm_budget)
     dev = torch.device("cuda", 0)
     torch.cuda.set_device(dev)
     stream = torch.cuda.current_stream()
