@@ -765,12 +765,14 @@ def stack_profile_main(args, spec):
         L = tda.LayerDesc(di, do, T, k, k, seed=0, layer=li)
         assert tda.tda_project_engine(L, tda.TDA_BF16, A, B) == 1
         wsb = tda.tda_workspace_size(tda.TDA_OP_PROJECT, L, tda.TDA_BF16, n, 0, tda.TDA_ROUTE_FACTORED)
+        if not (spec["balance"] if args.balance < 0 else bool(args.balance)):
+            wsb = 2 * k * (di + do) if k == 128 else 0  # sign tables only: whole examples per SM
         ws = torch.empty(max(wsb, 256), dtype=torch.uint8, device=dev)
         phi = torch.empty((n, D), device=dev)
         run = lambda: tda.tda_project(L, tda.TDA_BF16, A, B, n, phi, D, tda.TDA_ROUTE_FACTORED, ws, wsb)
         work = ("GB/s", n * (T * (di + do) * 2 + 4 * D) / 1e9)
         what = {"kernel": "factored projection", "linear": [di, do], "n": n, "T": T, "k": k,
-                "sign_tables": bool(wsb)}
+                "sign_tables": k == 128 and bool(wsb), "balanced": wsb > 2 * k * (di + do) * (k == 128)}
     else:
         nl = args.profile_linears or len(spec["layer"])
         per = tda.tda_precondition_state_bytes(D, tda.TDA_F32)

@@ -59,6 +59,8 @@ struct GParams {
     int splits;            // gridDim.y
     int batched;           // grid z = batch entry: A and B maps are 3-D (z the third coordinate)
     int64_t s_z;           // S element offset between batch entries
+    int64_t tiles_z;       // persistent kernel: tiles per batch entry
+    int nz;                // persistent kernel: batch entries
     unsigned int* err;
 };
 
@@ -361,6 +363,269 @@ score3x_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
         tmem_dealloc(tmem, C::kTmemCols);
     }
     cluster_sync();
+}
+
+// ---------------------------------------------------------------------------
+// Persistent variant of the same product for many tiles with short K (the
+// blocked Cholesky's trailing updates and the substitutions' block products,
+// K = 128 or 256): each CTA walks tiles blockIdx.x, blockIdx.x + gridDim.x, ...
+// over all batch entries with one set of barriers and one TMEM allocation. The
+// accumulators are double-buffered (kAcc per buffer), so a tile's epilogue
+// (TMEM -> registers -> S) overlaps the next tile's loads, splits and MMAs.
+// Warps 0-3 split, warps 4-7 epilogue, lane 0 of warp 8 issues the TMA copies,
+// lane 0 of warp 9 the MMAs. Same arithmetic per tile as score3x_kernel (the
+// K chunks rotate over kAcc accumulators, summed on CUDA cores). No clusters,
+// no split-K. All waits are bounded.
+constexpr int kThreadsP = 320;
+
+template <int BN>
+struct PCfg {
+    static constexpr int kStages = GCfg<BN>::kStages;
+    static constexpr uint32_t kABytes = GCfg<BN>::kABytes;
+    static constexpr uint32_t kBBytes = GCfg<BN>::kBBytes;
+    static constexpr uint32_t kStageBytes = GCfg<BN>::kStageBytes;
+    static constexpr int kAcc = 256 / BN;  // per buffer: two buffers fill the 512 TMEM columns
+    static constexpr size_t kSmem = 1024 + (size_t)kStages * kStageBytes + 8 * (3 * kStages + 5) + 16;
+};
+
+// Rows m0 (of A) and n0 (of B) and batch entry z of tile t.
+template <int BN>
+__device__ __forceinline__ void tile_at(const GParams& p, int64_t t, int64_t& m0, int64_t& n0, int& z) {
+    z = (int)(t / p.tiles_z);
+    const int64_t tile = t - (int64_t)z * p.tiles_z;
+    if (p.lower) {
+        int64_t i = (int64_t)((sqrt(8.0 * (double)tile + 1.0) - 1.0) * 0.5);
+        while (i * (i + 1) / 2 > tile) --i;
+        while ((i + 1) * (i + 2) / 2 <= tile) ++i;
+        n0 = i * BN;
+        m0 = (tile - i * (i + 1) / 2) * kBM;
+    } else {
+        m0 = (tile / p.tiles_n) * kBM;
+        n0 = (tile % p.tiles_n) * BN;
+    }
+}
+
+template <int BN>
+__global__ void __maxnreg__(200)
+gemm3x_persist_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
+                      const GParams p) {
+    using C = PCfg<BN>;
+    extern __shared__ uint8_t smem_raw[];
+    uint8_t* smem = (uint8_t*)(((uintptr_t)smem_raw + 1023) & ~(uintptr_t)1023);
+    uint64_t* bars = (uint64_t*)(smem + (size_t)C::kStages * C::kStageBytes);
+    uint64_t* raw_full = bars;                  // [kStages] TMA bytes landed (count 1 + tx)
+    uint64_t* full = raw_full + C::kStages;     // [kStages] split into hi/lo (count 4)
+    uint64_t* empty = full + C::kStages;        // [kStages] MMAs done reading (count 1)
+    uint64_t* tfull = empty + C::kStages;       // [2] accumulators ready (count 1)
+    uint64_t* tempty = tfull + 2;               // [2] accumulators drained (count 4)
+    uint64_t* mma_done = tempty + 2;            // count 1
+    uint32_t* tmem_slot = (uint32_t*)(mma_done + 1);
+    volatile int* abort = (volatile int*)(tmem_slot + 1);
+
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    if (threadIdx.x == 0) {
+        for (int s = 0; s < C::kStages; ++s) {
+            mbar_init(smem_u32(&raw_full[s]), 1);
+            mbar_init(smem_u32(&full[s]), 4);
+            mbar_init(smem_u32(&empty[s]), 1);
+        }
+        for (int b = 0; b < 2; ++b) {
+            mbar_init(smem_u32(&tfull[b]), 1);
+            mbar_init(smem_u32(&tempty[b]), 4);
+        }
+        mbar_init(smem_u32(mma_done), 1);
+        *abort = 0;
+        fence_mbar_init();
+    }
+    if (warp == 9) {
+        tmem_alloc(smem_u32(tmem_slot), 512);
+        tmem_relinquish();
+    }
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+    const uint32_t tmem = *tmem_slot;
+    const int64_t total = p.tiles_z * p.nz;
+    const int64_t nkc = (p.K + kKC - 1) / kKC;
+
+    if (warp < 4) {
+        // ---------------- split warps: raw fp32 (TMA) -> hi in place + lo
+        const int pt = threadIdx.x;
+        uint32_t it = 0;
+        bool ok = true;
+        for (int64_t t = blockIdx.x; ok && t < total; t += gridDim.x)
+            for (int64_t kc = 0; kc < nkc; ++kc, ++it) {
+                const int s = it % C::kStages;
+                const uint32_t ph = (it / C::kStages) & 1u;
+                bool got = true;
+                if (lane == 0) got = wait_bounded(smem_u32(&raw_full[s]), ph, abort, p.err);
+                got = __shfl_sync(0xffffffffu, got, 0);
+                __syncwarp();
+                if (!got) {
+                    ok = false;
+                    break;
+                }
+                uint8_t* st = smem + (size_t)s * C::kStageBytes;
+                split_tile<C::kABytes>(st, st + C::kABytes, pt);
+                split_tile<C::kBBytes>(st + 2 * C::kABytes, st + 2 * C::kABytes + C::kBBytes, pt);
+                fence_proxy_async();
+                __syncwarp();
+                if (lane == 0) mbar_arrive(smem_u32(&full[s]));
+            }
+    } else if (warp < 8) {
+        // ---------------- epilogue: TMEM -> registers (buffer released) -> S
+        const int q = warp & 3;
+        const int row = q * 32 + lane;
+        const int used = (int)(nkc < C::kAcc ? nkc : C::kAcc);
+        uint32_t lt = 0;
+        for (int64_t t = blockIdx.x; t < total; t += gridDim.x, ++lt) {
+            const uint32_t b = lt & 1u, ph = (lt >> 1) & 1u;
+            bool got = true;
+            if (lane == 0) got = wait_bounded(smem_u32(&tfull[b]), ph, abort, p.err);
+            got = __shfl_sync(0xffffffffu, got, 0);
+            if (epi_any(!got)) break;
+            tc_fence_after();
+            const uint32_t tbase = tmem + ((uint32_t)(q * 32) << 16) + b * (uint32_t)(C::kAcc * BN);
+            int64_t m0, n0;
+            int z;
+            tile_at<BN>(p, t, m0, n0, z);
+            float* Sz = p.S + (int64_t)z * p.s_z;
+            const int64_t m = m0 + row;
+            // 64 columns at a time (register budget); the buffer is released after the last read
+#pragma unroll 1
+            for (int h0 = 0; h0 < BN; h0 += 64) {
+                constexpr int HW = BN < 64 ? BN : 64;
+                float acc[HW];
+#pragma unroll
+                for (int c0 = 0; c0 < HW; c0 += 16) {
+#pragma unroll
+                    for (int i = 0; i < 16; ++i) acc[c0 + i] = 0.f;
+                    for (int a = 0; a < used; ++a) {
+                        float v[16];
+                        tmem_ld16(tbase + a * BN + h0 + c0, v);
+#pragma unroll
+                        for (int i = 0; i < 16; ++i) acc[c0 + i] += v[i];
+                    }
+                }
+                if (h0 + HW >= BN) {
+                    tc_fence_before();
+                    __syncwarp();
+                    if (lane == 0) mbar_arrive(smem_u32(&tempty[b]));
+                }
+                if (m < p.n_t) {
+                    if (p.beta == 0.f) {
+#pragma unroll
+                        for (int c = 0; c < HW; ++c) {
+                            const int64_t n = n0 + h0 + c;
+                            if (n < p.n_q) Sz[n * p.ld_S + m] = p.alpha * acc[c];
+                        }
+                    } else {
+#pragma unroll
+                        for (int c0 = 0; c0 < HW; c0 += 16) {
+                            float old[16];
+#pragma unroll
+                            for (int i = 0; i < 16; ++i) {
+                                const int64_t n = n0 + h0 + c0 + i;
+                                old[i] = n < p.n_q ? __ldcg(Sz + n * p.ld_S + m) : 0.f;
+                            }
+#pragma unroll
+                            for (int i = 0; i < 16; ++i) {
+                                const int64_t n = n0 + h0 + c0 + i;
+                                if (n < p.n_q) Sz[n * p.ld_S + m] = p.beta * old[i] + p.alpha * acc[c0 + i];
+                            }
+                        }
+                    }
+                }
+            }
+        }
+    } else if (warp == 8 && lane == 0) {
+        // ---------------- TMA producer
+        uint32_t it = 0, last_par[C::kStages];
+        bool issued[C::kStages];
+        for (int s = 0; s < C::kStages; ++s) issued[s] = false;
+        bool ok = true;
+        for (int64_t t = blockIdx.x; ok && t < total; t += gridDim.x) {
+            int64_t m0, n0;
+            int z;
+            tile_at<BN>(p, t, m0, n0, z);
+            for (int64_t kc = 0; kc < nkc; ++kc, ++it) {
+                const int s = it % C::kStages;
+                const uint32_t ph = (it / C::kStages) & 1u;
+                if (!wait_bounded(smem_u32(&empty[s]), ph ^ 1u, abort, p.err)) {
+                    ok = false;
+                    break;
+                }
+                const uint32_t st = smem_u32(smem + (size_t)s * C::kStageBytes), bar = smem_u32(&raw_full[s]);
+                const int k = (int)(kc * kKC);
+                mbar_arrive_tx(bar, C::kABytes + C::kBBytes);
+                if (p.batched) {
+                    tma_load_3d(st, &tmA, k, (int)m0, z, bar);
+                    tma_load_3d(st + 2 * C::kABytes, &tmB, k, (int)n0, z, bar);
+                } else {
+                    tma_load_2d(st, &tmA, k, (int)m0, bar);
+                    tma_load_2d(st + 2 * C::kABytes, &tmB, k, (int)n0, bar);
+                }
+                issued[s] = true;
+                last_par[s] = ph;
+            }
+        }
+        for (int s = 0; s < C::kStages; ++s)
+            if (issued[s]) {
+                const uint64_t t0 = global_ns();
+                while (!mbar_try_wait(smem_u32(&raw_full[s]), last_par[s]))
+                    if (global_ns() - t0 > kTimeoutNs) {
+                        atomicOr(p.err, kErrTimeout);
+                        break;
+                    }
+            }
+    } else if (warp == 9 && lane == 0) {
+        // ---------------- MMA issuer
+        const uint32_t idesc = idesc_tf32(kBM, BN);
+        uint32_t it = 0, lt = 0;
+        bool ok = true;
+        for (int64_t t = blockIdx.x; ok && t < total; t += gridDim.x, ++lt) {
+            const uint32_t b = lt & 1u, use = lt >> 1;
+            if (!wait_bounded(smem_u32(&tempty[b]), (use & 1u) ^ 1u, abort, p.err)) break;
+            tc_fence_after();
+            for (int64_t kc = 0; kc < nkc; ++kc, ++it) {
+                const int s = it % C::kStages;
+                const uint32_t ph = (it / C::kStages) & 1u;
+                if (!wait_bounded(smem_u32(&full[s]), ph, abort, p.err)) {
+                    ok = false;
+                    break;
+                }
+                tc_fence_after();
+                const uint32_t st = smem_u32(smem + (size_t)s * C::kStageBytes);
+                const uint64_t ahi = sw128_desc(st), alo = sw128_desc(st + C::kABytes);
+                const uint64_t bhi = sw128_desc(st + 2 * C::kABytes), blo = sw128_desc(st + 2 * C::kABytes + C::kBBytes);
+                const uint32_t d = tmem + (b * C::kAcc + (uint32_t)(kc % C::kAcc)) * BN;
+#pragma unroll
+                for (int k = 0; k < kKC / 8; ++k) {
+                    const uint32_t first = (kc < C::kAcc && k == 0) ? 0u : 1u;
+                    mma_tf32(d, ahi + 2 * k, bhi + 2 * k, idesc, first);
+                    mma_tf32(d, ahi + 2 * k, blo + 2 * k, idesc, 1u);
+                    mma_tf32(d, alo + 2 * k, bhi + 2 * k, idesc, 1u);
+                }
+                mma_commit(smem_u32(&empty[s]));
+            }
+            if (!ok) break;
+            mma_commit(smem_u32(&tfull[b]));
+        }
+        mma_commit(smem_u32(mma_done));
+        const uint64_t t0 = global_ns();
+        while (!mbar_try_wait(smem_u32(mma_done), 0))
+            if (global_ns() - t0 > kTimeoutNs) {
+                atomicOr(p.err, kErrTimeout);
+                break;
+            }
+    }
+
+    tc_fence_before();
+    __syncthreads();
+    if (warp == 9) {
+        tc_fence_after();
+        tmem_dealloc(tmem, 512);
+    }
 }
 
 // ---------------------------------------------------------------------------
@@ -730,6 +995,18 @@ cudaError_t launch_bn(GParams p, cudaStream_t s, int64_t nz = 1, size_t a_z_byte
     while (cs > 1 && (size_t)(cs - 1) * kBM * BN * 4 > (size_t)C::kStages * C::kStageBytes) cs >>= 1;
     p.cs = cs;
     p.tiles_n = (int)tiles_n;
+    if (cs == 1 && p.splits == 1 && !p.kslice && nkc <= 64 && tiles * nz > sms) {
+        // more tiles than SMs with short K: one persistent CTA per SM walks the tiles
+        using P = PCfg<BN>;
+        p.tiles_z = tiles;
+        p.nz = (int)nz;
+        cudaError_t e = cudaFuncSetAttribute(gemm3x_persist_kernel<BN>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                             (int)P::kSmem);
+        if (e != cudaSuccess) return e;
+        note_launches(1);
+        gemm3x_persist_kernel<BN><<<(unsigned)sms, kThreadsP, P::kSmem, s>>>(tmA, tmB, p);
+        return cudaGetLastError();
+    }
     cudaError_t e = cudaFuncSetAttribute(score3x_kernel<BN>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)C::kSmem);
     if (e != cudaSuccess) return e;
     cudaLaunchConfig_t cfg = {};

@@ -24,8 +24,8 @@
 //
 // Blocked path (fp32 state, D a multiple of 128 and at least 2048): the same
 // right-looking Cholesky in 256-column panels of two 128-column halves. Per
-// half: the 128 x 128 diagonal block is factored in shared memory (its four
-// 32-column steps as above, Dinv of its four 32 x 32 blocks) and the rows below
+// half: the 128 x 128 diagonal block is factored in shared memory (column by
+// column, left-looking; Dinv of its four 32 x 32 blocks) and the rows below
 // it are solved against it (x L_BB^T = a); the second half's columns first take
 // the first half's update. The trailing lower triangle then takes the rank-256
 // update M -= P P^T on the tensor cores (3xTF32, launch_gemm_nt_tc). After the
@@ -1041,18 +1041,17 @@ constexpr size_t kTrsmSmem =
     sizeof(float) * ((size_t)kBB * (kBB + 1) + (size_t)(kBB / kNB) * kNB * (kNB + 1) + (size_t)kTrsmWarps * kBB);
 
 // Factor the 128 x 128 diagonal block at lo of every layer (grid = layer) in
-// shared memory, in four 32-column steps: Cholesky of the 32 x 32 block by one
-// warp (warp_cholesky32: rolled steps, the pivot column in register 0), the
-// block's rows below it solved against it by forward substitution (one thread
-// per row, rolled loops), the rest of the block updated. L returns to M's lower
-// triangle; the inverses of the four 32 x 32 diagonal blocks go to Dinv (one
-// warp each, after the last step); a non-positive pivot is recorded in the header.
+// shared memory by the left-looking (Cholesky-Crout) order, one column per
+// step: L_ij = (A_ij - sum_{m<j} L_im L_jm) / L_jj for every row i >= j at
+// once, two threads per row (each half of the dot product, four independent
+// partial sums). The serial chain is one short dot product, one rsqrt and two
+// barriers per column. L returns to M's lower triangle; the inverses of the
+// four 32 x 32 diagonal blocks go to Dinv (one warp each); a non-positive
+// pivot is recorded in the header and its column turns NaN.
 __global__ void __launch_bounds__(256) diag_block_kernel(St<float> st, int64_t lo) {
     extern __shared__ __align__(16) float dsm[];
     float(*A)[kBB + 1] = reinterpret_cast<float(*)[kBB + 1]>(dsm);
-    __shared__ float Bk[kNB][kNB + 1];        // the step's diagonal block before factoring
-    __shared__ float LkT[kNB][2 * kNB + 1];   // its factor, transposed
-    __shared__ float dinv[kNB];
+    __shared__ float sinv[kBB];
     const int l = blockIdx.x;
     const int64_t D = st.D;
     float* M = st.M(l);
@@ -1062,45 +1061,37 @@ __global__ void __launch_bounds__(256) diag_block_kernel(St<float> st, int64_t l
         A[i][j] = (j <= i) ? M[(lo + i) * D + lo + j] : 0.f;
     }
     __syncthreads();
-    for (int c0 = 0; c0 < kBB; c0 += kNB) {
-        for (int e = tid; e < kNB * kNB; e += 256) Bk[e / kNB][e % kNB] = A[c0 + e / kNB][c0 + e % kNB];
-        __syncthreads();
-        if (warp == 0) {
-            const int bad = warp_cholesky32(Bk, LkT, dinv, lane);
-            if (lane == 0 && bad >= 0) {
-                double* h = st.header(l);
-                if (h[kPcFailedPivot] == 0.0) h[kPcFailedPivot] = (double)(lo + c0 + bad + 1);
-            }
-        }
-        __syncthreads();
-        for (int e = tid; e < kNB * kNB; e += 256) {
-            const int i = e / kNB, j = e % kNB;  // L of the step's block back into A
-            A[c0 + i][c0 + j] = (j <= i) ? LkT[j][i] : 0.f;
-        }
-        const int rows = kBB - c0 - kNB;  // rows of the block below this step's diagonal block
-        // x L_ss^T = a, one row per thread: x_j = (a_j - sum_{m<j} x_m L_jm) / L_jj, in place
-        if (tid < rows) {
-            float* a = A[c0 + kNB + tid] + c0;
+    const int i = tid >> 1, h = tid & 1;
 #pragma unroll 1
-            for (int jj = 0; jj < kNB; ++jj) {
-                float t = a[jj];
-#pragma unroll 4
-                for (int m = 0; m < jj; ++m) t -= a[m] * LkT[m][jj];
-                a[jj] = t * dinv[jj];
+    for (int j = 0; j < kBB; ++j) {
+        float s = 0.f;
+        if (i >= j) {
+            float a0 = 0.f, a1 = 0.f, a2 = 0.f, a3 = 0.f;
+            int m = h;
+            for (; m + 6 < j; m += 8) {
+                a0 = fmaf(A[i][m], A[j][m], a0);
+                a1 = fmaf(A[i][m + 2], A[j][m + 2], a1);
+                a2 = fmaf(A[i][m + 4], A[j][m + 4], a2);
+                a3 = fmaf(A[i][m + 6], A[j][m + 6], a3);
             }
+            for (; m < j; m += 2) a0 = fmaf(A[i][m], A[j][m], a0);
+            s = (a0 + a1) + (a2 + a3);
+        }
+        s += __shfl_xor_sync(0xffffffffu, s, 1);
+        s = (i >= j) ? A[i][j] - s : 0.f;
+        if (i == j && h == 0) {
+            const bool ok = s > 0.f;
+            if (!ok) {
+                double* hd = st.header(l);
+                if (hd[kPcFailedPivot] == 0.0) hd[kPcFailedPivot] = (double)(lo + j + 1);
+            }
+            // L_jj = s * rsqrt(s), 1 / L_jj = rsqrt(s)
+            const float inv = ok ? rsqrtf(s) : NAN;
+            sinv[j] = inv;
+            A[j][j] = s * inv;
         }
         __syncthreads();
-        // the block's trailing lower triangle
-        for (int e = tid; e < rows * rows; e += 256) {
-            const int i = e / rows, j = e % rows;
-            if (j > i) continue;
-            const float* xi = A[c0 + kNB + i] + c0;
-            const float* xj = A[c0 + kNB + j] + c0;
-            float acc = 0.f;
-#pragma unroll 8
-            for (int m = 0; m < kNB; ++m) acc += xi[m] * xj[m];
-            A[c0 + kNB + i][c0 + kNB + j] -= acc;
-        }
+        if (i > j && h == 0) A[i][j] = s * sinv[j];
         __syncthreads();
     }
     // inverses of the four diagonal blocks: warp w, lane c solves L X[:, c] = e_c
@@ -1108,20 +1099,20 @@ __global__ void __launch_bounds__(256) diag_block_kernel(St<float> st, int64_t l
         const int b0 = warp * kNB, c = lane;
         float x[kNB];
 #pragma unroll
-        for (int i = 0; i < kNB; ++i) x[i] = (i == c) ? 1.f : 0.f;
+        for (int r = 0; r < kNB; ++r) x[r] = (r == c) ? 1.f : 0.f;
 #pragma unroll
         for (int jj = 0; jj < kNB; ++jj) {
-            x[jj] = (jj < c) ? 0.f : x[jj] / A[b0 + jj][b0 + jj];
+            x[jj] = (jj < c) ? 0.f : x[jj] * sinv[b0 + jj];
 #pragma unroll
-            for (int i = jj + 1; i < kNB; ++i) x[i] -= A[b0 + i][b0 + jj] * x[jj];
+            for (int r = jj + 1; r < kNB; ++r) x[r] -= A[b0 + r][b0 + jj] * x[jj];
         }
         float* Dg = st.Dinv(l) + ((lo + b0) / kNB) * (kNB * kNB);
 #pragma unroll
-        for (int i = 0; i < kNB; ++i) Dg[i * kNB + c] = x[i];
+        for (int r = 0; r < kNB; ++r) Dg[r * kNB + c] = x[r];
     }
     for (int e = tid; e < kBB * kBB; e += 256) {
-        const int i = e / kBB, j = e % kBB;
-        if (j <= i) M[(lo + i) * D + lo + j] = A[i][j];
+        const int r = e / kBB, c = e % kBB;
+        if (c <= r) M[(lo + r) * D + lo + c] = A[r][c];
     }
 }
 
