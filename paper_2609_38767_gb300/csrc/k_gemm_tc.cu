@@ -375,7 +375,9 @@ score3x_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
 // Warps 0-3 split, warps 4-7 epilogue, lane 0 of warp 8 issues the TMA copies,
 // lane 0 of warp 9 the MMAs. Same arithmetic per tile as score3x_kernel (the
 // K chunks rotate over kAcc accumulators, summed on CUDA cores). No clusters,
-// no split-K. All waits are bounded.
+// no split-K. All waits are bounded. Ten warps share the register file's four
+// partitions unevenly (three warps on two of them), which caps a thread at 168
+// registers: the epilogue drains the accumulators 64 columns at a time.
 constexpr int kThreadsP = 320;
 
 template <int BN>
@@ -406,7 +408,7 @@ __device__ __forceinline__ void tile_at(const GParams& p, int64_t t, int64_t& m0
 }
 
 template <int BN>
-__global__ void __maxnreg__(200)
+__global__ void __launch_bounds__(kThreadsP, 1)
 gemm3x_persist_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
                       const GParams p) {
     using C = PCfg<BN>;
