@@ -1012,14 +1012,15 @@ def stack_main(args, spec):
             srcs = srcs[:-1]
         dsts = [torch.empty_like(x, device=dev) for x in srcs]
         nbytes = sum(x.numel() * 2 for x in srcs)
-        for rep in range(2):
+        h2d_gbs = 0.0
+        for rep in range(4):  # best of four: the link's ceiling, not a slow first pass
             torch.cuda.synchronize()
             c0 = time.perf_counter()
             for i, (hs, ds) in enumerate(zip(srcs, dsts)):
                 with torch.cuda.stream(copy_streams[i % 4]):
                     ds.copy_(hs, non_blocking=True)
             torch.cuda.synchronize()
-            h2d_gbs = nbytes / (time.perf_counter() - c0) / 1e9
+            h2d_gbs = max(h2d_gbs, nbytes / (time.perf_counter() - c0) / 1e9)
         del dsts
         idx_h = torch.empty((Nq, args.topk), dtype=torch.int32).pin_memory()
         val_h = torch.empty((Nq, args.topk), dtype=torch.float32).pin_memory()
@@ -1046,6 +1047,7 @@ def stack_main(args, spec):
         e2e = {"value": chunk / e2e_s, "unit": "examples/s", "h2d_bytes_per_step": h2d,
                "d2h_bytes_per_step": (Nq // C) * args.topk * 8, "ms_per_step": e2e_s * 1e3, "steps": n_e2e,
                "host_pool_examples": Ph, "h2d_gbs_measured_4_streams": h2d_gbs,
+               "h2d_gbs_achieved": h2d / e2e_s / 1e9,
                "h2d_bound_examples_per_s": chunk / (h2d / (h2d_gbs * 1e9)), "host_numa_node": numa}
         if saved_aff is not None:
             os.sched_setaffinity(0, saved_aff)

@@ -1078,9 +1078,11 @@ cudaError_t launch_k(const tda_layer_desc& L, const void* A, const void* B, int6
     // With the balanced-range workspace (one example per tile): contiguous runs of token tiles
     // per CTA, 32 token rows staged at a time (room for one or two more stages in the ring).
     // Without it, at least one example per SM (no cluster shares an example) stages 32 rows as
-    // well; fewer examples keep the larger staging rows, which hold the cluster's partial blocks.
+    // well for k >= 64 (k <= 32 measured faster with whole tiles: 7.1-7.3 against 6.9 TB/s on
+    // the Llama-1B block); fewer examples keep the larger staging rows, which hold the cluster's
+    // partial blocks.
     const bool bal = bal_ws && pack == 1;
-    const bool narrow = pack == 1 && N >= (int64_t)sm_count();
+    const bool narrow = K >= 64 && pack == 1 && N >= (int64_t)sm_count();
     if constexpr (K > 64) {
         if constexpr (!KF && !FO) {
             if (signs) {
