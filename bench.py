@@ -104,7 +104,9 @@ def parse_args():
     p.add_argument("--e2e-steps", type=int, default=2)
     p.add_argument("--no-e2e", action="store_true")
     p.add_argument("--no-cpu-baseline", action="store_true")
-    p.add_argument("--pool", type=int, default=128, help="pinned host examples per linear for e2e")
+    p.add_argument("--pool", type=int, default=16, help="pinned host examples per linear for e2e")
+    p.add_argument("--host-pool", type=int, default=None,
+                   help="stack workloads: pinned host examples per linear shape for e2e (default: the workload's)")
     p.add_argument("--linears", default="q,k,v,o,gate,up,down",
                    help="subset of the block's linears (profiling of a smaller case)")
     p.add_argument("--project-only", action="store_true",
@@ -605,7 +607,7 @@ STACKS = {
                   ("gate", 4096, 14336), ("up", 4096, 14336), ("down", 14336, 4096)],
         "n_layers": 32, "T": 1024, "k": 64, "n_train": 8192, "chunk": 256, "n_query": 256,
         "dist_a": 0, "sigma_b": math.sqrt(1e-3), "lambda_rel": 1e-2,
-        "train_pool": 512, "query_pool": 256, "host_pool": 128, "balance": False, "query_priority": 0, "sm_budget": 0,
+        "train_pool": 512, "query_pool": 256, "host_pool": 4, "balance": False, "query_priority": 0, "sm_budget": 0,
         "factors": "A~N(0,1), B~N(0,1e-3) (seeded synthetic)",
     },
     "large_model": {
@@ -982,7 +984,7 @@ def stack_main(args, spec):
     e2e = None
     if not args.no_e2e:
         saved_aff, numa = bind_to_gpu_numa(0)
-        Ph = spec["host_pool"]
+        Ph = spec["host_pool"] if args.host_pool is None else args.host_pool
         hpools = []
         for si in range(nshape):
             A, B, Aq, Bq = pools[si]
