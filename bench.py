@@ -54,15 +54,16 @@ METRIC = "train examples attributed/sec (project+score)"
 
 # DRAM traffic of the tensor-core projection kernel, from one ncu capture per k
 # (dram__bytes_read.sum + dram__bytes_write.sum over the algorithmic bytes of the
-# launch): k = 64, 160 examples of the 4096x4096 linear at T = 1024
-# (profiles/tc_projection_k64_llama3_q160.md); k = 128, 32 examples of the
-# 12288 -> 1536 linear at T = 2048 (profiles/tc_projection_k128_large_k32.md).
+# launch): k = 32, 608 examples of the 2048x2048 linear at T = 512; k = 64, 160
+# examples of the 4096x4096 linear at T = 1024, whole examples per SM; k = 128, 32
+# examples of the 12288 -> 1536 linear at T = 2048, balanced token-tile ranges
+# (the ncu summaries under profiles/).
 # Launches of other linears are scaled by their algorithmic bytes (every factor
 # byte is read once, so traffic grows in proportion). Valid only for the kernel
 # source it was measured on (the kernel file and its PTX helper header); any
 # change makes the bench report null.
-TRAFFIC_RATIO = {64: 1.0030041, 128: 1.0161786}
-TRAFFIC_KERNEL_SHA256 = "5e334442b0a93a40d94f1506bb2bc1776c1cb6a7702f4eb0eaf8e7beef7d17a7"
+TRAFFIC_RATIO = {32: 1.0010457, 64: 1.0016203, 128: 1.0161481}
+TRAFFIC_KERNEL_SHA256 = "7a4b0ecb95b9b806b08718b2caa1cf5c2e1f07e4aca5177447ad0cb59b9139da"
 
 
 def projection_kernel_sha256():
