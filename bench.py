@@ -652,9 +652,11 @@ def stack_config(args, spec):
 
 def stack_oracle_sample(spec, factors_of):
     """Time the fp64 oracle on a bounded sample of a stack job and extrapolate to the job's
-    examples/s: n_s train and 2 query examples through the 7 linears of one layer, the Fisher
-    of one linear over the n_s train features, the damped inverse (D x D Cholesky) applied to
-    the queries, and their scores. factors_of(role, li, n) returns float64 (A, B)."""
+    examples/s: n_s train and 2 query examples through the first two linears of one layer (q
+    and k; the oracle's projection time is proportional to T (d_in + d_out) per example, so
+    it is scaled to the layer's seven linears by that sum), the Fisher of one linear over the
+    n_s train features, the damped inverse (D x D Cholesky) applied to the queries, and their
+    scores. factors_of(role, li, n) returns float64 (A, B)."""
     import numpy as np
 
     import oracle
@@ -663,9 +665,12 @@ def stack_oracle_sample(spec, factors_of):
     threads = os.cpu_count() or 1
     oracle.set_threads(threads)
     n_s, nq_s, k, D = max(2, threads), 2, spec["k"], spec["k"] ** 2
+    sampled = (0, 1)
+    width = lambda li: spec["layer"][li][1] + spec["layer"][li][2]
+    scale = sum(width(li) for li in range(len(spec["layer"]))) / sum(width(li) for li in sampled)
     t_proj = t_qproj = 0.0
     phis, qs = [], []
-    for li in range(len(spec["layer"])):
+    for li in sampled:
         A, B = factors_of("train", li, n_s)
         t0 = time.perf_counter()
         phis.append(oracle.project(A, B, k, k, 0, li).reshape(n_s, D))
@@ -686,12 +691,13 @@ def stack_oracle_sample(spec, factors_of):
     t_score = time.perf_counter() - t0
     N, Nq, L = spec["n_train"], spec["n_query"], spec["n_layers"]
     nlin = L * len(spec["layer"])
-    total = (t_proj * L * N / n_s + t_qproj * L * Nq / nq_s + t_fit * nlin * N / n_s + t_fact * nlin
-             + t_score * nlin * (N / n_s) * (Nq / nq_s))
-    sample = (f"{n_s} train + {nq_s} query examples (fp64, {threads} threads) through the 7 linears of one layer, "
-              f"Fisher of one linear over them, D x D Cholesky + solves, scores; projection scaled by "
-              f"{L} layers x {N}/{n_s} (queries {Nq}/{nq_s}), Fisher by {nlin} linears x {N}/{n_s}, factorisation "
-              f"by {nlin} linears, score by {nlin} x {N}/{n_s} x {Nq}/{nq_s}")
+    total = (t_proj * scale * L * N / n_s + t_qproj * scale * L * Nq / nq_s + t_fit * nlin * N / n_s
+             + t_fact * nlin + t_score * nlin * (N / n_s) * (Nq / nq_s))
+    sample = (f"{n_s} train + {nq_s} query examples (fp64, {threads} threads) through the q and k linears of one "
+              f"layer, Fisher of one linear over them, D x D Cholesky + solves, scores; projection scaled by "
+              f"{scale:.2f} (the layer's sum of d_in + d_out over q's and k's) x {L} layers x {N}/{n_s} (queries "
+              f"{Nq}/{nq_s}), Fisher by {nlin} linears x {N}/{n_s}, factorisation by {nlin} linears, score by "
+              f"{nlin} x {N}/{n_s} x {Nq}/{nq_s}")
     wall = t_proj + t_qproj + t_fit + t_fact + t_score
     return N / total, threads, sample, wall
 
