@@ -493,10 +493,21 @@ gemm3x_persist_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_cons
             tile_at<BN>(p, t, m0, n0, z);
             float* Sz = p.S + (int64_t)z * p.s_z;
             const int64_t m = m0 + row;
-            // 64 columns at a time (register budget); the buffer is released after the last read
+            // 64 columns at a time (register budget): the part's previous values are loaded first,
+            // so the 64 loads are in flight while the part's accumulators are read from TMEM; the
+            // buffer is released after the last read
+            constexpr int HW = BN < 64 ? BN : 64;
+            const bool rmw = p.beta != 0.f && m < p.n_t;
 #pragma unroll 1
-            for (int h0 = 0; h0 < BN; h0 += 64) {
-                constexpr int HW = BN < 64 ? BN : 64;
+            for (int h0 = 0; h0 < BN; h0 += HW) {
+                float old[HW];
+                if (rmw) {
+#pragma unroll
+                    for (int i = 0; i < HW; ++i) {
+                        const int64_t n = n0 + h0 + i;
+                        old[i] = n < p.n_q ? __ldcg(Sz + n * p.ld_S + m) : 0.f;
+                    }
+                }
                 float acc[HW];
 #pragma unroll
                 for (int c0 = 0; c0 < HW; c0 += 16) {
@@ -515,27 +526,10 @@ gemm3x_persist_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_cons
                     if (lane == 0) mbar_arrive(smem_u32(&tempty[b]));
                 }
                 if (m < p.n_t) {
-                    if (p.beta == 0.f) {
 #pragma unroll
-                        for (int c = 0; c < HW; ++c) {
-                            const int64_t n = n0 + h0 + c;
-                            if (n < p.n_q) Sz[n * p.ld_S + m] = p.alpha * acc[c];
-                        }
-                    } else {
-#pragma unroll
-                        for (int c0 = 0; c0 < HW; c0 += 16) {
-                            float old[16];
-#pragma unroll
-                            for (int i = 0; i < 16; ++i) {
-                                const int64_t n = n0 + h0 + c0 + i;
-                                old[i] = n < p.n_q ? __ldcg(Sz + n * p.ld_S + m) : 0.f;
-                            }
-#pragma unroll
-                            for (int i = 0; i < 16; ++i) {
-                                const int64_t n = n0 + h0 + c0 + i;
-                                if (n < p.n_q) Sz[n * p.ld_S + m] = p.beta * old[i] + p.alpha * acc[c0 + i];
-                            }
-                        }
+                    for (int i = 0; i < HW; ++i) {
+                        const int64_t n = n0 + h0 + i;
+                        if (n < p.n_q) Sz[n * p.ld_S + m] = rmw ? p.beta * old[i] + p.alpha * acc[i] : p.alpha * acc[i];
                     }
                 }
             }
