@@ -982,10 +982,14 @@ def stack_main(args, spec):
         "topk": ("latency", 4.0 * Nq * N, hbm, "GB/s"),
     }
     phases = {}
+    side = bool(args.query_side_stream)
     for name, ms_ in ph.items():
         bound, work, peak, unit = per_job_lin[name]
         rate = work / C / (ms_ * 1e-3) / (1e9 if unit == "GB/s" else 1e12)
         phases[name] = {"ms": ms_, "bound": bound, "achieved": rate, "peak": peak, "unit": unit, "frac": rate / peak}
+        if side and name != "project_train":
+            # wall time on the query-side stream, beside the train projections that hold most SMs
+            phases[name]["stream"] = "query side, overlapped"
 
     # ---- e2e: the same steps with the factors in pinned host memory
     e2e = None
