@@ -81,11 +81,13 @@ __device__ __forceinline__ void split_tf32(float x, float& hi, float& lo) {
     lo = x - hi;
 }
 
-// Split a TMA-written fp32 tile in place: hi = x truncated to TF32 stays, lo =
-// x - hi goes to the lo tile at the same byte offset (the swizzle is the same
-// for both). 128 threads, one 16-byte group each per pass (conflict-free).
+// Split a TMA-written fp32 tile: lo = x - hi (hi = x truncated to TF32) goes to
+// the lo tile at the same byte offset (the swizzle is the same for both). The
+// fp32 tile itself serves as the hi operand: a kind::tf32 MMA reads only the
+// upper 19 bits of each element, which is hi exactly, so it is not rewritten.
+// 128 threads, one 16-byte group each per pass (conflict-free).
 template <uint32_t BYTES>
-__device__ __forceinline__ void split_tile(uint8_t* hi, uint8_t* lo, int pt) {
+__device__ __forceinline__ void split_tile(const uint8_t* hi, uint8_t* lo, int pt) {
 #pragma unroll 4
     for (uint32_t off = (uint32_t)pt * 16u; off < BYTES; off += 128u * 16u) {
         const float4 v = *reinterpret_cast<const float4*>(hi + off);
@@ -94,7 +96,6 @@ __device__ __forceinline__ void split_tile(uint8_t* hi, uint8_t* lo, int pt) {
         split_tf32(v.y, h.y, l.y);
         split_tf32(v.z, h.z, l.z);
         split_tf32(v.w, h.w, l.w);
-        *reinterpret_cast<float4*>(hi + off) = h;
         *reinterpret_cast<float4*>(lo + off) = l;
     }
 }
