@@ -27,11 +27,20 @@
 // HBM-bound and the pipeline is sized for bytes in flight.
 //
 // k = 128 (K = 128): At | Bt of one tile fill 256 TMEM columns, so the two
-// accumulator buffers take all 512 and a stage holds one token tile; the
-// epilogue stages and contracts the tile's tokens in two 64-row halves (the
-// fp32 rows of a whole tile would leave too little shared memory for the
-// stage ring), and at most 2-CTA clusters share an example (their partial
-// K x K blocks are reduced inside the leader's staging rows).
+// accumulator buffers take all 512 and a stage holds one token tile. With the
+// optional workspace both sides' sign tables are written once per call and
+// brought in by TMA beside the factor tiles instead of by the generator warps.
+//
+// Staging: the epilogue stages a tile's fp32 rows in shared memory in parts of
+// SR token rows (32 where every CTA owns whole examples or balanced ranges, 64
+// or 128 otherwise); fewer staged rows leave room for more stages in the ring.
+//
+// Work split: whole examples per CTA (example slots cid, cid + ncl, ...);
+// below one example per SM a cluster of 2 or 4 CTAs shares an example's token
+// tiles and reduces the partial K x K blocks over distributed shared memory;
+// with the workspace (balanced ranges) every CTA takes an equal contiguous run
+// of token tiles and an example split between CTAs is summed from partial
+// blocks, in CTA order, by the last of them to finish (store_phi_bal).
 //
 // Warp roles (256 threads, one persistent CTA per SM):
 //   warp 0  TMA producer: 128x64 bf16 factor tiles into the stage ring
