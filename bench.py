@@ -648,7 +648,9 @@ def stack_config(args, spec):
         "resident_pools": (f"{spec['train_pool']} train / {spec['query_pool']} query examples per linear shape in "
                            "HBM; each (chunk, layer) reads its own window of the train pool"),
         "l2": "inputs larger than L2 (no flush)",
-        "parallelism": "one GPU", "routes": "factored (every linear)",
+        "parallelism": ("one GPU" if int(os.environ.get("WORLD_SIZE", "1")) == 1 else
+                        f"replicas: an independent job on each of {os.environ.get('WORLD_SIZE')} GPUs"),
+        "routes": "factored (every linear)",
         "train_schedule": ("balanced token-tile ranges per launch"
                            if (spec["balance"] if args.balance < 0 else bool(args.balance))
                            else "whole examples per SM") + f", {args.train_streams} train streams"
@@ -833,14 +835,32 @@ def stack_main(args, spec):
     from paper_2609_38767_gb300 import synth
     from paper_2609_38767_gb300.stream import StackJob
 
-    if int(os.environ.get("WORLD_SIZE", "1")) > 1 and int(os.environ.get("RANK", "0")) != 0:
-        return 0  # one GPU: the stack job does not shard here
-    tbuild.build()
+    # Under torchrun every rank runs an independent replica of the job on its own GPU (the
+    # method runs on one GPU; replicas share nothing): barrier and max over ranks around the
+    # timed region, value = the replicas' examples over that time.
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    dev = torch.device("cuda", local)
+    torch.cuda.set_device(dev)
+    dist = None
+    if world > 1:
+        import torch.distributed as dist
+        dist.init_process_group("nccl", device_id=dev)
+    if rank == 0:
+        tbuild.build()
+    if dist:
+        dist.barrier()
     tda.load()
     sm_budget = spec["sm_budget"] if args.sm_budget is None else args.sm_budget
     tda.tda_set_sm_budget(sm_budget)
-    dev = torch.device("cuda", 0)
-    torch.cuda.set_device(dev)
+
+    def max_over_ranks(x):
+        if not dist:
+            return x
+        t = torch.tensor([x], dtype=torch.float64, device=dev)
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        return float(t.item())
     stream = torch.cuda.current_stream()
     lin, L = spec["layer"], spec["n_layers"]
     T, k, N, chunk, Nq = spec["T"], spec["k"], spec["n_train"], spec["chunk"], spec["n_query"]
@@ -924,11 +944,14 @@ def stack_main(args, spec):
             di, do = linears[li]
             ev.append((open_ev.pop(li), e, n * (T * (di + do) * 2 + 4 * D)))
 
-    clocks = ClockSampler(0)
+    clocks = ClockSampler(local)
     clocks.start()
     time.sleep(0.3)
     l0 = tda.tda_launch_count()
     t0, t1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    if dist:
+        dist.barrier()
+    torch.cuda.synchronize()
     if args.nvtx:
         torch.cuda.nvtx.range_push("timed")
     t0.record(stream)
@@ -939,11 +962,13 @@ def stack_main(args, spec):
     if args.nvtx:
         torch.cuda.nvtx.range_pop()
     torch.cuda.synchronize()
+    if dist:
+        dist.barrier()
     launches = tda.tda_launch_count() - l0
     ck = clocks.stop()
     tda.tda_device_status()
-    ms = t0.elapsed_time(t1) / steps
-    value = chunk / (ms * 1e-3)
+    ms = max_over_ranks(t0.elapsed_time(t1) / steps)
+    value = world * chunk / (ms * 1e-3)
 
     peaks = {}
     try:
@@ -1001,7 +1026,7 @@ def stack_main(args, spec):
     # ---- e2e: the same steps with the factors in pinned host memory
     e2e = None
     if not args.no_e2e:
-        saved_aff, numa = bind_to_gpu_numa(0)
+        saved_aff, numa = bind_to_gpu_numa(local)
         Ph = spec["host_pool"] if args.host_pool is None else args.host_pool
         hpools = []
         for si in range(nshape):
@@ -1057,23 +1082,28 @@ def stack_main(args, spec):
         e2e_step()
         torch.cuda.synchronize()
         n_e2e = max(1, args.e2e_steps)
+        if dist:
+            dist.barrier()
         c0 = time.perf_counter()
         for _ in range(n_e2e):
             e2e_step()
-        e2e_s = (time.perf_counter() - c0) / n_e2e
+        e2e_s = max_over_ranks((time.perf_counter() - c0) / n_e2e)
         tda.tda_device_status()
         h2d = (chunk * T * sum(di + do for di, do in linears) * 2
                + Nq * T * sum(di + do for di, do in linears) * 2 // C)
-        e2e = {"value": chunk / e2e_s, "unit": "examples/s", "h2d_bytes_per_step": h2d,
+        e2e = {"value": world * chunk / e2e_s, "unit": "examples/s", "h2d_bytes_per_step": world * h2d,
                "d2h_bytes_per_step": (Nq // C) * args.topk * 8, "ms_per_step": e2e_s * 1e3, "steps": n_e2e,
                "host_pool_examples": Ph, "h2d_gbs_measured_4_streams": h2d_gbs,
                "h2d_gbs_achieved": h2d / e2e_s / 1e9,
                "h2d_bound_examples_per_s": chunk / (h2d / (h2d_gbs * 1e9)), "host_numa_node": numa}
+        if world > 1:
+            e2e["d2h_bytes_per_step"] *= world
+            e2e["note"] = "per-rank H2D figures; value and bytes summed over the replicas"
         if saved_aff is not None:
             os.sched_setaffinity(0, saved_aff)
 
     cpu = None
-    if not args.no_cpu_baseline:
+    if not args.no_cpu_baseline and rank == 0:
         def factors_of(role, li, n):
             A, B, Aq, Bq = pools[li]
             X, Y = (A, B) if role == "train" else (Aq, Bq)
@@ -1083,12 +1113,16 @@ def stack_main(args, spec):
         cpu = {"value": v, "unit": "examples/s", "cores": cores, "kind": "oracle", "sample": sample}
 
     line = {
-        "metric": METRIC, "value": value, "unit": "examples/s", "n_gpus": 1, "steps": steps, "warmup": args.warmup,
-        "ms_per_step": ms, "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "bf16",
-        "data": "synthetic", "config": stack_config(args, spec), "roofline": roofline, "phases": phases,
-        "cpu_baseline": cpu, "e2e": e2e, "gpu_launches": launches, "clocks": ck,
+        "metric": METRIC, "value": value, "unit": "examples/s", "n_gpus": world, "steps": steps,
+        "warmup": args.warmup, "ms_per_step": ms, "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
+        "dtype": "bf16", "data": "synthetic", "config": stack_config(args, spec), "roofline": roofline,
+        "phases": phases, "cpu_baseline": cpu, "e2e": e2e, "gpu_launches": launches, "clocks": ck,
     }
-    print(json.dumps(line), flush=True)
+    if rank == 0:
+        print(json.dumps(line), flush=True)
+    if dist:
+        dist.barrier()
+        dist.destroy_process_group()
     return 0
 
 
