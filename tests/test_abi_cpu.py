@@ -180,3 +180,19 @@ def test_sm_budget_is_host_state(libs):
     assert tda.tda_get_sm_budget() == 100
     tda.tda_set_sm_budget(0)
     assert tda.tda_get_sm_budget() == 0
+
+
+@pytest.mark.parametrize("k", [16, 32, 64, 128])
+def test_factored_projection_workspace_layout(libs, k):
+    # bf16 factored projection: the optional workspace is [k = 128 sign tables, rounded up to
+    # 256 bytes][two k x k fp32 partial blocks and one counter per SM]; any other k or dtype
+    # needs none
+    di, do = 1000, 2056
+    L = tda.LayerDesc(di, do, 300, k, k)
+    b = tda.tda_workspace_size(tda.TDA_OP_PROJECT, L, tda.TDA_BF16, 7, 0, tda.TDA_ROUTE_FACTORED)
+    signs = (2 * k * (di + do) + 255) // 256 * 256 if k == 128 else 0
+    per_sm = 2 * k * k * 4 + 4
+    assert b > signs and (b - signs) % per_sm == 0
+    L2 = tda.LayerDesc(di, do, 300, k, k // 2 if k > 16 else 32)
+    assert tda.tda_workspace_size(tda.TDA_OP_PROJECT, L2, tda.TDA_BF16, 7, 0, tda.TDA_ROUTE_FACTORED) == 0
+    assert tda.tda_workspace_size(tda.TDA_OP_PROJECT, L, tda.TDA_F32, 7, 0, tda.TDA_ROUTE_FACTORED) == 0
