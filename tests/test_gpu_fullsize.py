@@ -273,6 +273,30 @@ def test_large_model_layer_from_pinned_host(dev, orc, li, di, do, pws):
         assert rel_fro(got[e], ref[e]) <= TOL
 
 
+def test_llama8b_gate_from_pinned_host_small_pieces(dev, orc):
+    # the Llama-3-8B stack's e2e leg: 4-example pieces of the gate linear (4096 -> 14336,
+    # T = 1024, k = 64) from pinned host memory, with the projection's workspace beside the
+    # staging halves (balanced token-tile ranges: 32 tiles over 32 SMs, no example split)
+    T, k, n, li = 1024, 64, 4, 4
+    di, do = 4096, 14336
+    A = synth.factors(synth.SEED_A, li, n, T, di, 1.0, 0, 0, "bf16")
+    B = synth.factors(synth.SEED_B, li, n, T, do, math.sqrt(1e-3), 0, 0, "bf16")
+    Ah = torch.from_numpy(A.view(np.int16)).view(torch.bfloat16).pin_memory()
+    Bh = torch.from_numpy(B.view(np.int16)).view(torch.bfloat16).pin_memory()
+    L = tda.LayerDesc(di, do, T, k, k, seed=0, layer=li)
+    p = tda.tda_workspace_size(tda.TDA_OP_PROJECT, L, tda.TDA_BF16, n, 0, tda.TDA_ROUTE_FACTORED)
+    wsb = n * tda.tda_project_host_ws_min(L, tda.TDA_BF16) + 2 * ((p + 255) // 256 * 256)
+    ws = torch.empty(wsb, dtype=torch.uint8, device=dev)
+    phi = torch.empty((n, k * k), device=dev)
+    for _ in range(2):  # the second call reuses the staging halves and the projection workspaces
+        tda.tda_project_host(L, tda.TDA_BF16, Ah, Bh, n, phi, k * k, ws, wsb)
+    tda.tda_device_status()
+    ref = orc.project(synth.to_f64(A, "bf16"), synth.to_f64(B, "bf16"), k, k, 0, li)
+    got = phi.cpu().numpy().reshape(n, k, k)
+    for e in range(n):
+        assert rel_fro(got[e], ref[e]) <= TOL
+
+
 def test_topk_at_large_model_query_shape(dev, orc):
     # 512 queries x 16384 train, top-100, descending with ties to the lower index
     rng = np.random.default_rng(2)

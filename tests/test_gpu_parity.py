@@ -679,9 +679,13 @@ def test_similarity_projected_routes_match_oracle(dev, orc, dtype, route):
 
 
 @pytest.mark.parametrize("nq,nt,D,beta", [(8, 64, 256, 0.0), (70, 300, 1024, 1.0), (64, 4096, 7168, 0.0),
-                                          (3, 130, 100, 0.5), (200, 257, 64, 0.0)])
+                                          (3, 130, 100, 0.5), (200, 257, 64, 0.0),
+                                          # more tiles than SMs with short K: the persistent kernel
+                                          # (double-buffered accumulators), ragged edge tiles
+                                          (300, 9000, 256, 0.0), (64, 20000, 512, 1.0), (129, 12001, 96, 0.5)])
 def test_score_tensor_core_matches_oracle(dev, orc, nq, nt, D, beta):
-    # fp32 scores on tcgen05 (3xTF32, cluster split-K): within the fp32 tolerance
+    # fp32 scores on tcgen05 (3xTF32; cluster split-K, or one persistent CTA per SM walking
+    # the tiles): within the fp32 tolerance
     rng = np.random.default_rng(nq + nt + D)
     Q = rng.standard_normal((nq, D)).astype(np.float32)
     P = (rng.standard_normal((nt, D)) * rng.uniform(0.1, 10.0, (nt, 1))).astype(np.float32)
