@@ -107,6 +107,13 @@ def parse_args():
                         "next chunks' projections, 0 = in line after each chunk")
     p.add_argument("--query-priority", type=int, default=None,
                    help="priority of that stream (lower = higher; default: the workload's)")
+    p.add_argument("--train-priority", type=int, default=None,
+                   help="stack workloads: priority of the train projection streams (lower = higher)")
+    p.add_argument("--bulk-priority", type=int, default=None,
+                   help="stack workloads: run the query side's Fisher fit and query projections on a stream of "
+                        "this priority (default: the workload's; none = on the query-side stream)")
+    p.add_argument("--side-thread", type=int, default=-1,
+                   help="stack workloads: 1 = a host thread of its own enqueues the query side (-1: the workload's)")
     p.add_argument("--query-streams", type=int, default=8,
                    help="streams the query projections of the linears are spread over (device-resident leg)")
     p.add_argument("--e2e-steps", type=int, default=2)
@@ -906,7 +913,10 @@ def stack_main(args, spec):
     job = StackJob(linears, T, k, N, chunk, Nq, topk=args.topk, lambda_rel=spec["lambda_rel"], device=dev,
                    train_streams=args.train_streams, query_stream=bool(args.query_side_stream),
                    query_priority=spec["query_priority"] if args.query_priority is None else args.query_priority,
-                   balance=balance)
+                   balance=balance,
+                   train_priority=spec.get("train_priority", 0) if args.train_priority is None else args.train_priority,
+                   bulk_priority=spec.get("bulk_priority") if args.bulk_priority is None else args.bulk_priority,
+                   side_thread=spec.get("side_thread", False) if args.side_thread < 0 else bool(args.side_thread))
     for si in range(nshape):  # every linear shape runs on the tensor-core projection kernel
         assert tda.tda_project_engine(job.layers[si], tda.TDA_BF16, pools[si][0], pools[si][1]) == 1
     state = {"j": 0, "s": 0}
@@ -926,17 +936,23 @@ def stack_main(args, spec):
     torch.cuda.synchronize()
 
     ev, phase_ev, open_ev = [], [], {}
+    # timing events created before the timed region (creating hundreds per step would add host
+    # time to every step): two per train launch and about ten phase marks per step
+    pool = [torch.cuda.Event(enable_timing=True) for _ in range(steps * (2 * nlin * (1 + max(1, chunk // Pt)) + 16))]
+
+    def new_event():
+        return pool.pop() if pool else torch.cuda.Event(enable_timing=True)
 
     def mark(name):
         st = torch.cuda.current_stream()  # phases are timed on the stream they run on
-        e = torch.cuda.Event(enable_timing=True)
+        e = new_event()
         e.record(st)
         phase_ev.append((name, e, st.cuda_stream))
 
     def hook(role, li, when, n):
         if role != "train":
             return
-        e = torch.cuda.Event(enable_timing=True)
+        e = new_event()
         e.record(torch.cuda.current_stream())
         if when == "begin":
             open_ev[li] = e
@@ -955,8 +971,10 @@ def stack_main(args, spec):
     if args.nvtx:
         torch.cuda.nvtx.range_push("timed")
     t0.record(stream)
+    h0 = time.perf_counter()
     for _ in range(steps):
         advance(dev_factors, mark, hook)
+    host_ms = (time.perf_counter() - h0) * 1e3 / steps  # host time to enqueue a step
     job.join()  # the query side queued in the timed steps is inside the timed region
     t1.record(stream)
     if args.nvtx:
@@ -1117,6 +1135,7 @@ def stack_main(args, spec):
         "warmup": args.warmup, "ms_per_step": ms, "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
         "dtype": "bf16", "data": "synthetic", "config": stack_config(args, spec), "roofline": roofline,
         "phases": phases, "cpu_baseline": cpu, "e2e": e2e, "gpu_launches": launches, "clocks": ck,
+        "host_enqueue_ms_per_step": host_ms,
     }
     if rank == 0:
         print(json.dumps(line), flush=True)

@@ -997,14 +997,13 @@ cudaError_t launch_bn(GParams p, cudaStream_t s, int64_t nz = 1, size_t a_z_byte
         using P = PCfg<BN>;
         p.tiles_z = tiles;
         p.nz = (int)nz;
-        cudaError_t e = cudaFuncSetAttribute(gemm3x_persist_kernel<BN>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                             (int)P::kSmem);
+        cudaError_t e = smem_attr_once<gemm3x_persist_kernel<BN>>((int)P::kSmem);
         if (e != cudaSuccess) return e;
         note_launches(1);
         gemm3x_persist_kernel<BN><<<(unsigned)sms, kThreadsP, P::kSmem, s>>>(tmA, tmB, p);
         return cudaGetLastError();
     }
-    cudaError_t e = cudaFuncSetAttribute(score3x_kernel<BN>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)C::kSmem);
+    cudaError_t e = smem_attr_once<score3x_kernel<BN>>((int)C::kSmem);
     if (e != cudaSuccess) return e;
     cudaLaunchConfig_t cfg = {};
     cudaLaunchAttribute attr[1];
@@ -1187,7 +1186,7 @@ cudaError_t launch_fit_tc(int n_layers, int64_t D, void* state, size_t state_byt
     p.n = n;
     p.tiles = (int)(nt * (nt + 1) / 2);
     p.err = err;
-    cudaError_t e = cudaFuncSetAttribute(fit3x_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)C::kSmem);
+    cudaError_t e = smem_attr_once<fit3x_kernel>((int)C::kSmem);
     if (e != cudaSuccess) return e;
     note_launches(1);
     fit3x_kernel<<<(unsigned)(p.tiles * n_layers), kFitThreads, C::kSmem, s>>>(tm, p);

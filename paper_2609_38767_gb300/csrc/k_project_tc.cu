@@ -1011,8 +1011,7 @@ cudaError_t launch_kg(const tda_layer_desc& L, const void* A, const void* B, int
     p.part = nullptr;
     p.cnt = nullptr;
     const int sms = sm_count();
-    cudaError_t e = cudaFuncSetAttribute(project_tc_kernel<K, G, KF, FO, SL, SR, BAL>,
-                                         cudaFuncAttributeMaxDynamicSharedMemorySize, (int)C::kSmem);
+    cudaError_t e = smem_attr_once<project_tc_kernel<K, G, KF, FO, SL, SR, BAL>>((int)C::kSmem);
     if (e != cudaSuccess) return e;
     // Fewer examples than SMs: a cluster of cs CTAs shares each example's token
     // tiles and reduces the partial features through distributed shared memory.
@@ -1031,11 +1030,8 @@ cudaError_t launch_kg(const tda_layer_desc& L, const void* A, const void* B, int
     cfg.stream = s;
     cfg.attrs = attr;
     cfg.numAttrs = 1;
-    int max_clusters = 0;
-    cfg.gridDim = dim3((unsigned)(cs * (sms / cs)));
-    if (cudaOccupancyMaxActiveClusters(&max_clusters, project_tc_kernel<K, G, KF, FO, SL, SR, BAL>, &cfg) != cudaSuccess ||
-        max_clusters < 1)
-        max_clusters = sms / cs;
+    cfg.gridDim = dim3((unsigned)(cs * (device_sms() / cs)));
+    int max_clusters = max_clusters_once<project_tc_kernel<K, G, KF, FO, SL, SR, BAL>>(cfg, cs, sms / cs);
     if (max_clusters > sms / cs) max_clusters = sms / cs;  // the SM budget (the occupancy query sees every SM)
     int64_t clusters = (FO || BAL) ? p.n_units : p.n_slots;
     if (clusters > max_clusters) clusters = max_clusters;

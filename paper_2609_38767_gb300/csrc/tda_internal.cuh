@@ -5,6 +5,8 @@
 #include <cuda_runtime.h>
 #include <stdint.h>
 
+#include <atomic>
+
 #include "../../include/tda.h"
 
 namespace tda {
@@ -221,5 +223,37 @@ cudaError_t launch_topk(const float* S, int64_t n_q, int64_t n_t, int64_t ld_S, 
 
 // State header layout of the preconditioner (doubles).
 enum { kPcLambda = 0, kPcMeanEig = 1, kPcFailedPivot = 2, kPcNTotal = 3, kPcHeaderDoubles = 8 };
+
+// Per-kernel launch set-up that does not change between launches, done once per device
+// (a stream job launches hundreds of kernels a step, and the host's time per launch adds up):
+// the dynamic shared-memory limit of kernel K, and K's maximum co-resident clusters of cs CTAs.
+template <auto Kernel>
+cudaError_t smem_attr_once(int bytes) {
+    static std::atomic<uint64_t> done{0};  // bit d: set on device d
+    int dev = 0;
+    cudaError_t e = cudaGetDevice(&dev);
+    if (e != cudaSuccess) return e;
+    const uint64_t bit = (dev >= 0 && dev < 64) ? (1ull << dev) : 0;
+    if (bit && (done.load(std::memory_order_acquire) & bit)) return cudaSuccess;
+    e = cudaFuncSetAttribute(Kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, bytes);
+    if (e == cudaSuccess && bit) done.fetch_or(bit, std::memory_order_release);
+    return e;
+}
+
+template <auto Kernel>
+int max_clusters_once(const cudaLaunchConfig_t& cfg, int cs, int fallback) {
+    static std::atomic<int> cache[64][3];  // 0 = not yet queried; cs 1, 2, 4
+    int dev = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) dev = -1;
+    const int slot = cs >= 4 ? 2 : cs - 1;
+    if (dev >= 0) {
+        const int v = cache[dev][slot].load(std::memory_order_relaxed);
+        if (v > 0) return v;
+    }
+    int n = 0;
+    if (cudaOccupancyMaxActiveClusters(&n, Kernel, &cfg) != cudaSuccess || n < 1) return fallback;
+    if (dev >= 0) cache[dev][slot].store(n, std::memory_order_relaxed);
+    return n;
+}
 
 }  // namespace tda

@@ -27,6 +27,9 @@ as pieces (device tensors, or pinned host tensors for tda_project_host).
 """
 from __future__ import annotations
 
+import queue
+import threading
+
 import torch
 
 import paper_2609_38767_gb300 as tda
@@ -35,7 +38,7 @@ import paper_2609_38767_gb300 as tda
 class StackJob:
     def __init__(self, linears, T, k, n_train, chunk, n_query, *, topk=100, lambda_rel=1e-2, lambda_abs=0.0,
                  seed=0, device="cuda", host_ws_bytes=0, train_streams=1, proj_ws=True, query_stream=False,
-                 query_priority=0, balance=True):
+                 query_priority=0, balance=True, train_priority=0, bulk_priority=None, side_thread=False):
         """linears: [(d_in, d_out)] of the whole stack, in layer order (linear i uses projection
         layer id i). n_train must be a multiple of chunk. train_streams > 1 spreads the train
         projections of a chunk round-robin over that many streams, so that a launch's CTAs fill
@@ -47,7 +50,14 @@ class StackJob:
         side and the top-k on a stream of their own (priority query_priority), beside the
         next chunks' projections; events order the two job-boundary dependencies (a job's
         query side starts after its last chunk is projected; a job's features are overwritten
-        two jobs later only after that query side has read them)."""
+        two jobs later only after that query side has read them). train_priority: priority of
+        the train projection streams. bulk_priority: with query_stream, run the query side's
+        bulk kernels (Fisher fit and query projections) on a third stream of this priority,
+        so that they can yield to the train projections while the latency-bound factorisation
+        chain keeps query_priority (lower number = higher priority). side_thread: with
+        query_stream, a host thread of its own enqueues the query side, so that a query-side
+        stream that the GPU serves late (a full launch queue) cannot hold up the enqueueing of
+        the next chunks' projections."""
         assert n_train % chunk == 0 and n_train >= topk >= 1
         self.layers = [tda.LayerDesc(di, do, T, k, k, seed=seed, layer=i) for i, (di, do) in enumerate(linears)]
         self.nl = len(self.layers)
@@ -78,6 +88,17 @@ class StackJob:
         self.proj_ws = [torch.empty(self.proj_wsb, dtype=torch.uint8, device=dev)
                         for _ in range(self.train_streams + 1)] if self.proj_wsb else None
         self.side = torch.cuda.Stream(device=dev, priority=query_priority) if query_stream else None
+        self.side_bulk = (torch.cuda.Stream(device=dev, priority=bulk_priority)
+                          if query_stream and bulk_priority is not None else None)
+        self.train_priority = train_priority
+        self._dev = dev
+        self._worker = None
+        self._qd_ready = {}  # job -> threading.Event: its query_done event has been recorded
+        if query_stream and side_thread:
+            self._tasks = queue.Queue()
+            self._err = None
+            self._worker = threading.Thread(target=self._run_side, name="tda-query-side", daemon=True)
+            self._worker.start()
         self._train_done = {}  # job -> event after its last chunk's projections (train stream)
         self._query_done = {}  # job -> event after its last query share (query stream)
 
@@ -112,7 +133,7 @@ class StackJob:
             return
         main = torch.cuda.current_stream()
         if len(self._streams) < n:
-            self._streams = [torch.cuda.Stream(device=main.device) for _ in range(n)]
+            self._streams = [torch.cuda.Stream(device=main.device, priority=self.train_priority) for _ in range(n)]
         for st in self._streams[:n]:
             st.wait_stream(main)
         for li, L in enumerate(self.layers):
@@ -133,13 +154,22 @@ class StackJob:
         D, DT = self.D, self.DT
         st = self.state[:(l1 - l0) * self.per]
         slot = self.train_streams  # the query side's own projection workspace
-        mark("fisher_fit")
-        tda.tda_precondition(tda.TDA_PC_RESET, l1 - l0, D, tda.TDA_F32, st)
-        tda.tda_precondition(tda.TDA_PC_FIT_ACCUM, l1 - l0, D, tda.TDA_F32, st, phi=self.Phi[b][:, l0 * D:],
-                             n=self.N, ld_phi=DT)
-        mark("project_query")
-        for li in range(l0, l1):
-            self._project(self.layers[li], factors("query", li, j, s), self.Q[:, li * D:], hook, li, "query", slot)
+        chain, bulk = torch.cuda.current_stream(), self.side_bulk
+        if bulk is not None:
+            bulk.wait_stream(chain)  # the previous share's factorisation is done with the state
+        with torch.cuda.stream(bulk if bulk is not None else chain):
+            mark("fisher_fit")
+            tda.tda_precondition(tda.TDA_PC_RESET, l1 - l0, D, tda.TDA_F32, st)
+            tda.tda_precondition(tda.TDA_PC_FIT_ACCUM, l1 - l0, D, tda.TDA_F32, st, phi=self.Phi[b][:, l0 * D:],
+                                 n=self.N, ld_phi=DT)
+            mark("project_query")
+            for li in range(l0, l1):
+                self._project(self.layers[li], factors("query", li, j, s), self.Q[:, li * D:], hook, li, "query",
+                              slot)
+            if bulk is not None:
+                mark(None)
+        if bulk is not None:
+            chain.wait_stream(bulk)
         mark("factor_apply")
         tda.tda_precondition(tda.TDA_PC_FACTOR_APPLY, l1 - l0, D, tda.TDA_F32, st, n_total=self.N,
                              lambda_abs=self.lambda_abs, lambda_rel_mean_eig=self.lambda_rel, q=self.Q[:, l0 * D:],
@@ -157,6 +187,41 @@ class StackJob:
             mark("topk")
         tda.tda_topk(self.S[j % 2][r0:], r1 - r0, self.N, self.N, self.topk, self.idx[r0:], self.val[r0:])
 
+    def _run_side(self):
+        torch.cuda.set_device(self._dev)
+        while True:
+            task = self._tasks.get()
+            try:
+                if task is None:
+                    return
+                if self._err is None:
+                    with torch.cuda.stream(self.side):
+                        task()
+            except BaseException as e:  # re-raised on the caller's thread by step() or join()
+                self._err = e
+                for ready in list(self._qd_ready.values()):
+                    ready.set()  # a caller waiting for a job boundary wakes up and raises
+            finally:
+                self._tasks.task_done()
+
+    def _side_part(self, j, s, factors, first_job, mark, hook, ready=None):
+        """The query side of step s of job j, on the query-side stream (current stream);
+        ready (threading.Event) is set once job j-1's query_done event is recorded."""
+        if j - 1 >= first_job:
+            if s == 0 and (j - 1) in self._train_done:
+                self.side.wait_event(self._train_done.pop(j - 1))
+            self.query_part(j - 1, s, factors, mark, hook)
+            if s == self.C - 1:
+                e = torch.cuda.Event()
+                e.record(self.side)
+                self._query_done[j - 1] = e
+                if ready is not None:
+                    ready.set()
+        if j - 2 >= first_job:
+            self.topk_part(j - 2, s, mark)
+        if mark:
+            mark(None)
+
     def step(self, j, s, factors, first_job=0, mark=None, hook=None):
         """Step s of job j: chunk s of job j, share s of job j-1's query side and of job
         j-2's top-k. Jobs before first_job do not exist (their shares are skipped)."""
@@ -170,8 +235,15 @@ class StackJob:
                 mark(None)
             return
         main = torch.cuda.current_stream()
-        if s == 0 and (j - 2) in self._query_done:
-            main.wait_event(self._query_done.pop(j - 2))  # job j overwrites job j-2's features
+        if s == 0 and j - 2 >= first_job:
+            ready = self._qd_ready.pop(j - 2, None)
+            if ready is not None:
+                ready.wait()  # the query-side thread has recorded job j-2's query_done
+                if self._err is not None:
+                    err, self._err = self._err, None
+                    raise err
+            if (j - 2) in self._query_done:
+                main.wait_event(self._query_done.pop(j - 2))  # job j overwrites job j-2's features
         self.train_part(j, s, factors, mark, hook)
         if mark:
             mark(None)
@@ -179,21 +251,29 @@ class StackJob:
             e = torch.cuda.Event()
             e.record(main)
             self._train_done[j] = e
-        with torch.cuda.stream(self.side):
-            if j - 1 >= first_job:
-                if s == 0 and (j - 1) in self._train_done:
-                    self.side.wait_event(self._train_done.pop(j - 1))
-                self.query_part(j - 1, s, factors, mark, hook)
-                if s == self.C - 1:
-                    e = torch.cuda.Event()
-                    e.record(self.side)
-                    self._query_done[j - 1] = e
-            if j - 2 >= first_job:
-                self.topk_part(j - 2, s, mark)
-            if mark:
-                mark(None)
+        if self._worker is None:
+            with torch.cuda.stream(self.side):
+                self._side_part(j, s, factors, first_job, mark, hook)
+            return
+        ready = None
+        if s == self.C - 1 and j - 1 >= first_job:
+            ready = self._qd_ready[j - 1] = threading.Event()
+        self._tasks.put(lambda: self._side_part(j, s, factors, first_job, mark, hook, ready))
 
     def join(self):
-        """Make the current stream wait for the query side's work queued so far."""
+        """Make the current stream wait for the query side's work queued so far (and, with
+        the query-side thread, wait until that thread has enqueued it)."""
+        if self._worker is not None:
+            self._tasks.join()
+            if self._err is not None:
+                err, self._err = self._err, None
+                raise err
         if self.side is not None:
             torch.cuda.current_stream().wait_stream(self.side)
+
+    def close(self):
+        """Stop the query-side thread (after join())."""
+        if self._worker is not None:
+            self._tasks.put(None)
+            self._worker.join()
+            self._worker = None

@@ -7,8 +7,9 @@ the first are complete; both are compared with the oracle's fp64 features,
 Fisher, damped inverse (Woodbury form: fewer examples than features), score
 matrix and top-k over the same factors. The shares of the query side differ in
 size (six linears over four steps), D = 4096 takes the blocked tensor-core
-preconditioner, and the train projections of a chunk run on one or on three
-streams, the query side in line or on a stream of its own.
+preconditioner, and the train projections of a chunk run on one, two or three
+streams, the query side in line, on a stream of its own, or enqueued by a host
+thread of its own with its bulk kernels on a third stream.
 """
 import os
 
@@ -51,8 +52,12 @@ def window(role, li, j, s):
     return [(2 * j + li + r) % PQ for r in range(NQ)]
 
 
-@pytest.mark.parametrize("train_streams,query_stream", [(1, False), (3, True)])
-def test_stack_job_matches_oracle(orc, train_streams, query_stream):
+@pytest.mark.parametrize("train_streams,query_stream,opts", [
+    (1, False, {}), (3, True, {}),
+    # the query side enqueued by a host thread of its own, its bulk kernels on a third stream,
+    # stream priorities train > factorisation chain > bulk
+    (2, True, {"side_thread": True, "bulk_priority": 0, "train_priority": -1, "query_priority": -2})])
+def test_stack_job_matches_oracle(orc, train_streams, query_stream, opts):
     assert torch.cuda.is_available(), "GPU tests need a CUDA device"
     tbuild.build()
     tda.load()
@@ -74,12 +79,13 @@ def test_stack_job_matches_oracle(orc, train_streams, query_stream):
         return pieces
 
     job = StackJob(LIN, T, K, N, CHUNK, NQ, topk=TOPK, lambda_rel=1e-2, device=dev, train_streams=train_streams,
-                   query_stream=query_stream)
+                   query_stream=query_stream, **opts)
     marks = []
     for j in range(3):
         for s in range(job.C):
             job.step(j, s, factors, mark=marks.append)
     job.join()
+    job.close()
     torch.cuda.synchronize()
     tda.tda_device_status()
     assert {"project_train", "fisher_fit", "project_query", "factor_apply", "score", "topk"} <= set(marks)
