@@ -11,12 +11,15 @@
 // CTA tile: 128 rows of Phi (MMA M, one TMEM lane each) x BN query columns
 // (MMA N). Lane 0 of warp 5 copies the fp32 chunks of both operands with TMA
 // (32 features = one 128-byte row per operand row, 128B swizzle: already the
-// K-major operand layout) into the hi tiles of a stage; warps 0-3 split them in
-// place (hi stays, lo goes to the lo tile at the same offset); lane 0 of warp 4
-// issues the MMAs; warps 4-7 read the fp32 accumulator tile from TMEM. A thread-block cluster of cs CTAs splits K; the
-// members' partial tiles are summed into the leader CTA over distributed shared
-// memory (deterministic, no workspace) before the leader writes S. All waits
-// are bounded (see tc_ptx.cuh).
+// K-major operand layout) into the hi tiles of a stage; warps 0-3 write lo to
+// the lo tile at the same offset (the fp32 tile itself is the hi operand: a
+// kind::tf32 MMA reads only the upper 19 bits); lane 0 of warp 4 issues the
+// MMAs; warps 4-7 read the fp32 accumulator tile from TMEM. A thread-block
+// cluster of cs CTAs splits K; the members' partial tiles are summed into the
+// leader CTA over distributed shared memory (deterministic, no workspace)
+// before the leader writes S. With more tiles than SMs and short K (the blocked
+// Cholesky's products) gemm3x_persist_kernel walks the tiles instead. All
+// waits are bounded (see tc_ptx.cuh).
 #include <cuda.h>
 
 #include <mutex>
