@@ -15,7 +15,8 @@ one by one, and stage by stage from the GPU's own features.
   D = 16384 Fisher fit, factorisation and query solves, the preconditioned
   score and the top-100; the factors are also streamed from pinned host memory.
 * The 8192 x 8192 linear of the route sweep: exact similarity by both routes.
-Tolerances: relative Frobenius error 2e-2 for bf16 factors (spec bound).
+Tolerances: relative Frobenius error 2e-2 for score matrices and features from bf16 factors
+(fp32 accumulation).
 """
 import math
 import os
