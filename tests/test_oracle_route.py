@@ -199,3 +199,17 @@ def test_exact_similarity_and_norm_costs_count_loop_nests(orc):
         np.testing.assert_allclose(n, ref, rtol=1e-12)
     _, c3 = orc.route_costs(orc.OP_NORM_PROJECTED, B1, 0, TT, DI, DO, KI, KO)
     assert c3[0] == 2 * ca.macs and c3[1] == 2 * cb.macs and c3[2] == 2 * cg.macs
+
+
+def test_exact_ties_prefer_gram_then_the_factored_projection(orc):
+    # The tie rule (a reading: App. A.4 prefers the factorised form for its memory): on equal
+    # counts the Gram route wins, then the factored projection, then materialisation.
+    # Projected similarity ties exactly at B1 = 1, B2 = 2, T = 2, k_a = k_g = 2: beyond the
+    # shared projection of the factors the factored route adds (B1+B2) 2 T k_a k_g + B1 B2 2 k_a k_g
+    # = 48 + 16 and the Gram route B1 B2 2 T^2 (k_a + k_g) = 64.
+    best, c = orc.route_costs(orc.OP_SIM_PROJECTED, 1, 2, 2, 64, 64, 2, 2)
+    assert c[0] == c[2] < c[1] and best == 2
+    # Projection ties at T = d_in = d_out = k = 1: factored 2T(d k + d k) + 2T k^2 = 6,
+    # materialised 2T d^2 + 2 d^2 k + 2 d k^2 = 6.
+    best, c = orc.route_costs(orc.OP_PROJECT, 1, 0, 1, 1, 1, 1, 1)
+    assert c[0] == c[1] == 6 and best == 0
