@@ -98,6 +98,26 @@ MUTANTS = [
      "cost[2] = B1 * B2 * 2.0 * t * t * (Ni + No);", "cost[2] = B1 * B2 * 2.0 * t * (Ni + No);"),
     ("route costs: norms without the sum of squares",
      "cost[0] = B1 * (proj_factors + contract + 2.0 * ka * kg);", "cost[0] = B1 * (proj_factors + contract);"),
+    ("damped inverse: lambda left off the diagonal",
+     "for (int64_t a = 0; a < D; ++a) L[a * D + a] += lambda;", "for (int64_t a = 0; a < D; ++a) L[a * D + a] += 0.0;"),
+    ("forward substitution without the division by the pivot",
+     "y[i] = s / L[i * D + i];", "y[i] = s;"),
+    ("Woodbury: final division by lambda dropped",
+     "x[a] = s / lambda;", "x[a] = s;"),
+    ("K-FAC eigenvalues: sum instead of product of the factors' eigenvalues",
+     "Lam[r * k_in + c] = wg[r] * wa[c];", "Lam[r * k_in + c] = wg[r] + wa[c];"),
+    ("EK-FAC eigenvalues: sum over the examples instead of the mean",
+     "Lam[e] = N > 0 ? s / (double)N : 0.0;", "Lam[e] = N > 0 ? s : 0.0;"),
+    ("K-FAC damping: mean over k_in entries instead of k_in k_out",
+     "return lambda_abs + lambda_rel * s / (double)(k_in * k_out);", "return lambda_abs + lambda_rel * s / (double)k_in;"),
+    ("Jacobi: eigenpairs sorted descending",
+     "if (w[j] < w[m]) m = j;", "if (w[j] > w[m]) m = j;"),
+    ("top-k: ascending scores",
+     "if (a->v > b->v) return -1;", "if (a->v < b->v) return -1;"),
+    ("route costs: projection without the token contraction",
+     "cost[0] = B1 * (proj_factors + contract);", "cost[0] = B1 * proj_factors;"),
+    ("route costs: exact norms by the Gram route with T instead of T^2",
+     "cost[2] = B1 * 2.0 * t * t * (Ni + No);", "cost[2] = B1 * 2.0 * t * (Ni + No);"),
     ("route choice: ties prefer the factored projection over the Gram route",
      "static const int32_t pref[3] = {2, 0, 1};", "static const int32_t pref[3] = {0, 2, 1};"),
 ]
