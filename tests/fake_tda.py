@@ -77,3 +77,20 @@ def install(fake, monkeypatch, cuda_streams=False):
     if cuda_streams:
         monkeypatch.setattr(torch.cuda, "current_stream", lambda *a, **k: None)
         monkeypatch.setattr(torch.cuda, "stream", lambda s: contextlib.nullcontext())
+
+
+def pipeline_class(module, name):
+    """The host pipeline class `name` of paper_2609_38767_gb300.<module>, or, when the
+    environment names another source for that module (TDA_<MODULE>_SOURCE; the mutation
+    test of the host-logic tests plants mistakes in a copy), the class from that copy."""
+    import importlib
+    import importlib.util
+    import os
+
+    src = os.environ.get(f"TDA_{module.upper()}_SOURCE")
+    if not src:
+        return getattr(importlib.import_module(f"paper_2609_38767_gb300.{module}"), name)
+    spec = importlib.util.spec_from_file_location(f"{module}_variant", src)
+    mod = importlib.util.module_from_spec(spec)
+    spec.loader.exec_module(mod)
+    return getattr(mod, name)

@@ -16,9 +16,10 @@ import torch
 import paper_2609_38767_gb300 as tda
 from paper_2609_38767_gb300 import build as tbuild
 from paper_2609_38767_gb300 import synth
-from paper_2609_38767_gb300.block import BlockPipeline
 
-from fake_tda import FakeLib, install
+from fake_tda import FakeLib, install, pipeline_class
+
+BlockPipeline = pipeline_class("block", "BlockPipeline")
 
 LIN = [(32, 16), (16, 48), (24, 24)]
 T, K, N, NQ, TOPK = 7, 4, 48, 5, 6

@@ -7,6 +7,7 @@ closed forms, identities, published vectors) against it in a fresh process.
 At least one pin must fail for every mistake; the unmodified copy must pass
 them all. The mistakes are planted only in temporary copies, on the CPU.
 """
+import concurrent.futures
 import os
 import shutil
 import subprocess
@@ -123,8 +124,7 @@ MUTANTS = [
 ]
 
 
-def _run_pins(tmp_path, source_text):
-    d = tmp_path / "oracle"
+def _run_pins(d, source_text):
     d.mkdir()
     (d / "oracle.c").write_text(source_text)
     shutil.copy(os.path.join(ROOT, "oracle", "oracle.h"), d / "oracle.h")
@@ -133,15 +133,27 @@ def _run_pins(tmp_path, source_text):
                           cwd=ROOT, env=env, capture_output=True, text=True, timeout=300)
 
 
-def test_unmodified_copy_passes_every_pin(tmp_path):
-    r = _run_pins(tmp_path, open(ORACLE_C).read())
+@pytest.fixture(scope="module")
+def runs(tmp_path_factory):
+    """Every copy's pin run, several at once (each is a compile and a short pytest process)."""
+    src = open(ORACLE_C).read()
+    texts = {"unmodified": src}
+    for what, old, new in MUTANTS:
+        assert src.count(old) == 1, f"mutation site not unique or missing: {old}"
+        texts[what] = src.replace(old, new)
+    base = tmp_path_factory.mktemp("oracle_copies")
+    with concurrent.futures.ThreadPoolExecutor(max_workers=max(1, min(8, os.cpu_count() or 1))) as ex:
+        futs = {k: ex.submit(_run_pins, base / f"copy{i}", t) for i, (k, t) in enumerate(texts.items())}
+        return {k: f.result() for k, f in futs.items()}
+
+
+def test_unmodified_copy_passes_every_pin(runs):
+    r = runs["unmodified"]
     assert r.returncode == 0, r.stdout[-2000:] + r.stderr[-2000:]
 
 
-@pytest.mark.parametrize("what,old,new", MUTANTS, ids=[m[0] for m in MUTANTS])
-def test_planted_mistake_fails_a_pin(tmp_path, what, old, new):
-    src = open(ORACLE_C).read()
-    assert src.count(old) == 1, f"mutation site not unique or missing: {old}"
-    r = _run_pins(tmp_path, src.replace(old, new))
+@pytest.mark.parametrize("what", [m[0] for m in MUTANTS])
+def test_planted_mistake_fails_a_pin(runs, what):
+    r = runs[what]
     # exit code 1: the pins ran and at least one failed (not a build or collection error)
     assert r.returncode == 1 and " failed" in r.stdout, (what, r.returncode, r.stdout[-2000:], r.stderr[-2000:])

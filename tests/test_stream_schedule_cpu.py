@@ -23,9 +23,9 @@ import numpy as np
 import pytest
 
 from paper_2609_38767_gb300 import synth
-from paper_2609_38767_gb300.stream import StackJob
+from fake_tda import FakeLib, bf16_tensor, install, pipeline_class
 
-from fake_tda import FakeLib, bf16_tensor, install
+StackJob = pipeline_class("stream", "StackJob")
 
 LIN = [(24, 16), (16, 40), (32, 24), (24, 24), (40, 16)]  # five linears over four steps: shares 1, 1, 1, 2
 T, K, N, CHUNK, NQ, TOPK, P, PQ = 6, 4, 64, 16, 6, 5, 40, 9
