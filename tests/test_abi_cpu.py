@@ -199,3 +199,20 @@ def test_factored_projection_workspace_layout(libs, k):
     L2 = tda.LayerDesc(di, do, 300, k, k // 2 if k > 16 else 32)
     assert tda.tda_workspace_size(tda.TDA_OP_PROJECT, L2, tda.TDA_BF16, 7, 0, tda.TDA_ROUTE_FACTORED) == 0
     assert tda.tda_workspace_size(tda.TDA_OP_PROJECT, L, tda.TDA_F32, 7, 0, tda.TDA_ROUTE_FACTORED) == 0
+
+
+def test_route_model_matches_oracle_on_random_shapes(libs, orc):
+    # 600 seeded random shapes over every op (the flop model does not depend on the dtype):
+    # the library's host-side cost model and choice equal the oracle's Table 2 counts
+    rng = np.random.default_rng(7)
+    for _ in range(600):
+        op = int(rng.integers(0, 5))
+        n1, n2 = int(rng.integers(0, 5000)), int(rng.integers(0, 5000))
+        T = int(2 ** rng.integers(0, 14)) if rng.random() < 0.5 else int(rng.integers(1, 9000))
+        di, do = int(rng.integers(1, 20000)), int(rng.integers(1, 20000))
+        ki, ko = int(rng.integers(1, 257)), int(rng.integers(1, 257))
+        L = tda.LayerDesc(di, do, T, ki, ko)
+        chosen, cost = tda.tda_route(L, op, n1, n2, tda.TDA_BF16)
+        best, ocost = orc.route_costs(op, n1, n2, T, di, do, ki, ko)
+        assert chosen == best, (op, n1, n2, T, di, do, ki, ko, cost, ocost)
+        np.testing.assert_allclose(cost, ocost, rtol=1e-12)
