@@ -316,8 +316,14 @@ cudaError_t launch_project_materialized(const tda_layer_desc& L, tda_dtype dt, c
     return cudaSuccess;
 }
 
+// The Frobenius dots' split-K partial sums (at most 256 feature slices per query x train pair of a
+// chunk) sit after the query and train gradients, so that even the smallest workspace (one train
+// gradient at a time) keeps the feature axis split: one unsplit row of millions of features
+// accumulated in the tensor pipe's truncating fp32 loses about 1e-2 of relative accuracy.
+static size_t simexact_part_floats(int64_t n_q, int64_t chunk) { return (size_t)256 * (size_t)(n_q * chunk); }
+
 size_t similarity_materialize_ws_bytes(const tda_layer_desc& L, int64_t n_q, int64_t chunk) {
-    return sizeof(float) * (size_t)((n_q + chunk) * L.d_out * L.d_in);
+    return sizeof(float) * ((size_t)((n_q + chunk) * L.d_out * L.d_in) + simexact_part_floats(n_q, chunk));
 }
 
 cudaError_t launch_similarity_materialized(const tda_layer_desc& L, tda_dtype dt, const void* Aq,
@@ -342,7 +348,10 @@ cudaError_t launch_similarity_materialized(const tda_layer_desc& L, tda_dtype dt
     float* part = nullptr;
     if (splits > 1) {
         const size_t need = (size_t)splits * (size_t)n_q * (size_t)chunk;
-        if (chunk > 1 && need <= (size_t)gsz) {
+        const size_t grads = (size_t)(n_q + chunk) * (size_t)gsz;  // floats of the query and train DW
+        if (ws_bytes / sizeof(float) >= grads + need) {
+            part = Gq + grads;  // the partials' room after the train gradients
+        } else if (chunk > 1 && need <= (size_t)gsz) {
             --chunk;
             part = Gt + chunk * gsz;
         } else {

@@ -117,8 +117,9 @@ def test_workspace_sizes(libs):
     assert tda.tda_workspace_size(tda.TDA_OP_PROJECT, L, tda.TDA_F32, 10, 0, tda.TDA_ROUTE_FACTORED) == 0
     assert tda.tda_workspace_size(tda.TDA_OP_PROJECT, L, tda.TDA_F32, 10, 0,
                                   tda.TDA_ROUTE_MATERIALIZE) == 4 * (128 * 256 + 128 * 16)
+    # the 3 query DW, one train DW and the split-K partials of 3 dots over at most 256 slices
     assert tda.tda_workspace_size(tda.TDA_OP_SIMILARITY_EXACT, L, tda.TDA_F32, 3, 9,
-                                  tda.TDA_ROUTE_MATERIALIZE) == 4 * 4 * 128 * 256
+                                  tda.TDA_ROUTE_MATERIALIZE) == 4 * (4 * 128 * 256 + 256 * 3)
     assert tda.tda_workspace_size(tda.TDA_OP_SIMILARITY_EXACT, L, tda.TDA_F32, 3, 9, tda.TDA_ROUTE_GRAM) == 0
     D = 16 * 16
     assert tda.tda_workspace_size(tda.TDA_OP_SIMILARITY_PROJECTED, L, tda.TDA_F32, 3, 9,

@@ -14,7 +14,8 @@ one by one, and stage by stage from the GPU's own features.
   T = 2048, Student-t activations): 7 x 16384 features per example, the
   D = 16384 Fisher fit, factorisation and query solves, the preconditioned
   score and the top-100; the factors are also streamed from pinned host memory.
-* The 8192 x 8192 linear of the route sweep: exact similarity by both routes.
+* The 8192 x 8192 linear of the route sweep: exact similarity by both routes at
+  T = 8 ... 512, the projection by both routes at T = 8 and 2048.
 Tolerances: relative Frobenius error 2e-2 for score matrices and features from bf16 factors
 (fp32 accumulation).
 """
@@ -311,7 +312,7 @@ def test_topk_at_large_model_query_shape(dev, orc):
     np.testing.assert_array_equal(val.cpu().numpy(), ov.astype(np.float32))
 
 
-@pytest.mark.parametrize("T", [8, 32])
+@pytest.mark.parametrize("T", [8, 32, 128, 512])
 def test_route_sweep_linear_exact_similarity(dev, orc, T):
     # 8192 x 8192 linear, A, B ~ N(0, 1): Gram route and materialise route vs the oracle
     d, nq, nt = 8192, 2, 2
@@ -330,6 +331,31 @@ def test_route_sweep_linear_exact_similarity(dev, orc, T):
         tda.tda_similarity_exact(L, tda.TDA_BF16, to(Aq), to(Bq), nq, to(At), to(Bt), nt, S, nt, 0.0, route, ws, wsb)
         tda.tda_device_status()
         assert rel_fro(S.cpu().numpy(), ref) <= TOL, route
+
+
+@pytest.mark.parametrize("T", [8, 2048])
+def test_route_sweep_linear_projection_both_routes(dev, orc, T):
+    # the 8192 x 8192 linear of the route sweep at a short and a long T, k = 64, A, B ~ N(0, 1): the
+    # factored tensor-core projection and the materialise route against the oracle (at T = 8192 the
+    # oracle's loops take minutes per example)
+    d, n, k = 8192, 2, 64
+    A = synth.factors(synth.SEED_A, 0, n, T, d, 1.0, dtype="bf16")
+    B = synth.factors(synth.SEED_B, 0, n, T, d, 1.0, dtype="bf16")
+    to = lambda x: torch.from_numpy(x.view(np.int16)).view(torch.bfloat16).to(dev)
+    L = tda.LayerDesc(d, d, T, k, k, seed=0, layer=0)
+    orc.set_threads(os.cpu_count() or 1)
+    ref = orc.project(synth.to_f64(A, "bf16"), synth.to_f64(B, "bf16"), k, k, 0, 0).reshape(n, k * k)
+    Ad, Bd = to(A), to(B)
+    assert tda.tda_project_engine(L, tda.TDA_BF16, Ad, Bd) == 1
+    for route in (tda.TDA_ROUTE_FACTORED, tda.TDA_ROUTE_MATERIALIZE):
+        wsb = tda.tda_workspace_size(tda.TDA_OP_PROJECT, L, tda.TDA_BF16, n, 0, route)
+        ws = torch.empty(max(wsb, 256), dtype=torch.uint8, device=dev)
+        phi = torch.full((n, k * k), float("nan"), device=dev)
+        tda.tda_project(L, tda.TDA_BF16, Ad, Bd, n, phi, k * k, route, ws, wsb)
+        tda.tda_device_status()
+        got = phi.cpu().numpy()
+        for e in range(n):
+            assert rel_fro(got[e], ref[e]) <= TOL, (route, e)
 
 
 def test_overlapped_query_side_matches_serial(dev):
