@@ -206,8 +206,10 @@ tda_status tda_project_materialized_noalloc(const tda_layer_desc* L, tda_dtype d
  *   S[q][i] = beta*S[q][i] + <DW_q, DW_i>_F
  * for n_q query and n_t train examples of one layer (Eq. 4's left side).
  *   route GRAM computes sum_{t,s} <a_t^q,a_s^i><g_t^q,g_s^i> (Eq. 4) without
- *   forming DW; MATERIALIZE forms DW (Eq. 1) in ws and takes Frobenius dots;
- *   AUTO asks tda_route (TDA_OP_SIMILARITY_EXACT).
+ *   forming DW; MATERIALIZE forms DW (Eq. 1) in ws and takes Frobenius dots
+ *   split over slices of the d_out*d_in features (ws also holds the slices'
+ *   partial sums; a larger ws holds more train DW at once); AUTO asks tda_route
+ *   (TDA_OP_SIMILARITY_EXACT).
  *   Aq/Bq: [n_q][T][d], At/Bt: [n_t][T][d], dtype as in tda_project.
  *   S: device fp32, row q at S + q*ld_S (ld_S >= n_t). beta 0 overwrites.
  * ------------------------------------------------------------------------- */
